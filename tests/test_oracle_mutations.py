@@ -1,0 +1,90 @@
+"""Plant plausible mistakes in the oracle (on the CPU) and check that a pin catches each."""
+import math
+
+import pytest
+import torch
+
+import oracle
+import oracle.model as om
+import tests.test_oracle_pins as pins
+
+
+def _patch(monkeypatch, name, fn):
+    monkeypatch.setattr(om, name, fn)
+    monkeypatch.setattr(oracle, name, fn)
+
+
+def bad_rope(x, theta):            # wrong rotation sign
+    S, hd = x.shape[1], x.shape[3]
+    half = hd // 2
+    inv = theta ** (-2.0 * torch.arange(half, dtype=torch.float64) / hd)
+    ang = torch.arange(S, dtype=torch.float64)[:, None] * inv[None, :]
+    c, s = torch.cos(ang)[None, :, None, :], torch.sin(ang)[None, :, None, :]
+    x1, x2 = x[..., :half], x[..., half:]
+    return torch.cat([x1 * c + x2 * s, x2 * c - x1 * s], dim=-1)
+
+
+def bad_attention(q, k, v):        # missing 1/sqrt(hd)
+    return om.attention.__wrapped__(q * math.sqrt(q.shape[-1]), k, v)
+
+
+def bad_kl(z, t, kl_dir=0):        # lse of the teacher dropped
+    lp = torch.log_softmax(z, -1)
+    return (lp.exp() * (lp - t)).sum(-1)
+
+
+def bad_rmsnorm(x, g, eps):        # eps outside the square root
+    return x / (torch.sqrt((x * x).mean(-1, keepdim=True)) + eps) * g
+
+
+def bad_adamw(theta, g, m, v, step, lr, b1, b2, eps, wd):   # no bias correction
+    theta.mul_(1 - lr * wd)
+    m.mul_(b1).add_((1 - b1) * g)
+    v.mul_(b2).add_((1 - b2) * g * g)
+    theta.sub_(lr * m / (torch.sqrt(v) + eps))
+
+
+def bad_gelu(x):                   # erf-GELU instead of the tanh form
+    return torch.nn.functional.gelu(x)
+
+
+MUTATIONS = [
+    ("rope", bad_rope, [pins.test_rope_is_the_complex_rotation, pins.test_layer_matches_library_composition]),
+    ("kl_rows", bad_kl, [pins.test_loss_closed_forms]),
+    ("rmsnorm", bad_rmsnorm, [pins.test_blocks_match_library_routines]),
+    ("adamw_update", bad_adamw, [pins.test_adamw_matches_torch_optim]),
+    ("gelu_tanh", bad_gelu, [pins.test_blocks_match_library_routines]),
+]
+
+
+@pytest.mark.parametrize("name,fn,tests", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_pins_catch_planted_mistake(monkeypatch, name, fn, tests):
+    _patch(monkeypatch, name, fn)
+    for t in tests:
+        with pytest.raises(AssertionError):
+            t()
+
+
+def test_pins_catch_unscaled_attention(monkeypatch):
+    orig = om.attention
+    _patch(monkeypatch, "attention", lambda q, k, v: orig(q * math.sqrt(q.shape[-1]), k, v))
+    with pytest.raises(AssertionError):
+        pins.test_attention_matches_sdpa(4, 2, 8)
+
+
+def test_pins_catch_wrong_gqa_grouping(monkeypatch):
+    orig = om.attention
+
+    def tiled(q, k, v):            # kv head h % Hkv instead of h // (H / Hkv)
+        rep = q.shape[2] // k.shape[2]
+        return orig(q, k.repeat(1, 1, rep, 1), v.repeat(1, 1, rep, 1))
+    _patch(monkeypatch, "attention", tiled)
+    with pytest.raises(AssertionError):
+        pins.test_attention_matches_sdpa(4, 2, 8)
+
+
+def test_pins_catch_dropped_residual(monkeypatch):
+    orig = om.layer_forward
+    _patch(monkeypatch, "layer_forward", lambda P, l, x, d: orig(P, l, x, d) - x)
+    with pytest.raises(AssertionError):
+        pins.test_layer_matches_library_composition()
