@@ -1,0 +1,348 @@
+#!/usr/bin/env python
+"""Throughput of ZeroLock's concurrent per-chunk update on GB300 (one JSON line on stdout).
+
+A step is one micro-batch through all K chunks (forward, readout, local objective, local
+backward, AdamW) via zl_step. Default workload: the GPT-2-small-shaped bf16 model (12 layers,
+d 768, vocab 50257, micro-batch 8 x 512 tokens, K = 4). Also reported: the same-engine
+backpropagation baseline (zl_bp_step), peak HBM of both, the GEMM roofline fraction measured
+live with CUDA events, the CPU oracle on a bounded sample, an end-to-end figure through the
+public API with host buffers, and SM clocks sampled during the timed region.
+
+Multi-GPU (torchrun): the path does not shard; every rank trains an independent replica on
+its own micro-batches ("replicas only"), value = tokens of all ranks / max rank time.
+
+--impl reference times the CPU oracle (the only reference implementation there is) on
+bounded samples of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+import synth  # noqa: E402
+
+WORKLOADS = {"gpt2": synth.GPT2_SMALL, "tiny": synth.TINY, "llama1b": synth.LLAMA_1B, "llama3b": synth.LLAMA_3B,
+             "llama7b": synth.LLAMA_7B}
+METRIC = "training tokens/s on 1 GB300 (ZeroLock vs same-engine BP), peak HBM GB, % roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="gpt2", choices=list(WORKLOADS))
+    ap.add_argument("--K", type=int, default=0, help="chunk count (default: the workload's)")
+    ap.add_argument("--max-live", type=int, default=2, help="chunks whose activations may be alive at once")
+    ap.add_argument("--no-bp", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def workload_desc(w, K):
+    d = w.dims
+    arch = "llama" if d.arch == synth.ARCH_LLAMA else "gpt2"
+    return (f"{w.name}: {arch}-style decoder, {d.n_layers} layers, d_model {d.d_model}, {d.n_heads} heads "
+            f"({d.n_kv_heads} kv), ffn {d.d_ff}, vocab {d.vocab}, micro-batch {w.batch} x seq {w.seq}, "
+            f"K={K} chunks, alpha {w.alpha}, AdamW")
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+# ---------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, local_rank: int):
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        self.gpu = vis.split(",")[local_rank] if vis else str(local_rank)
+        self.proc = None
+        self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.flush()
+        self.out.seek(0)
+        rows = [r.split(",") for r in self.out.read().strip().splitlines() if r.strip()]
+        os.unlink(self.out.name)
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx = max(mx, float(r[2]))
+                for n, v in zip(names, r[5:9]):
+                    if v.strip() == "Active":
+                        reasons.add(n)
+            except (ValueError, IndexError):
+                continue
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------------------
+# CPU oracle on a bounded sample
+# ---------------------------------------------------------------------------------------------
+def oracle_sample(w, K, params, n_samples: int):
+    """Times the oracle on `n_samples` local steps of one chunk on one 1 x seq sequence each.
+
+    One local step of one chunk costs about 1/K of a full ZeroLock step of the same tokens,
+    so the equivalent rate is (seq / K) tokens per sample time.
+    """
+    from oracle import Oracle, OracleConfig
+    bounds = synth.chunk_bounds(w.dims.n_layers, K)
+    P = {n: (synth.round_bf16(t) if (w.dtype == "bf16" and t.dim() == 2) else t) for n, t in params.items()}
+    dt = torch.float32 if w.dtype == "bf16" else torch.float64
+    orc = Oracle(OracleConfig(dims=w.dims, bounds=bounds, alpha=w.alpha, lr=w.lr), P, dtype=dt)
+    ids = synth.zipf_ids(w.seed + 77, 1, w.seq, w.dims.vocab)
+    labels = synth.next_token_labels(ids)
+    h0 = orc.embed(ids)
+    times = []
+    for i in range(n_samples):
+        k = i % K + 1
+        t0 = time.perf_counter()
+        orc.local_grad(k, h0, labels)
+        times.append(time.perf_counter() - t0)
+    return times, (w.seq / K), torch.get_num_threads()
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = WORKLOADS[args.workload]
+    K = args.K or w.K
+    params = synth.make_params(w.dims, w.seed)
+    times, tok, cores = oracle_sample(w, K, params, args.warmup + args.steps)
+    t = sum(times[args.warmup:])
+    value = tok * args.steps / t
+    sample = f"{args.steps} local steps of one chunk on 1 x {w.seq} tokens, round-robin over the K chunks"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32" if w.dtype == "bf16" else "f64", "data": "synthetic",
+            "config": {"workload": workload_desc(w, K), "K": K},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------------------------
+def run_ours(args):
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    import paper_2608_07974_gb300 as pkg
+    pkg.build()
+    from paper_2608_07974_gb300 import binding as zb
+
+    w = WORKLOADS[args.workload]
+    K = args.K or w.K
+    bounds = synth.chunk_bounds(w.dims.n_layers, K)
+    params = synth.make_params(w.dims, w.seed)
+
+    def make_engine(max_live):
+        e = zb.ZeroLock(w.dims, K, bounds, dtype=w.dtype, alpha=w.alpha, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
+                        eps=w.eps, weight_decay=w.weight_decay, max_live_chunks=max_live)
+        e.load(params)
+        return e
+
+    nb = 4   # distinct resident micro-batches, per rank
+    batches = [synth.make_batch(w, 1000 * rank + i) for i in range(nb)]
+    dev_batches = [(a.cuda(), b.cuda()) for a, b in batches]
+    tokens = w.batch * w.seq
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+
+    def timed(fn, steps):
+        barrier()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(steps):
+            fn(i)
+        t1.record(stream)
+        barrier()
+        ms = t0.elapsed_time(t1)
+        if world > 1:
+            x = torch.tensor([ms], device="cuda")
+            dist.all_reduce(x, op=dist.ReduceOp.MAX)
+            ms = float(x)
+        return ms
+
+    # ---- ZeroLock: device-resident inputs -----------------------------------------------------
+    eng = make_engine(args.max_live)
+
+    def zl(i):
+        ids, lab = dev_batches[i % nb]
+        zb.zl_step(eng.ctx, ids, lab, w.batch, w.seq, K, want_losses=False)
+        if i % 8 == 7:
+            zb.zl_join(eng.ctx)
+
+    def zl_joined(i):
+        zl(i)
+        zb.zl_join(eng.ctx)
+
+    for i in range(args.warmup):
+        zl(i)
+    eng.synchronize()
+    eng.reset_peak()
+    clocks = ClockSampler(local)
+    clocks.start()
+    n0 = zb.zl_kernel_launches()
+    ms = timed(zl_joined, args.steps)
+    launches = zb.zl_kernel_launches() - n0
+    clk = clocks.stop()
+    zl_peak = eng.peak_bytes()[0]
+    value = tokens * args.steps * world / (ms / 1e3)
+
+    # ---- live per-kernel-class timing (CUDA events on the launching streams) ------------------
+    zb.zl_profile(eng.ctx, True)
+    prof_steps = min(args.steps, 5)
+    for i in range(prof_steps):
+        zl(i)
+    prof = zb.zl_profile_read(eng.ctx)
+    zb.zl_profile(eng.ctx, False)
+    pk, pk_kind = peaks()
+    g = prof["gemm"]
+    gemm_tflops = g["flops"] / (g["ms"] / 1e3) / 1e12 if g["ms"] > 0 else 0.0
+    tot_ms = sum(v["ms"] for v in prof.values())
+    roof = {"bound": "tensor", "kernel": "gemm (all chunk and head GEMMs)", "achieved": gemm_tflops,
+            "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s", "frac": gemm_tflops / pk["bf16_tflops_sustained"],
+            "peak_kind": f"{pk_kind} bf16 sustained", "traffic": None,
+            "launches": g["launches"], "flops_per_launch": g["flops"] / max(g["launches"], 1),
+            "share_of_kernel_time": g["ms"] / tot_ms if tot_ms else None}
+    classes = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / prof_steps,
+                   "TFLOP/s" if v["flops"] else "GB/s":
+                       (v["flops"] / (v["ms"] / 1e3) / 1e12) if v["flops"] else (v["bytes"] / (v["ms"] / 1e3) / 1e9)
+                       if v["ms"] > 0 else 0.0}
+               for k, v in prof.items() if v["launches"]}
+
+    # ---- end to end through the public API with host buffers ---------------------------------
+    e2e = None
+    if not args.no_e2e:
+        host = [(a.pin_memory(), b.pin_memory()) for a, b in batches]
+        dids = torch.empty_like(dev_batches[0][0])
+        dlab = torch.empty_like(dev_batches[0][1])
+        out = torch.empty(K, dtype=torch.float32)
+
+        def e2e_step(i):
+            hi, hl = host[i % nb]
+            dids.copy_(hi, non_blocking=True)
+            dlab.copy_(hl, non_blocking=True)
+            zb.zl_step(eng.ctx, dids, dlab, w.batch, w.seq, K, want_losses=False)
+            out[:] = torch.tensor(zb.zl_read_losses(eng.ctx, K))
+        for i in range(2):
+            e2e_step(i)
+        ems = timed(e2e_step, args.steps)
+        e2e = {"value": tokens * args.steps * world / (ems / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": 2 * tokens * 4, "d2h_bytes_per_step": K * 4}
+    eng.close()
+    del eng
+    torch.cuda.empty_cache()
+
+    # ---- same-engine backpropagation ----------------------------------------------------------
+    bp = None
+    if not args.no_bp:
+        beng = make_engine(args.max_live)
+
+        def bps(i):
+            ids, lab = dev_batches[i % nb]
+            zb.zl_bp_step(beng.ctx, ids, lab, w.batch, w.seq, want_loss=False)
+            zb.zl_join(beng.ctx)
+        for i in range(args.warmup):
+            bps(i)
+        beng.synchronize()
+        beng.reset_peak()
+        bms = timed(bps, args.steps)
+        bp = {"value": tokens * args.steps * world / (bms / 1e3), "unit": "tokens/s",
+              "peak_hbm_gb": beng.peak_bytes()[0] / 1e9, "ms_per_step": bms / args.steps}
+        beng.close()
+
+    # ---- CPU oracle on a bounded sample (rank 0, one GPU only) --------------------------------
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        times, tok, cores = oracle_sample(w, K, params, 2)
+        cpu = {"value": tok / times[-1], "unit": "tokens/s", "cores": cores, "kind": "oracle",
+               "sample": f"one local step of chunk 2 on 1 x {w.seq} tokens (fp32 oracle, after one warm-up sample); "
+                         f"rate = ({w.seq}/K) tokens per sample time"}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+                "config": {"workload": workload_desc(w, K), "K": K, "bounds": bounds,
+                           "global_batch": w.batch * world, "seq_len": w.seq, "max_live_chunks": args.max_live,
+                           "parallelism": f"replicas x{world}" if world > 1 else "single GPU, K streams",
+                           "l2": "no flush: every step's working set (weights, AdamW state, logits) exceeds L2"},
+                "peak_hbm_gb": zl_peak / 1e9, "bp": bp,
+                "zl_vs_bp": {"throughput": value / bp["value"], "peak_hbm": (zl_peak / 1e9) / bp["peak_hbm_gb"]}
+                if bp else None,
+                "roofline": roof, "kernel_classes": classes, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": launches, "clocks": clk}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

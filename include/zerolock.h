@@ -1,0 +1,193 @@
+/*
+ * zerolock.h -- C ABI of the GB300 (sm_103a) engine for ZeroLock's decoupled per-chunk update.
+ *
+ * The method (paper Section II-A): a decoder-only transformer is cut into K
+ * chunks of consecutive layers (Eq. 1: h_0 = E(x), h_k = f_k(h_{k-1})). Every
+ * chunk reads its output through the model's frozen final norm and LM head
+ * (Eq. 2: z_k = Norm(h_k) W_lm^T), builds the local objective
+ *   L_k = alpha * CE(p_k, y) + (1 - alpha) * KL(p_k || sg(p_{k-1}))   (Eq. 3-5)
+ * averaged over the loss set Omega (positions whose label is >= 0), back-
+ * propagates inside the chunk only (Remark 1) and applies its own optimizer
+ * step (Eq. 6, here AdamW as in Section III-C). Chunks exchange only hidden
+ * states (Section III-A, technique III), so the K chunk updates run
+ * concurrently: one CUDA stream per chunk, chunk k's output h_k handed to
+ * chunk k+1 as soon as its forward ends (early forwarding, technique I).
+ *
+ * Conventions shared by every call:
+ *   - Chunks are numbered k = 1..K as in the paper; h_0 is the embedding output.
+ *   - Token-major activations: row n = b * S + s of a [N = B*S, d] row-major array.
+ *   - Device arrays are in the context's compute dtype (ZL_DTYPE_F32: float,
+ *     ZL_DTYPE_BF16: bfloat16) unless stated otherwise. ids and labels are
+ *     int32 device arrays of B*S entries; a label of -1 marks a position
+ *     outside Omega; ids must lie in [0, vocab), labels in [-1, vocab).
+ *   - Pointers passed in are borrowed: the library never frees them, and
+ *     device pointers given to a call must stay valid and unmodified until the
+ *     next zl_synchronize() on that context returns (work is asynchronous).
+ *   - Every call returns a zl_status. On failure zl_last_error() describes it;
+ *     the context stays usable unless ZL_ERR_STATE is returned. No C++
+ *     exception crosses this boundary.
+ *   - A context is used by one host thread at a time.
+ */
+#ifndef ZEROLOCK_H
+#define ZEROLOCK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct zl_ctx zl_ctx;
+
+typedef enum {
+  ZL_OK = 0,
+  ZL_ERR_ARG = -1,          /* invalid argument (size, index, pointer, id or label range)      */
+  ZL_ERR_CUDA = -2,         /* a CUDA runtime call failed                                      */
+  ZL_ERR_OOM = -3,          /* device allocation failed                                        */
+  ZL_ERR_STATE = -4,        /* the context is no longer usable (sticky CUDA error)              */
+  ZL_ERR_TIMEOUT = -5,      /* zl_synchronize gave up waiting                                  */
+  ZL_ERR_UNSUPPORTED = -6   /* valid but not implemented combination                           */
+} zl_status;
+
+enum { ZL_ARCH_LLAMA = 0, ZL_ARCH_GPT2 = 1 };
+enum { ZL_DTYPE_F32 = 0, ZL_DTYPE_BF16 = 1 };
+
+/* Model shape. arch ZL_ARCH_LLAMA: RMSNorm, rotate-half RoPE, grouped KV heads,
+ * SwiGLU FFN (w1 = [W_gate; W_up]), untied LM head. ZL_ARCH_GPT2: LayerNorm with
+ * bias, learned positions, GELU (tanh) MLP, biased linears, head tied to tok_emb.
+ * d_model must equal n_heads * head_dim with head_dim even and <= 128. */
+typedef struct {
+  int arch;
+  int dtype;                /* ZL_DTYPE_F32 or ZL_DTYPE_BF16 (fp32 master weights and AdamW state) */
+  int n_layers, d_model, n_heads, n_kv_heads, d_ff, vocab, max_seq;
+  float norm_eps, rope_theta;
+} zl_model_dims;
+
+/* Training settings of the local update (Eq. 3-6, step S3 of Section III-B). */
+typedef struct {
+  float alpha;              /* weight of the task term, 0 < alpha <= 1 (Eq. 3)                      */
+  int kl_dir;               /* 0: KL(p_k || p_{k-1}) (Eq. 5);  1: KL(p_{k-1} || p_k)                  */
+  int consis_first;         /* 1: chunk 1's consistency target is p_0 = readout(h_0); 0: alpha_1 = 1  */
+  float lr, beta1, beta2, eps, weight_decay;     /* decoupled AdamW                                  */
+  int accum_m;              /* micro-batches per update window (gradient = their mean), >= 1         */
+  int max_live_chunks;      /* chunks whose activations may be alive at once; 0 means K              */
+  int lr_schedule;          /* 0: constant lr;  1: lr / sqrt(t + lr_gamma), t = 0,1,.. (Theorem 1)    */
+  float lr_gamma;
+} zl_train_cfg;
+
+/* Create a context: parameters, AdamW state, K streams and events, a stream-ordered
+ * activation pool. bounds has K+1 entries, bounds[0] = 0 < bounds[1] < ... <
+ * bounds[K] = n_layers; chunk k owns layers bounds[k-1] .. bounds[k]-1 (Eq. 1).
+ * Parameters start at zero (norm gains at one); load them with zl_set_param.
+ * *out is owned by the caller and released with zl_free. */
+zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const zl_train_cfg* cfg,
+                    zl_ctx** out);
+
+/* Release everything the context owns (waits for its queued work first). NULL-safe. */
+void zl_free(zl_ctx* ctx);
+
+/* Order the context's work after `stream` (a cudaStream_t; NULL = legacy default stream):
+ * every call waits for the work queued on it so far. Results are joined back into it by
+ * zl_join / zl_synchronize. */
+zl_status zl_set_stream(zl_ctx* ctx, void* stream);
+
+/* Tensor names: tok_emb [V,d], pos_emb [max_seq,d] (GPT-2), norm_f.weight [d],
+ * norm_f.bias [d] (GPT-2), lm_head [V,d] (Llama), and per layer l
+ * layers.{l}.{attn_norm.weight, attn_norm.bias, wqkv, bqkv, wo, bo, ffn_norm.weight,
+ * ffn_norm.bias, w1, b1, w2, b2} (biases: GPT-2 only); weights are [out, in] row-major.
+ * zl_set_param copies `bytes` = numel * 4 of fp32 values from src (device memory if
+ * on_device, else host) into the master copy (and the compute copy). */
+zl_status zl_set_param(zl_ctx* ctx, const char* name, const void* src, size_t bytes, int on_device);
+
+/* Copy one tensor out as fp32 (waits for queued work). which: 0 value (master copy),
+ * 1 accumulated gradient, 2 AdamW first moment, 3 AdamW second moment (1-3: trainable only). */
+zl_status zl_get_param(zl_ctx* ctx, const char* name, int which, void* dst, size_t bytes, int on_device);
+
+/* Number of elements of a named tensor (0 with ZL_ERR_ARG if unknown). */
+zl_status zl_param_numel(zl_ctx* ctx, const char* name, size_t* numel);
+
+/* h_0 = E(x) (Eq. 1): h0_out [B*S, d] (caller-owned device array, compute dtype). */
+zl_status zl_embed(zl_ctx* ctx, const int32_t* ids, int B, int S, void* h0_out);
+
+/* h_k = f_k(h_{k-1}) (Eq. 1) for one chunk, no gradient state touched. h_in: [B*S,d]
+ * device array; may be NULL only for k = 1, in which case h_0 = E(ids) is formed
+ * internally. h_out: caller-owned [B*S,d] device array. */
+zl_status zl_forward_chunk(zl_ctx* ctx, int k, const void* h_in, const int32_t* ids, void* h_out,
+                           int B, int S);
+
+/* One local step of chunk k on one micro-batch (steps S1-S3 of Section III-B): forward,
+ * readout, local objective with the teacher p_{k-1} = readout(h_in) (stop-gradient),
+ * backward inside the chunk, gradient accumulation, AdamW at the end of the window.
+ * h_in as in zl_forward_chunk. h_out (optional, may be NULL) receives h_k.
+ * loss_out (optional host pointer): if non-NULL the call waits and stores L_k. */
+zl_status zl_local_step(zl_ctx* ctx, int k, const void* h_in, const int32_t* ids,
+                        const int32_t* labels, int B, int S, void* h_out, float* loss_out);
+
+/* One micro-batch through all K chunks, concurrently (one stream per chunk, early
+ * forwarding; chunk k's teacher is chunk k-1's logits). Same values as K calls of
+ * zl_local_step in order k = 1..K. losses_out: NULL (losses stay on the device, see
+ * zl_read_losses) or a host array of K floats, in which case the call waits. */
+zl_status zl_step(zl_ctx* ctx, const int32_t* ids, const int32_t* labels, int B, int S,
+                  float* losses_out);
+
+/* Same-engine backpropagation baseline: the chunks chained, one readout on h_K,
+ * CE over Omega, gradient through every chunk, AdamW on all (window rules as above). */
+zl_status zl_bp_step(zl_ctx* ctx, const int32_t* ids, const int32_t* labels, int B, int S,
+                     float* loss_out);
+
+/* Global objective L(p_K) = CE of the last chunk's readout over Omega (Section II-C). */
+zl_status zl_eval_global_loss(zl_ctx* ctx, const int32_t* ids, const int32_t* labels, int B, int S,
+                              float* loss_out);
+
+/* Wait for the last zl_step / zl_bp_step and copy its K (or 1) losses to host. */
+zl_status zl_read_losses(zl_ctx* ctx, float* losses_out, int n);
+
+/* Make the stream given to zl_set_stream wait for all queued work (no host wait). */
+zl_status zl_join(zl_ctx* ctx);
+
+/* Wait for all queued work, polling; ZL_ERR_TIMEOUT after timeout_ms (< 0: no limit).
+ * Also reports device-side argument errors (ids or labels out of range) of that work. */
+zl_status zl_synchronize(zl_ctx* ctx, int timeout_ms);
+
+/* Device bytes held by the context: peak since creation or the last reset, and now
+ * (parameters and optimizer state plus the activation pool's high-water mark). */
+zl_status zl_peak_bytes(zl_ctx* ctx, size_t* peak, size_t* current);
+zl_status zl_reset_peak(zl_ctx* ctx);
+
+/* Message of the last failed call on this thread (owned by the library). */
+const char* zl_last_error(void);
+
+/* Instrumentation. zl_profile(ctx, 1) brackets every kernel the context launches with CUDA
+ * events on the launching stream; zl_profile_read waits for queued work and writes a JSON
+ * object {class: {"launches", "ms", "flops", "bytes"}} (algorithmic FLOPs / HBM bytes of those
+ * launches) into buf (NUL-terminated, truncated to cap), then clears the records.
+ * zl_kernel_launches returns how many kernels the library has launched in this process. */
+zl_status zl_profile(zl_ctx* ctx, int on);
+zl_status zl_profile_read(zl_ctx* ctx, char* buf, size_t cap);
+zl_status zl_kernel_launches(uint64_t* count);
+
+/* ---------------------------------------------------------------------------------------
+ * Single-kernel entry points (used by the tests and the roofline measurement). All
+ * pointers are device pointers; `stream` is a cudaStream_t (NULL = legacy default).
+ * ------------------------------------------------------------------------------------- */
+
+/* Fused local objective (Eq. 3-5) over N rows of logits. z, t: [N, ldz] in `dtype`
+ * (columns >= V are padding and ignored); t may be NULL when alpha == 1.
+ * labels: [N] int32. Writes dz = dL/dz [N, ldz] (dtype; padding columns 0) and
+ * row_loss[N] (fp32, alpha*CE_i + (1-alpha)*KL_i, 0 outside Omega), and *loss
+ * (one fp32 on the device) = sum(row_loss) / |Omega|. */
+zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_t* labels, int N,
+                           int V, int ldz, float alpha, int kl_dir, void* dz, float* row_loss,
+                           float* loss, void* stream);
+
+/* C[M,N] (+)= A[M,K] . B^T where B is [N,K] (mode 0, "forward"), or A[M,K] . B with B
+ * [K,N] (mode 1, "dX"), or C[M,N] += A^T . B with A [K,M], B [K,N] (mode 2, "dW",
+ * C fp32 and always accumulated). dtype of A, B and (modes 0/1) C. Row-major, dense. */
+zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C,
+                     void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ZEROLOCK_H */

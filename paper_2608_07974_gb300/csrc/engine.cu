@@ -1,0 +1,1297 @@
+// ZeroLock engine behind the C ABI of include/zerolock.h: parameter slabs, the chunk forward /
+// local backward (Section II-A, Remark 1), the readout and local objective (Eq. 2-5), AdamW
+// (Eq. 6 as AdamW), and the K-stream scheduler with early forwarding, per-entry readiness
+// events and a bound on live activation arenas (Section III-A/B).
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cstdio>
+#include <chrono>
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include "common.cuh"
+#include "ops.h"
+#include "zerolock.h"
+
+namespace zl {
+static std::atomic<unsigned long long> g_launches{0};
+void note_launch(int n) { g_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed); }
+unsigned long long launches_so_far() { return g_launches.load(std::memory_order_relaxed); }
+}  // namespace zl
+
+namespace {
+
+using namespace zl;
+
+// Kernel classes of the per-launch profile (zl_profile).
+enum { PC_GEMM, PC_ATTN_F, PC_ATTN_B, PC_LOSS, PC_NORM, PC_ADAMW, PC_ELEM, PC_COUNT };
+const char* kPCName[PC_COUNT] = {"gemm", "attn_fwd", "attn_bwd", "local_loss", "norm", "adamw", "elementwise"};
+struct ProfRec {
+  int cls;
+  cudaEvent_t a, b;
+  double flops, bytes, launches;
+};
+
+thread_local std::string g_err;
+
+struct ZlError {
+  zl_status st;
+  std::string msg;
+};
+[[noreturn]] void raise_err(zl_status st, const std::string& msg) { throw ZlError{st, msg}; }
+
+bool sticky(cudaError_t e) {
+  return e == cudaErrorIllegalAddress || e == cudaErrorLaunchFailure || e == cudaErrorIllegalInstruction ||
+         e == cudaErrorMisalignedAddress || e == cudaErrorHardwareStackError || e == cudaErrorAssert ||
+         e == cudaErrorInvalidPc || e == cudaErrorInvalidAddressSpace;
+}
+
+#define CK(call)                                                                                  \
+  do {                                                                                            \
+    cudaError_t e_ = (call);                                                                      \
+    if (e_ != cudaSuccess) {                                                                      \
+      raise_err(e_ == cudaErrorMemoryAllocation ? ZL_ERR_OOM : (sticky(e_) ? ZL_ERR_STATE : ZL_ERR_CUDA), \
+                std::string(#call) + " failed: " + cudaGetErrorString(e_));                       \
+    }                                                                                             \
+  } while (0)
+
+#define CHECK_LAUNCH() CK(cudaGetLastError())
+
+// ----------------------------------------------------------------------------------------------
+// Parameter layout: per layer a fixed list of tensors, stored in one contiguous slab per chunk
+// (fp32 master, gradient, AdamW m and v; plus a bf16 compute copy in bf16 mode).
+// ----------------------------------------------------------------------------------------------
+enum PK { P_N1W, P_N1B, P_WQKV, P_BQKV, P_WO, P_BO, P_N2W, P_N2B, P_W1, P_B1, P_W2, P_B2, P_COUNT };
+const char* kPName[P_COUNT] = {"attn_norm.weight", "attn_norm.bias", "wqkv", "bqkv", "wo", "bo",
+                               "ffn_norm.weight", "ffn_norm.bias", "w1", "b1", "w2", "b2"};
+
+struct Layer {
+  size_t off[P_COUNT];
+  size_t numel[P_COUNT];
+  bool has[P_COUNT];
+};
+
+struct Chunk {
+  int k = 0, l0 = 0, l1 = 0;
+  size_t n = 0;
+  float *master = nullptr, *grad = nullptr, *m = nullptr, *v = nullptr;
+  void* comp = nullptr;
+  std::vector<Layer> layers;
+  int micro = 0;
+  long t = 0;
+  cudaStream_t s = nullptr;
+  cudaEvent_t ev_h = nullptr, ev_z = nullptr, ev_loss = nullptr, ev_hb = nullptr, ev_done = nullptr;
+};
+
+// Saved activations of one layer (pointers into the chunk's arena).
+struct LayerSave {
+  const void* x = nullptr;   // layer input
+  void *xn1, *qkv, *att, *x2, *xn2, *hid, *act, *y;
+  float *rstd1, *mean1, *rstd2, *mean2, *lse;
+};
+
+}  // namespace
+
+struct zl_ctx {
+  zl_model_dims dims;
+  zl_train_cfg cfg;
+  int K = 0;
+  std::vector<int> bounds;
+  int dt = 0;
+  bool llama = true;
+  int d = 0, hd = 0, H = 0, Hkv = 0, qkvw = 0, ad = 0, f = 0, f1 = 0, V = 0, Vp = 0;
+  std::vector<Chunk> ch;   // ch[1..K]
+  void *tok_emb = nullptr, *pos_emb = nullptr, *lm_head = nullptr;
+  float *normf_w = nullptr, *normf_b = nullptr;
+  float* rope_cs = nullptr;
+  cudaMemPool_t pool = nullptr;
+  size_t static_bytes = 0;
+  cudaStream_t user = nullptr, aux = nullptr;
+  cudaEvent_t ev_start = nullptr, ev_aux = nullptr, ev_sync = nullptr;
+  std::vector<cudaEvent_t> live_ring;
+  long live_seq = 0;
+  unsigned* d_err = nullptr;
+  int* d_count = nullptr;        // [K + 1] one |Omega| per stream
+  float* d_losses = nullptr;     // [K + 1]
+  float* h_losses = nullptr;     // pinned [K + 1]
+  int last_nloss = 0;
+  bool broken = false;
+  std::vector<void*> statics;
+  bool prof = false;
+  std::vector<ProfRec> recs;
+  std::vector<cudaEvent_t> evpool;
+  size_t evnext = 0;
+};
+
+namespace {
+
+// ----------------------------------------------------------------------------------------------
+// small helpers
+// ----------------------------------------------------------------------------------------------
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+void* salloc(zl_ctx* c, size_t bytes) {
+  void* p = nullptr;
+  CK(cudaMalloc(&p, std::max<size_t>(bytes, 256)));
+  c->statics.push_back(p);
+  c->static_bytes += std::max<size_t>(bytes, 256);
+  return p;
+}
+
+void* palloc(zl_ctx* c, size_t bytes, cudaStream_t s) {
+  void* p = nullptr;
+  CK(cudaMallocFromPoolAsync(&p, std::max<size_t>(bytes, 256), c->pool, s));
+  return p;
+}
+void pfree(void* p, cudaStream_t s) {
+  if (p) CK(cudaFreeAsync(p, s));
+}
+
+// A bump allocator over one pool allocation (256-byte aligned pieces).
+struct Arena {
+  char* base = nullptr;
+  size_t used = 0, cap = 0;
+  void* take(size_t bytes) {
+    void* p = base + used;
+    used += round_up(std::max<size_t>(bytes, 1), 256);
+    if (used > cap) raise_err(ZL_ERR_STATE, "internal: arena overflow");
+    return p;
+  }
+};
+
+const void* Wc(zl_ctx* c, Chunk& k, int li, PK p) {   // compute-dtype pointer of a matrix
+  const size_t off = k.layers[li].off[p];
+  return c->dt == BF16 ? (const void*)((const bf16*)k.comp + off) : (const void*)(k.master + off);
+}
+float* Wm(Chunk& k, int li, PK p) { return k.layers[li].has[p] ? k.master + k.layers[li].off[p] : nullptr; }
+float* Gm(Chunk& k, int li, PK p) { return k.layers[li].has[p] ? k.grad + k.layers[li].off[p] : nullptr; }
+
+size_t esz(zl_ctx* c) { return dt_size(c->dt); }
+
+void wait_ev(cudaStream_t s, cudaEvent_t e) { CK(cudaStreamWaitEvent(s, e, 0)); }
+void rec(cudaEvent_t e, cudaStream_t s) { CK(cudaEventRecord(e, s)); }
+
+cudaEvent_t take_ev(zl_ctx* c) {
+  if (c->evnext == c->evpool.size()) {
+    cudaEvent_t e;
+    CK(cudaEventCreate(&e));
+    c->evpool.push_back(e);
+  }
+  return c->evpool[c->evnext++];
+}
+
+// Brackets the launches of its scope with timing events when the context profiles.
+struct ProfScope {
+  zl_ctx* c;
+  cudaStream_t s;
+  int cls;
+  double flops, bytes, launches;
+  cudaEvent_t a = nullptr;
+  ProfScope(zl_ctx* c_, cudaStream_t s_, int cls_, double fl, double by, double nl = 1)
+      : c(c_), s(s_), cls(cls_), flops(fl), bytes(by), launches(nl) {
+    if (c->prof) {
+      a = take_ev(c);
+      CK(cudaEventRecord(a, s));
+    }
+  }
+  ~ProfScope() {
+    if (!a) return;
+    if (c->evnext == c->evpool.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return;
+      c->evpool.push_back(e);
+    }
+    cudaEvent_t b = c->evpool[c->evnext++];
+    cudaEventRecord(b, s);
+    c->recs.push_back(ProfRec{cls, a, b, flops, bytes, launches});
+  }
+};
+
+// ----------------------------------------------------------------------------------------------
+// Profiled launch wrappers (algorithmic FLOPs / bytes per launch)
+// ----------------------------------------------------------------------------------------------
+void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, const void* B, void* C,
+       const float* bias, const void* R) {
+  const double e = (double)esz(c);
+  const double out = mode == 2 ? 8.0 * M * N : (R ? 2.0 : 1.0) * e * M * N;
+  ProfScope p(c, s, PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
+  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s);
+}
+void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
+  const double e = (double)esz(c), N = (double)B * S;
+  ProfScope p(c, s, PC_ATTN_F, 2.0 * B * c->H * (double)S * S * c->hd, e * N * (c->qkvw + c->ad));
+  attn_fwd(c->dt, qkv, out, lse, B, S, c->H, c->Hkv, c->hd, s);
+}
+void AB(zl_ctx* c, cudaStream_t s, const void* qkv, const void* out, const void* dout, const float* lse, float* D,
+        void* dqkv, int B, int S) {
+  const double e = (double)esz(c), N = (double)B * S;
+  ProfScope p(c, s, PC_ATTN_B, 4.0 * B * c->H * (double)S * S * c->hd, e * N * (2.0 * c->qkvw + 2.0 * c->ad), 3);
+  attn_bwd(c->dt, qkv, out, dout, lse, D, dqkv, B, S, c->H, c->Hkv, c->hd, s);
+}
+void NF(zl_ctx* c, cudaStream_t s, const void* x, const float* g, const float* b, void* y, float* rstd, float* mean,
+        int N) {
+  ProfScope p(c, s, PC_NORM, 0, 2.0 * esz(c) * (double)N * c->d);
+  launch_norm_fwd(c->dt, !c->llama, x, g, b, y, rstd, mean, N, c->d, c->dims.norm_eps, s);
+}
+void NBX(zl_ctx* c, cudaStream_t s, const void* x, const float* g, const float* rstd, const float* mean, const void* dy,
+         const void* dres, void* dx, int N) {
+  ProfScope p(c, s, PC_NORM, 0, (dres ? 4.0 : 3.0) * esz(c) * (double)N * c->d);
+  launch_norm_bwd_dx(c->dt, !c->llama, x, g, rstd, mean, dy, dres, dx, N, c->d, s);
+}
+// ----------------------------------------------------------------------------------------------
+// Layer forward / backward
+// ----------------------------------------------------------------------------------------------
+size_t layer_save_bytes(zl_ctx* c, int N, int B, int S, bool with_y) {
+  const size_t e = esz(c);
+  size_t b = 0;
+  auto add = [&](size_t x) { b += round_up(std::max<size_t>(x, 1), 256); };
+  add((size_t)N * c->d * e);        // xn1
+  add((size_t)N * c->qkvw * e);     // qkv
+  add((size_t)N * c->ad * e);       // att
+  add((size_t)N * c->d * e);        // x2
+  add((size_t)N * c->d * e);        // xn2
+  add((size_t)N * c->f1 * e);       // hid
+  add((size_t)N * c->f * e);        // act
+  if (with_y) add((size_t)N * c->d * e);
+  for (int i = 0; i < 4; ++i) add((size_t)N * 4);
+  add((size_t)B * c->H * S * 4);    // lse
+  return b;
+}
+
+void carve_layer(zl_ctx* c, Arena& a, LayerSave& sv, int N, int B, int S, bool with_y) {
+  const size_t e = esz(c);
+  sv.xn1 = a.take((size_t)N * c->d * e);
+  sv.qkv = a.take((size_t)N * c->qkvw * e);
+  sv.att = a.take((size_t)N * c->ad * e);
+  sv.x2 = a.take((size_t)N * c->d * e);
+  sv.xn2 = a.take((size_t)N * c->d * e);
+  sv.hid = a.take((size_t)N * c->f1 * e);
+  sv.act = a.take((size_t)N * c->f * e);
+  sv.y = with_y ? a.take((size_t)N * c->d * e) : nullptr;
+  sv.rstd1 = (float*)a.take((size_t)N * 4);
+  sv.mean1 = (float*)a.take((size_t)N * 4);
+  sv.rstd2 = (float*)a.take((size_t)N * 4);
+  sv.mean2 = (float*)a.take((size_t)N * 4);
+  sv.lse = (float*)a.take((size_t)B * c->H * S * 4);
+}
+
+void layer_fwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* x, void* y, int B, int S, cudaStream_t s) {
+  const int N = B * S, dt = c->dt;
+  sv.x = x;
+  NF(c, s, x, Wm(k, li, P_N1W), Wm(k, li, P_N1B), sv.xn1, sv.rstd1, sv.mean1, N);
+  G(c, s, 0, N, c->qkvw, c->d, sv.xn1, Wc(c, k, li, P_WQKV), sv.qkv, Wm(k, li, P_BQKV), nullptr);
+  if (c->llama) {
+    ProfScope p(c, s, PC_ELEM, 0, 2.0 * esz(c) * (double)N * (c->H + c->Hkv) * c->hd);
+    launch_rope(dt, sv.qkv, c->rope_cs, N, S, c->H, c->Hkv, c->hd, 0, s);
+  }
+  AF(c, s, sv.qkv, sv.att, sv.lse, B, S);
+  G(c, s, 0, N, c->d, c->ad, sv.att, Wc(c, k, li, P_WO), sv.x2, Wm(k, li, P_BO), x);
+  NF(c, s, sv.x2, Wm(k, li, P_N2W), Wm(k, li, P_N2B), sv.xn2, sv.rstd2, sv.mean2, N);
+  G(c, s, 0, N, c->f1, c->d, sv.xn2, Wc(c, k, li, P_W1), sv.hid, Wm(k, li, P_B1), nullptr);
+  {
+    ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * (c->f1 + c->f));
+    if (c->llama) launch_swiglu_fwd(dt, sv.hid, sv.act, N, c->f, s);
+    else launch_gelu_fwd(dt, sv.hid, sv.act, (size_t)N * c->f, s);
+  }
+  G(c, s, 0, N, c->d, c->f, sv.act, Wc(c, k, li, P_W2), y, Wm(k, li, P_B2), sv.x2);
+  CHECK_LAUNCH();
+}
+
+// Backward workspace of one chunk.
+struct BwdWs {
+  void *da, *dhid, *dxn, *dx2, *datt, *dqkv, *dy0, *dy1;
+  float *part_g, *part_b, *D;
+};
+
+size_t bwd_ws_bytes(zl_ctx* c, int N, int B, int S) {
+  const size_t e = esz(c);
+  const size_t wmax = std::max({(size_t)c->d, (size_t)c->qkvw, (size_t)c->f1, (size_t)c->f});
+  size_t b = 0;
+  auto add = [&](size_t x) { b += round_up(std::max<size_t>(x, 1), 256); };
+  add((size_t)N * c->f * e);
+  add((size_t)N * c->f1 * e);
+  add((size_t)N * c->d * e);
+  add((size_t)N * c->d * e);
+  add((size_t)N * c->ad * e);
+  add((size_t)N * c->qkvw * e);
+  add((size_t)N * c->d * e);
+  add((size_t)N * c->d * e);
+  add((size_t)colsum_blocks(N) * wmax * 4);
+  add((size_t)colsum_blocks(N) * wmax * 4);
+  add((size_t)B * c->H * S * 4);
+  return b;
+}
+
+void carve_ws(zl_ctx* c, Arena& a, BwdWs& w, int N, int B, int S) {
+  const size_t e = esz(c);
+  const size_t wmax = std::max({(size_t)c->d, (size_t)c->qkvw, (size_t)c->f1, (size_t)c->f});
+  w.da = a.take((size_t)N * c->f * e);
+  w.dhid = a.take((size_t)N * c->f1 * e);
+  w.dxn = a.take((size_t)N * c->d * e);
+  w.dx2 = a.take((size_t)N * c->d * e);
+  w.datt = a.take((size_t)N * c->ad * e);
+  w.dqkv = a.take((size_t)N * c->qkvw * e);
+  w.dy0 = a.take((size_t)N * c->d * e);
+  w.dy1 = a.take((size_t)N * c->d * e);
+  w.part_g = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
+  w.part_b = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
+  w.D = (float*)a.take((size_t)B * c->H * S * 4);
+}
+
+void bias_grad(zl_ctx* c, const void* dY, int N, int cols, float* g, BwdWs& w, cudaStream_t s) {
+  if (!g) return;
+  ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * cols, 2);
+  launch_colsum(c->dt, dY, w.part_b, N, cols, s);
+  launch_partials_add(w.part_b, colsum_blocks(N), cols, g, s);
+}
+
+void norm_param_grad(zl_ctx* c, const void* x, const float* rstd, const float* mean, const void* dyn, int N,
+                     float* gw, float* gb, BwdWs& w, cudaStream_t s) {
+  const bool ln = !c->llama;
+  ProfScope p(c, s, PC_NORM, 0, 2.0 * esz(c) * (double)N * c->d, ln ? 3 : 2);
+  launch_norm_bwd_dparam(c->dt, ln, x, rstd, mean, dyn, w.part_g, w.part_b, N, c->d, s);
+  launch_partials_add(w.part_g, colsum_blocks(N), c->d, gw, s);
+  if (ln) launch_partials_add(w.part_b, colsum_blocks(N), c->d, gb, s);
+}
+
+// dy: gradient w.r.t. the layer output; dx (may be NULL): gradient w.r.t. the layer input.
+void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void* dx, BwdWs& w, int B, int S,
+               cudaStream_t s) {
+  const int N = B * S, dt = c->dt;
+  // FFN
+  G(c, s, 2, c->d, c->f, N, dy, sv.act, Gm(k, li, P_W2), nullptr, nullptr);
+  bias_grad(c, dy, N, c->d, Gm(k, li, P_B2), w, s);
+  G(c, s, 1, N, c->f, c->d, dy, Wc(c, k, li, P_W2), w.da, nullptr, nullptr);
+  {
+    ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * (2.0 * c->f1 + c->f));
+    if (c->llama) launch_swiglu_bwd(dt, sv.hid, w.da, w.dhid, N, c->f, s);
+    else launch_gelu_bwd(dt, sv.hid, w.da, w.dhid, (size_t)N * c->f, s);
+  }
+  G(c, s, 2, c->f1, c->d, N, w.dhid, sv.xn2, Gm(k, li, P_W1), nullptr, nullptr);
+  bias_grad(c, w.dhid, N, c->f1, Gm(k, li, P_B1), w, s);
+  G(c, s, 1, N, c->d, c->f1, w.dhid, Wc(c, k, li, P_W1), w.dxn, nullptr, nullptr);
+  NBX(c, s, sv.x2, Wm(k, li, P_N2W), sv.rstd2, sv.mean2, w.dxn, dy, w.dx2, N);
+  norm_param_grad(c, sv.x2, sv.rstd2, sv.mean2, w.dxn, N, Gm(k, li, P_N2W), Gm(k, li, P_N2B), w, s);
+  // attention
+  G(c, s, 2, c->d, c->ad, N, w.dx2, sv.att, Gm(k, li, P_WO), nullptr, nullptr);
+  bias_grad(c, w.dx2, N, c->d, Gm(k, li, P_BO), w, s);
+  G(c, s, 1, N, c->ad, c->d, w.dx2, Wc(c, k, li, P_WO), w.datt, nullptr, nullptr);
+  AB(c, s, sv.qkv, sv.att, w.datt, sv.lse, w.D, w.dqkv, B, S);
+  if (c->llama) {
+    ProfScope p(c, s, PC_ELEM, 0, 2.0 * esz(c) * (double)N * (c->H + c->Hkv) * c->hd);
+    launch_rope(dt, w.dqkv, c->rope_cs, N, S, c->H, c->Hkv, c->hd, 1, s);
+  }
+  G(c, s, 2, c->qkvw, c->d, N, w.dqkv, sv.xn1, Gm(k, li, P_WQKV), nullptr, nullptr);
+  bias_grad(c, w.dqkv, N, c->qkvw, Gm(k, li, P_BQKV), w, s);
+  G(c, s, 1, N, c->d, c->qkvw, w.dqkv, Wc(c, k, li, P_WQKV), w.dxn, nullptr, nullptr);
+  norm_param_grad(c, sv.x, sv.rstd1, sv.mean1, w.dxn, N, Gm(k, li, P_N1W), Gm(k, li, P_N1B), w, s);
+  if (dx) NBX(c, s, sv.x, Wm(k, li, P_N1W), sv.rstd1, sv.mean1, w.dxn, w.dx2, dx, N);
+  CHECK_LAUNCH();
+}
+
+// ----------------------------------------------------------------------------------------------
+// Chunk forward (saving or not) and the chunk backward
+// ----------------------------------------------------------------------------------------------
+struct ChunkActs {
+  void* mem = nullptr;
+  std::vector<LayerSave> L;
+};
+
+// Saving forward: the arena holds every layer's activations; the chunk output goes to h_out.
+void chunk_fwd_save(zl_ctx* c, Chunk& k, const void* h_in, void* h_out, int B, int S, ChunkActs& acts,
+                    cudaStream_t s) {
+  const int N = B * S, nl = k.l1 - k.l0;
+  size_t bytes = 0;
+  for (int i = 0; i < nl; ++i) bytes += layer_save_bytes(c, N, B, S, i + 1 < nl);
+  Arena a;
+  a.base = (char*)palloc(c, bytes, s);
+  a.cap = bytes;
+  acts.mem = a.base;
+  acts.L.assign(nl, LayerSave{});
+  const void* x = h_in;
+  for (int i = 0; i < nl; ++i) {
+    carve_layer(c, a, acts.L[i], N, B, S, i + 1 < nl);
+    void* y = i + 1 < nl ? acts.L[i].y : h_out;
+    layer_fwd(c, k, i, acts.L[i], x, y, B, S, s);
+    x = y;
+  }
+}
+
+// Forward without saving (one transient layer workspace, ping-pong outputs).
+void chunk_fwd_nosave(zl_ctx* c, Chunk& k, const void* h_in, void* h_out, int B, int S, cudaStream_t s) {
+  const int N = B * S, nl = k.l1 - k.l0;
+  const size_t lb = layer_save_bytes(c, N, B, S, true) + round_up((size_t)N * c->d * esz(c), 256);
+  Arena a;
+  a.base = (char*)palloc(c, lb, s);
+  a.cap = lb;
+  LayerSave sv;
+  carve_layer(c, a, sv, N, B, S, true);
+  void* pong = a.take((size_t)N * c->d * esz(c));
+  const void* x = h_in;
+  for (int i = 0; i < nl; ++i) {
+    void* y = (i + 1 == nl) ? h_out : ((i % 2 == 0) ? sv.y : pong);
+    layer_fwd(c, k, i, sv, x, y, B, S, s);
+    x = y;
+  }
+  pfree(a.base, s);
+}
+
+// Backward through the chunk from dh (gradient at its output). dh_in (may be NULL) receives the
+// gradient at its input (only the backpropagation baseline needs it).
+void chunk_bwd(zl_ctx* c, Chunk& k, ChunkActs& acts, const void* dh, void* dh_in, int B, int S, cudaStream_t s) {
+  const int N = B * S, nl = k.l1 - k.l0;
+  const size_t wb = bwd_ws_bytes(c, N, B, S);
+  Arena a;
+  a.base = (char*)palloc(c, wb, s);
+  a.cap = wb;
+  BwdWs w;
+  carve_ws(c, a, w, N, B, S);
+  const void* dy = dh;
+  for (int i = nl - 1; i >= 0; --i) {
+    void* dx = i > 0 ? ((i % 2) ? w.dy0 : w.dy1) : dh_in;
+    layer_bwd(c, k, i, acts.L[i], dy, dx, w, B, S, s);
+    dy = dx;
+  }
+  pfree(a.base, s);
+}
+
+void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s) {
+  k.micro += 1;
+  if (k.micro < c->cfg.accum_m) return;
+  k.t += 1;
+  const zl_train_cfg& g = c->cfg;
+  double lr = g.lr;
+  if (g.lr_schedule == 1) lr = g.lr / std::sqrt((double)(k.t - 1) + g.lr_gamma);
+  const double bc1 = 1.0 - std::pow((double)g.beta1, (double)k.t);
+  const double bc2 = 1.0 - std::pow((double)g.beta2, (double)k.t);
+  ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * (double)k.n);
+  launch_adamw(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, k.n, (float)lr, g.beta1, g.beta2, g.eps,
+               g.weight_decay, (float)bc1, (float)bc2, 1.f / (float)g.accum_m, s);
+  CHECK_LAUNCH();
+  k.micro = 0;
+}
+
+float alpha_of(zl_ctx* c, int k) { return (k == 1 && !c->cfg.consis_first) ? 1.f : c->cfg.alpha; }
+
+// ----------------------------------------------------------------------------------------------
+// Readout (Eq. 2) and its backward (frozen head: no parameter gradient)
+// ----------------------------------------------------------------------------------------------
+struct ReadoutSave {
+  void* n = nullptr;
+  float *rstd = nullptr, *mean = nullptr;
+};
+
+void readout_fwd(zl_ctx* c, const void* h, void* z, ReadoutSave* keep, int N, cudaStream_t s) {
+  const size_t e = esz(c);
+  void* n = palloc(c, (size_t)N * c->d * e, s);
+  float* st = (float*)palloc(c, (size_t)N * 8, s);
+  NF(c, s, h, c->normf_w, c->normf_b, n, st, st + N, N);
+  G(c, s, 0, N, c->Vp, c->d, n, c->lm_head, z, nullptr, nullptr);
+  CHECK_LAUNCH();
+  if (keep) {
+    keep->n = n;
+    keep->rstd = st;
+    keep->mean = st + N;
+  } else {
+    pfree(n, s);
+    pfree(st, s);
+  }
+}
+
+// dh = Norm_f'(h)^T (dz W_lm)
+void readout_bwd(zl_ctx* c, const void* h, ReadoutSave& rs, const void* dz, void* dh, int N, cudaStream_t s) {
+  G(c, s, 1, N, c->d, c->Vp, dz, c->lm_head, rs.n, nullptr, nullptr);   // reuse n as dn
+  NBX(c, s, h, c->normf_w, rs.rstd, rs.mean, rs.n, nullptr, dh, N);
+  CHECK_LAUNCH();
+  pfree(rs.n, s);
+  pfree(rs.rstd, s);
+  rs = ReadoutSave{};
+}
+
+// Loss of chunk slot `slot` into d_losses[slot]; returns dz (pool memory, caller frees).
+void* local_loss(zl_ctx* c, const void* z, const void* t, const int32_t* labels, float alpha, int N, int slot,
+                 cudaStream_t s) {
+  void* dz = palloc(c, (size_t)N * c->Vp * esz(c), s);
+  float* rl = (float*)palloc(c, (size_t)N * 4, s);
+  launch_count_valid(labels, N, c->V, c->d_count + slot, c->d_err, s);
+  {
+    ProfScope p(c, s, PC_LOSS, 0, (alpha < 1.f ? 3.0 : 2.0) * esz(c) * (double)N * c->Vp);
+    launch_local_loss(c->dt, z, alpha < 1.f ? t : nullptr, labels, N, c->V, c->Vp, alpha, c->cfg.kl_dir,
+                      c->d_count + slot, dz, rl, s);
+  }
+  launch_loss_reduce(rl, N, c->d_count + slot, c->d_losses + slot, s);
+  CHECK_LAUNCH();
+  pfree(rl, s);
+  return dz;
+}
+
+// ----------------------------------------------------------------------------------------------
+// synchronisation
+// ----------------------------------------------------------------------------------------------
+void join_all(zl_ctx* c) {
+  for (int k = 1; k <= c->K; ++k) {
+    rec(c->ch[k].ev_done, c->ch[k].s);
+    wait_ev(c->user, c->ch[k].ev_done);
+  }
+  rec(c->ev_aux, c->aux);
+  wait_ev(c->user, c->ev_aux);
+}
+
+zl_status sync_all(zl_ctx* c, int timeout_ms) {
+  join_all(c);
+  rec(c->ev_sync, c->user);
+  const auto t0 = std::chrono::steady_clock::now();
+  for (;;) {
+    cudaError_t e = cudaEventQuery(c->ev_sync);
+    if (e == cudaSuccess) break;
+    if (e != cudaErrorNotReady) CK(e);
+    if (timeout_ms >= 0 &&
+        std::chrono::duration_cast<std::chrono::milliseconds>(std::chrono::steady_clock::now() - t0).count() >
+            timeout_ms)
+      raise_err(ZL_ERR_TIMEOUT, "zl_synchronize: queued work did not finish in time");
+    std::this_thread::sleep_for(std::chrono::microseconds(50));
+  }
+  unsigned err = 0;
+  CK(cudaMemcpy(&err, c->d_err, 4, cudaMemcpyDeviceToHost));
+  if (err) {
+    CK(cudaMemset(c->d_err, 0, 4));
+    std::string m = "device-side argument error:";
+    if (err & ZL_DEVERR_BAD_ID) m += " token id out of [0, vocab);";
+    if (err & ZL_DEVERR_BAD_LABEL) m += " label out of [-1, vocab);";
+    if (err & ZL_DEVERR_TIMEOUT) m += " bounded wait expired in a kernel;";
+    raise_err(ZL_ERR_ARG, m);
+  }
+  return ZL_OK;
+}
+
+void start_on(zl_ctx* c, cudaStream_t s) {   // order s after the user's stream
+  rec(c->ev_start, c->user);
+  wait_ev(s, c->ev_start);
+}
+
+void check_bs(zl_ctx* c, int B, int S) {
+  if (B <= 0 || S <= 0) raise_err(ZL_ERR_ARG, "empty micro-batch (B and S must be >= 1)");
+  if (S > c->dims.max_seq) raise_err(ZL_ERR_ARG, "S exceeds max_seq");
+  if ((long)B * S > (1L << 26)) raise_err(ZL_ERR_ARG, "B*S too large");
+}
+
+// ----------------------------------------------------------------------------------------------
+// Name lookup
+// ----------------------------------------------------------------------------------------------
+struct Found {
+  void* dev = nullptr;          // compute-dtype or fp32 pointer of the tensor
+  bool fp32 = true;
+  size_t numel = 0;
+  Chunk* chunk = nullptr;       // trainable: owning chunk
+  size_t off = 0;
+  int frozen = 0;               // 1 tok_emb, 2 pos_emb, 3 norm_f.weight, 4 norm_f.bias, 5 lm_head
+};
+
+bool lookup(zl_ctx* c, const std::string& name, Found& f) {
+  const size_t Vd = (size_t)c->V * c->d;
+  if (name == "tok_emb") { f = Found{c->tok_emb, c->dt == F32, Vd, nullptr, 0, 1}; return true; }
+  if (name == "pos_emb" && !c->llama) {
+    f = Found{c->pos_emb, c->dt == F32, (size_t)c->dims.max_seq * c->d, nullptr, 0, 2};
+    return true;
+  }
+  if (name == "norm_f.weight") { f = Found{c->normf_w, true, (size_t)c->d, nullptr, 0, 3}; return true; }
+  if (name == "norm_f.bias" && !c->llama) { f = Found{c->normf_b, true, (size_t)c->d, nullptr, 0, 4}; return true; }
+  if (name == "lm_head" && c->llama) { f = Found{c->lm_head, c->dt == F32, Vd, nullptr, 0, 5}; return true; }
+  if (name.rfind("layers.", 0) != 0) return false;
+  const size_t dot = name.find('.', 7);
+  if (dot == std::string::npos) return false;
+  int l = -1;
+  try { l = std::stoi(name.substr(7, dot - 7)); } catch (...) { return false; }
+  if (l < 0 || l >= c->dims.n_layers) return false;
+  const std::string suf = name.substr(dot + 1);
+  for (int k = 1; k <= c->K; ++k) {
+    Chunk& ck = c->ch[k];
+    if (l < ck.l0 || l >= ck.l1) continue;
+    const Layer& L = ck.layers[l - ck.l0];
+    for (int p = 0; p < P_COUNT; ++p)
+      if (L.has[p] && suf == kPName[p]) {
+        f = Found{ck.master + L.off[p], true, L.numel[p], &ck, L.off[p], 0};
+        return true;
+      }
+  }
+  return false;
+}
+
+void free_ctx(zl_ctx* c) {
+  if (!c) return;
+  cudaDeviceSynchronize();
+  for (int k = 1; k < (int)c->ch.size(); ++k) {
+    Chunk& ck = c->ch[k];
+    if (ck.s) cudaStreamDestroy(ck.s);
+    for (cudaEvent_t e : {ck.ev_h, ck.ev_z, ck.ev_loss, ck.ev_hb, ck.ev_done})
+      if (e) cudaEventDestroy(e);
+  }
+  for (cudaEvent_t e : c->live_ring) cudaEventDestroy(e);
+  for (cudaEvent_t e : {c->ev_start, c->ev_aux, c->ev_sync})
+    if (e) cudaEventDestroy(e);
+  if (c->aux) cudaStreamDestroy(c->aux);
+  for (void* p : c->statics) cudaFree(p);
+  if (c->h_losses) cudaFreeHost(c->h_losses);
+  if (c->pool) cudaMemPoolDestroy(c->pool);
+  delete c;
+}
+
+template <typename F>
+zl_status guarded(zl_ctx* c, F&& fn) {
+  if (c && c->broken) { g_err = "context unusable after an earlier sticky CUDA error"; return ZL_ERR_STATE; }
+  try {
+    return fn();
+  } catch (const ZlError& e) {
+    g_err = e.msg;
+    if (c && e.st == ZL_ERR_STATE) c->broken = true;
+    return e.st;
+  } catch (const std::exception& e) {
+    g_err = std::string("internal error: ") + e.what();
+    return ZL_ERR_CUDA;
+  }
+}
+
+}  // namespace
+
+// ================================================================================================
+// C ABI
+// ================================================================================================
+extern "C" {
+
+const char* zl_last_error(void) { return g_err.c_str(); }
+
+zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const zl_train_cfg* cfg, zl_ctx** out) {
+  if (!dims || !bounds || !cfg || !out) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  *out = nullptr;
+  const zl_model_dims& D = *dims;
+  std::string why;
+  if (D.arch != ZL_ARCH_LLAMA && D.arch != ZL_ARCH_GPT2) why = "arch";
+  else if (D.dtype != ZL_DTYPE_F32 && D.dtype != ZL_DTYPE_BF16) why = "dtype";
+  else if (D.n_layers < 1 || D.d_model < 8 || D.n_heads < 1 || D.n_kv_heads < 1 || D.d_ff < 8 || D.vocab < 2 ||
+           D.max_seq < 1) why = "non-positive dimension";
+  else if (D.d_model % D.n_heads != 0) why = "d_model must be n_heads * head_dim";
+  else if ((D.d_model / D.n_heads) % 2 != 0 || D.d_model / D.n_heads > 128) why = "head_dim must be even and <= 128";
+  else if (D.n_heads % D.n_kv_heads != 0) why = "n_heads must be a multiple of n_kv_heads";
+  else if (D.arch == ZL_ARCH_GPT2 && D.n_kv_heads != D.n_heads) why = "GPT-2 blocks use n_kv_heads == n_heads";
+  else if (D.d_model % 8 != 0 || D.d_ff % 8 != 0) why = "d_model and d_ff must be multiples of 8";
+  else if (!(D.norm_eps > 0.f)) why = "norm_eps";
+  else if (K < 1 || K > D.n_layers) why = "K must be in [1, n_layers]";
+  else if (bounds[0] != 0 || bounds[K] != D.n_layers) why = "bounds[0] must be 0 and bounds[K] n_layers";
+  else if (!(cfg->alpha > 0.f && cfg->alpha <= 1.f)) why = "alpha must be in (0, 1]";
+  else if (cfg->kl_dir != 0 && cfg->kl_dir != 1) why = "kl_dir must be 0 or 1";
+  else if (cfg->accum_m < 1) why = "accum_m must be >= 1";
+  else if (cfg->max_live_chunks < 0) why = "max_live_chunks must be >= 0";
+  else if (cfg->lr_schedule != 0 && cfg->lr_schedule != 1) why = "lr_schedule";
+  else if (cfg->lr_schedule == 1 && !(cfg->lr_gamma > 0.f)) why = "lr_gamma must be > 0";
+  for (int k = 1; why.empty() && k <= K; ++k)
+    if (bounds[k] <= bounds[k - 1]) why = "bounds must be strictly increasing";
+  if (!why.empty()) { g_err = "zl_create: " + why; return ZL_ERR_ARG; }
+
+  zl_ctx* c = new zl_ctx();
+  zl_status st = guarded(nullptr, [&]() -> zl_status {
+    c->dims = D;
+    c->cfg = *cfg;
+    c->K = K;
+    c->bounds.assign(bounds, bounds + K + 1);
+    c->dt = D.dtype;
+    c->llama = D.arch == ZL_ARCH_LLAMA;
+    c->d = D.d_model;
+    c->H = D.n_heads;
+    c->Hkv = D.n_kv_heads;
+    c->hd = D.d_model / D.n_heads;
+    c->qkvw = (c->H + 2 * c->Hkv) * c->hd;
+    c->ad = c->H * c->hd;
+    c->f = D.d_ff;
+    c->f1 = c->llama ? 2 * D.d_ff : D.d_ff;
+    c->V = D.vocab;
+    c->Vp = (int)round_up((size_t)D.vocab, 128);
+    const size_t e = esz(c);
+
+    int dev = 0;
+    CK(cudaGetDevice(&dev));
+    cudaMemPoolProps props = {};
+    props.allocType = cudaMemAllocationTypePinned;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = dev;
+    CK(cudaMemPoolCreate(&c->pool, &props));
+    uint64_t thr = UINT64_MAX;
+    CK(cudaMemPoolSetAttribute(c->pool, cudaMemPoolAttrReleaseThreshold, &thr));
+
+    // frozen tensors
+    c->tok_emb = salloc(c, (size_t)c->V * c->d * e);
+    CK(cudaMemset(c->tok_emb, 0, (size_t)c->V * c->d * e));
+    if (!c->llama) {
+      c->pos_emb = salloc(c, (size_t)D.max_seq * c->d * e);
+      CK(cudaMemset(c->pos_emb, 0, (size_t)D.max_seq * c->d * e));
+    }
+    c->normf_w = (float*)salloc(c, (size_t)c->d * 4);
+    c->normf_b = (float*)salloc(c, (size_t)c->d * 4);
+    {
+      std::vector<float> ones(c->d, 1.f);
+      CK(cudaMemcpy(c->normf_w, ones.data(), (size_t)c->d * 4, cudaMemcpyHostToDevice));
+      CK(cudaMemset(c->normf_b, 0, (size_t)c->d * 4));
+    }
+    c->lm_head = salloc(c, (size_t)c->Vp * c->d * e);   // padded rows stay zero
+    CK(cudaMemset(c->lm_head, 0, (size_t)c->Vp * c->d * e));
+    if (c->llama) {   // rotary table (cos, sin) for positions 0..max_seq-1, computed in double
+      const int half = c->hd / 2;
+      std::vector<float> cs((size_t)D.max_seq * half * 2);
+      for (int s = 0; s < D.max_seq; ++s)
+        for (int i = 0; i < half; ++i) {
+          const double ang = (double)s * std::pow((double)D.rope_theta, -2.0 * i / c->hd);
+          cs[((size_t)s * half + i) * 2] = (float)std::cos(ang);
+          cs[((size_t)s * half + i) * 2 + 1] = (float)std::sin(ang);
+        }
+      c->rope_cs = (float*)salloc(c, cs.size() * 4);
+      CK(cudaMemcpy(c->rope_cs, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice));
+    }
+
+    // chunks
+    const int d = c->d;
+    c->ch.resize(K + 1);
+    for (int k = 1; k <= K; ++k) {
+      Chunk& ck = c->ch[k];
+      ck.k = k;
+      ck.l0 = bounds[k - 1];
+      ck.l1 = bounds[k];
+      size_t off = 0;
+      for (int l = ck.l0; l < ck.l1; ++l) {
+        Layer L;
+        size_t shp[P_COUNT] = {(size_t)d, (size_t)d, (size_t)c->qkvw * d, (size_t)c->qkvw, (size_t)d * c->ad, (size_t)d,
+                               (size_t)d, (size_t)d, (size_t)c->f1 * d, (size_t)c->f, (size_t)d * c->f, (size_t)d};
+        for (int p = 0; p < P_COUNT; ++p) {
+          const bool bias = (p == P_N1B || p == P_BQKV || p == P_BO || p == P_N2B || p == P_B1 || p == P_B2);
+          L.has[p] = !(c->llama && bias);
+          L.numel[p] = L.has[p] ? shp[p] : 0;
+          L.off[p] = off;
+          if (L.has[p]) off += round_up(shp[p], 64);
+        }
+        ck.layers.push_back(L);
+      }
+      ck.n = std::max<size_t>(off, 64);
+      ck.master = (float*)salloc(c, ck.n * 4);
+      ck.grad = (float*)salloc(c, ck.n * 4);
+      ck.m = (float*)salloc(c, ck.n * 4);
+      ck.v = (float*)salloc(c, ck.n * 4);
+      CK(cudaMemset(ck.master, 0, ck.n * 4));
+      CK(cudaMemset(ck.grad, 0, ck.n * 4));
+      CK(cudaMemset(ck.m, 0, ck.n * 4));
+      CK(cudaMemset(ck.v, 0, ck.n * 4));
+      if (c->dt == BF16) {
+        ck.comp = salloc(c, ck.n * 2);
+        CK(cudaMemset(ck.comp, 0, ck.n * 2));
+      }
+      // norm gains start at one
+      std::vector<float> ones(d, 1.f);
+      for (auto& L : ck.layers)
+        for (PK p : {P_N1W, P_N2W}) CK(cudaMemcpy(ck.master + L.off[p], ones.data(), (size_t)d * 4, cudaMemcpyHostToDevice));
+      if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
+      CK(cudaStreamCreateWithFlags(&ck.s, cudaStreamNonBlocking));
+      for (cudaEvent_t* e2 : {&ck.ev_h, &ck.ev_z, &ck.ev_loss, &ck.ev_hb, &ck.ev_done})
+        CK(cudaEventCreateWithFlags(e2, cudaEventDisableTiming));
+    }
+    CK(cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking));
+    for (cudaEvent_t* e2 : {&c->ev_start, &c->ev_aux, &c->ev_sync}) CK(cudaEventCreateWithFlags(e2, cudaEventDisableTiming));
+    const int cap = cfg->max_live_chunks > 0 ? std::min(cfg->max_live_chunks, K) : K;
+    c->live_ring.resize(cap);
+    for (auto& e2 : c->live_ring) CK(cudaEventCreateWithFlags(&e2, cudaEventDisableTiming));
+    c->d_err = (unsigned*)salloc(c, 4);
+    CK(cudaMemset(c->d_err, 0, 4));
+    c->d_count = (int*)salloc(c, (size_t)(K + 1) * 4);
+    c->d_losses = (float*)salloc(c, (size_t)(K + 1) * 4);
+    CK(cudaMemset(c->d_losses, 0, (size_t)(K + 1) * 4));
+    CK(cudaMallocHost(&c->h_losses, (size_t)(K + 1) * 4));
+    CK(cudaDeviceSynchronize());
+    return ZL_OK;
+  });
+  if (st != ZL_OK) {
+    std::string keep = g_err;
+    free_ctx(c);
+    g_err = keep;
+    return st;
+  }
+  *out = c;
+  return ZL_OK;
+}
+
+void zl_free(zl_ctx* ctx) { free_ctx(ctx); }
+
+zl_status zl_set_stream(zl_ctx* c, void* stream) {
+  if (!c) { g_err = "NULL context"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    c->user = (cudaStream_t)stream;
+    return ZL_OK;
+  });
+}
+
+zl_status zl_param_numel(zl_ctx* c, const char* name, size_t* numel) {
+  if (!c || !name || !numel) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  Found f;
+  if (!lookup(c, name, f)) { *numel = 0; g_err = std::string("unknown tensor ") + name; return ZL_ERR_ARG; }
+  *numel = f.numel;
+  return ZL_OK;
+}
+
+zl_status zl_set_param(zl_ctx* c, const char* name, const void* src, size_t bytes, int on_device) {
+  if (!c || !name || !src) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    Found f;
+    if (!lookup(c, name, f)) raise_err(ZL_ERR_ARG, std::string("unknown tensor ") + name);
+    if (bytes != f.numel * 4) raise_err(ZL_ERR_ARG, std::string("byte count mismatch for ") + name);
+    sync_all(c, -1);
+    const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    if (f.chunk) {
+      CK(cudaMemcpy(f.dev, src, bytes, kind));
+      if (c->dt == BF16) launch_f32_to_bf16((const float*)f.dev, (bf16*)f.chunk->comp + f.off, f.numel, 0);
+    } else if (f.fp32) {
+      CK(cudaMemcpy(f.dev, src, bytes, kind));
+    } else {   // frozen tensor held in bf16
+      float* tmp = nullptr;
+      CK(cudaMalloc(&tmp, bytes));
+      CK(cudaMemcpy(tmp, src, bytes, kind));
+      launch_f32_to_bf16(tmp, f.dev, f.numel, 0);
+      CK(cudaDeviceSynchronize());
+      CK(cudaFree(tmp));
+    }
+    // the LM head copy: lm_head (Llama) or the tied token embedding (GPT-2)
+    if ((f.frozen == 5) || (f.frozen == 1 && !c->llama))
+      CK(cudaMemcpy(c->lm_head, f.dev, (size_t)c->V * c->d * esz(c), cudaMemcpyDeviceToDevice));
+    CK(cudaDeviceSynchronize());
+    return ZL_OK;
+  });
+}
+
+zl_status zl_get_param(zl_ctx* c, const char* name, int which, void* dst, size_t bytes, int on_device) {
+  if (!c || !name || !dst) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    Found f;
+    if (!lookup(c, name, f)) raise_err(ZL_ERR_ARG, std::string("unknown tensor ") + name);
+    if (bytes != f.numel * 4) raise_err(ZL_ERR_ARG, std::string("byte count mismatch for ") + name);
+    if (which < 0 || which > 3 || (which > 0 && !f.chunk)) raise_err(ZL_ERR_ARG, "which: 0..3, 1..3 trainable only");
+    sync_all(c, -1);
+    const void* srcp = f.dev;
+    if (which > 0) {
+      float* base = which == 1 ? f.chunk->grad : which == 2 ? f.chunk->m : f.chunk->v;
+      srcp = base + f.off;
+    }
+    const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+    if (f.fp32 || which > 0) {
+      CK(cudaMemcpy(dst, srcp, bytes, kind));
+    } else {
+      std::vector<uint16_t> h(f.numel);
+      CK(cudaMemcpy(h.data(), srcp, f.numel * 2, cudaMemcpyDeviceToHost));
+      std::vector<float> o(f.numel);
+      for (size_t i = 0; i < f.numel; ++i) {
+        uint32_t u = (uint32_t)h[i] << 16;
+        std::memcpy(&o[i], &u, 4);
+      }
+      CK(cudaMemcpy(dst, o.data(), bytes, on_device ? cudaMemcpyHostToDevice : cudaMemcpyHostToHost));
+    }
+    return ZL_OK;
+  });
+}
+
+zl_status zl_embed(zl_ctx* c, const int32_t* ids, int B, int S, void* h0_out) {
+  if (!c || !ids || !h0_out) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    check_bs(c, B, S);
+    cudaStream_t s = c->ch[1].s;
+    start_on(c, s);
+    launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h0_out, B * S, S, c->d, c->V, c->d_err, s);
+    CHECK_LAUNCH();
+    return ZL_OK;
+  });
+}
+
+zl_status zl_forward_chunk(zl_ctx* c, int k, const void* h_in, const int32_t* ids, void* h_out, int B, int S) {
+  if (!c || !h_out) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    check_bs(c, B, S);
+    if (k < 1 || k > c->K) raise_err(ZL_ERR_ARG, "chunk index out of [1, K]");
+    if (!h_in && (k != 1 || !ids)) raise_err(ZL_ERR_ARG, "h_in may be NULL only for k = 1 with ids");
+    Chunk& ck = c->ch[k];
+    cudaStream_t s = ck.s;
+    start_on(c, s);
+    const int N = B * S;
+    void* h0 = nullptr;
+    if (!h_in) {
+      h0 = palloc(c, (size_t)N * c->d * esz(c), s);
+      launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h0, N, S, c->d, c->V, c->d_err, s);
+      h_in = h0;
+    }
+    chunk_fwd_nosave(c, ck, h_in, h_out, B, S, s);
+    pfree(h0, s);
+    return ZL_OK;
+  });
+}
+
+zl_status zl_local_step(zl_ctx* c, int k, const void* h_in, const int32_t* ids, const int32_t* labels, int B, int S,
+                        void* h_out, float* loss_out) {
+  if (!c || !labels) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    check_bs(c, B, S);
+    if (k < 1 || k > c->K) raise_err(ZL_ERR_ARG, "chunk index out of [1, K]");
+    if (!h_in && (k != 1 || !ids)) raise_err(ZL_ERR_ARG, "h_in may be NULL only for k = 1 with ids");
+    Chunk& ck = c->ch[k];
+    cudaStream_t s = ck.s;
+    start_on(c, s);
+    const int N = B * S;
+    const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+    void* h0 = nullptr;
+    if (!h_in) {
+      h0 = palloc(c, hb, s);
+      launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h0, N, S, c->d, c->V, c->d_err, s);
+      h_in = h0;
+    }
+    const float a = alpha_of(c, k);
+    void* t = nullptr;
+    if (a < 1.f) {   // teacher p_{k-1} = readout(h_{k-1}), recomputed from the detached input
+      t = palloc(c, zb, s);
+      readout_fwd(c, h_in, t, nullptr, N, s);
+    }
+    void* hk = palloc(c, hb, s);
+    ChunkActs acts;
+    chunk_fwd_save(c, ck, h_in, hk, B, S, acts, s);
+    if (h_out) CK(cudaMemcpyAsync(h_out, hk, hb, cudaMemcpyDeviceToDevice, s));
+    void* z = palloc(c, zb, s);
+    ReadoutSave rs;
+    readout_fwd(c, hk, z, &rs, N, s);
+    void* dz = local_loss(c, z, t, labels, a, N, k, s);
+    pfree(z, s);
+    pfree(t, s);
+    void* dh = palloc(c, hb, s);
+    readout_bwd(c, hk, rs, dz, dh, N, s);
+    pfree(dz, s);
+    chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
+    pfree(dh, s);
+    pfree(acts.mem, s);
+    pfree(hk, s);
+    pfree(h0, s);
+    adamw_window(c, ck, s);
+    if (loss_out) {
+      CK(cudaMemcpyAsync(c->h_losses + k, c->d_losses + k, 4, cudaMemcpyDeviceToHost, s));
+      sync_all(c, -1);
+      *loss_out = c->h_losses[k];
+    }
+    return ZL_OK;
+  });
+}
+
+// The concurrent ZeroLock step: chunk k runs on stream s_k; its forward waits only for the
+// readiness event of h_{k-1} (early forwarding), its loss waits for the teacher logits z_{k-1},
+// and at most `cap` chunks hold activation arenas at once.
+zl_status zl_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S, float* losses_out) {
+  if (!c || !ids || !labels) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    check_bs(c, B, S);
+    const int N = B * S, K = c->K;
+    const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+    rec(c->ev_start, c->user);
+    for (int k = 1; k <= K; ++k) wait_ev(c->ch[k].s, c->ev_start);
+    wait_ev(c->aux, c->ev_start);
+    std::vector<void*> h(K + 1, nullptr), z(K + 1, nullptr);
+    // h_0 = E(x) on s_1; the teacher of chunk 1, z_0 = readout(h_0), on the auxiliary stream
+    cudaStream_t s1 = c->ch[1].s;
+    h[0] = palloc(c, hb, s1);
+    launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h[0], N, S, c->d, c->V, c->d_err, s1);
+    CHECK_LAUNCH();
+    rec(c->ch[1].ev_h, s1);   // reused below as "h_0 ready" before chunk 1 records h_1
+    cudaEvent_t ev_h0 = c->ev_aux;
+    const float a1 = alpha_of(c, 1);
+    if (a1 < 1.f) {
+      wait_ev(c->aux, c->ch[1].ev_h);
+      z[0] = palloc(c, zb, c->aux);
+      readout_fwd(c, h[0], z[0], nullptr, N, c->aux);
+    }
+    rec(ev_h0, c->aux);      // z_0 ready (and aux done reading h_0)
+    const int cap = (int)c->live_ring.size();
+    for (int k = 1; k <= K; ++k) {
+      Chunk& ck = c->ch[k];
+      cudaStream_t s = ck.s;
+      const float a = alpha_of(c, k);
+      // S1: the upstream entry (h_{k-1}) and a free arena slot
+      if (k > 1) wait_ev(s, c->ch[k - 1].ev_h);
+      const long seq = c->live_seq++;
+      if (seq >= cap) wait_ev(s, c->live_ring[seq % cap]);
+      // S2: forward, then hand h_k downstream before the local backward (early forwarding)
+      h[k] = palloc(c, hb, s);
+      ChunkActs acts;
+      chunk_fwd_save(c, ck, h[k - 1], h[k], B, S, acts, s);
+      rec(ck.ev_h, s);
+      z[k] = palloc(c, zb, s);
+      ReadoutSave rs;
+      readout_fwd(c, h[k], z[k], &rs, N, s);
+      rec(ck.ev_z, s);
+      // S3: local objective against the stop-gradient teacher z_{k-1}
+      void* teacher = nullptr;
+      if (a < 1.f) {
+        if (k == 1) wait_ev(s, ev_h0);
+        else wait_ev(s, c->ch[k - 1].ev_z);
+        teacher = z[k - 1];
+      }
+      void* dz = local_loss(c, z[k], teacher, labels, a, N, k, s);
+      rec(ck.ev_loss, s);
+      // z_{k-1} is no longer needed once this loss and chunk k-1's own loss are done
+      if (k == 1) {
+        if (z[0]) { wait_ev(s, ev_h0); pfree(z[0], s); }
+      } else {
+        wait_ev(s, c->ch[k - 1].ev_loss);
+        pfree(z[k - 1], s);
+      }
+      if (k == K) pfree(z[K], s);
+      void* dh = palloc(c, hb, s);
+      readout_bwd(c, h[k], rs, dz, dh, N, s);
+      pfree(dz, s);
+      rec(ck.ev_hb, s);
+      chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
+      pfree(dh, s);
+      pfree(acts.mem, s);
+      rec(c->live_ring[seq % cap], s);
+      // h_{k-1}: read by this chunk's backward and by chunk k-1's readout backward
+      if (k == 1) wait_ev(s, ev_h0);
+      else wait_ev(s, c->ch[k - 1].ev_hb);
+      pfree(h[k - 1], s);
+      if (k == K) pfree(h[K], s);
+      adamw_window(c, ck, s);
+    }
+    c->last_nloss = K;
+    if (losses_out) {
+      for (int k = 1; k <= K; ++k)
+        CK(cudaMemcpyAsync(c->h_losses + k, c->d_losses + k, 4, cudaMemcpyDeviceToHost, c->ch[k].s));
+      sync_all(c, -1);
+      for (int k = 1; k <= K; ++k) losses_out[k - 1] = c->h_losses[k];
+    }
+    return ZL_OK;
+  });
+}
+
+// Backpropagation through all chunks (the same kernels, one stream, every arena alive until
+// the backward reaches it).
+zl_status zl_bp_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S, float* loss_out) {
+  if (!c || !ids || !labels) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    check_bs(c, B, S);
+    const int N = B * S, K = c->K;
+    const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+    cudaStream_t s = c->ch[1].s;
+    rec(c->ev_start, c->user);
+    wait_ev(s, c->ev_start);
+    for (int k = 2; k <= K; ++k) {   // previous work of the other chunk streams
+      rec(c->ch[k].ev_done, c->ch[k].s);
+      wait_ev(s, c->ch[k].ev_done);
+    }
+    std::vector<void*> h(K + 1, nullptr);
+    std::vector<ChunkActs> acts(K + 1);
+    h[0] = palloc(c, hb, s);
+    launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h[0], N, S, c->d, c->V, c->d_err, s);
+    for (int k = 1; k <= K; ++k) {
+      h[k] = palloc(c, hb, s);
+      chunk_fwd_save(c, c->ch[k], h[k - 1], h[k], B, S, acts[k], s);
+    }
+    void* z = palloc(c, zb, s);
+    ReadoutSave rs;
+    readout_fwd(c, h[K], z, &rs, N, s);
+    void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
+    pfree(z, s);
+    void* dh = palloc(c, hb, s);
+    void* dh2 = palloc(c, hb, s);
+    readout_bwd(c, h[K], rs, dz, dh, N, s);
+    pfree(dz, s);
+    for (int k = K; k >= 1; --k) {
+      chunk_bwd(c, c->ch[k], acts[k], dh, k > 1 ? dh2 : nullptr, B, S, s);
+      std::swap(dh, dh2);
+      pfree(acts[k].mem, s);
+      pfree(h[k], s);
+    }
+    pfree(h[0], s);
+    pfree(dh, s);
+    pfree(dh2, s);
+    for (int k = 1; k <= K; ++k) {
+      if (k > 1) {   // the optimizer step of chunk k stays on its own stream
+        rec(c->ch[1].ev_done, s);
+        wait_ev(c->ch[k].s, c->ch[1].ev_done);
+      }
+      adamw_window(c, c->ch[k], k == 1 ? s : c->ch[k].s);
+    }
+    c->last_nloss = 1;
+    if (loss_out) {
+      CK(cudaMemcpyAsync(c->h_losses, c->d_losses, 4, cudaMemcpyDeviceToHost, s));
+      sync_all(c, -1);
+      *loss_out = c->h_losses[0];
+    }
+    return ZL_OK;
+  });
+}
+
+zl_status zl_eval_global_loss(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S, float* loss_out) {
+  if (!c || !ids || !labels || !loss_out) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    check_bs(c, B, S);
+    const int N = B * S, K = c->K;
+    const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+    cudaStream_t s = c->aux;
+    rec(c->ev_start, c->user);
+    wait_ev(s, c->ev_start);
+    for (int k = 1; k <= K; ++k) {
+      rec(c->ch[k].ev_done, c->ch[k].s);
+      wait_ev(s, c->ch[k].ev_done);
+    }
+    void* a = palloc(c, hb, s);
+    void* b = palloc(c, hb, s);
+    launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, a, N, S, c->d, c->V, c->d_err, s);
+    for (int k = 1; k <= K; ++k) {
+      chunk_fwd_nosave(c, c->ch[k], a, b, B, S, s);
+      std::swap(a, b);
+    }
+    void* z = palloc(c, zb, s);
+    readout_fwd(c, a, z, nullptr, N, s);
+    void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
+    pfree(dz, s);
+    pfree(z, s);
+    pfree(a, s);
+    pfree(b, s);
+    CK(cudaMemcpyAsync(c->h_losses, c->d_losses, 4, cudaMemcpyDeviceToHost, s));
+    sync_all(c, -1);
+    *loss_out = c->h_losses[0];
+    return ZL_OK;
+  });
+}
+
+zl_status zl_read_losses(zl_ctx* c, float* out, int n) {
+  if (!c || !out) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    if (n != c->last_nloss) raise_err(ZL_ERR_ARG, "n must be K after zl_step, 1 after zl_bp_step");
+    sync_all(c, -1);
+    CK(cudaMemcpy(out, c->d_losses + (c->last_nloss == 1 ? 0 : 1), (size_t)n * 4, cudaMemcpyDeviceToHost));
+    return ZL_OK;
+  });
+}
+
+zl_status zl_join(zl_ctx* c) {
+  if (!c) { g_err = "NULL context"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    join_all(c);
+    return ZL_OK;
+  });
+}
+
+zl_status zl_synchronize(zl_ctx* c, int timeout_ms) {
+  if (!c) { g_err = "NULL context"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status { return sync_all(c, timeout_ms); });
+}
+
+zl_status zl_peak_bytes(zl_ctx* c, size_t* peak, size_t* current) {
+  if (!c) { g_err = "NULL context"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    uint64_t hi = 0, cur = 0;
+    CK(cudaMemPoolGetAttribute(c->pool, cudaMemPoolAttrUsedMemHigh, &hi));
+    CK(cudaMemPoolGetAttribute(c->pool, cudaMemPoolAttrUsedMemCurrent, &cur));
+    if (peak) *peak = c->static_bytes + hi;
+    if (current) *current = c->static_bytes + cur;
+    return ZL_OK;
+  });
+}
+
+zl_status zl_reset_peak(zl_ctx* c) {
+  if (!c) { g_err = "NULL context"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    sync_all(c, -1);
+    uint64_t zero = 0;
+    CK(cudaMemPoolSetAttribute(c->pool, cudaMemPoolAttrUsedMemHigh, &zero));
+    return ZL_OK;
+  });
+}
+
+zl_status zl_profile(zl_ctx* c, int on) {
+  if (!c) { g_err = "NULL context"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    if (on && c->evpool.size() < 8192) {
+      while (c->evpool.size() < 8192) {
+        cudaEvent_t e;
+        CK(cudaEventCreate(&e));
+        c->evpool.push_back(e);
+      }
+    }
+    c->prof = on != 0;
+    return ZL_OK;
+  });
+}
+
+zl_status zl_profile_read(zl_ctx* c, char* buf, size_t cap) {
+  if (!c || !buf || cap == 0) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    sync_all(c, -1);
+    double ms[PC_COUNT] = {}, fl[PC_COUNT] = {}, by[PC_COUNT] = {}, nl[PC_COUNT] = {};
+    for (const ProfRec& r : c->recs) {
+      float t = 0.f;
+      CK(cudaEventElapsedTime(&t, r.a, r.b));
+      ms[r.cls] += t;
+      fl[r.cls] += r.flops;
+      by[r.cls] += r.bytes;
+      nl[r.cls] += r.launches;
+    }
+    c->recs.clear();
+    c->evnext = 0;
+    std::string js = "{";
+    for (int i = 0; i < PC_COUNT; ++i) {
+      char tmp[256];
+      std::snprintf(tmp, sizeof tmp, "%s\"%s\": {\"launches\": %.0f, \"ms\": %.6f, \"flops\": %.6e, \"bytes\": %.6e}",
+                    i ? ", " : "", kPCName[i], nl[i], ms[i], fl[i], by[i]);
+      js += tmp;
+    }
+    js += "}";
+    std::snprintf(buf, cap, "%s", js.c_str());
+    return ZL_OK;
+  });
+}
+
+zl_status zl_kernel_launches(uint64_t* count) {
+  if (!count) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  *count = (uint64_t)launches_so_far();
+  return ZL_OK;
+}
+
+zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_t* labels, int N, int V, int ldz,
+                           float alpha, int kl_dir, void* dz, float* row_loss, float* loss, void* stream) {
+  if (!z || !labels || !dz || !row_loss || !loss) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if (dtype != 0 && dtype != 1) { g_err = "dtype"; return ZL_ERR_ARG; }
+  if (N < 1 || V < 2 || ldz < V || ldz % 8 != 0) { g_err = "need N >= 1, V >= 2, ldz >= V, ldz % 8 == 0"; return ZL_ERR_ARG; }
+  if (!(alpha > 0.f && alpha <= 1.f) || (alpha < 1.f && !t) || (kl_dir != 0 && kl_dir != 1)) {
+    g_err = "alpha in (0,1], t required when alpha < 1, kl_dir 0/1";
+    return ZL_ERR_ARG;
+  }
+  return guarded(nullptr, [&]() -> zl_status {
+    cudaStream_t s = (cudaStream_t)stream;
+    int* cnt = nullptr;
+    unsigned* err = nullptr;
+    CK(cudaMallocAsync((void**)&cnt, 256, s));
+    err = (unsigned*)((char*)cnt + 128);
+    CK(cudaMemsetAsync(err, 0, 4, s));
+    launch_count_valid(labels, N, V, cnt, err, s);
+    launch_local_loss(dtype, z, t, labels, N, V, ldz, alpha, kl_dir, cnt, dz, row_loss, s);
+    launch_loss_reduce(row_loss, N, cnt, loss, s);
+    CHECK_LAUNCH();
+    CK(cudaFreeAsync(cnt, s));
+    return ZL_OK;
+  });
+}
+
+zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C, void* stream) {
+  if (!A || !B || !C) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if ((dtype != 0 && dtype != 1) || mode < 0 || mode > 2 || M < 0 || N < 0 || K < 0) {
+    g_err = "bad dtype/mode/size";
+    return ZL_ERR_ARG;
+  }
+  return guarded(nullptr, [&]() -> zl_status {
+    gemm(dtype, mode, M, N, K, A, B, C, nullptr, nullptr, (cudaStream_t)stream);
+    CHECK_LAUNCH();
+    return ZL_OK;
+  });
+}
+
+}  // extern "C"

@@ -1,0 +1,584 @@
+// Memory-bound kernels of the ZeroLock local step: embedding gather, norms, RoPE, activations,
+// the fused local objective (Eq. 3-5) and the per-chunk AdamW update.
+#include <math.h>
+
+#include "common.cuh"
+#include "ops.h"
+
+namespace zl {
+
+static inline int grid_for(size_t work, int threads, int max_blocks = 152 * 16) {
+  size_t b = (work + threads - 1) / threads;
+  if (b < 1) b = 1;
+  return (int)(b > (size_t)max_blocks ? (size_t)max_blocks : b);
+}
+
+// ------------------------------------------------------------------------------------------
+// Embedding gather (Eq. 1: h_0 = E(x)); frozen E (and learned positions P for GPT-2).
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void embed_k(const int32_t* __restrict__ ids, const T* __restrict__ E, const T* __restrict__ P,
+                        T* __restrict__ h, int N, int S, int d, int V, unsigned* err) {
+  const int nv = d / 8;
+  const long total = (long)N * nv;
+  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
+    const int n = (int)(i / nv), c = (int)(i % nv) * 8;
+    const int id = ids[n];
+    T* dst = h + (size_t)n * d + c;
+    if (id < 0 || id >= V) {
+      if (c == 0) atomicOr(err, ZL_DEVERR_BAD_ID);
+      float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      Vec8<T>::store(dst, f);
+      continue;
+    }
+    const T* src = E + (size_t)id * d + c;
+    if (P == nullptr) {               // bit-exact row copy
+      const uint4* s4 = reinterpret_cast<const uint4*>(src);
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+      for (int q = 0; q < (int)(sizeof(T) * 8 / 16); ++q) d4[q] = s4[q];
+    } else {
+      float a[8], b[8];
+      Vec8<T>::load(src, a);
+      Vec8<T>::load(P + (size_t)(n % S) * d + c, b);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) a[q] += b[q];
+      Vec8<T>::store(dst, a);
+    }
+  }
+}
+
+void launch_embed(int dt, const int32_t* ids, const void* E, const void* P, void* h, int N, int S, int d,
+                  int V, unsigned* err, cudaStream_t s) {
+  note_launch(1);
+  const int th = 256, g = grid_for((size_t)N * (d / 8), th);
+  if (dt == BF16)
+    embed_k<bf16><<<g, th, 0, s>>>(ids, (const bf16*)E, (const bf16*)P, (bf16*)h, N, S, d, V, err);
+  else
+    embed_k<float><<<g, th, 0, s>>>(ids, (const float*)E, (const float*)P, (float*)h, N, S, d, V, err);
+}
+
+// ------------------------------------------------------------------------------------------
+// RMSNorm / LayerNorm forward and backward (one warp per row, 8-wide vector access, fp32 math).
+// ------------------------------------------------------------------------------------------
+template <typename T, bool LN>
+__global__ void norm_fwd_k(const T* __restrict__ x, const float* __restrict__ g, const float* __restrict__ b,
+                           T* __restrict__ y, float* __restrict__ rstd_o, float* __restrict__ mean_o, int N,
+                           int d, float eps) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= N) return;
+  const T* xr = x + (size_t)row * d;
+  float s = 0.f, ss = 0.f;
+  for (int c = lane * 8; c < d; c += 256) {
+    float f[8];
+    Vec8<T>::load(xr + c, f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { s += f[i]; ss += f[i] * f[i]; }
+  }
+  s = warp_sum(s);
+  float mean = 0.f, var;
+  if (LN) {
+    mean = s / d;
+    float v = 0.f;
+    for (int c = lane * 8; c < d; c += 256) {
+      float f[8];
+      Vec8<T>::load(xr + c, f);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { const float t = f[i] - mean; v += t * t; }
+    }
+    var = warp_sum(v) / d;
+  } else {
+    var = warp_sum(ss) / d;
+  }
+  const float rstd = 1.f / sqrtf(var + eps);
+  T* yr = y + (size_t)row * d;
+  for (int c = lane * 8; c < d; c += 256) {
+    float f[8];
+    Vec8<T>::load(xr + c, f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      f[i] = (f[i] - mean) * rstd * (g ? g[c + i] : 1.f);
+      if (LN && b) f[i] += b[c + i];
+    }
+    Vec8<T>::store(yr + c, f);
+  }
+  if (lane == 0) {
+    if (rstd_o) rstd_o[row] = rstd;
+    if (LN && mean_o) mean_o[row] = mean;
+  }
+}
+
+void launch_norm_fwd(int dt, bool ln, const void* x, const float* g, const float* b, void* y, float* rstd,
+                     float* mean, int N, int d, float eps, cudaStream_t s) {
+  note_launch(1);
+  const int th = 256, blocks = (N * 32 + th - 1) / th;
+#define NF(T, L) norm_fwd_k<T, L><<<blocks, th, 0, s>>>((const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
+  if (dt == BF16) { if (ln) NF(bf16, true); else NF(bf16, false); }
+  else { if (ln) NF(float, true); else NF(float, false); }
+#undef NF
+}
+
+// dx = rstd * (dyh - mean(dyh) [LN] - xhat * mean(dyh * xhat)), dyh = g * dy.
+template <typename T, bool LN>
+__global__ void norm_bwd_dx_k(const T* __restrict__ x, const float* __restrict__ g,
+                              const float* __restrict__ rstd, const float* __restrict__ mean,
+                              const T* __restrict__ dy, const T* __restrict__ dres, T* __restrict__ dx, int N,
+                              int d) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= N) return;
+  const size_t o = (size_t)row * d;
+  const float r = rstd[row], mu = LN ? mean[row] : 0.f;
+  float s1 = 0.f, s2 = 0.f;
+  for (int c = lane * 8; c < d; c += 256) {
+    float fx[8], fd[8];
+    Vec8<T>::load(x + o + c, fx);
+    Vec8<T>::load(dy + o + c, fd);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float dyh = fd[i] * (g ? g[c + i] : 1.f);
+      s1 += dyh;
+      s2 += dyh * (fx[i] - mu) * r;
+    }
+  }
+  s1 = warp_sum(s1) / d;
+  s2 = warp_sum(s2) / d;
+  for (int c = lane * 8; c < d; c += 256) {
+    float fx[8], fd[8], fr[8];
+    Vec8<T>::load(x + o + c, fx);
+    Vec8<T>::load(dy + o + c, fd);
+    if (dres) Vec8<T>::load(dres + o + c, fr);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float dyh = fd[i] * (g ? g[c + i] : 1.f);
+      const float xh = (fx[i] - mu) * r;
+      float v = r * (dyh - (LN ? s1 : 0.f) - xh * s2);
+      if (dres) v += fr[i];
+      fd[i] = v;
+    }
+    Vec8<T>::store(dx + o + c, fd);
+  }
+}
+
+void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const float* rstd, const float* mean,
+                        const void* dy, const void* dres, void* dx, int N, int d, cudaStream_t s) {
+  note_launch(1);
+  const int th = 256, blocks = (N * 32 + th - 1) / th;
+#define NB(T, L) \
+  norm_bwd_dx_k<T, L><<<blocks, th, 0, s>>>((const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, N, d)
+  if (dt == BF16) { if (ln) NB(bf16, true); else NB(bf16, false); }
+  else { if (ln) NB(float, true); else NB(float, false); }
+#undef NB
+}
+
+static constexpr int kColRows = 64;   // rows per partial-sum block
+int colsum_blocks(int N) { return (N + kColRows - 1) / kColRows; }
+
+// block (32, 8): 32 columns x 8 row lanes; grid (ceil(d/32), colsum_blocks(N)).
+template <typename T, bool NORM, bool LN>
+__global__ void colsum_k(const T* __restrict__ A, const T* __restrict__ x, const float* __restrict__ rstd,
+                         const float* __restrict__ mean, float* __restrict__ part_g,
+                         float* __restrict__ part_b, int N, int d) {
+  __shared__ float sg[8][33], sb[8][33];
+  const int c = blockIdx.x * 32 + threadIdx.x;
+  const int r0 = blockIdx.y * kColRows;
+  float ag = 0.f, ab = 0.f;
+  if (c < d) {
+    for (int r = r0 + threadIdx.y; r < min(r0 + kColRows, N); r += 8) {
+      const float a = to_f(A[(size_t)r * d + c]);
+      if (NORM) {
+        const float xh = (to_f(x[(size_t)r * d + c]) - (LN ? mean[r] : 0.f)) * rstd[r];
+        ag += a * xh;
+      }
+      ab += a;
+    }
+  }
+  sg[threadIdx.y][threadIdx.x] = ag;
+  sb[threadIdx.y][threadIdx.x] = ab;
+  __syncthreads();
+  if (threadIdx.y == 0 && c < d) {
+    float tg = 0.f, tb = 0.f;
+    for (int i = 0; i < 8; ++i) { tg += sg[i][threadIdx.x]; tb += sb[i][threadIdx.x]; }
+    if (NORM) {
+      part_g[(size_t)blockIdx.y * d + c] = tg;
+      if (LN) part_b[(size_t)blockIdx.y * d + c] = tb;
+    } else {
+      part_b[(size_t)blockIdx.y * d + c] = tb;
+    }
+  }
+}
+
+void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, const float* mean,
+                            const void* dy, float* part_g, float* part_b, int N, int d, cudaStream_t s) {
+  note_launch(1);
+  dim3 grid((d + 31) / 32, colsum_blocks(N)), block(32, 8);
+#define CS(T, L) \
+  colsum_k<T, true, L><<<grid, block, 0, s>>>((const T*)dy, (const T*)x, rstd, mean, part_g, part_b, N, d)
+  if (dt == BF16) { if (ln) CS(bf16, true); else CS(bf16, false); }
+  else { if (ln) CS(float, true); else CS(float, false); }
+#undef CS
+}
+
+void launch_colsum(int dt, const void* A, float* part, int N, int d, cudaStream_t s) {
+  note_launch(1);
+  dim3 grid((d + 31) / 32, colsum_blocks(N)), block(32, 8);
+  if (dt == BF16)
+    colsum_k<bf16, false, false><<<grid, block, 0, s>>>((const bf16*)A, nullptr, nullptr, nullptr, nullptr, part, N, d);
+  else
+    colsum_k<float, false, false><<<grid, block, 0, s>>>((const float*)A, nullptr, nullptr, nullptr, nullptr, part, N, d);
+}
+
+__global__ void partials_add_k(const float* __restrict__ part, int nb, int d, float* __restrict__ out) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= d) return;
+  float acc = 0.f;
+  for (int b = 0; b < nb; ++b) acc += part[(size_t)b * d + c];
+  out[c] += acc;
+}
+
+void launch_partials_add(const float* part, int nb, int d, float* out, cudaStream_t s) {
+  note_launch(1);
+  partials_add_k<<<(d + 255) / 256, 256, 0, s>>>(part, nb, d, out);
+}
+
+// ------------------------------------------------------------------------------------------
+// RoPE (rotate-half), SwiGLU, GELU(tanh)
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void rope_k(T* __restrict__ qkv, const float2* __restrict__ cs, int N, int S, int nh, int hd,
+                       int ld, int inverse) {
+  const int half = hd / 2;
+  const long total = (long)N * nh * half;
+  for (long idx = blockIdx.x * (long)blockDim.x + threadIdx.x; idx < total;
+       idx += (long)gridDim.x * blockDim.x) {
+    const int i = (int)(idx % half);
+    const int hh = (int)((idx / half) % nh);
+    const int n = (int)(idx / ((long)half * nh));
+    const float2 c = cs[(size_t)(n % S) * half + i];
+    const float sn = inverse ? -c.y : c.y;
+    T* p = qkv + (size_t)n * ld + (size_t)hh * hd;
+    const float x1 = to_f(p[i]), x2 = to_f(p[i + half]);
+    p[i] = from_f<T>(x1 * c.x - x2 * sn);
+    p[i + half] = from_f<T>(x2 * c.x + x1 * sn);
+  }
+}
+
+void launch_rope(int dt, void* qkv, const float* cs, int N, int S, int H, int Hkv, int hd, int inverse,
+                 cudaStream_t s) {
+  note_launch(1);
+  const int nh = H + Hkv, ld = (H + 2 * Hkv) * hd;
+  const int th = 256, g = grid_for((size_t)N * nh * (hd / 2), th);
+  if (dt == BF16) rope_k<bf16><<<g, th, 0, s>>>((bf16*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
+  else rope_k<float><<<g, th, 0, s>>>((float*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
+}
+
+__device__ __forceinline__ float sigmoidf_(float x) { return 1.f / (1.f + expf(-x)); }
+
+template <typename T>
+__global__ void swiglu_fwd_k(const T* __restrict__ gu, T* __restrict__ a, int N, int f) {
+  const int nv = f / 8;
+  const long total = (long)N * nv;
+  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
+    const int n = (int)(i / nv), c = (int)(i % nv) * 8;
+    float g[8], u[8];
+    Vec8<T>::load(gu + (size_t)n * 2 * f + c, g);
+    Vec8<T>::load(gu + (size_t)n * 2 * f + f + c, u);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) g[q] = g[q] * sigmoidf_(g[q]) * u[q];
+    Vec8<T>::store(a + (size_t)n * f + c, g);
+  }
+}
+
+template <typename T>
+__global__ void swiglu_bwd_k(const T* __restrict__ gu, const T* __restrict__ da, T* __restrict__ dgu, int N,
+                             int f) {
+  const int nv = f / 8;
+  const long total = (long)N * nv;
+  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
+    const int n = (int)(i / nv), c = (int)(i % nv) * 8;
+    float g[8], u[8], d[8], dg[8], du[8];
+    Vec8<T>::load(gu + (size_t)n * 2 * f + c, g);
+    Vec8<T>::load(gu + (size_t)n * 2 * f + f + c, u);
+    Vec8<T>::load(da + (size_t)n * f + c, d);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float sg = sigmoidf_(g[q]);
+      du[q] = d[q] * g[q] * sg;
+      dg[q] = d[q] * u[q] * sg * (1.f + g[q] * (1.f - sg));
+    }
+    Vec8<T>::store(dgu + (size_t)n * 2 * f + c, dg);
+    Vec8<T>::store(dgu + (size_t)n * 2 * f + f + c, du);
+  }
+}
+
+void launch_swiglu_fwd(int dt, const void* gu, void* a, int N, int f, cudaStream_t s) {
+  note_launch(1);
+  const int th = 256, g = grid_for((size_t)N * (f / 8), th);
+  if (dt == BF16) swiglu_fwd_k<bf16><<<g, th, 0, s>>>((const bf16*)gu, (bf16*)a, N, f);
+  else swiglu_fwd_k<float><<<g, th, 0, s>>>((const float*)gu, (float*)a, N, f);
+}
+void launch_swiglu_bwd(int dt, const void* gu, const void* da, void* dgu, int N, int f, cudaStream_t s) {
+  note_launch(1);
+  const int th = 256, g = grid_for((size_t)N * (f / 8), th);
+  if (dt == BF16) swiglu_bwd_k<bf16><<<g, th, 0, s>>>((const bf16*)gu, (const bf16*)da, (bf16*)dgu, N, f);
+  else swiglu_bwd_k<float><<<g, th, 0, s>>>((const float*)gu, (const float*)da, (float*)dgu, N, f);
+}
+
+__device__ __forceinline__ float gelu_inner(float x) { return 0.7978845608028654f * (x + 0.044715f * x * x * x); }
+
+template <typename T>
+__global__ void gelu_fwd_k(const T* __restrict__ x, T* __restrict__ y, size_t n8) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
+    float f[8];
+    Vec8<T>::load(x + i * 8, f);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) f[q] = 0.5f * f[q] * (1.f + tanhf(gelu_inner(f[q])));
+    Vec8<T>::store(y + i * 8, f);
+  }
+}
+
+template <typename T>
+__global__ void gelu_bwd_k(const T* __restrict__ x, const T* __restrict__ dy, T* __restrict__ dx, size_t n8) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
+    float f[8], d[8];
+    Vec8<T>::load(x + i * 8, f);
+    Vec8<T>::load(dy + i * 8, d);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float u = f[q], t = tanhf(gelu_inner(u));
+      const float du = 0.7978845608028654f * (1.f + 3.f * 0.044715f * u * u);
+      d[q] *= 0.5f * (1.f + t) + 0.5f * u * (1.f - t * t) * du;
+    }
+    Vec8<T>::store(dx + i * 8, d);
+  }
+}
+
+void launch_gelu_fwd(int dt, const void* x, void* y, size_t n, cudaStream_t s) {
+  note_launch(1);
+  const int th = 256, g = grid_for(n / 8, th);
+  if (dt == BF16) gelu_fwd_k<bf16><<<g, th, 0, s>>>((const bf16*)x, (bf16*)y, n / 8);
+  else gelu_fwd_k<float><<<g, th, 0, s>>>((const float*)x, (float*)y, n / 8);
+}
+void launch_gelu_bwd(int dt, const void* x, const void* dy, void* dx, size_t n, cudaStream_t s) {
+  note_launch(1);
+  const int th = 256, g = grid_for(n / 8, th);
+  if (dt == BF16) gelu_bwd_k<bf16><<<g, th, 0, s>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, n / 8);
+  else gelu_bwd_k<float><<<g, th, 0, s>>>((const float*)x, (const float*)dy, (float*)dx, n / 8);
+}
+
+// ------------------------------------------------------------------------------------------
+// Local objective (Eq. 3-5), fused: per row i in Omega with p = softmax(z_i), q = softmax(t_i):
+//   CE_i = lse_z - z_y;  KL_i = sum_j p_j (z_j - t_j) - lse_z + lse_t       (kl_dir 0: KL(p||q))
+//                        KL_i = sum_j q_j (t_j - z_j) - lse_t + lse_z       (kl_dir 1: KL(q||p))
+//   dz_j = (1/|Omega|) [alpha (p_j - [j = y]) + (1 - alpha) g_j],
+//   g_j = p_j ((z_j - t_j) - (lse_z - lse_t) - KL_i)   (kl_dir 0),   g_j = p_j - q_j   (kl_dir 1).
+// One block per row; pass 1 keeps online (max, sum) pairs, pass 2 writes dz. No probability
+// tensor is stored.
+// ------------------------------------------------------------------------------------------
+struct Lse3 { float m, s, a; };   // running max, sum e^(x-m), sum e^(x-m) * w
+
+__device__ __forceinline__ Lse3 lse_merge(Lse3 x, Lse3 y) {
+  const float M = fmaxf(x.m, y.m);
+  if (M == -INFINITY) return x;
+  const float ex = expf(x.m - M), ey = expf(y.m - M);
+  return Lse3{M, x.s * ex + y.s * ey, x.a * ex + y.a * ey};
+}
+
+__device__ __forceinline__ Lse3 warp_merge(Lse3 v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    Lse3 w{__shfl_xor_sync(0xffffffffu, v.m, o), __shfl_xor_sync(0xffffffffu, v.s, o),
+           __shfl_xor_sync(0xffffffffu, v.a, o)};
+    v = lse_merge(v, w);
+  }
+  return v;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(512) local_loss_k(const T* __restrict__ z, const T* __restrict__ t,
+                                                    const int32_t* __restrict__ labels, int V, int ldz,
+                                                    float alpha, int kl_dir, const int* __restrict__ count,
+                                                    T* __restrict__ dz, float* __restrict__ row_loss) {
+  __shared__ Lse3 shz[16], sht[16];
+  __shared__ float sh_stats[4];
+  const int row = blockIdx.x;
+  const T* zr = z + (size_t)row * ldz;
+  const T* tr = t ? t + (size_t)row * ldz : nullptr;
+  T* dr = dz + (size_t)row * ldz;
+  const int y = labels[row];
+  const bool valid = y >= 0 && y < V;
+  if (!valid) {   // rows outside Omega: no loss, zero gradient
+    for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) {
+      float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      Vec8<T>::store(dr + c, f);
+    }
+    if (threadIdx.x == 0) row_loss[row] = 0.f;
+    return;
+  }
+  Lse3 Z{-INFINITY, 0.f, 0.f}, Q{-INFINITY, 0.f, 0.f};
+  for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) {
+    float fz[8], ft[8];
+    Vec8<T>::load(zr + c, fz);
+    if (tr) Vec8<T>::load(tr + c, ft);
+    float lz = -INFINITY, lt = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (c + i < V) { lz = fmaxf(lz, fz[i]); if (tr) lt = fmaxf(lt, ft[i]); }
+    if (lz > Z.m) { const float sc = expf(Z.m - lz); Z.s *= sc; Z.a *= sc; Z.m = lz; }
+    if (tr && lt > Q.m) { const float sc = expf(Q.m - lt); Q.s *= sc; Q.a *= sc; Q.m = lt; }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (c + i >= V) continue;
+      const float ez = expf(fz[i] - Z.m);
+      Z.s += ez;
+      if (tr) {
+        const float et = expf(ft[i] - Q.m);
+        Q.s += et;
+        if (kl_dir == 0) Z.a += ez * (fz[i] - ft[i]);
+        else Q.a += et * (ft[i] - fz[i]);
+      }
+    }
+  }
+  Z = warp_merge(Z);
+  if (tr) Q = warp_merge(Q);
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  if (lane == 0) { shz[w] = Z; sht[w] = Q; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    Lse3 a = shz[0], b = sht[0];
+    for (int i = 1; i < nw; ++i) { a = lse_merge(a, shz[i]); if (tr) b = lse_merge(b, sht[i]); }
+    const float lse_z = a.m + logf(a.s);
+    float lse_t = 0.f, kl = 0.f;
+    if (tr) {
+      lse_t = b.m + logf(b.s);
+      kl = kl_dir == 0 ? a.a / a.s - lse_z + lse_t : b.a / b.s - lse_t + lse_z;
+    }
+    const float ce = lse_z - to_f(zr[y]);
+    row_loss[row] = alpha * ce + (tr ? (1.f - alpha) * kl : 0.f);
+    sh_stats[0] = lse_z;
+    sh_stats[1] = lse_t;
+    sh_stats[2] = kl;
+  }
+  __syncthreads();
+  const float lse_z = sh_stats[0], lse_t = sh_stats[1], kl = sh_stats[2];
+  const int cnt = *count;
+  const float inv_n = cnt > 0 ? 1.f / (float)cnt : 0.f;
+  const float wt = inv_n * alpha, wc = inv_n * (1.f - alpha);
+  for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) {
+    float fz[8], ft[8], o[8];
+    Vec8<T>::load(zr + c, fz);
+    if (tr) Vec8<T>::load(tr + c, ft);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int j = c + i;
+      if (j >= V) { o[i] = 0.f; continue; }
+      const float p = expf(fz[i] - lse_z);
+      float gsum = wt * (p - (j == y ? 1.f : 0.f));
+      if (tr) {
+        const float gc = kl_dir == 0 ? p * ((fz[i] - ft[i]) - (lse_z - lse_t) - kl) : p - expf(ft[i] - lse_t);
+        gsum += wc * gc;
+      }
+      o[i] = gsum;
+    }
+    Vec8<T>::store(dr + c, o);
+  }
+}
+
+void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labels, int N, int V, int ldz,
+                       float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s) {
+  note_launch(1);
+  if (N <= 0) return;
+  const int th = 512;
+  if (dt == BF16)
+    local_loss_k<bf16><<<N, th, 0, s>>>((const bf16*)z, (const bf16*)t, labels, V, ldz, alpha, kl_dir, count,
+                                        (bf16*)dz, row_loss);
+  else
+    local_loss_k<float><<<N, th, 0, s>>>((const float*)z, (const float*)t, labels, V, ldz, alpha, kl_dir, count,
+                                         (float*)dz, row_loss);
+}
+
+__global__ void count_valid_k(const int32_t* __restrict__ labels, int N, int V, int* count, unsigned* err) {
+  __shared__ float sh[32];
+  float c = 0.f;
+  bool bad = false;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    const int y = labels[i];
+    if (y >= 0 && y < V) c += 1.f;
+    if (y < -1 || y >= V) bad = true;
+  }
+  if (bad) atomicOr(err, ZL_DEVERR_BAD_LABEL);
+  c = block_sum(c, sh);
+  if (threadIdx.x == 0) *count = (int)(c + 0.5f);
+}
+
+void launch_count_valid(const int32_t* labels, int N, int V, int* count, unsigned* err, cudaStream_t s) {
+  note_launch(1);
+  count_valid_k<<<1, 1024, 0, s>>>(labels, N, V, count, err);
+}
+
+__global__ void loss_reduce_k(const float* __restrict__ rl, int N, const int* count, float* out) {
+  __shared__ double sh[1024];
+  double acc = 0.0;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) acc += (double)rl[i];
+  sh[threadIdx.x] = acc;
+  __syncthreads();
+  for (int o = blockDim.x / 2; o > 0; o >>= 1) {
+    if ((int)threadIdx.x < o) sh[threadIdx.x] += sh[threadIdx.x + o];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    const int c = *count;
+    *out = c > 0 ? (float)(sh[0] / (double)c) : 0.f;
+  }
+}
+
+void launch_loss_reduce(const float* row_loss, int N, const int* count, float* out, cudaStream_t s) {
+  note_launch(1);
+  loss_reduce_k<<<1, 1024, 0, s>>>(row_loss, N, count, out);
+}
+
+// ------------------------------------------------------------------------------------------
+// AdamW over one chunk's contiguous parameter slab (decoupled weight decay, bias correction).
+// ------------------------------------------------------------------------------------------
+__global__ void adamw_k(float4* __restrict__ th, float4* __restrict__ g, float4* __restrict__ m,
+                        float4* __restrict__ v, __nv_bfloat162* __restrict__ comp, size_t n4, float lr, float b1,
+                        float b2, float eps, float wd, float bc1, float bc2, float gscale) {
+  const float decay = 1.f - lr * wd;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
+    float4 t = th[i], gg = g[i], mm = m[i], vv = v[i];
+    float* tp = &t.x; float* gp = &gg.x; float* mp = &mm.x; float* vp = &vv.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float gq = gp[q] * gscale;
+      mp[q] = b1 * mp[q] + (1.f - b1) * gq;
+      vp[q] = b2 * vp[q] + (1.f - b2) * gq * gq;
+      tp[q] = tp[q] * decay - lr * (mp[q] / bc1) / (sqrtf(vp[q] / bc2) + eps);
+    }
+    th[i] = t; m[i] = mm; v[i] = vv;
+    g[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (comp) {
+      comp[2 * i] = __floats2bfloat162_rn(t.x, t.y);
+      comp[2 * i + 1] = __floats2bfloat162_rn(t.z, t.w);
+    }
+  }
+}
+
+void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, float lr, float b1, float b2,
+                  float eps, float wd, float bc1, float bc2, float gscale, cudaStream_t s) {
+  note_launch(1);
+  const size_t n4 = n / 4;   // slabs are padded to a multiple of 64 elements
+  const int th = 256, gr = grid_for(n4, th, 152 * 8);
+  adamw_k<<<gr, th, 0, s>>>((float4*)theta, (float4*)g, (float4*)m, (float4*)v, (__nv_bfloat162*)comp, n4, lr,
+                            b1, b2, eps, wd, bc1, bc2, gscale);
+}
+
+__global__ void f32_to_bf16_k(const float* __restrict__ a, bf16* __restrict__ b, size_t n) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+    b[i] = __float2bfloat16_rn(a[i]);
+}
+
+void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s) {
+  note_launch(1);
+  f32_to_bf16_k<<<grid_for(n, 256), 256, 0, s>>>(src, (bf16*)dst, n);
+}
+
+}  // namespace zl

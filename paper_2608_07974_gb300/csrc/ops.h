@@ -1,0 +1,72 @@
+// Host-side launchers of the engine's kernels (internal; the public ABI is include/zerolock.h).
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace zl {
+
+enum Dt { F32 = 0, BF16 = 1 };
+inline size_t dt_size(int dt) { return dt == BF16 ? 2 : 4; }
+
+// Count of kernels launched by the library (process-wide).
+void note_launch(int n);
+unsigned long long launches_so_far();
+
+// h_0 = E[ids] (+ P[s]); bad ids set ZL_DEVERR_BAD_ID in *err and give a zero row.
+void launch_embed(int dt, const int32_t* ids, const void* E, const void* P, void* h, int N, int S, int d,
+                  int V, unsigned* err, cudaStream_t s);
+
+// y = Norm(x) * g (+ b). RMSNorm (ln = false) or LayerNorm (ln = true). Saves rstd (and mean).
+void launch_norm_fwd(int dt, bool ln, const void* x, const float* g, const float* b, void* y, float* rstd,
+                     float* mean, int N, int d, float eps, cudaStream_t s);
+// dx = Norm'(x)^T (g * dy) (+ dres). g may be NULL (gain 1).
+void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const float* rstd, const float* mean,
+                        const void* dy, const void* dres, void* dx, int N, int d, cudaStream_t s);
+// Partial column sums over row blocks: part_g[b][c] = sum dy * xhat, part_b[b][c] = sum dy (LN only).
+int colsum_blocks(int N);
+void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, const float* mean,
+                            const void* dy, float* part_g, float* part_b, int N, int d, cudaStream_t s);
+// part[b][c] = sum over the rows of block b of A[r][c] (bias gradients).
+void launch_colsum(int dt, const void* A, float* part, int N, int d, cudaStream_t s);
+// out[c] += sum_b part[b][c], b in increasing order (deterministic).
+void launch_partials_add(const float* part, int nb, int d, float* out, cudaStream_t s);
+
+// Rotate q and k heads of qkv [N, (H + 2 Hkv) hd] in place by +angle (inverse = 0) or -angle.
+// cs: [S, hd/2] (cos, sin) pairs.
+void launch_rope(int dt, void* qkv, const float* cs, int N, int S, int H, int Hkv, int hd, int inverse,
+                 cudaStream_t s);
+void launch_swiglu_fwd(int dt, const void* gu, void* a, int N, int f, cudaStream_t s);
+void launch_swiglu_bwd(int dt, const void* gu, const void* da, void* dgu, int N, int f, cudaStream_t s);
+void launch_gelu_fwd(int dt, const void* x, void* y, size_t n, cudaStream_t s);
+void launch_gelu_bwd(int dt, const void* x, const void* dy, void* dx, size_t n, cudaStream_t s);
+
+// |Omega| = #(labels >= 0); labels outside [-1, V) set ZL_DEVERR_BAD_LABEL.
+void launch_count_valid(const int32_t* labels, int N, int V, int* count, unsigned* err, cudaStream_t s);
+// Fused local objective: dz and per-row loss (Eq. 3-5). t may be NULL iff alpha == 1.
+void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labels, int N, int V, int ldz,
+                       float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s);
+// *out = sum(row_loss) / count.
+void launch_loss_reduce(const float* row_loss, int N, const int* count, float* out, cudaStream_t s);
+
+// One AdamW step over a contiguous slab; zeroes g; refreshes the bf16 copy if comp != NULL.
+void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, float lr, float b1,
+                  float b2, float eps, float wd, float bc1, float bc2, float gscale, cudaStream_t s);
+void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
+
+// GEMM (row-major): mode 0: C = A[M,K] B[N,K]^T (+ bias[N]) (+ R[M,N]); mode 1: C = A[M,K] B[K,N] (+ R);
+// mode 2: C[M,N] (fp32) += A[K,M]^T B[K,N].
+void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
+          const void* R, cudaStream_t s);
+bool gemm_tc_available();
+void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
+               const void* R, cudaStream_t s);
+
+// Causal attention over qkv [N, (H + 2 Hkv) hd] (token-major, rows b*S + s): out [N, H hd], lse [B, H, S].
+void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,
+              cudaStream_t s);
+// Gradients into dqkv (same layout as qkv). Dbuf: [B, H, S] scratch.
+void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const float* lse, float* Dbuf,
+              void* dqkv, int B, int S, int H, int Hkv, int hd, cudaStream_t s);
+
+}  // namespace zl
