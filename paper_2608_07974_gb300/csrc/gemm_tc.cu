@@ -1,0 +1,400 @@
+// Tensor-core GEMM for sm_103a: TMA tiles (128-byte swizzle) -> tcgen05.mma (bf16 operands,
+// fp32 accumulator in TMEM, double buffered) -> tcgen05.ld epilogue (bias, residual, bf16 store,
+// or fp32 accumulate into a gradient). Persistent, warp-specialised: warp 0 issues TMA loads,
+// warp 1 owns TMEM and issues the MMAs (one thread), warps 2-5 drain the accumulator.
+// Every mbarrier wait is bounded: on expiry the kernel raises ZL_DEVERR_TIMEOUT and unwinds.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "ops.h"
+
+namespace zl {
+namespace tc {
+
+constexpr int BM = 128, BK = 64;
+constexpr int kThreads = 192;
+constexpr unsigned long long kTimeoutNs = 2000000000ull;   // 2 s per wait
+
+template <int BN>
+struct Cfg {
+  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+};
+
+struct Args {
+  int M, N, K, mode;       // mode 0/1: bf16 C (+bias, +R); mode 2: fp32 C += acc
+  void* C;
+  const float* bias;
+  const bf16* R;
+  unsigned* err;
+  int tiles_m, tiles_n;
+};
+
+__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ unsigned long long gtimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t n) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(n) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.b32 %0, 1, 0, p;\n}"
+      : "=r"(r)
+      : "r"(su32(b)), "r"(parity)
+      : "memory");
+  return r != 0;
+}
+// Waits for the phase of the given parity; false if the kernel is unwinding or the wait expired.
+__device__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, unsigned* err) {
+  if (mbar_test(b, parity)) return true;
+  const unsigned long long t0 = gtimer();
+  for (;;) {
+    if (mbar_test(b, parity)) return true;
+    if (*abort_flag) return false;
+    if (gtimer() - t0 > kTimeoutNs) {
+      *abort_flag = 1;
+      if (err) atomicOr(err, ZL_DEVERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma2d(void* dst, const CUtensorMap* m, uint64_t* bar, int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+          su32(dst)),
+      "l"((unsigned long long)m), "r"(su32(bar)), "r"(c0), "r"(c1)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor: start, leading / stride byte offsets, sm100 version bit,
+// 128-byte swizzle.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, operand majors, N, M.
+template <int BN, bool A_MN, bool B_MN>
+__device__ __forceinline__ constexpr uint32_t idesc() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((A_MN ? 1u : 0u) << 15) | ((B_MN ? 1u : 0u) << 16) |
+         ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d),
+      "l"(a), "l"(b), "r"(id), "r"(acc));
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+               : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int& tm, int& tn) {
+  constexpr int G = 8;   // groups of 8 tile rows share B tiles in L2
+  const int per_group = G * tiles_n;
+  const int gid = tile / per_group, first = gid * G;
+  const int gm = min(tiles_m - first, G);
+  const int r = tile % per_group;
+  tm = first + r % gm;
+  tn = r / gm;
+}
+
+template <int BN, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc_k(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, const Args g) {
+  using C_ = Cfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = (uint64_t*)(smem + C_::STAGES * C_::STAGE_BYTES);
+  uint64_t* empty = full + C_::STAGES;
+  uint64_t* tfull = empty + C_::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* fin = tempty + 2;
+  uint32_t* tbase = (uint32_t*)(fin + 1);
+  volatile int* abort_flag = (volatile int*)(tbase + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C_::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int a = 0; a < 2; ++a) { mbar_init(&tfull[a], 1); mbar_init(&tempty[a], 4); }
+    mbar_init(fin, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tbase)),
+                 "r"((uint32_t)C_::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tbase;
+  const int nk = (g.K + BK - 1) / BK;
+  const int num_tiles = g.tiles_m * g.tiles_n;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int issued[C_::STAGES];   // parity of the last fill of each stage, -1 if none
+#pragma unroll
+      for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
+      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
+        int tm, tn;
+        tile_coords(tile, g.tiles_m, g.tiles_n, tm, tn);
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
+          mbar_expect_tx(&full[stage], C_::STAGE_BYTES);
+          issued[stage] = (int)phase;
+          uint8_t* sa = smem + stage * C_::STAGE_BYTES;
+          uint8_t* sb = sa + C_::A_BYTES;
+          const int k0 = kb * BK;
+          if (!A_MN) {
+            tma2d(sa, &ta, &full[stage], k0, tm * BM);
+          } else {
+            tma2d(sa, &ta, &full[stage], tm * BM, k0);
+            tma2d(sa + 8192, &ta, &full[stage], tm * BM + 64, k0);
+          }
+          if (!B_MN) {
+            tma2d(sb, &tb, &full[stage], k0, tn * BN);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j) tma2d(sb + j * 8192, &tb, &full[stage], tn * BN + 64 * j, k0);
+          }
+          if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (!ok) {   // unwinding: let the copies already in flight land before the CTA exits
+        for (int s = 0; s < C_::STAGES; ++s) {
+          if (issued[s] < 0) continue;
+          const unsigned long long t0 = gtimer();
+          while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer (one thread) ----------------
+    if (lane == 0) {
+      constexpr uint32_t id = idesc<BN, A_MN, B_MN>();
+      int stage = 0, it = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++it) {
+        const int acc = it & 1;
+        const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+        if (!mbar_wait(&tempty[acc], aph ^ 1u, abort_flag, g.err)) break;
+        fence_after();
+        const uint32_t d = tmem + (uint32_t)(acc * BN);
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+          fence_after();
+          const uint32_t a0 = su32(smem + stage * C_::STAGE_BYTES), b0 = a0 + C_::A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t ad = A_MN ? sdesc(a0 + kk * 2048, 8192, 1024) : sdesc(a0 + kk * 32, 16, 1024);
+            const uint64_t bd = B_MN ? sdesc(b0 + kk * 2048, 8192, 1024) : sdesc(b0 + kk * 32, 16, 1024);
+            mma_bf16(d, ad, bd, id, (kb | kk) != 0 ? 1u : 0u);
+          }
+          mma_commit(&empty[stage]);
+          if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (ok) mma_commit(&tfull[acc]);
+      }
+      // all MMAs issued by this thread complete before TMEM is released
+      mma_commit(fin);
+    }
+  } else {
+    // ---------------- epilogue: warps 2..5, one accumulator row per thread ----------------
+    const int q = warp & 3;   // TMEM lanes 32q..32q+31 are the ones this warp may read
+    int it = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
+      int tm, tn;
+      tile_coords(tile, g.tiles_m, g.tiles_n, tm, tn);
+      const int acc = it & 1;
+      const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], aph, abort_flag, g.err) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      fence_after();
+      const int m = tm * BM + q * 32 + lane;
+      const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tmem_ld32(trow + (uint32_t)c, v);
+        const int n0 = tn * BN + c;
+        if (m >= g.M || n0 >= g.N) continue;
+        if (g.mode == 2) {
+          float* cr = (float*)g.C + (size_t)m * g.N + n0;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (n0 + 4 * j >= g.N) break;
+            float4 x = reinterpret_cast<float4*>(cr)[j];
+            x.x += v[4 * j]; x.y += v[4 * j + 1]; x.z += v[4 * j + 2]; x.w += v[4 * j + 3];
+            reinterpret_cast<float4*>(cr)[j] = x;
+          }
+        } else {
+          bf16* cr = (bf16*)g.C + (size_t)m * g.N + n0;
+          const bf16* rr = g.R ? g.R + (size_t)m * g.N + n0 : nullptr;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            if (n0 + 8 * j >= g.N) break;
+            float t[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) t[e] = v[8 * j + e];
+            if (g.bias) {
+#pragma unroll
+              for (int e = 0; e < 8; ++e) t[e] += g.bias[n0 + 8 * j + e];
+            }
+            if (rr) {
+              float r8[8];
+              Vec8<bf16>::load(rr + 8 * j, r8);
+#pragma unroll
+              for (int e = 0; e < 8; ++e) t[e] += r8[e];
+            }
+            Vec8<bf16>::store(cr + 8 * j, t);
+          }
+        }
+      }
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+    }
+  }
+
+  __syncthreads();
+  if (warp == 1) {
+    // wait (bounded) for the final commit issued above, then release TMEM
+    if (lane == 0) {
+      const unsigned long long t0 = gtimer();
+      while (!mbar_test(fin, 0) && gtimer() - t0 < 100000000ull) {
+      }
+    }
+    __syncwarp();
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)C_::TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------------------------------------------------
+// host side
+// ------------------------------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+int g_sms = 0;
+int g_avail = -1;
+
+bool init() {
+  if (g_avail >= 0) return g_avail == 1;
+  g_avail = 0;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (major != 10 || minor != 3) return false;
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess || !fn)
+    return false;
+  g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+  g_avail = 1;
+  return true;
+}
+
+// 2-D bf16 tensor [outer, inner] (inner contiguous), box [box_outer, box_inner], 128-byte swizzle.
+bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint32_t box_inner, uint32_t box_outer) {
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, bool A_MN, bool B_MN>
+bool launch(const Args& a, const void* A, const void* B, cudaStream_t s) {
+  using C_ = Cfg<BN>;
+  static bool attr = false;
+  auto kern = gemm_tc_k<BN, A_MN, B_MN>;
+  if (!attr) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM) != cudaSuccess) return false;
+    attr = true;
+  }
+  CUtensorMap ta, tb;
+  const bool okA = A_MN ? make_map(&ta, A, (uint64_t)a.M, (uint64_t)a.K, 64, 64)
+                        : make_map(&ta, A, (uint64_t)a.K, (uint64_t)a.M, 64, BM);
+  const bool okB = B_MN ? make_map(&tb, B, (uint64_t)a.N, (uint64_t)a.K, 64, 64)
+                        : make_map(&tb, B, (uint64_t)a.K, (uint64_t)a.N, 64, BN);
+  if (!okA || !okB) return false;
+  const int tiles = a.tiles_m * a.tiles_n;
+  const int grid = tiles < g_sms ? tiles : g_sms;
+  gemm_tc_k<BN, A_MN, B_MN><<<grid, kThreads, C_::SMEM, s>>>(ta, tb, a);
+  return true;
+}
+
+}  // namespace tc
+
+bool gemm_tc_available() { return tc::init(); }
+
+// Returns false when the shape / alignment is outside what the tensor-core path handles.
+bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
+             unsigned* err, cudaStream_t s) {
+  if (!tc::init()) return false;
+  if (M < 16 || N < 16 || K < 16) return false;
+  auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
+  if (!al16(A) || !al16(B) || !al16(C) || (R && !al16(R))) return false;
+  if (N % 8 != 0) return false;
+  if ((mode == 0 || mode == 1) && K % 8 != 0) return false;
+  if (mode == 2 && M % 8 != 0) return false;
+  tc::Args a;
+  a.M = M; a.N = N; a.K = K; a.mode = mode;
+  a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err;
+  a.tiles_m = (M + tc::BM - 1) / tc::BM;
+  const int t256 = a.tiles_m * ((N + 255) / 256);
+  const bool wide = t256 >= tc::g_sms;
+  a.tiles_n = wide ? (N + 255) / 256 : (N + 127) / 128;
+  note_launch(1);
+  if (mode == 0) return wide ? tc::launch<256, false, false>(a, A, B, s) : tc::launch<128, false, false>(a, A, B, s);
+  if (mode == 1) return wide ? tc::launch<256, false, true>(a, A, B, s) : tc::launch<128, false, true>(a, A, B, s);
+  return wide ? tc::launch<256, true, true>(a, A, B, s) : tc::launch<128, true, true>(a, A, B, s);
+}
+
+}  // namespace zl
