@@ -198,13 +198,28 @@ def zl_reset_peak(ctx) -> None:
     _check(_lib.zl_reset_peak(ctx))
 
 
+def _need(t, dtypes, what):
+    if t is not None and not isinstance(t, int) and str(t.dtype).replace("torch.", "") not in dtypes:
+        raise TypeError(f"{what}: dtype {t.dtype}, expected {dtypes}")
+
+
 def zl_op_local_loss(dtype: int, z, t, labels, N: int, V: int, ldz: int, alpha: float, kl_dir: int, dz, row_loss,
                      loss, stream: int = 0) -> None:
+    act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
+    for x, nm in ((z, "z"), (t, "t"), (dz, "dz")):
+        _need(x, act, nm)
+    _need(labels, ("int32",), "labels")
+    _need(row_loss, ("float32",), "row_loss")
+    _need(loss, ("float32",), "loss")
     _check(_lib.zl_op_local_loss(dtype, _p(z), _p(t), _p(labels), N, V, ldz, alpha, kl_dir, _p(dz), _p(row_loss),
                                  _p(loss), stream))
 
 
 def zl_op_gemm(dtype: int, mode: int, M: int, N: int, K: int, A, B, Cm, stream: int = 0) -> None:
+    act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
+    _need(A, act, "A")
+    _need(B, act, "B")
+    _need(Cm, ("float32",) if mode == 2 else act, "C")
     _check(_lib.zl_op_gemm(dtype, mode, M, N, K, _p(A), _p(B), _p(Cm), stream))
 
 

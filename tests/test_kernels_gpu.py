@@ -82,7 +82,7 @@ def test_gemm_matches_matmul(B, dtype, mode, M, N, K):
     else:
         a, b = torch.randn(K, M).to(td), torch.randn(K, N).to(td)
         ref = a.double().T @ b.double()
-    c0 = torch.randn(M, N) if mode == 2 else None
+    c0 = torch.randn(M, N, dtype=torch.float32) if mode == 2 else None
     c = c0.clone().cuda() if mode == 2 else torch.empty(M, N, dtype=td, device="cuda")
     B.zl_op_gemm(0 if dtype == "f32" else 1, mode, M, N, K, a.cuda(), b.cuda(), c)
     torch.cuda.synchronize()
@@ -118,7 +118,7 @@ def test_gemm_tensor_core_matches_fp32(B, mode, M, N, K):
         b = torch.randn(K, N, device="cuda", generator=g).to(bf)
         ref = a.float().T @ b.float()
     if mode == 2:
-        c0 = torch.randn(M, N, device="cuda", generator=g)
+        c0 = torch.randn(M, N, device="cuda", generator=g, dtype=torch.float32)
         c = c0.clone()
         ref = ref + c0
     else:

@@ -7,6 +7,7 @@ import torch
 import oracle
 import oracle.model as om
 import tests.test_oracle_pins as pins
+from tests.test_oracle_pins import float64_default  # noqa: F401  (autouse fixture)
 
 
 def _patch(monkeypatch, name, fn):

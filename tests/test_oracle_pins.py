@@ -15,7 +15,16 @@ from oracle.model import Oracle, OracleConfig
 import synth
 from synth import ARCH_GPT2, ARCH_LLAMA, ModelDims
 
-torch.set_default_dtype(torch.float64)
+
+
+@pytest.fixture(autouse=True)
+def float64_default():
+    """The pins run in float64; the default dtype is restored for the other test modules."""
+    old = torch.get_default_dtype()
+    torch.set_default_dtype(torch.float64)
+    yield
+    torch.set_default_dtype(old)
+
 
 LLAMA_T = ModelDims(ARCH_LLAMA, n_layers=2, d_model=16, n_heads=4, n_kv_heads=2, d_ff=24,
                     vocab=37, max_seq=8)
