@@ -181,6 +181,22 @@ zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_
                            int V, int ldz, float alpha, int kl_dir, void* dz, float* row_loss,
                            float* loss, void* stream);
 
+/* Allocation-free variant of zl_op_local_loss (no counterpart in the paper). For callers that
+ * cannot allocate device memory: a host framework whose own caching allocator has reserved the
+ * device budget, so an outside cudaMalloc fails or breaks its accounting, or a latency-critical
+ * loop that must not take the synchronisation cudaMalloc / cudaFree can imply. Same inputs and
+ * outputs as zl_op_local_loss except that the per-row losses stay internal; the scratch
+ * (per-row losses, |Omega|, an error word) is a file-scope device array of
+ * ZL_NOALLOC_MAX_ROWS + 128 floats (257 KB) that every GPU which loads the library holds until
+ * process exit. N > ZL_NOALLOC_MAX_ROWS is rejected with ZL_ERR_ARG. The first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress, with that device current); make
+ * that first call before any stream capture. All calls share the array: calls whose work
+ * overlaps on the GPU race on it, so order them on one stream (or synchronise between them).
+ * Calls no cudaMalloc, cudaFree or allocating library routine. */
+#define ZL_NOALLOC_MAX_ROWS 65536
+zl_status zl_op_local_loss_noalloc(int dtype, const void* z, const void* t, const int32_t* labels, int N, int V,
+                                   int ldz, float alpha, int kl_dir, void* dz, float* loss, void* stream);
+
 /* C[M,N] (+)= A[M,K] . B^T where B is [N,K] (mode 0, "forward"), or A[M,K] . B with B
  * [K,N] (mode 1, "dX"), or C[M,N] += A^T . B with A [K,M], B [K,N] (mode 2, "dW",
  * C fp32 and always accumulated). dtype of A, B and (modes 0/1) C. Row-major, dense. */

@@ -665,6 +665,14 @@ extern "C" {
 
 const char* zl_last_error(void) { return g_err.c_str(); }
 
+}  // extern "C"
+
+namespace zl {
+void set_last_error(const char* msg) { g_err = msg ? msg : ""; }
+}  // namespace zl
+
+extern "C" {
+
 zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const zl_train_cfg* cfg, zl_ctx** out) {
   if (!dims || !bounds || !cfg || !out) { g_err = "NULL argument"; return ZL_ERR_ARG; }
   *out = nullptr;

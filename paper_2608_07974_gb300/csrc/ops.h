@@ -4,10 +4,16 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <string>
+
 namespace zl {
 
 enum Dt { F32 = 0, BF16 = 1 };
 inline size_t dt_size(int dt) { return dt == BF16 ? 2 : 4; }
+
+// Message returned by zl_last_error() on this thread.
+void set_last_error(const char* msg);
+inline void set_last_error(const std::string& msg) { set_last_error(msg.c_str()); }
 
 // Count of kernels launched by the library (process-wide).
 void note_launch(int n);
