@@ -181,6 +181,16 @@ zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_
                            int V, int ldz, float alpha, int kl_dir, void* dz, float* row_loss,
                            float* loss, void* stream);
 
+/* Causal softmax attention with grouped KV heads (the attention of every transformer layer of
+ * Eq. 1): qkv [B*S, (H + 2*Hkv)*hd] token-major (per row: H query heads, Hkv key heads, Hkv value
+ * heads, each hd wide; query head h reads KV head h / (H/Hkv)), scale 1/sqrt(hd). Forward writes
+ * out [B*S, H*hd] and lse [B, H, S] (fp32 natural-log row log-sum-exp). Backward takes dout
+ * [B*S, H*hd] and writes dqkv (qkv layout). dtype of qkv/out/dout/dqkv; hd even and <= 128. */
+zl_status zl_op_attention(int dtype, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,
+                          void* stream);
+zl_status zl_op_attention_bwd(int dtype, const void* qkv, const void* out, const void* dout, const float* lse,
+                              void* dqkv, int B, int S, int H, int Hkv, int hd, void* stream);
+
 /* Allocation-free variant of zl_op_local_loss (no counterpart in the paper). For callers that
  * cannot allocate device memory: a host framework whose own caching allocator has reserved the
  * device budget, so an outside cudaMalloc fails or breaks its accounting, or a latency-critical

@@ -21,7 +21,7 @@ ZL_DTYPE_F32, ZL_DTYPE_BF16 = 0, 1
 EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_get_param", "zl_param_numel",
            "zl_embed", "zl_forward_chunk", "zl_local_step", "zl_step", "zl_bp_step", "zl_eval_global_loss",
            "zl_read_losses", "zl_join", "zl_synchronize", "zl_peak_bytes", "zl_reset_peak", "zl_last_error",
-           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_profile", "zl_profile_read", "zl_kernel_launches"]
+           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches"]
 
 
 class zl_model_dims(C.Structure):
@@ -71,6 +71,8 @@ def _load() -> C.CDLL:
         "zl_op_local_loss": [i, vp, vp, vp, i, i, i, f, i, vp, vp, vp, vp],
         "zl_op_local_loss_noalloc": [i, vp, vp, vp, i, i, i, f, i, vp, vp, vp],
         "zl_op_gemm": [i, i, i, i, i, vp, vp, vp, vp],
+        "zl_op_attention": [i, vp, vp, vp, i, i, i, i, i, vp],
+        "zl_op_attention_bwd": [i, vp, vp, vp, vp, vp, i, i, i, i, i, vp],
         "zl_profile": [vp, i],
         "zl_profile_read": [vp, C.c_char_p, sz],
         "zl_kernel_launches": [C.POINTER(C.c_uint64)],
@@ -226,6 +228,23 @@ def zl_op_local_loss_noalloc(dtype: int, z, t, labels, N: int, V: int, ldz: int,
     _need(loss, ("float32",), "loss")
     _check(_lib.zl_op_local_loss_noalloc(dtype, _p(z), _p(t), _p(labels), N, V, ldz, alpha, kl_dir, _p(dz),
                                          _p(loss), stream))
+
+
+def zl_op_attention(dtype: int, qkv, out, lse, B: int, S: int, H: int, Hkv: int, hd: int, stream: int = 0) -> None:
+    act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
+    _need(qkv, act, "qkv")
+    _need(out, act, "out")
+    _need(lse, ("float32",), "lse")
+    _check(_lib.zl_op_attention(dtype, _p(qkv), _p(out), _p(lse), B, S, H, Hkv, hd, stream))
+
+
+def zl_op_attention_bwd(dtype: int, qkv, out, dout, lse, dqkv, B: int, S: int, H: int, Hkv: int, hd: int,
+                        stream: int = 0) -> None:
+    act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
+    for x, nm in ((qkv, "qkv"), (out, "out"), (dout, "dout"), (dqkv, "dqkv")):
+        _need(x, act, nm)
+    _need(lse, ("float32",), "lse")
+    _check(_lib.zl_op_attention_bwd(dtype, _p(qkv), _p(out), _p(dout), _p(lse), _p(dqkv), B, S, H, Hkv, hd, stream))
 
 
 def zl_op_gemm(dtype: int, mode: int, M: int, N: int, K: int, A, B, Cm, stream: int = 0) -> None:

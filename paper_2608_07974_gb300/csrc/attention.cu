@@ -157,8 +157,13 @@ __global__ void attn_bwd_dkv_k(const T* __restrict__ qkv, const T* __restrict__ 
 inline int warps_grid(long rows) { return (int)((rows * 32 + 255) / 256); }
 }  // namespace
 
+bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s);
+bool attn_bwd_tc(const void* qkv, const void* dout, const float* lse, const float* D, void* dqkv, int B, int S, int H,
+                 int Hkv, int hd, cudaStream_t s);
+
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s) {
   note_launch(1);
+  if (dt == BF16 && attn_fwd_tc(qkv, out, lse, B, S, H, Hkv, hd, s)) return;
   const float scale = 1.f / sqrtf((float)hd);
   const int g = warps_grid((long)B * H * S);
   if (dt == BF16) attn_fwd_k<bf16><<<g, 256, 0, s>>>((const bf16*)qkv, (bf16*)out, lse, B, S, H, Hkv, hd, scale);
@@ -172,6 +177,7 @@ void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const 
   const int gq = warps_grid((long)B * H * S), gk = warps_grid((long)B * Hkv * S);
   if (dt == BF16) {
     attn_bwd_d_k<bf16><<<gq, 256, 0, s>>>((const bf16*)out, (const bf16*)dout, Dbuf, B, S, H, hd);
+    if (attn_bwd_tc(qkv, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s)) return;
     attn_bwd_dq_k<bf16><<<gq, 256, 0, s>>>((const bf16*)qkv, (const bf16*)dout, lse, Dbuf, (bf16*)dqkv, B, S, H, Hkv,
                                            hd, scale);
     attn_bwd_dkv_k<bf16><<<gk, 256, 0, s>>>((const bf16*)qkv, (const bf16*)dout, lse, Dbuf, (bf16*)dqkv, B, S, H,

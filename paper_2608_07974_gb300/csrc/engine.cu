@@ -1289,6 +1289,37 @@ zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_
   });
 }
 
+static bool attn_args_ok(int dtype, int B, int S, int H, int Hkv, int hd) {
+  return (dtype == 0 || dtype == 1) && B >= 1 && S >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0 && hd >= 2 &&
+         hd <= 128 && hd % 2 == 0;
+}
+
+zl_status zl_op_attention(int dtype, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,
+                          void* stream) {
+  if (!qkv || !out || !lse) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if (!attn_args_ok(dtype, B, S, H, Hkv, hd)) { g_err = "bad attention shape"; return ZL_ERR_ARG; }
+  return guarded(nullptr, [&]() -> zl_status {
+    attn_fwd(dtype, qkv, out, lse, B, S, H, Hkv, hd, (cudaStream_t)stream);
+    CHECK_LAUNCH();
+    return ZL_OK;
+  });
+}
+
+zl_status zl_op_attention_bwd(int dtype, const void* qkv, const void* out, const void* dout, const float* lse,
+                              void* dqkv, int B, int S, int H, int Hkv, int hd, void* stream) {
+  if (!qkv || !out || !dout || !lse || !dqkv) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if (!attn_args_ok(dtype, B, S, H, Hkv, hd)) { g_err = "bad attention shape"; return ZL_ERR_ARG; }
+  return guarded(nullptr, [&]() -> zl_status {
+    cudaStream_t s = (cudaStream_t)stream;
+    float* D = nullptr;
+    CK(cudaMallocAsync((void**)&D, (size_t)B * H * S * 4, s));
+    attn_bwd(dtype, qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
+    CHECK_LAUNCH();
+    CK(cudaFreeAsync(D, s));
+    return ZL_OK;
+  });
+}
+
 zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C, void* stream) {
   if (!A || !B || !C) { g_err = "NULL argument"; return ZL_ERR_ARG; }
   if ((dtype != 0 && dtype != 1) || mode < 0 || mode > 2 || M < 0 || N < 0 || K < 0) {

@@ -146,3 +146,49 @@ def test_gemm_tensor_core_throughput(B):
     tflops = 2 * M * N * K * 10 / (t0.elapsed_time(t1) / 1e3) / 1e12
     print(f"tcgen05 GEMM 4096^3: {tflops:.1f} TFLOP/s")
     assert tflops > 150, tflops
+
+
+# Causal attention with grouped KV heads against PyTorch's fp32 SDPA / autograd on the same values.
+ATTN_SHAPES = [(2, 512, 12, 12, 64), (1, 1024, 32, 4, 64), (1, 200, 4, 4, 32), (2, 130, 4, 2, 100),
+               (1, 300, 8, 8, 128), (3, 1, 4, 2, 64), (1, 64, 2, 1, 32)]
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("Bb,S,H,Hkv,hd", ATTN_SHAPES)
+def test_attention_matches_sdpa(B, dtype, Bb, S, H, Hkv, hd):
+    if dtype == "f32" and S * H > 4096:
+        pytest.skip("the CUDA-core path is checked on the small shapes")
+    g = torch.Generator(device="cuda").manual_seed(S * 31 + H * 7 + hd)
+    td = torch.bfloat16 if dtype == "bf16" else torch.float32
+    W = (H + 2 * Hkv) * hd
+    qkv = torch.randn(Bb * S, W, device="cuda", generator=g, dtype=torch.float32).to(td)
+    dout = torch.randn(Bb * S, H * hd, device="cuda", generator=g, dtype=torch.float32).to(td)
+    out = torch.empty(Bb * S, H * hd, device="cuda", dtype=td)
+    lse = torch.empty(Bb, H, S, device="cuda", dtype=torch.float32)
+    dq = torch.full_like(qkv, float("nan"))
+    dt = B.ZL_DTYPE_BF16 if dtype == "bf16" else B.ZL_DTYPE_F32
+    B.zl_op_attention(dt, qkv, out, lse, Bb, S, H, Hkv, hd)
+    B.zl_op_attention_bwd(dt, qkv, out, dout, lse, dq, Bb, S, H, Hkv, hd)
+    torch.cuda.synchronize()
+    x = qkv.float().view(Bb, S, W).requires_grad_(True)
+    q = x[..., : H * hd].view(Bb, S, H, hd).transpose(1, 2)
+    k = x[..., H * hd: (H + Hkv) * hd].view(Bb, S, Hkv, hd).transpose(1, 2)
+    v = x[..., (H + Hkv) * hd:].view(Bb, S, Hkv, hd).transpose(1, 2)
+    rep = H // Hkv
+    k, v = k.repeat_interleave(rep, 1), v.repeat_interleave(rep, 1)
+    s = (q @ k.transpose(-1, -2)) / hd ** 0.5
+    s = s.masked_fill(torch.triu(torch.ones(S, S, dtype=torch.bool, device="cuda"), 1), float("-inf"))
+    ref_lse = torch.logsumexp(s, -1)
+    ref = (torch.softmax(s, -1) @ v).transpose(1, 2).reshape(Bb * S, H * hd)
+    (gx,) = torch.autograd.grad(ref, x, dout.float().view(Bb * S, H * hd))
+    tol = 2e-2 if dtype == "bf16" else 1e-5
+    assert float((out.float() - ref).abs().max()) <= tol * max(1.0, float(ref.abs().max()))
+    assert float((lse - ref_lse).abs().max()) <= (1e-3 if dtype == "bf16" else 1e-5)
+    gx = gx.view(Bb * S, W)
+    err = float((dq.float() - gx).abs().max()) / max(1.0, float(gx.abs().max()))
+    assert err <= (3e-2 if dtype == "bf16" else 1e-5), err
+    # sections: cosine per q / k / v block must be tight
+    for lo, hi in ((0, H * hd), (H * hd, (H + Hkv) * hd), ((H + Hkv) * hd, W)):
+        a, r = dq.float()[:, lo:hi].reshape(-1).double(), gx[:, lo:hi].reshape(-1).double()
+        cos = float(a @ r / (a.norm() * r.norm() + 1e-30))
+        assert cos >= 0.9995, (lo, cos)
