@@ -180,8 +180,10 @@ def test_attention_matches_sdpa(B, dtype, Bb, S, H, Hkv, hd):
     s = s.masked_fill(torch.triu(torch.ones(S, S, dtype=torch.bool, device="cuda"), 1), float("-inf"))
     ref_lse = torch.logsumexp(s, -1)
     ref = (torch.softmax(s, -1) @ v).transpose(1, 2).reshape(Bb * S, H * hd)
-    (gx,) = torch.autograd.grad(ref, x, dout.float().view(Bb * S, H * hd))
+    (gx,) = torch.autograd.grad(ref, x, dout.float().view(Bb * S, H * hd), retain_graph=False)
+    ref_lse = ref_lse.detach()
     tol = 2e-2 if dtype == "bf16" else 1e-5
+    ref = ref.detach()
     assert float((out.float() - ref).abs().max()) <= tol * max(1.0, float(ref.abs().max()))
     assert float((lse - ref_lse).abs().max()) <= (1e-3 if dtype == "bf16" else 1e-5)
     gx = gx.view(Bb * S, W)
