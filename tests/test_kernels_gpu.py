@@ -192,5 +192,8 @@ def test_attention_matches_sdpa(B, dtype, Bb, S, H, Hkv, hd):
     # sections: cosine per q / k / v block must be tight
     for lo, hi in ((0, H * hd), (H * hd, (H + Hkv) * hd), ((H + Hkv) * hd, W)):
         a, r = dq.float()[:, lo:hi].reshape(-1).double(), gx[:, lo:hi].reshape(-1).double()
+        if float(r.norm()) <= 1e-3 * max(1.0, float(gx.norm())):   # dQ and dK are exactly 0 when S = 1
+            assert float(a.abs().max()) <= 1e-2, (lo, float(a.abs().max()))
+            continue
         cos = float(a @ r / (a.norm() * r.norm() + 1e-30))
         assert cos >= 0.9995, (lo, cos)
