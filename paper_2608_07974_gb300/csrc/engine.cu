@@ -220,7 +220,7 @@ void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, 
   const double e = (double)esz(c);
   const double out = mode == 2 ? 8.0 * M * N : (R ? 2.0 : 1.0) * e * M * N;
   ProfScope p(c, s, PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
-  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err);
+  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool);
 }
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
   const double e = (double)esz(c), N = (double)B * S;

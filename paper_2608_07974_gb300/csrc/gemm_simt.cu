@@ -98,8 +98,8 @@ void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void*
 namespace zl {
 // GEMM dispatch: the tensor-core kernel where it applies, else the CUDA-core kernel.
 void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-          const void* R, cudaStream_t s, unsigned* err) {
-  if (dt == BF16 && gemm_tc(mode, M, N, K, A, B, C, bias, R, err, s)) return;
+          const void* R, cudaStream_t s, unsigned* err, cudaMemPool_t pool) {
+  if (dt == BF16 && gemm_tc(mode, M, N, K, A, B, C, bias, R, err, s, pool)) return;
   gemm_simt(dt, mode, M, N, K, A, B, C, bias, R, s);
 }
 }  // namespace zl

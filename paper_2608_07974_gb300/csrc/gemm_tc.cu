@@ -6,6 +6,10 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
+#include <cstdio>
+#include <cstdlib>
+
 #include "common.cuh"
 #include "ops.h"
 
@@ -18,7 +22,8 @@ constexpr unsigned long long kTimeoutNs = 2000000000ull;   // 2 s per wait
 
 template <int BN>
 struct Cfg {
-  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  // BN = 64 stays under 114 KB of shared memory so two CTAs (and TMEM allocations) fit on an SM.
+  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 4);
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -27,12 +32,13 @@ struct Cfg {
 };
 
 struct Args {
-  int M, N, K, mode;       // mode 0/1: bf16 C (+bias, +R); mode 2: fp32 C += acc
+  int M, N, K, mode;       // mode 0/1: bf16 C (+bias, +R); 2: fp32 C += acc; 3: fp32 store into split slice
   void* C;
   const float* bias;
   const bf16* R;
   unsigned* err;
   int tiles_m, tiles_n;
+  int splits, kb_per_split;   // split-K: unit u -> split u / tiles, k blocks [s*kps, min(nk, (s+1)*kps))
 };
 
 __device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -162,6 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tbase;
   const int nk = (g.K + BK - 1) / BK;
   const int num_tiles = g.tiles_m * g.tiles_n;
+  const int num_units = num_tiles * g.splits;
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -172,10 +179,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       int issued[C_::STAGES];   // parity of the last fill of each stage, -1 if none
 #pragma unroll
       for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
-      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
+      for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
         int tm, tn;
-        tile_coords(tile, g.tiles_m, g.tiles_n, tm, tn);
-        for (int kb = 0; kb < nk; ++kb) {
+        tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+        const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
           mbar_expect_tx(&full[stage], C_::STAGE_BYTES);
           issued[stage] = (int)phase;
@@ -213,13 +221,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0, it = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++it) {
+      for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++it) {
         const int acc = it & 1;
         const uint32_t aph = (uint32_t)(it >> 1) & 1u;
         if (!mbar_wait(&tempty[acc], aph ^ 1u, abort_flag, g.err)) break;
         fence_after();
         const uint32_t d = tmem + (uint32_t)(acc * BN);
-        for (int kb = 0; kb < nk; ++kb) {
+        const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, g.err)) { ok = false; break; }
           fence_after();
           const uint32_t a0 = su32(smem + stage * C_::STAGE_BYTES), b0 = a0 + C_::A_BYTES;
@@ -227,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int kk = 0; kk < BK / 16; ++kk) {
             const uint64_t ad = A_MN ? sdesc(a0 + kk * 2048, 8192, 1024) : sdesc(a0 + kk * 32, 16, 1024);
             const uint64_t bd = B_MN ? sdesc(b0 + kk * 2048, 8192, 1024) : sdesc(b0 + kk * 32, 16, 1024);
-            mma_bf16(d, ad, bd, id, (kb | kk) != 0 ? 1u : 0u);
+            mma_bf16(d, ad, bd, id, (kb > kb0 || kk > 0) ? 1u : 0u);
           }
           mma_commit(&empty[stage]);
           if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
@@ -241,9 +250,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- epilogue: warps 2..5, one accumulator row per thread ----------------
     const int q = warp & 3;   // TMEM lanes 32q..32q+31 are the ones this warp may read
     int it = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
+    for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
       int tm, tn;
-      tile_coords(tile, g.tiles_m, g.tiles_n, tm, tn);
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      const size_t slice = (size_t)(unit / num_tiles) * g.M * g.N;
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
       int ok = 1;
@@ -267,6 +277,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             float4 x = reinterpret_cast<float4*>(cr)[j];
             x.x += v[4 * j]; x.y += v[4 * j + 1]; x.z += v[4 * j + 2]; x.w += v[4 * j + 3];
             reinterpret_cast<float4*>(cr)[j] = x;
+          }
+        } else if (g.mode == 3) {
+          float* cr = (float*)g.C + slice + (size_t)m * g.N + n0;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (n0 + 4 * j >= g.N) break;
+            reinterpret_cast<float4*>(cr)[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
           }
         } else {
           bf16* cr = (bf16*)g.C + (size_t)m * g.N + n0;
@@ -312,6 +329,43 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Sums the split-K partials in split order (deterministic) and applies the epilogue.
+__global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, int mode, void* C,
+                                const float* __restrict__ bias, const bf16* __restrict__ R) {
+  const size_t n8 = (size_t)M * N / 8, MN = (size_t)M * N;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
+    const size_t e = i * 8;
+    float acc[8];
+    Vec8<float>::load(ws + e, acc);
+    for (int s = 1; s < splits; ++s) {
+      float t[8];
+      Vec8<float>::load(ws + s * MN + e, t);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] += t[q];
+    }
+    if (mode == 2) {
+      float c[8];
+      Vec8<float>::load((float*)C + e, c);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) c[q] += acc[q];
+      Vec8<float>::store((float*)C + e, c);
+    } else {
+      const int n = (int)(e % N);
+      if (bias) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] += bias[n + q];
+      }
+      if (R) {
+        float r[8];
+        Vec8<bf16>::load(R + e, r);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] += r[q];
+      }
+      Vec8<bf16>::store((bf16*)C + e, acc);
+    }
+  }
+}
+
 // ------------------------------------------------------------------------------------------------
 // host side
 // ------------------------------------------------------------------------------------------------
@@ -350,7 +404,7 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
 }
 
 template <int BN, bool A_MN, bool B_MN>
-bool launch(const Args& a, const void* A, const void* B, cudaStream_t s) {
+bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int ctas_per_sm) {
   using C_ = Cfg<BN>;
   static bool attr = false;
   auto kern = gemm_tc_k<BN, A_MN, B_MN>;
@@ -364,10 +418,44 @@ bool launch(const Args& a, const void* A, const void* B, cudaStream_t s) {
   const bool okB = B_MN ? make_map(&tb, B, (uint64_t)a.N, (uint64_t)a.K, 64, 64)
                         : make_map(&tb, B, (uint64_t)a.K, (uint64_t)a.N, 64, BN);
   if (!okA || !okB) return false;
-  const int tiles = a.tiles_m * a.tiles_n;
-  const int grid = tiles < g_sms ? tiles : g_sms;
+  const int units = a.tiles_m * a.tiles_n * a.splits;
+  const int slots = g_sms * ctas_per_sm;
+  const int grid = units < slots ? units : slots;
   gemm_tc_k<BN, A_MN, B_MN><<<grid, kThreads, C_::SMEM, s>>>(ta, tb, a);
   return true;
+}
+
+template <bool A_MN, bool B_MN>
+bool launch_bn(int bn, const Args& a, const void* A, const void* B, cudaStream_t s) {
+  if (bn == 256) return launch<256, A_MN, B_MN>(a, A, B, s, 1);
+  if (bn == 128) return launch<128, A_MN, B_MN>(a, A, B, s, 1);
+  return launch<64, A_MN, B_MN>(a, A, B, s, 2);
+}
+
+// Tile width and split count from a wave model: units of 128 x BN x (K / splits) run on
+// 152 (BN 256/128) or 304 (BN 64) slots at one SM's share of the tensor rate, plus a fixed cost
+// per unit and, for splits, the fp32 partial traffic of the reduction.
+void choose(int M, int N, int K, int& bn_out, int& splits_out) {
+  const double rate = 1.45e15 / g_sms;        // flop/s of one SM
+  const double unit_fixed = 0.6e-6;           // pipeline fill and epilogue tail per unit (s)
+  const double hbm = 6.0e12;                  // bytes/s for the partials
+  const int nk = (K + BK - 1) / BK;
+  double best = 1e30;
+  for (int bn : {256, 128, 64}) {
+    const long tiles = (long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
+    const int cps = bn == 64 ? 2 : 1;
+    for (int sp : {1, 2, 3, 4, 6, 8}) {
+      if (sp > 1 && nk / sp < 6) continue;
+      const int kps = (nk + sp - 1) / sp;
+      const long units = tiles * sp;
+      const long slots = (long)g_sms * cps;
+      const long waves = (units + slots - 1) / slots;
+      const double unit_t = (2.0 * BM * bn * kps * BK) / (rate / cps) + unit_fixed;
+      double t = waves * unit_t;
+      if (sp > 1) t += (double)sp * M * N * 4.0 * 2.0 / hbm + 3e-6;
+      if (t < best * 0.97) { best = t; bn_out = bn; splits_out = sp; }
+    }
+  }
 }
 
 }  // namespace tc
@@ -376,7 +464,7 @@ bool gemm_tc_available() { return tc::init(); }
 
 // Returns false when the shape / alignment is outside what the tensor-core path handles.
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-             unsigned* err, cudaStream_t s) {
+             unsigned* err, cudaStream_t s, cudaMemPool_t pool) {
   if (!tc::init()) return false;
   if (M < 16 || N < 16 || K < 16) return false;
   auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
@@ -384,17 +472,59 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
   if (N % 8 != 0) return false;
   if ((mode == 0 || mode == 1) && K % 8 != 0) return false;
   if (mode == 2 && M % 8 != 0) return false;
+  int bn = 128, splits = 1;
+  tc::choose(M, N, K, bn, splits);
+  if (const char* force = std::getenv("ZL_GEMM_TILE")) {   // tuning override "BN:SPLITS"
+    int fb = 0, fs = 0;
+    if (std::sscanf(force, "%d:%d", &fb, &fs) == 2 && (fb == 64 || fb == 128 || fb == 256) && fs >= 1 && fs <= 16) {
+      bn = fb;
+      splits = std::max(1, std::min(fs, (K + tc::BK - 1) / tc::BK));
+    }
+  }
   tc::Args a;
   a.M = M; a.N = N; a.K = K; a.mode = mode;
   a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err;
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
-  const int t256 = a.tiles_m * ((N + 255) / 256);
-  const bool wide = t256 >= tc::g_sms;
-  a.tiles_n = wide ? (N + 255) / 256 : (N + 127) / 128;
+  a.tiles_n = (N + bn - 1) / bn;
+  const int nk = (K + tc::BK - 1) / tc::BK;
+  a.splits = splits;
+  a.kb_per_split = (nk + splits - 1) / splits;
+  float* ws = nullptr;
+  if (splits > 1) {
+    const size_t bytes = (size_t)splits * M * N * 4;
+    cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&ws, bytes, pool, s) : cudaMallocAsync((void**)&ws, bytes, s);
+    if (e != cudaSuccess) {   // no room for the partials: one split
+      cudaGetLastError();
+      ws = nullptr;
+      a.splits = 1;
+      a.kb_per_split = nk;
+    } else {
+      a.mode = 3;
+      a.C = ws;
+      a.bias = nullptr;
+      a.R = nullptr;
+    }
+  }
   note_launch(1);
-  if (mode == 0) return wide ? tc::launch<256, false, false>(a, A, B, s) : tc::launch<128, false, false>(a, A, B, s);
-  if (mode == 1) return wide ? tc::launch<256, false, true>(a, A, B, s) : tc::launch<128, false, true>(a, A, B, s);
-  return wide ? tc::launch<256, true, true>(a, A, B, s) : tc::launch<128, true, true>(a, A, B, s);
+  bool ok;
+  if (mode == 0) ok = tc::launch_bn<false, false>(bn, a, A, B, s);
+  else if (mode == 1) ok = tc::launch_bn<false, true>(bn, a, A, B, s);
+  else ok = tc::launch_bn<true, true>(bn, a, A, B, s);
+  if (ws) {
+    if (ok) {
+      note_launch(1);
+      const size_t n8 = (size_t)M * N / 8;
+      const int blocks = (int)std::min<size_t>((n8 + 255) / 256, (size_t)tc::g_sms * 8);
+      tc::splitk_reduce_k<<<blocks, 256, 0, s>>>(ws, a.splits, M, N, mode, C, bias, (const bf16*)R);
+    }
+    cudaFreeAsync(ws, s);
+  }
+  return ok;
+}
+
+void gemm_tc_plan(int M, int N, int K, int* bn, int* splits) {
+  if (!tc::init()) { *bn = 0; *splits = 0; return; }
+  tc::choose(M, N, K, *bn, *splits);
 }
 
 }  // namespace zl

@@ -62,12 +62,15 @@ void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
 
 // GEMM (row-major): mode 0: C = A[M,K] B[N,K]^T (+ bias[N]) (+ R[M,N]); mode 1: C = A[M,K] B[K,N] (+ R);
 // mode 2: C[M,N] (fp32) += A[K,M]^T B[K,N]. bf16 runs on the tcgen05 kernel where its shape and
-// alignment rules hold, everything else on the CUDA-core kernel. err: device word for timeouts.
+// alignment rules hold, everything else on the CUDA-core kernel. err: device word for timeouts;
+// pool: stream-ordered pool for split-K partials (NULL: the device's default pool).
 void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-          const void* R, cudaStream_t s, unsigned* err = nullptr);
+          const void* R, cudaStream_t s, unsigned* err = nullptr, cudaMemPool_t pool = nullptr);
 bool gemm_tc_available();
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-             unsigned* err, cudaStream_t s);
+             unsigned* err, cudaStream_t s, cudaMemPool_t pool);
+// Tile width and split-K count the tensor-core GEMM picks for a shape (0, 0 if unavailable).
+void gemm_tc_plan(int M, int N, int K, int* bn, int* splits);
 void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
                const void* R, cudaStream_t s);
 

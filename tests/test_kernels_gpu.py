@@ -98,7 +98,8 @@ def test_gemm_matches_matmul(B, dtype, mode, M, N, K):
 # takes every bf16 case here. Reference: fp32 torch.matmul of the same bf16 values.
 TC_SHAPES = [(0, 256, 384, 128), (0, 4096, 2304, 768), (1, 4096, 768, 3072), (2, 2304, 768, 4096),
              (0, 1024, 50304, 768), (1, 1024, 768, 50304), (0, 200, 136, 72), (1, 333, 264, 200),
-             (2, 136, 264, 333), (0, 4096, 8640, 512), (1, 512, 8640, 3200), (2, 3200, 8640, 256)]
+             (2, 136, 264, 333), (0, 4096, 8640, 512), (1, 512, 8640, 3200), (2, 3200, 8640, 256),
+             (2, 768, 768, 4096), (1, 4096, 768, 50304)]
 
 
 @pytest.mark.parametrize("mode,M,N,K", TC_SHAPES)
@@ -127,6 +128,14 @@ def test_gemm_tensor_core_matches_fp32(B, mode, M, N, K):
     torch.cuda.synchronize()
     err = float((c.float() - ref).abs().max()) / float(ref.abs().max())
     assert err <= (1e-5 if mode == 2 else 8e-3), err
+
+
+@pytest.mark.parametrize("tile", ["64:1", "128:1", "256:1", "64:3", "128:4", "256:2"])
+@pytest.mark.parametrize("mode,M,N,K", [(0, 384, 200, 1024), (1, 260, 136, 3000), (2, 136, 264, 2100)])
+def test_gemm_every_tile_and_split(B, monkeypatch, tile, mode, M, N, K):
+    """Each tile width and split-K count (forced) agrees with the fp32 reference on ragged shapes."""
+    monkeypatch.setenv("ZL_GEMM_TILE", tile)
+    test_gemm_tensor_core_matches_fp32(B, mode, M, N, K)
 
 
 def test_gemm_tensor_core_throughput(B):
