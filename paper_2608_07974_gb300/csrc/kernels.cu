@@ -173,31 +173,45 @@ void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const fl
 static constexpr int kColRows = 64;   // rows per partial-sum block
 int colsum_blocks(int N) { return (N + kColRows - 1) / kColRows; }
 
-// block (32, 8): 32 columns x 8 row lanes; grid (ceil(d/32), colsum_blocks(N)).
+// block (32, 8): 32 threads x 8 columns each (256 columns, 16-byte loads) x 8 row lanes;
+// grid (ceil(d/256), colsum_blocks(N)). Requires d % 8 == 0.
 template <typename T, bool NORM, bool LN>
-__global__ void colsum_k(const T* __restrict__ A, const T* __restrict__ x, const float* __restrict__ rstd,
-                         const float* __restrict__ mean, float* __restrict__ part_g,
-                         float* __restrict__ part_b, int N, int d) {
-  __shared__ float sg[8][33], sb[8][33];
-  const int c = blockIdx.x * 32 + threadIdx.x;
+__global__ void __launch_bounds__(256) colsum_k(const T* __restrict__ A, const T* __restrict__ x,
+                                                const float* __restrict__ rstd, const float* __restrict__ mean,
+                                                float* __restrict__ part_g, float* __restrict__ part_b, int N,
+                                                int d) {
+  __shared__ float sg[8][256], sb[8][256];
+  const int c0 = blockIdx.x * 256 + threadIdx.x * 8;
   const int r0 = blockIdx.y * kColRows;
-  float ag = 0.f, ab = 0.f;
-  if (c < d) {
-    for (int r = r0 + threadIdx.y; r < min(r0 + kColRows, N); r += 8) {
-      const float a = to_f(A[(size_t)r * d + c]);
+  const int r1 = min(r0 + kColRows, N);
+  float ag[8] = {0, 0, 0, 0, 0, 0, 0, 0}, ab[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  if (c0 < d) {
+    for (int r = r0 + threadIdx.y; r < r1; r += 8) {
+      float a[8];
+      Vec8<T>::load(A + (size_t)r * d + c0, a);
       if (NORM) {
-        const float xh = (to_f(x[(size_t)r * d + c]) - (LN ? mean[r] : 0.f)) * rstd[r];
-        ag += a * xh;
+        float xv[8];
+        Vec8<T>::load(x + (size_t)r * d + c0, xv);
+        const float mu = LN ? mean[r] : 0.f, rs = rstd[r];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ag[i] = fmaf(a[i], (xv[i] - mu) * rs, ag[i]);
       }
-      ab += a;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ab[i] += a[i];
     }
   }
-  sg[threadIdx.y][threadIdx.x] = ag;
-  sb[threadIdx.y][threadIdx.x] = ab;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    sg[threadIdx.y][threadIdx.x * 8 + i] = ag[i];
+    sb[threadIdx.y][threadIdx.x * 8 + i] = ab[i];
+  }
   __syncthreads();
-  if (threadIdx.y == 0 && c < d) {
+  const int t = threadIdx.y * 32 + threadIdx.x;   // 256 threads, one column each
+  const int c = blockIdx.x * 256 + t;
+  if (c < d) {
     float tg = 0.f, tb = 0.f;
-    for (int i = 0; i < 8; ++i) { tg += sg[i][threadIdx.x]; tb += sb[i][threadIdx.x]; }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { tg += sg[i][t]; tb += sb[i][t]; }
     if (NORM) {
       part_g[(size_t)blockIdx.y * d + c] = tg;
       if (LN) part_b[(size_t)blockIdx.y * d + c] = tb;
@@ -210,7 +224,7 @@ __global__ void colsum_k(const T* __restrict__ A, const T* __restrict__ x, const
 void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, const float* mean,
                             const void* dy, float* part_g, float* part_b, int N, int d, cudaStream_t s) {
   note_launch(1);
-  dim3 grid((d + 31) / 32, colsum_blocks(N)), block(32, 8);
+  dim3 grid((d + 255) / 256, colsum_blocks(N)), block(32, 8);
 #define CS(T, L) \
   colsum_k<T, true, L><<<grid, block, 0, s>>>((const T*)dy, (const T*)x, rstd, mean, part_g, part_b, N, d)
   if (dt == BF16) { if (ln) CS(bf16, true); else CS(bf16, false); }
@@ -220,7 +234,7 @@ void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, c
 
 void launch_colsum(int dt, const void* A, float* part, int N, int d, cudaStream_t s) {
   note_launch(1);
-  dim3 grid((d + 31) / 32, colsum_blocks(N)), block(32, 8);
+  dim3 grid((d + 255) / 256, colsum_blocks(N)), block(32, 8);
   if (dt == BF16)
     colsum_k<bf16, false, false><<<grid, block, 0, s>>>((const bf16*)A, nullptr, nullptr, nullptr, nullptr, part, N, d);
   else
@@ -374,12 +388,12 @@ void launch_gelu_bwd(int dt, const void* x, const void* dy, void* dx, size_t n, 
 // One block per row; pass 1 keeps online (max, sum) pairs, pass 2 writes dz. No probability
 // tensor is stored.
 // ------------------------------------------------------------------------------------------
-struct Lse3 { float m, s, a; };   // running max, sum e^(x-m), sum e^(x-m) * w
+struct Lse3 { float m, s, a; };   // running max (log2 units), sum 2^(x-m), sum 2^(x-m) * w
 
 __device__ __forceinline__ Lse3 lse_merge(Lse3 x, Lse3 y) {
   const float M = fmaxf(x.m, y.m);
   if (M == -INFINITY) return x;
-  const float ex = expf(x.m - M), ey = expf(y.m - M);
+  const float ex = exp2f(x.m - M), ey = exp2f(y.m - M);
   return Lse3{M, x.s * ex + y.s * ey, x.a * ex + y.a * ey};
 }
 
@@ -393,12 +407,36 @@ __device__ __forceinline__ Lse3 warp_merge(Lse3 v) {
   return v;
 }
 
+constexpr float kL2e = 1.4426950408889634f, kLn2 = 0.6931471805599453f;
+
+// Adds 8 values (natural-log logits f, weights w) to an online base-2 log-sum-exp.
+__device__ __forceinline__ void lse_add8(Lse3& A, const float* f, const float* w, int nvalid) {
+  float mx = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    if (i < nvalid) mx = fmaxf(mx, f[i] * kL2e);
+  if (mx > A.m) {
+    const float sc = exp2f(A.m - mx);
+    A.s *= sc;
+    A.a *= sc;
+    A.m = mx;
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if (i < nvalid) {
+      const float e = exp2f(fmaf(f[i], kL2e, -A.m));
+      A.s += e;
+      if (w) A.a = fmaf(e, w[i], A.a);
+    }
+  }
+}
+
 template <typename T>
-__global__ void __launch_bounds__(512) local_loss_k(const T* __restrict__ z, const T* __restrict__ t,
-                                                    const int32_t* __restrict__ labels, int V, int ldz,
-                                                    float alpha, int kl_dir, const int* __restrict__ count,
-                                                    T* __restrict__ dz, float* __restrict__ row_loss) {
-  __shared__ Lse3 shz[16], sht[16];
+__global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, const T* __restrict__ t,
+                                                     const int32_t* __restrict__ labels, int V, int ldz,
+                                                     float alpha, int kl_dir, const int* __restrict__ count,
+                                                     T* __restrict__ dz, float* __restrict__ row_loss) {
+  __shared__ Lse3 shz[32], sht[32];
   __shared__ float sh_stats[4];
   const int row = blockIdx.x;
   const T* zr = z + (size_t)row * ldz;
@@ -406,50 +444,63 @@ __global__ void __launch_bounds__(512) local_loss_k(const T* __restrict__ z, con
   T* dr = dz + (size_t)row * ldz;
   const int y = labels[row];
   const bool valid = y >= 0 && y < V;
+  const int step = blockDim.x * 8;
   if (!valid) {   // rows outside Omega: no loss, zero gradient
-    for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) {
-      float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-      Vec8<T>::store(dr + c, f);
-    }
+    float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    for (int c = threadIdx.x * 8; c < ldz; c += step) Vec8<T>::store(dr + c, f);
     if (threadIdx.x == 0) row_loss[row] = 0.f;
     return;
   }
+  // pass 1: base-2 online log-sum-exp of z and t, plus the KL cross term
   Lse3 Z{-INFINITY, 0.f, 0.f}, Q{-INFINITY, 0.f, 0.f};
-  for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) {
+  auto consume = [&](const float* fz, const float* ft, int nv) {
+    float w[8];
+    if (tr) {
+      if (kl_dir == 0) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) w[i] = fz[i] - ft[i];
+        lse_add8(Z, fz, w, nv);
+        lse_add8(Q, ft, nullptr, nv);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) w[i] = ft[i] - fz[i];
+        lse_add8(Z, fz, nullptr, nv);
+        lse_add8(Q, ft, w, nv);
+      }
+    } else {
+      lse_add8(Z, fz, nullptr, nv);
+    }
+  };
+  int c = threadIdx.x * 8;
+  for (; c + step + 8 <= V; c += 2 * step) {   // two full vectors per trip: twice the loads in flight
+    float z0[8], t0[8], z1[8], t1[8];
+    Vec8<T>::load(zr + c, z0);
+    Vec8<T>::load(zr + c + step, z1);
+    if (tr) {
+      Vec8<T>::load(tr + c, t0);
+      Vec8<T>::load(tr + c + step, t1);
+    }
+    consume(z0, t0, 8);
+    consume(z1, t1, 8);
+  }
+  for (; c < V; c += step) {
     float fz[8], ft[8];
     Vec8<T>::load(zr + c, fz);
     if (tr) Vec8<T>::load(tr + c, ft);
-    float lz = -INFINITY, lt = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      if (c + i < V) { lz = fmaxf(lz, fz[i]); if (tr) lt = fmaxf(lt, ft[i]); }
-    if (lz > Z.m) { const float sc = expf(Z.m - lz); Z.s *= sc; Z.a *= sc; Z.m = lz; }
-    if (tr && lt > Q.m) { const float sc = expf(Q.m - lt); Q.s *= sc; Q.a *= sc; Q.m = lt; }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      if (c + i >= V) continue;
-      const float ez = expf(fz[i] - Z.m);
-      Z.s += ez;
-      if (tr) {
-        const float et = expf(ft[i] - Q.m);
-        Q.s += et;
-        if (kl_dir == 0) Z.a += ez * (fz[i] - ft[i]);
-        else Q.a += et * (ft[i] - fz[i]);
-      }
-    }
+    consume(fz, ft, min(8, V - c));
   }
   Z = warp_merge(Z);
   if (tr) Q = warp_merge(Q);
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  if (lane == 0) { shz[w] = Z; sht[w] = Q; }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  if (lane == 0) { shz[wid] = Z; sht[wid] = Q; }
   __syncthreads();
   if (threadIdx.x == 0) {
     Lse3 a = shz[0], b = sht[0];
     for (int i = 1; i < nw; ++i) { a = lse_merge(a, shz[i]); if (tr) b = lse_merge(b, sht[i]); }
-    const float lse_z = a.m + logf(a.s);
+    const float lse_z = (a.m + log2f(a.s)) * kLn2;
     float lse_t = 0.f, kl = 0.f;
     if (tr) {
-      lse_t = b.m + logf(b.s);
+      lse_t = (b.m + log2f(b.s)) * kLn2;
       kl = kl_dir == 0 ? a.a / a.s - lse_z + lse_t : b.a / b.s - lse_t + lse_z;
     }
     const float ce = lse_z - to_f(zr[y]);
@@ -460,10 +511,12 @@ __global__ void __launch_bounds__(512) local_loss_k(const T* __restrict__ z, con
   }
   __syncthreads();
   const float lse_z = sh_stats[0], lse_t = sh_stats[1], kl = sh_stats[2];
+  const float lz2 = lse_z * kL2e, lt2 = lse_t * kL2e, dl = lse_z - lse_t;
   const int cnt = *count;
   const float inv_n = cnt > 0 ? 1.f / (float)cnt : 0.f;
   const float wt = inv_n * alpha, wc = inv_n * (1.f - alpha);
-  for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) {
+  // pass 2 (the row was just read by this block: L2 hits)
+  for (int c = threadIdx.x * 8; c < ldz; c += step) {
     float fz[8], ft[8], o[8];
     Vec8<T>::load(zr + c, fz);
     if (tr) Vec8<T>::load(tr + c, ft);
@@ -471,11 +524,11 @@ __global__ void __launch_bounds__(512) local_loss_k(const T* __restrict__ z, con
     for (int i = 0; i < 8; ++i) {
       const int j = c + i;
       if (j >= V) { o[i] = 0.f; continue; }
-      const float p = expf(fz[i] - lse_z);
+      const float p = exp2f(fmaf(fz[i], kL2e, -lz2));
       float gsum = wt * (p - (j == y ? 1.f : 0.f));
       if (tr) {
-        const float gc = kl_dir == 0 ? p * ((fz[i] - ft[i]) - (lse_z - lse_t) - kl) : p - expf(ft[i] - lse_t);
-        gsum += wc * gc;
+        const float gc = kl_dir == 0 ? p * ((fz[i] - ft[i]) - dl - kl) : p - exp2f(fmaf(ft[i], kL2e, -lt2));
+        gsum = fmaf(wc, gc, gsum);
       }
       o[i] = gsum;
     }
@@ -487,7 +540,10 @@ void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labe
                        float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s) {
   note_launch(1);
   if (N <= 0) return;
-  const int th = 512;
+  // enough threads for one 8-wide vector each up to 1024; at most two 1024-thread rows per SM, so a
+  // row read in pass 1 is still in L2 for pass 2
+  int th = 32;
+  while (th < 1024 && th * 8 < ldz) th *= 2;
   if (dt == BF16)
     local_loss_k<bf16><<<N, th, 0, s>>>((const bf16*)z, (const bf16*)t, labels, V, ldz, alpha, kl_dir, count,
                                         (bf16*)dz, row_loss);
