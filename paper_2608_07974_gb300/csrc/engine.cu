@@ -306,6 +306,7 @@ void layer_fwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* x, void* 
 struct BwdWs {
   void *da, *dhid, *dxn, *dx2, *datt, *dqkv, *dy0, *dy1;
   float *part_g, *part_b, *D;
+  unsigned* counter;   // column-sum completion ticket (zero between launches)
 };
 
 size_t bwd_ws_bytes(zl_ctx* c, int N, int B, int S) {
@@ -324,6 +325,7 @@ size_t bwd_ws_bytes(zl_ctx* c, int N, int B, int S) {
   add((size_t)colsum_blocks(N) * wmax * 4);
   add((size_t)colsum_blocks(N) * wmax * 4);
   add((size_t)B * c->H * S * 4);
+  add(4);
   return b;
 }
 
@@ -341,22 +343,20 @@ void carve_ws(zl_ctx* c, Arena& a, BwdWs& w, int N, int B, int S) {
   w.part_g = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
   w.part_b = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
   w.D = (float*)a.take((size_t)B * c->H * S * 4);
+  w.counter = (unsigned*)a.take(4);
 }
 
 void bias_grad(zl_ctx* c, const void* dY, int N, int cols, float* g, BwdWs& w, cudaStream_t s) {
   if (!g) return;
-  ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * cols, 2);
-  launch_colsum(c->dt, dY, w.part_b, N, cols, s);
-  launch_partials_add(w.part_b, colsum_blocks(N), cols, g, s);
+  ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * cols, 1);
+  launch_colsum(c->dt, dY, w.part_b, N, cols, g, w.counter, s);
 }
 
 void norm_param_grad(zl_ctx* c, const void* x, const float* rstd, const float* mean, const void* dyn, int N,
                      float* gw, float* gb, BwdWs& w, cudaStream_t s) {
   const bool ln = !c->llama;
-  ProfScope p(c, s, PC_NORM, 0, 2.0 * esz(c) * (double)N * c->d, ln ? 3 : 2);
-  launch_norm_bwd_dparam(c->dt, ln, x, rstd, mean, dyn, w.part_g, w.part_b, N, c->d, s);
-  launch_partials_add(w.part_g, colsum_blocks(N), c->d, gw, s);
-  if (ln) launch_partials_add(w.part_b, colsum_blocks(N), c->d, gb, s);
+  ProfScope p(c, s, PC_NORM, 0, 2.0 * esz(c) * (double)N * c->d, 1);
+  launch_norm_bwd_dparam(c->dt, ln, x, rstd, mean, dyn, w.part_g, w.part_b, N, c->d, gw, gb, w.counter, s);
 }
 
 // dy: gradient w.r.t. the layer output; dx (may be NULL): gradient w.r.t. the layer input.
@@ -451,6 +451,7 @@ void chunk_bwd(zl_ctx* c, Chunk& k, ChunkActs& acts, const void* dh, void* dh_in
   a.cap = wb;
   BwdWs w;
   carve_ws(c, a, w, N, B, S);
+  CK(cudaMemsetAsync(w.counter, 0, 4, s));
   const void* dy = dh;
   for (int i = nl - 1; i >= 0; --i) {
     void* dx = i > 0 ? ((i % 2) ? w.dy0 : w.dy1) : dh_in;

@@ -1,6 +1,7 @@
 // Memory-bound kernels of the ZeroLock local step: embedding gather, norms, RoPE, activations,
 // the fused local objective (Eq. 3-5) and the per-chunk AdamW update.
 #include <math.h>
+#include <stdlib.h>
 
 #include "common.cuh"
 #include "ops.h"
@@ -108,14 +109,132 @@ __global__ void norm_fwd_k(const T* __restrict__ x, const float* __restrict__ g,
   }
 }
 
+// Row held in registers (d <= 256 * VPL): one read of x, every load issued before the reductions.
+template <typename T, bool LN, int VPL>
+__global__ void norm_fwd_reg_k(const T* __restrict__ x, const float* __restrict__ g, const float* __restrict__ b,
+                               T* __restrict__ y, float* __restrict__ rstd_o, float* __restrict__ mean_o, int N, int d,
+                               float eps) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= N) return;
+  const T* xr = x + (size_t)row * d;
+  float f[VPL][8];
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int c = lane * 8 + v * 256;
+    if (c < d) Vec8<T>::load(xr + c, f[v]);
+    else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) f[v][i] = 0.f;
+    }
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int v = 0; v < VPL; ++v)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s += f[v][i];
+  const float mean = LN ? warp_sum(s) / d : 0.f;
+  float q = 0.f;
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int c = lane * 8 + v * 256;
+    if (c < d) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { const float t = f[v][i] - mean; q += t * t; }
+    }
+  }
+  const float rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
+  T* yr = y + (size_t)row * d;
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int c = lane * 8 + v * 256;
+    if (c >= d) continue;
+    float o[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      o[i] = (f[v][i] - mean) * rstd * (g ? g[c + i] : 1.f);
+      if (LN && b) o[i] += b[c + i];
+    }
+    Vec8<T>::store(yr + c, o);
+  }
+  if (lane == 0) {
+    if (rstd_o) rstd_o[row] = rstd;
+    if (LN && mean_o) mean_o[row] = mean;
+  }
+}
+
+template <typename T, bool LN, int VPL>
+__global__ void norm_bwd_dx_reg_k(const T* __restrict__ x, const float* __restrict__ g,
+                                  const float* __restrict__ rstd, const float* __restrict__ mean,
+                                  const T* __restrict__ dy, const T* __restrict__ dres, T* __restrict__ dx, int N,
+                                  int d) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= N) return;
+  const size_t o = (size_t)row * d;
+  const float r = rstd[row], mu = LN ? mean[row] : 0.f;
+  float fx[VPL][8], fd[VPL][8];
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int c = lane * 8 + v * 256;
+    if (c < d) {
+      Vec8<T>::load(x + o + c, fx[v]);
+      Vec8<T>::load(dy + o + c, fd[v]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) fx[v][i] = fd[v][i] = 0.f;
+    }
+  }
+  float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int c = lane * 8 + v * 256;
+    if (c >= d) continue;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      fd[v][i] *= (g ? g[c + i] : 1.f);       // dy * gain
+      fx[v][i] = (fx[v][i] - mu) * r;         // xhat
+      s1 += fd[v][i];
+      s2 += fd[v][i] * fx[v][i];
+    }
+  }
+  s1 = warp_sum(s1) / d;
+  s2 = warp_sum(s2) / d;
+#pragma unroll
+  for (int v = 0; v < VPL; ++v) {
+    const int c = lane * 8 + v * 256;
+    if (c >= d) continue;
+    float res[8], out[8];
+    if (dres) Vec8<T>::load(dres + o + c, res);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      out[i] = r * (fd[v][i] - (LN ? s1 : 0.f) - fx[v][i] * s2);
+      if (dres) out[i] += res[i];
+    }
+    Vec8<T>::store(dx + o + c, out);
+  }
+}
+
 void launch_norm_fwd(int dt, bool ln, const void* x, const float* g, const float* b, void* y, float* rstd,
                      float* mean, int N, int d, float eps, cudaStream_t s) {
   note_launch(1);
   const int th = 256, blocks = (N * 32 + th - 1) / th;
+  const int vpl = (d + 255) / 256;
+#define NFR(T, L, V) norm_fwd_reg_k<T, L, V><<<blocks, th, 0, s>>>((const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
+#define NFV(T, L)                     \
+  if (vpl == 1) NFR(T, L, 1);         \
+  else if (vpl == 2) NFR(T, L, 2);    \
+  else if (vpl == 3) NFR(T, L, 3);    \
+  else NFR(T, L, 4);
 #define NF(T, L) norm_fwd_k<T, L><<<blocks, th, 0, s>>>((const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
-  if (dt == BF16) { if (ln) NF(bf16, true); else NF(bf16, false); }
-  else { if (ln) NF(float, true); else NF(float, false); }
+  if (vpl <= 4) {
+    if (dt == BF16) { if (ln) { NFV(bf16, true) } else { NFV(bf16, false) } }
+    else { if (ln) { NFV(float, true) } else { NFV(float, false) } }
+  } else {
+    if (dt == BF16) { if (ln) NF(bf16, true); else NF(bf16, false); }
+    else { if (ln) NF(float, true); else NF(float, false); }
+  }
 #undef NF
+#undef NFV
+#undef NFR
 }
 
 // dx = rstd * (dyh - mean(dyh) [LN] - xhat * mean(dyh * xhat)), dyh = g * dy.
@@ -163,11 +282,27 @@ void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const fl
                         const void* dy, const void* dres, void* dx, int N, int d, cudaStream_t s) {
   note_launch(1);
   const int th = 256, blocks = (N * 32 + th - 1) / th;
+  const int vpl = (d + 255) / 256;
+#define NBR(T, L, V)                                                                                             \
+  norm_bwd_dx_reg_k<T, L, V><<<blocks, th, 0, s>>>((const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, \
+                                                   N, d)
+#define NBV(T, L)                     \
+  if (vpl == 1) NBR(T, L, 1);         \
+  else if (vpl == 2) NBR(T, L, 2);    \
+  else if (vpl == 3) NBR(T, L, 3);    \
+  else NBR(T, L, 4);
 #define NB(T, L) \
   norm_bwd_dx_k<T, L><<<blocks, th, 0, s>>>((const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, N, d)
-  if (dt == BF16) { if (ln) NB(bf16, true); else NB(bf16, false); }
-  else { if (ln) NB(float, true); else NB(float, false); }
+  if (vpl <= 4) {
+    if (dt == BF16) { if (ln) { NBV(bf16, true) } else { NBV(bf16, false) } }
+    else { if (ln) { NBV(float, true) } else { NBV(float, false) } }
+  } else {
+    if (dt == BF16) { if (ln) NB(bf16, true); else NB(bf16, false); }
+    else { if (ln) NB(float, true); else NB(float, false); }
+  }
 #undef NB
+#undef NBV
+#undef NBR
 }
 
 static constexpr int kColRows = 64;   // rows per partial-sum block
@@ -175,11 +310,15 @@ int colsum_blocks(int N) { return (N + kColRows - 1) / kColRows; }
 
 // block (32, 8): 32 threads x 8 columns each (256 columns, 16-byte loads) x 8 row lanes;
 // grid (ceil(d/256), colsum_blocks(N)). Requires d % 8 == 0.
+// After its partial sums, the last block to finish (ticket counter) adds sum_b part[b][c], b in
+// increasing order, into the outputs and re-arms the counter: deterministic, one launch.
 template <typename T, bool NORM, bool LN>
 __global__ void __launch_bounds__(256) colsum_k(const T* __restrict__ A, const T* __restrict__ x,
                                                 const float* __restrict__ rstd, const float* __restrict__ mean,
                                                 float* __restrict__ part_g, float* __restrict__ part_b, int N,
-                                                int d) {
+                                                int d, float* __restrict__ out_g, float* __restrict__ out_b,
+                                                unsigned* __restrict__ counter) {
+  __shared__ unsigned ticket;
   __shared__ float sg[8][256], sb[8][256];
   const int c0 = blockIdx.x * 256 + threadIdx.x * 8;
   const int r0 = blockIdx.y * kColRows;
@@ -219,26 +358,53 @@ __global__ void __launch_bounds__(256) colsum_k(const T* __restrict__ A, const T
       part_b[(size_t)blockIdx.y * d + c] = tb;
     }
   }
+  __threadfence();
+  __syncthreads();
+  if (t == 0) ticket = atomicAdd(counter, 1u);
+  __syncthreads();
+  if (ticket != gridDim.x * gridDim.y - 1) return;
+  __threadfence();
+  const int nb = gridDim.y;
+  for (int cc = t; cc < d; cc += 256) {
+    if (NORM) {
+      float a = 0.f, bsum = 0.f;
+      for (int bb = 0; bb < nb; ++bb) {
+        a += __ldcg(part_g + (size_t)bb * d + cc);
+        if (LN) bsum += __ldcg(part_b + (size_t)bb * d + cc);
+      }
+      out_g[cc] += a;
+      if (LN) out_b[cc] += bsum;
+    } else {
+      float bsum = 0.f;
+      for (int bb = 0; bb < nb; ++bb) bsum += __ldcg(part_b + (size_t)bb * d + cc);
+      out_b[cc] += bsum;
+    }
+  }
+  if (t == 0) *counter = 0u;
 }
 
 void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, const float* mean,
-                            const void* dy, float* part_g, float* part_b, int N, int d, cudaStream_t s) {
+                            const void* dy, float* part_g, float* part_b, int N, int d, float* out_g, float* out_b,
+                            unsigned* counter, cudaStream_t s) {
   note_launch(1);
   dim3 grid((d + 255) / 256, colsum_blocks(N)), block(32, 8);
-#define CS(T, L) \
-  colsum_k<T, true, L><<<grid, block, 0, s>>>((const T*)dy, (const T*)x, rstd, mean, part_g, part_b, N, d)
+#define CS(T, L)                                                                                             \
+  colsum_k<T, true, L><<<grid, block, 0, s>>>((const T*)dy, (const T*)x, rstd, mean, part_g, part_b, N, d, out_g, \
+                                              out_b, counter)
   if (dt == BF16) { if (ln) CS(bf16, true); else CS(bf16, false); }
   else { if (ln) CS(float, true); else CS(float, false); }
 #undef CS
 }
 
-void launch_colsum(int dt, const void* A, float* part, int N, int d, cudaStream_t s) {
+void launch_colsum(int dt, const void* A, float* part, int N, int d, float* out, unsigned* counter, cudaStream_t s) {
   note_launch(1);
   dim3 grid((d + 255) / 256, colsum_blocks(N)), block(32, 8);
   if (dt == BF16)
-    colsum_k<bf16, false, false><<<grid, block, 0, s>>>((const bf16*)A, nullptr, nullptr, nullptr, nullptr, part, N, d);
+    colsum_k<bf16, false, false><<<grid, block, 0, s>>>((const bf16*)A, nullptr, nullptr, nullptr, nullptr, part, N, d,
+                                                        nullptr, out, counter);
   else
-    colsum_k<float, false, false><<<grid, block, 0, s>>>((const float*)A, nullptr, nullptr, nullptr, nullptr, part, N, d);
+    colsum_k<float, false, false><<<grid, block, 0, s>>>((const float*)A, nullptr, nullptr, nullptr, nullptr, part, N,
+                                                         d, nullptr, out, counter);
 }
 
 __global__ void partials_add_k(const float* __restrict__ part, int nb, int d, float* __restrict__ out) {
@@ -388,12 +554,23 @@ void launch_gelu_bwd(int dt, const void* x, const void* dy, void* dx, size_t n, 
 // One block per row; pass 1 keeps online (max, sum) pairs, pass 2 writes dz. No probability
 // tensor is stored.
 // ------------------------------------------------------------------------------------------
+constexpr float kL2e = 1.4426950408889634f, kLn2 = 0.6931471805599453f;
+
+// 2^x by the SFU's ex2.approx (relative error about 2^-22; flushes subnormal results to zero,
+// which only affects probabilities below 1e-38).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+
 struct Lse3 { float m, s, a; };   // running max (log2 units), sum 2^(x-m), sum 2^(x-m) * w
 
 __device__ __forceinline__ Lse3 lse_merge(Lse3 x, Lse3 y) {
   const float M = fmaxf(x.m, y.m);
   if (M == -INFINITY) return x;
-  const float ex = exp2f(x.m - M), ey = exp2f(y.m - M);
+  const float ex = ex2(x.m - M), ey = ex2(y.m - M);
   return Lse3{M, x.s * ex + y.s * ey, x.a * ex + y.a * ey};
 }
 
@@ -407,7 +584,6 @@ __device__ __forceinline__ Lse3 warp_merge(Lse3 v) {
   return v;
 }
 
-constexpr float kL2e = 1.4426950408889634f, kLn2 = 0.6931471805599453f;
 
 // Adds 8 values (natural-log logits f, weights w) to an online base-2 log-sum-exp.
 __device__ __forceinline__ void lse_add8(Lse3& A, const float* f, const float* w, int nvalid) {
@@ -416,7 +592,7 @@ __device__ __forceinline__ void lse_add8(Lse3& A, const float* f, const float* w
   for (int i = 0; i < 8; ++i)
     if (i < nvalid) mx = fmaxf(mx, f[i] * kL2e);
   if (mx > A.m) {
-    const float sc = exp2f(A.m - mx);
+    const float sc = ex2(A.m - mx);
     A.s *= sc;
     A.a *= sc;
     A.m = mx;
@@ -424,7 +600,7 @@ __device__ __forceinline__ void lse_add8(Lse3& A, const float* f, const float* w
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     if (i < nvalid) {
-      const float e = exp2f(fmaf(f[i], kL2e, -A.m));
+      const float e = ex2(fmaf(f[i], kL2e, -A.m));
       A.s += e;
       if (w) A.a = fmaf(e, w[i], A.a);
     }
@@ -524,10 +700,10 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
     for (int i = 0; i < 8; ++i) {
       const int j = c + i;
       if (j >= V) { o[i] = 0.f; continue; }
-      const float p = exp2f(fmaf(fz[i], kL2e, -lz2));
+      const float p = ex2(fmaf(fz[i], kL2e, -lz2));
       float gsum = wt * (p - (j == y ? 1.f : 0.f));
       if (tr) {
-        const float gc = kl_dir == 0 ? p * ((fz[i] - ft[i]) - dl - kl) : p - exp2f(fmaf(ft[i], kL2e, -lt2));
+        const float gc = kl_dir == 0 ? p * ((fz[i] - ft[i]) - dl - kl) : p - ex2(fmaf(ft[i], kL2e, -lt2));
         gsum = fmaf(wc, gc, gsum);
       }
       o[i] = gsum;
@@ -542,8 +718,13 @@ void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labe
   if (N <= 0) return;
   // enough threads for one 8-wide vector each up to 1024; at most two 1024-thread rows per SM, so a
   // row read in pass 1 is still in L2 for pass 2
+  int cap = 512;   // two or more rows in flight per SM; the rows being read still fit in L2
+  if (const char* e = std::getenv("ZL_LOSS_THREADS")) {   // tuning override
+    const int v = std::atoi(e);
+    if (v == 128 || v == 256 || v == 512 || v == 1024) cap = v;
+  }
   int th = 32;
-  while (th < 1024 && th * 8 < ldz) th *= 2;
+  while (th < cap && th * 8 < ldz) th *= 2;
   if (dt == BF16)
     local_loss_k<bf16><<<N, th, 0, s>>>((const bf16*)z, (const bf16*)t, labels, V, ldz, alpha, kl_dir, count,
                                         (bf16*)dz, row_loss);
