@@ -29,8 +29,9 @@ namespace {
 using namespace zl;
 
 // Kernel classes of the per-launch profile (zl_profile).
-enum { PC_GEMM, PC_ATTN_F, PC_ATTN_B, PC_LOSS, PC_NORM, PC_ADAMW, PC_ELEM, PC_COUNT };
-const char* kPCName[PC_COUNT] = {"gemm", "attn_fwd", "attn_bwd", "local_loss", "norm", "adamw", "elementwise"};
+enum { PC_GEMM, PC_GEMM_HEAD, PC_ATTN_F, PC_ATTN_B, PC_LOSS, PC_NORM, PC_ADAMW, PC_ELEM, PC_COUNT };
+const char* kPCName[PC_COUNT] = {"gemm_layer", "gemm_head", "attn_fwd", "attn_bwd", "local_loss", "norm", "adamw",
+                                 "elementwise"};
 struct ProfRec {
   int cls;
   cudaEvent_t a, b;
@@ -219,7 +220,8 @@ void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, 
        const float* bias, const void* R) {
   const double e = (double)esz(c);
   const double out = mode == 2 ? 8.0 * M * N : (R ? 2.0 : 1.0) * e * M * N;
-  ProfScope p(c, s, PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
+  const bool head = B == c->lm_head;
+  ProfScope p(c, s, head ? PC_GEMM_HEAD : PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
   gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool);
 }
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
@@ -523,7 +525,7 @@ void* local_loss(zl_ctx* c, const void* z, const void* t, const int32_t* labels,
   {
     ProfScope p(c, s, PC_LOSS, 0, (alpha < 1.f ? 3.0 : 2.0) * esz(c) * (double)N * c->Vp);
     launch_local_loss(c->dt, z, alpha < 1.f ? t : nullptr, labels, N, c->V, c->Vp, alpha, c->cfg.kl_dir,
-                      c->d_count + slot, dz, rl, s);
+                      c->d_count + slot, dz, rl, s, c->d_err);
   }
   launch_loss_reduce(rl, N, c->d_count + slot, c->d_losses + slot, s);
   CHECK_LAUNCH();

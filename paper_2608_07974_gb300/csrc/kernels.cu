@@ -712,8 +712,185 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
   }
 }
 
+// ------------------------------------------------------------------------------------------
+// The same objective with the row streamed through shared memory by 1-D TMA bulk copies: a ring of
+// kLossStages chunks of z (and t) per CTA keeps tens of KB per SM in flight without registers.
+// Pass 1 streams the row from HBM, pass 2 streams it again (an L2 hit) and writes dz.
+// ------------------------------------------------------------------------------------------
+constexpr int kLossChunk = 4096;    // elements per chunk
+constexpr int kLossStages = 4;
+constexpr unsigned long long kLossTimeoutNs = 2000000000ull;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ unsigned long long gtime() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(512, 2) local_loss_tma_k(const T* __restrict__ z, const T* __restrict__ t,
+                                                          const int32_t* __restrict__ labels, int V, int ldz,
+                                                          float alpha, int kl_dir, const int* __restrict__ count,
+                                                          T* __restrict__ dz, float* __restrict__ row_loss,
+                                                          unsigned* err) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  __shared__ __align__(8) uint64_t full[kLossStages];
+  __shared__ Lse3 shz[16], sht[16];
+  __shared__ float sh_stats[4];
+  __shared__ int abort_flag;
+  T* zbuf = reinterpret_cast<T*>(sm);                        // [stages][chunk]
+  T* tbuf = zbuf + kLossStages * kLossChunk;                 // [stages][chunk] when t != NULL
+  const int row = blockIdx.x;
+  const T* zr = z + (size_t)row * ldz;
+  const T* tr = t ? t + (size_t)row * ldz : nullptr;
+  T* dr = dz + (size_t)row * ldz;
+  const int y = labels[row];
+  if (!(y >= 0 && y < V)) {   // rows outside Omega: no loss, zero gradient
+    float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) Vec8<T>::store(dr + c, f);
+    if (threadIdx.x == 0) row_loss[row] = 0.f;
+    return;
+  }
+  const int nch = (ldz + kLossChunk - 1) / kLossChunk;
+  const int total = 2 * nch;   // pass 1 then pass 2 over the same chunks
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kLossStages; ++s)
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full[s])) : "memory");
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  auto issue = [&](int i) {   // chunk i % nch of the row into stage i % kLossStages
+    const int ch = i % nch, st = i % kLossStages;
+    const int c0 = ch * kLossChunk, len = min(kLossChunk, ldz - c0);
+    const uint32_t bytes = (uint32_t)(len * sizeof(T));
+    const uint32_t bar = smem_u32(&full[st]);
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(tr ? 2 * bytes : bytes)
+                 : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(zbuf + st * kLossChunk)),
+                 "l"(zr + c0), "r"(bytes), "r"(bar)
+                 : "memory");
+    if (tr)
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                       smem_u32(tbuf + st * kLossChunk)),
+                   "l"(tr + c0), "r"(bytes), "r"(bar)
+                   : "memory");
+  };
+  if (threadIdx.x == 0)
+    for (int i = 0; i < kLossStages && i < total; ++i) issue(i);
+  Lse3 Z{-INFINITY, 0.f, 0.f}, Q{-INFINITY, 0.f, 0.f};
+  float lz2 = 0.f, lt2 = 0.f, dl = 0.f, kl = 0.f, wt = 0.f, wc = 0.f;
+  bool ok = true;
+  for (int i = 0; i < total; ++i) {
+    const int st = i % kLossStages;
+    const uint32_t parity = (uint32_t)(i / kLossStages) & 1u;
+    // bounded wait for the stage
+    {
+      uint32_t done = 0;
+      const unsigned long long t0 = gtime();
+      while (true) {
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.b32 %0, 1, 0, p;\n}"
+            : "=r"(done)
+            : "r"(smem_u32(&full[st])), "r"(parity)
+            : "memory");
+        if (done) break;
+        if (abort_flag || gtime() - t0 > kLossTimeoutNs) {
+          abort_flag = 1;
+          ok = false;
+          break;
+        }
+      }
+    }
+    if (!ok) break;
+    const int ch = i % nch;
+    const int c = ch * kLossChunk + threadIdx.x * 8;
+    const int nv = min(8, V - c);
+    if (i < nch) {
+      // pass 1
+      if (threadIdx.x * 8 < kLossChunk && nv > 0) {
+        float fz[8], ft[8], w[8];
+        Vec8<T>::load(zbuf + st * kLossChunk + threadIdx.x * 8, fz);
+        if (tr) {
+          Vec8<T>::load(tbuf + st * kLossChunk + threadIdx.x * 8, ft);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) w[k] = kl_dir == 0 ? fz[k] - ft[k] : ft[k] - fz[k];
+          lse_add8(Z, fz, kl_dir == 0 ? w : nullptr, nv);
+          lse_add8(Q, ft, kl_dir == 0 ? nullptr : w, nv);
+        } else {
+          lse_add8(Z, fz, nullptr, nv);
+        }
+      }
+      if (i == nch - 1) {   // row statistics
+        Z = warp_merge(Z);
+        if (tr) Q = warp_merge(Q);
+        const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+        if (lane == 0) { shz[wid] = Z; sht[wid] = Q; }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+          Lse3 a = shz[0], b = sht[0];
+          for (int k = 1; k < nw; ++k) { a = lse_merge(a, shz[k]); if (tr) b = lse_merge(b, sht[k]); }
+          const float lse_z = (a.m + log2f(a.s)) * kLn2;
+          float lse_t = 0.f, kld = 0.f;
+          if (tr) {
+            lse_t = (b.m + log2f(b.s)) * kLn2;
+            kld = kl_dir == 0 ? a.a / a.s - lse_z + lse_t : b.a / b.s - lse_t + lse_z;
+          }
+          row_loss[row] = alpha * (lse_z - to_f(zr[y])) + (tr ? (1.f - alpha) * kld : 0.f);
+          sh_stats[0] = lse_z;
+          sh_stats[1] = lse_t;
+          sh_stats[2] = kld;
+        }
+        __syncthreads();
+        const float lse_z = sh_stats[0], lse_t = sh_stats[1];
+        kl = sh_stats[2];
+        lz2 = lse_z * kL2e;
+        lt2 = lse_t * kL2e;
+        dl = lse_z - lse_t;
+        const int cnt = *count;
+        const float inv_n = cnt > 0 ? 1.f / (float)cnt : 0.f;
+        wt = inv_n * alpha;
+        wc = inv_n * (1.f - alpha);
+      }
+    } else if (threadIdx.x * 8 < kLossChunk && c < ldz) {
+      // pass 2: dz for this chunk
+      float fz[8], ft[8], o[8];
+      Vec8<T>::load(zbuf + st * kLossChunk + threadIdx.x * 8, fz);
+      if (tr) Vec8<T>::load(tbuf + st * kLossChunk + threadIdx.x * 8, ft);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int j = c + k;
+        if (j >= V) { o[k] = 0.f; continue; }
+        const float p = ex2(fmaf(fz[k], kL2e, -lz2));
+        float gsum = wt * (p - (j == y ? 1.f : 0.f));
+        if (tr) {
+          const float gc = kl_dir == 0 ? p * ((fz[k] - ft[k]) - dl - kl) : p - ex2(fmaf(ft[k], kL2e, -lt2));
+          gsum = fmaf(wc, gc, gsum);
+        }
+        o[k] = gsum;
+      }
+      Vec8<T>::store(dr + c, o);
+    }
+    __syncthreads();   // the stage is free again
+    if (threadIdx.x == 0 && i + kLossStages < total) issue(i + kLossStages);
+  }
+  if (!ok) {
+    if (threadIdx.x == 0) {
+      if (err) atomicOr(err, ZL_DEVERR_TIMEOUT);
+      // let copies still in flight land before the CTA's shared memory is reused
+      const unsigned long long t0 = gtime();
+      while (gtime() - t0 < 100000000ull) {
+      }
+    }
+    __syncthreads();
+  }
+}
+
 void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labels, int N, int V, int ldz,
-                       float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s) {
+                       float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s,
+                       unsigned* err) {
   note_launch(1);
   if (N <= 0) return;
   // enough threads for one 8-wide vector each up to 1024; at most two 1024-thread rows per SM, so a
@@ -725,6 +902,18 @@ void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labe
   }
   int th = 32;
   while (th < cap && th * 8 < ldz) th *= 2;
+  if (dt == BF16 && ldz % 8 == 0 && !std::getenv("ZL_LOSS_SIMPLE")) {
+    const int smem = kLossStages * kLossChunk * 2 * (t ? 2 : 1);
+    static bool attr = false;
+    if (!attr) {
+      cudaFuncSetAttribute(local_loss_tma_k<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kLossStages * kLossChunk * 2 * 2);
+      attr = true;
+    }
+    local_loss_tma_k<bf16><<<N, 512, smem, s>>>((const bf16*)z, (const bf16*)t, labels, V, ldz, alpha, kl_dir, count,
+                                                (bf16*)dz, row_loss, err);
+    return;
+  }
   if (dt == BF16)
     local_loss_k<bf16><<<N, th, 0, s>>>((const bf16*)z, (const bf16*)t, labels, V, ldz, alpha, kl_dir, count,
                                         (bf16*)dz, row_loss);
