@@ -525,7 +525,7 @@ void* local_loss(zl_ctx* c, const void* z, const void* t, const int32_t* labels,
   {
     ProfScope p(c, s, PC_LOSS, 0, (alpha < 1.f ? 3.0 : 2.0) * esz(c) * (double)N * c->Vp);
     launch_local_loss(c->dt, z, alpha < 1.f ? t : nullptr, labels, N, c->V, c->Vp, alpha, c->cfg.kl_dir,
-                      c->d_count + slot, dz, rl, s, c->d_err);
+                      c->d_count + slot, dz, rl, s);
   }
   launch_loss_reduce(rl, N, c->d_count + slot, c->d_losses + slot, s);
   CHECK_LAUNCH();

@@ -585,12 +585,14 @@ __device__ __forceinline__ Lse3 warp_merge(Lse3 v) {
 }
 
 
-// Adds 8 values (natural-log logits f, weights w) to an online base-2 log-sum-exp.
-__device__ __forceinline__ void lse_add8(Lse3& A, const float* f, const float* w, int nvalid) {
+// Online base-2 log-sum-exp of 8 values already scaled by log2(e) (xs), optionally with the cross
+// term sum 2^(xs - m) * w. nvalid < 8 only for the last, partial vector of a row.
+template <bool FULL>
+__device__ __forceinline__ void lse_add8(Lse3& A, const float* xs, const float* w, int nvalid) {
   float mx = -INFINITY;
 #pragma unroll
   for (int i = 0; i < 8; ++i)
-    if (i < nvalid) mx = fmaxf(mx, f[i] * kL2e);
+    if (FULL || i < nvalid) mx = fmaxf(mx, xs[i]);
   if (mx > A.m) {
     const float sc = ex2(A.m - mx);
     A.s *= sc;
@@ -599,327 +601,137 @@ __device__ __forceinline__ void lse_add8(Lse3& A, const float* f, const float* w
   }
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    if (i < nvalid) {
-      const float e = ex2(fmaf(f[i], kL2e, -A.m));
+    if (FULL || i < nvalid) {
+      const float e = ex2(xs[i] - A.m);
       A.s += e;
       if (w) A.a = fmaf(e, w[i], A.a);
     }
   }
 }
 
-template <typename T>
+template <typename T, bool TEACHER, int KLDIR, bool FULL>
+__device__ __forceinline__ void loss_pass1_vec(const T* zp, const T* tp, Lse3& Z, Lse3& Q, int nv) {
+  float zs[8], ts[8], w[8];
+  Vec8<T>::load(zp, zs);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) zs[i] *= kL2e;
+  if (TEACHER) {
+    Vec8<T>::load(tp, ts);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      ts[i] *= kL2e;
+      w[i] = KLDIR == 0 ? zs[i] - ts[i] : ts[i] - zs[i];   // in log2 units; scaled by ln 2 at the end
+    }
+    lse_add8<FULL>(Z, zs, KLDIR == 0 ? w : nullptr, nv);
+    lse_add8<FULL>(Q, ts, KLDIR == 0 ? nullptr : w, nv);
+  } else {
+    lse_add8<FULL>(Z, zs, nullptr, nv);
+  }
+}
+
+// One block per row of logits. Pass 1: base-2 online log-sum-exp of z and t and the KL cross term
+// (two full vectors per trip for loads in flight); pass 2 (the row is still in L2) writes dz.
+template <typename T, bool TEACHER, int KLDIR>
 __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, const T* __restrict__ t,
                                                      const int32_t* __restrict__ labels, int V, int ldz,
-                                                     float alpha, int kl_dir, const int* __restrict__ count,
+                                                     float alpha, const int* __restrict__ count,
                                                      T* __restrict__ dz, float* __restrict__ row_loss) {
   __shared__ Lse3 shz[32], sht[32];
   __shared__ float sh_stats[4];
   const int row = blockIdx.x;
   const T* zr = z + (size_t)row * ldz;
-  const T* tr = t ? t + (size_t)row * ldz : nullptr;
+  const T* tr = TEACHER ? t + (size_t)row * ldz : nullptr;
   T* dr = dz + (size_t)row * ldz;
   const int y = labels[row];
-  const bool valid = y >= 0 && y < V;
   const int step = blockDim.x * 8;
-  if (!valid) {   // rows outside Omega: no loss, zero gradient
+  if (!(y >= 0 && y < V)) {   // rows outside Omega: no loss, zero gradient
     float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     for (int c = threadIdx.x * 8; c < ldz; c += step) Vec8<T>::store(dr + c, f);
     if (threadIdx.x == 0) row_loss[row] = 0.f;
     return;
   }
-  // pass 1: base-2 online log-sum-exp of z and t, plus the KL cross term
   Lse3 Z{-INFINITY, 0.f, 0.f}, Q{-INFINITY, 0.f, 0.f};
-  auto consume = [&](const float* fz, const float* ft, int nv) {
-    float w[8];
-    if (tr) {
-      if (kl_dir == 0) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) w[i] = fz[i] - ft[i];
-        lse_add8(Z, fz, w, nv);
-        lse_add8(Q, ft, nullptr, nv);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) w[i] = ft[i] - fz[i];
-        lse_add8(Z, fz, nullptr, nv);
-        lse_add8(Q, ft, w, nv);
-      }
-    } else {
-      lse_add8(Z, fz, nullptr, nv);
-    }
-  };
   int c = threadIdx.x * 8;
-  for (; c + step + 8 <= V; c += 2 * step) {   // two full vectors per trip: twice the loads in flight
-    float z0[8], t0[8], z1[8], t1[8];
-    Vec8<T>::load(zr + c, z0);
-    Vec8<T>::load(zr + c + step, z1);
-    if (tr) {
-      Vec8<T>::load(tr + c, t0);
-      Vec8<T>::load(tr + c + step, t1);
-    }
-    consume(z0, t0, 8);
-    consume(z1, t1, 8);
+  for (; c + step + 8 <= V; c += 2 * step) {
+    loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c, tr + c, Z, Q, 8);
+    loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c + step, tr + c + step, Z, Q, 8);
   }
   for (; c < V; c += step) {
-    float fz[8], ft[8];
-    Vec8<T>::load(zr + c, fz);
-    if (tr) Vec8<T>::load(tr + c, ft);
-    consume(fz, ft, min(8, V - c));
+    if (c + 8 <= V) loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c, tr + c, Z, Q, 8);
+    else loss_pass1_vec<T, TEACHER, KLDIR, false>(zr + c, tr + c, Z, Q, V - c);
   }
   Z = warp_merge(Z);
-  if (tr) Q = warp_merge(Q);
+  if (TEACHER) Q = warp_merge(Q);
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   if (lane == 0) { shz[wid] = Z; sht[wid] = Q; }
   __syncthreads();
   if (threadIdx.x == 0) {
     Lse3 a = shz[0], b = sht[0];
-    for (int i = 1; i < nw; ++i) { a = lse_merge(a, shz[i]); if (tr) b = lse_merge(b, sht[i]); }
+    for (int i = 1; i < nw; ++i) { a = lse_merge(a, shz[i]); if (TEACHER) b = lse_merge(b, sht[i]); }
     const float lse_z = (a.m + log2f(a.s)) * kLn2;
     float lse_t = 0.f, kl = 0.f;
-    if (tr) {
+    if (TEACHER) {
       lse_t = (b.m + log2f(b.s)) * kLn2;
-      kl = kl_dir == 0 ? a.a / a.s - lse_z + lse_t : b.a / b.s - lse_t + lse_z;
+      kl = KLDIR == 0 ? a.a / a.s * kLn2 - lse_z + lse_t : b.a / b.s * kLn2 - lse_t + lse_z;
     }
-    const float ce = lse_z - to_f(zr[y]);
-    row_loss[row] = alpha * ce + (tr ? (1.f - alpha) * kl : 0.f);
+    row_loss[row] = alpha * (lse_z - to_f(zr[y])) + (TEACHER ? (1.f - alpha) * kl : 0.f);
     sh_stats[0] = lse_z;
     sh_stats[1] = lse_t;
     sh_stats[2] = kl;
   }
   __syncthreads();
   const float lse_z = sh_stats[0], lse_t = sh_stats[1], kl = sh_stats[2];
-  const float lz2 = lse_z * kL2e, lt2 = lse_t * kL2e, dl = lse_z - lse_t;
+  const float lz2 = lse_z * kL2e, lt2 = lse_t * kL2e, shift = (lse_z - lse_t) + kl;
   const int cnt = *count;
   const float inv_n = cnt > 0 ? 1.f / (float)cnt : 0.f;
   const float wt = inv_n * alpha, wc = inv_n * (1.f - alpha);
-  // pass 2 (the row was just read by this block: L2 hits)
-  for (int c = threadIdx.x * 8; c < ldz; c += step) {
+  for (c = threadIdx.x * 8; c < ldz; c += step) {
     float fz[8], ft[8], o[8];
     Vec8<T>::load(zr + c, fz);
-    if (tr) Vec8<T>::load(tr + c, ft);
+    if (TEACHER) Vec8<T>::load(tr + c, ft);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const int j = c + i;
-      if (j >= V) { o[i] = 0.f; continue; }
       const float p = ex2(fmaf(fz[i], kL2e, -lz2));
-      float gsum = wt * (p - (j == y ? 1.f : 0.f));
-      if (tr) {
-        const float gc = kl_dir == 0 ? p * ((fz[i] - ft[i]) - dl - kl) : p - ex2(fmaf(ft[i], kL2e, -lt2));
-        gsum = fmaf(wc, gc, gsum);
+      float g = wt * p;
+      if (TEACHER) {
+        const float gc = KLDIR == 0 ? p * ((fz[i] - ft[i]) - shift) : p - ex2(fmaf(ft[i], kL2e, -lt2));
+        g = fmaf(wc, gc, g);
       }
-      o[i] = gsum;
+      o[i] = g;
+    }
+    if (y >= c && y < c + 8) o[y - c] -= wt;   // the one-hot of the task term
+    if (c + 8 > V) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        if (c + i >= V) o[i] = 0.f;   // padding columns
     }
     Vec8<T>::store(dr + c, o);
   }
 }
 
-// ------------------------------------------------------------------------------------------
-// The same objective with the row streamed through shared memory by 1-D TMA bulk copies: a ring of
-// kLossStages chunks of z (and t) per CTA keeps tens of KB per SM in flight without registers.
-// Pass 1 streams the row from HBM, pass 2 streams it again (an L2 hit) and writes dz.
-// ------------------------------------------------------------------------------------------
-constexpr int kLossChunk = 4096;    // elements per chunk
-constexpr int kLossStages = 4;
-constexpr unsigned long long kLossTimeoutNs = 2000000000ull;
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-__device__ __forceinline__ unsigned long long gtime() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-template <typename T>
-__global__ void __launch_bounds__(512, 2) local_loss_tma_k(const T* __restrict__ z, const T* __restrict__ t,
-                                                          const int32_t* __restrict__ labels, int V, int ldz,
-                                                          float alpha, int kl_dir, const int* __restrict__ count,
-                                                          T* __restrict__ dz, float* __restrict__ row_loss,
-                                                          unsigned* err) {
-  extern __shared__ __align__(128) uint8_t sm[];
-  __shared__ __align__(8) uint64_t full[kLossStages];
-  __shared__ Lse3 shz[16], sht[16];
-  __shared__ float sh_stats[4];
-  __shared__ int abort_flag;
-  T* zbuf = reinterpret_cast<T*>(sm);                        // [stages][chunk]
-  T* tbuf = zbuf + kLossStages * kLossChunk;                 // [stages][chunk] when t != NULL
-  const int row = blockIdx.x;
-  const T* zr = z + (size_t)row * ldz;
-  const T* tr = t ? t + (size_t)row * ldz : nullptr;
-  T* dr = dz + (size_t)row * ldz;
-  const int y = labels[row];
-  if (!(y >= 0 && y < V)) {   // rows outside Omega: no loss, zero gradient
-    float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    for (int c = threadIdx.x * 8; c < ldz; c += blockDim.x * 8) Vec8<T>::store(dr + c, f);
-    if (threadIdx.x == 0) row_loss[row] = 0.f;
-    return;
-  }
-  const int nch = (ldz + kLossChunk - 1) / kLossChunk;
-  const int total = 2 * nch;   // pass 1 then pass 2 over the same chunks
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kLossStages; ++s)
-      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full[s])) : "memory");
-    abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  __syncthreads();
-  auto issue = [&](int i) {   // chunk i % nch of the row into stage i % kLossStages
-    const int ch = i % nch, st = i % kLossStages;
-    const int c0 = ch * kLossChunk, len = min(kLossChunk, ldz - c0);
-    const uint32_t bytes = (uint32_t)(len * sizeof(T));
-    const uint32_t bar = smem_u32(&full[st]);
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(tr ? 2 * bytes : bytes)
-                 : "memory");
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     smem_u32(zbuf + st * kLossChunk)),
-                 "l"(zr + c0), "r"(bytes), "r"(bar)
-                 : "memory");
-    if (tr)
-      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                       smem_u32(tbuf + st * kLossChunk)),
-                   "l"(tr + c0), "r"(bytes), "r"(bar)
-                   : "memory");
-  };
-  if (threadIdx.x == 0)
-    for (int i = 0; i < kLossStages && i < total; ++i) issue(i);
-  Lse3 Z{-INFINITY, 0.f, 0.f}, Q{-INFINITY, 0.f, 0.f};
-  float lz2 = 0.f, lt2 = 0.f, dl = 0.f, kl = 0.f, wt = 0.f, wc = 0.f;
-  bool ok = true;
-  for (int i = 0; i < total; ++i) {
-    const int st = i % kLossStages;
-    const uint32_t parity = (uint32_t)(i / kLossStages) & 1u;
-    // bounded wait for the stage
-    {
-      uint32_t done = 0;
-      const unsigned long long t0 = gtime();
-      while (true) {
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.b32 %0, 1, 0, p;\n}"
-            : "=r"(done)
-            : "r"(smem_u32(&full[st])), "r"(parity)
-            : "memory");
-        if (done) break;
-        if (abort_flag || gtime() - t0 > kLossTimeoutNs) {
-          abort_flag = 1;
-          ok = false;
-          break;
-        }
-      }
-    }
-    if (!ok) break;
-    const int ch = i % nch;
-    const int c = ch * kLossChunk + threadIdx.x * 8;
-    const int nv = min(8, V - c);
-    if (i < nch) {
-      // pass 1
-      if (threadIdx.x * 8 < kLossChunk && nv > 0) {
-        float fz[8], ft[8], w[8];
-        Vec8<T>::load(zbuf + st * kLossChunk + threadIdx.x * 8, fz);
-        if (tr) {
-          Vec8<T>::load(tbuf + st * kLossChunk + threadIdx.x * 8, ft);
-#pragma unroll
-          for (int k = 0; k < 8; ++k) w[k] = kl_dir == 0 ? fz[k] - ft[k] : ft[k] - fz[k];
-          lse_add8(Z, fz, kl_dir == 0 ? w : nullptr, nv);
-          lse_add8(Q, ft, kl_dir == 0 ? nullptr : w, nv);
-        } else {
-          lse_add8(Z, fz, nullptr, nv);
-        }
-      }
-      if (i == nch - 1) {   // row statistics
-        Z = warp_merge(Z);
-        if (tr) Q = warp_merge(Q);
-        const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-        if (lane == 0) { shz[wid] = Z; sht[wid] = Q; }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-          Lse3 a = shz[0], b = sht[0];
-          for (int k = 1; k < nw; ++k) { a = lse_merge(a, shz[k]); if (tr) b = lse_merge(b, sht[k]); }
-          const float lse_z = (a.m + log2f(a.s)) * kLn2;
-          float lse_t = 0.f, kld = 0.f;
-          if (tr) {
-            lse_t = (b.m + log2f(b.s)) * kLn2;
-            kld = kl_dir == 0 ? a.a / a.s - lse_z + lse_t : b.a / b.s - lse_t + lse_z;
-          }
-          row_loss[row] = alpha * (lse_z - to_f(zr[y])) + (tr ? (1.f - alpha) * kld : 0.f);
-          sh_stats[0] = lse_z;
-          sh_stats[1] = lse_t;
-          sh_stats[2] = kld;
-        }
-        __syncthreads();
-        const float lse_z = sh_stats[0], lse_t = sh_stats[1];
-        kl = sh_stats[2];
-        lz2 = lse_z * kL2e;
-        lt2 = lse_t * kL2e;
-        dl = lse_z - lse_t;
-        const int cnt = *count;
-        const float inv_n = cnt > 0 ? 1.f / (float)cnt : 0.f;
-        wt = inv_n * alpha;
-        wc = inv_n * (1.f - alpha);
-      }
-    } else if (threadIdx.x * 8 < kLossChunk && c < ldz) {
-      // pass 2: dz for this chunk
-      float fz[8], ft[8], o[8];
-      Vec8<T>::load(zbuf + st * kLossChunk + threadIdx.x * 8, fz);
-      if (tr) Vec8<T>::load(tbuf + st * kLossChunk + threadIdx.x * 8, ft);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const int j = c + k;
-        if (j >= V) { o[k] = 0.f; continue; }
-        const float p = ex2(fmaf(fz[k], kL2e, -lz2));
-        float gsum = wt * (p - (j == y ? 1.f : 0.f));
-        if (tr) {
-          const float gc = kl_dir == 0 ? p * ((fz[k] - ft[k]) - dl - kl) : p - ex2(fmaf(ft[k], kL2e, -lt2));
-          gsum = fmaf(wc, gc, gsum);
-        }
-        o[k] = gsum;
-      }
-      Vec8<T>::store(dr + c, o);
-    }
-    __syncthreads();   // the stage is free again
-    if (threadIdx.x == 0 && i + kLossStages < total) issue(i + kLossStages);
-  }
-  if (!ok) {
-    if (threadIdx.x == 0) {
-      if (err) atomicOr(err, ZL_DEVERR_TIMEOUT);
-      // let copies still in flight land before the CTA's shared memory is reused
-      const unsigned long long t0 = gtime();
-      while (gtime() - t0 < 100000000ull) {
-      }
-    }
-    __syncthreads();
-  }
-}
-
 void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labels, int N, int V, int ldz,
-                       float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s,
-                       unsigned* err) {
+                       float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s) {
   note_launch(1);
   if (N <= 0) return;
-  // enough threads for one 8-wide vector each up to 1024; at most two 1024-thread rows per SM, so a
-  // row read in pass 1 is still in L2 for pass 2
-  int cap = 512;   // two or more rows in flight per SM; the rows being read still fit in L2
+  // up to 512 threads per row (one 8-wide vector each): several rows in flight per SM, and the rows
+  // being read still fit in L2 for the second pass
+  int cap = 512;
   if (const char* e = std::getenv("ZL_LOSS_THREADS")) {   // tuning override
     const int v = std::atoi(e);
     if (v == 128 || v == 256 || v == 512 || v == 1024) cap = v;
   }
   int th = 32;
   while (th < cap && th * 8 < ldz) th *= 2;
-  if (dt == BF16 && ldz % 8 == 0 && !std::getenv("ZL_LOSS_SIMPLE")) {
-    const int smem = kLossStages * kLossChunk * 2 * (t ? 2 : 1);
-    static bool attr = false;
-    if (!attr) {
-      cudaFuncSetAttribute(local_loss_tma_k<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           kLossStages * kLossChunk * 2 * 2);
-      attr = true;
-    }
-    local_loss_tma_k<bf16><<<N, 512, smem, s>>>((const bf16*)z, (const bf16*)t, labels, V, ldz, alpha, kl_dir, count,
-                                                (bf16*)dz, row_loss, err);
-    return;
-  }
-  if (dt == BF16)
-    local_loss_k<bf16><<<N, th, 0, s>>>((const bf16*)z, (const bf16*)t, labels, V, ldz, alpha, kl_dir, count,
-                                        (bf16*)dz, row_loss);
-  else
-    local_loss_k<float><<<N, th, 0, s>>>((const float*)z, (const float*)t, labels, V, ldz, alpha, kl_dir, count,
-                                         (float*)dz, row_loss);
+#define LL(T, TE, KD)                                                                                        \
+  local_loss_k<T, TE, KD><<<N, th, 0, s>>>((const T*)z, (const T*)t, labels, V, ldz, alpha, count, (T*)dz, \
+                                           row_loss)
+#define LLT(T)                      \
+  if (!t) LL(T, false, 0);          \
+  else if (kl_dir == 0) LL(T, true, 0); \
+  else LL(T, true, 1);
+  if (dt == BF16) { LLT(bf16) } else { LLT(float) }
+#undef LLT
+#undef LL
 }
 
 __global__ void count_valid_k(const int32_t* __restrict__ labels, int N, int V, int* count, unsigned* err) {
