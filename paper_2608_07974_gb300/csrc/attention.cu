@@ -158,8 +158,8 @@ inline int warps_grid(long rows) { return (int)((rows * 32 + 255) / 256); }
 }  // namespace
 
 bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s);
-bool attn_bwd_tc(const void* qkv, const void* dout, const float* lse, const float* D, void* dqkv, int B, int S, int H,
-                 int Hkv, int hd, cudaStream_t s);
+bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
+                 int H, int Hkv, int hd, cudaStream_t s);
 
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s) {
   note_launch(1);
@@ -172,12 +172,12 @@ void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int 
 
 void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const float* lse, float* Dbuf, void* dqkv,
               int B, int S, int H, int Hkv, int hd, cudaStream_t s) {
-  note_launch(3);
+  note_launch(dt == BF16 ? 2 : 3);
   const float scale = 1.f / sqrtf((float)hd);
   const int gq = warps_grid((long)B * H * S), gk = warps_grid((long)B * Hkv * S);
+  if (dt == BF16 && attn_bwd_tc(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s)) return;
   if (dt == BF16) {
     attn_bwd_d_k<bf16><<<gq, 256, 0, s>>>((const bf16*)out, (const bf16*)dout, Dbuf, B, S, H, hd);
-    if (attn_bwd_tc(qkv, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s)) return;
     attn_bwd_dq_k<bf16><<<gq, 256, 0, s>>>((const bf16*)qkv, (const bf16*)dout, lse, Dbuf, (bf16*)dqkv, B, S, H, Hkv,
                                            hd, scale);
     attn_bwd_dkv_k<bf16><<<gk, 256, 0, s>>>((const bf16*)qkv, (const bf16*)dout, lse, Dbuf, (bf16*)dqkv, B, S, H,

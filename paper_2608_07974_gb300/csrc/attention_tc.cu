@@ -90,6 +90,13 @@ __device__ __forceinline__ void load_tile(bf16* t, const bf16* g, long ld, int n
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// 2^x on the SFU (ex2.approx, relative error about 2^-22; subnormal results flush to zero).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // ----------------------------------------------------------------------------------------------
 // forward
 // ----------------------------------------------------------------------------------------------
@@ -162,7 +169,7 @@ __global__ void __launch_bounds__(NT) fwd_k(const bf16* __restrict__ qkv, bf16* 
     float corr[2];
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
-      corr[i] = mx[i] == -INFINITY ? 1.f : exp2f(m[i] - mx[i]);
+      corr[i] = mx[i] == -INFINITY ? 1.f : ex2(m[i] - mx[i]);
       m[i] = mx[i];
       l[i] *= corr[i];
     }
@@ -171,7 +178,7 @@ __global__ void __launch_bounds__(NT) fwd_k(const bf16* __restrict__ qkv, bf16* 
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const float mm = m[e >> 1];
-        const float p = mm == -INFINITY ? 0.f : exp2f(s[nt][e] - mm);
+        const float p = mm == -INFINITY ? 0.f : ex2(s[nt][e] - mm);
         s[nt][e] = p;
         l[e >> 1] += p;
       }
@@ -219,9 +226,10 @@ __global__ void __launch_bounds__(NT) fwd_k(const bf16* __restrict__ qkv, bf16* 
 // backward: dQ (one CTA per query block of one head)
 // ----------------------------------------------------------------------------------------------
 template <int HDP>
-__global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, const bf16* __restrict__ dout,
-                                               const float* __restrict__ lse, const float* __restrict__ Dv,
-                                               bf16* __restrict__ dqkv, int S, int H, int Hkv, int hd, float scale) {
+__global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, const bf16* __restrict__ outp,
+                                               const bf16* __restrict__ dout, const float* __restrict__ lse,
+                                               float* __restrict__ Dv, bf16* __restrict__ dqkv, int S, int H,
+                                               int Hkv, int hd, float scale) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* Qs = reinterpret_cast<bf16*>(smem);
   bf16* dOs = Qs + BR * HDP;
@@ -240,11 +248,26 @@ __global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, con
   load_tile<HDP>(Ks, base + (H + kvh) * hd, ld, S, hd, vec);
   load_tile<HDP>(Vs, base + (H + Hkv + kvh) * hd, ld, S, hd, vec);
   cp_commit();
-  for (int i = threadIdx.x; i < BR; i += NT) {
+  // D_i = sum_d dO_i[d] O_i[d] for this block's rows (written for the dK/dV kernel that follows)
+  for (int i = threadIdx.x >> 1; i < BR; i += NT / 2) {
     const int r = q0 + i;
-    const size_t si = ((size_t)b * H + h) * S + r;
-    Ls[i] = r < S ? lse[si] * kLog2e : 0.f;
-    Ds[i] = r < S ? Dv[si] : 0.f;
+    float acc = 0.f;
+    if (r < S) {
+      const bf16* orow = outp + ((size_t)b * S + r) * HD + h * hd;
+      const bf16* drow = dout + ((size_t)b * S + r) * HD + h * hd;
+      for (int dd = (threadIdx.x & 1) * 2; dd < hd; dd += 4) {
+        const float2 o2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(orow + dd));
+        const float2 g2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(drow + dd));
+        acc = fmaf(o2.x, g2.x, fmaf(o2.y, g2.y, acc));
+      }
+    }
+    acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+    if ((threadIdx.x & 1) == 0) {
+      const size_t si = ((size_t)b * H + h) * S + r;
+      Ls[i] = r < S ? lse[si] * kLog2e : 0.f;
+      Ds[i] = r < S ? acc : 0.f;
+      if (r < S) Dv[si] = acc;
+    }
   }
   float dq[HDP / 8][4];
 #pragma unroll
@@ -292,7 +315,7 @@ __global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, con
         const int lr = lr0 + ((e >> 1) << 3);
         const int row = q0 + lr;
         const bool ok = col <= row && col < S && row < S;
-        const float p = ok ? exp2f(s[nt][e] * sl2 - Ls[lr]) : 0.f;
+        const float p = ok ? ex2(s[nt][e] * sl2 - Ls[lr]) : 0.f;
         s[nt][e] = p * (dp[nt][e] - Ds[lr]);   // dS
       }
 #pragma unroll
@@ -408,7 +431,7 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
         const int q = q0 + lq;
         const int key = k0 + lr0 + ((e >> 1) << 3);
         const bool ok = q >= key && q < S && key < S;
-        const float p = ok ? exp2f(st[nt][e] * sl2 - Lt[lq]) : 0.f;
+        const float p = ok ? ex2(st[nt][e] * sl2 - Lt[lq]) : 0.f;
         st[nt][e] = p;
         dpt[nt][e] = p * (dpt[nt][e] - Dt[lq]);
       }
@@ -458,8 +481,8 @@ void fwd_t(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv,
 }
 
 template <int HDP>
-void bwd_t(const void* qkv, const void* dout, const float* lse, const float* D, void* dqkv, int B, int S, int H,
-           int Hkv, int hd, cudaStream_t s) {
+void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
+           int H, int Hkv, int hd, cudaStream_t s) {
   const float scale = 1.f / sqrtf((float)hd);
   const int smem = 6 * BR * HDP * 2 + 4 * BR * 4;
   static bool attr = false;
@@ -469,7 +492,8 @@ void bwd_t(const void* qkv, const void* dout, const float* lse, const float* D, 
     attr = true;
   }
   dim3 gq((S + BR - 1) / BR, H, B), gk((S + BR - 1) / BR, Hkv, B);
-  bwd_dq_k<HDP><<<gq, NT, smem, s>>>((const bf16*)qkv, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, hd, scale);
+  bwd_dq_k<HDP><<<gq, NT, smem, s>>>((const bf16*)qkv, (const bf16*)out, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H,
+                                     Hkv, hd, scale);
   bwd_dkv_k<HDP><<<gk, NT, smem, s>>>((const bf16*)qkv, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, hd, scale);
 }
 
@@ -483,12 +507,12 @@ bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, in
   return true;
 }
 
-bool attn_bwd_tc(const void* qkv, const void* dout, const float* lse, const float* D, void* dqkv, int B, int S, int H,
-                 int Hkv, int hd, cudaStream_t s) {
+bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
+                 int H, int Hkv, int hd, cudaStream_t s) {
   if (hd > 128 || hd % 2) return false;
-  if (hd <= 32) fa::bwd_t<32>(qkv, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
-  else if (hd <= 64) fa::bwd_t<64>(qkv, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
-  else fa::bwd_t<128>(qkv, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
+  if (hd <= 32) fa::bwd_t<32>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
+  else if (hd <= 64) fa::bwd_t<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
+  else fa::bwd_t<128>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
   return true;
 }
 
