@@ -159,7 +159,7 @@ inline int warps_grid(long rows) { return (int)((rows * 32 + 255) / 256); }
 
 bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s);
 bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
-                 int H, int Hkv, int hd, cudaStream_t s);
+                 int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool);
 
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s) {
   note_launch(1);
@@ -171,11 +171,11 @@ void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int 
 }
 
 void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const float* lse, float* Dbuf, void* dqkv,
-              int B, int S, int H, int Hkv, int hd, cudaStream_t s) {
-  note_launch(dt == BF16 ? 2 : 3);
+              int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool) {
+  note_launch(dt == BF16 ? (H > Hkv ? 3 : 2) : 3);
   const float scale = 1.f / sqrtf((float)hd);
   const int gq = warps_grid((long)B * H * S), gk = warps_grid((long)B * Hkv * S);
-  if (dt == BF16 && attn_bwd_tc(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s)) return;
+  if (dt == BF16 && attn_bwd_tc(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s, pool)) return;
   if (dt == BF16) {
     attn_bwd_d_k<bf16><<<gq, 256, 0, s>>>((const bf16*)out, (const bf16*)dout, Dbuf, B, S, H, hd);
     attn_bwd_dq_k<bf16><<<gq, 256, 0, s>>>((const bf16*)qkv, (const bf16*)dout, lse, Dbuf, (bf16*)dqkv, B, S, H, Hkv,

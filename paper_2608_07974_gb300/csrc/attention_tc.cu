@@ -7,6 +7,8 @@
 // gradient is a fixed-order sum: no atomics, bit-reproducible under any schedule.
 #include <math.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "ops.h"
 
@@ -348,10 +350,14 @@ __global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, con
 // ----------------------------------------------------------------------------------------------
 // backward: dK, dV (one CTA per key block of one KV head; loops over its query heads)
 // ----------------------------------------------------------------------------------------------
+// part == NULL: one CTA per (key block, KV head) looping over the group's query heads, writing dK, dV.
+// part != NULL: one CTA per (key block, query head); fp32 partials part[2][H][B*S][hd] (dK unscaled,
+// dV), reduced over each group by reduce_dkv_k.
 template <int HDP>
 __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, const bf16* __restrict__ dout,
                                                 const float* __restrict__ lse, const float* __restrict__ Dv,
-                                                bf16* __restrict__ dqkv, int S, int H, int Hkv, int hd, float scale) {
+                                                bf16* __restrict__ dqkv, int S, int H, int Hkv, int hd, float scale,
+                                                float* __restrict__ part) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* Ks = reinterpret_cast<bf16*>(smem);
   bf16* Vs = Ks + BR * HDP;
@@ -359,9 +365,12 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
   bf16* dOs = Qs + 2 * BR * HDP;       // [2]
   float* Ls = reinterpret_cast<float*>(dOs + 2 * BR * HDP);   // [2][BR]
   float* Ds = Ls + 2 * BR;                                     // [2][BR]
-  const int kb = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
+  const int kb = blockIdx.x, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int rep = H / Hkv, ld = (H + 2 * Hkv) * hd, HD = H * hd;
+  const int ld = (H + 2 * Hkv) * hd, HD = H * hd;
+  const int kvh = part ? blockIdx.y / (H / Hkv) : blockIdx.y;
+  const int rep = part ? 1 : H / Hkv;                  // query heads this CTA loops over
+  const int h_first = part ? blockIdx.y : kvh * (H / Hkv);
   const bool vec = (hd & 7) == 0;
   const bf16* base = qkv + (size_t)b * S * ld;
   const int k0 = kb * BR;
@@ -371,7 +380,7 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
   load_tile<HDP>(Ks, base + (size_t)k0 * ld + (H + kvh) * hd, ld, S - k0, hd, vec);
   load_tile<HDP>(Vs, base + (size_t)k0 * ld + (H + Hkv + kvh) * hd, ld, S - k0, hd, vec);
   auto stage = [&](int it, int buf) {
-    const int h = kvh * rep + it / per_head, qb = kb + it % per_head, q0 = qb * BR;
+    const int h = h_first + it / per_head, qb = kb + it % per_head, q0 = qb * BR;
     load_tile<HDP>(Qs + buf * BR * HDP, base + (size_t)q0 * ld + h * hd, ld, S - q0, hd, vec);
     load_tile<HDP>(dOs + buf * BR * HDP, dout + ((size_t)b * S + q0) * HD + h * hd, HD, S - q0, hd, vec);
     for (int i = threadIdx.x; i < BR; i += NT) {
@@ -458,6 +467,20 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
   for (int i = 0; i < 2; ++i) {
     const int key = k0 + lr0 + 8 * i;
     if (key >= S) continue;
+    if (part) {
+      const size_t NS = (size_t)gridDim.z * S;
+      float* pk = part + ((size_t)h_first * NS + (size_t)b * S + key) * hd;
+      float* pv = pk + (size_t)H * NS * hd;
+#pragma unroll
+      for (int nt = 0; nt < HDP / 8; ++nt) {
+        const int col = nt * 8 + 2 * (lane & 3);
+        if (col < hd) {
+          *reinterpret_cast<float2*>(pk + col) = make_float2(dk[nt][2 * i], dk[nt][2 * i + 1]);
+          *reinterpret_cast<float2*>(pv + col) = make_float2(dv[nt][2 * i], dv[nt][2 * i + 1]);
+        }
+      }
+      continue;
+    }
     bf16* dkr = dqkv + ((size_t)b * S + key) * ld + (H + kvh) * hd;
     bf16* dvr = dqkv + ((size_t)b * S + key) * ld + (H + Hkv + kvh) * hd;
 #pragma unroll
@@ -480,9 +503,32 @@ void fwd_t(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv,
   fwd_k<HDP><<<grid, NT, smem, s>>>((const bf16*)qkv, (bf16*)out, lse, S, H, Hkv, hd, 1.f / sqrtf((float)hd));
 }
 
+// dK, dV of each KV head = fixed-order sums of its query heads' partials.
+__global__ void reduce_dkv_k(const float* __restrict__ part, bf16* __restrict__ dqkv, int NS, int H, int Hkv, int hd,
+                             float scale) {
+  const int rep = H / Hkv, ld = (H + 2 * Hkv) * hd;
+  const size_t total = (size_t)NS * Hkv * (hd / 2);
+  const size_t HNS = (size_t)H * NS * hd;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
+    const int dd = (int)(i % (hd / 2)) * 2;
+    const int kvh = (int)((i / (hd / 2)) % Hkv);
+    const size_t n = i / ((size_t)(hd / 2) * Hkv);
+    float k0 = 0.f, k1 = 0.f, v0 = 0.f, v1 = 0.f;
+    for (int hh = 0; hh < rep; ++hh) {
+      const size_t o = ((size_t)(kvh * rep + hh) * NS + n) * hd + dd;
+      const float2 a = *reinterpret_cast<const float2*>(part + o);
+      const float2 c = *reinterpret_cast<const float2*>(part + HNS + o);
+      k0 += a.x; k1 += a.y; v0 += c.x; v1 += c.y;
+    }
+    bf16* row = dqkv + n * ld;
+    *reinterpret_cast<uint32_t*>(row + (H + kvh) * hd + dd) = pack(k0 * scale, k1 * scale);
+    *reinterpret_cast<uint32_t*>(row + (H + Hkv + kvh) * hd + dd) = pack(v0, v1);
+  }
+}
+
 template <int HDP>
 void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
-           int H, int Hkv, int hd, cudaStream_t s) {
+           int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool) {
   const float scale = 1.f / sqrtf((float)hd);
   const int smem = 6 * BR * HDP * 2 + 4 * BR * 4;
   static bool attr = false;
@@ -491,10 +537,24 @@ void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse,
     cudaFuncSetAttribute(bwd_dkv_k<HDP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     attr = true;
   }
-  dim3 gq((S + BR - 1) / BR, H, B), gk((S + BR - 1) / BR, Hkv, B);
+  dim3 gq((S + BR - 1) / BR, H, B);
   bwd_dq_k<HDP><<<gq, NT, smem, s>>>((const bf16*)qkv, (const bf16*)out, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H,
                                      Hkv, hd, scale);
-  bwd_dkv_k<HDP><<<gk, NT, smem, s>>>((const bf16*)qkv, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, hd, scale);
+  float* part = nullptr;
+  if (H > Hkv) {   // grouped heads: one CTA per query head, then a fixed-order group reduction
+    const size_t bytes = 2ull * H * B * S * hd * sizeof(float);
+    cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&part, bytes, pool, s) : cudaMallocAsync((void**)&part, bytes, s);
+    if (e != cudaSuccess) { cudaGetLastError(); part = nullptr; }
+  }
+  dim3 gk((S + BR - 1) / BR, part ? H : Hkv, B);
+  bwd_dkv_k<HDP><<<gk, NT, smem, s>>>((const bf16*)qkv, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, hd, scale,
+                                      part);
+  if (part) {
+    const size_t total = (size_t)B * S * Hkv * (hd / 2);
+    const int blocks = (int)std::min<size_t>((total + 255) / 256, 152 * 16);
+    reduce_dkv_k<<<blocks, 256, 0, s>>>(part, (bf16*)dqkv, B * S, H, Hkv, hd, scale);
+    cudaFreeAsync(part, s);
+  }
 }
 
 }  // namespace fa
@@ -508,11 +568,11 @@ bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, in
 }
 
 bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
-                 int H, int Hkv, int hd, cudaStream_t s) {
+                 int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool) {
   if (hd > 128 || hd % 2) return false;
-  if (hd <= 32) fa::bwd_t<32>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
-  else if (hd <= 64) fa::bwd_t<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
-  else fa::bwd_t<128>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s);
+  if (hd <= 32) fa::bwd_t<32>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s, pool);
+  else if (hd <= 64) fa::bwd_t<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s, pool);
+  else fa::bwd_t<128>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, hd, s, pool);
   return true;
 }
 

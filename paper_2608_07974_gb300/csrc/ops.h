@@ -82,6 +82,6 @@ void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int 
               cudaStream_t s);
 // Gradients into dqkv (same layout as qkv). Dbuf: [B, H, S] scratch.
 void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const float* lse, float* Dbuf,
-              void* dqkv, int B, int S, int H, int Hkv, int hd, cudaStream_t s);
+              void* dqkv, int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool = nullptr);
 
 }  // namespace zl
