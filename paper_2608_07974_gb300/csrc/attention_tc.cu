@@ -32,6 +32,9 @@ __device__ __forceinline__ uint32_t s32(const void* p) { return (uint32_t)__cvta
 __device__ __forceinline__ void cp16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s32(dst)), "l"(src) : "memory");
 }
+__device__ __forceinline__ void cp8(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(s32(dst)), "l"(src) : "memory");
+}
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
@@ -74,18 +77,28 @@ __device__ __forceinline__ void frag_b_kn(uint32_t* b, const bf16* t, int k0, in
 }
 
 // rows [r0, r0 + 64) of a head slice (row stride ld elements) into a swizzled tile; rows >= nrows
-// and columns >= hd read as zero.
+// and columns >= hd read as zero. vec: 16-byte copies (hd % 8 == 0); otherwise 8-byte copies of
+// 4-element halves when hd % 4 == 0 (e.g. hd = 100, whose head slices are 8-byte aligned).
 template <int HDP>
 __device__ __forceinline__ void load_tile(bf16* t, const bf16* g, long ld, int nrows, int hd, bool vec) {
+  const bool vec8 = (hd & 3) == 0;
   for (int i = threadIdx.x; i < BR * Tile<HDP>::CH; i += NT) {
     const int r = i / Tile<HDP>::CH, c = i % Tile<HDP>::CH;
     bf16* dst = t + Tile<HDP>::off(r, c);
     const bf16* src = g + (size_t)r * ld + c * 8;
-    if (vec && r < nrows && c * 8 < hd) {
+    if (r >= nrows || c * 8 >= hd) {
+      *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+    } else if (vec) {
       cp16(dst, src);
+    } else if (vec8) {
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {
+        if (c * 8 + hf * 4 < hd) cp8(dst + hf * 4, src + hf * 4);
+        else *reinterpret_cast<uint2*>(dst + hf * 4) = make_uint2(0u, 0u);
+      }
     } else {
 #pragma unroll
-      for (int e = 0; e < 8; ++e) dst[e] = (r < nrows && c * 8 + e < hd) ? src[e] : __float2bfloat16_rn(0.f);
+      for (int e = 0; e < 8; ++e) dst[e] = c * 8 + e < hd ? src[e] : __float2bfloat16_rn(0.f);
     }
   }
 }
@@ -153,16 +166,27 @@ __global__ void __launch_bounds__(NT) fwd_k(const bf16* __restrict__ qkv, bf16* 
       }
     }
     float mx[2] = {m[0], m[1]};
+    if (kb < qb && (kb + 1) * BR <= S) {   // strictly below the diagonal and inside the sequence: no mask
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
+      for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int col = kb * BR + nt * 8 + 2 * (lane & 3) + (e & 1);
-        const int row = row0 + ((e >> 1) << 3);
-        const float v = (col <= row && col < S) ? s[nt][e] * sl2 : -INFINITY;
-        s[nt][e] = v;
-        mx[e >> 1] = fmaxf(mx[e >> 1], v);
-      }
+        for (int e = 0; e < 4; ++e) {
+          const float v = s[nt][e] * sl2;
+          s[nt][e] = v;
+          mx[e >> 1] = fmaxf(mx[e >> 1], v);
+        }
+    } else {
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int col = kb * BR + nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int row = row0 + ((e >> 1) << 3);
+          const float v = (col <= row && col < S) ? s[nt][e] * sl2 : -INFINITY;
+          s[nt][e] = v;
+          mx[e >> 1] = fmaxf(mx[e >> 1], v);
+        }
+    }
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
       mx[i] = fmaxf(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 1));
@@ -309,14 +333,18 @@ __global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, con
         mma(dp[2 * np + 1], ad, bvv[2], bvv[3]);
       }
     }
+    const bool inner = kb < qb && (qb + 1) * BR <= S;   // no causal or length mask in this block
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const int col = kb * BR + nt * 8 + 2 * (lane & 3) + (e & 1);
         const int lr = lr0 + ((e >> 1) << 3);
-        const int row = q0 + lr;
-        const bool ok = col <= row && col < S && row < S;
+        bool ok = true;
+        if (!inner) {
+          const int col = kb * BR + nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int row = q0 + lr;
+          ok = col <= row && col < S && row < S;
+        }
         const float p = ok ? ex2(s[nt][e] * sl2 - Ls[lr]) : 0.f;
         s[nt][e] = p * (dp[nt][e] - Ds[lr]);   // dS
       }
@@ -432,14 +460,18 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
       }
     }
     // P^T and dS^T for this warp's 16 keys x 64 queries
+    const bool inner = q0 > k0 && q0 + BR <= S;   // every query after every key, all in range
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int lq = nt * 8 + 2 * (lane & 3) + (e & 1);
-        const int q = q0 + lq;
-        const int key = k0 + lr0 + ((e >> 1) << 3);
-        const bool ok = q >= key && q < S && key < S;
+        bool ok = true;
+        if (!inner) {
+          const int q = q0 + lq;
+          const int key = k0 + lr0 + ((e >> 1) << 3);
+          ok = q >= key && q < S && key < S;
+        }
         const float p = ok ? ex2(st[nt][e] * sl2 - Lt[lq]) : 0.f;
         st[nt][e] = p;
         dpt[nt][e] = p * (dpt[nt][e] - Dt[lq]);
