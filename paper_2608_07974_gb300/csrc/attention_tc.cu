@@ -333,21 +333,27 @@ __global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, con
         mma(dp[2 * np + 1], ad, bvv[2], bvv[3]);
       }
     }
-    const bool inner = kb < qb && (qb + 1) * BR <= S;   // no causal or length mask in this block
+    const float L0 = Ls[lr0], L1 = Ls[lr0 + 8], D0 = Ds[lr0], D1 = Ds[lr0 + 8];
+    if (kb < qb && (qb + 1) * BR <= S) {   // no causal or length mask in this block
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
+      for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int lr = lr0 + ((e >> 1) << 3);
-        bool ok = true;
-        if (!inner) {
-          const int col = kb * BR + nt * 8 + 2 * (lane & 3) + (e & 1);
-          const int row = q0 + lr;
-          ok = col <= row && col < S && row < S;
+        for (int e = 0; e < 4; ++e) {
+          const float p = ex2(s[nt][e] * sl2 - (e < 2 ? L0 : L1));
+          s[nt][e] = p * (dp[nt][e] - (e < 2 ? D0 : D1));   // dS
         }
-        const float p = ok ? ex2(s[nt][e] * sl2 - Ls[lr]) : 0.f;
-        s[nt][e] = p * (dp[nt][e] - Ds[lr]);   // dS
-      }
+    } else {
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int col = kb * BR + nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int row = q0 + lr0 + ((e >> 1) << 3);
+          const bool ok = col <= row && col < S && row < S;
+          const float p = ok ? ex2(s[nt][e] * sl2 - (e < 2 ? L0 : L1)) : 0.f;
+          s[nt][e] = p * (dp[nt][e] - (e < 2 ? D0 : D1));
+        }
+    }
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
       uint32_t pa[4] = {pack(s[2 * kk][0], s[2 * kk][1]), pack(s[2 * kk][2], s[2 * kk][3]),
@@ -460,22 +466,33 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
       }
     }
     // P^T and dS^T for this warp's 16 keys x 64 queries
-    const bool inner = q0 > k0 && q0 + BR <= S;   // every query after every key, all in range
+    if (q0 > k0 && q0 + BR <= S) {   // every query after every key, all in range: no mask
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
+      for (int nt = 0; nt < 8; ++nt) {
+        const int lq = nt * 8 + 2 * (lane & 3);
+        const float2 L2 = *reinterpret_cast<const float2*>(Lt + lq);
+        const float2 D2 = *reinterpret_cast<const float2*>(Dt + lq);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int lq = nt * 8 + 2 * (lane & 3) + (e & 1);
-        bool ok = true;
-        if (!inner) {
+        for (int e = 0; e < 4; ++e) {
+          const float p = ex2(st[nt][e] * sl2 - ((e & 1) ? L2.y : L2.x));
+          st[nt][e] = p;
+          dpt[nt][e] = p * (dpt[nt][e] - ((e & 1) ? D2.y : D2.x));
+        }
+      }
+    } else {
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int lq = nt * 8 + 2 * (lane & 3) + (e & 1);
           const int q = q0 + lq;
           const int key = k0 + lr0 + ((e >> 1) << 3);
-          ok = q >= key && q < S && key < S;
+          const bool ok = q >= key && q < S && key < S;
+          const float p = ok ? ex2(st[nt][e] * sl2 - Lt[lq]) : 0.f;
+          st[nt][e] = p;
+          dpt[nt][e] = p * (dpt[nt][e] - Dt[lq]);
         }
-        const float p = ok ? ex2(st[nt][e] * sl2 - Lt[lq]) : 0.f;
-        st[nt][e] = p;
-        dpt[nt][e] = p * (dpt[nt][e] - Dt[lq]);
-      }
+    }
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
       uint32_t pa[4] = {pack(st[2 * kk][0], st[2 * kk][1]), pack(st[2 * kk][2], st[2 * kk][3]),
