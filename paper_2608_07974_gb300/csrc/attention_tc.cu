@@ -444,70 +444,85 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
     const bf16* dOt = dOs + cur * BR * HDP;
     const float* Lt = Ls + cur * BR;
     const float* Dt = Ds + cur * BR;
-    float st[8][4], dpt[8][4];
+    // phase 1: S^T = K Q^T, then P^T, kept only as the packed bf16 A fragments of the dV product
+    uint32_t pa[4][4];
+    const bool inner = q0 > k0 && q0 + BR <= S;   // every query after every key, all in range: no mask
+    {
+      float st[8][4];
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+      for (int i = 0; i < 8; ++i) st[i][0] = st[i][1] = st[i][2] = st[i][3] = 0.f;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) st[i][e] = dpt[i][e] = 0.f;
+      for (int ks = 0; ks < HDP / 16; ++ks) {
+        uint32_t ak[4];
+        frag_a<HDP>(ak, Ks, warp * 16, ks * 16, lane);
 #pragma unroll
-    for (int ks = 0; ks < HDP / 16; ++ks) {
-      uint32_t ak[4], av[4];
-      frag_a<HDP>(ak, Ks, warp * 16, ks * 16, lane);
-      frag_a<HDP>(av, Vs, warp * 16, ks * 16, lane);
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        uint32_t bq[4], bd[4];
-        frag_b_nk<HDP>(bq, Qt, np * 16, ks * 16, lane);
-        frag_b_nk<HDP>(bd, dOt, np * 16, ks * 16, lane);
-        mma(st[2 * np], ak, bq[0], bq[1]);
-        mma(st[2 * np + 1], ak, bq[2], bq[3]);
-        mma(dpt[2 * np], av, bd[0], bd[1]);
-        mma(dpt[2 * np + 1], av, bd[2], bd[3]);
+        for (int np = 0; np < 4; ++np) {
+          uint32_t bq[4];
+          frag_b_nk<HDP>(bq, Qt, np * 16, ks * 16, lane);
+          mma(st[2 * np], ak, bq[0], bq[1]);
+          mma(st[2 * np + 1], ak, bq[2], bq[3]);
+        }
       }
-    }
-    // P^T and dS^T for this warp's 16 keys x 64 queries
-    if (q0 > k0 && q0 + BR <= S) {   // every query after every key, all in range: no mask
 #pragma unroll
       for (int nt = 0; nt < 8; ++nt) {
         const int lq = nt * 8 + 2 * (lane & 3);
         const float2 L2 = *reinterpret_cast<const float2*>(Lt + lq);
-        const float2 D2 = *reinterpret_cast<const float2*>(Dt + lq);
+        float p[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const float p = ex2(st[nt][e] * sl2 - ((e & 1) ? L2.y : L2.x));
-          st[nt][e] = p;
-          dpt[nt][e] = p * (dpt[nt][e] - ((e & 1) ? D2.y : D2.x));
+          bool ok = true;
+          if (!inner) {
+            const int q = q0 + lq + (e & 1);
+            const int key = k0 + lr0 + ((e >> 1) << 3);
+            ok = q >= key && q < S && key < S;
+          }
+          p[e] = ok ? ex2(st[nt][e] * sl2 - ((e & 1) ? L2.y : L2.x)) : 0.f;
+        }
+        pa[nt >> 1][(nt & 1) * 2] = pack(p[0], p[1]);
+        pa[nt >> 1][(nt & 1) * 2 + 1] = pack(p[2], p[3]);
+      }
+    }
+    // phase 2: dP^T = V dO^T, dS^T = P^T (dP^T - D) with P^T from the bf16 fragments
+    uint32_t da[4][4];
+    {
+      float dpt[8][4];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) dpt[i][0] = dpt[i][1] = dpt[i][2] = dpt[i][3] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < HDP / 16; ++ks) {
+        uint32_t av[4];
+        frag_a<HDP>(av, Vs, warp * 16, ks * 16, lane);
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {
+          uint32_t bd[4];
+          frag_b_nk<HDP>(bd, dOt, np * 16, ks * 16, lane);
+          mma(dpt[2 * np], av, bd[0], bd[1]);
+          mma(dpt[2 * np + 1], av, bd[2], bd[3]);
         }
       }
-    } else {
 #pragma unroll
-      for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int lq = nt * 8 + 2 * (lane & 3) + (e & 1);
-          const int q = q0 + lq;
-          const int key = k0 + lr0 + ((e >> 1) << 3);
-          const bool ok = q >= key && q < S && key < S;
-          const float p = ok ? ex2(st[nt][e] * sl2 - Lt[lq]) : 0.f;
-          st[nt][e] = p;
-          dpt[nt][e] = p * (dpt[nt][e] - Dt[lq]);
-        }
+      for (int nt = 0; nt < 8; ++nt) {
+        const int lq = nt * 8 + 2 * (lane & 3);
+        const float2 D2 = *reinterpret_cast<const float2*>(Dt + lq);
+        const uint32_t u01 = pa[nt >> 1][(nt & 1) * 2], u23 = pa[nt >> 1][(nt & 1) * 2 + 1];
+        const float2 p01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u01));
+        const float2 p23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u23));
+        da[nt >> 1][(nt & 1) * 2] = pack(p01.x * (dpt[nt][0] - D2.x), p01.y * (dpt[nt][1] - D2.y));
+        da[nt >> 1][(nt & 1) * 2 + 1] = pack(p23.x * (dpt[nt][2] - D2.x), p23.y * (dpt[nt][3] - D2.y));
+      }
     }
+    // dV += P^T dO, dK += dS^T Q
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
-      uint32_t pa[4] = {pack(st[2 * kk][0], st[2 * kk][1]), pack(st[2 * kk][2], st[2 * kk][3]),
-                        pack(st[2 * kk + 1][0], st[2 * kk + 1][1]), pack(st[2 * kk + 1][2], st[2 * kk + 1][3])};
-      uint32_t da[4] = {pack(dpt[2 * kk][0], dpt[2 * kk][1]), pack(dpt[2 * kk][2], dpt[2 * kk][3]),
-                        pack(dpt[2 * kk + 1][0], dpt[2 * kk + 1][1]), pack(dpt[2 * kk + 1][2], dpt[2 * kk + 1][3])};
 #pragma unroll
       for (int np = 0; np < HDP / 16; ++np) {
         uint32_t bdo[4], bq[4];
         frag_b_kn<HDP>(bdo, dOt, kk * 16, np * 16, lane);
         frag_b_kn<HDP>(bq, Qt, kk * 16, np * 16, lane);
-        mma(dv[2 * np], pa, bdo[0], bdo[1]);
-        mma(dv[2 * np + 1], pa, bdo[2], bdo[3]);
-        mma(dk[2 * np], da, bq[0], bq[1]);
-        mma(dk[2 * np + 1], da, bq[2], bq[3]);
+        mma(dv[2 * np], pa[kk], bdo[0], bdo[1]);
+        mma(dv[2 * np + 1], pa[kk], bdo[2], bdo[3]);
+        mma(dk[2 * np], da[kk], bq[0], bq[1]);
+        mma(dk[2 * np + 1], da[kk], bq[2], bq[3]);
       }
     }
     __syncthreads();
@@ -547,7 +562,11 @@ template <int HDP>
 void fwd_t(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s) {
   const int smem = 5 * BR * HDP * 2;
   static bool attr = false;
-  if (!attr) { cudaFuncSetAttribute(fwd_k<HDP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem); attr = true; }
+  if (!attr) {
+    cudaFuncSetAttribute(fwd_k<HDP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(fwd_k<HDP>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    attr = true;
+  }
   dim3 grid((S + BR - 1) / BR, H, B);
   fwd_k<HDP><<<grid, NT, smem, s>>>((const bf16*)qkv, (bf16*)out, lse, S, H, Hkv, hd, 1.f / sqrtf((float)hd));
 }
@@ -584,6 +603,8 @@ void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse,
   if (!attr) {
     cudaFuncSetAttribute(bwd_dq_k<HDP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(bwd_dkv_k<HDP>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(bwd_dq_k<HDP>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    cudaFuncSetAttribute(bwd_dkv_k<HDP>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     attr = true;
   }
   dim3 gq((S + BR - 1) / BR, H, B);
