@@ -53,6 +53,64 @@ def parse():
     return ap.parse_args()
 
 
+def max_over_ranks(ms: float, world: int, device: str = "cuda") -> float:
+    """The slowest rank's time (all_reduce MAX over the default process group)."""
+    if world <= 1:
+        return ms
+    import torch.distributed as dist
+    x = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(x, op=dist.ReduceOp.MAX)
+    return float(x)
+
+
+def job_tokens_per_s(tokens_per_step: int, steps: int, world: int, max_ms: float) -> float:
+    """Whole-job throughput: every rank's tokens over the slowest rank's time."""
+    return tokens_per_step * steps * world / (max_ms / 1e3)
+
+
+def roofline_of(prof):
+    """Roofline entry of the kernel class with the largest time share in a zl_profile_read result."""
+    pk, pk_kind = peaks()
+    tot_ms = sum(v["ms"] for v in prof.values())
+    dom = max(prof, key=lambda k: prof[k]["ms"])
+    g = prof[dom]
+    tensor = g["flops"] > 0
+    if tensor:
+        achieved = g["flops"] / (g["ms"] / 1e3) / 1e12
+        peak_v, unit, kind = pk["bf16_tflops_sustained"], "TFLOP/s", f"{pk_kind} bf16 sustained"
+    else:
+        achieved = g["bytes"] / (g["ms"] / 1e3) / 1e9
+        peak_v, unit, kind = pk["hbm_gbs"], "GB/s", f"{pk_kind} HBM copy"
+    traffic = measured_traffic(dom)
+    return {"bound": "tensor" if tensor else "hbm", "kernel": dom, "achieved": achieved, "peak": peak_v,
+            "unit": unit, "frac": achieved / peak_v, "peak_kind": kind, "traffic": traffic,
+            "launches": g["launches"],
+            "work_per_launch": (g["flops"] if tensor else g["bytes"]) / max(g["launches"], 1),
+            "share_of_kernel_time": g["ms"] / tot_ms if tot_ms else None}
+
+
+# DRAM bytes per launch (read + write) from ncu captures, valid only for the kernel sources they were
+# taken on (sha256 prefix of the file); any change to that source makes the figure null.
+TRAFFIC = {}
+
+
+def measured_traffic(cls):
+    import hashlib
+    ent = TRAFFIC.get(cls)
+    if not ent:
+        return None
+    src = os.path.join(ROOT, "paper_2608_07974_gb300", "csrc", ent["source"])
+    with open(src, "rb") as f:
+        if hashlib.sha256(f.read()).hexdigest()[:16] != ent["sha256"]:
+            return None
+    return ent["bytes_per_launch"]
+
+
+def rank_batch_ids(rank: int, n: int):
+    """Micro-batch indices of one replica (distinct per rank)."""
+    return [1000 * rank + i for i in range(n)]
+
+
 def workload_desc(w, K):
     d = w.dims
     arch = "llama" if d.arch == synth.ARCH_LLAMA else "gpt2"
@@ -188,14 +246,14 @@ def run_ours(args):
     bounds = synth.chunk_bounds(w.dims.n_layers, K)
     params = synth.make_params(w.dims, w.seed)
 
-    def make_engine(max_live):
+    def make_engine(max_live, serialize=False):
         e = zb.ZeroLock(w.dims, K, bounds, dtype=w.dtype, alpha=w.alpha, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
-                        eps=w.eps, weight_decay=w.weight_decay, max_live_chunks=max_live)
+                        eps=w.eps, weight_decay=w.weight_decay, max_live_chunks=max_live, serialize=serialize)
         e.load(params)
         return e
 
     nb = 4   # distinct resident micro-batches, per rank
-    batches = [synth.make_batch(w, 1000 * rank + i) for i in range(nb)]
+    batches = [synth.make_batch(w, i) for i in rank_batch_ids(rank, nb)]
     dev_batches = [(a.cuda(), b.cuda()) for a, b in batches]
     tokens = w.batch * w.seq
     stream = torch.cuda.current_stream()
@@ -214,12 +272,7 @@ def run_ours(args):
             fn(i)
         t1.record(stream)
         barrier()
-        ms = t0.elapsed_time(t1)
-        if world > 1:
-            x = torch.tensor([ms], device="cuda")
-            dist.all_reduce(x, op=dist.ReduceOp.MAX)
-            ms = float(x)
-        return ms
+        return max_over_ranks(t0.elapsed_time(t1), world)
 
     # ---- ZeroLock: device-resident inputs -----------------------------------------------------
     eng = make_engine(args.max_live)
@@ -245,7 +298,7 @@ def run_ours(args):
     launches = zb.zl_kernel_launches() - n0
     clk = clocks.stop()
     zl_peak = eng.peak_bytes()[0]
-    value = tokens * args.steps * world / (ms / 1e3)
+    value = job_tokens_per_s(tokens, args.steps, world, ms)
 
     # ---- live per-kernel-class timing (CUDA events on the launching streams) ------------------
     zb.zl_profile(eng.ctx, True)
@@ -254,22 +307,7 @@ def run_ours(args):
         zl(i)
     prof = zb.zl_profile_read(eng.ctx)
     zb.zl_profile(eng.ctx, False)
-    pk, pk_kind = peaks()
-    tot_ms = sum(v["ms"] for v in prof.values())
-    dom = max(prof, key=lambda k: prof[k]["ms"])          # the kernel class with the largest time share
-    g = prof[dom]
-    tensor = g["flops"] > 0
-    if tensor:
-        achieved = g["flops"] / (g["ms"] / 1e3) / 1e12
-        peak_v, unit, kind = pk["bf16_tflops_sustained"], "TFLOP/s", f"{pk_kind} bf16 sustained"
-    else:
-        achieved = g["bytes"] / (g["ms"] / 1e3) / 1e9
-        peak_v, unit, kind = pk["hbm_gbs"], "GB/s", f"{pk_kind} HBM copy"
-    roof = {"bound": "tensor" if tensor else "hbm", "kernel": dom, "achieved": achieved, "peak": peak_v,
-            "unit": unit, "frac": achieved / peak_v, "peak_kind": kind, "traffic": None,
-            "launches": g["launches"],
-            "work_per_launch": (g["flops"] if tensor else g["bytes"]) / max(g["launches"], 1),
-            "share_of_kernel_time": g["ms"] / tot_ms if tot_ms else None}
+    roof = roofline_of(prof)
     classes = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / prof_steps,
                    "TFLOP/s" if v["flops"] else "GB/s":
                        (v["flops"] / (v["ms"] / 1e3) / 1e12) if v["flops"] else (v["bytes"] / (v["ms"] / 1e3) / 1e9)
@@ -293,7 +331,7 @@ def run_ours(args):
         for i in range(2):
             e2e_step(i)
         ems = timed(e2e_step, args.steps)
-        e2e = {"value": tokens * args.steps * world / (ems / 1e3), "unit": "tokens/s",
+        e2e = {"value": job_tokens_per_s(tokens, args.steps, world, ems), "unit": "tokens/s",
                "h2d_bytes_per_step": 2 * tokens * 4, "d2h_bytes_per_step": K * 4}
     eng.close()
     del eng
@@ -313,9 +351,20 @@ def run_ours(args):
         beng.synchronize()
         beng.reset_peak()
         bms = timed(bps, args.steps)
-        bp = {"value": tokens * args.steps * world / (bms / 1e3), "unit": "tokens/s",
+        bp = {"value": job_tokens_per_s(tokens, args.steps, world, bms), "unit": "tokens/s",
               "peak_hbm_gb": beng.peak_bytes()[0] / 1e9, "ms_per_step": bms / args.steps}
         beng.close()
+
+    # ---- the same step with every chunk on one stream: per-launch times without the other chunks' kernels
+    seng = make_engine(args.max_live, serialize=True)
+    for i in range(2):
+        zb.zl_step(seng.ctx, dev_batches[i % nb][0], dev_batches[i % nb][1], w.batch, w.seq, K, want_losses=False)
+    zb.zl_profile(seng.ctx, True)
+    for i in range(prof_steps):
+        zb.zl_step(seng.ctx, dev_batches[i % nb][0], dev_batches[i % nb][1], w.batch, w.seq, K, want_losses=False)
+    sprof = zb.zl_profile_read(seng.ctx)
+    seng.close()
+    roof_serial = roofline_of(sprof)
 
     # ---- CPU oracle on a bounded sample (rank 0, one GPU only) --------------------------------
     cpu = None
@@ -336,7 +385,7 @@ def run_ours(args):
                 "peak_hbm_gb": zl_peak / 1e9, "bp": bp,
                 "zl_vs_bp": {"throughput": value / bp["value"], "peak_hbm": (zl_peak / 1e9) / bp["peak_hbm_gb"]}
                 if bp else None,
-                "roofline": roof, "kernel_classes": classes, "cpu_baseline": cpu, "e2e": e2e,
+                "roofline": roof, "roofline_serial": roof_serial, "kernel_classes": classes, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": launches, "clocks": clk}
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -74,6 +74,7 @@ typedef struct {
   int max_live_chunks;      /* chunks whose activations may be alive at once; 0 means K              */
   int lr_schedule;          /* 0: constant lr;  1: lr / sqrt(t + lr_gamma), t = 0,1,.. (Theorem 1)    */
   float lr_gamma;
+  int serialize;            /* 1: every chunk on one stream (no overlap; for measurement), 0: K streams */
 } zl_train_cfg;
 
 /* Create a context: parameters, AdamW state, K streams and events, a stream-ordered

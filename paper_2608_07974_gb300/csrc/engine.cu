@@ -628,16 +628,17 @@ bool lookup(zl_ctx* c, const std::string& name, Found& f) {
 void free_ctx(zl_ctx* c) {
   if (!c) return;
   cudaDeviceSynchronize();
+  const bool shared = c->cfg.serialize != 0;
   for (int k = 1; k < (int)c->ch.size(); ++k) {
     Chunk& ck = c->ch[k];
-    if (ck.s) cudaStreamDestroy(ck.s);
+    if (ck.s && (!shared || k == 1)) cudaStreamDestroy(ck.s);
     for (cudaEvent_t e : {ck.ev_h, ck.ev_z, ck.ev_loss, ck.ev_hb, ck.ev_done})
       if (e) cudaEventDestroy(e);
   }
   for (cudaEvent_t e : c->live_ring) cudaEventDestroy(e);
   for (cudaEvent_t e : {c->ev_start, c->ev_aux, c->ev_sync})
     if (e) cudaEventDestroy(e);
-  if (c->aux) cudaStreamDestroy(c->aux);
+  if (c->aux && !shared) cudaStreamDestroy(c->aux);
   for (void* p : c->statics) cudaFree(p);
   if (c->h_losses) cudaFreeHost(c->h_losses);
   if (c->pool) cudaMemPoolDestroy(c->pool);
@@ -699,6 +700,7 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (cfg->max_live_chunks < 0) why = "max_live_chunks must be >= 0";
   else if (cfg->lr_schedule != 0 && cfg->lr_schedule != 1) why = "lr_schedule";
   else if (cfg->lr_schedule == 1 && !(cfg->lr_gamma > 0.f)) why = "lr_gamma must be > 0";
+  else if (cfg->serialize != 0 && cfg->serialize != 1) why = "serialize must be 0 or 1";
   for (int k = 1; why.empty() && k <= K; ++k)
     if (bounds[k] <= bounds[k - 1]) why = "bounds must be strictly increasing";
   if (!why.empty()) { g_err = "zl_create: " + why; return ZL_ERR_ARG; }
@@ -802,11 +804,13 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       for (auto& L : ck.layers)
         for (PK p : {P_N1W, P_N2W}) CK(cudaMemcpy(ck.master + L.off[p], ones.data(), (size_t)d * 4, cudaMemcpyHostToDevice));
       if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
-      CK(cudaStreamCreateWithFlags(&ck.s, cudaStreamNonBlocking));
+      if (cfg->serialize && k > 1) ck.s = c->ch[1].s;   // one stream for every chunk
+      else CK(cudaStreamCreateWithFlags(&ck.s, cudaStreamNonBlocking));
       for (cudaEvent_t* e2 : {&ck.ev_h, &ck.ev_z, &ck.ev_loss, &ck.ev_hb, &ck.ev_done})
         CK(cudaEventCreateWithFlags(e2, cudaEventDisableTiming));
     }
-    CK(cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking));
+    if (cfg->serialize) c->aux = c->ch[1].s;
+    else CK(cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking));
     for (cudaEvent_t* e2 : {&c->ev_start, &c->ev_aux, &c->ev_sync}) CK(cudaEventCreateWithFlags(e2, cudaEventDisableTiming));
     const int cap = cfg->max_live_chunks > 0 ? std::min(cfg->max_live_chunks, K) : K;
     c->live_ring.resize(cap);
