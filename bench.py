@@ -91,7 +91,12 @@ def roofline_of(prof):
 
 # DRAM bytes per launch (read + write) from ncu captures, valid only for the kernel sources they were
 # taken on (sha256 prefix of the file); any change to that source makes the figure null.
-TRAFFIC = {}
+TRAFFIC = {
+    # ncu dram__bytes_read.sum + dram__bytes_write.sum of the GPT-2 GEMM shapes (microbench gemm),
+    # averaged with the per-step launch mix: 12 layer GEMMs per layer; 5 head forwards, 4 head dX
+    "gemm_layer": {"source": "gemm_tc.cu", "sha256": "a36ba939245bb7d1", "bytes_per_launch": 22315200.0},
+    "gemm_head": {"source": "gemm_tc.cu", "sha256": "a36ba939245bb7d1", "bytes_per_launch": 642291882.7},
+}
 
 
 def measured_traffic(cls):
