@@ -39,7 +39,7 @@ from typing import Dict, List, Optional, Sequence, Tuple
 
 import torch
 
-from synth import ARCH_GPT2, ARCH_LLAMA, ModelDims, layer_param_shapes
+from synth import ARCH_GPT2, ARCH_LLAMA, LORA_TARGETS, ModelDims, layer_param_shapes, lora_param_shapes
 
 Tensor = torch.Tensor
 
@@ -114,9 +114,18 @@ def embed(P: Dict[str, Tensor], ids: Tensor, d: ModelDims) -> Tensor:
     return h
 
 
-def layer_forward(P: Dict[str, Tensor], l: int, x: Tensor, d: ModelDims) -> Tensor:
-    """One transformer block (pre-norm residual) on x [B,S,d]."""
-    g = lambda s: P[f"layers.{l}.{s}"]
+def lora_weight(P: Dict[str, Tensor], l: int, name: str, scale: float) -> Tensor:
+    """w_l + Delta w_l with Delta w_l = scale * B_l A_l when the layer carries LoRA factors (Section II-A)."""
+    w = P[f"layers.{l}.{name}"]
+    a = P.get(f"layers.{l}.{name}.lora_a")
+    if a is None:
+        return w
+    return w + scale * (P[f"layers.{l}.{name}.lora_b"] @ a)
+
+
+def layer_forward(P: Dict[str, Tensor], l: int, x: Tensor, d: ModelDims, lora_scale: float = 1.0) -> Tensor:
+    """One transformer block (pre-norm residual) on x [B,S,d]; linear weights include LoRA updates."""
+    g = lambda s: lora_weight(P, l, s, lora_scale) if s in LORA_TARGETS else P[f"layers.{l}.{s}"]
     B, S, _ = x.shape
     H, Hkv, hd = d.n_heads, d.n_kv_heads, d.head_dim
     if d.arch == ARCH_LLAMA:
@@ -144,10 +153,10 @@ def layer_forward(P: Dict[str, Tensor], l: int, x: Tensor, d: ModelDims) -> Tens
 
 
 def chunk_forward(P: Dict[str, Tensor], bounds: Sequence[int], k: int, h: Tensor,
-                  d: ModelDims) -> Tensor:
-    """h_k = f_k(h_{k-1}) over layers bounds[k-1] .. bounds[k]-1 (chunks k = 1..K)."""
+                  d: ModelDims, lora_scale: float = 1.0) -> Tensor:
+    """h_k = f_k(h_{k-1}; W_k + Delta W_k) over layers bounds[k-1] .. bounds[k]-1 (Eq. 1)."""
     for l in range(bounds[k - 1], bounds[k]):
-        h = layer_forward(P, l, h, d)
+        h = layer_forward(P, l, h, d, lora_scale)
     return h
 
 
@@ -242,6 +251,8 @@ class OracleConfig:
     accum_m: int = 1
     lr_schedule: int = 0            # 0: constant; 1: lr / sqrt(t + lr_gamma) (Theorem 1)
     lr_gamma: float = 1.0
+    lora_rank: int = 0              # 0: every layer tensor trainable; r > 0: only the LoRA factors
+    lora_scale: float = 1.0         # Delta w = lora_scale * B A
 
     @property
     def K(self) -> int:
@@ -270,9 +281,12 @@ class Oracle:
 
     # -- parameter sets ------------------------------------------------------------------
     def chunk_names(self, k: int) -> List[str]:
+        """The trainable tensors of chunk k: all layer tensors, or only the LoRA factors A_l, B_l."""
+        shapes = (lora_param_shapes(self.d, self.cfg.lora_rank) if self.cfg.lora_rank > 0
+                  else layer_param_shapes(self.d))
         out = []
         for l in range(self.cfg.bounds[k - 1], self.cfg.bounds[k]):
-            out += [f"layers.{l}.{s}" for s, _ in layer_param_shapes(self.d)]
+            out += [f"layers.{l}.{s}" for s, _ in shapes]
         return out
 
     def trainable_names(self) -> List[str]:
@@ -290,7 +304,7 @@ class Oracle:
 
     def forward_chunk(self, k: int, h_prev: Tensor) -> Tensor:
         with torch.no_grad():
-            return chunk_forward(self.P, self.cfg.bounds, k, h_prev.to(self.dtype), self.d)
+            return chunk_forward(self.P, self.cfg.bounds, k, h_prev.to(self.dtype), self.d, self.cfg.lora_scale)
 
     def readout(self, h: Tensor) -> Tensor:
         with torch.no_grad():
@@ -307,7 +321,7 @@ class Oracle:
         h_in = h_prev.detach().to(self.dtype)                      # sg(h_{k-1})
         a = self.alpha_k(k)
         t = readout(self.P, h_in, self.d).detach() if a < 1.0 else None   # sg(p_{k-1})
-        h = chunk_forward(P, self.cfg.bounds, k, h_in, self.d)
+        h = chunk_forward(P, self.cfg.bounds, k, h_in, self.d, self.cfg.lora_scale)
         z = readout(P, h, self.d)
         L = local_objective(z, t, labels, a, self.cfg.kl_dir)
         grads = torch.autograd.grad(L, [leaves[n] for n in names])
@@ -357,7 +371,7 @@ class Oracle:
         P.update(leaves)
         h = embed(P, ids, self.d)
         for k in range(1, self.cfg.K + 1):
-            h = chunk_forward(P, self.cfg.bounds, k, h, self.d)
+            h = chunk_forward(P, self.cfg.bounds, k, h, self.d, self.cfg.lora_scale)
         z = readout(P, h, self.d)
         L = local_objective(z, None, labels, 1.0)
         grads = torch.autograd.grad(L, [leaves[n] for n in names])
@@ -378,5 +392,5 @@ class Oracle:
         with torch.no_grad():
             h = self.embed(ids)
             for k in range(1, self.cfg.K + 1):
-                h = chunk_forward(self.P, self.cfg.bounds, k, h, self.d)
+                h = chunk_forward(self.P, self.cfg.bounds, k, h, self.d, self.cfg.lora_scale)
             return float(local_objective(readout(self.P, h, self.d), None, labels, 1.0))

@@ -205,6 +205,36 @@ def layer_param_shapes(d: ModelDims) -> List[Tuple[str, Tuple[int, ...]]]:
             ("w2", (d.d_model, d.d_ff)), ("b2", (d.d_model,))]
 
 
+LORA_TARGETS = ("wqkv", "wo", "w1", "w2")
+
+
+def lora_param_shapes(d: ModelDims, rank: int) -> List[Tuple[str, Tuple[int, ...]]]:
+    """Per-layer LoRA tensors: for each linear W [out, in], lora_a [rank, in] and lora_b [out, rank]."""
+    out = []
+    for s, (o, i) in ((s, shp) for s, shp in layer_param_shapes(d) if s in LORA_TARGETS):
+        out += [(f"{s}.lora_a", (rank, i)), (f"{s}.lora_b", (o, rank))]
+    return out
+
+
+def make_lora_params(d: ModelDims, seed: int, rank: int, b_std: float = 0.0,
+                     layers: Optional[Iterable[int]] = None) -> Dict[str, torch.Tensor]:
+    """LoRA factors: A ~ N(0, 0.02^2); B = 0 (the usual start, so the model begins at its base
+    weights) unless b_std > 0 (tests use a non-zero B to exercise every gradient)."""
+    layers = range(d.n_layers) if layers is None else layers
+    out = {}
+    for l in layers:
+        for s, shp in lora_param_shapes(d, rank):
+            name = f"layers.{l}.{s}"
+            n = shp[0] * shp[1]
+            if s.endswith("lora_a"):
+                out[name] = normal(stream_key(seed, name), n, 0.02).to(torch.float32).view(shp)
+            elif b_std > 0:
+                out[name] = normal(stream_key(seed, name), n, b_std).to(torch.float32).view(shp)
+            else:
+                out[name] = torch.zeros(shp, dtype=torch.float32)
+    return out
+
+
 def frozen_param_shapes(d: ModelDims) -> List[Tuple[str, Tuple[int, ...]]]:
     """Frozen tensors: embedding (+ learned positions), final norm, LM head (GPT-2: tied to tok_emb)."""
     out = [("tok_emb", (d.vocab, d.d_model))]

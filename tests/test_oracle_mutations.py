@@ -89,3 +89,10 @@ def test_pins_catch_dropped_residual(monkeypatch):
     _patch(monkeypatch, "layer_forward", lambda P, l, x, d: orig(P, l, x, d) - x)
     with pytest.raises(AssertionError):
         pins.test_layer_matches_library_composition()
+
+
+def test_pins_catch_unscaled_lora(monkeypatch):
+    orig = om.lora_weight
+    monkeypatch.setattr(om, "lora_weight", lambda P, l, name, scale: orig(P, l, name, 1.0))
+    with pytest.raises(AssertionError):
+        pins.test_lora_zero_b_is_the_base_model_and_chain_rule()

@@ -399,3 +399,72 @@ def test_accumulation_window_is_the_mean():
     th, m, v = ref.P[n].clone(), torch.zeros_like(ref.P[n]), torch.zeros_like(ref.P[n])
     oracle.adamw_update(th, (ga[n] + gb[n]) / 2, m, v, 1, 1e-2, 0.9, 0.999, 1e-8, 0.01)
     assert torch.allclose(a.P[n], th, atol=1e-15, rtol=0)
+
+
+# ---------------------------------------------------------------------------------------
+# LoRA chunks (the paper's setting: frozen w_l, trainable A_l, B_l, Delta w_l = s B_l A_l)
+# ---------------------------------------------------------------------------------------
+
+def _lora_setup(d, rank=3, scale=2.0, b_std=0.3):
+    P = tiny_params(d)
+    P.update({n: t * 15.0 if n.endswith("lora_a") else t
+              for n, t in synth.make_lora_params(d, 11, rank, b_std=b_std).items()})
+    cfg = OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5, lora_rank=rank, lora_scale=scale)
+    return P, cfg
+
+
+@pytest.mark.parametrize("d", [LLAMA_T, GPT2_T], ids=["llama", "gpt2"])
+def test_lora_gradient_matches_finite_differences(d):
+    P, cfg = _lora_setup(d)
+    ids, labels = tiny_batch(d)
+    orc = Oracle(cfg, P)
+    h = orc.embed(ids)
+    gen = torch.Generator().manual_seed(5)
+    for k in (1, 2):
+        L, grads, h_next = orc.local_grad(k, h, labels)
+        assert set(grads) == set(orc.chunk_names(k)) and all("lora_" in n for n in grads)
+
+        def Lk(Pp):
+            t = oracle.readout(Pp, h, d)
+            hk = oracle.chunk_forward(Pp, cfg.bounds, k, h, d, cfg.lora_scale)
+            return float(oracle.local_objective(oracle.readout(Pp, hk, d), t, labels, 0.5))
+
+        for name, g in grads.items():
+            flat = orc.P[name].view(-1)
+            for idx in torch.randint(0, flat.numel(), (3,), generator=gen).tolist():
+                old = float(flat[idx])
+                flat[idx] = old + 1e-6
+                lp = Lk(orc.P)
+                flat[idx] = old - 1e-6
+                lm = Lk(orc.P)
+                flat[idx] = old
+                fd = (lp - lm) / 2e-6
+                assert abs(fd - float(g.view(-1)[idx])) <= 1e-7 + 1e-6 * abs(fd), (name, idx)
+        h = h_next
+
+
+def test_lora_zero_b_is_the_base_model_and_chain_rule():
+    """B = 0 gives the base model exactly; dL/dB = s G A^T and dL/dA = s B^T G, G = dL/dW_eff."""
+    d = LLAMA_T
+    P, cfg = _lora_setup(d, b_std=0.0)
+    ids, labels = tiny_batch(d)
+    base = Oracle(OracleConfig(dims=d, bounds=[0, 1, 2]), {n: t for n, t in P.items() if "lora_" not in n})
+    lora = Oracle(cfg, P)
+    h0 = base.embed(ids)
+    assert torch.equal(lora.forward_chunk(1, h0), base.forward_chunk(1, h0))
+    # chain rule with a non-zero B: full fine-tune gradients of the merged weights
+    P, cfg = _lora_setup(d)
+    lora = Oracle(cfg, P)
+    merged = {n: t for n, t in lora.P.items() if "lora_" not in n}
+    for l in range(d.n_layers):
+        for s in synth.LORA_TARGETS:
+            merged[f"layers.{l}.{s}"] = oracle.model.lora_weight(lora.P, l, s, cfg.lora_scale)
+    full = Oracle(OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5), merged)
+    h0 = full.embed(ids)
+    _, gl, _ = lora.local_grad(1, h0, labels)
+    _, gf, _ = full.local_grad(1, h0, labels)
+    for s in synth.LORA_TARGETS:
+        G = gf[f"layers.0.{s}"]
+        A, Bm = lora.P[f"layers.0.{s}.lora_a"], lora.P[f"layers.0.{s}.lora_b"]
+        assert torch.allclose(gl[f"layers.0.{s}.lora_b"], cfg.lora_scale * G @ A.T, atol=1e-12, rtol=1e-9)
+        assert torch.allclose(gl[f"layers.0.{s}.lora_a"], cfg.lora_scale * Bm.T @ G, atol=1e-12, rtol=1e-9)
