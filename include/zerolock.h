@@ -75,6 +75,8 @@ typedef struct {
   int lr_schedule;          /* 0: constant lr;  1: lr / sqrt(t + lr_gamma), t = 0,1,.. (Theorem 1)    */
   float lr_gamma;
   int serialize;            /* 1: every chunk on one stream (no overlap; for measurement), 0: K streams */
+  int lora_rank;            /* 0: full fine-tune; r > 0: LoRA (Section II-A) on the QKV, output and FFN  */
+  float lora_scale;         /*   linears, w + lora_scale * B A, only A [r, in] and B [out, r] trainable  */
 } zl_train_cfg;
 
 /* Create a context: parameters, AdamW state, K streams and events, a stream-ordered
@@ -96,7 +98,8 @@ zl_status zl_set_stream(zl_ctx* ctx, void* stream);
 /* Tensor names: tok_emb [V,d], pos_emb [max_seq,d] (GPT-2), norm_f.weight [d],
  * norm_f.bias [d] (GPT-2), lm_head [V,d] (Llama), and per layer l
  * layers.{l}.{attn_norm.weight, attn_norm.bias, wqkv, bqkv, wo, bo, ffn_norm.weight,
- * ffn_norm.bias, w1, b1, w2, b2} (biases: GPT-2 only); weights are [out, in] row-major.
+ * ffn_norm.bias, w1, b1, w2, b2} (biases: GPT-2 only); weights are [out, in] row-major. With
+ * lora_rank r > 0 also layers.{l}.{wqkv, wo, w1, w2}.{lora_a [r, in], lora_b [out, r]}.
  * zl_set_param copies `bytes` = numel * 4 of fp32 values from src (device memory if
  * on_device, else host) into the master copy (and the compute copy). */
 zl_status zl_set_param(zl_ctx* ctx, const char* name, const void* src, size_t bytes, int on_device);

@@ -71,10 +71,18 @@ enum PK { P_N1W, P_N1B, P_WQKV, P_BQKV, P_WO, P_BO, P_N2W, P_N2B, P_W1, P_B1, P_
 const char* kPName[P_COUNT] = {"attn_norm.weight", "attn_norm.bias", "wqkv", "bqkv", "wo", "bo",
                                "ffn_norm.weight", "ffn_norm.bias", "w1", "b1", "w2", "b2"};
 
+// Where a tensor lives: the trainable slab (fp32 master, grad, AdamW m/v, compute copy), the frozen
+// fp32 vector slab, or the frozen matrix slab (compute dtype only).
+enum Slab { S_TRAIN = 0, S_FVEC = 1, S_FMAT = 2 };
+constexpr int kLoraP[4] = {P_WQKV, P_WO, P_W1, P_W2};   // the linears that carry LoRA factors
+
 struct Layer {
   size_t off[P_COUNT];
   size_t numel[P_COUNT];
   bool has[P_COUNT];
+  int slab[P_COUNT];
+  size_t la[4], lb[4];        // LoRA A [r, in] and B [out, r] offsets in the trainable slab
+  int lin_in[4], lin_out[4];  // shapes of the four linears
 };
 
 struct Chunk {
@@ -82,6 +90,9 @@ struct Chunk {
   size_t n = 0;
   float *master = nullptr, *grad = nullptr, *m = nullptr, *v = nullptr;
   void* comp = nullptr;
+  float* fvec = nullptr;   // frozen vectors (norm gains, biases) in LoRA mode
+  void* fmat = nullptr;    // frozen base matrices in LoRA mode (compute dtype)
+  size_t fvec_n = 0, fmat_n = 0;
   std::vector<Layer> layers;
   int micro = 0;
   long t = 0;
@@ -94,6 +105,7 @@ struct LayerSave {
   const void* x = nullptr;   // layer input
   void *xn1, *qkv, *att, *x2, *xn2, *hid, *act, *y;
   float *rstd1, *mean1, *rstd2, *mean2, *lse;
+  void* u[4];                // LoRA: x A^T of each linear [N, r]
 };
 
 }  // namespace
@@ -166,11 +178,24 @@ struct Arena {
 };
 
 const void* Wc(zl_ctx* c, Chunk& k, int li, PK p) {   // compute-dtype pointer of a matrix
-  const size_t off = k.layers[li].off[p];
+  const Layer& L = k.layers[li];
+  const size_t off = L.off[p];
+  if (L.slab[p] == S_FMAT)
+    return c->dt == BF16 ? (const void*)((const bf16*)k.fmat + off) : (const void*)((const float*)k.fmat + off);
   return c->dt == BF16 ? (const void*)((const bf16*)k.comp + off) : (const void*)(k.master + off);
 }
-float* Wm(Chunk& k, int li, PK p) { return k.layers[li].has[p] ? k.master + k.layers[li].off[p] : nullptr; }
-float* Gm(Chunk& k, int li, PK p) { return k.layers[li].has[p] ? k.grad + k.layers[li].off[p] : nullptr; }
+float* Wm(Chunk& k, int li, PK p) {   // fp32 pointer of a vector (gain or bias)
+  const Layer& L = k.layers[li];
+  if (!L.has[p]) return nullptr;
+  return L.slab[p] == S_FVEC ? k.fvec + L.off[p] : k.master + L.off[p];
+}
+float* Gm(Chunk& k, int li, PK p) {   // gradient accumulator; NULL for frozen tensors
+  const Layer& L = k.layers[li];
+  return (L.has[p] && L.slab[p] == S_TRAIN) ? k.grad + L.off[p] : nullptr;
+}
+const void* LoraC(zl_ctx* c, Chunk& k, size_t off) {
+  return c->dt == BF16 ? (const void*)((const bf16*)k.comp + off) : (const void*)(k.master + off);
+}
 
 size_t esz(zl_ctx* c) { return dt_size(c->dt); }
 
@@ -217,12 +242,13 @@ struct ProfScope {
 // Profiled launch wrappers (algorithmic FLOPs / bytes per launch)
 // ----------------------------------------------------------------------------------------------
 void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, const void* B, void* C,
-       const float* bias, const void* R) {
+       const float* bias, const void* R, float alpha = 1.f) {
+  if (!C) return;   // frozen weight: no gradient to form
   const double e = (double)esz(c);
   const double out = mode == 2 ? 8.0 * M * N : (R ? 2.0 : 1.0) * e * M * N;
   const bool head = B == c->lm_head;
   ProfScope p(c, s, head ? PC_GEMM_HEAD : PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
-  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool);
+  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool, alpha);
 }
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
   const double e = (double)esz(c), N = (double)B * S;
@@ -262,6 +288,9 @@ size_t layer_save_bytes(zl_ctx* c, int N, int B, int S, bool with_y) {
   if (with_y) add((size_t)N * c->d * e);
   for (int i = 0; i < 4; ++i) add((size_t)N * 4);
   add((size_t)B * c->H * S * 4);    // lse
+  const int r = c->cfg.lora_rank;
+  if (r > 0)
+    for (int i = 0; i < 4; ++i) add((size_t)N * r * e);
   return b;
 }
 
@@ -280,6 +309,30 @@ void carve_layer(zl_ctx* c, Arena& a, LayerSave& sv, int N, int B, int S, bool w
   sv.rstd2 = (float*)a.take((size_t)N * 4);
   sv.mean2 = (float*)a.take((size_t)N * 4);
   sv.lse = (float*)a.take((size_t)B * c->H * S * 4);
+  const int r = c->cfg.lora_rank;
+  for (int i = 0; i < 4; ++i) sv.u[i] = r > 0 ? a.take((size_t)N * r * e) : nullptr;
+}
+
+// LoRA on linear i (Delta w = s B A): u = X A^T, out += s u B^T (Section II-A).
+void lora_fwd(zl_ctx* c, Chunk& k, int li, int i, const void* X, void* out, void* u, int N, cudaStream_t s) {
+  const int r = c->cfg.lora_rank;
+  if (r <= 0) return;
+  const Layer& L = k.layers[li];
+  G(c, s, 0, N, r, L.lin_in[i], X, LoraC(c, k, L.la[i]), u, nullptr, nullptr);
+  G(c, s, 0, N, L.lin_out[i], r, u, LoraC(c, k, L.lb[i]), out, nullptr, out, c->cfg.lora_scale);
+}
+
+// LoRA backward of linear i, after dX holds dY W: du = s dY B; dB += s dY^T u; dA += du^T X; dX += du A.
+void lora_bwd(zl_ctx* c, Chunk& k, int li, int i, const void* X, const void* u, const void* dY, void* dX, void* du,
+              int N, cudaStream_t s) {
+  const int r = c->cfg.lora_rank;
+  if (r <= 0) return;
+  const Layer& L = k.layers[li];
+  const float sc = c->cfg.lora_scale;
+  G(c, s, 1, N, r, L.lin_out[i], dY, LoraC(c, k, L.lb[i]), du, nullptr, nullptr, sc);
+  G(c, s, 2, L.lin_out[i], r, N, dY, u, k.grad + L.lb[i], nullptr, nullptr, sc);
+  G(c, s, 2, r, L.lin_in[i], N, du, X, k.grad + L.la[i], nullptr, nullptr);
+  G(c, s, 1, N, L.lin_in[i], r, du, LoraC(c, k, L.la[i]), dX, nullptr, dX);
 }
 
 void layer_fwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* x, void* y, int B, int S, cudaStream_t s) {
@@ -287,26 +340,30 @@ void layer_fwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* x, void* 
   sv.x = x;
   NF(c, s, x, Wm(k, li, P_N1W), Wm(k, li, P_N1B), sv.xn1, sv.rstd1, sv.mean1, N);
   G(c, s, 0, N, c->qkvw, c->d, sv.xn1, Wc(c, k, li, P_WQKV), sv.qkv, Wm(k, li, P_BQKV), nullptr);
+  lora_fwd(c, k, li, 0, sv.xn1, sv.qkv, sv.u[0], N, s);
   if (c->llama) {
     ProfScope p(c, s, PC_ELEM, 0, 2.0 * esz(c) * (double)N * (c->H + c->Hkv) * c->hd);
     launch_rope(dt, sv.qkv, c->rope_cs, N, S, c->H, c->Hkv, c->hd, 0, s);
   }
   AF(c, s, sv.qkv, sv.att, sv.lse, B, S);
   G(c, s, 0, N, c->d, c->ad, sv.att, Wc(c, k, li, P_WO), sv.x2, Wm(k, li, P_BO), x);
+  lora_fwd(c, k, li, 1, sv.att, sv.x2, sv.u[1], N, s);
   NF(c, s, sv.x2, Wm(k, li, P_N2W), Wm(k, li, P_N2B), sv.xn2, sv.rstd2, sv.mean2, N);
   G(c, s, 0, N, c->f1, c->d, sv.xn2, Wc(c, k, li, P_W1), sv.hid, Wm(k, li, P_B1), nullptr);
+  lora_fwd(c, k, li, 2, sv.xn2, sv.hid, sv.u[2], N, s);
   {
     ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * (c->f1 + c->f));
     if (c->llama) launch_swiglu_fwd(dt, sv.hid, sv.act, N, c->f, s);
     else launch_gelu_fwd(dt, sv.hid, sv.act, (size_t)N * c->f, s);
   }
   G(c, s, 0, N, c->d, c->f, sv.act, Wc(c, k, li, P_W2), y, Wm(k, li, P_B2), sv.x2);
+  lora_fwd(c, k, li, 3, sv.act, y, sv.u[3], N, s);
   CHECK_LAUNCH();
 }
 
 // Backward workspace of one chunk.
 struct BwdWs {
-  void *da, *dhid, *dxn, *dx2, *datt, *dqkv, *dy0, *dy1;
+  void *da, *dhid, *dxn, *dx2, *datt, *dqkv, *dy0, *dy1, *du;
   float *part_g, *part_b, *D;
   unsigned* counter;   // column-sum completion ticket (zero between launches)
 };
@@ -328,6 +385,7 @@ size_t bwd_ws_bytes(zl_ctx* c, int N, int B, int S) {
   add((size_t)colsum_blocks(N) * wmax * 4);
   add((size_t)B * c->H * S * 4);
   add(4);
+  add((size_t)N * std::max(c->cfg.lora_rank, 1) * e);
   return b;
 }
 
@@ -346,6 +404,7 @@ void carve_ws(zl_ctx* c, Arena& a, BwdWs& w, int N, int B, int S) {
   w.part_b = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
   w.D = (float*)a.take((size_t)B * c->H * S * 4);
   w.counter = (unsigned*)a.take(4);
+  w.du = a.take((size_t)N * std::max(c->cfg.lora_rank, 1) * e);
 }
 
 void bias_grad(zl_ctx* c, const void* dY, int N, int cols, float* g, BwdWs& w, cudaStream_t s) {
@@ -356,6 +415,7 @@ void bias_grad(zl_ctx* c, const void* dY, int N, int cols, float* g, BwdWs& w, c
 
 void norm_param_grad(zl_ctx* c, const void* x, const float* rstd, const float* mean, const void* dyn, int N,
                      float* gw, float* gb, BwdWs& w, cudaStream_t s) {
+  if (!gw) return;   // frozen norm
   const bool ln = !c->llama;
   ProfScope p(c, s, PC_NORM, 0, 2.0 * esz(c) * (double)N * c->d, 1);
   launch_norm_bwd_dparam(c->dt, ln, x, rstd, mean, dyn, w.part_g, w.part_b, N, c->d, gw, gb, w.counter, s);
@@ -369,6 +429,7 @@ void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void*
   G(c, s, 2, c->d, c->f, N, dy, sv.act, Gm(k, li, P_W2), nullptr, nullptr);
   bias_grad(c, dy, N, c->d, Gm(k, li, P_B2), w, s);
   G(c, s, 1, N, c->f, c->d, dy, Wc(c, k, li, P_W2), w.da, nullptr, nullptr);
+  lora_bwd(c, k, li, 3, sv.act, sv.u[3], dy, w.da, w.du, N, s);
   {
     ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * (2.0 * c->f1 + c->f));
     if (c->llama) launch_swiglu_bwd(dt, sv.hid, w.da, w.dhid, N, c->f, s);
@@ -377,12 +438,14 @@ void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void*
   G(c, s, 2, c->f1, c->d, N, w.dhid, sv.xn2, Gm(k, li, P_W1), nullptr, nullptr);
   bias_grad(c, w.dhid, N, c->f1, Gm(k, li, P_B1), w, s);
   G(c, s, 1, N, c->d, c->f1, w.dhid, Wc(c, k, li, P_W1), w.dxn, nullptr, nullptr);
+  lora_bwd(c, k, li, 2, sv.xn2, sv.u[2], w.dhid, w.dxn, w.du, N, s);
   NBX(c, s, sv.x2, Wm(k, li, P_N2W), sv.rstd2, sv.mean2, w.dxn, dy, w.dx2, N);
   norm_param_grad(c, sv.x2, sv.rstd2, sv.mean2, w.dxn, N, Gm(k, li, P_N2W), Gm(k, li, P_N2B), w, s);
   // attention
   G(c, s, 2, c->d, c->ad, N, w.dx2, sv.att, Gm(k, li, P_WO), nullptr, nullptr);
   bias_grad(c, w.dx2, N, c->d, Gm(k, li, P_BO), w, s);
   G(c, s, 1, N, c->ad, c->d, w.dx2, Wc(c, k, li, P_WO), w.datt, nullptr, nullptr);
+  lora_bwd(c, k, li, 1, sv.att, sv.u[1], w.dx2, w.datt, w.du, N, s);
   AB(c, s, sv.qkv, sv.att, w.datt, sv.lse, w.D, w.dqkv, B, S);
   if (c->llama) {
     ProfScope p(c, s, PC_ELEM, 0, 2.0 * esz(c) * (double)N * (c->H + c->Hkv) * c->hd);
@@ -391,6 +454,7 @@ void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void*
   G(c, s, 2, c->qkvw, c->d, N, w.dqkv, sv.xn1, Gm(k, li, P_WQKV), nullptr, nullptr);
   bias_grad(c, w.dqkv, N, c->qkvw, Gm(k, li, P_BQKV), w, s);
   G(c, s, 1, N, c->d, c->qkvw, w.dqkv, Wc(c, k, li, P_WQKV), w.dxn, nullptr, nullptr);
+  lora_bwd(c, k, li, 0, sv.xn1, sv.u[0], w.dqkv, w.dxn, w.du, N, s);
   norm_param_grad(c, sv.x, sv.rstd1, sv.mean1, w.dxn, N, Gm(k, li, P_N1W), Gm(k, li, P_N1B), w, s);
   if (dx) NBX(c, s, sv.x, Wm(k, li, P_N1W), sv.rstd1, sv.mean1, w.dxn, w.dx2, dx, N);
   CHECK_LAUNCH();
@@ -618,8 +682,17 @@ bool lookup(zl_ctx* c, const std::string& name, Found& f) {
     const Layer& L = ck.layers[l - ck.l0];
     for (int p = 0; p < P_COUNT; ++p)
       if (L.has[p] && suf == kPName[p]) {
-        f = Found{ck.master + L.off[p], true, L.numel[p], &ck, L.off[p], 0};
+        if (L.slab[p] == S_TRAIN) f = Found{ck.master + L.off[p], true, L.numel[p], &ck, L.off[p], 0};
+        else if (L.slab[p] == S_FVEC) f = Found{ck.fvec + L.off[p], true, L.numel[p], nullptr, 0, 0};
+        else f = Found{(char*)ck.fmat + L.off[p] * esz(c), c->dt == F32, L.numel[p], nullptr, 0, 0};
         return true;
+      }
+    if (c->cfg.lora_rank > 0)
+      for (int i = 0; i < 4; ++i) {
+        const std::string base = kPName[kLoraP[i]];
+        const size_t r = (size_t)c->cfg.lora_rank;
+        if (suf == base + ".lora_a") { f = Found{ck.master + L.la[i], true, r * L.lin_in[i], &ck, L.la[i], 0}; return true; }
+        if (suf == base + ".lora_b") { f = Found{ck.master + L.lb[i], true, r * L.lin_out[i], &ck, L.lb[i], 0}; return true; }
       }
   }
   return false;
@@ -701,6 +774,8 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (cfg->lr_schedule != 0 && cfg->lr_schedule != 1) why = "lr_schedule";
   else if (cfg->lr_schedule == 1 && !(cfg->lr_gamma > 0.f)) why = "lr_gamma must be > 0";
   else if (cfg->serialize != 0 && cfg->serialize != 1) why = "serialize must be 0 or 1";
+  else if (cfg->lora_rank < 0 || cfg->lora_rank > 256) why = "lora_rank must be in [0, 256]";
+  else if (cfg->lora_rank > 0 && !(std::isfinite(cfg->lora_scale))) why = "lora_scale must be finite";
   for (int k = 1; why.empty() && k <= K; ++k)
     if (bounds[k] <= bounds[k - 1]) why = "bounds must be strictly increasing";
   if (!why.empty()) { g_err = "zl_create: " + why; return ZL_ERR_ARG; }
@@ -772,21 +847,49 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       ck.k = k;
       ck.l0 = bounds[k - 1];
       ck.l1 = bounds[k];
-      size_t off = 0;
+      // Full fine-tune: every layer tensor in the trainable slab. LoRA: the base matrices and the
+      // vectors are frozen and only the factors A [r, in], B [out, r] of the four linears train.
+      const int r = cfg->lora_rank;
+      size_t off = 0, fvec = 0, fmat = 0;
       for (int l = ck.l0; l < ck.l1; ++l) {
         Layer L;
         size_t shp[P_COUNT] = {(size_t)d, (size_t)d, (size_t)c->qkvw * d, (size_t)c->qkvw, (size_t)d * c->ad, (size_t)d,
                                (size_t)d, (size_t)d, (size_t)c->f1 * d, (size_t)c->f, (size_t)d * c->f, (size_t)d};
         for (int p = 0; p < P_COUNT; ++p) {
           const bool bias = (p == P_N1B || p == P_BQKV || p == P_BO || p == P_N2B || p == P_B1 || p == P_B2);
+          const bool mat = (p == P_WQKV || p == P_WO || p == P_W1 || p == P_W2);
           L.has[p] = !(c->llama && bias);
           L.numel[p] = L.has[p] ? shp[p] : 0;
-          L.off[p] = off;
-          if (L.has[p]) off += round_up(shp[p], 64);
+          L.slab[p] = r == 0 ? S_TRAIN : (mat ? S_FMAT : S_FVEC);
+          size_t& cur = L.slab[p] == S_TRAIN ? off : (L.slab[p] == S_FMAT ? fmat : fvec);
+          L.off[p] = cur;
+          if (L.has[p]) cur += round_up(shp[p], 64);
+        }
+        const int ins[4] = {d, c->ad, d, c->f}, outs[4] = {c->qkvw, d, c->f1, d};
+        for (int i = 0; i < 4; ++i) {
+          L.lin_in[i] = ins[i];
+          L.lin_out[i] = outs[i];
+          L.la[i] = L.lb[i] = 0;
+          if (r > 0) {
+            L.la[i] = off;
+            off += round_up((size_t)r * ins[i], 64);
+            L.lb[i] = off;
+            off += round_up((size_t)outs[i] * r, 64);
+          }
         }
         ck.layers.push_back(L);
       }
       ck.n = std::max<size_t>(off, 64);
+      ck.fvec_n = fvec;
+      ck.fmat_n = fmat;
+      if (fvec) {
+        ck.fvec = (float*)salloc(c, fvec * 4);
+        CK(cudaMemset(ck.fvec, 0, fvec * 4));
+      }
+      if (fmat) {
+        ck.fmat = salloc(c, fmat * esz(c));
+        CK(cudaMemset(ck.fmat, 0, fmat * esz(c)));
+      }
       ck.master = (float*)salloc(c, ck.n * 4);
       ck.grad = (float*)salloc(c, ck.n * 4);
       ck.m = (float*)salloc(c, ck.n * 4);
@@ -802,7 +905,9 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       // norm gains start at one
       std::vector<float> ones(d, 1.f);
       for (auto& L : ck.layers)
-        for (PK p : {P_N1W, P_N2W}) CK(cudaMemcpy(ck.master + L.off[p], ones.data(), (size_t)d * 4, cudaMemcpyHostToDevice));
+        for (PK p : {P_N1W, P_N2W})
+          CK(cudaMemcpy((L.slab[p] == S_FVEC ? ck.fvec : ck.master) + L.off[p], ones.data(), (size_t)d * 4,
+                        cudaMemcpyHostToDevice));
       if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
       if (cfg->serialize && k > 1) ck.s = c->ch[1].s;   // one stream for every chunk
       else CK(cudaStreamCreateWithFlags(&ck.s, cudaStreamNonBlocking));

@@ -22,8 +22,8 @@ __device__ __forceinline__ float ldB(const T* B, int N, int K, int k, int n) {
 
 template <typename T, typename TC, int MODE>
 __global__ void __launch_bounds__(256) gemm_simt_k(int M, int N, int K, const T* __restrict__ A,
-                                                   const T* __restrict__ B, TC* __restrict__ C,
-                                                   const float* __restrict__ bias, const TC* __restrict__ R) {
+                                                   const T* __restrict__ B, TC* C,
+                                                   const float* __restrict__ bias, const TC* R, float alpha) {
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
@@ -60,7 +60,7 @@ __global__ void __launch_bounds__(256) gemm_simt_k(int M, int N, int K, const T*
       const int n = bn + tx + 16 * j;
       if (n >= N) continue;
       const size_t o = (size_t)m * N + n;
-      float v = acc[i][j];
+      float v = alpha * acc[i][j];
       if (MODE == 2) {
         reinterpret_cast<float*>(C)[o] += v;
       } else {
@@ -74,23 +74,25 @@ __global__ void __launch_bounds__(256) gemm_simt_k(int M, int N, int K, const T*
 
 template <typename T>
 void gemm_simt_t(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-                 const void* R, cudaStream_t s) {
+                 const void* R, cudaStream_t s, float alpha) {
   dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM), block(256);
   if (mode == 0)
-    gemm_simt_k<T, T, 0><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, bias, (const T*)R);
+    gemm_simt_k<T, T, 0><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, bias, (const T*)R, alpha);
   else if (mode == 1)
-    gemm_simt_k<T, T, 1><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, nullptr, (const T*)R);
+    gemm_simt_k<T, T, 1><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, nullptr, (const T*)R,
+                                                 alpha);
   else
-    gemm_simt_k<T, float, 2><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (float*)C, nullptr, nullptr);
+    gemm_simt_k<T, float, 2><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (float*)C, nullptr, nullptr,
+                                                    alpha);
 }
 }  // namespace
 
 void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-               const void* R, cudaStream_t s) {
+               const void* R, cudaStream_t s, float alpha) {
   note_launch(1);
   if (M <= 0 || N <= 0) return;
-  if (dt == BF16) gemm_simt_t<bf16>(mode, M, N, K, A, B, C, bias, R, s);
-  else gemm_simt_t<float>(mode, M, N, K, A, B, C, bias, R, s);
+  if (dt == BF16) gemm_simt_t<bf16>(mode, M, N, K, A, B, C, bias, R, s, alpha);
+  else gemm_simt_t<float>(mode, M, N, K, A, B, C, bias, R, s, alpha);
 }
 
 }  // namespace zl
@@ -98,8 +100,8 @@ void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void*
 namespace zl {
 // GEMM dispatch: the tensor-core kernel where it applies, else the CUDA-core kernel.
 void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-          const void* R, cudaStream_t s, unsigned* err, cudaMemPool_t pool) {
-  if (dt == BF16 && gemm_tc(mode, M, N, K, A, B, C, bias, R, err, s, pool)) return;
-  gemm_simt(dt, mode, M, N, K, A, B, C, bias, R, s);
+          const void* R, cudaStream_t s, unsigned* err, cudaMemPool_t pool, float alpha) {
+  if (dt == BF16 && gemm_tc(mode, M, N, K, A, B, C, bias, R, err, s, pool, alpha)) return;
+  gemm_simt(dt, mode, M, N, K, A, B, C, bias, R, s, alpha);
 }
 }  // namespace zl

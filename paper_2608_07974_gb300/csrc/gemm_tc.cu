@@ -39,6 +39,7 @@ struct Args {
   unsigned* err;
   int tiles_m, tiles_n;
   int splits, kb_per_split;   // split-K: unit u -> split u / tiles, k blocks [s*kps, min(nk, (s+1)*kps))
+  float alpha;                // scale of the product
 };
 
 __device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -267,6 +268,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int c = 0; c < BN; c += 32) {
         float v[32];
         tmem_ld32(trow + (uint32_t)c, v);
+        if (g.alpha != 1.f) {
+#pragma unroll
+          for (int q2 = 0; q2 < 32; ++q2) v[q2] *= g.alpha;
+        }
         const int n0 = tn * BN + c;
         if (m >= g.M || n0 >= g.N) continue;
         if (g.mode == 2) {
@@ -331,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // Sums the split-K partials in split order (deterministic) and applies the epilogue.
 __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, int mode, void* C,
-                                const float* __restrict__ bias, const bf16* __restrict__ R) {
+                                const float* __restrict__ bias, const bf16* R, float alpha) {
   const size_t n8 = (size_t)M * N / 8, MN = (size_t)M * N;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
     const size_t e = i * 8;
@@ -343,6 +348,8 @@ __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M,
 #pragma unroll
       for (int q = 0; q < 8; ++q) acc[q] += t[q];
     }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] *= alpha;
     if (mode == 2) {
       float c[8];
       Vec8<float>::load((float*)C + e, c);
@@ -464,7 +471,7 @@ bool gemm_tc_available() { return tc::init(); }
 
 // Returns false when the shape / alignment is outside what the tensor-core path handles.
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-             unsigned* err, cudaStream_t s, cudaMemPool_t pool) {
+             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha) {
   if (!tc::init()) return false;
   if (M < 16 || N < 16 || K < 16) return false;
   auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
@@ -483,7 +490,7 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
   }
   tc::Args a;
   a.M = M; a.N = N; a.K = K; a.mode = mode;
-  a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err;
+  a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err; a.alpha = alpha;
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
   a.tiles_n = (N + bn - 1) / bn;
   const int nk = (K + tc::BK - 1) / tc::BK;
@@ -503,6 +510,7 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
       a.C = ws;
       a.bias = nullptr;
       a.R = nullptr;
+      a.alpha = 1.f;   // applied by the reduction
     }
   }
   note_launch(1);
@@ -515,7 +523,7 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
       note_launch(1);
       const size_t n8 = (size_t)M * N / 8;
       const int blocks = (int)std::min<size_t>((n8 + 255) / 256, (size_t)tc::g_sms * 8);
-      tc::splitk_reduce_k<<<blocks, 256, 0, s>>>(ws, a.splits, M, N, mode, C, bias, (const bf16*)R);
+      tc::splitk_reduce_k<<<blocks, 256, 0, s>>>(ws, a.splits, M, N, mode, C, bias, (const bf16*)R, alpha);
     }
     cudaFreeAsync(ws, s);
   }

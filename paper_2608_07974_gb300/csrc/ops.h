@@ -67,15 +67,16 @@ void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
 // mode 2: C[M,N] (fp32) += A[K,M]^T B[K,N]. bf16 runs on the tcgen05 kernel where its shape and
 // alignment rules hold, everything else on the CUDA-core kernel. err: device word for timeouts;
 // pool: stream-ordered pool for split-K partials (NULL: the device's default pool).
+// alpha scales the product: C = alpha A op(B) (+ bias) (+ R), or C += alpha A^T B. R may alias C.
 void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-          const void* R, cudaStream_t s, unsigned* err = nullptr, cudaMemPool_t pool = nullptr);
+          const void* R, cudaStream_t s, unsigned* err = nullptr, cudaMemPool_t pool = nullptr, float alpha = 1.f);
 bool gemm_tc_available();
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-             unsigned* err, cudaStream_t s, cudaMemPool_t pool);
+             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha);
 // Tile width and split-K count the tensor-core GEMM picks for a shape (0, 0 if unavailable).
 void gemm_tc_plan(int M, int N, int K, int* bn, int* splits);
 void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-               const void* R, cudaStream_t s);
+               const void* R, cudaStream_t s, float alpha = 1.f);
 
 // Causal attention over qkv [N, (H + 2 Hkv) hd] (token-major, rows b*S + s): out [N, H hd], lse [B, H, S].
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,
