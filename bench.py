@@ -47,6 +47,7 @@ def parse():
     ap.add_argument("--workload", default="gpt2", choices=list(WORKLOADS))
     ap.add_argument("--K", type=int, default=0, help="chunk count (default: the workload's)")
     ap.add_argument("--max-live", type=int, default=2, help="chunks whose activations may be alive at once")
+    ap.add_argument("--lora", type=int, default=0, help="LoRA rank (0: full fine-tune); scale 16 / rank")
     ap.add_argument("--no-bp", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -116,12 +117,13 @@ def rank_batch_ids(rank: int, n: int):
     return [1000 * rank + i for i in range(n)]
 
 
-def workload_desc(w, K):
+def workload_desc(w, K, lora=0):
     d = w.dims
     arch = "llama" if d.arch == synth.ARCH_LLAMA else "gpt2"
+    tune = f"LoRA rank {lora} scale {16 / lora:g} on QKV/O/FFN" if lora else "full fine-tune"
     return (f"{w.name}: {arch}-style decoder, {d.n_layers} layers, d_model {d.d_model}, {d.n_heads} heads "
             f"({d.n_kv_heads} kv), ffn {d.d_ff}, vocab {d.vocab}, micro-batch {w.batch} x seq {w.seq}, "
-            f"K={K} chunks, alpha {w.alpha}, AdamW")
+            f"K={K} chunks, alpha {w.alpha}, AdamW, {tune}")
 
 
 def peaks():
@@ -250,10 +252,13 @@ def run_ours(args):
     K = args.K or w.K
     bounds = synth.chunk_bounds(w.dims.n_layers, K)
     params = synth.make_params(w.dims, w.seed)
+    if args.lora:
+        params.update(synth.make_lora_params(w.dims, w.seed, args.lora))
 
     def make_engine(max_live, serialize=False):
         e = zb.ZeroLock(w.dims, K, bounds, dtype=w.dtype, alpha=w.alpha, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
-                        eps=w.eps, weight_decay=w.weight_decay, max_live_chunks=max_live, serialize=serialize)
+                        eps=w.eps, weight_decay=w.weight_decay, max_live_chunks=max_live, serialize=serialize,
+                        lora_rank=args.lora, lora_scale=16.0 / args.lora if args.lora else 1.0)
         e.load(params)
         return e
 
@@ -373,7 +378,7 @@ def run_ours(args):
 
     # ---- CPU oracle on a bounded sample (rank 0, one GPU only) --------------------------------
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu:
+    if rank == 0 and world == 1 and not args.no_cpu and not args.lora:
         times, tok, cores = oracle_sample(w, K, params, 2)
         cpu = {"value": tok / times[-1], "unit": "tokens/s", "cores": cores, "kind": "oracle",
                "sample": f"one local step of chunk 2 on 1 x {w.seq} tokens (fp32 oracle, after one warm-up sample); "
@@ -383,7 +388,7 @@ def run_ours(args):
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-                "config": {"workload": workload_desc(w, K), "K": K, "bounds": bounds,
+                "config": {"workload": workload_desc(w, K, args.lora), "K": K, "bounds": bounds,
                            "global_batch": w.batch * world, "seq_len": w.seq, "max_live_chunks": args.max_live,
                            "parallelism": f"replicas x{world}" if world > 1 else "single GPU, K streams",
                            "l2": "no flush: every step's working set (weights, AdamW state, logits) exceeds L2"},
