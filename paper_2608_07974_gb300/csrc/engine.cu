@@ -81,7 +81,7 @@ struct Layer {
   size_t numel[P_COUNT];
   bool has[P_COUNT];
   int slab[P_COUNT];
-  size_t la[4], lb[4];        // LoRA A [r, in] and B [out, r] offsets in the trainable slab
+  size_t la[4], lb[4];        // LoRA A [r16, in] and B^T [r16, out] offsets in the trainable slab
   int lin_in[4], lin_out[4];  // shapes of the four linears
 };
 
@@ -193,6 +193,8 @@ float* Gm(Chunk& k, int li, PK p) {   // gradient accumulator; NULL for frozen t
   const Layer& L = k.layers[li];
   return (L.has[p] && L.slab[p] == S_TRAIN) ? k.grad + L.off[p] : nullptr;
 }
+int lora_r16(int r) { return r > 0 ? (r + 15) / 16 * 16 : 0; }
+
 const void* LoraC(zl_ctx* c, Chunk& k, size_t off) {
   return c->dt == BF16 ? (const void*)((const bf16*)k.comp + off) : (const void*)(k.master + off);
 }
@@ -288,7 +290,7 @@ size_t layer_save_bytes(zl_ctx* c, int N, int B, int S, bool with_y) {
   if (with_y) add((size_t)N * c->d * e);
   for (int i = 0; i < 4; ++i) add((size_t)N * 4);
   add((size_t)B * c->H * S * 4);    // lse
-  const int r = c->cfg.lora_rank;
+  const int r = lora_r16(c->cfg.lora_rank);
   if (r > 0)
     for (int i = 0; i < 4; ++i) add((size_t)N * r * e);
   return b;
@@ -309,28 +311,29 @@ void carve_layer(zl_ctx* c, Arena& a, LayerSave& sv, int N, int B, int S, bool w
   sv.rstd2 = (float*)a.take((size_t)N * 4);
   sv.mean2 = (float*)a.take((size_t)N * 4);
   sv.lse = (float*)a.take((size_t)B * c->H * S * 4);
-  const int r = c->cfg.lora_rank;
+  const int r = lora_r16(c->cfg.lora_rank);
   for (int i = 0; i < 4; ++i) sv.u[i] = r > 0 ? a.take((size_t)N * r * e) : nullptr;
 }
 
-// LoRA on linear i (Delta w = s B A): u = X A^T, out += s u B^T (Section II-A).
+// LoRA on linear i (Delta w = s B A, Section II-A): u = X A^T [N, r16], out += s u (B^T).
 void lora_fwd(zl_ctx* c, Chunk& k, int li, int i, const void* X, void* out, void* u, int N, cudaStream_t s) {
-  const int r = c->cfg.lora_rank;
+  const int r = lora_r16(c->cfg.lora_rank);
   if (r <= 0) return;
   const Layer& L = k.layers[li];
   G(c, s, 0, N, r, L.lin_in[i], X, LoraC(c, k, L.la[i]), u, nullptr, nullptr);
-  G(c, s, 0, N, L.lin_out[i], r, u, LoraC(c, k, L.lb[i]), out, nullptr, out, c->cfg.lora_scale);
+  G(c, s, 1, N, L.lin_out[i], r, u, LoraC(c, k, L.lb[i]), out, nullptr, out, c->cfg.lora_scale);
 }
 
-// LoRA backward of linear i, after dX holds dY W: du = s dY B; dB += s dY^T u; dA += du^T X; dX += du A.
+// LoRA backward of linear i, after dX holds dY W: du = s dY B; d(B^T) += s u^T dY; dA += du^T X;
+// dX += du A.
 void lora_bwd(zl_ctx* c, Chunk& k, int li, int i, const void* X, const void* u, const void* dY, void* dX, void* du,
               int N, cudaStream_t s) {
-  const int r = c->cfg.lora_rank;
+  const int r = lora_r16(c->cfg.lora_rank);
   if (r <= 0) return;
   const Layer& L = k.layers[li];
   const float sc = c->cfg.lora_scale;
-  G(c, s, 1, N, r, L.lin_out[i], dY, LoraC(c, k, L.lb[i]), du, nullptr, nullptr, sc);
-  G(c, s, 2, L.lin_out[i], r, N, dY, u, k.grad + L.lb[i], nullptr, nullptr, sc);
+  G(c, s, 0, N, r, L.lin_out[i], dY, LoraC(c, k, L.lb[i]), du, nullptr, nullptr, sc);
+  G(c, s, 2, r, L.lin_out[i], N, u, dY, k.grad + L.lb[i], nullptr, nullptr, sc);
   G(c, s, 2, r, L.lin_in[i], N, du, X, k.grad + L.la[i], nullptr, nullptr);
   G(c, s, 1, N, L.lin_in[i], r, du, LoraC(c, k, L.la[i]), dX, nullptr, dX);
 }
@@ -385,7 +388,7 @@ size_t bwd_ws_bytes(zl_ctx* c, int N, int B, int S) {
   add((size_t)colsum_blocks(N) * wmax * 4);
   add((size_t)B * c->H * S * 4);
   add(4);
-  add((size_t)N * std::max(c->cfg.lora_rank, 1) * e);
+  add((size_t)N * std::max(lora_r16(c->cfg.lora_rank), 1) * e);
   return b;
 }
 
@@ -404,7 +407,7 @@ void carve_ws(zl_ctx* c, Arena& a, BwdWs& w, int N, int B, int S) {
   w.part_b = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
   w.D = (float*)a.take((size_t)B * c->H * S * 4);
   w.counter = (unsigned*)a.take(4);
-  w.du = a.take((size_t)N * std::max(c->cfg.lora_rank, 1) * e);
+  w.du = a.take((size_t)N * std::max(lora_r16(c->cfg.lora_rank), 1) * e);
 }
 
 void bias_grad(zl_ctx* c, const void* dY, int N, int cols, float* g, BwdWs& w, cudaStream_t s) {
@@ -657,6 +660,7 @@ struct Found {
   Chunk* chunk = nullptr;       // trainable: owning chunk
   size_t off = 0;
   int frozen = 0;               // 1 tok_emb, 2 pos_emb, 3 norm_f.weight, 4 norm_f.bias, 5 lm_head
+  int trows = 0, tcols = 0;     // > 0: user layout [tcols, trows], stored transposed as [trows, tcols]
 };
 
 bool lookup(zl_ctx* c, const std::string& name, Found& f) {
@@ -692,7 +696,12 @@ bool lookup(zl_ctx* c, const std::string& name, Found& f) {
         const std::string base = kPName[kLoraP[i]];
         const size_t r = (size_t)c->cfg.lora_rank;
         if (suf == base + ".lora_a") { f = Found{ck.master + L.la[i], true, r * L.lin_in[i], &ck, L.la[i], 0}; return true; }
-        if (suf == base + ".lora_b") { f = Found{ck.master + L.lb[i], true, r * L.lin_out[i], &ck, L.lb[i], 0}; return true; }
+        if (suf == base + ".lora_b") {
+          f = Found{ck.master + L.lb[i], true, r * L.lin_out[i], &ck, L.lb[i], 0};
+          f.trows = (int)r;
+          f.tcols = L.lin_out[i];
+          return true;
+        }
       }
   }
   return false;
@@ -865,16 +874,20 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
           L.off[p] = cur;
           if (L.has[p]) cur += round_up(shp[p], 64);
         }
+        // LoRA factors are stored with the rank padded to a multiple of 16 (rows beyond r stay exactly
+        // zero: zero start, zero gradient), A as [r16, in] and B transposed as [r16, out], so every
+        // LoRA product is a tensor-core GEMM.
         const int ins[4] = {d, c->ad, d, c->f}, outs[4] = {c->qkvw, d, c->f1, d};
+        const size_t r16 = (size_t)lora_r16(r);
         for (int i = 0; i < 4; ++i) {
           L.lin_in[i] = ins[i];
           L.lin_out[i] = outs[i];
           L.la[i] = L.lb[i] = 0;
           if (r > 0) {
             L.la[i] = off;
-            off += round_up((size_t)r * ins[i], 64);
+            off += round_up(r16 * ins[i], 64);
             L.lb[i] = off;
-            off += round_up((size_t)outs[i] * r, 64);
+            off += round_up(r16 * outs[i], 64);
           }
         }
         ck.layers.push_back(L);
@@ -965,7 +978,14 @@ zl_status zl_set_param(zl_ctx* c, const char* name, const void* src, size_t byte
     if (bytes != f.numel * 4) raise_err(ZL_ERR_ARG, std::string("byte count mismatch for ") + name);
     sync_all(c, -1);
     const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
-    if (f.chunk) {
+    if (f.trows > 0) {   // user layout [tcols, trows] -> stored [trows, tcols]
+      std::vector<float> h(f.numel), t(f.numel);
+      CK(cudaMemcpy(h.data(), src, bytes, on_device ? cudaMemcpyDeviceToHost : cudaMemcpyHostToHost));
+      for (int o = 0; o < f.tcols; ++o)
+        for (int j = 0; j < f.trows; ++j) t[(size_t)j * f.tcols + o] = h[(size_t)o * f.trows + j];
+      CK(cudaMemcpy(f.dev, t.data(), bytes, cudaMemcpyHostToDevice));
+      if (c->dt == BF16) launch_f32_to_bf16((const float*)f.dev, (bf16*)f.chunk->comp + f.off, f.numel, 0);
+    } else if (f.chunk) {
       CK(cudaMemcpy(f.dev, src, bytes, kind));
       if (c->dt == BF16) launch_f32_to_bf16((const float*)f.dev, (bf16*)f.chunk->comp + f.off, f.numel, 0);
     } else if (f.fp32) {
@@ -1000,7 +1020,13 @@ zl_status zl_get_param(zl_ctx* c, const char* name, int which, void* dst, size_t
       srcp = base + f.off;
     }
     const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
-    if (f.fp32 || which > 0) {
+    if (f.trows > 0) {   // stored [trows, tcols] -> user layout [tcols, trows]
+      std::vector<float> h(f.numel), t(f.numel);
+      CK(cudaMemcpy(h.data(), srcp, bytes, cudaMemcpyDeviceToHost));
+      for (int j = 0; j < f.trows; ++j)
+        for (int o = 0; o < f.tcols; ++o) t[(size_t)o * f.trows + j] = h[(size_t)j * f.tcols + o];
+      CK(cudaMemcpy(dst, t.data(), bytes, on_device ? cudaMemcpyHostToDevice : cudaMemcpyHostToHost));
+    } else if (f.fp32 || which > 0) {
       CK(cudaMemcpy(dst, srcp, bytes, kind));
     } else {
       std::vector<uint16_t> h(f.numel);

@@ -206,3 +206,10 @@ def test_attention_matches_sdpa(B, dtype, Bb, S, H, Hkv, hd):
             continue
         cos = float(a @ r / (a.norm() * r.norm() + 1e-30))
         assert cos >= 0.9995, (lo, cos)
+
+
+@pytest.mark.parametrize("mode,M,N,K", [(0, 4096, 16, 768), (1, 4096, 2304, 16), (2, 16, 2304, 4096),
+                                        (2, 16, 768, 4096), (0, 512, 16, 3072), (1, 300, 768, 16)])
+def test_gemm_rank16_shapes(B, mode, M, N, K):
+    """The LoRA products: one of M, N, K is the padded rank 16 (tensor-core path, partial tiles)."""
+    test_gemm_tensor_core_matches_fp32(B, mode, M, N, K)
