@@ -77,6 +77,7 @@ typedef struct {
   int serialize;            /* 1: every chunk on one stream (no overlap; for measurement), 0: K streams */
   int lora_rank;            /* 0: full fine-tune; r > 0: LoRA (Section II-A) on the QKV, output and FFN  */
   float lora_scale;         /*   linears, w + lora_scale * B A, only A [r, in] and B [out, r] trainable  */
+  int replay_depth;         /* D >= 0: zl_step keeps each chunk's last D inputs for zl_replay          */
 } zl_train_cfg;
 
 /* Create a context: parameters, AdamW state, K streams and events, a stream-ordered
@@ -139,6 +140,20 @@ zl_status zl_step(zl_ctx* ctx, const int32_t* ids, const int32_t* labels, int B,
  * CE over Omega, gradient through every chunk, AdamW on all (window rules as above). */
 zl_status zl_bp_step(zl_ctx* ctx, const int32_t* ids, const int32_t* labels, int B, int S,
                      float* loss_out);
+
+/* Failure recovery (Section III-B-3). Proactive checkpointing: zl_chunk_save writes chunk k's
+ * state (fp32 master weights, gradient accumulator, AdamW moments, optimizer step, progress) into a
+ * caller-owned host buffer of zl_chunk_state_bytes bytes; zl_chunk_load restores it (ZL_ERR_ARG if
+ * the blob belongs to another chunk or shape). Reactive recovery: with replay_depth D > 0, zl_step
+ * keeps each chunk's inputs h_{k-1} and labels of the last D micro-batches in a device ring (the
+ * paper's hidden-state buffer); zl_replay re-runs chunk k's local steps for every buffered
+ * micro-batch after its restored progress, catching it up to the pipeline frontier while the other
+ * chunks keep their state. *replayed (optional) gets the count, *loss_out (optional) the last L_k.
+ * ZL_ERR_ARG if a needed micro-batch has left the ring. */
+zl_status zl_chunk_state_bytes(zl_ctx* ctx, int k, size_t* bytes);
+zl_status zl_chunk_save(zl_ctx* ctx, int k, void* host_dst, size_t bytes);
+zl_status zl_chunk_load(zl_ctx* ctx, int k, const void* host_src, size_t bytes);
+zl_status zl_replay(zl_ctx* ctx, int k, int* replayed, float* loss_out);
 
 /* Global objective L(p_K) = CE of the last chunk's readout over Omega (Section II-C). */
 zl_status zl_eval_global_loss(zl_ctx* ctx, const int32_t* ids, const int32_t* labels, int B, int S,

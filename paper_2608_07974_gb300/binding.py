@@ -21,7 +21,8 @@ ZL_DTYPE_F32, ZL_DTYPE_BF16 = 0, 1
 EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_get_param", "zl_param_numel",
            "zl_embed", "zl_forward_chunk", "zl_local_step", "zl_step", "zl_bp_step", "zl_eval_global_loss",
            "zl_read_losses", "zl_join", "zl_synchronize", "zl_peak_bytes", "zl_reset_peak", "zl_last_error",
-           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches"]
+           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
+           "zl_chunk_load", "zl_replay"]
 
 
 class zl_model_dims(C.Structure):
@@ -35,7 +36,7 @@ class zl_train_cfg(C.Structure):
                 ("beta1", C.c_float), ("beta2", C.c_float), ("eps", C.c_float), ("weight_decay", C.c_float),
                 ("accum_m", C.c_int), ("max_live_chunks", C.c_int), ("lr_schedule", C.c_int),
                 ("lr_gamma", C.c_float), ("serialize", C.c_int), ("lora_rank", C.c_int),
-                ("lora_scale", C.c_float)]
+                ("lora_scale", C.c_float), ("replay_depth", C.c_int)]
 
 
 class ZLError(RuntimeError):
@@ -77,6 +78,10 @@ def _load() -> C.CDLL:
         "zl_profile": [vp, i],
         "zl_profile_read": [vp, C.c_char_p, sz],
         "zl_kernel_launches": [C.POINTER(C.c_uint64)],
+        "zl_chunk_state_bytes": [vp, i, C.POINTER(sz)],
+        "zl_chunk_save": [vp, i, vp, sz],
+        "zl_chunk_load": [vp, i, vp, sz],
+        "zl_replay": [vp, i, C.POINTER(C.c_int), C.POINTER(f)],
     }
     for name, args in sig.items():
         fn = getattr(lib, name)
@@ -273,6 +278,24 @@ def zl_kernel_launches() -> int:
     return n.value
 
 
+def zl_chunk_save(ctx, k: int) -> bytes:
+    n = C.c_size_t()
+    _check(_lib.zl_chunk_state_bytes(ctx, k, C.byref(n)))
+    buf = C.create_string_buffer(n.value)
+    _check(_lib.zl_chunk_save(ctx, k, buf, n.value))
+    return buf.raw
+
+
+def zl_chunk_load(ctx, k: int, blob: bytes) -> None:
+    _check(_lib.zl_chunk_load(ctx, k, blob, len(blob)))
+
+
+def zl_replay(ctx, k: int):
+    n, loss = C.c_int(), C.c_float()
+    _check(_lib.zl_replay(ctx, k, C.byref(n), C.byref(loss)))
+    return n.value, loss.value
+
+
 # ---- convenience object ----------------------------------------------------------------------
 class ZeroLock:
     """One engine context: a model cut into K chunks, its AdamW state and K CUDA streams."""
@@ -281,7 +304,7 @@ class ZeroLock:
                  kl_dir: int = 0, consis_first: int = 1, lr: float = 1e-3, beta1: float = 0.9,
                  beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.01, accum_m: int = 1,
                  max_live_chunks: int = 0, lr_schedule: int = 0, lr_gamma: float = 1.0, serialize: bool = False,
-                 lora_rank: int = 0, lora_scale: float = 1.0, stream=None):
+                 lora_rank: int = 0, lora_scale: float = 1.0, replay_depth: int = 0, stream=None):
         import torch
         self.dims = dims
         self.K = K
@@ -290,7 +313,8 @@ class ZeroLock:
                            dims.d_model, dims.n_heads, dims.n_kv_heads, dims.d_ff, dims.vocab, dims.max_seq,
                            dims.norm_eps, dims.rope_theta)
         cfg = zl_train_cfg(alpha, kl_dir, consis_first, lr, beta1, beta2, eps, weight_decay, accum_m,
-                           max_live_chunks, lr_schedule, lr_gamma, int(serialize), lora_rank, lora_scale)
+                           max_live_chunks, lr_schedule, lr_gamma, int(serialize), lora_rank, lora_scale,
+                           replay_depth)
         self.ctx = zl_create(md, K, list(bounds), cfg)
         s = stream if stream is not None else torch.cuda.current_stream()
         zl_set_stream(self.ctx, s.cuda_stream)

@@ -96,6 +96,16 @@ struct Chunk {
   std::vector<Layer> layers;
   int micro = 0;
   long t = 0;
+  long done = 0;             // micro-batches this chunk has processed (progress metadata)
+  // hidden-state buffer (Section III-B-3): the last replay_depth inputs h_{k-1} with their labels
+  struct Entry {
+    long seq = -1;
+    int B = 0, S = 0;
+    size_t cap = 0;          // tokens the buffers hold
+    void* h = nullptr;
+    int32_t* labels = nullptr;
+  };
+  std::vector<Entry> ring;
   cudaStream_t s = nullptr;
   cudaEvent_t ev_h = nullptr, ev_z = nullptr, ev_loss = nullptr, ev_hb = nullptr, ev_done = nullptr;
 };
@@ -133,6 +143,7 @@ struct zl_ctx {
   float* d_losses = nullptr;     // [K + 1]
   float* h_losses = nullptr;     // pinned [K + 1]
   int last_nloss = 0;
+  long seq = 0;              // micro-batches seen by zl_step (the pipeline frontier)
   bool broken = false;
   std::vector<void*> statics;
   bool prof = false;
@@ -548,6 +559,29 @@ void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s) {
 
 float alpha_of(zl_ctx* c, int k) { return (k == 1 && !c->cfg.consis_first) ? 1.f : c->cfg.alpha; }
 
+// Keeps chunk k's input of micro-batch `seq` (h_{k-1} and the labels) in its hidden-state buffer.
+void ring_put(zl_ctx* c, Chunk& ck, long seq, const void* h_in, const int32_t* labels, int B, int S, cudaStream_t s) {
+  const int D = c->cfg.replay_depth;
+  if (D <= 0) return;
+  if ((int)ck.ring.size() != D) ck.ring.resize(D);
+  Chunk::Entry& e = ck.ring[seq % D];
+  const size_t N = (size_t)B * S;
+  if (e.cap < N) {   // grow (rare): wait for this stream's use of the old buffers first
+    CK(cudaStreamSynchronize(s));
+    if (e.h) { CK(cudaFree(e.h)); c->static_bytes -= e.cap * c->d * esz(c); }
+    if (e.labels) { CK(cudaFree(e.labels)); c->static_bytes -= e.cap * 4; }
+    CK(cudaMalloc(&e.h, N * c->d * esz(c)));
+    CK(cudaMalloc((void**)&e.labels, N * 4));
+    c->static_bytes += N * c->d * esz(c) + N * 4;
+    e.cap = N;
+  }
+  CK(cudaMemcpyAsync(e.h, h_in, N * c->d * esz(c), cudaMemcpyDeviceToDevice, s));
+  CK(cudaMemcpyAsync(e.labels, labels, N * 4, cudaMemcpyDeviceToDevice, s));
+  e.seq = seq;
+  e.B = B;
+  e.S = S;
+}
+
 // ----------------------------------------------------------------------------------------------
 // Readout (Eq. 2) and its backward (frozen head: no parameter gradient)
 // ----------------------------------------------------------------------------------------------
@@ -713,6 +747,10 @@ void free_ctx(zl_ctx* c) {
   const bool shared = c->cfg.serialize != 0;
   for (int k = 1; k < (int)c->ch.size(); ++k) {
     Chunk& ck = c->ch[k];
+    for (auto& e : ck.ring) {
+      if (e.h) cudaFree(e.h);
+      if (e.labels) cudaFree(e.labels);
+    }
     if (ck.s && (!shared || k == 1)) cudaStreamDestroy(ck.s);
     for (cudaEvent_t e : {ck.ev_h, ck.ev_z, ck.ev_loss, ck.ev_hb, ck.ev_done})
       if (e) cudaEventDestroy(e);
@@ -784,6 +822,7 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (cfg->lr_schedule == 1 && !(cfg->lr_gamma > 0.f)) why = "lr_gamma must be > 0";
   else if (cfg->serialize != 0 && cfg->serialize != 1) why = "serialize must be 0 or 1";
   else if (cfg->lora_rank < 0 || cfg->lora_rank > 256) why = "lora_rank must be in [0, 256]";
+  else if (cfg->replay_depth < 0 || cfg->replay_depth > 4096) why = "replay_depth must be in [0, 4096]";
   else if (cfg->lora_rank > 0 && !(std::isfinite(cfg->lora_scale))) why = "lora_scale must be finite";
   for (int k = 1; why.empty() && k <= K; ++k)
     if (bounds[k] <= bounds[k - 1]) why = "bounds must be strictly increasing";
@@ -1076,6 +1115,47 @@ zl_status zl_forward_chunk(zl_ctx* c, int k, const void* h_in, const int32_t* id
   });
 }
 
+// Steps S1-S3 of Section III-B for chunk k on one micro-batch, queued on the chunk's stream.
+void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, const int32_t* labels, int B, int S,
+                     void* h_out) {
+  Chunk& ck = c->ch[k];
+  cudaStream_t s = ck.s;
+  const int N = B * S;
+  const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+  void* h0 = nullptr;
+  if (!h_in) {
+    h0 = palloc(c, hb, s);
+    launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h0, N, S, c->d, c->V, c->d_err, s);
+    h_in = h0;
+  }
+  const float a = alpha_of(c, k);
+  void* t = nullptr;
+  if (a < 1.f) {   // teacher p_{k-1} = readout(h_{k-1}), recomputed from the detached input
+    t = palloc(c, zb, s);
+    readout_fwd(c, h_in, t, nullptr, N, s);
+  }
+  void* hk = palloc(c, hb, s);
+  ChunkActs acts;
+  chunk_fwd_save(c, ck, h_in, hk, B, S, acts, s);
+  if (h_out) CK(cudaMemcpyAsync(h_out, hk, hb, cudaMemcpyDeviceToDevice, s));
+  void* z = palloc(c, zb, s);
+  ReadoutSave rs;
+  readout_fwd(c, hk, z, &rs, N, s);
+  void* dz = local_loss(c, z, t, labels, a, N, k, s);
+  pfree(z, s);
+  pfree(t, s);
+  void* dh = palloc(c, hb, s);
+  readout_bwd(c, hk, rs, dz, dh, N, s);
+  pfree(dz, s);
+  chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
+  pfree(dh, s);
+  pfree(acts.mem, s);
+  pfree(hk, s);
+  pfree(h0, s);
+  adamw_window(c, ck, s);
+  ck.done += 1;
+}
+
 zl_status zl_local_step(zl_ctx* c, int k, const void* h_in, const int32_t* ids, const int32_t* labels, int B, int S,
                         void* h_out, float* loss_out) {
   if (!c || !labels) { g_err = "NULL argument"; return ZL_ERR_ARG; }
@@ -1083,47 +1163,105 @@ zl_status zl_local_step(zl_ctx* c, int k, const void* h_in, const int32_t* ids, 
     check_bs(c, B, S);
     if (k < 1 || k > c->K) raise_err(ZL_ERR_ARG, "chunk index out of [1, K]");
     if (!h_in && (k != 1 || !ids)) raise_err(ZL_ERR_ARG, "h_in may be NULL only for k = 1 with ids");
-    Chunk& ck = c->ch[k];
-    cudaStream_t s = ck.s;
-    start_on(c, s);
-    const int N = B * S;
-    const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
-    void* h0 = nullptr;
-    if (!h_in) {
-      h0 = palloc(c, hb, s);
-      launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h0, N, S, c->d, c->V, c->d_err, s);
-      h_in = h0;
-    }
-    const float a = alpha_of(c, k);
-    void* t = nullptr;
-    if (a < 1.f) {   // teacher p_{k-1} = readout(h_{k-1}), recomputed from the detached input
-      t = palloc(c, zb, s);
-      readout_fwd(c, h_in, t, nullptr, N, s);
-    }
-    void* hk = palloc(c, hb, s);
-    ChunkActs acts;
-    chunk_fwd_save(c, ck, h_in, hk, B, S, acts, s);
-    if (h_out) CK(cudaMemcpyAsync(h_out, hk, hb, cudaMemcpyDeviceToDevice, s));
-    void* z = palloc(c, zb, s);
-    ReadoutSave rs;
-    readout_fwd(c, hk, z, &rs, N, s);
-    void* dz = local_loss(c, z, t, labels, a, N, k, s);
-    pfree(z, s);
-    pfree(t, s);
-    void* dh = palloc(c, hb, s);
-    readout_bwd(c, hk, rs, dz, dh, N, s);
-    pfree(dz, s);
-    chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
-    pfree(dh, s);
-    pfree(acts.mem, s);
-    pfree(hk, s);
-    pfree(h0, s);
-    adamw_window(c, ck, s);
+    start_on(c, c->ch[k].s);
+    local_step_impl(c, k, h_in, ids, labels, B, S, h_out);
     if (loss_out) {
-      CK(cudaMemcpyAsync(c->h_losses + k, c->d_losses + k, 4, cudaMemcpyDeviceToHost, s));
+      CK(cudaMemcpyAsync(c->h_losses + k, c->d_losses + k, 4, cudaMemcpyDeviceToHost, c->ch[k].s));
       sync_all(c, -1);
       *loss_out = c->h_losses[k];
     }
+    return ZL_OK;
+  });
+}
+
+// Catch chunk k up to the pipeline frontier from its hidden-state buffer (reactive recovery,
+// Section III-B-3): re-runs its local steps for every buffered micro-batch after its progress.
+zl_status zl_replay(zl_ctx* c, int k, int* replayed, float* loss_out) {
+  if (!c) { g_err = "NULL context"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    if (k < 1 || k > c->K) raise_err(ZL_ERR_ARG, "chunk index out of [1, K]");
+    Chunk& ck = c->ch[k];
+    const int D = c->cfg.replay_depth;
+    if (ck.done > c->seq) raise_err(ZL_ERR_STATE, "chunk progress is ahead of the pipeline frontier");
+    if (ck.done < c->seq && (D <= 0 || c->seq - ck.done > D))
+      raise_err(ZL_ERR_ARG, "the micro-batches to replay are no longer in the hidden-state buffer");
+    start_on(c, ck.s);
+    int n = 0;
+    for (long q = ck.done; q < c->seq; ++q) {
+      Chunk::Entry& e = ck.ring[q % D];
+      if (e.seq != q) raise_err(ZL_ERR_ARG, "hidden-state buffer entry missing");
+      local_step_impl(c, k, e.h, nullptr, e.labels, e.B, e.S, nullptr);
+      ++n;
+    }
+    if (replayed) *replayed = n;
+    if (loss_out && n > 0) {
+      CK(cudaMemcpyAsync(c->h_losses + k, c->d_losses + k, 4, cudaMemcpyDeviceToHost, ck.s));
+      sync_all(c, -1);
+      *loss_out = c->h_losses[k];
+    }
+    return ZL_OK;
+  });
+}
+
+// Per-chunk checkpoint (proactive checkpointing, Section III-B-3): header, then the trainable
+// slab's fp32 master, gradient accumulator and AdamW moments.
+struct CkptHeader {
+  uint64_t magic;
+  int32_t k, l0, l1, lora_rank;
+  int64_t n, t, done;
+  int32_t micro, dtype;
+};
+constexpr uint64_t kCkptMagic = 0x31304B434C5A4C5AULL;   // "ZLZLCK01"
+
+zl_status zl_chunk_state_bytes(zl_ctx* c, int k, size_t* bytes) {
+  if (!c || !bytes) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if (k < 1 || k > c->K) { g_err = "chunk index out of [1, K]"; return ZL_ERR_ARG; }
+  *bytes = sizeof(CkptHeader) + 4 * c->ch[k].n * sizeof(float);
+  return ZL_OK;
+}
+
+zl_status zl_chunk_save(zl_ctx* c, int k, void* dst, size_t bytes) {
+  if (!c || !dst) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    if (k < 1 || k > c->K) raise_err(ZL_ERR_ARG, "chunk index out of [1, K]");
+    Chunk& ck = c->ch[k];
+    if (bytes != sizeof(CkptHeader) + 4 * ck.n * sizeof(float)) raise_err(ZL_ERR_ARG, "checkpoint size mismatch");
+    sync_all(c, -1);
+    CkptHeader h{kCkptMagic, k, ck.l0, ck.l1, c->cfg.lora_rank, (int64_t)ck.n, ck.t, ck.done, ck.micro, c->dt};
+    std::memcpy(dst, &h, sizeof h);
+    float* p = reinterpret_cast<float*>(static_cast<char*>(dst) + sizeof h);
+    const size_t sz = ck.n * sizeof(float);
+    CK(cudaMemcpy(p, ck.master, sz, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(p + ck.n, ck.grad, sz, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(p + 2 * ck.n, ck.m, sz, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(p + 3 * ck.n, ck.v, sz, cudaMemcpyDeviceToHost));
+    return ZL_OK;
+  });
+}
+
+zl_status zl_chunk_load(zl_ctx* c, int k, const void* src, size_t bytes) {
+  if (!c || !src) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    if (k < 1 || k > c->K) raise_err(ZL_ERR_ARG, "chunk index out of [1, K]");
+    Chunk& ck = c->ch[k];
+    if (bytes != sizeof(CkptHeader) + 4 * ck.n * sizeof(float)) raise_err(ZL_ERR_ARG, "checkpoint size mismatch");
+    CkptHeader h;
+    std::memcpy(&h, src, sizeof h);
+    if (h.magic != kCkptMagic || h.k != k || h.l0 != ck.l0 || h.l1 != ck.l1 || h.lora_rank != c->cfg.lora_rank ||
+        h.n != (int64_t)ck.n || h.dtype != c->dt)
+      raise_err(ZL_ERR_ARG, "checkpoint does not belong to this chunk");
+    sync_all(c, -1);
+    const float* p = reinterpret_cast<const float*>(static_cast<const char*>(src) + sizeof h);
+    const size_t sz = ck.n * sizeof(float);
+    CK(cudaMemcpy(ck.master, p, sz, cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(ck.grad, p + ck.n, sz, cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(ck.m, p + 2 * ck.n, sz, cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(ck.v, p + 3 * ck.n, sz, cudaMemcpyHostToDevice));
+    if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
+    CK(cudaDeviceSynchronize());
+    ck.t = h.t;
+    ck.done = h.done;
+    ck.micro = h.micro;
     return ZL_OK;
   });
 }
@@ -1162,6 +1300,8 @@ zl_status zl_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
       const float a = alpha_of(c, k);
       // S1: the upstream entry (h_{k-1}) and a free arena slot
       if (k > 1) wait_ev(s, c->ch[k - 1].ev_h);
+      ring_put(c, ck, c->seq, h[k - 1], labels, B, S, s);
+      ck.done += 1;
       const long seq = c->live_seq++;
       if (seq >= cap) wait_ev(s, c->live_ring[seq % cap]);
       // S2: forward, then hand h_k downstream before the local backward (early forwarding)
@@ -1206,6 +1346,7 @@ zl_status zl_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
       adamw_window(c, ck, s);
     }
     c->last_nloss = K;
+    c->seq += 1;
     if (losses_out) {
       for (int k = 1; k <= K; ++k)
         CK(cudaMemcpyAsync(c->h_losses + k, c->d_losses + k, 4, cudaMemcpyDeviceToHost, c->ch[k].s));
@@ -1265,6 +1406,7 @@ zl_status zl_bp_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B
       adamw_window(c, c->ch[k], k == 1 ? s : c->ch[k].s);
     }
     c->last_nloss = 1;
+    for (int k = 1; k <= K; ++k) c->ch[k].done += 1;
     if (loss_out) {
       CK(cudaMemcpyAsync(c->h_losses, c->d_losses, 4, cudaMemcpyDeviceToHost, s));
       sync_all(c, -1);

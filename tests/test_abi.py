@@ -42,12 +42,12 @@ def test_bad_arguments_are_rejected_on_the_host(lib):
     """zl_create validates its arguments before touching the device."""
     from paper_2608_07974_gb300 import binding as b
     dims = b.zl_model_dims(0, 0, 4, 128, 4, 4, 344, 512, 64, 1e-5, 1e4)
-    cfg = b.zl_train_cfg(0.5, 0, 1, 1e-3, 0.9, 0.999, 1e-8, 0.01, 1, 0, 0, 1.0, 0, 0, 1.0)
+    cfg = b.zl_train_cfg(0.5, 0, 1, 1e-3, 0.9, 0.999, 1e-8, 0.01, 1, 0, 0, 1.0, 0, 0, 1.0, 0)
     for bounds, K in ([[0, 3, 2], 2], [[0, 2, 5], 2], [[1, 4], 1], [[0, 4], 0]):
         with pytest.raises(b.ZLError) as e:
             b.zl_create(dims, K, bounds, cfg)
         assert e.value.status == b.ZL_ERR_ARG
-    bad = b.zl_train_cfg(1.5, 0, 1, 1e-3, 0.9, 0.999, 1e-8, 0.01, 1, 0, 0, 1.0, 0, 0, 1.0)
+    bad = b.zl_train_cfg(1.5, 0, 1, 1e-3, 0.9, 0.999, 1e-8, 0.01, 1, 0, 0, 1.0, 0, 0, 1.0, 0)
     with pytest.raises(b.ZLError):
         b.zl_create(dims, 2, [0, 2, 4], bad)
     odd = b.zl_model_dims(0, 0, 4, 130, 4, 4, 344, 512, 64, 1e-5, 1e4)
