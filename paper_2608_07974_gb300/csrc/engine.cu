@@ -379,7 +379,7 @@ void layer_fwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* x, void* 
 struct BwdWs {
   void *da, *dhid, *dxn, *dx2, *datt, *dqkv, *dy0, *dy1, *du;
   float *part_g, *part_b, *D;
-  unsigned* counter;   // column-sum completion ticket (zero between launches)
+  unsigned* counter;   // column-sum completion tickets, one per 256-column group (zero between launches)
 };
 
 size_t bwd_ws_bytes(zl_ctx* c, int N, int B, int S) {
@@ -398,7 +398,7 @@ size_t bwd_ws_bytes(zl_ctx* c, int N, int B, int S) {
   add((size_t)colsum_blocks(N) * wmax * 4);
   add((size_t)colsum_blocks(N) * wmax * 4);
   add((size_t)B * c->H * S * 4);
-  add(4);
+  add((size_t)colsum_groups((int)wmax) * 4);
   add((size_t)N * std::max(lora_r16(c->cfg.lora_rank), 1) * e);
   return b;
 }
@@ -417,7 +417,7 @@ void carve_ws(zl_ctx* c, Arena& a, BwdWs& w, int N, int B, int S) {
   w.part_g = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
   w.part_b = (float*)a.take((size_t)colsum_blocks(N) * wmax * 4);
   w.D = (float*)a.take((size_t)B * c->H * S * 4);
-  w.counter = (unsigned*)a.take(4);
+  w.counter = (unsigned*)a.take((size_t)colsum_groups((int)wmax) * 4);
   w.du = a.take((size_t)N * std::max(lora_r16(c->cfg.lora_rank), 1) * e);
 }
 
@@ -531,7 +531,8 @@ void chunk_bwd(zl_ctx* c, Chunk& k, ChunkActs& acts, const void* dh, void* dh_in
   a.cap = wb;
   BwdWs w;
   carve_ws(c, a, w, N, B, S);
-  CK(cudaMemsetAsync(w.counter, 0, 4, s));
+  const size_t wmax = std::max({(size_t)c->d, (size_t)c->qkvw, (size_t)c->f1, (size_t)c->f});
+  CK(cudaMemsetAsync(w.counter, 0, (size_t)colsum_groups((int)wmax) * 4, s));
   const void* dy = dh;
   for (int i = nl - 1; i >= 0; --i) {
     void* dx = i > 0 ? ((i % 2) ? w.dy0 : w.dy1) : dh_in;
@@ -811,6 +812,7 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (D.n_heads % D.n_kv_heads != 0) why = "n_heads must be a multiple of n_kv_heads";
   else if (D.arch == ZL_ARCH_GPT2 && D.n_kv_heads != D.n_heads) why = "GPT-2 blocks use n_kv_heads == n_heads";
   else if (D.d_model % 8 != 0 || D.d_ff % 8 != 0) why = "d_model and d_ff must be multiples of 8";
+  else if (D.d_model > 16384) why = "d_model above 16384 is not supported";
   else if (!(D.norm_eps > 0.f)) why = "norm_eps";
   else if (K < 1 || K > D.n_layers) why = "K must be in [1, n_layers]";
   else if (bounds[0] != 0 || bounds[K] != D.n_layers) why = "bounds[0] must be 0 and bounds[K] n_layers";

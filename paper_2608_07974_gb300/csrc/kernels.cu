@@ -62,54 +62,14 @@ void launch_embed(int dt, const int32_t* ids, const void* E, const void* P, void
 // ------------------------------------------------------------------------------------------
 // RMSNorm / LayerNorm forward and backward (one warp per row, 8-wide vector access, fp32 math).
 // ------------------------------------------------------------------------------------------
-template <typename T, bool LN>
-__global__ void norm_fwd_k(const T* __restrict__ x, const float* __restrict__ g, const float* __restrict__ b,
-                           T* __restrict__ y, float* __restrict__ rstd_o, float* __restrict__ mean_o, int N,
-                           int d, float eps) {
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (row >= N) return;
-  const T* xr = x + (size_t)row * d;
-  float s = 0.f, ss = 0.f;
-  for (int c = lane * 8; c < d; c += 256) {
-    float f[8];
-    Vec8<T>::load(xr + c, f);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) { s += f[i]; ss += f[i] * f[i]; }
-  }
-  s = warp_sum(s);
-  float mean = 0.f, var;
-  if (LN) {
-    mean = s / d;
-    float v = 0.f;
-    for (int c = lane * 8; c < d; c += 256) {
-      float f[8];
-      Vec8<T>::load(xr + c, f);
-#pragma unroll
-      for (int i = 0; i < 8; ++i) { const float t = f[i] - mean; v += t * t; }
-    }
-    var = warp_sum(v) / d;
-  } else {
-    var = warp_sum(ss) / d;
-  }
-  const float rstd = 1.f / sqrtf(var + eps);
-  T* yr = y + (size_t)row * d;
-  for (int c = lane * 8; c < d; c += 256) {
-    float f[8];
-    Vec8<T>::load(xr + c, f);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      f[i] = (f[i] - mean) * rstd * (g ? g[c + i] : 1.f);
-      if (LN && b) f[i] += b[c + i];
-    }
-    Vec8<T>::store(yr + c, f);
-  }
-  if (lane == 0) {
-    if (rstd_o) rstd_o[row] = rstd;
-    if (LN && mean_o) mean_o[row] = mean;
-  }
+// 8 consecutive fp32 values (32-byte aligned) as two 16-byte loads.
+__device__ __forceinline__ void load8f(const float* p, float* f) {
+  const float4 u = reinterpret_cast<const float4*>(p)[0], v = reinterpret_cast<const float4*>(p)[1];
+  f[0] = u.x; f[1] = u.y; f[2] = u.z; f[3] = u.w; f[4] = v.x; f[5] = v.y; f[6] = v.z; f[7] = v.w;
 }
 
-// Row held in registers (d <= 256 * VPL): one read of x, every load issued before the reductions.
+// Row held in registers (d <= 256 * VPL), one warp per row: one read of x; every load of the row, its
+// gains and biases is issued before the reductions, so a warp waits for memory once.
 template <typename T, bool LN, int VPL>
 __global__ void norm_fwd_reg_k(const T* __restrict__ x, const float* __restrict__ g, const float* __restrict__ b,
                                T* __restrict__ y, float* __restrict__ rstd_o, float* __restrict__ mean_o, int N, int d,
@@ -117,12 +77,15 @@ __global__ void norm_fwd_reg_k(const T* __restrict__ x, const float* __restrict_
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= N) return;
   const T* xr = x + (size_t)row * d;
-  float f[VPL][8];
+  float f[VPL][8], gv[VPL][8], bv[VPL][8];
 #pragma unroll
   for (int v = 0; v < VPL; ++v) {
     const int c = lane * 8 + v * 256;
-    if (c < d) Vec8<T>::load(xr + c, f[v]);
-    else {
+    if (c < d) {
+      Vec8<T>::load(xr + c, f[v]);
+      if (g) load8f(g + c, gv[v]);
+      if (LN && b) load8f(b + c, bv[v]);
+    } else {
 #pragma unroll
       for (int i = 0; i < 8; ++i) f[v][i] = 0.f;
     }
@@ -151,8 +114,8 @@ __global__ void norm_fwd_reg_k(const T* __restrict__ x, const float* __restrict_
     float o[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      o[i] = (f[v][i] - mean) * rstd * (g ? g[c + i] : 1.f);
-      if (LN && b) o[i] += b[c + i];
+      o[i] = (f[v][i] - mean) * rstd * (g ? gv[v][i] : 1.f);
+      if (LN && b) o[i] += bv[v][i];
     }
     Vec8<T>::store(yr + c, o);
   }
@@ -162,6 +125,7 @@ __global__ void norm_fwd_reg_k(const T* __restrict__ x, const float* __restrict_
   }
 }
 
+// dx = rstd * (dyh - mean(dyh) [LN] - xhat * mean(dyh * xhat)) (+ dres), dyh = g * dy; one warp per row.
 template <typename T, bool LN, int VPL>
 __global__ void norm_bwd_dx_reg_k(const T* __restrict__ x, const float* __restrict__ g,
                                   const float* __restrict__ rstd, const float* __restrict__ mean,
@@ -171,13 +135,20 @@ __global__ void norm_bwd_dx_reg_k(const T* __restrict__ x, const float* __restri
   if (row >= N) return;
   const size_t o = (size_t)row * d;
   const float r = rstd[row], mu = LN ? mean[row] : 0.f;
-  float fx[VPL][8], fd[VPL][8];
+  float fx[VPL][8], fd[VPL][8], fr[VPL][8];
 #pragma unroll
   for (int v = 0; v < VPL; ++v) {
     const int c = lane * 8 + v * 256;
     if (c < d) {
       Vec8<T>::load(x + o + c, fx[v]);
       Vec8<T>::load(dy + o + c, fd[v]);
+      if (dres) Vec8<T>::load(dres + o + c, fr[v]);
+      if (g) {
+        float gv[8];
+        load8f(g + c, gv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) fd[v][i] *= gv[i];
+      }
     } else {
 #pragma unroll
       for (int i = 0; i < 8; ++i) fx[v][i] = fd[v][i] = 0.f;
@@ -190,7 +161,6 @@ __global__ void norm_bwd_dx_reg_k(const T* __restrict__ x, const float* __restri
     if (c >= d) continue;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      fd[v][i] *= (g ? g[c + i] : 1.f);       // dy * gain
       fx[v][i] = (fx[v][i] - mu) * r;         // xhat
       s1 += fd[v][i];
       s2 += fd[v][i] * fx[v][i];
@@ -202,15 +172,131 @@ __global__ void norm_bwd_dx_reg_k(const T* __restrict__ x, const float* __restri
   for (int v = 0; v < VPL; ++v) {
     const int c = lane * 8 + v * 256;
     if (c >= d) continue;
-    float res[8], out[8];
-    if (dres) Vec8<T>::load(dres + o + c, res);
+    float out[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       out[i] = r * (fd[v][i] - (LN ? s1 : 0.f) - fx[v][i] * s2);
-      if (dres) out[i] += res[i];
+      if (dres) out[i] += fr[v][i];
     }
     Vec8<T>::store(dx + o + c, out);
   }
+}
+
+// One block per row (1024 < d <= 16384): thread t holds vectors t + j * blockDim.x, j < VPT, of the
+// row, every load issued before the block reductions.
+template <typename T, bool LN, int VPT>
+__global__ void __launch_bounds__(512) norm_fwd_blk_k(const T* __restrict__ x, const float* __restrict__ g,
+                                                      const float* __restrict__ b, T* __restrict__ y,
+                                                      float* __restrict__ rstd_o, float* __restrict__ mean_o, int N,
+                                                      int d, float eps) {
+  __shared__ float sh[32];
+  const size_t o = (size_t)blockIdx.x * d;
+  float f[VPT][8], gv[VPT][8], bv[VPT][8];
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int c = (threadIdx.x + j * blockDim.x) * 8;
+    if (c < d) {
+      Vec8<T>::load(x + o + c, f[j]);
+      if (g) load8f(g + c, gv[j]);
+      if (LN && b) load8f(b + c, bv[j]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) f[j][i] = 0.f;
+    }
+  }
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < VPT; ++j)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sum += f[j][i];
+  const float mean = LN ? block_sum(sum, sh) / d : 0.f;
+  float q = 0.f;
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    if ((int)(threadIdx.x + j * blockDim.x) * 8 >= d) continue;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { const float t = f[j][i] - mean; q += t * t; }
+  }
+  const float rstd = 1.f / sqrtf(block_sum(q, sh) / d + eps);
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int c = (threadIdx.x + j * blockDim.x) * 8;
+    if (c >= d) continue;
+    float out[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      out[i] = (f[j][i] - mean) * rstd * (g ? gv[j][i] : 1.f);
+      if (LN && b) out[i] += bv[j][i];
+    }
+    Vec8<T>::store(y + o + c, out);
+  }
+  if (threadIdx.x == 0) {
+    if (rstd_o) rstd_o[blockIdx.x] = rstd;
+    if (LN && mean_o) mean_o[blockIdx.x] = mean;
+  }
+}
+
+template <typename T, bool LN, int VPT>
+__global__ void __launch_bounds__(512) norm_bwd_dx_blk_k(const T* __restrict__ x, const float* __restrict__ g,
+                                                         const float* __restrict__ rstd,
+                                                         const float* __restrict__ mean, const T* __restrict__ dy,
+                                                         const T* __restrict__ dres, T* __restrict__ dx, int N,
+                                                         int d) {
+  __shared__ float sh[32];
+  const size_t o = (size_t)blockIdx.x * d;
+  const float r = rstd[blockIdx.x], mu = LN ? mean[blockIdx.x] : 0.f;
+  float fx[VPT][8], fd[VPT][8], fr[VPT][8];
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int c = (threadIdx.x + j * blockDim.x) * 8;
+    if (c < d) {
+      Vec8<T>::load(x + o + c, fx[j]);
+      Vec8<T>::load(dy + o + c, fd[j]);
+      if (dres) Vec8<T>::load(dres + o + c, fr[j]);
+      if (g) {
+        float gv[8];
+        load8f(g + c, gv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) fd[j][i] *= gv[i];
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) fx[j][i] = fd[j][i] = 0.f;
+    }
+  }
+  float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    if ((int)(threadIdx.x + j * blockDim.x) * 8 >= d) continue;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      fx[j][i] = (fx[j][i] - mu) * r;
+      s1 += fd[j][i];
+      s2 += fd[j][i] * fx[j][i];
+    }
+  }
+  s1 = LN ? block_sum(s1, sh) / d : 0.f;
+  s2 = block_sum(s2, sh) / d;
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int c = (threadIdx.x + j * blockDim.x) * 8;
+    if (c >= d) continue;
+    float out[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      out[i] = r * (fd[j][i] - s1 - fx[j][i] * s2);
+      if (dres) out[i] += fr[j][i];
+    }
+    Vec8<T>::store(dx + o + c, out);
+  }
+}
+
+// Threads per block (<= 512) and vectors per thread of the block-per-row kernels.
+static void blk_shape(int d, int& threads, int& vpt) {
+  const int nvec = d / 8;
+  vpt = 1;
+  while (vpt < 4 && (nvec + vpt - 1) / vpt > 512) vpt *= 2;
+  threads = ((nvec + vpt - 1) / vpt + 31) / 32 * 32;
 }
 
 void launch_norm_fwd(int dt, bool ln, const void* x, const float* g, const float* b, void* y, float* rstd,
@@ -224,58 +310,24 @@ void launch_norm_fwd(int dt, bool ln, const void* x, const float* g, const float
   else if (vpl == 2) NFR(T, L, 2);    \
   else if (vpl == 3) NFR(T, L, 3);    \
   else NFR(T, L, 4);
-#define NF(T, L) norm_fwd_k<T, L><<<blocks, th, 0, s>>>((const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
+#define NFB(T, L, V) norm_fwd_blk_k<T, L, V><<<N, bt, 0, s>>>((const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
+#define NF(T, L)                      \
+  if (vpt == 1) NFB(T, L, 1);         \
+  else if (vpt == 2) NFB(T, L, 2);    \
+  else NFB(T, L, 4);
   if (vpl <= 4) {
     if (dt == BF16) { if (ln) { NFV(bf16, true) } else { NFV(bf16, false) } }
     else { if (ln) { NFV(float, true) } else { NFV(float, false) } }
   } else {
-    if (dt == BF16) { if (ln) NF(bf16, true); else NF(bf16, false); }
-    else { if (ln) NF(float, true); else NF(float, false); }
+    int bt, vpt;
+    blk_shape(d, bt, vpt);
+    if (dt == BF16) { if (ln) { NF(bf16, true) } else { NF(bf16, false) } }
+    else { if (ln) { NF(float, true) } else { NF(float, false) } }
   }
 #undef NF
+#undef NFB
 #undef NFV
 #undef NFR
-}
-
-// dx = rstd * (dyh - mean(dyh) [LN] - xhat * mean(dyh * xhat)), dyh = g * dy.
-template <typename T, bool LN>
-__global__ void norm_bwd_dx_k(const T* __restrict__ x, const float* __restrict__ g,
-                              const float* __restrict__ rstd, const float* __restrict__ mean,
-                              const T* __restrict__ dy, const T* __restrict__ dres, T* __restrict__ dx, int N,
-                              int d) {
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (row >= N) return;
-  const size_t o = (size_t)row * d;
-  const float r = rstd[row], mu = LN ? mean[row] : 0.f;
-  float s1 = 0.f, s2 = 0.f;
-  for (int c = lane * 8; c < d; c += 256) {
-    float fx[8], fd[8];
-    Vec8<T>::load(x + o + c, fx);
-    Vec8<T>::load(dy + o + c, fd);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float dyh = fd[i] * (g ? g[c + i] : 1.f);
-      s1 += dyh;
-      s2 += dyh * (fx[i] - mu) * r;
-    }
-  }
-  s1 = warp_sum(s1) / d;
-  s2 = warp_sum(s2) / d;
-  for (int c = lane * 8; c < d; c += 256) {
-    float fx[8], fd[8], fr[8];
-    Vec8<T>::load(x + o + c, fx);
-    Vec8<T>::load(dy + o + c, fd);
-    if (dres) Vec8<T>::load(dres + o + c, fr);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float dyh = fd[i] * (g ? g[c + i] : 1.f);
-      const float xh = (fx[i] - mu) * r;
-      float v = r * (dyh - (LN ? s1 : 0.f) - xh * s2);
-      if (dres) v += fr[i];
-      fd[i] = v;
-    }
-    Vec8<T>::store(dx + o + c, fd);
-  }
 }
 
 void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const float* rstd, const float* mean,
@@ -291,53 +343,86 @@ void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const fl
   else if (vpl == 2) NBR(T, L, 2);    \
   else if (vpl == 3) NBR(T, L, 3);    \
   else NBR(T, L, 4);
-#define NB(T, L) \
-  norm_bwd_dx_k<T, L><<<blocks, th, 0, s>>>((const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, N, d)
+#define NBB(T, L, V)                                                                                          \
+  norm_bwd_dx_blk_k<T, L, V><<<N, bt, 0, s>>>((const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, N, d)
+#define NB(T, L)                      \
+  if (vpt == 1) NBB(T, L, 1);         \
+  else if (vpt == 2) NBB(T, L, 2);    \
+  else NBB(T, L, 4);
   if (vpl <= 4) {
     if (dt == BF16) { if (ln) { NBV(bf16, true) } else { NBV(bf16, false) } }
     else { if (ln) { NBV(float, true) } else { NBV(float, false) } }
   } else {
-    if (dt == BF16) { if (ln) NB(bf16, true); else NB(bf16, false); }
-    else { if (ln) NB(float, true); else NB(float, false); }
+    int bt, vpt;
+    blk_shape(d, bt, vpt);
+    if (dt == BF16) { if (ln) { NB(bf16, true) } else { NB(bf16, false) } }
+    else { if (ln) { NB(float, true) } else { NB(float, false) } }
   }
 #undef NB
+#undef NBB
 #undef NBV
 #undef NBR
 }
 
 static constexpr int kColRows = 64;   // rows per partial-sum block
+static constexpr int kColLanes = 8;   // row lanes per block: each thread sums kColRows / kColLanes rows
 int colsum_blocks(int N) { return (N + kColRows - 1) / kColRows; }
+int colsum_groups(int d) { return (d + 255) / 256; }
 
 // block (32, 8): 32 threads x 8 columns each (256 columns, 16-byte loads) x 8 row lanes;
-// grid (ceil(d/256), colsum_blocks(N)). Requires d % 8 == 0.
-// After its partial sums, the last block to finish (ticket counter) adds sum_b part[b][c], b in
-// increasing order, into the outputs and re-arms the counter: deterministic, one launch.
+// grid (colsum_groups(d), colsum_blocks(N)). Requires d % 8 == 0.
+// Every row load of a thread is issued before the first add (8 rows, 16 B each, in flight at once).
+// After its partial sums, the last block of each 256-column group (one ticket counter per group)
+// adds sum_b part[b][c], b in increasing order, into the outputs and re-arms its counter:
+// deterministic, one launch, and the final sums of the groups run in parallel.
 template <typename T, bool NORM, bool LN>
 __global__ void __launch_bounds__(256) colsum_k(const T* __restrict__ A, const T* __restrict__ x,
                                                 const float* __restrict__ rstd, const float* __restrict__ mean,
                                                 float* __restrict__ part_g, float* __restrict__ part_b, int N,
                                                 int d, float* __restrict__ out_g, float* __restrict__ out_b,
-                                                unsigned* __restrict__ counter) {
+                                                unsigned* __restrict__ counters) {
+  constexpr int R = kColRows / kColLanes;
   __shared__ unsigned ticket;
-  __shared__ float sg[8][256], sb[8][256];
+  __shared__ float sg[kColLanes][256], sb[kColLanes][256];
   const int c0 = blockIdx.x * 256 + threadIdx.x * 8;
-  const int r0 = blockIdx.y * kColRows;
-  const int r1 = min(r0 + kColRows, N);
+  const int rb = blockIdx.y * kColRows + threadIdx.y;
   float ag[8] = {0, 0, 0, 0, 0, 0, 0, 0}, ab[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   if (c0 < d) {
-    for (int r = r0 + threadIdx.y; r < r1; r += 8) {
-      float a[8];
-      Vec8<T>::load(A + (size_t)r * d + c0, a);
-      if (NORM) {
-        float xv[8];
-        Vec8<T>::load(x + (size_t)r * d + c0, xv);
-        const float mu = LN ? mean[r] : 0.f, rs = rstd[r];
+    float a[R][8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) ag[i] = fmaf(a[i], (xv[i] - mu) * rs, ag[i]);
+    for (int j = 0; j < R; ++j) {
+      const int r = rb + j * kColLanes;
+      if (r < N) Vec8<T>::load(A + (size_t)r * d + c0, a[j]);
+      else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a[j][i] = 0.f;
+      }
+    }
+    if (NORM) {
+      float xs[R][8], mu[R], rs[R];
+#pragma unroll
+      for (int j = 0; j < R; ++j) {
+        const int r = rb + j * kColLanes;
+        if (r < N) {
+          Vec8<T>::load(x + (size_t)r * d + c0, xs[j]);
+          mu[j] = LN ? mean[r] : 0.f;
+          rs[j] = rstd[r];
+        } else {
+          mu[j] = 0.f;
+          rs[j] = 0.f;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) xs[j][i] = 0.f;
+        }
       }
 #pragma unroll
-      for (int i = 0; i < 8; ++i) ab[i] += a[i];
+      for (int j = 0; j < R; ++j)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ag[i] = fmaf(a[j][i], (xs[j][i] - mu[j]) * rs[j], ag[i]);
     }
+#pragma unroll
+    for (int j = 0; j < R; ++j)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ab[i] += a[j][i];
   }
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
@@ -350,7 +435,7 @@ __global__ void __launch_bounds__(256) colsum_k(const T* __restrict__ A, const T
   if (c < d) {
     float tg = 0.f, tb = 0.f;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) { tg += sg[i][t]; tb += sb[i][t]; }
+    for (int i = 0; i < kColLanes; ++i) { tg += sg[i][t]; tb += sb[i][t]; }
     if (NORM) {
       part_g[(size_t)blockIdx.y * d + c] = tg;
       if (LN) part_b[(size_t)blockIdx.y * d + c] = tb;
@@ -360,51 +445,63 @@ __global__ void __launch_bounds__(256) colsum_k(const T* __restrict__ A, const T
   }
   __threadfence();
   __syncthreads();
-  if (t == 0) ticket = atomicAdd(counter, 1u);
+  if (t == 0) ticket = atomicAdd(counters + blockIdx.x, 1u);
   __syncthreads();
-  if (ticket != gridDim.x * gridDim.y - 1) return;
+  if (ticket != gridDim.y - 1) return;
   __threadfence();
-  const int nb = gridDim.y;
-  for (int cc = t; cc < d; cc += 256) {
-    if (NORM) {
-      float a = 0.f, bsum = 0.f;
-      for (int bb = 0; bb < nb; ++bb) {
-        a += __ldcg(part_g + (size_t)bb * d + cc);
-        if (LN) bsum += __ldcg(part_b + (size_t)bb * d + cc);
+  if (c < d) {
+    const int nb = gridDim.y;
+    float a = 0.f, bsum = 0.f;
+    int bb = 0;
+    for (; bb + 16 <= nb; bb += 16) {   // 16 loads in flight, added in increasing b
+      float vg[16], vb[16];
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        if (NORM) vg[q] = __ldcg(part_g + (size_t)(bb + q) * d + c);
+        if (!NORM || LN) vb[q] = __ldcg(part_b + (size_t)(bb + q) * d + c);
       }
-      out_g[cc] += a;
-      if (LN) out_b[cc] += bsum;
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        if (NORM) a += vg[q];
+        if (!NORM || LN) bsum += vb[q];
+      }
+    }
+    for (; bb < nb; ++bb) {
+      if (NORM) a += __ldcg(part_g + (size_t)bb * d + c);
+      if (!NORM || LN) bsum += __ldcg(part_b + (size_t)bb * d + c);
+    }
+    if (NORM) {
+      out_g[c] += a;
+      if (LN) out_b[c] += bsum;
     } else {
-      float bsum = 0.f;
-      for (int bb = 0; bb < nb; ++bb) bsum += __ldcg(part_b + (size_t)bb * d + cc);
-      out_b[cc] += bsum;
+      out_b[c] += bsum;
     }
   }
-  if (t == 0) *counter = 0u;
+  if (t == 0) counters[blockIdx.x] = 0u;
 }
 
 void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, const float* mean,
                             const void* dy, float* part_g, float* part_b, int N, int d, float* out_g, float* out_b,
-                            unsigned* counter, cudaStream_t s) {
+                            unsigned* counters, cudaStream_t s) {
   note_launch(1);
-  dim3 grid((d + 255) / 256, colsum_blocks(N)), block(32, 8);
+  dim3 grid(colsum_groups(d), colsum_blocks(N)), block(32, kColLanes);
 #define CS(T, L)                                                                                             \
   colsum_k<T, true, L><<<grid, block, 0, s>>>((const T*)dy, (const T*)x, rstd, mean, part_g, part_b, N, d, out_g, \
-                                              out_b, counter)
+                                              out_b, counters)
   if (dt == BF16) { if (ln) CS(bf16, true); else CS(bf16, false); }
   else { if (ln) CS(float, true); else CS(float, false); }
 #undef CS
 }
 
-void launch_colsum(int dt, const void* A, float* part, int N, int d, float* out, unsigned* counter, cudaStream_t s) {
+void launch_colsum(int dt, const void* A, float* part, int N, int d, float* out, unsigned* counters, cudaStream_t s) {
   note_launch(1);
-  dim3 grid((d + 255) / 256, colsum_blocks(N)), block(32, 8);
+  dim3 grid(colsum_groups(d), colsum_blocks(N)), block(32, kColLanes);
   if (dt == BF16)
     colsum_k<bf16, false, false><<<grid, block, 0, s>>>((const bf16*)A, nullptr, nullptr, nullptr, nullptr, part, N, d,
-                                                        nullptr, out, counter);
+                                                        nullptr, out, counters);
   else
     colsum_k<float, false, false><<<grid, block, 0, s>>>((const float*)A, nullptr, nullptr, nullptr, nullptr, part, N,
-                                                         d, nullptr, out, counter);
+                                                         d, nullptr, out, counters);
 }
 
 __global__ void partials_add_k(const float* __restrict__ part, int nb, int d, float* __restrict__ out) {
@@ -756,7 +853,14 @@ void launch_count_valid(const int32_t* labels, int N, int V, int* count, unsigne
 __global__ void loss_reduce_k(const float* __restrict__ rl, int N, const int* count, float* out) {
   __shared__ double sh[1024];
   double acc = 0.0;
-  for (int i = threadIdx.x; i < N; i += blockDim.x) acc += (double)rl[i];
+  for (int i0 = threadIdx.x; i0 < N; i0 += 4 * blockDim.x) {   // 4 loads in flight, added in index order
+    float v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = i0 + q * (int)blockDim.x < N ? rl[i0 + q * blockDim.x] : 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (i0 + q * (int)blockDim.x < N) acc += (double)v[q];
+  }
   sh[threadIdx.x] = acc;
   __syncthreads();
   for (int o = blockDim.x / 2; o > 0; o >>= 1) {

@@ -29,15 +29,17 @@ void launch_norm_fwd(int dt, bool ln, const void* x, const float* g, const float
 // dx = Norm'(x)^T (g * dy) (+ dres). g may be NULL (gain 1).
 void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const float* rstd, const float* mean,
                         const void* dy, const void* dres, void* dx, int N, int d, cudaStream_t s);
-// Column sums over rows, deterministic: per-row-block partials (part_*[b][c]), then the last block adds
-// sum_b part_*[b][c] into the outputs. Norm parameters: out_g += sum dy * xhat, out_b += sum dy (LN).
-// counter: a device word that is 0 before the launch and is 0 again after it (one per stream).
+// Column sums over rows, deterministic: per-row-block partials (part_*[b][c]), then the last block of
+// each 256-column group adds sum_b part_*[b][c] into the outputs. Norm parameters: out_g += sum dy * xhat,
+// out_b += sum dy (LN). counters: colsum_groups(d) device words, 0 before the launch and 0 again after
+// it (one array per stream).
 int colsum_blocks(int N);
+int colsum_groups(int d);
 void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, const float* mean,
                             const void* dy, float* part_g, float* part_b, int N, int d, float* out_g, float* out_b,
-                            unsigned* counter, cudaStream_t s);
+                            unsigned* counters, cudaStream_t s);
 // Bias gradients: out[c] += sum_r A[r][c].
-void launch_colsum(int dt, const void* A, float* part, int N, int d, float* out, unsigned* counter, cudaStream_t s);
+void launch_colsum(int dt, const void* A, float* part, int N, int d, float* out, unsigned* counters, cudaStream_t s);
 // out[c] += sum_b part[b][c], b in increasing order (deterministic).
 void launch_partials_add(const float* part, int nb, int d, float* out, cudaStream_t s);
 
