@@ -52,3 +52,24 @@ def test_wide_rows_match_oracle(name):
             ref = ref[list(range(d)) + list(range(d + kv, d + 2 * kv))]
         assert fro_rel(got, ref) <= TOL, n
     eng.close()
+
+
+def test_wide_gpt2_lora_matches_oracle():
+    """GPT-2 blocks with LoRA factors (rank 4, non-zero B) at the wide width: biased linears, GELU
+    and the block-per-row LayerNorms with frozen base weights, only A and B training."""
+    w = WIDE["gpt2-d1280"]
+    rank, scale = 4, 4.0
+    P = synth.make_params(w.dims, w.seed)
+    P.update(synth.make_lora_params(w.dims, w.seed, rank, b_std=0.05))
+    eng = engine_for(w, lora_rank=rank, lora_scale=scale)
+    eng.load(P)
+    orc = oracle_for(w, P, lora_rank=rank, lora_scale=scale)
+    for s in range(w.steps):
+        ids, labels = synth.make_batch(w, s)
+        lg = eng.step(ids.cuda(), labels.cuda())
+        lo = orc.step(ids, labels)
+        for a, b in zip(lg, lo):
+            assert rel(a, b) <= TOL, (s, lg, lo)
+    for n in orc.trainable_names():
+        assert fro_rel(eng.get(n), orc.P[n]) <= TOL, n
+    eng.close()
