@@ -27,7 +27,8 @@ def _loss_ref(z, t, labels, V, alpha, kl_dir):
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("N,V,alpha,kl_dir", [(37, 512, 0.5, 0), (64, 1000, 0.3, 1), (5, 50257, 0.5, 0),
-                                               (300, 32000, 1.0, 0), (1, 2, 0.7, 0)])
+                                               (300, 32000, 1.0, 0), (1, 2, 0.7, 0), (6, 50257, 0.4, 1),
+                                               (3, 65536, 0.5, 0), (3, 100000, 0.5, 1)])
 def test_local_loss_matches_oracle(B, dtype, N, V, alpha, kl_dir):
     torch.manual_seed(N + V)
     ldz = (V + 127) // 128 * 128
