@@ -439,16 +439,17 @@ bool launch_bn(int bn, const Args& a, const void* A, const void* B, cudaStream_t
   return launch<64, A_MN, B_MN>(a, A, B, s, 2);
 }
 
-// Tile width and split count from a wave model: units of 128 x BN x (K / splits) run on
-// 152 (BN 256/128) or 304 (BN 64) slots at one SM's share of the tensor rate, plus a fixed cost
-// per unit and, for splits, the fp32 partial traffic of the reduction.
-void choose(int M, int N, int K, int& bn_out, int& splits_out) {
-  const double rate = 1.45e15 / g_sms;        // flop/s of one SM
-  const double unit_fixed = 0.6e-6;           // pipeline fill and epilogue tail per unit (s)
+// Tile width and split count from a wave model: units of 128 x BN x (K / splits) run on 152 (BN
+// 256/128) or 304 (BN 64) slots, each k block (64 deep) of a unit taking the time measured for that
+// tile on GB300 (4096^3 and transformer-shape sweeps; the operands of the mode-2 kernel are both
+// MN-major and load in more boxes), plus, for splits, the fp32 partial traffic and the reduction.
+void choose(int mode, int M, int N, int K, int& bn_out, int& splits_out) {
   const double hbm = 6.0e12;                  // bytes/s for the partials
   const int nk = (K + BK - 1) / BK;
   double best = 1e30;
   for (int bn : {256, 128, 64}) {
+    const double kb = mode == 2 ? (bn == 256 ? 0.60e-6 : bn == 128 ? 0.41e-6 : 0.44e-6)
+                                : (bn == 256 ? 0.36e-6 : bn == 128 ? 0.29e-6 : 0.32e-6);
     const long tiles = (long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
     const int cps = bn == 64 ? 2 : 1;
     for (int sp : {1, 2, 3, 4, 6, 8}) {
@@ -457,8 +458,7 @@ void choose(int M, int N, int K, int& bn_out, int& splits_out) {
       const long units = tiles * sp;
       const long slots = (long)g_sms * cps;
       const long waves = (units + slots - 1) / slots;
-      const double unit_t = (2.0 * BM * bn * kps * BK) / (rate / cps) + unit_fixed;
-      double t = waves * unit_t;
+      double t = waves * kps * kb;
       if (sp > 1) t += (double)sp * M * N * 4.0 * 2.0 / hbm + 3e-6;
       if (t < best * 0.97) { best = t; bn_out = bn; splits_out = sp; }
     }
@@ -480,7 +480,7 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
   if ((mode == 0 || mode == 1) && K % 8 != 0) return false;
   if (mode == 2 && M % 8 != 0) return false;
   int bn = 128, splits = 1;
-  tc::choose(M, N, K, bn, splits);
+  tc::choose(mode, M, N, K, bn, splits);
   if (const char* force = std::getenv("ZL_GEMM_TILE")) {   // tuning override "BN:SPLITS"
     int fb = 0, fs = 0;
     if (std::sscanf(force, "%d:%d", &fb, &fs) == 2 && (fb == 64 || fb == 128 || fb == 256) && fs >= 1 && fs <= 16) {
@@ -528,11 +528,6 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
     cudaFreeAsync(ws, s);
   }
   return ok;
-}
-
-void gemm_tc_plan(int M, int N, int K, int* bn, int* splits) {
-  if (!tc::init()) { *bn = 0; *splits = 0; return; }
-  tc::choose(M, N, K, *bn, *splits);
 }
 
 }  // namespace zl

@@ -75,8 +75,6 @@ void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, v
 bool gemm_tc_available();
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
              unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha);
-// Tile width and split-K count the tensor-core GEMM picks for a shape (0, 0 if unavailable).
-void gemm_tc_plan(int M, int N, int K, int* bn, int* splits);
 void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
                const void* R, cudaStream_t s, float alpha = 1.f);
 

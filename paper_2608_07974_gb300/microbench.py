@@ -1,12 +1,12 @@
 """Single-kernel timings through the C ABI (CUDA events, after warm-up), for tuning and profiling.
 
     python -m paper_2608_07974_gb300.microbench loss [--rows 1024] [--vocab 50257] [--reps 4]
-    python -m paper_2608_07974_gb300.microbench gemm [--sweep]
+    python -m paper_2608_07974_gb300.microbench gemm [--sweep] [--workload gpt2|llama-1b]
     python -m paper_2608_07974_gb300.microbench attention [--batch 8 --seq 512 --heads 12 --kv-heads 12 --head-dim 64]
 
 `loss` runs the fused local objective on random bf16 logits; `gemm` times the GEMM shapes of the
-GPT-2-small workload (12 layers, d 768, FFN 3072, vocab 50304 padded, 4096 tokens), with --sweep
-every tile width / split-K count; `attention` the causal attention forward and backward.
+GPT-2-small workload (12 layers, d 768, FFN 3072, vocab 50304 padded, 4096 tokens) or of the
+Llama-style 1.1B one, with --sweep every tile width / split-K count; `attention` the causal attention forward and backward.
 """
 from __future__ import annotations
 
@@ -62,10 +62,22 @@ GPT2_SHAPES = [("qkv fwd", 0, 4096, 2304, 768), ("o fwd", 0, 4096, 768, 768), ("
                ("fc dW", 2, 3072, 768, 4096), ("proj dW", 2, 768, 3072, 4096), ("4096^3", 0, 4096, 4096, 4096)]
 
 
+def _shapes_of(d, d_qkv, f1, f, V, n=4096):
+    return [("qkv fwd", 0, n, d_qkv, d), ("o fwd", 0, n, d, d), ("ffn-in fwd", 0, n, f1, d), ("ffn-out fwd", 0, n, d, f),
+            ("head fwd", 0, n, V, d), ("qkv dX", 1, n, d, d_qkv), ("o dX", 1, n, d, d), ("ffn-in dX", 1, n, d, f1),
+            ("ffn-out dX", 1, n, f, d), ("head dX", 1, n, d, V), ("qkv dW", 2, d_qkv, d, n), ("o dW", 2, d, d, n),
+            ("ffn-in dW", 2, f1, d, n), ("ffn-out dW", 2, d, f, n), ("4096^3", 0, 4096, 4096, 4096)]
+
+
+# Llama-style 1.1B: d 2048, 32 query / 4 key-value heads of 64, SwiGLU 5632 (gate and up fused), vocab 32000
+LLAMA1B_SHAPES = _shapes_of(2048, 2560, 11264, 5632, 32000)
+
+
 def gemm(args):
     B = _lib()
     tiles = ["auto"] + ([f"{bn}:{s}" for bn in (64, 128, 256) for s in (1, 2, 3, 4, 6)] if args.sweep else [])
-    for name, mode, M, N, K in GPT2_SHAPES:
+    shapes = {"gpt2": GPT2_SHAPES, "llama-1b": LLAMA1B_SHAPES}[args.workload]
+    for name, mode, M, N, K in shapes:
         bf = torch.bfloat16
         if mode == 0:
             a, b = torch.randn(M, K, device="cuda").to(bf), torch.randn(N, K, device="cuda").to(bf)
@@ -115,6 +127,7 @@ def main():
     p.add_argument("--reps", type=int, default=4)
     p = sub.add_parser("gemm")
     p.add_argument("--sweep", action="store_true")
+    p.add_argument("--workload", choices=["gpt2", "llama-1b"], default="gpt2")
     p.add_argument("--reps", type=int, default=20)
     p = sub.add_parser("attention")
     p.add_argument("--batch", type=int, default=8)
