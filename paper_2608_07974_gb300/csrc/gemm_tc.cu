@@ -23,12 +23,14 @@ constexpr unsigned long long kTimeoutNs = 2000000000ull;   // 2 s per wait
 template <int BN>
 struct Cfg {
   // BN = 64 stays under 114 KB of shared memory so two CTAs (and TMEM allocations) fit on an SM.
-  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 4);
+  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 3);
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  // epilogue staging: per epilogue warp two buffers of 32 rows x 128 B (the TMA store box)
+  static constexpr int OUT_BYTES = 4 * 2 * 32 * 128;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + OUT_BYTES + 1024 + 256;
 };
 
 struct Args {
@@ -80,6 +82,31 @@ __device__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag
     }
   }
 }
+
+// Epilogue stores: shared memory -> global through the tensor map of C (bulk-group completion).
+__device__ __forceinline__ void tma_store2d(const CUtensorMap* m, const void* src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   (unsigned long long)m),
+               "r"(su32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void tma_store3d(const CUtensorMap* m, const void* src, int c0, int c1, int c2) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   (unsigned long long)m),
+               "r"(su32(src)), "r"(c0), "r"(c1), "r"(c2)
+               : "memory");
+}
+// fp32 C += tile, added by the TMA unit (one add per element: deterministic).
+__device__ __forceinline__ void tma_reduce_add2d(const CUtensorMap* m, const void* src, int c0, int c1) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   (unsigned long long)m),
+               "r"(su32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 __device__ __forceinline__ void tma2d(void* dst, const CUtensorMap* m, uint64_t* bar, int c0, int c1) {
   asm volatile(
@@ -137,11 +164,13 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
 
 template <int BN, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_tc_k(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, const Args g) {
+    gemm_tc_k(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+              const __grid_constant__ CUtensorMap tcm, const Args g) {
   using C_ = Cfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint64_t* full = (uint64_t*)(smem + C_::STAGES * C_::STAGE_BYTES);
+  uint8_t* outbuf = smem + C_::STAGES * C_::STAGE_BYTES;   // 1024-byte aligned (stage sizes are)
+  uint64_t* full = (uint64_t*)(outbuf + C_::OUT_BYTES);
   uint64_t* empty = full + C_::STAGES;
   uint64_t* tfull = empty + C_::STAGES;
   uint64_t* tempty = tfull + 2;
@@ -249,12 +278,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------- epilogue: warps 2..5, one accumulator row per thread ----------------
+    // Per 128-byte column chunk (64 bf16 or 32 fp32 columns): TMEM -> registers (alpha, bias,
+    // residual) -> this warp's staging buffer in the TMA 128-byte swizzle -> one TMA store (modes
+    // 0, 1: bf16 C; 3: fp32 split slice) or TMA reduce-add (mode 2: fp32 C += tile) by lane 0.
+    // The TMA clips rows >= M and columns >= N; two buffers per warp let a store drain while the
+    // next chunk is formed.
     const int q = warp & 3;   // TMEM lanes 32q..32q+31 are the ones this warp may read
-    int it = 0;
+    uint8_t* stage_out = outbuf + q * (2 * 32 * 128);
+    const bool f32out = g.mode >= 2;
+    const int ccols = f32out ? 32 : 64;   // columns per chunk
+    int it = 0, nchunk = 0;
     for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
       int tm, tn;
       tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
-      const size_t slice = (size_t)(unit / num_tiles) * g.M * g.N;
+      const int split = unit / num_tiles;
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
       int ok = 1;
@@ -262,61 +299,81 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       fence_after();
-      const int m = tm * BM + q * 32 + lane;
+      const int row0 = tm * BM + q * 32;
+      const int m = row0 + lane;
       const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        float v[32];
-        tmem_ld32(trow + (uint32_t)c, v);
-        if (g.alpha != 1.f) {
-#pragma unroll
-          for (int q2 = 0; q2 < 32; ++q2) v[q2] *= g.alpha;
-        }
+      for (int c = 0; c < BN; c += ccols, ++nchunk) {
         const int n0 = tn * BN + c;
-        if (m >= g.M || n0 >= g.N) continue;
-        if (g.mode == 2) {
-          float* cr = (float*)g.C + (size_t)m * g.N + n0;
+        uint8_t* sbuf = stage_out + (nchunk & 1) * (32 * 128);
+        if (lane == 0) bulk_wait_read1();   // the store that last used this buffer has read it
+        __syncwarp();
+        uint8_t* srow = sbuf + lane * 128;
+        // 32 columns at a time: f32 chunks are one half, bf16 chunks two (16-byte pieces 4h .. 4h+3)
+#pragma unroll 1
+        for (int h = 0; h < ccols / 32; ++h) {
+          const int nh = n0 + 32 * h;
+          float v[32];
+          tmem_ld32(trow + (uint32_t)(c + 32 * h), v);
+          if (g.alpha != 1.f) {
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (n0 + 4 * j >= g.N) break;
-            float4 x = reinterpret_cast<float4*>(cr)[j];
-            x.x += v[4 * j]; x.y += v[4 * j + 1]; x.z += v[4 * j + 2]; x.w += v[4 * j + 3];
-            reinterpret_cast<float4*>(cr)[j] = x;
+            for (int e = 0; e < 32; ++e) v[e] *= g.alpha;
           }
-        } else if (g.mode == 3) {
-          float* cr = (float*)g.C + slice + (size_t)m * g.N + n0;
+          if (f32out) {
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (n0 + 4 * j >= g.N) break;
-            reinterpret_cast<float4*>(cr)[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-          }
-        } else {
-          bf16* cr = (bf16*)g.C + (size_t)m * g.N + n0;
-          const bf16* rr = g.R ? g.R + (size_t)m * g.N + n0 : nullptr;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            if (n0 + 8 * j >= g.N) break;
-            float t[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) t[e] = v[8 * j + e];
+            for (int k = 0; k < 8; ++k) {
+              const uint4 u = make_uint4(__float_as_uint(v[4 * k]), __float_as_uint(v[4 * k + 1]),
+                                         __float_as_uint(v[4 * k + 2]), __float_as_uint(v[4 * k + 3]));
+              *reinterpret_cast<uint4*>(srow + ((k ^ (lane & 7)) << 4)) = u;
+            }
+          } else {
             if (g.bias) {
 #pragma unroll
-              for (int e = 0; e < 8; ++e) t[e] += g.bias[n0 + 8 * j + e];
+              for (int j = 0; j < 8; ++j) {
+                if (nh + 4 * j < g.N) {
+                  const float4 b4 = *reinterpret_cast<const float4*>(g.bias + nh + 4 * j);
+                  v[4 * j] += b4.x; v[4 * j + 1] += b4.y; v[4 * j + 2] += b4.z; v[4 * j + 3] += b4.w;
+                }
+              }
             }
-            if (rr) {
-              float r8[8];
-              Vec8<bf16>::load(rr + 8 * j, r8);
+            if (g.R && m < g.M) {
+              const bf16* rr = g.R + (size_t)m * g.N + nh;
 #pragma unroll
-              for (int e = 0; e < 8; ++e) t[e] += r8[e];
+              for (int j = 0; j < 4; ++j) {
+                if (nh + 8 * j < g.N) {
+                  float r8[8];
+                  Vec8<bf16>::load(rr + 8 * j, r8);
+#pragma unroll
+                  for (int e = 0; e < 8; ++e) v[8 * j + e] += r8[e];
+                }
+              }
             }
-            Vec8<bf16>::store(cr + 8 * j, t);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              __nv_bfloat162 hv[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) hv[e] = __floats2bfloat162_rn(v[8 * k + 2 * e], v[8 * k + 2 * e + 1]);
+              const int piece = 4 * h + k;
+              *reinterpret_cast<uint4*>(srow + ((piece ^ (lane & 7)) << 4)) = *reinterpret_cast<const uint4*>(hv);
+            }
           }
+        }
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          if (row0 < g.M && n0 < g.N) {
+            if (g.mode == 2) tma_reduce_add2d(&tcm, sbuf, n0, row0);
+            else if (g.mode == 3) tma_store3d(&tcm, sbuf, n0, row0, split);
+            else tma_store2d(&tcm, sbuf, n0, row0);
+          }
+          bulk_commit();
         }
       }
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
     }
+    if (lane == 0) bulk_wait_all();   // every store of this warp has landed in global memory
   }
 
   __syncthreads();
@@ -410,6 +467,21 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tensor map of C for the epilogue's TMA stores: bf16 [M, N] in boxes of 32 rows x 64 columns (modes
+// 0, 1), fp32 [M, N] in 32 x 32 (mode 2, reduce-add), fp32 [splits, M, N] in 1 x 32 x 32 (mode 3), all
+// in the 128-byte swizzle the epilogue writes its staging buffers in.
+bool make_map_c(CUtensorMap* m, const Args& a) {
+  const bool f32 = a.mode >= 2;
+  const uint64_t esz = f32 ? 4 : 2;
+  cuuint64_t dims[3] = {(cuuint64_t)a.N, (cuuint64_t)a.M, (cuuint64_t)a.splits};
+  cuuint64_t strides[2] = {(cuuint64_t)a.N * esz, (cuuint64_t)a.M * a.N * esz};
+  cuuint32_t box[3] = {f32 ? 32u : 64u, 32u, 1u};
+  cuuint32_t es[3] = {1, 1, 1};
+  return g_encode(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.mode == 3 ? 3 : 2,
+                  a.C, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int BN, bool A_MN, bool B_MN>
 bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int ctas_per_sm) {
   using C_ = Cfg<BN>;
@@ -424,11 +496,12 @@ bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int cta
                         : make_map(&ta, A, (uint64_t)a.K, (uint64_t)a.M, 64, BM);
   const bool okB = B_MN ? make_map(&tb, B, (uint64_t)a.N, (uint64_t)a.K, 64, 64)
                         : make_map(&tb, B, (uint64_t)a.K, (uint64_t)a.N, 64, BN);
-  if (!okA || !okB) return false;
+  CUtensorMap tcm;
+  if (!okA || !okB || !make_map_c(&tcm, a)) return false;
   const int units = a.tiles_m * a.tiles_n * a.splits;
   const int slots = g_sms * ctas_per_sm;
   const int grid = units < slots ? units : slots;
-  gemm_tc_k<BN, A_MN, B_MN><<<grid, kThreads, C_::SMEM, s>>>(ta, tb, a);
+  gemm_tc_k<BN, A_MN, B_MN><<<grid, kThreads, C_::SMEM, s>>>(ta, tb, tcm, a);
   return true;
 }
 
