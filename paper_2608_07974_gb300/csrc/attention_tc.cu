@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(NT) fwd_k(const bf16* __restrict__ qkv, bf16* 
   bf16* Qs = reinterpret_cast<bf16*>(smem);
   bf16* Ks = Qs + BR * HDP;            // [2]
   bf16* Vs = Ks + 2 * BR * HDP;        // [2]
-  const int qb = gridDim.x - 1 - blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int qb = gridDim.z - 1 - blockIdx.z, h = blockIdx.x, b = blockIdx.y;   // longest blocks launch first
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kvh = h / (H / Hkv), ld = (H + 2 * Hkv) * hd;
   const bool vec = (hd & 7) == 0;
@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, con
   bf16* Vs = Ks + 2 * BR * HDP;        // [2]
   float* Ls = reinterpret_cast<float*>(Vs + 2 * BR * HDP);
   float* Ds = Ls + BR;
-  const int qb = gridDim.x - 1 - blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int qb = gridDim.z - 1 - blockIdx.z, h = blockIdx.x, b = blockIdx.y;   // longest blocks launch first
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kvh = h / (H / Hkv), ld = (H + 2 * Hkv) * hd, HD = H * hd;
   const bool vec = (hd & 7) == 0;
@@ -399,12 +399,12 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
   bf16* dOs = Qs + 2 * BR * HDP;       // [2]
   float* Ls = reinterpret_cast<float*>(dOs + 2 * BR * HDP);   // [2][BR]
   float* Ds = Ls + 2 * BR;                                     // [2][BR]
-  const int kb = blockIdx.x, b = blockIdx.z;
+  const int kb = blockIdx.z, b = blockIdx.y;   // key block 0 (the longest) launches first
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ld = (H + 2 * Hkv) * hd, HD = H * hd;
-  const int kvh = part ? blockIdx.y / (H / Hkv) : blockIdx.y;
+  const int kvh = part ? blockIdx.x / (H / Hkv) : blockIdx.x;
   const int rep = part ? 1 : H / Hkv;                  // query heads this CTA loops over
-  const int h_first = part ? blockIdx.y : kvh * (H / Hkv);
+  const int h_first = part ? blockIdx.x : kvh * (H / Hkv);
   const bool vec = (hd & 7) == 0;
   const bf16* base = qkv + (size_t)b * S * ld;
   const int k0 = kb * BR;
@@ -532,7 +532,7 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
     const int key = k0 + lr0 + 8 * i;
     if (key >= S) continue;
     if (part) {
-      const size_t NS = (size_t)gridDim.z * S;
+      const size_t NS = (size_t)gridDim.y * S;
       float* pk = part + ((size_t)h_first * NS + (size_t)b * S + key) * hd;
       float* pv = pk + (size_t)H * NS * hd;
 #pragma unroll
@@ -567,7 +567,7 @@ void fwd_t(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv,
     cudaFuncSetAttribute(fwd_k<HDP>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     attr = true;
   }
-  dim3 grid((S + BR - 1) / BR, H, B);
+  dim3 grid(H, B, (S + BR - 1) / BR);
   fwd_k<HDP><<<grid, NT, smem, s>>>((const bf16*)qkv, (bf16*)out, lse, S, H, Hkv, hd, 1.f / sqrtf((float)hd));
 }
 
@@ -607,7 +607,7 @@ void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse,
     cudaFuncSetAttribute(bwd_dkv_k<HDP>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     attr = true;
   }
-  dim3 gq((S + BR - 1) / BR, H, B);
+  dim3 gq(H, B, (S + BR - 1) / BR);
   bwd_dq_k<HDP><<<gq, NT, smem, s>>>((const bf16*)qkv, (const bf16*)out, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H,
                                      Hkv, hd, scale);
   float* part = nullptr;
@@ -616,7 +616,7 @@ void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse,
     cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&part, bytes, pool, s) : cudaMallocAsync((void**)&part, bytes, s);
     if (e != cudaSuccess) { cudaGetLastError(); part = nullptr; }
   }
-  dim3 gk((S + BR - 1) / BR, part ? H : Hkv, B);
+  dim3 gk(part ? H : Hkv, B, (S + BR - 1) / BR);
   bwd_dkv_k<HDP><<<gk, NT, smem, s>>>((const bf16*)qkv, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, hd, scale,
                                       part);
   if (part) {

@@ -683,6 +683,7 @@ void check_bs(zl_ctx* c, int B, int S) {
   if (B <= 0 || S <= 0) raise_err(ZL_ERR_ARG, "empty micro-batch (B and S must be >= 1)");
   if (S > c->dims.max_seq) raise_err(ZL_ERR_ARG, "S exceeds max_seq");
   if ((long)B * S > (1L << 26)) raise_err(ZL_ERR_ARG, "B*S too large");
+  if (B > 65535) raise_err(ZL_ERR_ARG, "B above 65535");
 }
 
 // ----------------------------------------------------------------------------------------------
@@ -1572,8 +1573,8 @@ zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_
 }
 
 static bool attn_args_ok(int dtype, int B, int S, int H, int Hkv, int hd) {
-  return (dtype == 0 || dtype == 1) && B >= 1 && S >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0 && hd >= 2 &&
-         hd <= 128 && hd % 2 == 0;
+  return (dtype == 0 || dtype == 1) && B >= 1 && B <= 65535 && S >= 1 && (long)B * S <= (1L << 26) && H >= 1 &&
+         Hkv >= 1 && H % Hkv == 0 && hd >= 2 && hd <= 128 && hd % 2 == 0;
 }
 
 zl_status zl_op_attention(int dtype, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,

@@ -521,7 +521,7 @@ void choose(int mode, int M, int N, int K, int& bn_out, int& splits_out) {
   const int nk = (K + BK - 1) / BK;
   double best = 1e30;
   for (int bn : {256, 128, 64}) {
-    const double kb = mode == 2 ? (bn == 256 ? 0.60e-6 : bn == 128 ? 0.41e-6 : 0.44e-6)
+    const double kb = mode == 2 ? (bn == 256 ? 0.40e-6 : bn == 128 ? 0.30e-6 : 0.36e-6)
                                 : (bn == 256 ? 0.36e-6 : bn == 128 ? 0.29e-6 : 0.32e-6);
     const long tiles = (long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
     const int cps = bn == 64 ? 2 : 1;
