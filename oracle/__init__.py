@@ -17,10 +17,10 @@ mixture), Lemma 3 (stop-gradient block structure) and K=1, alpha=1 == BP.
 Parity unpinned: the convergence statements (Proposition 1, Theorem 1) need
 trained weights and data and are not checked.
 """
-from .model import (Oracle, OracleConfig, embed, layer_forward, chunk_forward, readout,
+from .model import (Oracle, OracleConfig, embed, layer_forward, chunk_forward, readout, adapter,
                     local_objective, local_objective_rows, rmsnorm, layernorm, rope,
                     attention, gelu_tanh, silu, kl_rows, adamw_update)
 
-__all__ = ["Oracle", "OracleConfig", "embed", "layer_forward", "chunk_forward", "readout",
+__all__ = ["Oracle", "OracleConfig", "embed", "layer_forward", "chunk_forward", "readout", "adapter",
            "local_objective", "local_objective_rows", "rmsnorm", "layernorm", "rope",
            "attention", "gelu_tanh", "silu", "kl_rows", "adamw_update"]

@@ -39,7 +39,8 @@ from typing import Dict, List, Optional, Sequence, Tuple
 
 import torch
 
-from synth import ARCH_GPT2, ARCH_LLAMA, LORA_TARGETS, ModelDims, layer_param_shapes, lora_param_shapes
+from synth import (ARCH_GPT2, ARCH_LLAMA, LORA_TARGETS, ModelDims, adapter_param_shapes, layer_param_shapes,
+                   lora_param_shapes)
 
 Tensor = torch.Tensor
 
@@ -169,6 +170,12 @@ def readout(P: Dict[str, Tensor], h: Tensor, d: ModelDims) -> Tensor:
     return n @ P["tok_emb"].T
 
 
+def adapter(P: Dict[str, Tensor], k: int, h: Tensor) -> Tensor:
+    """Readout adapter of chunk k (Section III-B, Local Update Interface, option (b)): a small residual
+    MLP before the frozen head, a_k(h) = h + GELU(h D_k^T) U_k^T, which is the identity while U_k = 0."""
+    return h + gelu_tanh(h @ P[f"adapters.{k}.down"].T) @ P[f"adapters.{k}.up"].T
+
+
 # ----------------------------------------------------------------------------------------
 # Local objective (Eq. 3-5)
 # ----------------------------------------------------------------------------------------
@@ -253,6 +260,7 @@ class OracleConfig:
     lr_gamma: float = 1.0
     lora_rank: int = 0              # 0: every layer tensor trainable; r > 0: only the LoRA factors
     lora_scale: float = 1.0         # Delta w = lora_scale * B A
+    adapter_dim: int = 0            # > 0: chunk k's own readout goes through its adapter a_k
 
     @property
     def K(self) -> int:
@@ -287,6 +295,8 @@ class Oracle:
         out = []
         for l in range(self.cfg.bounds[k - 1], self.cfg.bounds[k]):
             out += [f"layers.{l}.{s}" for s, _ in shapes]
+        if self.cfg.adapter_dim > 0:
+            out += [f"adapters.{k}.{s}" for s, _ in adapter_param_shapes(self.d, self.cfg.adapter_dim)]
         return out
 
     def trainable_names(self) -> List[str]:
@@ -310,6 +320,13 @@ class Oracle:
         with torch.no_grad():
             return readout(self.P, h.to(self.dtype), self.d)
 
+    def student_readout(self, P: Dict[str, Tensor], k: int, h: Tensor) -> Tensor:
+        """Chunk k's own readout z_k: through its adapter when adapters are on. The teacher p_{k-1} is
+        always the frozen head on h_{k-1} (chunk k builds it from its input hidden state alone)."""
+        if self.cfg.adapter_dim > 0:
+            h = adapter(P, k, h)
+        return readout(P, h, self.d)
+
     # -- one chunk's local objective and gradient -----------------------------------------
     def local_grad(self, k: int, h_prev: Tensor, labels: Tensor
                    ) -> Tuple[float, Dict[str, Tensor], Tensor]:
@@ -322,16 +339,18 @@ class Oracle:
         a = self.alpha_k(k)
         t = readout(self.P, h_in, self.d).detach() if a < 1.0 else None   # sg(p_{k-1})
         h = chunk_forward(P, self.cfg.bounds, k, h_in, self.d, self.cfg.lora_scale)
-        z = readout(P, h, self.d)
+        z = self.student_readout(P, k, h)
         L = local_objective(z, t, labels, a, self.cfg.kl_dir)
         grads = torch.autograd.grad(L, [leaves[n] for n in names])
         return float(L.detach()), dict(zip(names, grads)), h.detach()
 
-    def _apply_window(self, k: int) -> None:
+    def _apply_window(self, k: int, adapters: bool = True) -> None:
         c = self.cfg
         self.t[k] += 1
         lr = c.lr if c.lr_schedule == 0 else c.lr / math.sqrt(self.t[k] - 1 + c.lr_gamma)
         for n in self.chunk_names(k):
+            if not adapters and n.startswith("adapters."):
+                continue
             g = self.acc[n] / c.accum_m
             adamw_update(self.P[n], g, self.m[n], self.v[n], self.t[k], lr,
                          c.beta1, c.beta2, c.eps, c.weight_decay)
@@ -364,8 +383,9 @@ class Oracle:
 
     # -- backpropagation baseline and the global objective ------------------------------
     def bp_grad(self, ids: Tensor, labels: Tensor) -> Tuple[float, Dict[str, Tensor]]:
-        """Global CE of the last readout and its gradient through all chunks."""
-        names = self.trainable_names()
+        """Global CE of the last readout and its gradient through all chunks (no adapters: they only
+        serve the local objectives)."""
+        names = [n for n in self.trainable_names() if not n.startswith("adapters.")]
         leaves = {n: self.P[n].clone().requires_grad_(True) for n in names}
         P = dict(self.P)
         P.update(leaves)
@@ -384,7 +404,7 @@ class Oracle:
         for k in range(1, self.cfg.K + 1):
             self.micro[k] += 1
             if self.micro[k] == self.cfg.accum_m:
-                self._apply_window(k)
+                self._apply_window(k, adapters=False)
         return L
 
     def global_loss(self, ids: Tensor, labels: Tensor) -> float:

@@ -235,6 +235,29 @@ def make_lora_params(d: ModelDims, seed: int, rank: int, b_std: float = 0.0,
     return out
 
 
+def adapter_param_shapes(d: ModelDims, dim: int) -> List[Tuple[str, Tuple[int, ...]]]:
+    """Readout adapter of one chunk (residual bottleneck MLP a(h) = h + up(GELU(down(h)))):
+    down [dim, d_model], up [d_model, dim]."""
+    return [("down", (dim, d.d_model)), ("up", (d.d_model, dim))]
+
+
+def make_adapter_params(d: ModelDims, K: int, seed: int, dim: int, up_std: float = 0.0) -> Dict[str, torch.Tensor]:
+    """Adapters of chunks 1..K: down ~ N(0, 0.02^2); up = 0 (the adapter starts as the identity map)
+    unless up_std > 0 (tests use a non-zero up to exercise every gradient)."""
+    out = {}
+    for k in range(1, K + 1):
+        for s, shp in adapter_param_shapes(d, dim):
+            name = f"adapters.{k}.{s}"
+            n = shp[0] * shp[1]
+            if s == "down":
+                out[name] = normal(stream_key(seed, name), n, 0.02).to(torch.float32).view(shp)
+            elif up_std > 0:
+                out[name] = normal(stream_key(seed, name), n, up_std).to(torch.float32).view(shp)
+            else:
+                out[name] = torch.zeros(shp, dtype=torch.float32)
+    return out
+
+
 def frozen_param_shapes(d: ModelDims) -> List[Tuple[str, Tuple[int, ...]]]:
     """Frozen tensors: embedding (+ learned positions), final norm, LM head (GPT-2: tied to tok_emb)."""
     out = [("tok_emb", (d.vocab, d.d_model))]

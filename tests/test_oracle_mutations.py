@@ -96,3 +96,21 @@ def test_pins_catch_unscaled_lora(monkeypatch):
     monkeypatch.setattr(om, "lora_weight", lambda P, l, name, scale: orig(P, l, name, 1.0))
     with pytest.raises(AssertionError):
         pins.test_lora_zero_b_is_the_base_model_and_chain_rule()
+
+
+def test_pins_catch_adapter_without_residual(monkeypatch):
+    def bad_adapter(P, k, h):      # the residual connection dropped
+        return oracle.gelu_tanh(h @ P[f"adapters.{k}.down"].T) @ P[f"adapters.{k}.up"].T
+    _patch(monkeypatch, "adapter", bad_adapter)
+    with pytest.raises(AssertionError):
+        pins.test_adapter_gradient_matches_finite_differences(pins.LLAMA_T)
+
+
+def test_pins_catch_adapter_on_the_teacher(monkeypatch):
+    real = om.readout
+
+    def readout_through_adapter(P, h, d):   # an upstream chunk's adapter leaks into the teacher
+        return real(P, om.adapter(P, 1, h) if "adapters.1.down" in P else h, d)
+    _patch(monkeypatch, "readout", readout_through_adapter)
+    with pytest.raises(AssertionError):
+        pins.test_adapter_teacher_is_the_frozen_head_and_bp_ignores_adapters()

@@ -468,3 +468,104 @@ def test_lora_zero_b_is_the_base_model_and_chain_rule():
         A, Bm = lora.P[f"layers.0.{s}.lora_a"], lora.P[f"layers.0.{s}.lora_b"]
         assert torch.allclose(gl[f"layers.0.{s}.lora_b"], cfg.lora_scale * G @ A.T, atol=1e-12, rtol=1e-9)
         assert torch.allclose(gl[f"layers.0.{s}.lora_a"], cfg.lora_scale * Bm.T @ G, atol=1e-12, rtol=1e-9)
+
+
+# ---------------------------------------------------------------------------------------
+# Readout adapters (Section III-B, option (b)): a_k(h) = h + GELU(h D^T) U^T before the frozen head
+# ---------------------------------------------------------------------------------------
+
+def _adapter_setup(d, dim=4, up_std=0.3):
+    P = tiny_params(d)
+    A = synth.make_adapter_params(d, 2, 13, dim, up_std=up_std)
+    P.update({n: t * 15.0 if n.endswith("down") else t for n, t in A.items()})
+    return P, OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5, adapter_dim=dim)
+
+
+def _library_adapter(P, k, h):
+    """The adapter written with torch.nn.functional's linear and tanh-GELU."""
+    F = torch.nn.functional
+    return h + F.linear(F.gelu(F.linear(h, P[f"adapters.{k}.down"]), approximate="tanh"), P[f"adapters.{k}.up"])
+
+
+@pytest.mark.parametrize("d", [LLAMA_T, GPT2_T], ids=["llama", "gpt2"])
+def test_adapter_gradient_matches_finite_differences(d):
+    """L_k with chunk k's adapter on its own readout, the teacher the frozen head on h_{k-1}: autograd
+    gradients of every chunk tensor (layers and adapter) against central differences of the loss
+    composed from library routines."""
+    P, cfg = _adapter_setup(d)
+    ids, labels = tiny_batch(d)
+    orc = Oracle(cfg, P)
+    h = orc.embed(ids)
+    gen = torch.Generator().manual_seed(9)
+    for k in (1, 2):
+        L, grads, h_next = orc.local_grad(k, h, labels)
+        assert {n for n in grads if n.startswith("adapters.")} == {f"adapters.{k}.down", f"adapters.{k}.up"}
+
+        def Lk(Pp):
+            t = oracle.readout(Pp, h, d)
+            hk = oracle.chunk_forward(Pp, cfg.bounds, k, h, d)
+            z = oracle.readout(Pp, _library_adapter(Pp, k, hk), d)
+            return float(oracle.local_objective(z, t, labels, 0.5))
+
+        assert abs(Lk(orc.P) - L) < 1e-12
+        for name, g in grads.items():
+            flat = orc.P[name].view(-1)
+            for idx in torch.randint(0, flat.numel(), (3,), generator=gen).tolist():
+                old = float(flat[idx])
+                flat[idx] = old + 1e-6
+                lp = Lk(orc.P)
+                flat[idx] = old - 1e-6
+                lm = Lk(orc.P)
+                flat[idx] = old
+                fd = (lp - lm) / 2e-6
+                assert abs(fd - float(g.view(-1)[idx])) <= 1e-7 + 1e-6 * abs(fd), (name, idx)
+        h = h_next
+
+
+def test_adapter_zero_up_is_identity_and_chain_rule():
+    """U = 0: the loss and every layer gradient equal the static-head ones exactly, dL/dD = 0, and
+    dL/dU = G^T GELU(h_k D^T) with G = dL/dh_k of the static-head objective (chain rule)."""
+    d = GPT2_T
+    P, cfg = _adapter_setup(d, up_std=0.0)
+    ids, labels = tiny_batch(d)
+    static = Oracle(OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5),
+                    {n: t for n, t in P.items() if not n.startswith("adapters.")})
+    ad = Oracle(cfg, P)
+    h0 = static.embed(ids)
+    Ls, gs, h1 = static.local_grad(1, h0, labels)
+    La, ga, _ = ad.local_grad(1, h0, labels)
+    assert La == Ls
+    for n, g in gs.items():
+        assert torch.equal(ga[n], g), n
+    assert torch.count_nonzero(ga["adapters.1.down"]) == 0
+    hk = h1.clone().requires_grad_(True)
+    t = oracle.readout(static.P, h0, d)
+    G, = torch.autograd.grad(oracle.local_objective(oracle.readout(static.P, hk, d), t, labels, 0.5), hk)
+    act = oracle.gelu_tanh(h1 @ ad.P["adapters.1.down"].T)
+    ref = torch.einsum("bsd,bsr->dr", G, act)
+    assert torch.allclose(ga["adapters.1.up"], ref, atol=1e-13, rtol=1e-10)
+
+
+def test_adapter_teacher_is_the_frozen_head_and_bp_ignores_adapters():
+    """Chunk 2's loss, with h_1 fixed, does not depend on chunk 1's adapter (its teacher is the frozen
+    head on h_1); the global objective and the backpropagation step leave every adapter untouched."""
+    d = LLAMA_T
+    P, cfg = _adapter_setup(d)
+    ids, labels = tiny_batch(d)
+    orc = Oracle(cfg, P)
+    h1 = orc.forward_chunk(1, orc.embed(ids))
+    L2, _, _ = orc.local_grad(2, h1, labels)
+    orc.P["adapters.1.down"].mul_(3.0)
+    orc.P["adapters.1.up"].add_(0.5)
+    assert orc.local_grad(2, h1, labels)[0] == L2
+    base = Oracle(OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5),
+                  {n: t for n, t in P.items() if not n.startswith("adapters.")})
+    bp = Oracle(cfg, P)
+    assert bp.global_loss(ids, labels) == base.global_loss(ids, labels)
+    before = {n: t.clone() for n, t in bp.P.items() if n.startswith("adapters.")}
+    bp.bp_step(ids, labels)
+    base.bp_step(ids, labels)
+    for n, t in before.items():
+        assert torch.equal(bp.P[n], t), n
+    for n, t in base.P.items():
+        assert torch.equal(bp.P[n], t), n
