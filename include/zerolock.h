@@ -78,6 +78,9 @@ typedef struct {
   int lora_rank;            /* 0: full fine-tune; r > 0: LoRA (Section II-A) on the QKV, output and FFN  */
   float lora_scale;         /*   linears, w + lora_scale * B A, only A [r, in] and B [out, r] trainable  */
   int replay_depth;         /* D >= 0: zl_step keeps each chunk's last D inputs for zl_replay          */
+  int adapter_dim;          /* 0: static readout head; r > 0 (a multiple of 16): chunk k's own readout  */
+                            /*   goes through its adapter a_k(h) = h + GELU(h D_k^T) U_k^T (Section     */
+                            /*   III-B, local update interface (b)), D_k [r, d], U_k [d, r] trainable   */
 } zl_train_cfg;
 
 /* Create a context: parameters, AdamW state, K streams and events, a stream-ordered
@@ -100,7 +103,10 @@ zl_status zl_set_stream(zl_ctx* ctx, void* stream);
  * norm_f.bias [d] (GPT-2), lm_head [V,d] (Llama), and per layer l
  * layers.{l}.{attn_norm.weight, attn_norm.bias, wqkv, bqkv, wo, bo, ffn_norm.weight,
  * ffn_norm.bias, w1, b1, w2, b2} (biases: GPT-2 only); weights are [out, in] row-major. With
- * lora_rank r > 0 also layers.{l}.{wqkv, wo, w1, w2}.{lora_a [r, in], lora_b [out, r]}.
+ * lora_rank r > 0 also layers.{l}.{wqkv, wo, w1, w2}.{lora_a [r, in], lora_b [out, r]}. With
+ * adapter_dim r > 0 also adapters.{k}.down [r, d] and adapters.{k}.up [d, r], k = 1..K (up starts
+ * at zero: the adapter is the identity until it trains). The teacher p_{k-1} of chunk k stays the
+ * frozen head on h_{k-1}; the backpropagation step and the global loss use no adapter.
  * zl_set_param copies `bytes` = numel * 4 of fp32 values from src (device memory if
  * on_device, else host) into the master copy (and the compute copy). */
 zl_status zl_set_param(zl_ctx* ctx, const char* name, const void* src, size_t bytes, int on_device);

@@ -94,6 +94,8 @@ struct Chunk {
   void* fmat = nullptr;    // frozen base matrices in LoRA mode (compute dtype)
   size_t fvec_n = 0, fmat_n = 0;
   std::vector<Layer> layers;
+  size_t ad_down = 0, ad_up = 0;   // readout adapter D [r, d] and U [d, r] in the trainable slab
+  size_t n_layers_slab = 0;        // trainable floats before the adapter (what backpropagation updates)
   int micro = 0;
   long t = 0;
   long done = 0;             // micro-batches this chunk has processed (progress metadata)
@@ -206,7 +208,7 @@ float* Gm(Chunk& k, int li, PK p) {   // gradient accumulator; NULL for frozen t
 }
 int lora_r16(int r) { return r > 0 ? (r + 15) / 16 * 16 : 0; }
 
-const void* LoraC(zl_ctx* c, Chunk& k, size_t off) {
+const void* TrainC(zl_ctx* c, Chunk& k, size_t off) {
   return c->dt == BF16 ? (const void*)((const bf16*)k.comp + off) : (const void*)(k.master + off);
 }
 
@@ -331,8 +333,8 @@ void lora_fwd(zl_ctx* c, Chunk& k, int li, int i, const void* X, void* out, void
   const int r = lora_r16(c->cfg.lora_rank);
   if (r <= 0) return;
   const Layer& L = k.layers[li];
-  G(c, s, 0, N, r, L.lin_in[i], X, LoraC(c, k, L.la[i]), u, nullptr, nullptr);
-  G(c, s, 1, N, L.lin_out[i], r, u, LoraC(c, k, L.lb[i]), out, nullptr, out, c->cfg.lora_scale);
+  G(c, s, 0, N, r, L.lin_in[i], X, TrainC(c, k, L.la[i]), u, nullptr, nullptr);
+  G(c, s, 1, N, L.lin_out[i], r, u, TrainC(c, k, L.lb[i]), out, nullptr, out, c->cfg.lora_scale);
 }
 
 // LoRA backward of linear i, after dX holds dY W: du = s dY B; d(B^T) += s u^T dY; dA += du^T X;
@@ -343,10 +345,10 @@ void lora_bwd(zl_ctx* c, Chunk& k, int li, int i, const void* X, const void* u, 
   if (r <= 0) return;
   const Layer& L = k.layers[li];
   const float sc = c->cfg.lora_scale;
-  G(c, s, 0, N, r, L.lin_out[i], dY, LoraC(c, k, L.lb[i]), du, nullptr, nullptr, sc);
+  G(c, s, 0, N, r, L.lin_out[i], dY, TrainC(c, k, L.lb[i]), du, nullptr, nullptr, sc);
   G(c, s, 2, r, L.lin_out[i], N, u, dY, k.grad + L.lb[i], nullptr, nullptr, sc);
   G(c, s, 2, r, L.lin_in[i], N, du, X, k.grad + L.la[i], nullptr, nullptr);
-  G(c, s, 1, N, L.lin_in[i], r, du, LoraC(c, k, L.la[i]), dX, nullptr, dX);
+  G(c, s, 1, N, L.lin_in[i], r, du, TrainC(c, k, L.la[i]), dX, nullptr, dX);
 }
 
 void layer_fwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* x, void* y, int B, int S, cudaStream_t s) {
@@ -542,7 +544,8 @@ void chunk_bwd(zl_ctx* c, Chunk& k, ChunkActs& acts, const void* dh, void* dh_in
   pfree(a.base, s);
 }
 
-void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s) {
+// adapters = false (the backpropagation step): the readout adapter, at the end of the slab, is left as is.
+void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s, bool adapters = true) {
   k.micro += 1;
   if (k.micro < c->cfg.accum_m) return;
   k.t += 1;
@@ -551,8 +554,11 @@ void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s) {
   if (g.lr_schedule == 1) lr = g.lr / std::sqrt((double)(k.t - 1) + g.lr_gamma);
   const double bc1 = 1.0 - std::pow((double)g.beta1, (double)k.t);
   const double bc2 = 1.0 - std::pow((double)g.beta2, (double)k.t);
-  ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * (double)k.n);
-  launch_adamw(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, k.n, (float)lr, g.beta1, g.beta2, g.eps,
+  const size_t n = (adapters || g.adapter_dim == 0) ? k.n : k.n_layers_slab;
+  k.micro = 0;
+  if (n == 0) return;
+  ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * (double)n);
+  launch_adamw(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, n, (float)lr, g.beta1, g.beta2, g.eps,
                g.weight_decay, (float)bc1, (float)bc2, 1.f / (float)g.accum_m, s);
   CHECK_LAUNCH();
   k.micro = 0;
@@ -589,29 +595,81 @@ void ring_put(zl_ctx* c, Chunk& ck, long seq, const void* h_in, const int32_t* l
 struct ReadoutSave {
   void* n = nullptr;
   float *rstd = nullptr, *mean = nullptr;
+  void *a = nullptr, *u = nullptr;   // adapter: a_k(h) and h D^T
 };
 
-void readout_fwd(zl_ctx* c, const void* h, void* z, ReadoutSave* keep, int N, cudaStream_t s) {
+// z = Norm_f(x) W_lm^T with x = h, or x = a_k(h) = h + GELU(h D^T) U^T when `ad` (chunk k's readout
+// adapter, Section III-B (b)) is given.
+void readout_fwd(zl_ctx* c, const void* h, void* z, ReadoutSave* keep, int N, cudaStream_t s,
+                 Chunk* ad = nullptr) {
   const size_t e = esz(c);
+  const void* x = h;
+  void *a = nullptr, *u = nullptr;
+  if (ad && c->cfg.adapter_dim > 0) {
+    const int ra = c->cfg.adapter_dim;
+    u = palloc(c, (size_t)N * ra * e, s);
+    void* gact = palloc(c, (size_t)N * ra * e, s);
+    a = palloc(c, (size_t)N * c->d * e, s);
+    G(c, s, 0, N, ra, c->d, h, TrainC(c, *ad, ad->ad_down), u, nullptr, nullptr);
+    {
+      ProfScope p(c, s, PC_ELEM, 0, 2.0 * e * (double)N * ra);
+      launch_gelu_fwd(c->dt, u, gact, (size_t)N * ra, s);
+    }
+    G(c, s, 0, N, c->d, ra, gact, TrainC(c, *ad, ad->ad_up), a, nullptr, h);
+    pfree(gact, s);
+    x = a;
+  }
   void* n = palloc(c, (size_t)N * c->d * e, s);
   float* st = (float*)palloc(c, (size_t)N * 8, s);
-  NF(c, s, h, c->normf_w, c->normf_b, n, st, st + N, N);
+  NF(c, s, x, c->normf_w, c->normf_b, n, st, st + N, N);
   G(c, s, 0, N, c->Vp, c->d, n, c->lm_head, z, nullptr, nullptr);
   CHECK_LAUNCH();
   if (keep) {
     keep->n = n;
     keep->rstd = st;
     keep->mean = st + N;
+    keep->a = a;
+    keep->u = u;
   } else {
     pfree(n, s);
     pfree(st, s);
+    pfree(a, s);
+    pfree(u, s);
   }
 }
 
-// dh = Norm_f'(h)^T (dz W_lm)
-void readout_bwd(zl_ctx* c, const void* h, ReadoutSave& rs, const void* dz, void* dh, int N, cudaStream_t s) {
+// dh = d/dh of the readout: Norm_f'(x)^T (dz W_lm), through the adapter when it was applied:
+// da = Norm_f'(a)^T dn;  dU += da^T GELU(u);  du = (da U) * GELU'(u);  dD += du^T h;  dh = da + du D.
+void readout_bwd(zl_ctx* c, const void* h, ReadoutSave& rs, const void* dz, void* dh, int N, cudaStream_t s,
+                 Chunk* ad = nullptr) {
   G(c, s, 1, N, c->d, c->Vp, dz, c->lm_head, rs.n, nullptr, nullptr);   // reuse n as dn
-  NBX(c, s, h, c->normf_w, rs.rstd, rs.mean, rs.n, nullptr, dh, N);
+  if (!rs.a) {
+    NBX(c, s, h, c->normf_w, rs.rstd, rs.mean, rs.n, nullptr, dh, N);
+  } else {
+    const int ra = c->cfg.adapter_dim;
+    const size_t e = esz(c);
+    void* da = palloc(c, (size_t)N * c->d * e, s);
+    void* gact = palloc(c, (size_t)N * ra * e, s);
+    void* dg = palloc(c, (size_t)N * ra * e, s);
+    NBX(c, s, rs.a, c->normf_w, rs.rstd, rs.mean, rs.n, nullptr, da, N);
+    {
+      ProfScope p(c, s, PC_ELEM, 0, 2.0 * e * (double)N * ra);
+      launch_gelu_fwd(c->dt, rs.u, gact, (size_t)N * ra, s);
+    }
+    G(c, s, 2, c->d, ra, N, da, gact, ad->grad + ad->ad_up, nullptr, nullptr);
+    G(c, s, 1, N, ra, c->d, da, TrainC(c, *ad, ad->ad_up), dg, nullptr, nullptr);
+    {
+      ProfScope p(c, s, PC_ELEM, 0, 3.0 * e * (double)N * ra);
+      launch_gelu_bwd(c->dt, rs.u, dg, gact, (size_t)N * ra, s);   // gact now holds du
+    }
+    G(c, s, 2, ra, c->d, N, gact, h, ad->grad + ad->ad_down, nullptr, nullptr);
+    G(c, s, 1, N, c->d, ra, gact, TrainC(c, *ad, ad->ad_down), dh, nullptr, da);
+    pfree(da, s);
+    pfree(gact, s);
+    pfree(dg, s);
+    pfree(rs.a, s);
+    pfree(rs.u, s);
+  }
   CHECK_LAUNCH();
   pfree(rs.n, s);
   pfree(rs.rstd, s);
@@ -709,6 +767,19 @@ bool lookup(zl_ctx* c, const std::string& name, Found& f) {
   if (name == "norm_f.weight") { f = Found{c->normf_w, true, (size_t)c->d, nullptr, 0, 3}; return true; }
   if (name == "norm_f.bias" && !c->llama) { f = Found{c->normf_b, true, (size_t)c->d, nullptr, 0, 4}; return true; }
   if (name == "lm_head" && c->llama) { f = Found{c->lm_head, c->dt == F32, Vd, nullptr, 0, 5}; return true; }
+  if (name.rfind("adapters.", 0) == 0 && c->cfg.adapter_dim > 0) {
+    const size_t dot = name.find('.', 9);
+    if (dot == std::string::npos) return false;
+    int k = -1;
+    try { k = std::stoi(name.substr(9, dot - 9)); } catch (...) { return false; }
+    if (k < 1 || k > c->K || name.substr(9, dot - 9) != std::to_string(k)) return false;
+    Chunk& ck = c->ch[k];
+    const std::string suf = name.substr(dot + 1);
+    const size_t n = (size_t)c->cfg.adapter_dim * c->d;
+    if (suf == "down") { f = Found{ck.master + ck.ad_down, true, n, &ck, ck.ad_down, 0}; return true; }
+    if (suf == "up") { f = Found{ck.master + ck.ad_up, true, n, &ck, ck.ad_up, 0}; return true; }
+    return false;
+  }
   if (name.rfind("layers.", 0) != 0) return false;
   const size_t dot = name.find('.', 7);
   if (dot == std::string::npos) return false;
@@ -814,6 +885,8 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (D.arch == ZL_ARCH_GPT2 && D.n_kv_heads != D.n_heads) why = "GPT-2 blocks use n_kv_heads == n_heads";
   else if (D.d_model % 8 != 0 || D.d_ff % 8 != 0) why = "d_model and d_ff must be multiples of 8";
   else if (D.d_model > 16384) why = "d_model above 16384 is not supported";
+  else if (cfg->adapter_dim < 0 || cfg->adapter_dim % 16 != 0 || cfg->adapter_dim > D.d_model)
+    why = "adapter_dim must be 0 or a multiple of 16 up to d_model";
   else if (!(D.norm_eps > 0.f)) why = "norm_eps";
   else if (K < 1 || K > D.n_layers) why = "K must be in [1, n_layers]";
   else if (bounds[0] != 0 || bounds[K] != D.n_layers) why = "bounds[0] must be 0 and bounds[K] n_layers";
@@ -933,6 +1006,14 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
           }
         }
         ck.layers.push_back(L);
+      }
+      ck.n_layers_slab = off;
+      if (cfg->adapter_dim > 0) {
+        const size_t ra = (size_t)cfg->adapter_dim;
+        ck.ad_down = off;
+        off += round_up(ra * d, 64);
+        ck.ad_up = off;
+        off += round_up((size_t)d * ra, 64);
       }
       ck.n = std::max<size_t>(off, 64);
       ck.fvec_n = fvec;
@@ -1143,12 +1224,13 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
   if (h_out) CK(cudaMemcpyAsync(h_out, hk, hb, cudaMemcpyDeviceToDevice, s));
   void* z = palloc(c, zb, s);
   ReadoutSave rs;
-  readout_fwd(c, hk, z, &rs, N, s);
+  Chunk* ad = c->cfg.adapter_dim > 0 ? &ck : nullptr;
+  readout_fwd(c, hk, z, &rs, N, s, ad);
   void* dz = local_loss(c, z, t, labels, a, N, k, s);
   pfree(z, s);
   pfree(t, s);
   void* dh = palloc(c, hb, s);
-  readout_bwd(c, hk, rs, dz, dh, N, s);
+  readout_bwd(c, hk, rs, dz, dh, N, s, ad);
   pfree(dz, s);
   chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
   pfree(dh, s);
@@ -1297,6 +1379,7 @@ zl_status zl_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
     }
     rec(ev_h0, c->aux);      // z_0 ready (and aux done reading h_0)
     const int cap = (int)c->live_ring.size();
+    const bool adp = c->cfg.adapter_dim > 0;
     for (int k = 1; k <= K; ++k) {
       Chunk& ck = c->ch[k];
       cudaStream_t s = ck.s;
@@ -1314,27 +1397,38 @@ zl_status zl_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
       rec(ck.ev_h, s);
       z[k] = palloc(c, zb, s);
       ReadoutSave rs;
-      readout_fwd(c, h[k], z[k], &rs, N, s);
+      readout_fwd(c, h[k], z[k], &rs, N, s, adp ? &ck : nullptr);
       rec(ck.ev_z, s);
-      // S3: local objective against the stop-gradient teacher z_{k-1}
+      // S3: local objective against the stop-gradient teacher: the frozen head on h_{k-1}, which is
+      // chunk k-1's own readout z_{k-1} (reused) unless chunk k-1 read out through its adapter
       void* teacher = nullptr;
+      void* own_t = nullptr;
       if (a < 1.f) {
-        if (k == 1) wait_ev(s, ev_h0);
-        else wait_ev(s, c->ch[k - 1].ev_z);
-        teacher = z[k - 1];
+        if (k == 1) {
+          wait_ev(s, ev_h0);
+          teacher = z[0];
+        } else if (adp) {
+          own_t = palloc(c, zb, s);
+          readout_fwd(c, h[k - 1], own_t, nullptr, N, s);
+          teacher = own_t;
+        } else {
+          wait_ev(s, c->ch[k - 1].ev_z);
+          teacher = z[k - 1];
+        }
       }
       void* dz = local_loss(c, z[k], teacher, labels, a, N, k, s);
       rec(ck.ev_loss, s);
+      pfree(own_t, s);
       // z_{k-1} is no longer needed once this loss and chunk k-1's own loss are done
       if (k == 1) {
         if (z[0]) { wait_ev(s, ev_h0); pfree(z[0], s); }
-      } else {
+      } else if (!adp) {
         wait_ev(s, c->ch[k - 1].ev_loss);
         pfree(z[k - 1], s);
       }
-      if (k == K) pfree(z[K], s);
+      if (k == K || adp) pfree(z[k], s);   // with adapters no later chunk reads z_k
       void* dh = palloc(c, hb, s);
-      readout_bwd(c, h[k], rs, dz, dh, N, s);
+      readout_bwd(c, h[k], rs, dz, dh, N, s, adp ? &ck : nullptr);
       pfree(dz, s);
       rec(ck.ev_hb, s);
       chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
@@ -1406,7 +1500,7 @@ zl_status zl_bp_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B
         rec(c->ch[1].ev_done, s);
         wait_ev(c->ch[k].s, c->ch[1].ev_done);
       }
-      adamw_window(c, c->ch[k], k == 1 ? s : c->ch[k].s);
+      adamw_window(c, c->ch[k], k == 1 ? s : c->ch[k].s, false);
     }
     c->last_nloss = 1;
     for (int k = 1; k <= K; ++k) c->ch[k].done += 1;
