@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--K", type=int, default=0, help="chunk count (default: the workload's)")
     ap.add_argument("--max-live", type=int, default=2, help="chunks whose activations may be alive at once")
     ap.add_argument("--lora", type=int, default=0, help="LoRA rank (0: full fine-tune); scale 16 / rank")
+    ap.add_argument("--adapter", type=int, default=0,
+                    help="readout adapter width per chunk (0: static head; a multiple of 16)")
     ap.add_argument("--no-bp", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -95,8 +97,8 @@ def roofline_of(prof):
 TRAFFIC = {
     # ncu dram__bytes_read.sum + dram__bytes_write.sum of the GPT-2 GEMM shapes (microbench gemm),
     # averaged with the per-step launch mix: 12 layer GEMMs per layer; 5 head forwards, 4 head dX
-    "gemm_layer": {"source": "gemm_tc.cu", "sha256": "fe8bf38df965d0c2", "bytes_per_launch": 22315200.0},
-    "gemm_head": {"source": "gemm_tc.cu", "sha256": "fe8bf38df965d0c2", "bytes_per_launch": 642291882.7},
+    "gemm_layer": {"source": "gemm_tc.cu", "sha256": "8f86aa41f702a435", "bytes_per_launch": 22309760.0},
+    "gemm_head": {"source": "gemm_tc.cu", "sha256": "8f86aa41f702a435", "bytes_per_launch": 642934072.9},
 }
 
 
@@ -117,13 +119,13 @@ def rank_batch_ids(rank: int, n: int):
     return [1000 * rank + i for i in range(n)]
 
 
-def workload_desc(w, K, lora=0):
+def workload_desc(w, K, lora=0, adapter=0):
     d = w.dims
     arch = "llama" if d.arch == synth.ARCH_LLAMA else "gpt2"
     tune = f"LoRA rank {lora} scale {16 / lora:g} on QKV/O/FFN" if lora else "full fine-tune"
     return (f"{w.name}: {arch}-style decoder, {d.n_layers} layers, d_model {d.d_model}, {d.n_heads} heads "
             f"({d.n_kv_heads} kv), ffn {d.d_ff}, vocab {d.vocab}, micro-batch {w.batch} x seq {w.seq}, "
-            f"K={K} chunks, alpha {w.alpha}, AdamW, {tune}")
+            f"K={K} chunks, alpha {w.alpha}, AdamW, {tune}" + (f", readout adapters of width {adapter}" if adapter else ""))
 
 
 def peaks():
@@ -254,11 +256,14 @@ def run_ours(args):
     params = synth.make_params(w.dims, w.seed)
     if args.lora:
         params.update(synth.make_lora_params(w.dims, w.seed, args.lora))
+    if args.adapter:
+        params.update(synth.make_adapter_params(w.dims, K, w.seed, args.adapter))
 
     def make_engine(max_live, serialize=False):
         e = zb.ZeroLock(w.dims, K, bounds, dtype=w.dtype, alpha=w.alpha, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
                         eps=w.eps, weight_decay=w.weight_decay, max_live_chunks=max_live, serialize=serialize,
-                        lora_rank=args.lora, lora_scale=16.0 / args.lora if args.lora else 1.0)
+                        lora_rank=args.lora, lora_scale=16.0 / args.lora if args.lora else 1.0,
+                        adapter_dim=args.adapter)
         e.load(params)
         return e
 
@@ -378,7 +383,7 @@ def run_ours(args):
 
     # ---- CPU oracle on a bounded sample (rank 0, one GPU only) --------------------------------
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu and not args.lora:
+    if rank == 0 and world == 1 and not args.no_cpu and not args.lora and not args.adapter:
         times, tok, cores = oracle_sample(w, K, params, 2)
         cpu = {"value": tok / times[-1], "unit": "tokens/s", "cores": cores, "kind": "oracle",
                "sample": f"one local step of chunk 2 on 1 x {w.seq} tokens (fp32 oracle, after one warm-up sample); "
@@ -388,7 +393,7 @@ def run_ours(args):
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-                "config": {"workload": workload_desc(w, K, args.lora), "K": K, "bounds": bounds,
+                "config": {"workload": workload_desc(w, K, args.lora, args.adapter), "K": K, "bounds": bounds,
                            "global_batch": w.batch * world, "seq_len": w.seq, "max_live_chunks": args.max_live,
                            "parallelism": f"replicas x{world}" if world > 1 else "single GPU, K streams",
                            "l2": "no flush: every step's working set (weights, AdamW state, logits) exceeds L2"},
