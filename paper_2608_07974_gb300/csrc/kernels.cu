@@ -682,14 +682,16 @@ __device__ __forceinline__ Lse3 warp_merge(Lse3 v) {
 }
 
 
-// Online base-2 log-sum-exp of 8 values already scaled by log2(e) (xs), optionally with the cross
-// term sum 2^(xs - m) * w. nvalid < 8 only for the last, partial vector of a row.
+// Online base-2 log-sum-exp of 8 raw logits x (the running max A.m is kept in log2 units, x * log2 e),
+// optionally with the cross term sum 2^(x log2 e - m) * w. nvalid < 8 only for the last, partial
+// vector of a row. The scale by log2 e is folded into the exponent's FMA.
 template <bool FULL>
-__device__ __forceinline__ void lse_add8(Lse3& A, const float* xs, const float* w, int nvalid) {
+__device__ __forceinline__ void lse_add8(Lse3& A, const float* x, const float* w, int nvalid) {
   float mx = -INFINITY;
 #pragma unroll
   for (int i = 0; i < 8; ++i)
-    if (FULL || i < nvalid) mx = fmaxf(mx, xs[i]);
+    if (FULL || i < nvalid) mx = fmaxf(mx, x[i]);
+  mx *= kL2e;
   if (mx > A.m) {
     const float sc = ex2(A.m - mx);
     A.s *= sc;
@@ -699,7 +701,7 @@ __device__ __forceinline__ void lse_add8(Lse3& A, const float* xs, const float* 
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     if (FULL || i < nvalid) {
-      const float e = ex2(xs[i] - A.m);
+      const float e = ex2(fmaf(x[i], kL2e, -A.m));
       A.s += e;
       if (w) A.a = fmaf(e, w[i], A.a);
     }
@@ -710,15 +712,10 @@ template <typename T, bool TEACHER, int KLDIR, bool FULL>
 __device__ __forceinline__ void loss_pass1_vec(const T* zp, const T* tp, Lse3& Z, Lse3& Q, int nv) {
   float zs[8], ts[8], w[8];
   Vec8<T>::load(zp, zs);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) zs[i] *= kL2e;
   if (TEACHER) {
     Vec8<T>::load(tp, ts);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      ts[i] *= kL2e;
-      w[i] = KLDIR == 0 ? zs[i] - ts[i] : ts[i] - zs[i];   // in log2 units; scaled by ln 2 at the end
-    }
+    for (int i = 0; i < 8; ++i) w[i] = KLDIR == 0 ? zs[i] - ts[i] : ts[i] - zs[i];   // natural units
     lse_add8<FULL>(Z, zs, KLDIR == 0 ? w : nullptr, nv);
     lse_add8<FULL>(Q, ts, KLDIR == 0 ? nullptr : w, nv);
   } else {
@@ -769,7 +766,7 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
     float lse_t = 0.f, kl = 0.f;
     if (TEACHER) {
       lse_t = (b.m + log2f(b.s)) * kLn2;
-      kl = KLDIR == 0 ? a.a / a.s * kLn2 - lse_z + lse_t : b.a / b.s * kLn2 - lse_t + lse_z;
+      kl = KLDIR == 0 ? a.a / a.s - lse_z + lse_t : b.a / b.s - lse_t + lse_z;
     }
     row_loss[row] = alpha * (lse_z - to_f(zr[y])) + (TEACHER ? (1.f - alpha) * kl : 0.f);
     sh_stats[0] = lse_z;
@@ -782,6 +779,8 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
   const int cnt = *count;
   const float inv_n = cnt > 0 ? 1.f / (float)cnt : 0.f;
   const float wt = inv_n * alpha, wc = inv_n * (1.f - alpha);
+  //   kl_dir 0: dz = p (wt + wc ((z - t) - shift));  kl_dir 1: dz = (wt + wc) p - wc q;  no teacher: wt p
+  const float k0 = wt - wc * shift, wtc = wt + wc;
   for (c = threadIdx.x * 8; c < ldz; c += step) {
     float fz[8], ft[8], o[8];
     Vec8<T>::load(zr + c, fz);
@@ -789,12 +788,9 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const float p = ex2(fmaf(fz[i], kL2e, -lz2));
-      float g = wt * p;
-      if (TEACHER) {
-        const float gc = KLDIR == 0 ? p * ((fz[i] - ft[i]) - shift) : p - ex2(fmaf(ft[i], kL2e, -lt2));
-        g = fmaf(wc, gc, g);
-      }
-      o[i] = g;
+      if (!TEACHER) o[i] = wt * p;
+      else if (KLDIR == 0) o[i] = p * fmaf(wc, fz[i] - ft[i], k0);
+      else o[i] = fmaf(wtc, p, -wc * ex2(fmaf(ft[i], kL2e, -lt2)));
     }
     if (y >= c && y < c + 8) o[y - c] -= wt;   // the one-hot of the task term
     if (c + 8 > V) {
