@@ -196,6 +196,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   fence_after();
   const uint32_t tmem = *tbase;
+  // Programmatic dependent launch: the set-up above may overlap the previous kernel of the stream;
+  // every thread waits for that kernel (and its memory) before touching global memory, and lets the
+  // next GEMM of the stream begin its own set-up.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int nk = (g.K + BK - 1) / BK;
   const int num_tiles = g.tiles_m * g.tiles_n;
   const int num_units = num_tiles * g.splits;
@@ -501,8 +506,17 @@ bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int cta
   const int units = a.tiles_m * a.tiles_n * a.splits;
   const int slots = g_sms * ctas_per_sm;
   const int grid = units < slots ? units : slots;
-  gemm_tc_k<BN, A_MN, B_MN><<<grid, kThreads, C_::SMEM, s>>>(ta, tb, tcm, a);
-  return true;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3((unsigned)kThreads);
+  cfg.dynamicSmemBytes = C_::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, tcm, a) == cudaSuccess;
 }
 
 template <bool A_MN, bool B_MN>
