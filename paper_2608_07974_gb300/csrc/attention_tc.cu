@@ -118,6 +118,8 @@ __device__ __forceinline__ float ex2(float x) {
 template <int HDP>
 __global__ void __launch_bounds__(NT) fwd_k(const bf16* __restrict__ qkv, bf16* __restrict__ out,
                                             float* __restrict__ lse, int S, int H, int Hkv, int hd, float scale) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* Qs = reinterpret_cast<bf16*>(smem);
   bf16* Ks = Qs + BR * HDP;            // [2]
@@ -256,6 +258,8 @@ __global__ void __launch_bounds__(NT) bwd_dq_k(const bf16* __restrict__ qkv, con
                                                const bf16* __restrict__ dout, const float* __restrict__ lse,
                                                float* __restrict__ Dv, bf16* __restrict__ dqkv, int S, int H,
                                                int Hkv, int hd, float scale) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* Qs = reinterpret_cast<bf16*>(smem);
   bf16* dOs = Qs + BR * HDP;
@@ -392,6 +396,8 @@ __global__ void __launch_bounds__(NT) bwd_dkv_k(const bf16* __restrict__ qkv, co
                                                 const float* __restrict__ lse, const float* __restrict__ Dv,
                                                 bf16* __restrict__ dqkv, int S, int H, int Hkv, int hd, float scale,
                                                 float* __restrict__ part) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* Ks = reinterpret_cast<bf16*>(smem);
   bf16* Vs = Ks + BR * HDP;
@@ -568,12 +574,14 @@ void fwd_t(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv,
     attr = true;
   }
   dim3 grid(H, B, (S + BR - 1) / BR);
-  fwd_k<HDP><<<grid, NT, smem, s>>>((const bf16*)qkv, (bf16*)out, lse, S, H, Hkv, hd, 1.f / sqrtf((float)hd));
+  launch_pdl(fwd_k<HDP>, grid, NT, smem, s, (const bf16*)qkv, (bf16*)out, lse, S, H, Hkv, hd, 1.f / sqrtf((float)hd));
 }
 
 // dK, dV of each KV head = fixed-order sums of its query heads' partials.
 __global__ void reduce_dkv_k(const float* __restrict__ part, bf16* __restrict__ dqkv, int NS, int H, int Hkv, int hd,
                              float scale) {
+  pdl_wait();
+  pdl_trigger();
   const int rep = H / Hkv, ld = (H + 2 * Hkv) * hd;
   const size_t total = (size_t)NS * Hkv * (hd / 2);
   const size_t HNS = (size_t)H * NS * hd;
@@ -608,7 +616,7 @@ void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse,
     attr = true;
   }
   dim3 gq(H, B, (S + BR - 1) / BR);
-  bwd_dq_k<HDP><<<gq, NT, smem, s>>>((const bf16*)qkv, (const bf16*)out, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H,
+  launch_pdl(bwd_dq_k<HDP>, gq, NT, smem, s, (const bf16*)qkv, (const bf16*)out, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H,
                                      Hkv, hd, scale);
   float* part = nullptr;
   if (H > Hkv) {   // grouped heads: one CTA per query head, then a fixed-order group reduction
@@ -617,12 +625,12 @@ void bwd_t(const void* qkv, const void* out, const void* dout, const float* lse,
     if (e != cudaSuccess) { cudaGetLastError(); part = nullptr; }
   }
   dim3 gk(part ? H : Hkv, B, (S + BR - 1) / BR);
-  bwd_dkv_k<HDP><<<gk, NT, smem, s>>>((const bf16*)qkv, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, hd, scale,
+  launch_pdl(bwd_dkv_k<HDP>, gk, NT, smem, s, (const bf16*)qkv, (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, hd, scale,
                                       part);
   if (part) {
     const size_t total = (size_t)B * S * Hkv * (hd / 2);
     const int blocks = (int)std::min<size_t>((total + 255) / 256, 152 * 16);
-    reduce_dkv_k<<<blocks, 256, 0, s>>>(part, (bf16*)dqkv, B * S, H, Hkv, hd, scale);
+    launch_pdl(reduce_dkv_k, blocks, 256, 0, s, part, (bf16*)dqkv, B * S, H, Hkv, hd, scale);
     cudaFreeAsync(part, s);
   }
 }

@@ -399,6 +399,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Sums the split-K partials in split order (deterministic) and applies the epilogue.
 __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, int mode, void* C,
                                 const float* __restrict__ bias, const bf16* R, float alpha) {
+  pdl_wait();
+  pdl_trigger();
   const size_t n8 = (size_t)M * N / 8, MN = (size_t)M * N;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
     const size_t e = i * 8;
@@ -610,7 +612,7 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
       note_launch(1);
       const size_t n8 = (size_t)M * N / 8;
       const int blocks = (int)std::min<size_t>((n8 + 255) / 256, (size_t)tc::g_sms * 8);
-      tc::splitk_reduce_k<<<blocks, 256, 0, s>>>(ws, a.splits, M, N, mode, C, bias, (const bf16*)R, alpha);
+      launch_pdl(tc::splitk_reduce_k, blocks, 256, 0, s, ws, a.splits, M, N, mode, C, bias, (const bf16*)R, alpha);
     }
     cudaFreeAsync(ws, s);
   }

@@ -20,6 +20,8 @@ static inline int grid_for(size_t work, int threads, int max_blocks = 152 * 16) 
 template <typename T>
 __global__ void embed_k(const int32_t* __restrict__ ids, const T* __restrict__ E, const T* __restrict__ P,
                         T* __restrict__ h, int N, int S, int d, int V, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int nv = d / 8;
   const long total = (long)N * nv;
   for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
@@ -54,9 +56,9 @@ void launch_embed(int dt, const int32_t* ids, const void* E, const void* P, void
   note_launch(1);
   const int th = 256, g = grid_for((size_t)N * (d / 8), th);
   if (dt == BF16)
-    embed_k<bf16><<<g, th, 0, s>>>(ids, (const bf16*)E, (const bf16*)P, (bf16*)h, N, S, d, V, err);
+    launch_pdl(embed_k<bf16>, g, th, 0, s, ids, (const bf16*)E, (const bf16*)P, (bf16*)h, N, S, d, V, err);
   else
-    embed_k<float><<<g, th, 0, s>>>(ids, (const float*)E, (const float*)P, (float*)h, N, S, d, V, err);
+    launch_pdl(embed_k<float>, g, th, 0, s, ids, (const float*)E, (const float*)P, (float*)h, N, S, d, V, err);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -74,6 +76,8 @@ template <typename T, bool LN, int VPL>
 __global__ void norm_fwd_reg_k(const T* __restrict__ x, const float* __restrict__ g, const float* __restrict__ b,
                                T* __restrict__ y, float* __restrict__ rstd_o, float* __restrict__ mean_o, int N, int d,
                                float eps) {
+  pdl_wait();
+  pdl_trigger();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= N) return;
   const T* xr = x + (size_t)row * d;
@@ -131,6 +135,8 @@ __global__ void norm_bwd_dx_reg_k(const T* __restrict__ x, const float* __restri
                                   const float* __restrict__ rstd, const float* __restrict__ mean,
                                   const T* __restrict__ dy, const T* __restrict__ dres, T* __restrict__ dx, int N,
                                   int d) {
+  pdl_wait();
+  pdl_trigger();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= N) return;
   const size_t o = (size_t)row * d;
@@ -189,6 +195,8 @@ __global__ void __launch_bounds__(512) norm_fwd_blk_k(const T* __restrict__ x, c
                                                       const float* __restrict__ b, T* __restrict__ y,
                                                       float* __restrict__ rstd_o, float* __restrict__ mean_o, int N,
                                                       int d, float eps) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float sh[32];
   const size_t o = (size_t)blockIdx.x * d;
   float f[VPT][8], gv[VPT][8], bv[VPT][8];
@@ -242,6 +250,8 @@ __global__ void __launch_bounds__(512) norm_bwd_dx_blk_k(const T* __restrict__ x
                                                          const float* __restrict__ mean, const T* __restrict__ dy,
                                                          const T* __restrict__ dres, T* __restrict__ dx, int N,
                                                          int d) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float sh[32];
   const size_t o = (size_t)blockIdx.x * d;
   const float r = rstd[blockIdx.x], mu = LN ? mean[blockIdx.x] : 0.f;
@@ -304,13 +314,13 @@ void launch_norm_fwd(int dt, bool ln, const void* x, const float* g, const float
   note_launch(1);
   const int th = 256, blocks = (N * 32 + th - 1) / th;
   const int vpl = (d + 255) / 256;
-#define NFR(T, L, V) norm_fwd_reg_k<T, L, V><<<blocks, th, 0, s>>>((const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
+#define NFR(T, L, V) launch_pdl(norm_fwd_reg_k<T, L, V>, blocks, th, 0, s, (const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
 #define NFV(T, L)                     \
   if (vpl == 1) NFR(T, L, 1);         \
   else if (vpl == 2) NFR(T, L, 2);    \
   else if (vpl == 3) NFR(T, L, 3);    \
   else NFR(T, L, 4);
-#define NFB(T, L, V) norm_fwd_blk_k<T, L, V><<<N, bt, 0, s>>>((const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
+#define NFB(T, L, V) launch_pdl(norm_fwd_blk_k<T, L, V>, N, bt, 0, s, (const T*)x, g, b, (T*)y, rstd, mean, N, d, eps)
 #define NF(T, L)                      \
   if (vpt == 1) NFB(T, L, 1);         \
   else if (vpt == 2) NFB(T, L, 2);    \
@@ -336,7 +346,7 @@ void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const fl
   const int th = 256, blocks = (N * 32 + th - 1) / th;
   const int vpl = (d + 255) / 256;
 #define NBR(T, L, V)                                                                                             \
-  norm_bwd_dx_reg_k<T, L, V><<<blocks, th, 0, s>>>((const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, \
+  launch_pdl(norm_bwd_dx_reg_k<T, L, V>, blocks, th, 0, s, (const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, \
                                                    N, d)
 #define NBV(T, L)                     \
   if (vpl == 1) NBR(T, L, 1);         \
@@ -344,7 +354,7 @@ void launch_norm_bwd_dx(int dt, bool ln, const void* x, const float* g, const fl
   else if (vpl == 3) NBR(T, L, 3);    \
   else NBR(T, L, 4);
 #define NBB(T, L, V)                                                                                          \
-  norm_bwd_dx_blk_k<T, L, V><<<N, bt, 0, s>>>((const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, N, d)
+  launch_pdl(norm_bwd_dx_blk_k<T, L, V>, N, bt, 0, s, (const T*)x, g, rstd, mean, (const T*)dy, (const T*)dres, (T*)dx, N, d)
 #define NB(T, L)                      \
   if (vpt == 1) NBB(T, L, 1);         \
   else if (vpt == 2) NBB(T, L, 2);    \
@@ -381,6 +391,8 @@ __global__ void __launch_bounds__(256) colsum_k(const T* __restrict__ A, const T
                                                 float* __restrict__ part_g, float* __restrict__ part_b, int N,
                                                 int d, float* __restrict__ out_g, float* __restrict__ out_b,
                                                 unsigned* __restrict__ counters) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int R = kColRows / kColLanes;
   __shared__ unsigned ticket;
   __shared__ float sg[kColLanes][256], sb[kColLanes][256];
@@ -486,7 +498,7 @@ void launch_norm_bwd_dparam(int dt, bool ln, const void* x, const float* rstd, c
   note_launch(1);
   dim3 grid(colsum_groups(d), colsum_blocks(N)), block(32, kColLanes);
 #define CS(T, L)                                                                                             \
-  colsum_k<T, true, L><<<grid, block, 0, s>>>((const T*)dy, (const T*)x, rstd, mean, part_g, part_b, N, d, out_g, \
+  launch_pdl(colsum_k<T, true, L>, grid, block, 0, s, (const T*)dy, (const T*)x, rstd, mean, part_g, part_b, N, d, out_g, \
                                               out_b, counters)
   if (dt == BF16) { if (ln) CS(bf16, true); else CS(bf16, false); }
   else { if (ln) CS(float, true); else CS(float, false); }
@@ -497,10 +509,10 @@ void launch_colsum(int dt, const void* A, float* part, int N, int d, float* out,
   note_launch(1);
   dim3 grid(colsum_groups(d), colsum_blocks(N)), block(32, kColLanes);
   if (dt == BF16)
-    colsum_k<bf16, false, false><<<grid, block, 0, s>>>((const bf16*)A, nullptr, nullptr, nullptr, nullptr, part, N, d,
+    launch_pdl(colsum_k<bf16, false, false>, grid, block, 0, s, (const bf16*)A, nullptr, nullptr, nullptr, nullptr, part, N, d,
                                                         nullptr, out, counters);
   else
-    colsum_k<float, false, false><<<grid, block, 0, s>>>((const float*)A, nullptr, nullptr, nullptr, nullptr, part, N,
+    launch_pdl(colsum_k<float, false, false>, grid, block, 0, s, (const float*)A, nullptr, nullptr, nullptr, nullptr, part, N,
                                                          d, nullptr, out, counters);
 }
 
@@ -523,6 +535,8 @@ void launch_partials_add(const float* part, int nb, int d, float* out, cudaStrea
 template <typename T>
 __global__ void rope_k(T* __restrict__ qkv, const float2* __restrict__ cs, int N, int S, int nh, int hd,
                        int ld, int inverse) {
+  pdl_wait();
+  pdl_trigger();
   const int half = hd / 2;
   const long total = (long)N * nh * half;
   for (long idx = blockIdx.x * (long)blockDim.x + threadIdx.x; idx < total;
@@ -544,14 +558,16 @@ void launch_rope(int dt, void* qkv, const float* cs, int N, int S, int H, int Hk
   note_launch(1);
   const int nh = H + Hkv, ld = (H + 2 * Hkv) * hd;
   const int th = 256, g = grid_for((size_t)N * nh * (hd / 2), th);
-  if (dt == BF16) rope_k<bf16><<<g, th, 0, s>>>((bf16*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
-  else rope_k<float><<<g, th, 0, s>>>((float*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
+  if (dt == BF16) launch_pdl(rope_k<bf16>, g, th, 0, s, (bf16*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
+  else launch_pdl(rope_k<float>, g, th, 0, s, (float*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
 }
 
 __device__ __forceinline__ float sigmoidf_(float x) { return 1.f / (1.f + expf(-x)); }
 
 template <typename T>
 __global__ void swiglu_fwd_k(const T* __restrict__ gu, T* __restrict__ a, int N, int f) {
+  pdl_wait();
+  pdl_trigger();
   const int nv = f / 8;
   const long total = (long)N * nv;
   for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
@@ -568,6 +584,8 @@ __global__ void swiglu_fwd_k(const T* __restrict__ gu, T* __restrict__ a, int N,
 template <typename T>
 __global__ void swiglu_bwd_k(const T* __restrict__ gu, const T* __restrict__ da, T* __restrict__ dgu, int N,
                              int f) {
+  pdl_wait();
+  pdl_trigger();
   const int nv = f / 8;
   const long total = (long)N * nv;
   for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
@@ -590,20 +608,22 @@ __global__ void swiglu_bwd_k(const T* __restrict__ gu, const T* __restrict__ da,
 void launch_swiglu_fwd(int dt, const void* gu, void* a, int N, int f, cudaStream_t s) {
   note_launch(1);
   const int th = 256, g = grid_for((size_t)N * (f / 8), th);
-  if (dt == BF16) swiglu_fwd_k<bf16><<<g, th, 0, s>>>((const bf16*)gu, (bf16*)a, N, f);
-  else swiglu_fwd_k<float><<<g, th, 0, s>>>((const float*)gu, (float*)a, N, f);
+  if (dt == BF16) launch_pdl(swiglu_fwd_k<bf16>, g, th, 0, s, (const bf16*)gu, (bf16*)a, N, f);
+  else launch_pdl(swiglu_fwd_k<float>, g, th, 0, s, (const float*)gu, (float*)a, N, f);
 }
 void launch_swiglu_bwd(int dt, const void* gu, const void* da, void* dgu, int N, int f, cudaStream_t s) {
   note_launch(1);
   const int th = 256, g = grid_for((size_t)N * (f / 8), th);
-  if (dt == BF16) swiglu_bwd_k<bf16><<<g, th, 0, s>>>((const bf16*)gu, (const bf16*)da, (bf16*)dgu, N, f);
-  else swiglu_bwd_k<float><<<g, th, 0, s>>>((const float*)gu, (const float*)da, (float*)dgu, N, f);
+  if (dt == BF16) launch_pdl(swiglu_bwd_k<bf16>, g, th, 0, s, (const bf16*)gu, (const bf16*)da, (bf16*)dgu, N, f);
+  else launch_pdl(swiglu_bwd_k<float>, g, th, 0, s, (const float*)gu, (const float*)da, (float*)dgu, N, f);
 }
 
 __device__ __forceinline__ float gelu_inner(float x) { return 0.7978845608028654f * (x + 0.044715f * x * x * x); }
 
 template <typename T>
 __global__ void gelu_fwd_k(const T* __restrict__ x, T* __restrict__ y, size_t n8) {
+  pdl_wait();
+  pdl_trigger();
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
     float f[8];
     Vec8<T>::load(x + i * 8, f);
@@ -615,6 +635,8 @@ __global__ void gelu_fwd_k(const T* __restrict__ x, T* __restrict__ y, size_t n8
 
 template <typename T>
 __global__ void gelu_bwd_k(const T* __restrict__ x, const T* __restrict__ dy, T* __restrict__ dx, size_t n8) {
+  pdl_wait();
+  pdl_trigger();
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
     float f[8], d[8];
     Vec8<T>::load(x + i * 8, f);
@@ -632,14 +654,14 @@ __global__ void gelu_bwd_k(const T* __restrict__ x, const T* __restrict__ dy, T*
 void launch_gelu_fwd(int dt, const void* x, void* y, size_t n, cudaStream_t s) {
   note_launch(1);
   const int th = 256, g = grid_for(n / 8, th);
-  if (dt == BF16) gelu_fwd_k<bf16><<<g, th, 0, s>>>((const bf16*)x, (bf16*)y, n / 8);
-  else gelu_fwd_k<float><<<g, th, 0, s>>>((const float*)x, (float*)y, n / 8);
+  if (dt == BF16) launch_pdl(gelu_fwd_k<bf16>, g, th, 0, s, (const bf16*)x, (bf16*)y, n / 8);
+  else launch_pdl(gelu_fwd_k<float>, g, th, 0, s, (const float*)x, (float*)y, n / 8);
 }
 void launch_gelu_bwd(int dt, const void* x, const void* dy, void* dx, size_t n, cudaStream_t s) {
   note_launch(1);
   const int th = 256, g = grid_for(n / 8, th);
-  if (dt == BF16) gelu_bwd_k<bf16><<<g, th, 0, s>>>((const bf16*)x, (const bf16*)dy, (bf16*)dx, n / 8);
-  else gelu_bwd_k<float><<<g, th, 0, s>>>((const float*)x, (const float*)dy, (float*)dx, n / 8);
+  if (dt == BF16) launch_pdl(gelu_bwd_k<bf16>, g, th, 0, s, (const bf16*)x, (const bf16*)dy, (bf16*)dx, n / 8);
+  else launch_pdl(gelu_bwd_k<float>, g, th, 0, s, (const float*)x, (const float*)dy, (float*)dx, n / 8);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -730,6 +752,8 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
                                                      const int32_t* __restrict__ labels, int V, int ldz,
                                                      float alpha, const int* __restrict__ count,
                                                      T* __restrict__ dz, float* __restrict__ row_loss) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ Lse3 shz[32], sht[32];
   __shared__ float sh_stats[4];
   const int row = blockIdx.x;
@@ -816,7 +840,7 @@ void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labe
   int th = 32;
   while (th < cap && th * 8 < ldz) th *= 2;
 #define LL(T, TE, KD)                                                                                        \
-  local_loss_k<T, TE, KD><<<N, th, 0, s>>>((const T*)z, (const T*)t, labels, V, ldz, alpha, count, (T*)dz, \
+  launch_pdl(local_loss_k<T, TE, KD>, N, th, 0, s, (const T*)z, (const T*)t, labels, V, ldz, alpha, count, (T*)dz, \
                                            row_loss)
 #define LLT(T)                      \
   if (!t) LL(T, false, 0);          \
@@ -828,6 +852,8 @@ void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labe
 }
 
 __global__ void count_valid_k(const int32_t* __restrict__ labels, int N, int V, int* count, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float sh[32];
   float c = 0.f;
   bool bad = false;
@@ -843,10 +869,12 @@ __global__ void count_valid_k(const int32_t* __restrict__ labels, int N, int V, 
 
 void launch_count_valid(const int32_t* labels, int N, int V, int* count, unsigned* err, cudaStream_t s) {
   note_launch(1);
-  count_valid_k<<<1, 1024, 0, s>>>(labels, N, V, count, err);
+  launch_pdl(count_valid_k, 1, 1024, 0, s, labels, N, V, count, err);
 }
 
 __global__ void loss_reduce_k(const float* __restrict__ rl, int N, const int* count, float* out) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ double sh[1024];
   double acc = 0.0;
   for (int i0 = threadIdx.x; i0 < N; i0 += 4 * blockDim.x) {   // 4 loads in flight, added in index order
@@ -871,7 +899,7 @@ __global__ void loss_reduce_k(const float* __restrict__ rl, int N, const int* co
 
 void launch_loss_reduce(const float* row_loss, int N, const int* count, float* out, cudaStream_t s) {
   note_launch(1);
-  loss_reduce_k<<<1, 1024, 0, s>>>(row_loss, N, count, out);
+  launch_pdl(loss_reduce_k, 1, 1024, 0, s, row_loss, N, count, out);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -880,6 +908,8 @@ void launch_loss_reduce(const float* row_loss, int N, const int* count, float* o
 __global__ void adamw_k(float4* __restrict__ th, float4* __restrict__ g, float4* __restrict__ m,
                         float4* __restrict__ v, __nv_bfloat162* __restrict__ comp, size_t n4, float lr, float b1,
                         float b2, float eps, float wd, float bc1, float bc2, float gscale) {
+  pdl_wait();
+  pdl_trigger();
   const float decay = 1.f - lr * wd;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
     float4 t = th[i], gg = g[i], mm = m[i], vv = v[i];
@@ -905,7 +935,7 @@ void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t
   note_launch(1);
   const size_t n4 = n / 4;   // slabs are padded to a multiple of 64 elements
   const int th = 256, gr = grid_for(n4, th, 152 * 8);
-  adamw_k<<<gr, th, 0, s>>>((float4*)theta, (float4*)g, (float4*)m, (float4*)v, (__nv_bfloat162*)comp, n4, lr,
+  launch_pdl(adamw_k, gr, th, 0, s, (float4*)theta, (float4*)g, (float4*)m, (float4*)v, (__nv_bfloat162*)comp, n4, lr,
                             b1, b2, eps, wd, bc1, bc2, gscale);
 }
 
