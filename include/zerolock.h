@@ -81,6 +81,9 @@ typedef struct {
   int adapter_dim;          /* 0: static readout head; r > 0 (a multiple of 16): chunk k's own readout  */
                             /*   goes through its adapter a_k(h) = h + GELU(h D_k^T) U_k^T (Section     */
                             /*   III-B, local update interface (b)), D_k [r, d], U_k [d, r] trainable   */
+  int graph;                /* 1: zl_step / zl_bp_step are captured as a CUDA graph once per micro-batch */
+                            /*   shape (after one eager call at that shape) and replayed; taken only    */
+                            /*   with accum_m = 1, replay_depth = 0 and profiling off (else eager)      */
 } zl_train_cfg;
 
 /* Create a context: parameters, AdamW state, K streams and events, a stream-ordered

@@ -36,7 +36,8 @@ class zl_train_cfg(C.Structure):
                 ("beta1", C.c_float), ("beta2", C.c_float), ("eps", C.c_float), ("weight_decay", C.c_float),
                 ("accum_m", C.c_int), ("max_live_chunks", C.c_int), ("lr_schedule", C.c_int),
                 ("lr_gamma", C.c_float), ("serialize", C.c_int), ("lora_rank", C.c_int),
-                ("lora_scale", C.c_float), ("replay_depth", C.c_int), ("adapter_dim", C.c_int)]
+                ("lora_scale", C.c_float), ("replay_depth", C.c_int), ("adapter_dim", C.c_int),
+                ("graph", C.c_int)]
 
 
 class ZLError(RuntimeError):
@@ -305,7 +306,7 @@ class ZeroLock:
                  beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.01, accum_m: int = 1,
                  max_live_chunks: int = 0, lr_schedule: int = 0, lr_gamma: float = 1.0, serialize: bool = False,
                  lora_rank: int = 0, lora_scale: float = 1.0, replay_depth: int = 0, adapter_dim: int = 0,
-                 stream=None):
+                 graph: bool = False, stream=None):
         import torch
         self.dims = dims
         self.K = K
@@ -315,7 +316,7 @@ class ZeroLock:
                            dims.norm_eps, dims.rope_theta)
         cfg = zl_train_cfg(alpha, kl_dir, consis_first, lr, beta1, beta2, eps, weight_decay, accum_m,
                            max_live_chunks, lr_schedule, lr_gamma, int(serialize), lora_rank, lora_scale,
-                           replay_depth, adapter_dim)
+                           replay_depth, adapter_dim, int(graph))
         self.ctx = zl_create(md, K, list(bounds), cfg)
         s = stream if stream is not None else torch.cuda.current_stream()
         zl_set_stream(self.ctx, s.cuda_stream)

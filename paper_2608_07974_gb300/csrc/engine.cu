@@ -97,7 +97,9 @@ struct Chunk {
   size_t ad_down = 0, ad_up = 0;   // readout adapter D [r, d] and U [d, r] in the trainable slab
   size_t n_layers_slab = 0;        // trainable floats before the adapter (what backpropagation updates)
   int micro = 0;
-  long t = 0;
+  long t = 0;                // optimizer steps (host mirror of *d_t)
+  long long* d_t = nullptr;  // optimizer steps on the device, advanced by the AdamW launch
+  float* d_hp = nullptr;     // this step's lr and bias corrections (written on the device)
   long done = 0;             // micro-batches this chunk has processed (progress metadata)
   // hidden-state buffer (Section III-B-3): the last replay_depth inputs h_{k-1} with their labels
   struct Entry {
@@ -152,6 +154,17 @@ struct zl_ctx {
   std::vector<ProfRec> recs;
   std::vector<cudaEvent_t> evpool;
   size_t evnext = 0;
+  // CUDA-graph form of zl_step / zl_bp_step: one capture per micro-batch shape, then replays
+  struct StepGraph {
+    int B = 0, S = 0;
+    int seen = 0;                 // calls at this shape so far (the first runs eagerly)
+    cudaGraphExec_t exec = nullptr;
+    int32_t *ids = nullptr, *labels = nullptr;   // staging copies of the inputs the graph reads
+    size_t cap = 0;
+    unsigned long long launches = 0;             // kernel launches the captured step contains
+  } zg, bg;
+  bool capturing = false;
+  cudaStream_t cap = nullptr;   // capture origin (the user's stream may be the uncapturable legacy stream)
 };
 
 namespace {
@@ -550,16 +563,11 @@ void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s, bool adapters = true) {
   if (k.micro < c->cfg.accum_m) return;
   k.t += 1;
   const zl_train_cfg& g = c->cfg;
-  double lr = g.lr;
-  if (g.lr_schedule == 1) lr = g.lr / std::sqrt((double)(k.t - 1) + g.lr_gamma);
-  const double bc1 = 1.0 - std::pow((double)g.beta1, (double)k.t);
-  const double bc2 = 1.0 - std::pow((double)g.beta2, (double)k.t);
   const size_t n = (adapters || g.adapter_dim == 0) ? k.n : k.n_layers_slab;
   k.micro = 0;
-  if (n == 0) return;
   ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * (double)n);
-  launch_adamw(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, n, (float)lr, g.beta1, g.beta2, g.eps,
-               g.weight_decay, (float)bc1, (float)bc2, 1.f / (float)g.accum_m, s);
+  launch_adamw(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, n, k.d_t, k.d_hp, g.lr, g.lr_schedule,
+               g.lr_gamma, g.beta1, g.beta2, g.eps, g.weight_decay, 1.f / (float)g.accum_m, s);
   CHECK_LAUNCH();
   k.micro = 0;
 }
@@ -817,6 +825,12 @@ bool lookup(zl_ctx* c, const std::string& name, Found& f) {
 void free_ctx(zl_ctx* c) {
   if (!c) return;
   cudaDeviceSynchronize();
+  for (zl_ctx::StepGraph* g : {&c->zg, &c->bg}) {
+    if (g->exec) cudaGraphExecDestroy(g->exec);
+    if (g->ids) cudaFree(g->ids);
+    if (g->labels) cudaFree(g->labels);
+  }
+  if (c->cap) cudaStreamDestroy(c->cap);
   const bool shared = c->cfg.serialize != 0;
   for (int k = 1; k < (int)c->ch.size(); ++k) {
     Chunk& ck = c->ch[k];
@@ -1026,6 +1040,9 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
         ck.fmat = salloc(c, fmat * esz(c));
         CK(cudaMemset(ck.fmat, 0, fmat * esz(c)));
       }
+      ck.d_t = (long long*)salloc(c, 64);
+      ck.d_hp = (float*)(ck.d_t + 1);
+      CK(cudaMemset(ck.d_t, 0, 64));
       ck.master = (float*)salloc(c, ck.n * 4);
       ck.grad = (float*)salloc(c, ck.n * 4);
       ck.m = (float*)salloc(c, ck.n * 4);
@@ -1345,6 +1362,8 @@ zl_status zl_chunk_load(zl_ctx* c, int k, const void* src, size_t bytes) {
     if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
     CK(cudaDeviceSynchronize());
     ck.t = h.t;
+    const long long tt = h.t;
+    CK(cudaMemcpy(ck.d_t, &tt, sizeof(tt), cudaMemcpyHostToDevice));
     ck.done = h.done;
     ck.micro = h.micro;
     return ZL_OK;
@@ -1354,96 +1373,209 @@ zl_status zl_chunk_load(zl_ctx* c, int k, const void* src, size_t bytes) {
 // The concurrent ZeroLock step: chunk k runs on stream s_k; its forward waits only for the
 // readiness event of h_{k-1} (early forwarding), its loss waits for the teacher logits z_{k-1},
 // and at most `cap` chunks hold activation arenas at once.
+}  // extern "C"
+
+namespace {
+
+// CUDA graphs (cfg.graph): a step is captured once per micro-batch shape and replayed. The first call
+// at a shape runs eagerly (it also performs the one-time set-up some launches do); the inputs are
+// staged into context-owned buffers that the graph reads. Graphs are used only where a step's work
+// is the same every time: no profiling, one micro-batch per window, no replay buffer.
+bool graph_ok(zl_ctx* c) {
+  return c->cfg.graph != 0 && !c->prof && c->cfg.accum_m == 1 && c->cfg.replay_depth == 0;
+}
+
+template <typename E, typename A>
+bool run_graph(zl_ctx* c, zl_ctx::StepGraph& g, const int32_t* ids, const int32_t* labels, int B, int S, E&& enqueue,
+               A&& advance) {
+  if (!graph_ok(c)) return false;
+  const size_t N = (size_t)B * S;
+  if (g.B != B || g.S != S) {
+    if (g.exec) {
+      sync_all(c, -1);
+      CK(cudaGraphExecDestroy(g.exec));
+      g.exec = nullptr;
+    }
+    g.B = B;
+    g.S = S;
+    g.seen = 0;
+  }
+  if (g.seen++ < 1) return false;
+  if (g.cap < N) {   // (re)allocate the staging buffers, outside any capture
+    sync_all(c, -1);
+    if (g.ids) CK(cudaFree(g.ids));
+    if (g.labels) CK(cudaFree(g.labels));
+    g.ids = g.labels = nullptr;
+    g.cap = 0;
+    CK(cudaMalloc((void**)&g.ids, N * 4));
+    CK(cudaMalloc((void**)&g.labels, N * 4));
+    g.cap = N;
+  }
+  CK(cudaMemcpyAsync(g.ids, ids, N * 4, cudaMemcpyDeviceToDevice, c->user));
+  CK(cudaMemcpyAsync(g.labels, labels, N * 4, cudaMemcpyDeviceToDevice, c->user));
+  join_all(c);   // every stream's earlier work before the graph
+  if (!g.exec) {
+    // capture on a stream of the context, standing in for the user's stream
+    if (!c->cap) CK(cudaStreamCreateWithFlags(&c->cap, cudaStreamNonBlocking));
+    const cudaStream_t user = c->user;
+    CK(cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal));
+    c->capturing = true;
+    c->user = c->cap;
+    const unsigned long long n0 = g_launches.load();
+    try {
+      enqueue(g.ids, g.labels);
+      join_all(c);
+      g.launches = g_launches.load() - n0;
+    } catch (...) {
+      c->capturing = false;
+      c->user = user;
+      cudaGraph_t junk = nullptr;
+      cudaStreamEndCapture(c->cap, &junk);
+      if (junk) cudaGraphDestroy(junk);
+      cudaGetLastError();
+      throw;
+    }
+    c->capturing = false;
+    c->user = user;
+    cudaGraph_t graph = nullptr;
+    CK(cudaStreamEndCapture(c->cap, &graph));
+    const cudaError_t e = cudaGraphInstantiate(&g.exec, graph, 0);
+    cudaGraphDestroy(graph);
+    CK(e);
+  } else {
+    advance();
+    note_launch((int)g.launches);   // the replay runs the same kernels
+  }
+  CK(cudaGraphLaunch(g.exec, c->user));
+  // The context's events were last recorded inside the capture, which does not count as a record
+  // outside it: record them all after the graph (a later point than the one they stood for, so every
+  // later wait on them stays correct). Later work on the chunk and auxiliary streams (loss read-back,
+  // the next eager step) follows the graph.
+  for (cudaEvent_t e : c->live_ring) rec(e, c->user);
+  for (int k = 1; k <= c->K; ++k)
+    for (cudaEvent_t e : {c->ch[k].ev_h, c->ch[k].ev_z, c->ch[k].ev_loss, c->ch[k].ev_hb, c->ch[k].ev_done})
+      rec(e, c->user);
+  for (cudaEvent_t e : {c->ev_aux, c->ev_sync}) rec(e, c->user);
+  rec(c->ev_start, c->user);
+  for (int k = 1; k <= c->K; ++k) wait_ev(c->ch[k].s, c->ev_start);
+  wait_ev(c->aux, c->ev_start);
+  return true;
+}
+
+// The work of one zl_step, queued on the chunk streams (eagerly or into a capture).
+void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S) {
+  const int N = B * S, K = c->K;
+  const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+  rec(c->ev_start, c->user);
+  for (int k = 1; k <= K; ++k) wait_ev(c->ch[k].s, c->ev_start);
+  wait_ev(c->aux, c->ev_start);
+  std::vector<void*> h(K + 1, nullptr), z(K + 1, nullptr);
+  // h_0 = E(x) on s_1; the teacher of chunk 1, z_0 = readout(h_0), on the auxiliary stream
+  cudaStream_t s1 = c->ch[1].s;
+  h[0] = palloc(c, hb, s1);
+  launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h[0], N, S, c->d, c->V, c->d_err, s1);
+  CHECK_LAUNCH();
+  rec(c->ch[1].ev_h, s1);   // reused below as "h_0 ready" before chunk 1 records h_1
+  cudaEvent_t ev_h0 = c->ev_aux;
+  const float a1 = alpha_of(c, 1);
+  if (a1 < 1.f) {
+    wait_ev(c->aux, c->ch[1].ev_h);
+    z[0] = palloc(c, zb, c->aux);
+    readout_fwd(c, h[0], z[0], nullptr, N, c->aux);
+  }
+  rec(ev_h0, c->aux);      // z_0 ready (and aux done reading h_0)
+  const int cap = (int)c->live_ring.size();
+  const bool adp = c->cfg.adapter_dim > 0;
+  for (int k = 1; k <= K; ++k) {
+    Chunk& ck = c->ch[k];
+    cudaStream_t s = ck.s;
+    const float a = alpha_of(c, k);
+    // S1: the upstream entry (h_{k-1}) and a free arena slot
+    if (k > 1) wait_ev(s, c->ch[k - 1].ev_h);
+    ring_put(c, ck, c->seq, h[k - 1], labels, B, S, s);
+    ck.done += 1;
+    // a capture sees only this step's events: slots are numbered within the step (graph launches
+    // on the user stream already order one step after the previous one)
+    const long seq0 = c->live_seq++;
+    const long seq = c->capturing ? (long)(k - 1) : seq0;
+    if (seq >= cap) wait_ev(s, c->live_ring[seq % cap]);
+    // S2: forward, then hand h_k downstream before the local backward (early forwarding)
+    h[k] = palloc(c, hb, s);
+    ChunkActs acts;
+    chunk_fwd_save(c, ck, h[k - 1], h[k], B, S, acts, s);
+    rec(ck.ev_h, s);
+    z[k] = palloc(c, zb, s);
+    ReadoutSave rs;
+    readout_fwd(c, h[k], z[k], &rs, N, s, adp ? &ck : nullptr);
+    rec(ck.ev_z, s);
+    // S3: local objective against the stop-gradient teacher: the frozen head on h_{k-1}, which is
+    // chunk k-1's own readout z_{k-1} (reused) unless chunk k-1 read out through its adapter
+    void* teacher = nullptr;
+    void* own_t = nullptr;
+    if (a < 1.f) {
+      if (k == 1) {
+        wait_ev(s, ev_h0);
+        teacher = z[0];
+      } else if (adp) {
+        own_t = palloc(c, zb, s);
+        readout_fwd(c, h[k - 1], own_t, nullptr, N, s);
+        teacher = own_t;
+      } else {
+        wait_ev(s, c->ch[k - 1].ev_z);
+        teacher = z[k - 1];
+      }
+    }
+    void* dz = local_loss(c, z[k], teacher, labels, a, N, k, s);
+    rec(ck.ev_loss, s);
+    pfree(own_t, s);
+    // z_{k-1} is no longer needed once this loss and chunk k-1's own loss are done
+    if (k == 1) {
+      if (z[0]) { wait_ev(s, ev_h0); pfree(z[0], s); }
+    } else if (!adp) {
+      wait_ev(s, c->ch[k - 1].ev_loss);
+      pfree(z[k - 1], s);
+    }
+    if (k == K || adp) pfree(z[k], s);   // with adapters no later chunk reads z_k
+    void* dh = palloc(c, hb, s);
+    readout_bwd(c, h[k], rs, dz, dh, N, s, adp ? &ck : nullptr);
+    pfree(dz, s);
+    rec(ck.ev_hb, s);
+    chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
+    pfree(dh, s);
+    pfree(acts.mem, s);
+    rec(c->live_ring[seq % cap], s);
+    // h_{k-1}: read by this chunk's backward and by chunk k-1's readout backward
+    if (k == 1) wait_ev(s, ev_h0);
+    else wait_ev(s, c->ch[k - 1].ev_hb);
+    pfree(h[k - 1], s);
+    if (k == K) pfree(h[K], s);
+    adamw_window(c, ck, s);
+  }
+  c->last_nloss = K;
+  c->seq += 1;
+}
+
+}  // namespace
+
+extern "C" {
+
 zl_status zl_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S, float* losses_out) {
   if (!c || !ids || !labels) { g_err = "NULL argument"; return ZL_ERR_ARG; }
   return guarded(c, [&]() -> zl_status {
     check_bs(c, B, S);
-    const int N = B * S, K = c->K;
-    const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
-    rec(c->ev_start, c->user);
-    for (int k = 1; k <= K; ++k) wait_ev(c->ch[k].s, c->ev_start);
-    wait_ev(c->aux, c->ev_start);
-    std::vector<void*> h(K + 1, nullptr), z(K + 1, nullptr);
-    // h_0 = E(x) on s_1; the teacher of chunk 1, z_0 = readout(h_0), on the auxiliary stream
-    cudaStream_t s1 = c->ch[1].s;
-    h[0] = palloc(c, hb, s1);
-    launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h[0], N, S, c->d, c->V, c->d_err, s1);
-    CHECK_LAUNCH();
-    rec(c->ch[1].ev_h, s1);   // reused below as "h_0 ready" before chunk 1 records h_1
-    cudaEvent_t ev_h0 = c->ev_aux;
-    const float a1 = alpha_of(c, 1);
-    if (a1 < 1.f) {
-      wait_ev(c->aux, c->ch[1].ev_h);
-      z[0] = palloc(c, zb, c->aux);
-      readout_fwd(c, h[0], z[0], nullptr, N, c->aux);
-    }
-    rec(ev_h0, c->aux);      // z_0 ready (and aux done reading h_0)
-    const int cap = (int)c->live_ring.size();
-    const bool adp = c->cfg.adapter_dim > 0;
-    for (int k = 1; k <= K; ++k) {
-      Chunk& ck = c->ch[k];
-      cudaStream_t s = ck.s;
-      const float a = alpha_of(c, k);
-      // S1: the upstream entry (h_{k-1}) and a free arena slot
-      if (k > 1) wait_ev(s, c->ch[k - 1].ev_h);
-      ring_put(c, ck, c->seq, h[k - 1], labels, B, S, s);
-      ck.done += 1;
-      const long seq = c->live_seq++;
-      if (seq >= cap) wait_ev(s, c->live_ring[seq % cap]);
-      // S2: forward, then hand h_k downstream before the local backward (early forwarding)
-      h[k] = palloc(c, hb, s);
-      ChunkActs acts;
-      chunk_fwd_save(c, ck, h[k - 1], h[k], B, S, acts, s);
-      rec(ck.ev_h, s);
-      z[k] = palloc(c, zb, s);
-      ReadoutSave rs;
-      readout_fwd(c, h[k], z[k], &rs, N, s, adp ? &ck : nullptr);
-      rec(ck.ev_z, s);
-      // S3: local objective against the stop-gradient teacher: the frozen head on h_{k-1}, which is
-      // chunk k-1's own readout z_{k-1} (reused) unless chunk k-1 read out through its adapter
-      void* teacher = nullptr;
-      void* own_t = nullptr;
-      if (a < 1.f) {
-        if (k == 1) {
-          wait_ev(s, ev_h0);
-          teacher = z[0];
-        } else if (adp) {
-          own_t = palloc(c, zb, s);
-          readout_fwd(c, h[k - 1], own_t, nullptr, N, s);
-          teacher = own_t;
-        } else {
-          wait_ev(s, c->ch[k - 1].ev_z);
-          teacher = z[k - 1];
-        }
-      }
-      void* dz = local_loss(c, z[k], teacher, labels, a, N, k, s);
-      rec(ck.ev_loss, s);
-      pfree(own_t, s);
-      // z_{k-1} is no longer needed once this loss and chunk k-1's own loss are done
-      if (k == 1) {
-        if (z[0]) { wait_ev(s, ev_h0); pfree(z[0], s); }
-      } else if (!adp) {
-        wait_ev(s, c->ch[k - 1].ev_loss);
-        pfree(z[k - 1], s);
-      }
-      if (k == K || adp) pfree(z[k], s);   // with adapters no later chunk reads z_k
-      void* dh = palloc(c, hb, s);
-      readout_bwd(c, h[k], rs, dz, dh, N, s, adp ? &ck : nullptr);
-      pfree(dz, s);
-      rec(ck.ev_hb, s);
-      chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
-      pfree(dh, s);
-      pfree(acts.mem, s);
-      rec(c->live_ring[seq % cap], s);
-      // h_{k-1}: read by this chunk's backward and by chunk k-1's readout backward
-      if (k == 1) wait_ev(s, ev_h0);
-      else wait_ev(s, c->ch[k - 1].ev_hb);
-      pfree(h[k - 1], s);
-      if (k == K) pfree(h[K], s);
-      adamw_window(c, ck, s);
-    }
-    c->last_nloss = K;
-    c->seq += 1;
+    const int K = c->K;
+    const bool graphed = run_graph(
+        c, c->zg, ids, labels, B, S, [&](const int32_t* gi, const int32_t* gl) { step_enqueue(c, gi, gl, B, S); },
+        [&]() {   // the host bookkeeping step_enqueue does, for a replay
+          for (int k = 1; k <= K; ++k) {
+            c->ch[k].done += 1;
+            c->ch[k].t += 1;
+          }
+          c->live_seq += K;
+          c->last_nloss = K;
+          c->seq += 1;
+        });
+    if (!graphed) step_enqueue(c, ids, labels, B, S);
     if (losses_out) {
       for (int k = 1; k <= K; ++k)
         CK(cudaMemcpyAsync(c->h_losses + k, c->d_losses + k, 4, cudaMemcpyDeviceToHost, c->ch[k].s));
@@ -1456,54 +1588,80 @@ zl_status zl_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
 
 // Backpropagation through all chunks (the same kernels, one stream, every arena alive until
 // the backward reaches it).
-zl_status zl_bp_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S, float* loss_out) {
-  if (!c || !ids || !labels) { g_err = "NULL argument"; return ZL_ERR_ARG; }
-  return guarded(c, [&]() -> zl_status {
-    check_bs(c, B, S);
-    const int N = B * S, K = c->K;
-    const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
-    cudaStream_t s = c->ch[1].s;
-    rec(c->ev_start, c->user);
-    wait_ev(s, c->ev_start);
+}  // extern "C"
+
+namespace {
+
+// The work of one zl_bp_step (eagerly or into a capture).
+void bp_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S) {
+  const int N = B * S, K = c->K;
+  const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+  cudaStream_t s = c->ch[1].s;
+  rec(c->ev_start, c->user);
+  wait_ev(s, c->ev_start);
+  wait_ev(c->aux, c->ev_start);    // (keeps every stream of the context in a capture)
+  if (!c->capturing)
     for (int k = 2; k <= K; ++k) {   // previous work of the other chunk streams
       rec(c->ch[k].ev_done, c->ch[k].s);
       wait_ev(s, c->ch[k].ev_done);
     }
-    std::vector<void*> h(K + 1, nullptr);
-    std::vector<ChunkActs> acts(K + 1);
-    h[0] = palloc(c, hb, s);
-    launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h[0], N, S, c->d, c->V, c->d_err, s);
-    for (int k = 1; k <= K; ++k) {
-      h[k] = palloc(c, hb, s);
-      chunk_fwd_save(c, c->ch[k], h[k - 1], h[k], B, S, acts[k], s);
+  std::vector<void*> h(K + 1, nullptr);
+  std::vector<ChunkActs> acts(K + 1);
+  h[0] = palloc(c, hb, s);
+  launch_embed(c->dt, ids, c->tok_emb, c->pos_emb, h[0], N, S, c->d, c->V, c->d_err, s);
+  for (int k = 1; k <= K; ++k) {
+    h[k] = palloc(c, hb, s);
+    chunk_fwd_save(c, c->ch[k], h[k - 1], h[k], B, S, acts[k], s);
+  }
+  void* z = palloc(c, zb, s);
+  ReadoutSave rs;
+  readout_fwd(c, h[K], z, &rs, N, s);
+  void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
+  pfree(z, s);
+  void* dh = palloc(c, hb, s);
+  void* dh2 = palloc(c, hb, s);
+  readout_bwd(c, h[K], rs, dz, dh, N, s);
+  pfree(dz, s);
+  for (int k = K; k >= 1; --k) {
+    chunk_bwd(c, c->ch[k], acts[k], dh, k > 1 ? dh2 : nullptr, B, S, s);
+    std::swap(dh, dh2);
+    pfree(acts[k].mem, s);
+    pfree(h[k], s);
+  }
+  pfree(h[0], s);
+  pfree(dh, s);
+  pfree(dh2, s);
+  for (int k = 1; k <= K; ++k) {
+    if (k > 1) {   // the optimizer step of chunk k stays on its own stream
+      rec(c->ch[1].ev_done, s);
+      wait_ev(c->ch[k].s, c->ch[1].ev_done);
     }
-    void* z = palloc(c, zb, s);
-    ReadoutSave rs;
-    readout_fwd(c, h[K], z, &rs, N, s);
-    void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
-    pfree(z, s);
-    void* dh = palloc(c, hb, s);
-    void* dh2 = palloc(c, hb, s);
-    readout_bwd(c, h[K], rs, dz, dh, N, s);
-    pfree(dz, s);
-    for (int k = K; k >= 1; --k) {
-      chunk_bwd(c, c->ch[k], acts[k], dh, k > 1 ? dh2 : nullptr, B, S, s);
-      std::swap(dh, dh2);
-      pfree(acts[k].mem, s);
-      pfree(h[k], s);
-    }
-    pfree(h[0], s);
-    pfree(dh, s);
-    pfree(dh2, s);
-    for (int k = 1; k <= K; ++k) {
-      if (k > 1) {   // the optimizer step of chunk k stays on its own stream
-        rec(c->ch[1].ev_done, s);
-        wait_ev(c->ch[k].s, c->ch[1].ev_done);
-      }
-      adamw_window(c, c->ch[k], k == 1 ? s : c->ch[k].s, false);
-    }
-    c->last_nloss = 1;
-    for (int k = 1; k <= K; ++k) c->ch[k].done += 1;
+    adamw_window(c, c->ch[k], k == 1 ? s : c->ch[k].s, false);
+  }
+  c->last_nloss = 1;
+  for (int k = 1; k <= K; ++k) c->ch[k].done += 1;
+}
+
+}  // namespace
+
+extern "C" {
+
+zl_status zl_bp_step(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int S, float* loss_out) {
+  if (!c || !ids || !labels) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  return guarded(c, [&]() -> zl_status {
+    check_bs(c, B, S);
+    const int K = c->K;
+    const bool graphed = run_graph(
+        c, c->bg, ids, labels, B, S, [&](const int32_t* gi, const int32_t* gl) { bp_enqueue(c, gi, gl, B, S); },
+        [&]() {
+          for (int k = 1; k <= K; ++k) {
+            c->ch[k].done += 1;
+            c->ch[k].t += 1;
+          }
+          c->last_nloss = 1;
+        });
+    if (!graphed) bp_enqueue(c, ids, labels, B, S);
+    const cudaStream_t s = c->ch[1].s;
     if (loss_out) {
       CK(cudaMemcpyAsync(c->h_losses, c->d_losses, 4, cudaMemcpyDeviceToHost, s));
       sync_all(c, -1);
@@ -1576,6 +1734,15 @@ zl_status zl_peak_bytes(zl_ctx* c, size_t* peak, size_t* current) {
     uint64_t hi = 0, cur = 0;
     CK(cudaMemPoolGetAttribute(c->pool, cudaMemPoolAttrUsedMemHigh, &hi));
     CK(cudaMemPoolGetAttribute(c->pool, cudaMemPoolAttrUsedMemCurrent, &cur));
+    if (c->cfg.graph) {   // a captured step's activations live in the device's graph memory
+      int dev = 0;
+      uint64_t ghi = 0, gcur = 0;
+      CK(cudaGetDevice(&dev));
+      CK(cudaDeviceGetGraphMemAttribute(dev, cudaGraphMemAttrUsedMemHigh, &ghi));
+      CK(cudaDeviceGetGraphMemAttribute(dev, cudaGraphMemAttrUsedMemCurrent, &gcur));
+      hi += ghi;
+      cur += gcur;
+    }
     if (peak) *peak = c->static_bytes + hi;
     if (current) *current = c->static_bytes + cur;
     return ZL_OK;
@@ -1588,6 +1755,11 @@ zl_status zl_reset_peak(zl_ctx* c) {
     sync_all(c, -1);
     uint64_t zero = 0;
     CK(cudaMemPoolSetAttribute(c->pool, cudaMemPoolAttrUsedMemHigh, &zero));
+    if (c->cfg.graph) {
+      int dev = 0;
+      CK(cudaGetDevice(&dev));
+      CK(cudaDeviceSetGraphMemAttribute(dev, cudaGraphMemAttrUsedMemHigh, &zero));
+    }
     return ZL_OK;
   });
 }

@@ -905,11 +905,26 @@ void launch_loss_reduce(const float* row_loss, int N, const int* count, float* o
 // ------------------------------------------------------------------------------------------
 // AdamW over one chunk's contiguous parameter slab (decoupled weight decay, bias correction).
 // ------------------------------------------------------------------------------------------
-__global__ void adamw_k(float4* __restrict__ th, float4* __restrict__ g, float4* __restrict__ m,
-                        float4* __restrict__ v, __nv_bfloat162* __restrict__ comp, size_t n4, float lr, float b1,
-                        float b2, float eps, float wd, float bc1, float bc2, float gscale) {
+// Advances a chunk's optimizer step count t (device memory, so a replayed CUDA graph keeps counting)
+// and writes this step's learning rate and bias corrections: hp = {lr_t, 1 - beta1^t, 1 - beta2^t}.
+__global__ void adamw_tick_k(long long* __restrict__ t, float* __restrict__ hp, float lr0, int schedule,
+                             float gamma, float b1, float b2) {
   pdl_wait();
   pdl_trigger();
+  const long long tt = *t + 1;
+  *t = tt;
+  const double lr = schedule == 1 ? (double)lr0 / sqrt((double)(tt - 1) + (double)gamma) : (double)lr0;
+  hp[0] = (float)lr;
+  hp[1] = (float)(1.0 - pow((double)b1, (double)tt));
+  hp[2] = (float)(1.0 - pow((double)b2, (double)tt));
+}
+
+__global__ void adamw_k(float4* __restrict__ th, float4* __restrict__ g, float4* __restrict__ m,
+                        float4* __restrict__ v, __nv_bfloat162* __restrict__ comp, size_t n4,
+                        const float* __restrict__ hp, float b1, float b2, float eps, float wd, float gscale) {
+  pdl_wait();
+  pdl_trigger();
+  const float lr = hp[0], bc1 = hp[1], bc2 = hp[2];
   const float decay = 1.f - lr * wd;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
     float4 t = th[i], gg = g[i], mm = m[i], vv = v[i];
@@ -930,13 +945,16 @@ __global__ void adamw_k(float4* __restrict__ th, float4* __restrict__ g, float4*
   }
 }
 
-void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, float lr, float b1, float b2,
-                  float eps, float wd, float bc1, float bc2, float gscale, cudaStream_t s) {
-  note_launch(1);
+void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, long long* t, float* hp,
+                  float lr0, int schedule, float gamma, float b1, float b2, float eps, float wd, float gscale,
+                  cudaStream_t s) {
+  note_launch(2);
+  launch_pdl(adamw_tick_k, 1, 1, 0, s, t, hp, lr0, schedule, gamma, b1, b2);
   const size_t n4 = n / 4;   // slabs are padded to a multiple of 64 elements
+  if (n4 == 0) return;
   const int th = 256, gr = grid_for(n4, th, 152 * 8);
-  launch_pdl(adamw_k, gr, th, 0, s, (float4*)theta, (float4*)g, (float4*)m, (float4*)v, (__nv_bfloat162*)comp, n4, lr,
-                            b1, b2, eps, wd, bc1, bc2, gscale);
+  launch_pdl(adamw_k, gr, th, 0, s, (float4*)theta, (float4*)g, (float4*)m, (float4*)v, (__nv_bfloat162*)comp, n4,
+             (const float*)hp, b1, b2, eps, wd, gscale);
 }
 
 __global__ void f32_to_bf16_k(const float* __restrict__ a, bf16* __restrict__ b, size_t n) {

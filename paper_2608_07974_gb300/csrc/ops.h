@@ -60,9 +60,12 @@ void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labe
 // *out = sum(row_loss) / count.
 void launch_loss_reduce(const float* row_loss, int N, const int* count, float* out, cudaStream_t s);
 
-// One AdamW step over a contiguous slab; zeroes g; refreshes the bf16 copy if comp != NULL.
-void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, float lr, float b1,
-                  float b2, float eps, float wd, float bc1, float bc2, float gscale, cudaStream_t s);
+// One AdamW step over a contiguous slab; zeroes g; refreshes the bf16 copy if comp != NULL. The step
+// count t lives in device memory (advanced here by one); hp (3 floats) receives lr_t and the bias
+// corrections; lr_t = lr0 or lr0 / sqrt(t - 1 + gamma) (schedule 1).
+void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, long long* t, float* hp,
+                  float lr0, int schedule, float gamma, float b1, float b2, float eps, float wd, float gscale,
+                  cudaStream_t s);
 void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
 
 // GEMM (row-major): mode 0: C = A[M,K] B[N,K]^T (+ bias[N]) (+ R[M,N]); mode 1: C = A[M,K] B[K,N] (+ R);
