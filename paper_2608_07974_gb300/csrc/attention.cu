@@ -158,10 +158,14 @@ inline int warps_grid(long rows) { return (int)((rows * 32 + 255) / 256); }
 }  // namespace
 
 bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s);
+bool attn_fwd_tcgen05(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
+                      unsigned* err);
 bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
                  int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool);
 
-void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s) {
+void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
+              unsigned* err) {
+  if (dt == BF16 && attn_fwd_tcgen05(qkv, out, lse, B, S, H, Hkv, hd, s, err)) return;
   note_launch(1);
   if (dt == BF16 && attn_fwd_tc(qkv, out, lse, B, S, H, Hkv, hd, s)) return;
   const float scale = 1.f / sqrtf((float)hd);
