@@ -162,6 +162,8 @@ bool attn_fwd_tcgen05(const void* qkv, void* out, float* lse, int B, int S, int 
                       unsigned* err);
 bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
                  int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool);
+bool attn_bwd_tcgen05(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv,
+                      int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err);
 
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
               unsigned* err) {
@@ -175,10 +177,11 @@ void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int 
 }
 
 void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const float* lse, float* Dbuf, void* dqkv,
-              int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool) {
+              int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
   note_launch(dt == BF16 ? (H > Hkv ? 3 : 2) : 3);
   const float scale = 1.f / sqrtf((float)hd);
   const int gq = warps_grid((long)B * H * S), gk = warps_grid((long)B * Hkv * S);
+  if (dt == BF16 && attn_bwd_tcgen05(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s, pool, err)) return;
   if (dt == BF16 && attn_bwd_tc(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s, pool)) return;
   if (dt == BF16) {
     attn_bwd_d_k<bf16><<<gq, 256, 0, s>>>((const bf16*)out, (const bf16*)dout, Dbuf, B, S, H, hd);

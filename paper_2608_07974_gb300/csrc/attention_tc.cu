@@ -645,6 +645,12 @@ bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, in
   return true;
 }
 
+void launch_reduce_dkv(const float* part, void* dqkv, int NS, int H, int Hkv, int hd, float scale, cudaStream_t s) {
+  const size_t total = (size_t)NS * Hkv * (hd / 2);
+  const int blocks = (int)std::min<size_t>((total + 255) / 256, 152 * 16);
+  launch_pdl(fa::reduce_dkv_k, blocks, 256, 0, s, part, (bf16*)dqkv, NS, H, Hkv, hd, scale);
+}
+
 bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
                  int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool) {
   if (hd > 128 || hd % 2) return false;

@@ -1,6 +1,7 @@
-// Causal attention forward on the 5th-generation tensor cores (sm_103a), head dim 128 (the kernel is
-// written for 64 and 128).
+// Causal attention on the 5th-generation tensor cores (sm_103a): the forward for head dim 128 (the
+// kernel is written for 64 and 128), the backward for head dims 64 and 128.
 //
+// Forward.
 // One CTA per 128 query rows of one (batch, head). TMA brings Q once and K / V tiles of 128 keys
 // through a stage ring (128-byte swizzle; a 3-D tensor map over [batch, token, feature] reads rows past
 // the sequence end as zeros); one thread issues tcgen05.mma with fp32 accumulators in TMEM; eight
@@ -332,6 +333,513 @@ __global__ void __launch_bounds__(NTHR, 1)
   }
 }
 
+// ==============================================================================================
+// Backward: two kernels, each a fixed-order sum per output row (no atomics).
+//   dQ kernel: one CTA per 128 queries; 64-key inner blocks j: S = Q K_j^T, dP = dO V_j^T (TMEM),
+//              dS = P * (dP - D) (shared memory, bf16), dQ += dS K_j (TMEM); also writes D = rowsum(dO * O).
+//   dK/dV kernel: one CTA per 128 keys; 64-query inner blocks i: S^T = K Q_i^T, dP^T = V dO_i^T,
+//              P^T and dS^T (shared memory), dV += P^T dO_i, dK += dS^T Q_i.
+// The 128 x 64 S / dP blocks are double-buffered in TMEM (columns 0 and 128, dP 64 columns after S); the
+// accumulators start at column 256. A 64-row tile of Q / dO / K / V is one K-major [64 x 64] block per 64
+// head-dim columns (8 KB each); the same bytes are the MN-major B operand of the accumulating product
+// (16-row steps 2 KB apart, head-dim blocks 8 KB apart).
+// ==============================================================================================
+constexpr int IB = 64;   // inner block rows
+
+template <int HD>
+struct BCfg {
+  static constexpr int T128 = 128 * HD * 2;
+  static constexpr int T64 = IB * HD * 2;
+  static constexpr int NST = HD == 64 ? 4 : 3;   // pipeline stages of (Q_i, dO_i) or (K_j, V_j)
+  static constexpr int OPB = 128 * IB * 2;       // one bf16 [128 x 64] operand (P^T, dS^T or dS)
+  static constexpr int SMEM_DKV = 2 * T128 + NST * 2 * T64 + 2 * OPB + NST * 2 * IB * 4 + 256 + 1024;
+  static constexpr int SMEM_DQ = 2 * T128 + NST * 2 * T64 + OPB + 2 * 128 * 4 + 256 + 1024;
+};
+
+// Stores 32 bf16 values (64 bytes: 16-byte chunks 4 half .. 4 half + 3) into row r of a swizzled
+// [128 x 64] K-major operand.
+__device__ __forceinline__ void put_quarter_row(uint8_t* g, int half, int r, const uint32_t* pk) {
+  uint8_t* row = g + r * 128;
+#pragma unroll
+  for (int u = 0; u < 4; ++u)
+    *reinterpret_cast<uint4*>(row + (((4 * half + u) ^ (r & 7)) << 4)) =
+        make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+}
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Warp-uniform bounded wait by lane 0.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, unsigned* err) {
+  int w = 1;
+  if ((threadIdx.x & 31) == 0) w = mbar_wait(bar, parity, abort_flag, err) ? 1 : 0;
+  return __shfl_sync(0xffffffffu, w, 0) != 0;
+}
+
+// Lane 0 of the producer, after a failed wait: lets the copies it issued land (bounded) before exit.
+template <int N>
+__device__ __forceinline__ void drain(uint64_t* full, const int* issued, uint64_t* first) {
+  for (int s = 0; s < N; ++s) {
+    if (issued[s] < 0) continue;
+    const unsigned long long t0 = gtimer();
+    while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
+    }
+  }
+  const unsigned long long t0 = gtimer();
+  while (!mbar_test(first, 0) && gtimer() - t0 < 100000000ull) {
+  }
+}
+
+__device__ __forceinline__ void tmem_alloc512(uint32_t* dst) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(dst)), "r"(512u)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+// Warp 1 after the final __syncthreads: waits (bounded) for the last MMAs, frees the TMEM.
+__device__ __forceinline__ void tmem_release(uint64_t* fin, uint32_t tmem) {
+  if ((threadIdx.x & 31) == 0) {
+    const unsigned long long t0 = gtimer();
+    while (!mbar_test(fin, 0) && gtimer() - t0 < 100000000ull) {
+    }
+  }
+  __syncwarp();
+  fence_after();
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512u) : "memory");
+}
+
+// dQ (and D) kernel. Maps: tq = qkv in 128-row boxes, tdo = dO in 128-row boxes, tkv = qkv in 64-row boxes.
+template <int HD>
+__global__ void __launch_bounds__(NTHR, 1)
+    attn_bwd_dq_tg_k(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tdo,
+                     const __grid_constant__ CUtensorMap tkv, const bf16* __restrict__ outp,
+                     const bf16* __restrict__ dout, const float* __restrict__ lse, float* __restrict__ Dv,
+                     bf16* __restrict__ dqkv, int S, int H, int Hkv, float scale, unsigned* err) {
+  using C_ = BCfg<HD>;
+  constexpr int NST = C_::NST;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sq = smem;
+  uint8_t* sdo = sq + C_::T128;
+  uint8_t* sst = sdo + C_::T128;                  // stage s: K_j at s * 2 T64, V_j after it
+  uint8_t* sds = sst + NST * 2 * C_::T64;
+  float* dpart = (float*)(sds + C_::OPB);         // [2][128] halves of D
+  uint64_t* full = (uint64_t*)(dpart + 256);
+  uint64_t* empty = full + NST;
+  uint64_t* qfull = empty + NST;
+  uint64_t* sfull = qfull + 1;                    // [2]
+  uint64_t* sempty = sfull + 2;                   // [2]
+  uint64_t* dsfull = sempty + 2;
+  uint64_t* dsempty = dsfull + 1;
+  uint64_t* ofull = dsempty + 1;
+  uint64_t* fin = ofull + 1;
+  uint32_t* tbase = (uint32_t*)(fin + 1);
+  volatile int* abort_flag = (volatile int*)(tbase + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x, b = blockIdx.y, qb = gridDim.z - 1 - blockIdx.z;   // longest first
+  const int kvh = h / (H / Hkv);
+  const int q0 = qb * 128;
+  const int nkb = min(2 * qb + 2, (S + IB - 1) / IB);
+  const int ld = (H + 2 * Hkv) * HD, HDall = H * HD;
+  const int xq = h * HD, xk = (H + kvh) * HD, xv = (H + Hkv + kvh) * HD;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    mbar_init(qfull, 1);
+    for (int u = 0; u < 2; ++u) { mbar_init(&sfull[u], 1); mbar_init(&sempty[u], NSM); }
+    mbar_init(dsfull, NSM);
+    mbar_init(dsempty, 1);
+    mbar_init(ofull, 1);
+    mbar_init(fin, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc512(tbase);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tbase;
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int issued[NST];
+#pragma unroll
+      for (int s = 0; s < NST; ++s) issued[s] = -1;
+      mbar_expect_tx(qfull, 2 * C_::T128);
+#pragma unroll
+      for (int c = 0; c < HD / 64; ++c) {
+        tma3d(sq + c * 16384, &tq, qfull, xq + 64 * c, q0, b);
+        tma3d(sdo + c * 16384, &tdo, qfull, h * HD + 64 * c, q0, b);
+      }
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int j = 0; j < nkb; ++j) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+        mbar_expect_tx(&full[stage], 2 * C_::T64);
+        issued[stage] = (int)phase;
+        uint8_t* st = sst + stage * 2 * C_::T64;
+#pragma unroll
+        for (int c = 0; c < HD / 64; ++c) {
+          tma3d(st + c * 8192, &tkv, &full[stage], xk + 64 * c, j * IB, b);
+          tma3d(st + C_::T64 + c * 8192, &tkv, &full[stage], xv + 64 * c, j * IB, b);
+        }
+        if (++stage == NST) { stage = 0; phase ^= 1u; }
+      }
+      if (!ok) drain<NST>(full, issued, qfull);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t id_s = idesc_f16(128, IB, false, false);
+      constexpr uint32_t id_q = idesc_f16(128, HD, false, true);
+      const uint32_t q_addr = su32(sq), do_addr = su32(sdo), ds_addr = su32(sds);
+      bool ok = mbar_wait(qfull, 0, abort_flag, err);
+      fence_after();
+      int stage = 0, pstage = 0;
+      uint32_t phase = 0;
+      auto dq = [&](int jb, int st) -> bool {   // dQ += dS_jb K_jb
+        if (!mbar_wait(dsfull, (uint32_t)(jb & 1), abort_flag, err)) return false;
+        fence_after();
+        const uint32_t k_addr = su32(sst + st * 2 * C_::T64);
+#pragma unroll
+        for (int ks = 0; ks < IB / 16; ++ks)
+          mma_bf16(tmem + 256, sdesc(ds_addr + ks * 32, 16, 1024), sdesc(k_addr + ks * 2048, 8192, 1024), id_q,
+                   (jb > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&empty[st]);
+        mma_commit(dsempty);
+        return true;
+      };
+      for (int j = 0; ok && j < nkb; ++j) {
+        const int buf = j & 1;
+        if (!mbar_wait(&sempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+        if (!mbar_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
+        fence_after();
+        const uint32_t k_addr = su32(sst + stage * 2 * C_::T64), v_addr = k_addr + C_::T64;
+        const uint32_t ts = tmem + (uint32_t)(buf * 128);
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          const int kq = ks / 4, kr = ks % 4;
+          mma_bf16(ts, sdesc(q_addr + kq * 16384 + kr * 32, 16, 1024), sdesc(k_addr + kq * 8192 + kr * 32, 16, 1024),
+                   id_s, ks > 0 ? 1u : 0u);
+          mma_bf16(ts + IB, sdesc(do_addr + kq * 16384 + kr * 32, 16, 1024),
+                   sdesc(v_addr + kq * 8192 + kr * 32, 16, 1024), id_s, ks > 0 ? 1u : 0u);
+        }
+        mma_commit(&sfull[buf]);
+        if (j > 0 && !dq(j - 1, pstage)) { ok = false; break; }
+        pstage = stage;
+        if (++stage == NST) { stage = 0; phase ^= 1u; }
+      }
+      if (ok && !dq(nkb - 1, pstage)) ok = false;
+      if (ok) mma_commit(ofull);
+      mma_commit(fin);
+    }
+  } else {
+    const int quad = warp & 3, half = (warp - 2) / 4;
+    const int r = quad * 32 + lane;
+    const int q = q0 + r, qc = min(q, S - 1);
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    const float sl2 = scale * kL2e;
+    const size_t si = ((size_t)b * H + h) * S + qc;
+    const float lse2 = q < S ? lse[si] * kL2e : INFINITY;
+    {   // D = rowsum(dO * O): each half sums half of the row, fixed-order combination
+      const bf16* orow = outp + ((size_t)b * S + qc) * HDall + (size_t)h * HD + half * (HD / 2);
+      const bf16* grow = dout + ((size_t)b * S + qc) * HDall + (size_t)h * HD + half * (HD / 2);
+      float acc = 0.f;
+#pragma unroll
+      for (int c = 0; c < HD / 2; c += 8) {
+        float o8[8], g8[8];
+        Vec8<bf16>::load(orow + c, o8);
+        Vec8<bf16>::load(grow + c, g8);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc = fmaf(o8[e], g8[e], acc);
+      }
+      dpart[half * 128 + r] = acc;
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * NSM) : "memory");
+    const float Dq = dpart[r] + dpart[128 + r];
+    if (q < S && half == 0) Dv[si] = Dq;
+    const int qlim = min(q, S - 1);
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      const int buf = j & 1;
+      if (!warp_wait(&sfull[buf], (uint32_t)(j >> 1) & 1u, abort_flag, err)) { ok = false; break; }
+      fence_after();
+      float sv[32], dp[32];
+      tmem_ld32(trow + (uint32_t)(buf * 128 + half * 32), sv);
+      tmem_ld32(trow + (uint32_t)(buf * 128 + IB + half * 32), dp);
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sempty[buf]);
+      const int kmax = qlim - (j * IB + half * 32);   // columns e <= kmax are causal and inside S
+      uint32_t pk[16];
+#pragma unroll
+      for (int e = 0; e < 32; e += 2) {
+        const float p0 = e <= kmax ? ex2(fmaf(sv[e], sl2, -lse2)) : 0.f;
+        const float p1 = e + 1 <= kmax ? ex2(fmaf(sv[e + 1], sl2, -lse2)) : 0.f;
+        pk[e / 2] = pack2(p0 * (dp[e] - Dq), p1 * (dp[e + 1] - Dq));
+      }
+      if (!warp_wait(dsempty, ((uint32_t)j & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+      put_quarter_row(sds, half, r, pk);
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(dsfull);
+    }
+    if (ok && warp_wait(ofull, 0, abort_flag, err)) {
+      fence_after();
+      bf16* drow = dqkv + ((size_t)b * S + qc) * ld + (size_t)h * HD;
+#pragma unroll
+      for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
+        float v[32];
+        tmem_ld32(trow + 256 + (uint32_t)c, v);
+        if (q < S) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] *= scale;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) Vec8<bf16>::store(drow + c + 8 * u, v + 8 * u);
+        }
+      }
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_release(fin, tmem);
+}
+
+// dK / dV kernel. One CTA per 128 keys of one query head (grouped heads: fp32 partials
+// part[2][H][B*S][HD], dK unscaled, summed per group afterwards) or of one KV head (H == Hkv: bf16 straight
+// into dqkv). Maps: tkv = qkv in 128-row boxes, tq = qkv in 64-row boxes, tdo = dO in 64-row boxes.
+template <int HD>
+__global__ void __launch_bounds__(NTHR, 1)
+    attn_bwd_dkv_tg_k(const __grid_constant__ CUtensorMap tkv, const __grid_constant__ CUtensorMap tq,
+                      const __grid_constant__ CUtensorMap tdo, const float* __restrict__ lse,
+                      const float* __restrict__ Dv, bf16* __restrict__ dqkv, int S, int H, int Hkv, float scale,
+                      float* __restrict__ part, unsigned* err) {
+  using C_ = BCfg<HD>;
+  constexpr int NST = C_::NST;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sk = smem;
+  uint8_t* sv = sk + C_::T128;
+  uint8_t* sst = sv + C_::T128;                   // stage s: Q_i at s * 2 T64, dO_i after it
+  uint8_t* sp = sst + NST * 2 * C_::T64;          // P^T
+  uint8_t* sds = sp + C_::OPB;                    // dS^T
+  float* stats = (float*)(sds + C_::OPB);         // stage s: lse2[64], D[64]
+  uint64_t* full = (uint64_t*)(stats + NST * 2 * IB);
+  uint64_t* empty = full + NST;
+  uint64_t* kvfull = empty + NST;
+  uint64_t* sfull = kvfull + 1;                   // [2]
+  uint64_t* sempty = sfull + 2;                   // [2]
+  uint64_t* pfull = sempty + 2;
+  uint64_t* pempty = pfull + 1;
+  uint64_t* ofull = pempty + 1;
+  uint64_t* fin = ofull + 1;
+  uint32_t* tbase = (uint32_t*)(fin + 1);
+  volatile int* abort_flag = (volatile int*)(tbase + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x, b = blockIdx.y, kb = blockIdx.z;   // key block 0 (the longest) first
+  const int kvh = part ? h / (H / Hkv) : h;
+  const int k0 = kb * 128, i0 = 2 * kb;
+  const int nit = (S + IB - 1) / IB - i0;
+  const int ld = (H + 2 * Hkv) * HD;
+  const int xq = h * HD, xk = (H + kvh) * HD, xv = (H + Hkv + kvh) * HD;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 2); mbar_init(&empty[s], 1); }
+    mbar_init(kvfull, 1);
+    for (int u = 0; u < 2; ++u) { mbar_init(&sfull[u], 1); mbar_init(&sempty[u], NSM); }
+    mbar_init(pfull, NSM);
+    mbar_init(pempty, 1);
+    mbar_init(ofull, 1);
+    mbar_init(fin, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc512(tbase);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tbase;
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    // lane 0: TMA of K, V once and of (Q_i, dO_i) per block; every lane: two of the block's lse2 and D
+    int issued[NST];
+#pragma unroll
+    for (int s = 0; s < NST; ++s) issued[s] = -1;
+    if (lane == 0) {
+      mbar_expect_tx(kvfull, 2 * C_::T128);
+#pragma unroll
+      for (int c = 0; c < HD / 64; ++c) {
+        tma3d(sk + c * 16384, &tkv, kvfull, xk + 64 * c, k0, b);
+        tma3d(sv + c * 16384, &tkv, kvfull, xv + 64 * c, k0, b);
+      }
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int it = 0; it < nit; ++it) {
+      const int qi0 = (i0 + it) * IB;
+      if (!warp_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+      uint8_t* st = sst + stage * 2 * C_::T64;
+      if (lane == 0) {
+        mbar_expect_tx(&full[stage], 2 * C_::T64);
+        issued[stage] = (int)phase;
+#pragma unroll
+        for (int c = 0; c < HD / 64; ++c) {
+          tma3d(st + c * 8192, &tq, &full[stage], xq + 64 * c, qi0, b);
+          tma3d(st + C_::T64 + c * 8192, &tdo, &full[stage], h * HD + 64 * c, qi0, b);
+        }
+      }
+      float* sl = stats + stage * 2 * IB;
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int cq = lane * 2 + u, qq = qi0 + cq;
+        const size_t si = ((size_t)b * H + h) * S + (qq < S ? qq : 0);
+        sl[cq] = qq < S ? lse[si] * kL2e : INFINITY;
+        sl[IB + cq] = qq < S ? Dv[si] : 0.f;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&full[stage]);
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (!ok && lane == 0) drain<NST>(full, issued, kvfull);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t id_s = idesc_f16(128, IB, false, false);
+      constexpr uint32_t id_g = idesc_f16(128, HD, false, true);
+      const uint32_t k_addr = su32(sk), v_addr = su32(sv), p_addr = su32(sp), ds_addr = su32(sds);
+      bool ok = mbar_wait(kvfull, 0, abort_flag, err);
+      fence_after();
+      int stage = 0, pstage = 0;
+      uint32_t phase = 0;
+      auto grads = [&](int ib, int st) -> bool {   // dV += P^T dO_ib, dK += dS^T Q_ib
+        if (!mbar_wait(pfull, (uint32_t)(ib & 1), abort_flag, err)) return false;
+        fence_after();
+        const uint32_t qa = su32(sst + st * 2 * C_::T64), da = qa + C_::T64;
+#pragma unroll
+        for (int ks = 0; ks < IB / 16; ++ks) {
+          const uint32_t acc = (ib > 0 || ks > 0) ? 1u : 0u;
+          mma_bf16(tmem + 256, sdesc(p_addr + ks * 32, 16, 1024), sdesc(da + ks * 2048, 8192, 1024), id_g, acc);
+          mma_bf16(tmem + 256 + HD, sdesc(ds_addr + ks * 32, 16, 1024), sdesc(qa + ks * 2048, 8192, 1024), id_g,
+                   acc);
+        }
+        mma_commit(&empty[st]);
+        mma_commit(pempty);
+        return true;
+      };
+      for (int it = 0; ok && it < nit; ++it) {
+        const int buf = it & 1;
+        if (!mbar_wait(&sempty[buf], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+        if (!mbar_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
+        fence_after();
+        const uint32_t qa = su32(sst + stage * 2 * C_::T64), da = qa + C_::T64;
+        const uint32_t ts = tmem + (uint32_t)(buf * 128);
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          const int kq = ks / 4, kr = ks % 4;
+          mma_bf16(ts, sdesc(k_addr + kq * 16384 + kr * 32, 16, 1024), sdesc(qa + kq * 8192 + kr * 32, 16, 1024),
+                   id_s, ks > 0 ? 1u : 0u);
+          mma_bf16(ts + IB, sdesc(v_addr + kq * 16384 + kr * 32, 16, 1024), sdesc(da + kq * 8192 + kr * 32, 16, 1024),
+                   id_s, ks > 0 ? 1u : 0u);
+        }
+        mma_commit(&sfull[buf]);
+        if (it > 0 && !grads(it - 1, pstage)) { ok = false; break; }
+        pstage = stage;
+        if (++stage == NST) { stage = 0; phase ^= 1u; }
+      }
+      if (ok && !grads(nit - 1, pstage)) ok = false;
+      if (ok) mma_commit(ofull);
+      mma_commit(fin);
+    }
+  } else {
+    const int quad = warp & 3, half = (warp - 2) / 4;
+    const int r = quad * 32 + lane;                 // key row = TMEM lane
+    const int key = k0 + r;
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    const float sl2 = scale * kL2e;
+    bool ok = true;
+    int stage = 0;
+    uint32_t phase = 0;
+    for (int it = 0; it < nit; ++it) {
+      const int buf = it & 1;
+      if (!warp_wait(&sfull[buf], (uint32_t)(it >> 1) & 1u, abort_flag, err)) { ok = false; break; }
+      fence_after();
+      float sv[32], dp[32];
+      tmem_ld32(trow + (uint32_t)(buf * 128 + half * 32), sv);
+      tmem_ld32(trow + (uint32_t)(buf * 128 + IB + half * 32), dp);
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sempty[buf]);
+      // this stage's lse2 and D: its full phase has completed (the S MMA waited on it); the wait
+      // orders the producer's stores before these loads
+      if (!warp_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
+      const float* sl = stats + stage * 2 * IB + half * 32;
+      const float* sd = sl + IB;
+      const int qbase = (i0 + it) * IB + half * 32;   // query of column 0 of this thread's 32
+      const int qlo = key - qbase;                     // columns e >= qlo are causal
+      const int qhi = S - qbase;                       // columns e < qhi are inside S
+      const bool krow = key < S;
+      uint32_t pk[16], dk[16];
+#pragma unroll
+      for (int e = 0; e < 32; e += 2) {
+        const bool v0 = krow && e >= qlo && e < qhi;
+        const bool v1 = krow && e + 1 >= qlo && e + 1 < qhi;
+        const float p0 = v0 ? ex2(fmaf(sv[e], sl2, -sl[e])) : 0.f;
+        const float p1 = v1 ? ex2(fmaf(sv[e + 1], sl2, -sl[e + 1])) : 0.f;
+        pk[e / 2] = pack2(p0, p1);
+        dk[e / 2] = pack2(p0 * (dp[e] - sd[e]), p1 * (dp[e + 1] - sd[e + 1]));
+      }
+      if (!warp_wait(pempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+      put_quarter_row(sp, half, r, pk);
+      put_quarter_row(sds, half, r, dk);
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(pfull);
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (ok && warp_wait(ofull, 0, abort_flag, err)) {
+      fence_after();
+      const int kc = min(key, S - 1);
+      const size_t NS = (size_t)gridDim.y * S;
+#pragma unroll
+      for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
+        float gv[32], gk[32];
+        tmem_ld32(trow + 256 + (uint32_t)c, gv);
+        tmem_ld32(trow + 256 + HD + (uint32_t)c, gk);
+        if (key < S) {
+          if (part) {
+            float* pk2 = part + ((size_t)h * NS + (size_t)b * S + kc) * HD + c;
+            float* pv2 = pk2 + (size_t)H * NS * HD;
+#pragma unroll
+            for (int e = 0; e < 32; e += 4) {
+              *reinterpret_cast<float4*>(pk2 + e) = make_float4(gk[e], gk[e + 1], gk[e + 2], gk[e + 3]);
+              *reinterpret_cast<float4*>(pv2 + e) = make_float4(gv[e], gv[e + 1], gv[e + 2], gv[e + 3]);
+            }
+          } else {
+            bf16* dkr = dqkv + ((size_t)b * S + kc) * ld + (size_t)xk + c;
+            bf16* dvr = dqkv + ((size_t)b * S + kc) * ld + (size_t)xv + c;
+#pragma unroll
+            for (int e = 0; e < 32; ++e) gk[e] *= scale;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              Vec8<bf16>::store(dkr + 8 * u, gk + 8 * u);
+              Vec8<bf16>::store(dvr + 8 * u, gv + 8 * u);
+            }
+          }
+        }
+      }
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_release(fin, tmem);
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
 
 bool enc_init() {
@@ -381,6 +889,44 @@ bool fwd_launch(const void* qkv, void* out, float* lse, int B, int S, int H, int
                     err) == cudaSuccess;
 }
 
+template <int HD>
+bool bwd_launch(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B,
+                int S, int H, int Hkv, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
+  using C_ = BCfg<HD>;
+  static bool attr = false;
+  auto kq = attn_bwd_dq_tg_k<HD>;
+  auto kkv = attn_bwd_dkv_tg_k<HD>;
+  if (!attr) {
+    if (cudaFuncSetAttribute(kq, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM_DQ) != cudaSuccess ||
+        cudaFuncSetAttribute(kkv, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM_DKV) != cudaSuccess)
+      return false;
+    attr = true;
+  }
+  const int W = (H + 2 * Hkv) * HD, Wo = H * HD;
+  CUtensorMap q128, q64, do128, do64;
+  if (!qkv_map(&q128, qkv, B, S, W, 128) || !qkv_map(&q64, qkv, B, S, W, IB) || !qkv_map(&do128, dout, B, S, Wo, 128) ||
+      !qkv_map(&do64, dout, B, S, Wo, IB))
+    return false;
+  float* part = nullptr;
+  if (H > Hkv) {   // grouped heads: one CTA per query head, then a fixed-order group reduction
+    const size_t bytes = 2ull * H * B * S * HD * sizeof(float);
+    cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&part, bytes, pool, s) : cudaMallocAsync((void**)&part, bytes, s);
+    if (e != cudaSuccess) { cudaGetLastError(); return false; }
+  }
+  const float scale = 1.f / sqrtf((float)HD);
+  const int nqb = (S + 127) / 128;
+  cudaError_t e = launch_pdl(kq, dim3(H, B, nqb), NTHR, C_::SMEM_DQ, s, q128, do128, q64, (const bf16*)out,
+                             (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, scale, err);
+  if (e == cudaSuccess)
+    e = launch_pdl(kkv, dim3(part ? H : Hkv, B, nqb), NTHR, C_::SMEM_DKV, s, q128, q64, do64, (const float*)lse,
+                   (const float*)D, (bf16*)dqkv, S, H, Hkv, scale, part, err);
+  if (part) {
+    if (e == cudaSuccess) launch_reduce_dkv(part, dqkv, B * S, H, Hkv, HD, scale, s);
+    cudaFreeAsync(part, s);
+  }
+  return e == cudaSuccess;
+}
+
 }  // namespace tg
 
 // Returns false when the shape is outside this kernel: head dim 128 only (at 64 the mma.sync kernel is
@@ -393,6 +939,19 @@ bool attn_fwd_tcgen05(const void* qkv, void* out, float* lse, int B, int S, int 
   if (!tg::enc_init()) return false;
   note_launch(1);
   return tg::fwd_launch<128>(qkv, out, lse, B, S, H, Hkv, s, err);
+}
+
+// Returns false when the shape is outside these kernels (head dim 64 or 128, alignment, no sm_103a) or the
+// grouped-head partials could not be allocated; the caller then uses the mma.sync kernels.
+bool attn_bwd_tcgen05(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv,
+                      int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
+  if (hd != 64 && hd != 128) return false;
+  if ((((uintptr_t)qkv | (uintptr_t)out | (uintptr_t)dout | (uintptr_t)dqkv) & 15u) || B > 65535 ||
+      (S + 127) / 128 > 65535)
+    return false;
+  if (!tg::enc_init()) return false;
+  return hd == 64 ? tg::bwd_launch<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err)
+                  : tg::bwd_launch<128>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err);
 }
 
 }  // namespace zl

@@ -287,7 +287,7 @@ void AB(zl_ctx* c, cudaStream_t s, const void* qkv, const void* out, const void*
         void* dqkv, int B, int S) {
   const double e = (double)esz(c), N = (double)B * S;
   ProfScope p(c, s, PC_ATTN_B, 4.0 * B * c->H * (double)S * S * c->hd, e * N * (2.0 * c->qkvw + 2.0 * c->ad), 3);
-  attn_bwd(c->dt, qkv, out, dout, lse, D, dqkv, B, S, c->H, c->Hkv, c->hd, s, c->pool);
+  attn_bwd(c->dt, qkv, out, dout, lse, D, dqkv, B, S, c->H, c->Hkv, c->hd, s, c->pool, c->d_err);
 }
 void NF(zl_ctx* c, cudaStream_t s, const void* x, const float* g, const float* b, void* y, float* rstd, float* mean,
         int N) {

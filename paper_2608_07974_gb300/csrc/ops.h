@@ -86,8 +86,13 @@ void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void*
 // other bf16 shapes: mma.sync; fp32: CUDA cores.
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,
               cudaStream_t s, unsigned* err = nullptr);
-// Gradients into dqkv (same layout as qkv). Dbuf: [B, H, S] scratch.
+// Gradients into dqkv (same layout as qkv). Dbuf: [B, H, S] scratch. bf16 with head dim 64 or 128: the
+// tcgen05 kernels (err as for attn_fwd); other bf16 shapes: mma.sync; fp32: CUDA cores.
 void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const float* lse, float* Dbuf,
-              void* dqkv, int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool = nullptr);
+              void* dqkv, int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool = nullptr,
+              unsigned* err = nullptr);
+// dK, dV of each KV head (bf16, into dqkv) = fixed-order sums over its query heads of the fp32 partials
+// part[2][H][NS][hd] (dK unscaled; times scale here).
+void launch_reduce_dkv(const float* part, void* dqkv, int NS, int H, int Hkv, int hd, float scale, cudaStream_t s);
 
 }  // namespace zl
