@@ -352,8 +352,11 @@ struct BCfg {
   static constexpr int T64 = IB * HD * 2;
   static constexpr int NST = HD == 64 ? 4 : 3;   // pipeline stages of (Q_i, dO_i) or (K_j, V_j)
   static constexpr int OPB = 128 * IB * 2;       // one bf16 [128 x 64] operand (P^T, dS^T or dS)
-  static constexpr int SMEM_DKV = 2 * T128 + NST * 2 * T64 + 2 * OPB + NST * 2 * IB * 4 + 256 + 1024;
-  static constexpr int SMEM_DQ = 2 * T128 + NST * 2 * T64 + OPB + 2 * 128 * 4 + 256 + 1024;
+  // K, V | stages | P^T, dS^T double-buffered | stats (-lse2, D) per stage | barriers | alignment
+  static constexpr int SMEM_DKV = 2 * T128 + NST * 2 * T64 + 4 * OPB + NST * 2 * IB * 4 + 256 + 1024;
+  // Q, dO | stages | dS double-buffered | D halves | barriers | alignment
+  static constexpr int SMEM_DQ = 2 * T128 + NST * 2 * T64 + 2 * OPB + 2 * 128 * 4 + 256 + 1024;
+  static_assert(SMEM_DKV <= 232448 && SMEM_DQ <= 232448, "shared memory per CTA");
 };
 
 // Stores 32 bf16 values (64 bytes: 16-byte chunks 4 half .. 4 half + 3) into row r of a swizzled
@@ -371,11 +374,31 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// Warp-uniform bounded wait by lane 0.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, unsigned* err) {
-  int w = 1;
-  if ((threadIdx.x & 31) == 0) w = mbar_wait(bar, parity, abort_flag, err) ? 1 : 0;
-  return __shfl_sync(0xffffffffu, w, 0) != 0;
+// Packed fp32 pairs (sm_100 and later): one instruction for two lanes' worth of FMA / FSUB / FMUL.
+__device__ __forceinline__ uint64_t f2(float x, float y) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+  return r;
+}
+__device__ __forceinline__ float2 uf2(uint64_t r) {
+  float2 v;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(v.x), "=f"(v.y) : "l"(r));
+  return v;
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ uint64_t sub2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
 }
 
 // Lane 0 of the producer, after a failed wait: lets the copies it issued land (bounded) before exit.
@@ -410,6 +433,9 @@ __device__ __forceinline__ void tmem_release(uint64_t* fin, uint32_t tmem) {
   asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512u) : "memory");
 }
 
+// The TMA and MMA warps run their loops with the whole warp (uniform control flow, so addresses and
+// descriptors stay in uniform registers); one elected lane issues each group of copies or products.
+
 // dQ (and D) kernel. Maps: tq = qkv in 128-row boxes, tdo = dO in 128-row boxes, tkv = qkv in 64-row boxes.
 template <int HD>
 __global__ void __launch_bounds__(NTHR, 1)
@@ -424,16 +450,16 @@ __global__ void __launch_bounds__(NTHR, 1)
   uint8_t* sq = smem;
   uint8_t* sdo = sq + C_::T128;
   uint8_t* sst = sdo + C_::T128;                  // stage s: K_j at s * 2 T64, V_j after it
-  uint8_t* sds = sst + NST * 2 * C_::T64;
-  float* dpart = (float*)(sds + C_::OPB);         // [2][128] halves of D
+  uint8_t* sds = sst + NST * 2 * C_::T64;         // dS, two buffers
+  float* dpart = (float*)(sds + 2 * C_::OPB);     // [2][128] halves of D
   uint64_t* full = (uint64_t*)(dpart + 256);
   uint64_t* empty = full + NST;
   uint64_t* qfull = empty + NST;
   uint64_t* sfull = qfull + 1;                    // [2]
   uint64_t* sempty = sfull + 2;                   // [2]
-  uint64_t* dsfull = sempty + 2;
-  uint64_t* dsempty = dsfull + 1;
-  uint64_t* ofull = dsempty + 1;
+  uint64_t* dsfull = sempty + 2;                  // [2]
+  uint64_t* dsempty = dsfull + 2;                 // [2]
+  uint64_t* ofull = dsempty + 2;
   uint64_t* fin = ofull + 1;
   uint32_t* tbase = (uint32_t*)(fin + 1);
   volatile int* abort_flag = (volatile int*)(tbase + 1);
@@ -448,9 +474,12 @@ __global__ void __launch_bounds__(NTHR, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(qfull, 1);
-    for (int u = 0; u < 2; ++u) { mbar_init(&sfull[u], 1); mbar_init(&sempty[u], NSM); }
-    mbar_init(dsfull, NSM);
-    mbar_init(dsempty, 1);
+    for (int u = 0; u < 2; ++u) {
+      mbar_init(&sfull[u], 1);
+      mbar_init(&sempty[u], NSM);
+      mbar_init(&dsfull[u], NSM);
+      mbar_init(&dsempty[u], 1);
+    }
     mbar_init(ofull, 1);
     mbar_init(fin, 1);
     *abort_flag = 0;
@@ -465,59 +494,71 @@ __global__ void __launch_bounds__(NTHR, 1)
   pdl_trigger();
 
   if (warp == 0) {
-    if (lane == 0) {
-      int issued[NST];
+    int issued[NST];
 #pragma unroll
-      for (int s = 0; s < NST; ++s) issued[s] = -1;
+    for (int s = 0; s < NST; ++s) issued[s] = -1;
+    const bool leader = elect_one();
+    if (leader) {
       mbar_expect_tx(qfull, 2 * C_::T128);
 #pragma unroll
       for (int c = 0; c < HD / 64; ++c) {
         tma3d(sq + c * 16384, &tq, qfull, xq + 64 * c, q0, b);
         tma3d(sdo + c * 16384, &tdo, qfull, h * HD + 64 * c, q0, b);
       }
-      int stage = 0;
-      uint32_t phase = 0;
-      bool ok = true;
-      for (int j = 0; j < nkb; ++j) {
-        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      if (!uwait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+      issued[stage] = (int)phase;
+      if (leader) {
         mbar_expect_tx(&full[stage], 2 * C_::T64);
-        issued[stage] = (int)phase;
         uint8_t* st = sst + stage * 2 * C_::T64;
 #pragma unroll
         for (int c = 0; c < HD / 64; ++c) {
           tma3d(st + c * 8192, &tkv, &full[stage], xk + 64 * c, j * IB, b);
           tma3d(st + C_::T64 + c * 8192, &tkv, &full[stage], xv + 64 * c, j * IB, b);
         }
-        if (++stage == NST) { stage = 0; phase ^= 1u; }
       }
-      if (!ok) drain<NST>(full, issued, qfull);
+      __syncwarp();
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
     }
+    if (!ok && lane == 0) drain<NST>(full, issued, qfull);
   } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t id_s = idesc_f16(128, IB, false, false);
-      constexpr uint32_t id_q = idesc_f16(128, HD, false, true);
-      const uint32_t q_addr = su32(sq), do_addr = su32(sdo), ds_addr = su32(sds);
-      bool ok = mbar_wait(qfull, 0, abort_flag, err);
+    constexpr uint32_t id_s = idesc_f16(128, IB, false, false);
+    constexpr uint32_t id_q = idesc_f16(128, HD, false, true);
+    const uint32_t q_addr = su32(sq), do_addr = su32(sdo), ds_addr = su32(sds);
+    const bool leader = elect_one();   // issues every product and every commit that tracks them
+    bool ok = uwait(qfull, 0, abort_flag, err);
+    fence_after();
+    int stage = 0, pstage = 0;
+    uint32_t phase = 0;
+    auto dq = [&](int jb, int st) -> bool {   // dQ += dS_jb K_jb
+      const int db = jb & 1;
+      if (!uwait(&dsfull[db], (uint32_t)(jb >> 1) & 1u, abort_flag, err)) return false;
       fence_after();
-      int stage = 0, pstage = 0;
-      uint32_t phase = 0;
-      auto dq = [&](int jb, int st) -> bool {   // dQ += dS_jb K_jb
-        if (!mbar_wait(dsfull, (uint32_t)(jb & 1), abort_flag, err)) return false;
-        fence_after();
-        const uint32_t k_addr = su32(sst + st * 2 * C_::T64);
+      if (leader) {
+        const uint32_t k_addr = su32(sst + st * 2 * C_::T64), a_addr = ds_addr + db * C_::OPB;
 #pragma unroll
         for (int ks = 0; ks < IB / 16; ++ks)
-          mma_bf16(tmem + 256, sdesc(ds_addr + ks * 32, 16, 1024), sdesc(k_addr + ks * 2048, 8192, 1024), id_q,
+          mma_bf16(tmem + 256, sdesc(a_addr + ks * 32, 16, 1024), sdesc(k_addr + ks * 2048, 8192, 1024), id_q,
                    (jb > 0 || ks > 0) ? 1u : 0u);
         mma_commit(&empty[st]);
-        mma_commit(dsempty);
-        return true;
-      };
-      for (int j = 0; ok && j < nkb; ++j) {
-        const int buf = j & 1;
-        if (!mbar_wait(&sempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-        if (!mbar_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
-        fence_after();
+        mma_commit(&dsempty[db]);
+      }
+      __syncwarp();
+      return true;
+    };
+    for (int j = 0; ok && j < nkb; ++j) {
+      const int buf = j & 1;
+      if (!uwait(&sempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err) ||
+          !uwait(&full[stage], phase, abort_flag, err)) {
+        ok = false;
+        break;
+      }
+      fence_after();
+      if (leader) {
         const uint32_t k_addr = su32(sst + stage * 2 * C_::T64), v_addr = k_addr + C_::T64;
         const uint32_t ts = tmem + (uint32_t)(buf * 128);
 #pragma unroll
@@ -529,22 +570,25 @@ __global__ void __launch_bounds__(NTHR, 1)
                    sdesc(v_addr + kq * 8192 + kr * 32, 16, 1024), id_s, ks > 0 ? 1u : 0u);
         }
         mma_commit(&sfull[buf]);
-        if (j > 0 && !dq(j - 1, pstage)) { ok = false; break; }
-        pstage = stage;
-        if (++stage == NST) { stage = 0; phase ^= 1u; }
       }
-      if (ok && !dq(nkb - 1, pstage)) ok = false;
+      __syncwarp();
+      if (j > 0 && !dq(j - 1, pstage)) { ok = false; break; }
+      pstage = stage;
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (ok && !dq(nkb - 1, pstage)) ok = false;
+    if (leader) {
       if (ok) mma_commit(ofull);
       mma_commit(fin);
     }
+    __syncwarp();
   } else {
     const int quad = warp & 3, half = (warp - 2) / 4;
     const int r = quad * 32 + lane;
     const int q = q0 + r, qc = min(q, S - 1);
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-    const float sl2 = scale * kL2e;
     const size_t si = ((size_t)b * H + h) * S + qc;
-    const float lse2 = q < S ? lse[si] * kL2e : INFINITY;
+    const float nlse2 = q < S ? -lse[si] * kL2e : -INFINITY;
     {   // D = rowsum(dO * O): each half sums half of the row, fixed-order combination
       const bf16* orow = outp + ((size_t)b * S + qc) * HDall + (size_t)h * HD + half * (HD / 2);
       const bf16* grow = dout + ((size_t)b * S + qc) * HDall + (size_t)h * HD + half * (HD / 2);
@@ -562,11 +606,13 @@ __global__ void __launch_bounds__(NTHR, 1)
     asm volatile("bar.sync 1, %0;" ::"n"(32 * NSM) : "memory");
     const float Dq = dpart[r] + dpart[128 + r];
     if (q < S && half == 0) Dv[si] = Dq;
-    const int qlim = min(q, S - 1);
+    const uint64_t SL2 = f2(scale * kL2e, scale * kL2e), NL = f2(nlse2, nlse2), DD = f2(Dq, Dq);
+    // keys >= S need no mask: their K rows are zero-filled, so dS there adds nothing to dQ
+    const int qmin = q0 + quad * 32;   // smallest query row of this warp
     bool ok = true;
     for (int j = 0; j < nkb; ++j) {
       const int buf = j & 1;
-      if (!warp_wait(&sfull[buf], (uint32_t)(j >> 1) & 1u, abort_flag, err)) { ok = false; break; }
+      if (!uwait(&sfull[buf], (uint32_t)(j >> 1) & 1u, abort_flag, err)) { ok = false; break; }
       fence_after();
       float sv[32], dp[32];
       tmem_ld32(trow + (uint32_t)(buf * 128 + half * 32), sv);
@@ -574,21 +620,29 @@ __global__ void __launch_bounds__(NTHR, 1)
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sempty[buf]);
-      const int kmax = qlim - (j * IB + half * 32);   // columns e <= kmax are causal and inside S
+      const int kbase = j * IB + half * 32;
+      const bool diag = kbase + 31 > qmin;   // warp-uniform: some column may lie above the diagonal
+      const int kmax = q - kbase;            // causal: columns e <= kmax
       uint32_t pk[16];
 #pragma unroll
       for (int e = 0; e < 32; e += 2) {
-        const float p0 = e <= kmax ? ex2(fmaf(sv[e], sl2, -lse2)) : 0.f;
-        const float p1 = e + 1 <= kmax ? ex2(fmaf(sv[e + 1], sl2, -lse2)) : 0.f;
-        pk[e / 2] = pack2(p0 * (dp[e] - Dq), p1 * (dp[e + 1] - Dq));
+        float2 x = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, NL));
+        if (diag) {
+          if (e > kmax) x.x = -INFINITY;
+          if (e + 1 > kmax) x.y = -INFINITY;
+        }
+        const float p0 = ex2(x.x), p1 = ex2(x.y);
+        const float2 ds = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), DD)));
+        pk[e / 2] = pack2(ds.x, ds.y);
       }
-      if (!warp_wait(dsempty, ((uint32_t)j & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-      put_quarter_row(sds, half, r, pk);
+      const int db = j & 1;
+      if (!uwait(&dsempty[db], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+      put_quarter_row(sds + db * C_::OPB, half, r, pk);
       fence_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(dsfull);
+      if (lane == 0) mbar_arrive(&dsfull[db]);
     }
-    if (ok && warp_wait(ofull, 0, abort_flag, err)) {
+    if (ok && uwait(ofull, 0, abort_flag, err)) {
       fence_after();
       bf16* drow = dqkv + ((size_t)b * S + qc) * ld + (size_t)h * HD;
 #pragma unroll
@@ -625,17 +679,16 @@ __global__ void __launch_bounds__(NTHR, 1)
   uint8_t* sk = smem;
   uint8_t* sv = sk + C_::T128;
   uint8_t* sst = sv + C_::T128;                   // stage s: Q_i at s * 2 T64, dO_i after it
-  uint8_t* sp = sst + NST * 2 * C_::T64;          // P^T
-  uint8_t* sds = sp + C_::OPB;                    // dS^T
-  float* stats = (float*)(sds + C_::OPB);         // stage s: lse2[64], D[64]
+  uint8_t* sp = sst + NST * 2 * C_::T64;          // buffer u: P^T at sp + 2 u OPB, dS^T after it
+  float* stats = (float*)(sp + 4 * C_::OPB);      // stage s: -lse2[64], D[64]
   uint64_t* full = (uint64_t*)(stats + NST * 2 * IB);
   uint64_t* empty = full + NST;
   uint64_t* kvfull = empty + NST;
   uint64_t* sfull = kvfull + 1;                   // [2]
   uint64_t* sempty = sfull + 2;                   // [2]
-  uint64_t* pfull = sempty + 2;
-  uint64_t* pempty = pfull + 1;
-  uint64_t* ofull = pempty + 1;
+  uint64_t* pfull = sempty + 2;                   // [2]
+  uint64_t* pempty = pfull + 2;                   // [2]
+  uint64_t* ofull = pempty + 2;
   uint64_t* fin = ofull + 1;
   uint32_t* tbase = (uint32_t*)(fin + 1);
   volatile int* abort_flag = (volatile int*)(tbase + 1);
@@ -650,9 +703,12 @@ __global__ void __launch_bounds__(NTHR, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 2); mbar_init(&empty[s], 1); }
     mbar_init(kvfull, 1);
-    for (int u = 0; u < 2; ++u) { mbar_init(&sfull[u], 1); mbar_init(&sempty[u], NSM); }
-    mbar_init(pfull, NSM);
-    mbar_init(pempty, 1);
+    for (int u = 0; u < 2; ++u) {
+      mbar_init(&sfull[u], 1);
+      mbar_init(&sempty[u], NSM);
+      mbar_init(&pfull[u], NSM);
+      mbar_init(&pempty[u], 1);
+    }
     mbar_init(ofull, 1);
     mbar_init(fin, 1);
     *abort_flag = 0;
@@ -667,11 +723,13 @@ __global__ void __launch_bounds__(NTHR, 1)
   pdl_trigger();
 
   if (warp == 0) {
-    // lane 0: TMA of K, V once and of (Q_i, dO_i) per block; every lane: two of the block's lse2 and D
+    // one elected lane: TMA of K, V once and of (Q_i, dO_i) per block; every lane: two of the block's
+    // -lse2 and D
     int issued[NST];
 #pragma unroll
     for (int s = 0; s < NST; ++s) issued[s] = -1;
-    if (lane == 0) {
+    const bool leader = elect_one();
+    if (leader) {
       mbar_expect_tx(kvfull, 2 * C_::T128);
 #pragma unroll
       for (int c = 0; c < HD / 64; ++c) {
@@ -682,13 +740,25 @@ __global__ void __launch_bounds__(NTHR, 1)
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
+    // this lane's two statistics of the next block, loaded one block ahead
+    float nl[2], dd[2];
+    auto fetch = [&](int it) {
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int qq = (i0 + it) * IB + lane * 2 + u;
+        const size_t si = ((size_t)b * H + h) * S + (qq < S ? qq : 0);
+        nl[u] = qq < S ? -lse[si] * kL2e : -INFINITY;
+        dd[u] = qq < S ? Dv[si] : 0.f;
+      }
+    };
+    fetch(0);
     for (int it = 0; it < nit; ++it) {
       const int qi0 = (i0 + it) * IB;
-      if (!warp_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
-      uint8_t* st = sst + stage * 2 * C_::T64;
-      if (lane == 0) {
+      if (!uwait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+      issued[stage] = (int)phase;
+      if (leader) {
         mbar_expect_tx(&full[stage], 2 * C_::T64);
-        issued[stage] = (int)phase;
+        uint8_t* st = sst + stage * 2 * C_::T64;
 #pragma unroll
         for (int c = 0; c < HD / 64; ++c) {
           tma3d(st + c * 8192, &tq, &full[stage], xq + 64 * c, qi0, b);
@@ -696,47 +766,51 @@ __global__ void __launch_bounds__(NTHR, 1)
         }
       }
       float* sl = stats + stage * 2 * IB;
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int cq = lane * 2 + u, qq = qi0 + cq;
-        const size_t si = ((size_t)b * H + h) * S + (qq < S ? qq : 0);
-        sl[cq] = qq < S ? lse[si] * kL2e : INFINITY;
-        sl[IB + cq] = qq < S ? Dv[si] : 0.f;
-      }
+      *reinterpret_cast<float2*>(sl + lane * 2) = make_float2(nl[0], nl[1]);
+      *reinterpret_cast<float2*>(sl + IB + lane * 2) = make_float2(dd[0], dd[1]);
       __syncwarp();
       if (lane == 0) mbar_arrive(&full[stage]);
+      if (it + 1 < nit) fetch(it + 1);
       if (++stage == NST) { stage = 0; phase ^= 1u; }
     }
     if (!ok && lane == 0) drain<NST>(full, issued, kvfull);
   } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t id_s = idesc_f16(128, IB, false, false);
-      constexpr uint32_t id_g = idesc_f16(128, HD, false, true);
-      const uint32_t k_addr = su32(sk), v_addr = su32(sv), p_addr = su32(sp), ds_addr = su32(sds);
-      bool ok = mbar_wait(kvfull, 0, abort_flag, err);
+    constexpr uint32_t id_s = idesc_f16(128, IB, false, false);
+    constexpr uint32_t id_g = idesc_f16(128, HD, false, true);
+    const uint32_t k_addr = su32(sk), v_addr = su32(sv), p_addr = su32(sp);
+    const bool leader = elect_one();   // issues every product and every commit that tracks them
+    bool ok = uwait(kvfull, 0, abort_flag, err);
+    fence_after();
+    int stage = 0, pstage = 0;
+    uint32_t phase = 0;
+    auto grads = [&](int ib, int st) -> bool {   // dV += P^T dO_ib, dK += dS^T Q_ib
+      const int pb = ib & 1;
+      if (!uwait(&pfull[pb], (uint32_t)(ib >> 1) & 1u, abort_flag, err)) return false;
       fence_after();
-      int stage = 0, pstage = 0;
-      uint32_t phase = 0;
-      auto grads = [&](int ib, int st) -> bool {   // dV += P^T dO_ib, dK += dS^T Q_ib
-        if (!mbar_wait(pfull, (uint32_t)(ib & 1), abort_flag, err)) return false;
-        fence_after();
+      if (leader) {
         const uint32_t qa = su32(sst + st * 2 * C_::T64), da = qa + C_::T64;
+        const uint32_t pa = p_addr + pb * 2 * C_::OPB, dsa = pa + C_::OPB;
 #pragma unroll
         for (int ks = 0; ks < IB / 16; ++ks) {
           const uint32_t acc = (ib > 0 || ks > 0) ? 1u : 0u;
-          mma_bf16(tmem + 256, sdesc(p_addr + ks * 32, 16, 1024), sdesc(da + ks * 2048, 8192, 1024), id_g, acc);
-          mma_bf16(tmem + 256 + HD, sdesc(ds_addr + ks * 32, 16, 1024), sdesc(qa + ks * 2048, 8192, 1024), id_g,
-                   acc);
+          mma_bf16(tmem + 256, sdesc(pa + ks * 32, 16, 1024), sdesc(da + ks * 2048, 8192, 1024), id_g, acc);
+          mma_bf16(tmem + 256 + HD, sdesc(dsa + ks * 32, 16, 1024), sdesc(qa + ks * 2048, 8192, 1024), id_g, acc);
         }
         mma_commit(&empty[st]);
-        mma_commit(pempty);
-        return true;
-      };
-      for (int it = 0; ok && it < nit; ++it) {
-        const int buf = it & 1;
-        if (!mbar_wait(&sempty[buf], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-        if (!mbar_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
-        fence_after();
+        mma_commit(&pempty[pb]);
+      }
+      __syncwarp();
+      return true;
+    };
+    for (int it = 0; ok && it < nit; ++it) {
+      const int buf = it & 1;
+      if (!uwait(&sempty[buf], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err) ||
+          !uwait(&full[stage], phase, abort_flag, err)) {
+        ok = false;
+        break;
+      }
+      fence_after();
+      if (leader) {
         const uint32_t qa = su32(sst + stage * 2 * C_::T64), da = qa + C_::T64;
         const uint32_t ts = tmem + (uint32_t)(buf * 128);
 #pragma unroll
@@ -744,30 +818,37 @@ __global__ void __launch_bounds__(NTHR, 1)
           const int kq = ks / 4, kr = ks % 4;
           mma_bf16(ts, sdesc(k_addr + kq * 16384 + kr * 32, 16, 1024), sdesc(qa + kq * 8192 + kr * 32, 16, 1024),
                    id_s, ks > 0 ? 1u : 0u);
-          mma_bf16(ts + IB, sdesc(v_addr + kq * 16384 + kr * 32, 16, 1024), sdesc(da + kq * 8192 + kr * 32, 16, 1024),
-                   id_s, ks > 0 ? 1u : 0u);
+          mma_bf16(ts + IB, sdesc(v_addr + kq * 16384 + kr * 32, 16, 1024),
+                   sdesc(da + kq * 8192 + kr * 32, 16, 1024), id_s, ks > 0 ? 1u : 0u);
         }
         mma_commit(&sfull[buf]);
-        if (it > 0 && !grads(it - 1, pstage)) { ok = false; break; }
-        pstage = stage;
-        if (++stage == NST) { stage = 0; phase ^= 1u; }
       }
-      if (ok && !grads(nit - 1, pstage)) ok = false;
+      __syncwarp();
+      if (it > 0 && !grads(it - 1, pstage)) { ok = false; break; }
+      pstage = stage;
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (ok && !grads(nit - 1, pstage)) ok = false;
+    if (leader) {
       if (ok) mma_commit(ofull);
       mma_commit(fin);
     }
+    __syncwarp();
   } else {
     const int quad = warp & 3, half = (warp - 2) / 4;
     const int r = quad * 32 + lane;                 // key row = TMEM lane
     const int key = k0 + r;
+    const int kmaxw = k0 + quad * 32 + 31;          // largest key of this warp
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-    const float sl2 = scale * kL2e;
+    const uint64_t SL2 = f2(scale * kL2e, scale * kL2e);
+    // Only the causal mask is applied: queries >= S have -lse2 = -inf (P = 0) and D = 0, and rows of
+    // keys >= S are never stored.
     bool ok = true;
     int stage = 0;
     uint32_t phase = 0;
     for (int it = 0; it < nit; ++it) {
       const int buf = it & 1;
-      if (!warp_wait(&sfull[buf], (uint32_t)(it >> 1) & 1u, abort_flag, err)) { ok = false; break; }
+      if (!uwait(&sfull[buf], (uint32_t)(it >> 1) & 1u, abort_flag, err)) { ok = false; break; }
       fence_after();
       float sv[32], dp[32];
       tmem_ld32(trow + (uint32_t)(buf * 128 + half * 32), sv);
@@ -775,34 +856,45 @@ __global__ void __launch_bounds__(NTHR, 1)
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sempty[buf]);
-      // this stage's lse2 and D: its full phase has completed (the S MMA waited on it); the wait
-      // orders the producer's stores before these loads
-      if (!warp_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
-      const float* sl = stats + stage * 2 * IB + half * 32;
-      const float* sd = sl + IB;
+      // this stage's statistics: its full phase has completed (the S MMA waited on it); the wait orders
+      // the producer's stores before these loads
+      if (!uwait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
+      const float4* sl4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + half * 32);
+      const float4* sd4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + IB + half * 32);
       const int qbase = (i0 + it) * IB + half * 32;   // query of column 0 of this thread's 32
-      const int qlo = key - qbase;                     // columns e >= qlo are causal
-      const int qhi = S - qbase;                       // columns e < qhi are inside S
-      const bool krow = key < S;
+      const bool diag = qbase < kmaxw;                 // warp-uniform: some column may precede its key
+      const int qlo = key - qbase;                     // causal: columns e >= qlo
       uint32_t pk[16], dk[16];
 #pragma unroll
-      for (int e = 0; e < 32; e += 2) {
-        const bool v0 = krow && e >= qlo && e < qhi;
-        const bool v1 = krow && e + 1 >= qlo && e + 1 < qhi;
-        const float p0 = v0 ? ex2(fmaf(sv[e], sl2, -sl[e])) : 0.f;
-        const float p1 = v1 ? ex2(fmaf(sv[e + 1], sl2, -sl[e + 1])) : 0.f;
-        pk[e / 2] = pack2(p0, p1);
-        dk[e / 2] = pack2(p0 * (dp[e] - sd[e]), p1 * (dp[e + 1] - sd[e + 1]));
+      for (int e4 = 0; e4 < 8; ++e4) {
+        const float4 l = sl4[e4], d = sd4[e4];
+        const int e = 4 * e4;
+        float2 xa = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, f2(l.x, l.y)));
+        float2 xb = uf2(fma2(f2(sv[e + 2], sv[e + 3]), SL2, f2(l.z, l.w)));
+        if (diag) {
+          if (e < qlo) xa.x = -INFINITY;
+          if (e + 1 < qlo) xa.y = -INFINITY;
+          if (e + 2 < qlo) xb.x = -INFINITY;
+          if (e + 3 < qlo) xb.y = -INFINITY;
+        }
+        const float p0 = ex2(xa.x), p1 = ex2(xa.y), p2 = ex2(xb.x), p3 = ex2(xb.y);
+        const float2 da = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), f2(d.x, d.y))));
+        const float2 db = uf2(mul2(f2(p2, p3), sub2(f2(dp[e + 2], dp[e + 3]), f2(d.z, d.w))));
+        pk[2 * e4] = pack2(p0, p1);
+        pk[2 * e4 + 1] = pack2(p2, p3);
+        dk[2 * e4] = pack2(da.x, da.y);
+        dk[2 * e4 + 1] = pack2(db.x, db.y);
       }
-      if (!warp_wait(pempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-      put_quarter_row(sp, half, r, pk);
-      put_quarter_row(sds, half, r, dk);
+      const int pb = it & 1;
+      if (!uwait(&pempty[pb], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+      put_quarter_row(sp + pb * 2 * C_::OPB, half, r, pk);
+      put_quarter_row(sp + pb * 2 * C_::OPB + C_::OPB, half, r, dk);
       fence_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(pfull);
+      if (lane == 0) mbar_arrive(&pfull[pb]);
       if (++stage == NST) { stage = 0; phase ^= 1u; }
     }
-    if (ok && warp_wait(ofull, 0, abort_flag, err)) {
+    if (ok && uwait(ofull, 0, abort_flag, err)) {
       fence_after();
       const int kc = min(key, S - 1);
       const size_t NS = (size_t)gridDim.y * S;

@@ -106,21 +106,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0;
-      bool ok = true;
-      int issued[C_::STAGES];   // parity of the last fill of each stage, -1 if none
+    // The whole warp runs the loop (uniform control flow keeps coordinates and addresses in uniform
+    // registers); one elected lane issues the copies.
+    const bool leader = elect_one();
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    int issued[C_::STAGES];   // parity of the last fill of each stage, -1 if none
 #pragma unroll
-      for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
-      for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
-        int tm, tn;
-        tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
-        const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
-        for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
+    for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
+    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
+      int tm, tn;
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (!uwait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
+        issued[stage] = (int)phase;
+        if (leader) {
           mbar_expect_tx(&full[stage], C_::STAGE_BYTES);
-          issued[stage] = (int)phase;
           uint8_t* sa = smem + stage * C_::STAGE_BYTES;
           uint8_t* sb = sa + C_::A_BYTES;
           const int k0 = kb * BK;
@@ -136,35 +139,39 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int j = 0; j < BN / 64; ++j) tma2d(sb + j * 8192, &tb, &full[stage], tn * BN + 64 * j, k0);
           }
-          if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
         }
+        __syncwarp();
+        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
       }
-      if (!ok) {   // unwinding: let the copies already in flight land before the CTA exits
-        for (int s = 0; s < C_::STAGES; ++s) {
-          if (issued[s] < 0) continue;
-          const unsigned long long t0 = gtimer();
-          while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
-          }
+    }
+    if (!ok && lane == 0) {   // unwinding: let the copies already in flight land before the CTA exits
+      for (int s = 0; s < C_::STAGES; ++s) {
+        if (issued[s] < 0) continue;
+        const unsigned long long t0 = gtimer();
+        while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
         }
       }
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer (one thread) ----------------
-    if (lane == 0) {
-      constexpr uint32_t id = idesc<BN, A_MN, B_MN>();
-      int stage = 0, it = 0;
-      uint32_t phase = 0;
-      bool ok = true;
-      for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++it) {
-        const int acc = it & 1;
-        const uint32_t aph = (uint32_t)(it >> 1) & 1u;
-        if (!mbar_wait(&tempty[acc], aph ^ 1u, abort_flag, g.err)) break;
+    // ---------------- MMA issuer ----------------
+    // The whole warp runs the loop and the waits; one elected lane issues every product and every
+    // commit that tracks them.
+    constexpr uint32_t id = idesc<BN, A_MN, B_MN>();
+    const bool leader = elect_one();
+    int stage = 0, it = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++it) {
+      const int acc = it & 1;
+      const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+      if (!uwait(&tempty[acc], aph ^ 1u, abort_flag, g.err)) break;
+      fence_after();
+      const uint32_t d = tmem + (uint32_t)(acc * BN);
+      const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (!uwait(&full[stage], phase, abort_flag, g.err)) { ok = false; break; }
         fence_after();
-        const uint32_t d = tmem + (uint32_t)(acc * BN);
-        const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
-        for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag, g.err)) { ok = false; break; }
-          fence_after();
+        if (leader) {
           const uint32_t a0 = su32(smem + stage * C_::STAGE_BYTES), b0 = a0 + C_::A_BYTES;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
@@ -173,13 +180,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_bf16(d, ad, bd, id, (kb > kb0 || kk > 0) ? 1u : 0u);
           }
           mma_commit(&empty[stage]);
-          if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
         }
-        if (ok) mma_commit(&tfull[acc]);
+        __syncwarp();
+        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
       }
-      // all MMAs issued by this thread complete before TMEM is released
-      mma_commit(fin);
+      if (ok && leader) mma_commit(&tfull[acc]);
+      __syncwarp();
     }
+    // all MMAs issued by the leader complete before TMEM is released
+    if (leader) mma_commit(fin);
+    __syncwarp();
   } else {
     // ---------------- epilogue: warps 2..5, one accumulator row per thread ----------------
     // Per 128-byte column chunk (64 bf16 or 32 fp32 columns): TMEM -> registers (alpha, bias,

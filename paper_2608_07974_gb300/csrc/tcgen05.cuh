@@ -8,7 +8,8 @@
 namespace zl {
 namespace tc {
 
-constexpr unsigned long long kTimeoutNs = 2000000000ull;   // 2 s per wait
+constexpr unsigned long long kTimeoutNs = 2000000000ull;   // 2 s (drain loops, %globaltimer)
+constexpr long long kTimeoutCycles = 4000000000ll;          // about 2 s of SM clock per mbarrier wait
 
 __device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ unsigned long long gtimer() {
@@ -34,19 +35,33 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
       : "memory");
   return r != 0;
 }
-// Waits for the phase of the given parity; false if the kernel is unwinding or the wait expired.
+// Waits for the phase of the given parity; false if the kernel is unwinding or the wait expired. The
+// limit is counted in SM cycles (clock64 is cheap to read; at lower clocks the limit only grows).
 __device__ inline bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, unsigned* err) {
   if (mbar_test(b, parity)) return true;
-  const unsigned long long t0 = gtimer();
+  const long long t0 = clock64();
   for (;;) {
     if (mbar_test(b, parity)) return true;
     if (*abort_flag) return false;
-    if (gtimer() - t0 > kTimeoutNs) {
+    if (clock64() - t0 > kTimeoutCycles) {
       *abort_flag = 1;
       if (err) atomicOr(err, ZL_DEVERR_TIMEOUT);
       return false;
     }
   }
+}
+
+// The same wait by every lane of a warp (warp-uniform control flow); true only if it held for all.
+__device__ __forceinline__ bool uwait(uint64_t* b, uint32_t parity, volatile int* abort_flag, unsigned* err) {
+  const bool ok = mbar_wait(b, parity, abort_flag, err);
+  return __all_sync(0xffffffffu, ok);
+}
+// One lane of the (converged) warp; tcgen05.mma and the tcgen05.commit that tracks it are issued inside
+// the same elected region.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t p;
+  asm volatile("{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n selp.b32 %0, 1, 0, e;\n}" : "=r"(p));
+  return p != 0;
 }
 
 // Epilogue stores: shared memory -> global through the tensor map of C (bulk-group completion).
