@@ -107,23 +107,26 @@ __global__ void __launch_bounds__(NTHR, 1)
   pdl_trigger();
 
   if (warp == 0) {
-    // ---------------- TMA producer ----------------
-    if (lane == 0) {
-      bool ok = true;
-      int issued[C_::STAGES];
+    // ---------------- TMA producer (whole warp, one elected lane issues) ----------------
+    const bool leader = elect_one();
+    bool ok = true;
+    int issued[C_::STAGES];
 #pragma unroll
-      for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
+    for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
+    if (leader) {
       mbar_expect_tx(qfull, C_::QBYTES);
 #pragma unroll
       for (int c = 0; c < HD / 64; ++c) tma3d(sq + c * 16384, &tqk, qfull, xq + 64 * c, q0, b);
-      int stage = 0;
-      uint32_t phase = 0;
-      for (int it = 0; ok && it < total; ++it) {
-        const bool withv = it >= nkb;
-        const int j = withv ? it - nkb : it;
-        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    for (int it = 0; ok && it < total; ++it) {
+      const bool withv = it >= nkb;
+      const int j = withv ? it - nkb : it;
+      if (!uwait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+      issued[stage] = (int)phase;
+      if (leader) {
         mbar_expect_tx(&full[stage], C_::KBYTES + (withv ? C_::VBYTES : 0));
-        issued[stage] = (int)phase;
         uint8_t* sk = sst + stage * C_::STAGE;
 #pragma unroll
         for (int c = 0; c < HD / 64; ++c) tma3d(sk + c * 16384, &tqk, &full[stage], xk + 64 * c, j * KB, b);
@@ -135,35 +138,37 @@ __global__ void __launch_bounds__(NTHR, 1)
             for (int nb = 0; nb < HD / 64; ++nb)
               tma3d(sv + (kh * (HD / 64) + nb) * 8192, &tvv, &full[stage], xv + 64 * nb, j * KB + 64 * kh, b);
         }
-        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
       }
-      if (!ok) {   // unwinding: let the copies in flight land before the CTA exits
-        for (int s = 0; s < C_::STAGES; ++s) {
-          if (issued[s] < 0) continue;
-          const unsigned long long t0 = gtimer();
-          while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
-          }
-        }
+      __syncwarp();
+      if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
+    }
+    if (!ok && lane == 0) {   // unwinding: let the copies in flight land before the CTA exits
+      for (int s = 0; s < C_::STAGES; ++s) {
+        if (issued[s] < 0) continue;
         const unsigned long long t0 = gtimer();
-        while (!mbar_test(qfull, 0) && gtimer() - t0 < 100000000ull) {
+        while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
         }
+      }
+      const unsigned long long t0 = gtimer();
+      while (!mbar_test(qfull, 0) && gtimer() - t0 < 100000000ull) {
       }
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer (one thread) ----------------
-    if (lane == 0) {
-      constexpr uint32_t id_s = idesc_f16(QB, KB, false, false);
-      constexpr uint32_t id_o = idesc_f16(QB, HD, false, true);
-      const uint32_t tso = tmem + 256;   // O
-      bool ok = mbar_wait(qfull, 0, abort_flag, err);
+    // ---------------- MMA issuer (whole warp, one elected lane issues and commits) ----------------
+    constexpr uint32_t id_s = idesc_f16(QB, KB, false, false);
+    constexpr uint32_t id_o = idesc_f16(QB, HD, false, true);
+    const uint32_t tso = tmem + 256;   // O
+    const bool leader = elect_one();
+    bool ok = uwait(qfull, 0, abort_flag, err);
+    fence_after();
+    int stage = 0, pstage = 0;
+    uint32_t phase = 0;
+    const uint32_t q_addr = su32(sq), p_addr = su32(sp);
+    // P V of pass-2 block jb, reading the V tile of the stage that held it; frees that stage and P
+    auto pv = [&](int jb, int st) -> bool {
+      if (!uwait(pfull, (uint32_t)(jb & 1), abort_flag, err)) return false;
       fence_after();
-      int stage = 0, pstage = 0;
-      uint32_t phase = 0;
-      const uint32_t q_addr = su32(sq), p_addr = su32(sp);
-      // P V of pass-2 block jb, reading the V tile of the stage that held it; frees that stage and P
-      auto pv = [&](int jb, int st) -> bool {
-        if (!mbar_wait(pfull, (uint32_t)(jb & 1), abort_flag, err)) return false;
-        fence_after();
+      if (leader) {
         const uint32_t v_addr = su32(sst + st * C_::STAGE + C_::KBYTES);
 #pragma unroll
         for (int ks = 0; ks < KB / 16; ++ks) {
@@ -174,13 +179,19 @@ __global__ void __launch_bounds__(NTHR, 1)
         }
         mma_commit(&empty[st]);
         mma_commit(pempty);
-        return true;
-      };
-      for (int it = 0; ok && it < total; ++it) {
-        const int sb = it & 1;
-        if (!mbar_wait(&sempty[sb], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-        if (!mbar_wait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
-        fence_after();
+      }
+      __syncwarp();
+      return true;
+    };
+    for (int it = 0; ok && it < total; ++it) {
+      const int sb = it & 1;
+      if (!uwait(&sempty[sb], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err) ||
+          !uwait(&full[stage], phase, abort_flag, err)) {
+        ok = false;
+        break;
+      }
+      fence_after();
+      if (leader) {
         const uint32_t k_addr = su32(sst + stage * C_::STAGE);
 #pragma unroll
         for (int ks = 0; ks < HD / 16; ++ks) {
@@ -190,18 +201,19 @@ __global__ void __launch_bounds__(NTHR, 1)
           mma_bf16(tmem + sb * 128, ad, bd, id_s, ks > 0 ? 1u : 0u);
         }
         mma_commit(&sfull[sb]);
-        if (it < nkb) {
-          mma_commit(&empty[stage]);   // pass 1: the K tile is done
-        } else if (it > nkb) {
-          if (!pv(it - nkb - 1, pstage)) { ok = false; break; }   // the previous block's P V
-        }
-        if (it >= nkb) pstage = stage;   // the stage this pass-2 block's V sits in
-        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
+        if (it < nkb) mma_commit(&empty[stage]);   // pass 1: the K tile is done
       }
-      if (ok && !pv(nkb - 1, pstage)) ok = false;
-      if (ok) mma_commit(ofull);
-      mma_commit(fin);   // every MMA of this thread completes before TMEM is released
+      __syncwarp();
+      if (it > nkb && !pv(it - nkb - 1, pstage)) { ok = false; break; }   // the previous block's P V
+      if (it >= nkb) pstage = stage;   // the stage this pass-2 block's V sits in
+      if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
     }
+    if (ok && !pv(nkb - 1, pstage)) ok = false;
+    if (leader) {
+      if (ok) mma_commit(ofull);
+      mma_commit(fin);   // every MMA of the leader completes before TMEM is released
+    }
+    __syncwarp();
   } else {
     // ---------------- softmax and output: warps 2..9, one query row per thread ----------------
     const int quad = warp & 3, half = (warp - 2) / 4;    // TMEM lane quadrant; key half of every block
@@ -215,10 +227,7 @@ __global__ void __launch_bounds__(NTHR, 1)
       const int sb = it & 1;
       const bool pass2 = it >= nkb;
       const int j = pass2 ? it - nkb : it;
-      int w = 1;
-      if (lane == 0) w = mbar_wait(&sfull[sb], (uint32_t)(it >> 1) & 1u, abort_flag, err) ? 1 : 0;
-      w = __shfl_sync(0xffffffffu, w, 0);
-      if (!w) { ok = false; break; }
+      if (!uwait(&sfull[sb], (uint32_t)(it >> 1) & 1u, abort_flag, err)) { ok = false; break; }
       fence_after();
       // keys of this half a row may see: k <= q (causal) and k < S
       const int kmax = min(q, S - 1) - j * KB - half * 64;   // last visible key offset in the half
@@ -250,13 +259,9 @@ __global__ void __launch_bounds__(NTHR, 1)
           stat[(half * QB + r) * 2] = m;
           stat[(half * QB + r) * 2 + 1] = l;
           __syncwarp();
-          if (lane == 0) {
-            mbar_arrive(statb);
-            w = mbar_wait(statb, 0, abort_flag, err) ? 1 : 0;
-          }
-          w = __shfl_sync(0xffffffffu, w, 0);
-          __syncwarp();   // lane 0's acquire orders the partner warp's statistics for the whole warp
-          if (!w) { ok = false; break; }
+          if (lane == 0) mbar_arrive(statb);
+          // every lane's own acquire orders the partner warp's statistics before its loads
+          if (!uwait(statb, 0, abort_flag, err)) { ok = false; break; }
           const float mo = stat[((1 - half) * QB + r) * 2], lo = stat[((1 - half) * QB + r) * 2 + 1];
           const float mt = fmaxf(m, mo);
           const float lt = mt > -INFINITY ? l * ex2(m - mt) + lo * ex2(mo - mt) : 0.f;
@@ -264,9 +269,7 @@ __global__ void __launch_bounds__(NTHR, 1)
         }
       } else {
         // P may be written once the previous block's P V has read it
-        if (lane == 0) w = mbar_wait(pempty, ((uint32_t)j & 1u) ^ 1u, abort_flag, err) ? 1 : 0;
-        w = __shfl_sync(0xffffffffu, w, 0);
-        if (!w) { ok = false; break; }
+        if (!uwait(pempty, ((uint32_t)j & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
         uint8_t* prow = sp + half * 16384 + r * 128;   // this half's P block, row r (128-byte swizzle)
 #pragma unroll 1
         for (int c = 0; c < 64; c += 32) {
@@ -298,10 +301,7 @@ __global__ void __launch_bounds__(NTHR, 1)
     }
     // output: O = sum_j P_j V_j is already normalised; each warp of a quadrant stores half of the columns
     if (ok) {
-      int w = 1;
-      if (lane == 0) w = mbar_wait(ofull, 0, abort_flag, err) ? 1 : 0;
-      w = __shfl_sync(0xffffffffu, w, 0);
-      if (w) {
+      if (uwait(ofull, 0, abort_flag, err)) {
         fence_after();
         bf16* orow = out + ((size_t)b * S + min(q, S - 1)) * ((size_t)H * HD) + (size_t)h * HD;
 #pragma unroll 1
@@ -345,6 +345,8 @@ __global__ void __launch_bounds__(NTHR, 1)
 // (16-row steps 2 KB apart, head-dim blocks 8 KB apart).
 // ==============================================================================================
 constexpr int IB = 64;   // inner block rows
+constexpr int NEW = 16;  // elementwise warps: four per TMEM lane quadrant, one 16-column quarter each
+constexpr int NTHR_B = 64 + 32 * NEW;
 
 template <int HD>
 struct BCfg {
@@ -354,18 +356,18 @@ struct BCfg {
   static constexpr int OPB = 128 * IB * 2;       // one bf16 [128 x 64] operand (P^T, dS^T or dS)
   // K, V | stages | P^T, dS^T double-buffered | stats (-lse2, D) per stage | barriers | alignment
   static constexpr int SMEM_DKV = 2 * T128 + NST * 2 * T64 + 4 * OPB + NST * 2 * IB * 4 + 256 + 1024;
-  // Q, dO | stages | dS double-buffered | D halves | barriers | alignment
-  static constexpr int SMEM_DQ = 2 * T128 + NST * 2 * T64 + 2 * OPB + 2 * 128 * 4 + 256 + 1024;
+  // Q, dO | stages | dS double-buffered | D quarters | barriers | alignment
+  static constexpr int SMEM_DQ = 2 * T128 + NST * 2 * T64 + 2 * OPB + 4 * 128 * 4 + 256 + 1024;
   static_assert(SMEM_DKV <= 232448 && SMEM_DQ <= 232448, "shared memory per CTA");
 };
 
-// Stores 32 bf16 values (64 bytes: 16-byte chunks 4 half .. 4 half + 3) into row r of a swizzled
+// Stores 16 bf16 values (32 bytes: 16-byte chunks 2 qu and 2 qu + 1) into row r of a swizzled
 // [128 x 64] K-major operand.
-__device__ __forceinline__ void put_quarter_row(uint8_t* g, int half, int r, const uint32_t* pk) {
+__device__ __forceinline__ void put_row16(uint8_t* g, int qu, int r, const uint32_t* pk) {
   uint8_t* row = g + r * 128;
 #pragma unroll
-  for (int u = 0; u < 4; ++u)
-    *reinterpret_cast<uint4*>(row + (((4 * half + u) ^ (r & 7)) << 4)) =
+  for (int u = 0; u < 2; ++u)
+    *reinterpret_cast<uint4*>(row + (((2 * qu + u) ^ (r & 7)) << 4)) =
         make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
 }
 
@@ -438,7 +440,7 @@ __device__ __forceinline__ void tmem_release(uint64_t* fin, uint32_t tmem) {
 
 // dQ (and D) kernel. Maps: tq = qkv in 128-row boxes, tdo = dO in 128-row boxes, tkv = qkv in 64-row boxes.
 template <int HD>
-__global__ void __launch_bounds__(NTHR, 1)
+__global__ void __launch_bounds__(NTHR_B, 1)
     attn_bwd_dq_tg_k(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tdo,
                      const __grid_constant__ CUtensorMap tkv, const bf16* __restrict__ outp,
                      const bf16* __restrict__ dout, const float* __restrict__ lse, float* __restrict__ Dv,
@@ -451,8 +453,8 @@ __global__ void __launch_bounds__(NTHR, 1)
   uint8_t* sdo = sq + C_::T128;
   uint8_t* sst = sdo + C_::T128;                  // stage s: K_j at s * 2 T64, V_j after it
   uint8_t* sds = sst + NST * 2 * C_::T64;         // dS, two buffers
-  float* dpart = (float*)(sds + 2 * C_::OPB);     // [2][128] halves of D
-  uint64_t* full = (uint64_t*)(dpart + 256);
+  float* dpart = (float*)(sds + 2 * C_::OPB);     // [4][128] quarters of D
+  uint64_t* full = (uint64_t*)(dpart + 512);
   uint64_t* empty = full + NST;
   uint64_t* qfull = empty + NST;
   uint64_t* sfull = qfull + 1;                    // [2]
@@ -476,8 +478,8 @@ __global__ void __launch_bounds__(NTHR, 1)
     mbar_init(qfull, 1);
     for (int u = 0; u < 2; ++u) {
       mbar_init(&sfull[u], 1);
-      mbar_init(&sempty[u], NSM);
-      mbar_init(&dsfull[u], NSM);
+      mbar_init(&sempty[u], NEW);
+      mbar_init(&dsfull[u], NEW);
       mbar_init(&dsempty[u], 1);
     }
     mbar_init(ofull, 1);
@@ -583,49 +585,48 @@ __global__ void __launch_bounds__(NTHR, 1)
     }
     __syncwarp();
   } else {
-    const int quad = warp & 3, half = (warp - 2) / 4;
+    const int quad = warp & 3, qu = (warp - 2) / 4;   // TMEM lane quadrant, 16-column quarter
     const int r = quad * 32 + lane;
     const int q = q0 + r, qc = min(q, S - 1);
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     const size_t si = ((size_t)b * H + h) * S + qc;
     const float nlse2 = q < S ? -lse[si] * kL2e : -INFINITY;
-    {   // D = rowsum(dO * O): each half sums half of the row, fixed-order combination
-      const bf16* orow = outp + ((size_t)b * S + qc) * HDall + (size_t)h * HD + half * (HD / 2);
-      const bf16* grow = dout + ((size_t)b * S + qc) * HDall + (size_t)h * HD + half * (HD / 2);
+    {   // D = rowsum(dO * O): each quarter sums a quarter of the row, fixed-order combination
+      const bf16* orow = outp + ((size_t)b * S + qc) * HDall + (size_t)h * HD + qu * (HD / 4);
+      const bf16* grow = dout + ((size_t)b * S + qc) * HDall + (size_t)h * HD + qu * (HD / 4);
       float acc = 0.f;
 #pragma unroll
-      for (int c = 0; c < HD / 2; c += 8) {
+      for (int c = 0; c < HD / 4; c += 8) {
         float o8[8], g8[8];
         Vec8<bf16>::load(orow + c, o8);
         Vec8<bf16>::load(grow + c, g8);
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc = fmaf(o8[e], g8[e], acc);
       }
-      dpart[half * 128 + r] = acc;
+      dpart[qu * 128 + r] = acc;
     }
-    asm volatile("bar.sync 1, %0;" ::"n"(32 * NSM) : "memory");
-    const float Dq = dpart[r] + dpart[128 + r];
-    if (q < S && half == 0) Dv[si] = Dq;
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * NEW) : "memory");
+    const float Dq = (dpart[r] + dpart[128 + r]) + (dpart[256 + r] + dpart[384 + r]);
+    if (q < S && qu == 0) Dv[si] = Dq;
     const uint64_t SL2 = f2(scale * kL2e, scale * kL2e), NL = f2(nlse2, nlse2), DD = f2(Dq, Dq);
-    // keys >= S need no mask: their K rows are zero-filled, so dS there adds nothing to dQ
     const int qmin = q0 + quad * 32;   // smallest query row of this warp
     bool ok = true;
     for (int j = 0; j < nkb; ++j) {
       const int buf = j & 1;
       if (!uwait(&sfull[buf], (uint32_t)(j >> 1) & 1u, abort_flag, err)) { ok = false; break; }
       fence_after();
-      float sv[32], dp[32];
-      tmem_ld32(trow + (uint32_t)(buf * 128 + half * 32), sv);
-      tmem_ld32(trow + (uint32_t)(buf * 128 + IB + half * 32), dp);
+      float sv[16], dp[16];
+      tmem_ld16(trow + (uint32_t)(buf * 128 + qu * 16), sv);
+      tmem_ld16(trow + (uint32_t)(buf * 128 + IB + qu * 16), dp);
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sempty[buf]);
-      const int kbase = j * IB + half * 32;
-      const bool diag = kbase + 31 > qmin;   // warp-uniform: some column may lie above the diagonal
+      const int kbase = j * IB + qu * 16;
+      const bool diag = kbase + 15 > qmin;   // warp-uniform: some column may lie above the diagonal
       const int kmax = q - kbase;            // causal: columns e <= kmax
-      uint32_t pk[16];
+      uint32_t pk[8];
 #pragma unroll
-      for (int e = 0; e < 32; e += 2) {
+      for (int e = 0; e < 16; e += 2) {
         float2 x = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, NL));
         if (diag) {
           if (e > kmax) x.x = -INFINITY;
@@ -637,7 +638,7 @@ __global__ void __launch_bounds__(NTHR, 1)
       }
       const int db = j & 1;
       if (!uwait(&dsempty[db], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-      put_quarter_row(sds + db * C_::OPB, half, r, pk);
+      put_row16(sds + db * C_::OPB, qu, r, pk);
       fence_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&dsfull[db]);
@@ -646,14 +647,14 @@ __global__ void __launch_bounds__(NTHR, 1)
       fence_after();
       bf16* drow = dqkv + ((size_t)b * S + qc) * ld + (size_t)h * HD;
 #pragma unroll
-      for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
-        float v[32];
-        tmem_ld32(trow + 256 + (uint32_t)c, v);
+      for (int c = qu * (HD / 4); c < (qu + 1) * (HD / 4); c += 16) {
+        float v[16];
+        tmem_ld16(trow + 256 + (uint32_t)c, v);
         if (q < S) {
 #pragma unroll
-          for (int e = 0; e < 32; ++e) v[e] *= scale;
-#pragma unroll
-          for (int u = 0; u < 4; ++u) Vec8<bf16>::store(drow + c + 8 * u, v + 8 * u);
+          for (int e = 0; e < 16; ++e) v[e] *= scale;
+          Vec8<bf16>::store(drow + c, v);
+          Vec8<bf16>::store(drow + c + 8, v + 8);
         }
       }
     }
@@ -667,7 +668,7 @@ __global__ void __launch_bounds__(NTHR, 1)
 // part[2][H][B*S][HD], dK unscaled, summed per group afterwards) or of one KV head (H == Hkv: bf16 straight
 // into dqkv). Maps: tkv = qkv in 128-row boxes, tq = qkv in 64-row boxes, tdo = dO in 64-row boxes.
 template <int HD>
-__global__ void __launch_bounds__(NTHR, 1)
+__global__ void __launch_bounds__(NTHR_B, 1)
     attn_bwd_dkv_tg_k(const __grid_constant__ CUtensorMap tkv, const __grid_constant__ CUtensorMap tq,
                       const __grid_constant__ CUtensorMap tdo, const float* __restrict__ lse,
                       const float* __restrict__ Dv, bf16* __restrict__ dqkv, int S, int H, int Hkv, float scale,
@@ -705,8 +706,8 @@ __global__ void __launch_bounds__(NTHR, 1)
     mbar_init(kvfull, 1);
     for (int u = 0; u < 2; ++u) {
       mbar_init(&sfull[u], 1);
-      mbar_init(&sempty[u], NSM);
-      mbar_init(&pfull[u], NSM);
+      mbar_init(&sempty[u], NEW);
+      mbar_init(&pfull[u], NEW);
       mbar_init(&pempty[u], 1);
     }
     mbar_init(ofull, 1);
@@ -835,10 +836,10 @@ __global__ void __launch_bounds__(NTHR, 1)
     }
     __syncwarp();
   } else {
-    const int quad = warp & 3, half = (warp - 2) / 4;
-    const int r = quad * 32 + lane;                 // key row = TMEM lane
+    const int quad = warp & 3, qu = (warp - 2) / 4;   // TMEM lane quadrant, 16-column quarter
+    const int r = quad * 32 + lane;                    // key row = TMEM lane
     const int key = k0 + r;
-    const int kmaxw = k0 + quad * 32 + 31;          // largest key of this warp
+    const int kmaxw = k0 + quad * 32 + 31;             // largest key of this warp
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     const uint64_t SL2 = f2(scale * kL2e, scale * kL2e);
     // Only the causal mask is applied: queries >= S have -lse2 = -inf (P = 0) and D = 0, and rows of
@@ -850,27 +851,29 @@ __global__ void __launch_bounds__(NTHR, 1)
       const int buf = it & 1;
       if (!uwait(&sfull[buf], (uint32_t)(it >> 1) & 1u, abort_flag, err)) { ok = false; break; }
       fence_after();
-      float sv[32], dp[32];
-      tmem_ld32(trow + (uint32_t)(buf * 128 + half * 32), sv);
-      tmem_ld32(trow + (uint32_t)(buf * 128 + IB + half * 32), dp);
+      float sv[16], dp[16];
+      tmem_ld16(trow + (uint32_t)(buf * 128 + qu * 16), sv);
+      tmem_ld16(trow + (uint32_t)(buf * 128 + IB + qu * 16), dp);
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sempty[buf]);
       // this stage's statistics: its full phase has completed (the S MMA waited on it); the wait orders
       // the producer's stores before these loads
       if (!uwait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
-      const float4* sl4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + half * 32);
-      const float4* sd4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + IB + half * 32);
-      const int qbase = (i0 + it) * IB + half * 32;   // query of column 0 of this thread's 32
-      const bool diag = qbase < kmaxw;                 // warp-uniform: some column may precede its key
-      const int qlo = key - qbase;                     // causal: columns e >= qlo
-      uint32_t pk[16], dk[16];
+      const float4* sl4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + qu * 16);
+      const float4* sd4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + IB + qu * 16);
+      float4 l[4], d[4];
 #pragma unroll
-      for (int e4 = 0; e4 < 8; ++e4) {
-        const float4 l = sl4[e4], d = sd4[e4];
+      for (int u = 0; u < 4; ++u) { l[u] = sl4[u]; d[u] = sd4[u]; }
+      const int qbase = (i0 + it) * IB + qu * 16;   // query of column 0 of this thread's 16
+      const bool diag = qbase < kmaxw;               // warp-uniform: some column may precede its key
+      const int qlo = key - qbase;                   // causal: columns e >= qlo
+      uint32_t pk[8], dk[8];
+#pragma unroll
+      for (int e4 = 0; e4 < 4; ++e4) {
         const int e = 4 * e4;
-        float2 xa = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, f2(l.x, l.y)));
-        float2 xb = uf2(fma2(f2(sv[e + 2], sv[e + 3]), SL2, f2(l.z, l.w)));
+        float2 xa = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, f2(l[e4].x, l[e4].y)));
+        float2 xb = uf2(fma2(f2(sv[e + 2], sv[e + 3]), SL2, f2(l[e4].z, l[e4].w)));
         if (diag) {
           if (e < qlo) xa.x = -INFINITY;
           if (e + 1 < qlo) xa.y = -INFINITY;
@@ -878,8 +881,8 @@ __global__ void __launch_bounds__(NTHR, 1)
           if (e + 3 < qlo) xb.y = -INFINITY;
         }
         const float p0 = ex2(xa.x), p1 = ex2(xa.y), p2 = ex2(xb.x), p3 = ex2(xb.y);
-        const float2 da = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), f2(d.x, d.y))));
-        const float2 db = uf2(mul2(f2(p2, p3), sub2(f2(dp[e + 2], dp[e + 3]), f2(d.z, d.w))));
+        const float2 da = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), f2(d[e4].x, d[e4].y))));
+        const float2 db = uf2(mul2(f2(p2, p3), sub2(f2(dp[e + 2], dp[e + 3]), f2(d[e4].z, d[e4].w))));
         pk[2 * e4] = pack2(p0, p1);
         pk[2 * e4 + 1] = pack2(p2, p3);
         dk[2 * e4] = pack2(da.x, da.y);
@@ -887,8 +890,8 @@ __global__ void __launch_bounds__(NTHR, 1)
       }
       const int pb = it & 1;
       if (!uwait(&pempty[pb], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-      put_quarter_row(sp + pb * 2 * C_::OPB, half, r, pk);
-      put_quarter_row(sp + pb * 2 * C_::OPB + C_::OPB, half, r, dk);
+      put_row16(sp + pb * 2 * C_::OPB, qu, r, pk);
+      put_row16(sp + pb * 2 * C_::OPB + C_::OPB, qu, r, dk);
       fence_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&pfull[pb]);
@@ -899,16 +902,16 @@ __global__ void __launch_bounds__(NTHR, 1)
       const int kc = min(key, S - 1);
       const size_t NS = (size_t)gridDim.y * S;
 #pragma unroll
-      for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
-        float gv[32], gk[32];
-        tmem_ld32(trow + 256 + (uint32_t)c, gv);
-        tmem_ld32(trow + 256 + HD + (uint32_t)c, gk);
+      for (int c = qu * (HD / 4); c < (qu + 1) * (HD / 4); c += 16) {
+        float gv[16], gk[16];
+        tmem_ld16(trow + 256 + (uint32_t)c, gv);
+        tmem_ld16(trow + 256 + HD + (uint32_t)c, gk);
         if (key < S) {
           if (part) {
             float* pk2 = part + ((size_t)h * NS + (size_t)b * S + kc) * HD + c;
             float* pv2 = pk2 + (size_t)H * NS * HD;
 #pragma unroll
-            for (int e = 0; e < 32; e += 4) {
+            for (int e = 0; e < 16; e += 4) {
               *reinterpret_cast<float4*>(pk2 + e) = make_float4(gk[e], gk[e + 1], gk[e + 2], gk[e + 3]);
               *reinterpret_cast<float4*>(pv2 + e) = make_float4(gv[e], gv[e + 1], gv[e + 2], gv[e + 3]);
             }
@@ -916,12 +919,11 @@ __global__ void __launch_bounds__(NTHR, 1)
             bf16* dkr = dqkv + ((size_t)b * S + kc) * ld + (size_t)xk + c;
             bf16* dvr = dqkv + ((size_t)b * S + kc) * ld + (size_t)xv + c;
 #pragma unroll
-            for (int e = 0; e < 32; ++e) gk[e] *= scale;
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              Vec8<bf16>::store(dkr + 8 * u, gk + 8 * u);
-              Vec8<bf16>::store(dvr + 8 * u, gv + 8 * u);
-            }
+            for (int e = 0; e < 16; ++e) gk[e] *= scale;
+            Vec8<bf16>::store(dkr, gk);
+            Vec8<bf16>::store(dkr + 8, gk + 8);
+            Vec8<bf16>::store(dvr, gv);
+            Vec8<bf16>::store(dvr + 8, gv + 8);
           }
         }
       }
@@ -1007,10 +1009,10 @@ bool bwd_launch(const void* qkv, const void* out, const void* dout, const float*
   }
   const float scale = 1.f / sqrtf((float)HD);
   const int nqb = (S + 127) / 128;
-  cudaError_t e = launch_pdl(kq, dim3(H, B, nqb), NTHR, C_::SMEM_DQ, s, q128, do128, q64, (const bf16*)out,
+  cudaError_t e = launch_pdl(kq, dim3(H, B, nqb), NTHR_B, C_::SMEM_DQ, s, q128, do128, q64, (const bf16*)out,
                              (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, scale, err);
   if (e == cudaSuccess)
-    e = launch_pdl(kkv, dim3(part ? H : Hkv, B, nqb), NTHR, C_::SMEM_DKV, s, q128, q64, do64, (const float*)lse,
+    e = launch_pdl(kkv, dim3(part ? H : Hkv, B, nqb), NTHR_B, C_::SMEM_DKV, s, q128, q64, do64, (const float*)lse,
                    (const float*)D, (bf16*)dqkv, S, H, Hkv, scale, part, err);
   if (part) {
     if (e == cudaSuccess) launch_reduce_dkv(part, dqkv, B * S, H, Hkv, HD, scale, s);
