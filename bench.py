@@ -95,24 +95,31 @@ def roofline_of(prof):
 
 
 # DRAM bytes per launch (read + write) from ncu captures, valid only for the kernel sources they were
-# taken on (sha256 prefix of the file); any change to that source makes the figure null.
+# taken on (sha256 prefix over the listed files, in order); any change to them makes the figure null.
+GEMM_SOURCES = ["gemm_tc.cu", "tcgen05.cuh"]
 TRAFFIC = {
     # ncu dram__bytes_read.sum + dram__bytes_write.sum of the GPT-2 GEMM shapes (microbench gemm),
     # averaged with the per-step launch mix: 12 layer GEMMs per layer; 5 head forwards, 4 head dX
-    "gemm_layer": {"source": "gemm_tc.cu", "sha256": "8f86aa41f702a435", "bytes_per_launch": 22309760.0},
-    "gemm_head": {"source": "gemm_tc.cu", "sha256": "8f86aa41f702a435", "bytes_per_launch": 642934072.9},
+    "gemm_layer": {"sources": GEMM_SOURCES, "sha256": "c89e8b6031725702", "bytes_per_launch": 22310314.7},
+    "gemm_head": {"sources": GEMM_SOURCES, "sha256": "c89e8b6031725702", "bytes_per_launch": 643574129.8},
 }
 
 
-def measured_traffic(cls):
+def sources_sha(names):
     import hashlib
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2608_07974_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(cls):
     ent = TRAFFIC.get(cls)
-    if not ent:
+    if not ent or ent["bytes_per_launch"] is None:
         return None
-    src = os.path.join(ROOT, "paper_2608_07974_gb300", "csrc", ent["source"])
-    with open(src, "rb") as f:
-        if hashlib.sha256(f.read()).hexdigest()[:16] != ent["sha256"]:
-            return None
+    if sources_sha(ent["sources"]) != ent["sha256"]:
+        return None
     return ent["bytes_per_launch"]
 
 
