@@ -3,6 +3,8 @@
 #include <math.h>
 #include <stdlib.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "ops.h"
 
@@ -745,6 +747,53 @@ __device__ __forceinline__ void loss_pass1_vec(const T* zp, const T* tp, Lse3& Z
   }
 }
 
+// bf16 vectors in packed form: the running sums in two lanes (fp32 pairs), the block maximum from the
+// raw bf16 pairs (exact), every FMA / add on pairs. Same terms as lse_add8, about a third fewer
+// instructions per element.
+struct Lse2 { float m; uint64_t s, a; };   // running max (log2 units), two-lane sum 2^(x-m), cross sum
+
+__device__ __forceinline__ Lse3 lse2_fold(const Lse2& A) {
+  const float2 s = uf2(A.s), a = uf2(A.a);
+  return Lse3{A.m, s.x + s.y, a.x + a.y};
+}
+
+__device__ __forceinline__ void lse2_add8(Lse2& A, const uint4& raw, const uint64_t* x2, const uint64_t* w2) {
+  const uint32_t mm = bf2_max(bf2_max(raw.x, raw.y), bf2_max(raw.z, raw.w));
+  const float mx = fmaxf(__uint_as_float(mm << 16), __uint_as_float(mm & 0xffff0000u)) * kL2e;
+  if (mx > A.m) {
+    const float sc = ex2(A.m - mx);
+    const uint64_t sc2 = f2(sc, sc);
+    A.s = mul2(A.s, sc2);
+    if (w2) A.a = mul2(A.a, sc2);
+    A.m = mx;
+  }
+  const uint64_t l2 = f2(kL2e, kL2e), nm = f2(-A.m, -A.m);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 x = uf2(fma2(x2[i], l2, nm));
+    const uint64_t e = f2(ex2(x.x), ex2(x.y));
+    A.s = add2(A.s, e);
+    if (w2) A.a = fma2(e, w2[i], A.a);
+  }
+}
+
+template <bool TEACHER, int KLDIR>
+__device__ __forceinline__ void loss_pass1_bf16(const bf16* zp, const bf16* tp, Lse2& Z, Lse2& Q) {
+  const uint4 zr = *reinterpret_cast<const uint4*>(zp);
+  const uint64_t z2[4] = {bf2_to_f2(zr.x), bf2_to_f2(zr.y), bf2_to_f2(zr.z), bf2_to_f2(zr.w)};
+  if (TEACHER) {
+    const uint4 tr = *reinterpret_cast<const uint4*>(tp);
+    const uint64_t t2[4] = {bf2_to_f2(tr.x), bf2_to_f2(tr.y), bf2_to_f2(tr.z), bf2_to_f2(tr.w)};
+    uint64_t w2[4];   // natural units
+#pragma unroll
+    for (int i = 0; i < 4; ++i) w2[i] = KLDIR == 0 ? sub2(z2[i], t2[i]) : sub2(t2[i], z2[i]);
+    lse2_add8(Z, zr, z2, KLDIR == 0 ? w2 : nullptr);
+    lse2_add8(Q, tr, t2, KLDIR == 0 ? nullptr : w2);
+  } else {
+    lse2_add8(Z, zr, z2, nullptr);
+  }
+}
+
 // One block per row of logits. Pass 1: base-2 online log-sum-exp of z and t and the KL cross term
 // (two full vectors per trip for loads in flight); pass 2 (the row is still in L2) writes dz.
 template <typename T, bool TEACHER, int KLDIR>
@@ -770,13 +819,25 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
   }
   Lse3 Z{-INFINITY, 0.f, 0.f}, Q{-INFINITY, 0.f, 0.f};
   int c = threadIdx.x * 8;
-  for (; c + step + 8 <= V; c += 2 * step) {
-    loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c, tr + c, Z, Q, 8);
-    loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c + step, tr + c + step, Z, Q, 8);
-  }
-  for (; c < V; c += step) {
-    if (c + 8 <= V) loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c, tr + c, Z, Q, 8);
-    else loss_pass1_vec<T, TEACHER, KLDIR, false>(zr + c, tr + c, Z, Q, V - c);
+  if constexpr (std::is_same<T, bf16>::value) {
+    Lse2 Z2{-INFINITY, 0ull, 0ull}, Q2{-INFINITY, 0ull, 0ull};   // (0ull is the pair (+0, +0))
+    for (; c + step + 8 <= V; c += 2 * step) {
+      loss_pass1_bf16<TEACHER, KLDIR>(zr + c, tr + c, Z2, Q2);
+      loss_pass1_bf16<TEACHER, KLDIR>(zr + c + step, tr + c + step, Z2, Q2);
+    }
+    for (; c + 8 <= V; c += step) loss_pass1_bf16<TEACHER, KLDIR>(zr + c, tr + c, Z2, Q2);
+    if (c < V) loss_pass1_vec<T, TEACHER, KLDIR, false>(zr + c, tr + c, Z, Q, V - c);
+    Z = lse_merge(lse2_fold(Z2), Z);
+    if (TEACHER) Q = lse_merge(lse2_fold(Q2), Q);
+  } else {
+    for (; c + step + 8 <= V; c += 2 * step) {
+      loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c, tr + c, Z, Q, 8);
+      loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c + step, tr + c + step, Z, Q, 8);
+    }
+    for (; c < V; c += step) {
+      if (c + 8 <= V) loss_pass1_vec<T, TEACHER, KLDIR, true>(zr + c, tr + c, Z, Q, 8);
+      else loss_pass1_vec<T, TEACHER, KLDIR, false>(zr + c, tr + c, Z, Q, V - c);
+    }
   }
   Z = warp_merge(Z);
   if (TEACHER) Q = warp_merge(Q);
@@ -805,24 +866,70 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
   const float wt = inv_n * alpha, wc = inv_n * (1.f - alpha);
   //   kl_dir 0: dz = p (wt + wc ((z - t) - shift));  kl_dir 1: dz = (wt + wc) p - wc q;  no teacher: wt p
   const float k0 = wt - wc * shift, wtc = wt + wc;
-  for (c = threadIdx.x * 8; c < ldz; c += step) {
-    float fz[8], ft[8], o[8];
-    Vec8<T>::load(zr + c, fz);
-    if (TEACHER) Vec8<T>::load(tr + c, ft);
+  const uint64_t L2 = f2(kL2e, kL2e), NLZ = f2(-lz2, -lz2), NLT = f2(-lt2, -lt2), WT = f2(wt, wt), WC = f2(wc, wc),
+                 K0 = f2(k0, k0), WTC = f2(wtc, wtc), NWC = f2(-wc, -wc);
+  // dz of one 8-wide vector at column c from its raw z (and t) words (bf16 rows)
+  auto emit_bf16 = [&](int cc, const uint4& zr4, const uint4& tr4) {
+    const uint32_t zw[4] = {zr4.x, zr4.y, zr4.z, zr4.w}, tw[4] = {tr4.x, tr4.y, tr4.z, tr4.w};
+    float o[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float p = ex2(fmaf(fz[i], kL2e, -lz2));
-      if (!TEACHER) o[i] = wt * p;
-      else if (KLDIR == 0) o[i] = p * fmaf(wc, fz[i] - ft[i], k0);
-      else o[i] = fmaf(wtc, p, -wc * ex2(fmaf(ft[i], kL2e, -lt2)));
+    for (int i = 0; i < 4; ++i) {
+      const uint64_t z2 = bf2_to_f2(zw[i]);
+      const float2 x = uf2(fma2(z2, L2, NLZ));
+      const uint64_t p = f2(ex2(x.x), ex2(x.y));
+      uint64_t r;
+      if (!TEACHER) {
+        r = mul2(WT, p);
+      } else if (KLDIR == 0) {
+        r = mul2(p, fma2(WC, sub2(z2, bf2_to_f2(tw[i])), K0));
+      } else {
+        const float2 xt = uf2(fma2(bf2_to_f2(tw[i]), L2, NLT));
+        r = fma2(WTC, p, mul2(NWC, f2(ex2(xt.x), ex2(xt.y))));
+      }
+      const float2 rf = uf2(r);
+      o[2 * i] = rf.x;
+      o[2 * i + 1] = rf.y;
     }
-    if (y >= c && y < c + 8) o[y - c] -= wt;   // the one-hot of the task term
-    if (c + 8 > V) {
+    if (y >= cc && y < cc + 8) o[y - cc] -= wt;   // the one-hot of the task term
+    if (cc + 8 > V) {
 #pragma unroll
       for (int i = 0; i < 8; ++i)
-        if (c + i >= V) o[i] = 0.f;   // padding columns
+        if (cc + i >= V) o[i] = 0.f;   // padding columns
     }
-    Vec8<T>::store(dr + c, o);
+    Vec8<T>::store(dr + cc, o);
+  };
+  c = threadIdx.x * 8;
+  if constexpr (std::is_same<T, bf16>::value) {
+    const uint4 zero4 = make_uint4(0u, 0u, 0u, 0u);
+    for (; c + step < ldz; c += 2 * step) {   // two vectors' loads in flight per trip
+      const uint4 za = *reinterpret_cast<const uint4*>(zr + c), zb = *reinterpret_cast<const uint4*>(zr + c + step);
+      const uint4 ta = TEACHER ? *reinterpret_cast<const uint4*>(tr + c) : zero4;
+      const uint4 tb = TEACHER ? *reinterpret_cast<const uint4*>(tr + c + step) : zero4;
+      emit_bf16(c, za, ta);
+      emit_bf16(c + step, zb, tb);
+    }
+    if (c < ldz) emit_bf16(c, *reinterpret_cast<const uint4*>(zr + c),
+                           TEACHER ? *reinterpret_cast<const uint4*>(tr + c) : zero4);
+  } else {
+    for (; c < ldz; c += step) {
+      float fz[8], ft[8], o[8];
+      Vec8<T>::load(zr + c, fz);
+      if (TEACHER) Vec8<T>::load(tr + c, ft);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float p = ex2(fmaf(fz[i], kL2e, -lz2));
+        if (!TEACHER) o[i] = wt * p;
+        else if (KLDIR == 0) o[i] = p * fmaf(wc, fz[i] - ft[i], k0);
+        else o[i] = fmaf(wtc, p, -wc * ex2(fmaf(ft[i], kL2e, -lt2)));
+      }
+      if (y >= c && y < c + 8) o[y - c] -= wt;   // the one-hot of the task term
+      if (c + 8 > V) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if (c + i >= V) o[i] = 0.f;   // padding columns
+      }
+      Vec8<T>::store(dr + c, o);
+    }
   }
 }
 
