@@ -112,6 +112,9 @@ struct Chunk {
   std::vector<Entry> ring;
   cudaStream_t s = nullptr;
   cudaEvent_t ev_h = nullptr, ev_z = nullptr, ev_loss = nullptr, ev_hb = nullptr, ev_done = nullptr;
+  // side stream of the backward's column sums (the chunk stream itself when serialised) and its events
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_sin = nullptr, ev_ln2 = nullptr, ev_layer = nullptr, ev_ln1 = nullptr, ev_send = nullptr;
 };
 
 // Saved activations of one layer (pointers into the chunk's arena).
@@ -436,27 +439,57 @@ void carve_ws(zl_ctx* c, Arena& a, BwdWs& w, int N, int B, int S) {
   w.du = a.take((size_t)N * std::max(lora_r16(c->cfg.lora_rank), 1) * e);
 }
 
-void bias_grad(zl_ctx* c, const void* dY, int N, int cols, float* g, BwdWs& w, cudaStream_t s) {
+// The column sums of one chunk backward (bias and norm-parameter gradients) run in order on the
+// chunk's side stream: nothing reads them before the optimizer step, so they leave the layer-to-layer
+// chain of the chunk stream. They share the workspace's partials and tickets, which nothing else uses.
+// The main stream waits only where it overwrites a buffer that a queued sum still reads; every wait
+// refers to a record made in the same backward (the flags), so none crosses a graph capture.
+struct SideQ {
+  Chunk* k;
+  cudaStream_t s, sd;
+  bool any = false, layer = false, ln2 = false, ln1 = false;
+  bool on() const { return sd != s; }
+  void fork() {   // the side stream waits for what the main stream has produced so far
+    if (!on()) return;
+    rec(k->ev_sin, s);
+    wait_ev(sd, k->ev_sin);
+    any = true;
+  }
+  bool mark(cudaEvent_t e) {   // record the side stream's position; true if recorded
+    if (!on() || !any) return false;
+    rec(e, sd);
+    return true;
+  }
+  void need(cudaEvent_t e, bool recorded) {
+    if (on() && recorded) wait_ev(s, e);
+  }
+};
+
+void bias_grad(zl_ctx* c, const void* dY, int N, int cols, float* g, BwdWs& w, SideQ& q) {
   if (!g) return;
-  ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * cols, 1);
-  launch_colsum(c->dt, dY, w.part_b, N, cols, g, w.counter, s);
+  q.fork();
+  ProfScope p(c, q.sd, PC_ELEM, 0, esz(c) * (double)N * cols, 1);
+  launch_colsum(c->dt, dY, w.part_b, N, cols, g, w.counter, q.sd);
 }
 
 void norm_param_grad(zl_ctx* c, const void* x, const float* rstd, const float* mean, const void* dyn, int N,
-                     float* gw, float* gb, BwdWs& w, cudaStream_t s) {
+                     float* gw, float* gb, BwdWs& w, SideQ& q) {
   if (!gw) return;   // frozen norm
   const bool ln = !c->llama;
-  ProfScope p(c, s, PC_NORM, 0, 2.0 * esz(c) * (double)N * c->d, 1);
-  launch_norm_bwd_dparam(c->dt, ln, x, rstd, mean, dyn, w.part_g, w.part_b, N, c->d, gw, gb, w.counter, s);
+  q.fork();
+  ProfScope p(c, q.sd, PC_NORM, 0, 2.0 * esz(c) * (double)N * c->d, 1);
+  launch_norm_bwd_dparam(c->dt, ln, x, rstd, mean, dyn, w.part_g, w.part_b, N, c->d, gw, gb, w.counter, q.sd);
 }
 
 // dy: gradient w.r.t. the layer output; dx (may be NULL): gradient w.r.t. the layer input.
 void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void* dx, BwdWs& w, int B, int S,
-               cudaStream_t s) {
+               cudaStream_t s, SideQ& q) {
   const int N = B * S, dt = c->dt;
+  // the layer above queued sums over dy's buffer, dhid, dx2 and dqkv, which this layer overwrites
+  q.need(k.ev_layer, q.layer);
   // FFN
   G(c, s, 2, c->d, c->f, N, dy, sv.act, Gm(k, li, P_W2), nullptr, nullptr);
-  bias_grad(c, dy, N, c->d, Gm(k, li, P_B2), w, s);
+  bias_grad(c, dy, N, c->d, Gm(k, li, P_B2), w, q);
   G(c, s, 1, N, c->f, c->d, dy, Wc(c, k, li, P_W2), w.da, nullptr, nullptr);
   lora_bwd(c, k, li, 3, sv.act, sv.u[3], dy, w.da, w.du, N, s);
   {
@@ -465,14 +498,16 @@ void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void*
     else launch_gelu_bwd(dt, sv.hid, w.da, w.dhid, (size_t)N * c->f, s);
   }
   G(c, s, 2, c->f1, c->d, N, w.dhid, sv.xn2, Gm(k, li, P_W1), nullptr, nullptr);
-  bias_grad(c, w.dhid, N, c->f1, Gm(k, li, P_B1), w, s);
+  bias_grad(c, w.dhid, N, c->f1, Gm(k, li, P_B1), w, q);
+  q.need(k.ev_ln1, q.ln1);   // the layer above's LN1 parameter sums read dxn
   G(c, s, 1, N, c->d, c->f1, w.dhid, Wc(c, k, li, P_W1), w.dxn, nullptr, nullptr);
   lora_bwd(c, k, li, 2, sv.xn2, sv.u[2], w.dhid, w.dxn, w.du, N, s);
   NBX(c, s, sv.x2, Wm(k, li, P_N2W), sv.rstd2, sv.mean2, w.dxn, dy, w.dx2, N);
-  norm_param_grad(c, sv.x2, sv.rstd2, sv.mean2, w.dxn, N, Gm(k, li, P_N2W), Gm(k, li, P_N2B), w, s);
+  norm_param_grad(c, sv.x2, sv.rstd2, sv.mean2, w.dxn, N, Gm(k, li, P_N2W), Gm(k, li, P_N2B), w, q);
+  q.ln2 = q.mark(k.ev_ln2);
   // attention
   G(c, s, 2, c->d, c->ad, N, w.dx2, sv.att, Gm(k, li, P_WO), nullptr, nullptr);
-  bias_grad(c, w.dx2, N, c->d, Gm(k, li, P_BO), w, s);
+  bias_grad(c, w.dx2, N, c->d, Gm(k, li, P_BO), w, q);
   G(c, s, 1, N, c->ad, c->d, w.dx2, Wc(c, k, li, P_WO), w.datt, nullptr, nullptr);
   lora_bwd(c, k, li, 1, sv.att, sv.u[1], w.dx2, w.datt, w.du, N, s);
   AB(c, s, sv.qkv, sv.att, w.datt, sv.lse, w.D, w.dqkv, B, S);
@@ -481,10 +516,13 @@ void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void*
     launch_rope(dt, w.dqkv, c->rope_cs, N, S, c->H, c->Hkv, c->hd, 1, s);
   }
   G(c, s, 2, c->qkvw, c->d, N, w.dqkv, sv.xn1, Gm(k, li, P_WQKV), nullptr, nullptr);
-  bias_grad(c, w.dqkv, N, c->qkvw, Gm(k, li, P_BQKV), w, s);
+  bias_grad(c, w.dqkv, N, c->qkvw, Gm(k, li, P_BQKV), w, q);
+  q.layer = q.mark(k.ev_layer);   // after this layer's sums over dy, dhid, dx2 and dqkv
+  q.need(k.ev_ln2, q.ln2);        // LN2 parameter sums read dxn, which the next product overwrites
   G(c, s, 1, N, c->d, c->qkvw, w.dqkv, Wc(c, k, li, P_WQKV), w.dxn, nullptr, nullptr);
   lora_bwd(c, k, li, 0, sv.xn1, sv.u[0], w.dqkv, w.dxn, w.du, N, s);
-  norm_param_grad(c, sv.x, sv.rstd1, sv.mean1, w.dxn, N, Gm(k, li, P_N1W), Gm(k, li, P_N1B), w, s);
+  norm_param_grad(c, sv.x, sv.rstd1, sv.mean1, w.dxn, N, Gm(k, li, P_N1W), Gm(k, li, P_N1B), w, q);
+  q.ln1 = q.mark(k.ev_ln1);
   if (dx) NBX(c, s, sv.x, Wm(k, li, P_N1W), sv.rstd1, sv.mean1, w.dxn, w.dx2, dx, N);
   CHECK_LAUNCH();
 }
@@ -548,12 +586,14 @@ void chunk_bwd(zl_ctx* c, Chunk& k, ChunkActs& acts, const void* dh, void* dh_in
   carve_ws(c, a, w, N, B, S);
   const size_t wmax = std::max({(size_t)c->d, (size_t)c->qkvw, (size_t)c->f1, (size_t)c->f});
   CK(cudaMemsetAsync(w.counter, 0, (size_t)colsum_groups((int)wmax) * 4, s));
+  SideQ q{&k, s, k.side ? k.side : s};
   const void* dy = dh;
   for (int i = nl - 1; i >= 0; --i) {
     void* dx = i > 0 ? ((i % 2) ? w.dy0 : w.dy1) : dh_in;
-    layer_bwd(c, k, i, acts.L[i], dy, dx, w, B, S, s);
+    layer_bwd(c, k, i, acts.L[i], dy, dx, w, B, S, s, q);
     dy = dx;
   }
+  if (q.mark(k.ev_send)) wait_ev(s, k.ev_send);   // the sums are done before the workspace goes back
   pfree(a.base, s);
 }
 
@@ -839,7 +879,9 @@ void free_ctx(zl_ctx* c) {
       if (e.labels) cudaFree(e.labels);
     }
     if (ck.s && (!shared || k == 1)) cudaStreamDestroy(ck.s);
-    for (cudaEvent_t e : {ck.ev_h, ck.ev_z, ck.ev_loss, ck.ev_hb, ck.ev_done})
+    if (ck.side && !shared) cudaStreamDestroy(ck.side);
+    for (cudaEvent_t e : {ck.ev_h, ck.ev_z, ck.ev_loss, ck.ev_hb, ck.ev_done, ck.ev_sin, ck.ev_ln2, ck.ev_layer,
+                          ck.ev_ln1, ck.ev_send})
       if (e) cudaEventDestroy(e);
   }
   for (cudaEvent_t e : c->live_ring) cudaEventDestroy(e);
@@ -1064,7 +1106,10 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
       if (cfg->serialize && k > 1) ck.s = c->ch[1].s;   // one stream for every chunk
       else CK(cudaStreamCreateWithFlags(&ck.s, cudaStreamNonBlocking));
-      for (cudaEvent_t* e2 : {&ck.ev_h, &ck.ev_z, &ck.ev_loss, &ck.ev_hb, &ck.ev_done})
+      if (cfg->serialize) ck.side = ck.s;
+      else CK(cudaStreamCreateWithFlags(&ck.side, cudaStreamNonBlocking));
+      for (cudaEvent_t* e2 : {&ck.ev_h, &ck.ev_z, &ck.ev_loss, &ck.ev_hb, &ck.ev_done, &ck.ev_sin, &ck.ev_ln2,
+                              &ck.ev_layer, &ck.ev_ln1, &ck.ev_send})
         CK(cudaEventCreateWithFlags(e2, cudaEventDisableTiming));
     }
     if (cfg->serialize) c->aux = c->ch[1].s;
