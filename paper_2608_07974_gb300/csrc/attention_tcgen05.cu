@@ -345,7 +345,8 @@ __global__ void __launch_bounds__(NTHR, 1)
 // (16-row steps 2 KB apart, head-dim blocks 8 KB apart).
 // ==============================================================================================
 constexpr int IB = 64;   // inner block rows
-constexpr int NEW = 16;  // elementwise warps: four per TMEM lane quadrant, one 16-column quarter each
+constexpr int NEW = 16;  // elementwise warps: two groups of eight (two per TMEM lane quadrant, one
+                         // 32-column half each); group g takes the inner blocks of parity g
 constexpr int NTHR_B = 64 + 32 * NEW;
 
 template <int HD>
@@ -449,10 +450,10 @@ __global__ void __launch_bounds__(NTHR_B, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(qfull, 1);
-    for (int u = 0; u < 2; ++u) {
+    for (int u = 0; u < 2; ++u) {   // buffer u is used by elementwise group u only
       mbar_init(&sfull[u], 1);
-      mbar_init(&sempty[u], NEW);
-      mbar_init(&dsfull[u], NEW);
+      mbar_init(&sempty[u], NEW / 2);
+      mbar_init(&dsfull[u], NEW / 2);
       mbar_init(&dsempty[u], 1);
     }
     mbar_init(ofull, 1);
@@ -583,38 +584,46 @@ __global__ void __launch_bounds__(NTHR_B, 1)
     if (q < S && qu == 0) Dv[si] = Dq;
     const uint64_t SL2 = f2(scale * kL2e, scale * kL2e), NL = f2(nlse2, nlse2), DD = f2(Dq, Dq);
     const int qmin = q0 + quad * 32;   // smallest query row of this warp
+    // inner blocks alternate between the two groups, so each group's chain of waits, TMEM loads,
+    // arithmetic and stores has two blocks' time; a thread takes 32 columns in two 16-column passes
+    const int grp = (warp - 2) >> 3, half = ((warp - 2) >> 2) & 1;
     bool ok = true;
-    for (int j = 0; j < nkb; ++j) {
+    for (int j = grp; j < nkb; j += 2) {
       const int buf = j & 1;
       if (!uwait(&sfull[buf], (uint32_t)(j >> 1) & 1u, abort_flag, err)) { ok = false; break; }
       fence_after();
-      float sv[16], dp[16];
-      tmem_ld16(trow + (uint32_t)(buf * 128 + qu * 16), sv);
-      tmem_ld16(trow + (uint32_t)(buf * 128 + IB + qu * 16), dp);
-      fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sempty[buf]);
-      const int kbase = j * IB + qu * 16;
-      const bool diag = kbase + 15 > qmin;   // warp-uniform: some column may lie above the diagonal
-      const int kmax = q - kbase;            // causal: columns e <= kmax
-      uint32_t pk[8];
-#pragma unroll
-      for (int e = 0; e < 16; e += 2) {
-        float2 x = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, NL));
-        if (diag) {
-          if (e > kmax) x.x = -INFINITY;
-          if (e + 1 > kmax) x.y = -INFINITY;
+      for (int sub = 0; sub < 2; ++sub) {
+        const int c0 = half * 32 + sub * 16;
+        float sv[16], dp[16];
+        tmem_ld16(trow + (uint32_t)(buf * 128 + c0), sv);
+        tmem_ld16(trow + (uint32_t)(buf * 128 + IB + c0), dp);
+        if (sub == 1) {
+          fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sempty[buf]);
         }
-        const float p0 = ex2(x.x), p1 = ex2(x.y);
-        const float2 ds = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), DD)));
-        pk[e / 2] = pack2(ds.x, ds.y);
+        const int kbase = j * IB + c0;
+        const bool diag = kbase + 15 > qmin;   // warp-uniform: some column may lie above the diagonal
+        const int kmax = q - kbase;            // causal: columns e <= kmax
+        uint32_t pk[8];
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          float2 x = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, NL));
+          if (diag) {
+            if (e > kmax) x.x = -INFINITY;
+            if (e + 1 > kmax) x.y = -INFINITY;
+          }
+          const float p0 = ex2(x.x), p1 = ex2(x.y);
+          const float2 ds = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), DD)));
+          pk[e / 2] = pack2(ds.x, ds.y);
+        }
+        if (sub == 0 && !uwait(&dsempty[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+        put_row16(sds + buf * C_::OPB, c0 >> 4, r, pk);
       }
-      const int db = j & 1;
-      if (!uwait(&dsempty[db], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-      put_row16(sds + db * C_::OPB, qu, r, pk);
+      if (!ok) break;
       fence_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&dsfull[db]);
+      if (lane == 0) mbar_arrive(&dsfull[buf]);
     }
     if (ok && uwait(ofull, 0, abort_flag, err)) {
       fence_after();
@@ -677,10 +686,10 @@ __global__ void __launch_bounds__(NTHR_B, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 2); mbar_init(&empty[s], 1); }
     mbar_init(kvfull, 1);
-    for (int u = 0; u < 2; ++u) {
+    for (int u = 0; u < 2; ++u) {   // buffer u is used by elementwise group u only
       mbar_init(&sfull[u], 1);
-      mbar_init(&sempty[u], NEW);
-      mbar_init(&pfull[u], NEW);
+      mbar_init(&sempty[u], NEW / 2);
+      mbar_init(&pfull[u], NEW / 2);
       mbar_init(&pempty[u], 1);
     }
     mbar_init(ofull, 1);
@@ -816,59 +825,63 @@ __global__ void __launch_bounds__(NTHR_B, 1)
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     const uint64_t SL2 = f2(scale * kL2e, scale * kL2e);
     // Only the causal mask is applied: queries >= S have -lse2 = -inf (P = 0) and D = 0, and rows of
-    // keys >= S are never stored.
+    // keys >= S are never stored. Inner blocks alternate between the two groups (as in the dQ kernel).
+    const int grp = (warp - 2) >> 3, half = ((warp - 2) >> 2) & 1;
     bool ok = true;
-    int stage = 0;
-    uint32_t phase = 0;
-    for (int it = 0; it < nit; ++it) {
-      const int buf = it & 1;
+    for (int it = grp; it < nit; it += 2) {
+      const int buf = it & 1, stage = it % NST;
+      const uint32_t phase = (uint32_t)(it / NST) & 1u;
       if (!uwait(&sfull[buf], (uint32_t)(it >> 1) & 1u, abort_flag, err)) { ok = false; break; }
       fence_after();
-      float sv[16], dp[16];
-      tmem_ld16(trow + (uint32_t)(buf * 128 + qu * 16), sv);
-      tmem_ld16(trow + (uint32_t)(buf * 128 + IB + qu * 16), dp);
-      fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sempty[buf]);
       // this stage's statistics: its full phase has completed (the S MMA waited on it); the wait orders
       // the producer's stores before these loads
       if (!uwait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
-      const float4* sl4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + qu * 16);
-      const float4* sd4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + IB + qu * 16);
-      float4 l[4], d[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) { l[u] = sl4[u]; d[u] = sd4[u]; }
-      const int qbase = (i0 + it) * IB + qu * 16;   // query of column 0 of this thread's 16
-      const bool diag = qbase < kmaxw;               // warp-uniform: some column may precede its key
-      const int qlo = key - qbase;                   // causal: columns e >= qlo
-      uint32_t pk[8], dk[8];
-#pragma unroll
-      for (int e4 = 0; e4 < 4; ++e4) {
-        const int e = 4 * e4;
-        float2 xa = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, f2(l[e4].x, l[e4].y)));
-        float2 xb = uf2(fma2(f2(sv[e + 2], sv[e + 3]), SL2, f2(l[e4].z, l[e4].w)));
-        if (diag) {
-          if (e < qlo) xa.x = -INFINITY;
-          if (e + 1 < qlo) xa.y = -INFINITY;
-          if (e + 2 < qlo) xb.x = -INFINITY;
-          if (e + 3 < qlo) xb.y = -INFINITY;
+      for (int sub = 0; sub < 2; ++sub) {
+        const int c0 = half * 32 + sub * 16;
+        float sv[16], dp[16];
+        tmem_ld16(trow + (uint32_t)(buf * 128 + c0), sv);
+        tmem_ld16(trow + (uint32_t)(buf * 128 + IB + c0), dp);
+        if (sub == 1) {
+          fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sempty[buf]);
         }
-        const float p0 = ex2(xa.x), p1 = ex2(xa.y), p2 = ex2(xb.x), p3 = ex2(xb.y);
-        const float2 da = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), f2(d[e4].x, d[e4].y))));
-        const float2 db = uf2(mul2(f2(p2, p3), sub2(f2(dp[e + 2], dp[e + 3]), f2(d[e4].z, d[e4].w))));
-        pk[2 * e4] = pack2(p0, p1);
-        pk[2 * e4 + 1] = pack2(p2, p3);
-        dk[2 * e4] = pack2(da.x, da.y);
-        dk[2 * e4 + 1] = pack2(db.x, db.y);
+        const float4* sl4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + c0);
+        const float4* sd4 = reinterpret_cast<const float4*>(stats + stage * 2 * IB + IB + c0);
+        float4 l[4], d[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) { l[u] = sl4[u]; d[u] = sd4[u]; }
+        const int qbase = (i0 + it) * IB + c0;   // query of column 0 of these 16
+        const bool diag = qbase < kmaxw;          // warp-uniform: some column may precede its key
+        const int qlo = key - qbase;              // causal: columns e >= qlo
+        uint32_t pk[8], dk[8];
+#pragma unroll
+        for (int e4 = 0; e4 < 4; ++e4) {
+          const int e = 4 * e4;
+          float2 xa = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, f2(l[e4].x, l[e4].y)));
+          float2 xb = uf2(fma2(f2(sv[e + 2], sv[e + 3]), SL2, f2(l[e4].z, l[e4].w)));
+          if (diag) {
+            if (e < qlo) xa.x = -INFINITY;
+            if (e + 1 < qlo) xa.y = -INFINITY;
+            if (e + 2 < qlo) xb.x = -INFINITY;
+            if (e + 3 < qlo) xb.y = -INFINITY;
+          }
+          const float p0 = ex2(xa.x), p1 = ex2(xa.y), p2 = ex2(xb.x), p3 = ex2(xb.y);
+          const float2 da = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), f2(d[e4].x, d[e4].y))));
+          const float2 db = uf2(mul2(f2(p2, p3), sub2(f2(dp[e + 2], dp[e + 3]), f2(d[e4].z, d[e4].w))));
+          pk[2 * e4] = pack2(p0, p1);
+          pk[2 * e4 + 1] = pack2(p2, p3);
+          dk[2 * e4] = pack2(da.x, da.y);
+          dk[2 * e4 + 1] = pack2(db.x, db.y);
+        }
+        if (sub == 0 && !uwait(&pempty[buf], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+        put_row16(sp + buf * 2 * C_::OPB, c0 >> 4, r, pk);
+        put_row16(sp + buf * 2 * C_::OPB + C_::OPB, c0 >> 4, r, dk);
       }
-      const int pb = it & 1;
-      if (!uwait(&pempty[pb], ((uint32_t)(it >> 1) & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
-      put_row16(sp + pb * 2 * C_::OPB, qu, r, pk);
-      put_row16(sp + pb * 2 * C_::OPB + C_::OPB, qu, r, dk);
+      if (!ok) break;
       fence_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&pfull[pb]);
-      if (++stage == NST) { stage = 0; phase ^= 1u; }
+      if (lane == 0) mbar_arrive(&pfull[buf]);
     }
     if (ok && uwait(ofull, 0, abort_flag, err)) {
       fence_after();
