@@ -809,10 +809,10 @@ __device__ __forceinline__ void loss_pass1_bf16(const bf16* zp, const bf16* tp, 
 // One block per row of logits. Pass 1: base-2 online log-sum-exp of z and t and the KL cross term
 // (two full vectors per trip for loads in flight); pass 2 (the row is still in L2) writes dz.
 template <typename T, bool TEACHER, int KLDIR>
-__global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, const T* __restrict__ t,
-                                                     const int32_t* __restrict__ labels, int V, int ldz,
-                                                     float alpha, const int* __restrict__ count,
-                                                     T* __restrict__ dz, float* __restrict__ row_loss) {
+__device__ __forceinline__ void local_loss_row(const T* __restrict__ z, const T* __restrict__ t,
+                                               const int32_t* __restrict__ labels, int V, int ldz, float alpha,
+                                               const int* __restrict__ count, T* __restrict__ dz,
+                                               float* __restrict__ row_loss) {
   pdl_wait();
   pdl_trigger();
   __shared__ Lse3 shz[32], sht[32];
@@ -945,29 +945,59 @@ __global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, co
   }
 }
 
+// Two rows per SM (the compiler's own register choice) and three rows per SM (at most 40 registers).
+template <typename T, bool TEACHER, int KLDIR>
+__global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, const T* __restrict__ t,
+                                                     const int32_t* __restrict__ labels, int V, int ldz,
+                                                     float alpha, const int* __restrict__ count,
+                                                     T* __restrict__ dz, float* __restrict__ row_loss) {
+  local_loss_row<T, TEACHER, KLDIR>(z, t, labels, V, ldz, alpha, count, dz, row_loss);
+}
+template <typename T, bool TEACHER, int KLDIR>
+__global__ void __launch_bounds__(512, 3) local_loss3_k(const T* __restrict__ z, const T* __restrict__ t,
+                                                        const int32_t* __restrict__ labels, int V, int ldz,
+                                                        float alpha, const int* __restrict__ count,
+                                                        T* __restrict__ dz, float* __restrict__ row_loss) {
+  local_loss_row<T, TEACHER, KLDIR>(z, t, labels, V, ldz, alpha, count, dz, row_loss);
+}
+
 void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labels, int N, int V, int ldz,
                        float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s) {
   note_launch(1);
   if (N <= 0) return;
   // up to 512 threads per row (one 8-wide vector each): several rows in flight per SM, and the rows
-  // being read still fit in L2 for the second pass
+  // being read still fit in L2 for the second pass. Three rows per SM (40 registers) where the rows in
+  // flight on every SM stay well inside L2 (V = 32000: 58 MB), two otherwise (V = 50257: three would
+  // hold 92 MB, and pass 2 would go back to DRAM: 293 against 260 us at 4096 rows).
   int cap = 512;
   if (const char* e = std::getenv("ZL_LOSS_THREADS")) {   // tuning override
     const int v = std::atoi(e);
-    if (v == 128 || v == 256 || v == 512 || v == 1024) cap = v;
+    if (v == 128 || v == 256 || v == 512) cap = v;
   }
   int th = 32;
   while (th < cap && th * 8 < ldz) th *= 2;
-#define LL(T, TE, KD)                                                                                        \
+  const size_t row_bytes = (size_t)ldz * dt_size(dt) * (t ? 2 : 1);
+  const bool three = dt == BF16 && 3ull * 152 * row_bytes <= (64ull << 20);
+#define LL2(T, TE, KD)                                                                                            \
   launch_pdl(local_loss_k<T, TE, KD>, N, th, 0, s, (const T*)z, (const T*)t, labels, V, ldz, alpha, count, (T*)dz, \
-                                           row_loss)
-#define LLT(T)                      \
-  if (!t) LL(T, false, 0);          \
-  else if (kl_dir == 0) LL(T, true, 0); \
-  else LL(T, true, 1);
-  if (dt == BF16) { LLT(bf16) } else { LLT(float) }
-#undef LLT
+             row_loss)
+#define LL(T, TE, KD)                                                                                           \
+  if (three)                                                                                                    \
+    launch_pdl(local_loss3_k<T, TE, KD>, N, th, 0, s, (const T*)z, (const T*)t, labels, V, ldz, alpha, count,   \
+               (T*)dz, row_loss);                                                                               \
+  else                                                                                                          \
+    LL2(T, TE, KD);
+  if (dt == BF16) {
+    if (!t) { LL(bf16, false, 0) }
+    else if (kl_dir == 0) { LL(bf16, true, 0) }
+    else { LL(bf16, true, 1) }
+  } else {   // fp32 rows: two per SM
+    if (!t) LL2(float, false, 0);
+    else if (kl_dir == 0) LL2(float, true, 0);
+    else LL2(float, true, 1);
+  }
 #undef LL
+#undef LL2
 }
 
 __global__ void count_valid_k(const int32_t* __restrict__ labels, int N, int V, int* count, unsigned* err) {
