@@ -73,6 +73,19 @@ def job_tokens_per_s(tokens_per_step: int, steps: int, world: int, max_ms: float
     return tokens_per_step * steps * world / (max_ms / 1e3)
 
 
+def step_roofline(prof, steps: int, ms_per_step: float):
+    """Whole-step roofline: the step time if every tensor-core class ran at the measured sustained bf16
+    peak and every memory-bound class at the measured HBM copy rate (algorithmic FLOPs and bytes per
+    step from the live profile), and the measured step's fraction of it."""
+    pk, pk_kind = peaks()
+    t_tensor = sum(v["flops"] for v in prof.values() if v["flops"] > 0) / steps / (pk["bf16_tflops_sustained"] * 1e12)
+    t_hbm = sum(v["bytes"] for v in prof.values() if v["flops"] == 0) / steps / (pk["hbm_gbs"] * 1e9)
+    ideal_ms = (t_tensor + t_hbm) * 1e3
+    return {"ideal_ms": ideal_ms, "tensor_ms": t_tensor * 1e3, "hbm_ms": t_hbm * 1e3, "measured_ms": ms_per_step,
+            "frac": ideal_ms / ms_per_step if ms_per_step > 0 else None,
+            "peak_kind": f"{pk_kind} bf16 sustained / HBM copy"}
+
+
 def roofline_of(prof):
     """Roofline entry of the kernel class with the largest time share in a zl_profile_read result."""
     pk, pk_kind = peaks()
@@ -332,6 +345,7 @@ def run_ours(args):
     prof = zb.zl_profile_read(eng.ctx)
     zb.zl_profile(eng.ctx, False)
     roof = roofline_of(prof)
+    step_roof = step_roofline(prof, prof_steps, ms / args.steps)
     classes = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / prof_steps,
                    "TFLOP/s" if v["flops"] else "GB/s":
                        (v["flops"] / (v["ms"] / 1e3) / 1e12) if v["flops"] else (v["bytes"] / (v["ms"] / 1e3) / 1e9)
@@ -410,7 +424,7 @@ def run_ours(args):
                 "peak_hbm_gb": zl_peak / 1e9, "bp": bp,
                 "zl_vs_bp": {"throughput": value / bp["value"], "peak_hbm": (zl_peak / 1e9) / bp["peak_hbm_gb"]}
                 if bp else None,
-                "roofline": roof, "roofline_serial": roof_serial, "kernel_classes": classes, "cpu_baseline": cpu, "e2e": e2e,
+                "roofline": roof, "roofline_serial": roof_serial, "step_roofline": step_roof, "kernel_classes": classes, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": launches, "clocks": clk}
         print(json.dumps(line), flush=True)
     if world > 1:

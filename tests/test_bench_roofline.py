@@ -1,0 +1,32 @@
+"""Host-side roofline logic of bench.py (no GPU): the whole-step roofline and the source-hash gate on the
+DRAM traffic figures."""
+import pytest
+
+import bench
+
+
+def test_step_roofline_is_flops_over_tensor_peak_plus_bytes_over_hbm():
+    pk, _ = bench.peaks()
+    steps = 4
+    # one step's worth: 2 ms of tensor work and 1 ms of memory work at the measured peaks
+    prof = {
+        "gemm_layer": {"flops": 2e-3 * pk["bf16_tflops_sustained"] * 1e12 * steps, "bytes": 1.0, "ms": 9.0, "launches": 8},
+        "local_loss": {"flops": 0.0, "bytes": 1e-3 * pk["hbm_gbs"] * 1e9 * steps, "ms": 5.0, "launches": 4},
+        "adamw": {"flops": 0.0, "bytes": 0.0, "ms": 0.0, "launches": 0},
+    }
+    r = bench.step_roofline(prof, steps, ms_per_step=6.0)
+    assert r["tensor_ms"] == pytest.approx(2.0)
+    assert r["hbm_ms"] == pytest.approx(1.0)   # bytes of tensor classes are not counted twice
+    assert r["ideal_ms"] == pytest.approx(3.0)
+    assert r["frac"] == pytest.approx(0.5)
+
+
+def test_traffic_figures_are_tied_to_the_kernel_sources(monkeypatch):
+    sha = bench.sources_sha(bench.GEMM_SOURCES)
+    monkeypatch.setitem(bench.TRAFFIC, "gemm_layer",
+                        {"sources": bench.GEMM_SOURCES, "sha256": sha, "bytes_per_launch": 123.0})
+    assert bench.measured_traffic("gemm_layer") == 123.0
+    monkeypatch.setitem(bench.TRAFFIC, "gemm_layer",
+                        {"sources": bench.GEMM_SOURCES, "sha256": "0" * 16, "bytes_per_launch": 123.0})
+    assert bench.measured_traffic("gemm_layer") is None
+    assert bench.measured_traffic("no_such_class") is None
