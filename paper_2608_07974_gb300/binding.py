@@ -21,7 +21,7 @@ ZL_DTYPE_F32, ZL_DTYPE_BF16 = 0, 1
 EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_get_param", "zl_param_numel",
            "zl_embed", "zl_forward_chunk", "zl_local_step", "zl_step", "zl_bp_step", "zl_eval_global_loss",
            "zl_read_losses", "zl_join", "zl_synchronize", "zl_peak_bytes", "zl_reset_peak", "zl_last_error",
-           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
+           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_gemm_ex", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
            "zl_chunk_load", "zl_replay"]
 
 
@@ -74,6 +74,7 @@ def _load() -> C.CDLL:
         "zl_op_local_loss": [i, vp, vp, vp, i, i, i, f, i, vp, vp, vp, vp],
         "zl_op_local_loss_noalloc": [i, vp, vp, vp, i, i, i, f, i, vp, vp, vp],
         "zl_op_gemm": [i, i, i, i, i, vp, vp, vp, vp],
+        "zl_op_gemm_ex": [i, i, i, i, i, vp, vp, vp, vp, vp, i, vp],
         "zl_op_attention": [i, vp, vp, vp, i, i, i, i, i, vp],
         "zl_op_attention_bwd": [i, vp, vp, vp, vp, vp, i, i, i, i, i, vp],
         "zl_profile": [vp, i],
@@ -260,6 +261,20 @@ def zl_op_gemm(dtype: int, mode: int, M: int, N: int, K: int, A, B, Cm, stream: 
     _need(B, act, "B")
     _need(Cm, ("float32",) if mode == 2 else act, "C")
     _check(_lib.zl_op_gemm(dtype, mode, M, N, K, _p(A), _p(B), _p(Cm), stream))
+
+
+def zl_op_gemm_ex(dtype: int, mode: int, M: int, N: int, K: int, A, B, Cm, bias=None, R=None, r_mode: int = 0,
+                  stream: int = 0) -> None:
+    act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
+    _need(A, act, "A")
+    _need(B, act, "B")
+    _need(Cm, act, "C")
+    if bias is not None:
+        _need(bias, ("float32",), "bias")
+    if R is not None:
+        _need(R, act, "R")
+    _check(_lib.zl_op_gemm_ex(dtype, mode, M, N, K, _p(A), _p(B), _p(Cm), _p(bias) if bias is not None else None,
+                              _p(R) if R is not None else None, r_mode, stream))
 
 
 def zl_profile(ctx, on: bool) -> None:

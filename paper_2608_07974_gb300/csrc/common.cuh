@@ -88,6 +88,18 @@ __device__ __forceinline__ uint32_t bf2_max(uint32_t a, uint32_t b) {
   return r;
 }
 
+// Derivative of the tanh-form GELU g(u) = 0.5 u (1 + tanh(k (u + c u^3))), k = sqrt(2 / pi), c = 0.044715:
+// g'(u) = 0.5 (1 + t) + 0.5 u (1 - t^2) k (1 + 3 c u^2) with t = tanh(k (u + c u^3)). approx: the SFU's
+// tanh.approx (relative error about 2^-11; for bf16 activations), else tanhf.
+__device__ __forceinline__ float gelu_tanh_grad(float u, bool approx) {
+  const float k = 0.7978845608028654f, c = 0.044715f;
+  const float a = k * (u + c * u * u * u);
+  float t;
+  if (approx) asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(a));
+  else t = tanhf(a);
+  return 0.5f * (1.f + t) + 0.5f * u * (1.f - t * t) * k * (1.f + 3.f * c * u * u);
+}
+
 template <typename T> struct Vec8;
 template <> struct Vec8<bf16> {
   __device__ __forceinline__ static void load(const bf16* p, float* f) {

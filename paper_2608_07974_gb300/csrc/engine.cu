@@ -273,13 +273,13 @@ struct ProfScope {
 // Profiled launch wrappers (algorithmic FLOPs / bytes per launch)
 // ----------------------------------------------------------------------------------------------
 void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, const void* B, void* C,
-       const float* bias, const void* R, float alpha = 1.f) {
+       const float* bias, const void* R, float alpha = 1.f, int rmode = 0) {
   if (!C) return;   // frozen weight: no gradient to form
   const double e = (double)esz(c);
   const double out = mode == 2 ? 8.0 * M * N : (R ? 2.0 : 1.0) * e * M * N;
   const bool head = B == c->lm_head;
   ProfScope p(c, s, head ? PC_GEMM_HEAD : PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
-  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool, alpha);
+  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool, alpha, rmode);
 }
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
   const double e = (double)esz(c), N = (double)B * S;
@@ -1922,6 +1922,21 @@ zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, co
   }
   return guarded(nullptr, [&]() -> zl_status {
     gemm(dtype, mode, M, N, K, A, B, C, nullptr, nullptr, (cudaStream_t)stream);
+    CHECK_LAUNCH();
+    return ZL_OK;
+  });
+}
+
+zl_status zl_op_gemm_ex(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C,
+                        const float* bias, const void* R, int r_mode, void* stream) {
+  if (!A || !B || !C) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if ((dtype != 0 && dtype != 1) || mode < 0 || mode > 1 || M < 0 || N < 0 || K < 0 || (r_mode != 0 && r_mode != 1) ||
+      (r_mode == 1 && !R)) {
+    g_err = "bad dtype/mode/size/r_mode (modes 0 and 1; r_mode 1 needs R)";
+    return ZL_ERR_ARG;
+  }
+  return guarded(nullptr, [&]() -> zl_status {
+    gemm(dtype, mode, M, N, K, A, B, C, bias, R, (cudaStream_t)stream, nullptr, nullptr, 1.f, r_mode);
     CHECK_LAUNCH();
     return ZL_OK;
   });

@@ -1,6 +1,8 @@
 // CUDA-core GEMM with fp32 accumulation: the fp32 path (the tiny fp32 workload needs fp32
 // accuracy, which rules out TF32 tensor cores) and the reference the tensor-core GEMM is tested
 // against. Row-major operands; the three modes of ops.h.
+#include <type_traits>
+
 #include "common.cuh"
 #include "ops.h"
 
@@ -23,7 +25,8 @@ __device__ __forceinline__ float ldB(const T* B, int N, int K, int k, int n) {
 template <typename T, typename TC, int MODE>
 __global__ void __launch_bounds__(256) gemm_simt_k(int M, int N, int K, const T* __restrict__ A,
                                                    const T* __restrict__ B, TC* C,
-                                                   const float* __restrict__ bias, const TC* R, float alpha) {
+                                                   const float* __restrict__ bias, const TC* R, float alpha,
+                                                   int rmode) {
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
@@ -65,7 +68,7 @@ __global__ void __launch_bounds__(256) gemm_simt_k(int M, int N, int K, const T*
         reinterpret_cast<float*>(C)[o] += v;
       } else {
         if (bias) v += bias[n];
-        if (R) v += to_f(R[o]);
+        if (R) v = rmode ? v * gelu_tanh_grad(to_f(R[o]), std::is_same<TC, bf16>::value) : v + to_f(R[o]);
         C[o] = from_f<TC>(v);
       }
     }
@@ -74,25 +77,26 @@ __global__ void __launch_bounds__(256) gemm_simt_k(int M, int N, int K, const T*
 
 template <typename T>
 void gemm_simt_t(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-                 const void* R, cudaStream_t s, float alpha) {
+                 const void* R, cudaStream_t s, float alpha, int rmode) {
   dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM), block(256);
   if (mode == 0)
-    gemm_simt_k<T, T, 0><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, bias, (const T*)R, alpha);
+    gemm_simt_k<T, T, 0><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, bias, (const T*)R, alpha,
+                                                 rmode);
   else if (mode == 1)
-    gemm_simt_k<T, T, 1><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, nullptr, (const T*)R,
-                                                 alpha);
+    gemm_simt_k<T, T, 1><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (T*)C, bias, (const T*)R,
+                                                 alpha, rmode);
   else
     gemm_simt_k<T, float, 2><<<grid, block, 0, s>>>(M, N, K, (const T*)A, (const T*)B, (float*)C, nullptr, nullptr,
-                                                    alpha);
+                                                    alpha, 0);
 }
 }  // namespace
 
 void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-               const void* R, cudaStream_t s, float alpha) {
+               const void* R, cudaStream_t s, float alpha, int rmode) {
   note_launch(1);
   if (M <= 0 || N <= 0) return;
-  if (dt == BF16) gemm_simt_t<bf16>(mode, M, N, K, A, B, C, bias, R, s, alpha);
-  else gemm_simt_t<float>(mode, M, N, K, A, B, C, bias, R, s, alpha);
+  if (dt == BF16) gemm_simt_t<bf16>(mode, M, N, K, A, B, C, bias, R, s, alpha, rmode);
+  else gemm_simt_t<float>(mode, M, N, K, A, B, C, bias, R, s, alpha, rmode);
 }
 
 }  // namespace zl
@@ -100,8 +104,8 @@ void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void*
 namespace zl {
 // GEMM dispatch: the tensor-core kernel where it applies, else the CUDA-core kernel.
 void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-          const void* R, cudaStream_t s, unsigned* err, cudaMemPool_t pool, float alpha) {
-  if (dt == BF16 && gemm_tc(mode, M, N, K, A, B, C, bias, R, err, s, pool, alpha)) return;
-  gemm_simt(dt, mode, M, N, K, A, B, C, bias, R, s, alpha);
+          const void* R, cudaStream_t s, unsigned* err, cudaMemPool_t pool, float alpha, int rmode) {
+  if (dt == BF16 && gemm_tc(mode, M, N, K, A, B, C, bias, R, err, s, pool, alpha, rmode)) return;
+  gemm_simt(dt, mode, M, N, K, A, B, C, bias, R, s, alpha, rmode);
 }
 }  // namespace zl

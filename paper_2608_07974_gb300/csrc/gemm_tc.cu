@@ -42,6 +42,7 @@ struct Args {
   int tiles_m, tiles_n;
   int splits, kb_per_split;   // split-K: unit u -> split u / tiles, k blocks [s*kps, min(nk, (s+1)*kps))
   float alpha;                // scale of the product
+  int rmode;                  // R in modes 0/1: 0 adds it (residual); 1 multiplies by GELU'(R) (R = the GELU input)
 };
 
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, operand majors, N, M.
@@ -257,8 +258,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (nh + 8 * j < g.N) {
                   float r8[8];
                   Vec8<bf16>::load(rr + 8 * j, r8);
+                  if (g.rmode) {
 #pragma unroll
-                  for (int e = 0; e < 8; ++e) v[8 * j + e] += r8[e];
+                    for (int e = 0; e < 8; ++e) v[8 * j + e] *= gelu_tanh_grad(r8[e], true);
+                  } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[8 * j + e] += r8[e];
+                  }
                 }
               }
             }
@@ -307,7 +313,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // Sums the split-K partials in split order (deterministic) and applies the epilogue.
 __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, int mode, void* C,
-                                const float* __restrict__ bias, const bf16* R, float alpha) {
+                                const float* __restrict__ bias, const bf16* R, float alpha, int rmode) {
   pdl_wait();
   pdl_trigger();
   const size_t n8 = (size_t)M * N / 8, MN = (size_t)M * N;
@@ -338,8 +344,13 @@ __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M,
       if (R) {
         float r[8];
         Vec8<bf16>::load(R + e, r);
+        if (rmode) {
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc[q] += r[q];
+          for (int q = 0; q < 8; ++q) acc[q] *= gelu_tanh_grad(r[q], true);
+        } else {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) acc[q] += r[q];
+        }
       }
       Vec8<bf16>::store((bf16*)C + e, acc);
     }
@@ -469,7 +480,7 @@ bool gemm_tc_available() { return tc::init(); }
 
 // Returns false when the shape / alignment is outside what the tensor-core path handles.
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha) {
+             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode) {
   if (!tc::init()) return false;
   if (M < 16 || N < 16 || K < 16) return false;
   auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
@@ -488,15 +499,15 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
   }
   tc::Args a;
   a.M = M; a.N = N; a.K = K; a.mode = mode;
-  a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err; a.alpha = alpha;
+  a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err; a.alpha = alpha; a.rmode = rmode;
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
   a.tiles_n = (N + bn - 1) / bn;
   const int nk = (K + tc::BK - 1) / tc::BK;
-  a.splits = splits;
   a.kb_per_split = (nk + splits - 1) / splits;
+  a.splits = (nk + a.kb_per_split - 1) / a.kb_per_split;   // no empty split (its slice would never be formed)
   float* ws = nullptr;
-  if (splits > 1) {
-    const size_t bytes = (size_t)splits * M * N * 4;
+  if (a.splits > 1) {
+    const size_t bytes = (size_t)a.splits * M * N * 4;
     cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&ws, bytes, pool, s) : cudaMallocAsync((void**)&ws, bytes, s);
     if (e != cudaSuccess) {   // no room for the partials: one split
       cudaGetLastError();
@@ -521,7 +532,8 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
       note_launch(1);
       const size_t n8 = (size_t)M * N / 8;
       const int blocks = (int)std::min<size_t>((n8 + 255) / 256, (size_t)tc::g_sms * 8);
-      launch_pdl(tc::splitk_reduce_k, blocks, 256, 0, s, ws, a.splits, M, N, mode, C, bias, (const bf16*)R, alpha);
+      launch_pdl(tc::splitk_reduce_k, blocks, 256, 0, s, ws, a.splits, M, N, mode, C, bias, (const bf16*)R, alpha,
+                 rmode);
     }
     cudaFreeAsync(ws, s);
   }

@@ -656,11 +656,7 @@ __global__ void gelu_bwd_k(const T* __restrict__ x, const T* __restrict__ dy, T*
     Vec8<T>::load(x + i * 8, f);
     Vec8<T>::load(dy + i * 8, d);
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const float u = f[q], t = gelu_tanh<T>(gelu_inner(u));
-      const float du = 0.7978845608028654f * (1.f + 3.f * 0.044715f * u * u);
-      d[q] *= 0.5f * (1.f + t) + 0.5f * u * (1.f - t * t) * du;
-    }
+    for (int q = 0; q < 8; ++q) d[q] *= gelu_tanh_grad(f[q], std::is_same<T, bf16>::value);
     Vec8<T>::store(dx + i * 8, d);
   }
 }

@@ -73,13 +73,16 @@ void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
 // alignment rules hold, everything else on the CUDA-core kernel. err: device word for timeouts;
 // pool: stream-ordered pool for split-K partials (NULL: the device's default pool).
 // alpha scales the product: C = alpha A op(B) (+ bias) (+ R), or C += alpha A^T B. R may alias C.
+// rmode 1 (modes 0 and 1): C = alpha A op(B) * GELU'(R) instead of + R (R is the GELU input; bf16 uses
+// the SFU tanh, as the GELU backward kernel does).
 void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-          const void* R, cudaStream_t s, unsigned* err = nullptr, cudaMemPool_t pool = nullptr, float alpha = 1.f);
+          const void* R, cudaStream_t s, unsigned* err = nullptr, cudaMemPool_t pool = nullptr, float alpha = 1.f,
+          int rmode = 0);
 bool gemm_tc_available();
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha);
+             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode = 0);
 void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
-               const void* R, cudaStream_t s, float alpha = 1.f);
+               const void* R, cudaStream_t s, float alpha = 1.f, int rmode = 0);
 
 // Causal attention over qkv [N, (H + 2 Hkv) hd] (token-major, rows b*S + s): out [N, H hd], lse [B, H, S].
 // bf16 with head dim 64 or 128: the tcgen05 kernel (err: device word for its bounded waits, may be NULL);

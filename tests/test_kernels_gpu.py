@@ -95,6 +95,53 @@ def test_gemm_matches_matmul(B, dtype, mode, M, N, K):
     assert err <= tol, err
 
 
+def _gelu_tanh_grad(u):
+    """d/du of the tanh-form GELU, by autograd through PyTorch's own GELU (fp64)."""
+    u = u.detach().double().requires_grad_(True)
+    (g,) = torch.autograd.grad(torch.nn.functional.gelu(u, approximate="tanh").sum(), u)
+    return g
+
+
+# The fused epilogue of modes 0 / 1 (zl_op_gemm_ex): bias, residual add, and the GELU-gradient product
+# the GPT-2 FFN backward uses; on the tensor-core path with and without split-K ("BN:SPLITS" forces the
+# tile), and on the CUDA-core path (fp32).
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("r_mode,with_bias", [(0, True), (0, False), (1, False)])
+@pytest.mark.parametrize("tile", [None, "128:3"])
+@pytest.mark.parametrize("M,N,K", [(256, 384, 512), (130, 136, 200)])
+def test_gemm_fused_epilogue(B, monkeypatch, dtype, mode, r_mode, with_bias, tile, M, N, K):
+    if dtype == "f32" and tile:
+        pytest.skip("the tile override applies to the tensor-core path")
+    if tile:
+        monkeypatch.setenv("ZL_GEMM_TILE", tile)
+    g = torch.Generator(device="cuda").manual_seed(M + 5 * N + 11 * K + mode + 3 * r_mode)
+    td = torch.bfloat16 if dtype == "bf16" else torch.float32
+    a = torch.randn(M, K, device="cuda", generator=g).to(td)
+    b = (torch.randn(N, K, device="cuda", generator=g) if mode == 0 else
+         torch.randn(K, N, device="cuda", generator=g)).to(td)
+    R = (2.5 * torch.randn(M, N, device="cuda", generator=g)).to(td)
+    bias = torch.randn(N, device="cuda", generator=g) if with_bias else None
+    prod = a.double() @ (b.double().T if mode == 0 else b.double())
+    if r_mode == 0:
+        ref = prod + R.double() + (bias.double() if with_bias else 0.0)
+    else:
+        ref = prod * _gelu_tanh_grad(R)
+    c = torch.full((M, N), float("nan"), device="cuda", dtype=td)
+    B.zl_op_gemm_ex(1 if dtype == "bf16" else 0, mode, M, N, K, a, b, c, bias=bias, R=R, r_mode=r_mode)
+    torch.cuda.synchronize()
+    err = float((c.double() - ref).abs().max()) / float(ref.abs().max())
+    assert err <= (1e-2 if dtype == "bf16" else 1e-5), err
+
+
+def test_gemm_fused_epilogue_rejects_bad_arguments(B):
+    a = torch.zeros(16, 16, device="cuda")
+    with pytest.raises(B.ZLError):
+        B.zl_op_gemm_ex(0, 2, 16, 16, 16, a, a, a, R=a, r_mode=0)    # mode 2 has no epilogue inputs
+    with pytest.raises(B.ZLError):
+        B.zl_op_gemm_ex(0, 0, 16, 16, 16, a, a, a, r_mode=1)         # r_mode 1 needs R
+
+
 # Shapes of the layer GEMMs (GPT-2 and Llama workloads) plus ragged tiles; the tensor-core path
 # takes every bf16 case here. Reference: fp32 torch.matmul of the same bf16 values.
 TC_SHAPES = [(0, 256, 384, 128), (0, 4096, 2304, 768), (1, 4096, 768, 3072), (2, 2304, 768, 4096),
