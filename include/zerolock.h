@@ -241,13 +241,15 @@ zl_status zl_op_local_loss_noalloc(int dtype, const void* z, const void* t, cons
 zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C,
                      void* stream);
 
-/* zl_op_gemm with the fused epilogue of modes 0 and 1 (the chunk forward and backward use it):
- * C = A op(B) (+ bias[N], fp32) (+ R[M,N]) when r_mode == 0, or C = A op(B) * GELU'(R) when
- * r_mode == 1 (R the input of the tanh-form GELU, so C is the gradient at that input; the
- * backward of the GPT-2 FFN activation). bias and R may be NULL (R is required for r_mode 1);
- * R has the dtype and layout of C and may alias it. Mode 2 takes neither (ZL_ERR_ARG). */
+/* zl_op_gemm with the fused epilogues the chunk forward and backward use. Modes 0 and 1:
+ * C = A op(B) (+ bias[N], fp32, read) (+ R[M,N]) when r_mode == 0, or C = A op(B) * GELU'(R) when
+ * r_mode == 1 (R the input of the tanh-form GELU, so C is the gradient at that input). bias and R
+ * may be NULL (R is required for r_mode 1); R has the dtype and layout of C and may alias it.
+ * Mode 2 (dW): C += A^T B and, if bias is not NULL, bias[M] += the column sums of A[K,M] (the bias
+ * gradient that goes with the weight gradient, by the engine's column-sum kernel); R must be NULL
+ * and r_mode 0 (else ZL_ERR_ARG). */
 zl_status zl_op_gemm_ex(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C,
-                        const float* bias, const void* R, int r_mode, void* stream);
+                        float* bias, const void* R, int r_mode, void* stream);
 
 #ifdef __cplusplus
 }

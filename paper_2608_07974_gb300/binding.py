@@ -268,7 +268,7 @@ def zl_op_gemm_ex(dtype: int, mode: int, M: int, N: int, K: int, A, B, Cm, bias=
     act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
     _need(A, act, "A")
     _need(B, act, "B")
-    _need(Cm, act, "C")
+    _need(Cm, ("float32",) if mode == 2 else act, "C")
     if bias is not None:
         _need(bias, ("float32",), "bias")
     if R is not None:

@@ -1928,15 +1928,27 @@ zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, co
 }
 
 zl_status zl_op_gemm_ex(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C,
-                        const float* bias, const void* R, int r_mode, void* stream) {
+                        float* bias, const void* R, int r_mode, void* stream) {
   if (!A || !B || !C) { g_err = "NULL argument"; return ZL_ERR_ARG; }
-  if ((dtype != 0 && dtype != 1) || mode < 0 || mode > 1 || M < 0 || N < 0 || K < 0 || (r_mode != 0 && r_mode != 1) ||
-      (r_mode == 1 && !R)) {
-    g_err = "bad dtype/mode/size/r_mode (modes 0 and 1; r_mode 1 needs R)";
+  if ((dtype != 0 && dtype != 1) || mode < 0 || mode > 2 || M < 0 || N < 0 || K < 0 || (r_mode != 0 && r_mode != 1) ||
+      (r_mode == 1 && !R) || (mode == 2 && (R || r_mode))) {
+    g_err = "bad dtype/mode/size/r_mode (r_mode 1 needs R; mode 2 takes no R)";
     return ZL_ERR_ARG;
   }
+  if (mode == 2 && bias && M % 8 != 0) { g_err = "mode 2 column sums need M % 8 == 0"; return ZL_ERR_ARG; }
   return guarded(nullptr, [&]() -> zl_status {
-    gemm(dtype, mode, M, N, K, A, B, C, bias, R, (cudaStream_t)stream, nullptr, nullptr, 1.f, r_mode);
+    cudaStream_t s = (cudaStream_t)stream;
+    gemm(dtype, mode, M, N, K, A, B, C, mode == 2 ? nullptr : bias, R, s, nullptr, nullptr, 1.f, r_mode);
+    if (mode == 2 && bias && K > 0) {   // the column sums of A: the column-sum kernel of the bias gradients
+      float* part = nullptr;
+      unsigned* cnt = nullptr;
+      CK(cudaMallocAsync((void**)&part, (size_t)colsum_blocks(K) * M * 4, s));
+      CK(cudaMallocAsync((void**)&cnt, (size_t)colsum_groups(M) * 4, s));
+      CK(cudaMemsetAsync(cnt, 0, (size_t)colsum_groups(M) * 4, s));
+      launch_colsum(dtype, A, part, K, M, bias, cnt, s);
+      CK(cudaFreeAsync(part, s));
+      CK(cudaFreeAsync(cnt, s));
+    }
     CHECK_LAUNCH();
     return ZL_OK;
   });

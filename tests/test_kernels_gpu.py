@@ -134,10 +134,35 @@ def test_gemm_fused_epilogue(B, monkeypatch, dtype, mode, r_mode, with_bias, til
     assert err <= (1e-2 if dtype == "bf16" else 1e-5), err
 
 
+# dW with the bias gradient: C += A^T B (tensor-core GEMM for bf16 under the default and forced tiles,
+# CUDA cores for fp32) and db += column sums of A (the column-sum kernel of the bias gradients).
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("tile", [None, "64:1", "256:1", "128:3"])
+@pytest.mark.parametrize("M,N,K", [(768, 768, 4096), (2304, 768, 512), (136, 264, 333)])
+def test_gemm_dw_with_bias_gradient(B, monkeypatch, dtype, tile, M, N, K):
+    if dtype == "f32" and tile:
+        pytest.skip("the tile override applies to the tensor-core path")
+    if tile:
+        monkeypatch.setenv("ZL_GEMM_TILE", tile)
+    g = torch.Generator(device="cuda").manual_seed(M + 7 * N + 13 * K)
+    td = torch.bfloat16 if dtype == "bf16" else torch.float32
+    a = torch.randn(K, M, device="cuda", generator=g).to(td)
+    b = torch.randn(K, N, device="cuda", generator=g).to(td)
+    c0 = torch.randn(M, N, device="cuda", generator=g)
+    db0 = torch.randn(M, device="cuda", generator=g)
+    c, db = c0.clone(), db0.clone()
+    B.zl_op_gemm_ex(1 if dtype == "bf16" else 0, 2, M, N, K, a, b, c, bias=db)
+    torch.cuda.synchronize()
+    ref = c0.double() + a.double().T @ b.double()
+    ref_db = db0.double() + a.double().sum(0)
+    assert float((c.double() - ref).abs().max()) / float(ref.abs().max()) <= 1e-5
+    assert float((db.double() - ref_db).abs().max()) / float(ref_db.abs().max()) <= 1e-5
+
+
 def test_gemm_fused_epilogue_rejects_bad_arguments(B):
     a = torch.zeros(16, 16, device="cuda")
     with pytest.raises(B.ZLError):
-        B.zl_op_gemm_ex(0, 2, 16, 16, 16, a, a, a, R=a, r_mode=0)    # mode 2 has no epilogue inputs
+        B.zl_op_gemm_ex(0, 2, 16, 16, 16, a, a, a, R=a, r_mode=0)    # mode 2 takes no R
     with pytest.raises(B.ZLError):
         B.zl_op_gemm_ex(0, 0, 16, 16, 16, a, a, a, r_mode=1)         # r_mode 1 needs R
 
