@@ -85,8 +85,8 @@ void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void*
                const void* R, cudaStream_t s, float alpha = 1.f, int rmode = 0);
 
 // Causal attention over qkv [N, (H + 2 Hkv) hd] (token-major, rows b*S + s): out [N, H hd], lse [B, H, S].
-// bf16 with head dim 64 or 128: the tcgen05 kernel (err: device word for its bounded waits, may be NULL);
-// other bf16 shapes: mma.sync; fp32: CUDA cores.
+// bf16 with head dim 64 or 128: the one-pass tcgen05 kernel (err: device word for its bounded waits, may
+// be NULL); other bf16 shapes: mma.sync; fp32: CUDA cores.
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,
               cudaStream_t s, unsigned* err = nullptr);
 // Gradients into dqkv (same layout as qkv). Dbuf: [B, H, S] scratch. bf16 with head dim 64 or 128: the
