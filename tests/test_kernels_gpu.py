@@ -282,6 +282,61 @@ def test_attention_matches_sdpa(B, dtype, Bb, S, H, Hkv, hd):
         assert cos >= 0.9995, (lo, cos)
 
 
+# Scores that grow along the sequence (keys aligned with a shared direction, scaled by position): every
+# 128-key block's maximum exceeds the previous one by far more than the rescale threshold, so the
+# one-pass forward rescales O in TMEM at every block; outputs, log-sum-exp and gradients against the
+# fp32 reference as in test_attention_matches_sdpa.
+@pytest.mark.parametrize("Bb,S,H,Hkv,hd", [(1, 700, 2, 2, 64), (2, 520, 4, 2, 64), (1, 600, 2, 2, 128)])
+def test_attention_rescales_on_growing_scores(B, Bb, S, H, Hkv, hd):
+    g = torch.Generator(device="cuda").manual_seed(S + hd)
+    W = (H + 2 * Hkv) * hd
+    u = torch.ones(hd, device="cuda") / hd ** 0.5
+    qkv = torch.randn(Bb * S, W, device="cuda", generator=g)
+    qkv[:, : (H + Hkv) * hd] *= 0.05          # small noise on queries and keys; values stay N(0, 1)
+    pos = torch.arange(S, device="cuda", dtype=torch.float32).repeat(Bb)
+    for hh in range(H):                       # queries ~ 4 u
+        qkv[:, hh * hd:(hh + 1) * hd] += 4.0 * u
+    ramp = 0.08 * hd ** 0.5 / 4.0            # keys ~ ramp pos u: scores grow by ~ 0.08 per key, ~ 15 (log2) per block
+    for kk in range(Hkv):
+        c = (H + kk) * hd
+        qkv[:, c:c + hd] += (ramp * pos)[:, None] * u
+    qkv = qkv.to(torch.bfloat16)
+    dout = torch.randn(Bb * S, H * hd, device="cuda", generator=g).to(torch.bfloat16)
+    out = torch.empty(Bb * S, H * hd, device="cuda", dtype=torch.bfloat16)
+    lse = torch.empty(Bb, H, S, device="cuda", dtype=torch.float32)
+    dq = torch.full_like(qkv, float("nan"))
+    B.zl_op_attention(B.ZL_DTYPE_BF16, qkv, out, lse, Bb, S, H, Hkv, hd)
+    B.zl_op_attention_bwd(B.ZL_DTYPE_BF16, qkv, out, dout, lse, dq, Bb, S, H, Hkv, hd)
+    torch.cuda.synchronize()
+    x = qkv.float().view(Bb, S, W).requires_grad_(True)
+    q = x[..., : H * hd].view(Bb, S, H, hd).transpose(1, 2)
+    k = x[..., H * hd: (H + Hkv) * hd].view(Bb, S, Hkv, hd).transpose(1, 2)
+    v = x[..., (H + Hkv) * hd:].view(Bb, S, Hkv, hd).transpose(1, 2)
+    rep = H // Hkv
+    k, v = k.repeat_interleave(rep, 1), v.repeat_interleave(rep, 1)
+    sc = (q @ k.transpose(-1, -2)) / hd ** 0.5
+    sc = sc.masked_fill(torch.triu(torch.ones(S, S, dtype=torch.bool, device="cuda"), 1), float("-inf"))
+    ref_lse = torch.logsumexp(sc, -1)
+    ref = (torch.softmax(sc, -1) @ v).transpose(1, 2).reshape(Bb * S, H * hd)
+    (gx,) = torch.autograd.grad(ref, x, dout.float().view(Bb * S, H * hd))
+    # the scores really grow: maxima of the last query row over full 128-key blocks rise by more than 8
+    # (log2 units)
+    last = sc[0, 0, S - 1] * 1.4426950408889634
+    bm = torch.stack([last[j:j + 128].max() for j in range(0, S - 127, 128)])
+    assert float((bm[1:] - bm[:-1]).min()) > 8.0
+    ref, ref_lse = ref.detach(), ref_lse.detach()
+    assert float((out.float() - ref).abs().max()) <= 2e-2 * max(1.0, float(ref.abs().max()))
+    assert float((lse - ref_lse).abs().max()) <= 1e-3 * max(1.0, float(ref_lse.abs().max()))
+    # Gradients: a sanity bound only. With keys sharing a large aligned component, dQ = sum_k dS K is a
+    # small residue of large, mostly cancelling terms, so the bf16 rounding of dS (as in any bf16
+    # backward) costs a few 1e-3 of cosine here; the forward checks above are the point of this test.
+    gx = gx.view(Bb * S, W)
+    for lo, hi in ((0, H * hd), (H * hd, (H + Hkv) * hd), ((H + Hkv) * hd, W)):
+        a, r = dq.float()[:, lo:hi].reshape(-1).double(), gx[:, lo:hi].reshape(-1).double()
+        cos = float(a @ r / (a.norm() * r.norm() + 1e-30))
+        assert cos >= 0.99, (lo, cos)
+
+
 @pytest.mark.parametrize("mode,M,N,K", [(0, 4096, 16, 768), (1, 4096, 2304, 16), (2, 16, 2304, 4096),
                                         (2, 16, 768, 4096), (0, 512, 16, 3072), (1, 300, 768, 16)])
 def test_gemm_rank16_shapes(B, mode, M, N, K):
