@@ -321,7 +321,7 @@ def test_attention_rescales_on_growing_scores(B, Bb, S, H, Hkv, hd):
     (gx,) = torch.autograd.grad(ref, x, dout.float().view(Bb * S, H * hd))
     # the scores really grow: maxima of the last query row over full 128-key blocks rise by more than 8
     # (log2 units)
-    last = sc[0, 0, S - 1] * 1.4426950408889634
+    last = sc[0, 0, S - 1].detach() * 1.4426950408889634
     bm = torch.stack([last[j:j + 128].max() for j in range(0, S - 127, 128)])
     assert float((bm[1:] - bm[:-1]).min()) > 8.0
     ref, ref_lse = ref.detach(), ref_lse.detach()
