@@ -273,13 +273,13 @@ struct ProfScope {
 // Profiled launch wrappers (algorithmic FLOPs / bytes per launch)
 // ----------------------------------------------------------------------------------------------
 void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, const void* B, void* C,
-       const float* bias, const void* R, float alpha = 1.f, int rmode = 0) {
+       const float* bias, const void* R, float alpha = 1.f) {
   if (!C) return;   // frozen weight: no gradient to form
   const double e = (double)esz(c);
   const double out = mode == 2 ? 8.0 * M * N : (R ? 2.0 : 1.0) * e * M * N;
   const bool head = B == c->lm_head;
   ProfScope p(c, s, head ? PC_GEMM_HEAD : PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
-  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool, alpha, rmode);
+  gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool, alpha);
 }
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
   const double e = (double)esz(c), N = (double)B * S;
