@@ -1,5 +1,6 @@
 // Causal attention on the 5th-generation tensor cores (sm_103a), head dims 64 and 128: a one-pass
-// forward with lazy rescaling and a two-kernel backward (dQ; dK and dV).
+// forward with lazy rescaling and a two-kernel backward (dQ; dK and dV) with 64-row (head dim 128) or
+// 128-row (head dim 64) inner blocks.
 //
 // One CTA per 128 rows of one (batch, head). TMA brings the CTA's fixed tile once and the streamed tiles
 // through a stage ring (128-byte swizzle; a 3-D tensor map over [batch, token, feature] reads rows past
@@ -331,7 +332,8 @@ __global__ void __launch_bounds__(NTHR, 1)
 }
 
 // ==============================================================================================
-// Backward: two kernels, each a fixed-order sum per output row (no atomics).
+// Backward: two kernels, each a fixed-order sum per output row (no atomics). Head dim 128 runs the
+// kernels of this section (64-row inner blocks); head dim 64 the 128-row variant that follows them.
 //   dQ kernel: one CTA per 128 queries; 64-key inner blocks j: S = Q K_j^T, dP = dO V_j^T (TMEM),
 //              dS = P * (dP - D) (shared memory, bf16), dQ += dS K_j (TMEM); also writes D = rowsum(dO * O).
 //   dK/dV kernel: one CTA per 128 keys; 64-query inner blocks i: S^T = K Q_i^T, dP^T = V dO_i^T,
@@ -917,6 +919,528 @@ __global__ void __launch_bounds__(NTHR_B, 1)
   if (warp == 1) tmem_release(fin, tmem);
 }
 
+// ----------------------------------------------------------------------------------------------
+// Backward with 128-wide inner blocks (head dim 64): per 128 keys (dQ) or 128 queries (dK / dV), one
+// round of hand-offs and 24 products instead of two rounds and 32. S / dP are single-buffered in TMEM
+// (columns 0 and 128): the elementwise warps read them into registers in two 16-column passes and
+// release them after the second, so the next block's products still overlap the arithmetic. Sixteen
+// elementwise warps, four per lane quadrant, 32 columns each. A 128-row tile of Q / dO / K / V is one
+// K-major [128 x 64] block per 64 head-dim columns (16 KB); as the MN-major B operand of the
+// accumulating product its 16-row steps are 2 KB apart.
+// ----------------------------------------------------------------------------------------------
+constexpr int WB = 128;   // inner block rows
+
+template <int HD>
+struct WCfg {
+  static constexpr int T128 = 128 * HD * 2;
+  static constexpr int NST = 3;             // stages of (Q_i, dO_i) or (K_j, V_j), 128 rows each
+  static constexpr int OPB = 128 * WB * 2;  // one bf16 [128 x 128] operand: two 64-column halves of 16 KB
+  // K, V | stages | P^T, dS^T | statistics (-lse2, D) per stage | barriers | alignment
+  static constexpr int SMEM_DKV = 2 * T128 + NST * 2 * T128 + 2 * OPB + NST * 2 * WB * 4 + 256 + 1024;
+  // Q, dO | stages | dS | D quarters | barriers | alignment
+  static constexpr int SMEM_DQ = 2 * T128 + NST * 2 * T128 + OPB + 4 * 128 * 4 + 256 + 1024;
+  static_assert(SMEM_DKV <= 232448 && SMEM_DQ <= 232448, "shared memory per CTA");
+};
+
+// 16 bf16 values (columns 16 s .. 16 s + 15 of a thread's 32, qq the 32-column quarter) into row r of a
+// swizzled [128 x 128] K-major operand (two 64-column halves of 16 KB).
+__device__ __forceinline__ void put_row16w(uint8_t* g, int qq, int sub, int r, const uint32_t* pk) {
+  uint8_t* row = g + (qq >> 1) * 16384 + r * 128;
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int chunk = ((qq & 1) * 4 + sub * 2 + u) ^ (r & 7);
+    *reinterpret_cast<uint4*>(row + (chunk << 4)) = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+  }
+}
+
+// dQ (and D) kernel, 128-key inner blocks. Maps: tq, tdo, tkv, all in 128-row boxes.
+template <int HD>
+__global__ void __launch_bounds__(NTHR_B, 1)
+    attn_bwd_dq_w_k(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tdo,
+                    const __grid_constant__ CUtensorMap tkv, const bf16* __restrict__ outp,
+                    const bf16* __restrict__ dout, const float* __restrict__ lse, float* __restrict__ Dv,
+                    bf16* __restrict__ dqkv, int S, int H, int Hkv, float scale, unsigned* err) {
+  using C_ = WCfg<HD>;
+  constexpr int NST = C_::NST;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sq = smem;
+  uint8_t* sdo = sq + C_::T128;
+  uint8_t* sst = sdo + C_::T128;                  // stage s: K_j at s * 2 T128, V_j after it
+  uint8_t* sds = sst + NST * 2 * C_::T128;        // dS
+  float* dpart = (float*)(sds + C_::OPB);         // [4][128] quarters of D
+  uint64_t* full = (uint64_t*)(dpart + 512);
+  uint64_t* empty = full + NST;
+  uint64_t* qfull = empty + NST;
+  uint64_t* sfull = qfull + 1;
+  uint64_t* sempty = sfull + 1;
+  uint64_t* dsfull = sempty + 1;
+  uint64_t* dsempty = dsfull + 1;
+  uint64_t* ofull = dsempty + 1;
+  uint64_t* fin = ofull + 1;
+  uint32_t* tbase = (uint32_t*)(fin + 1);
+  volatile int* abort_flag = (volatile int*)(tbase + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x, b = blockIdx.y, qb = gridDim.z - 1 - blockIdx.z;   // longest first
+  const int kvh = h / (H / Hkv);
+  const int q0 = qb * 128;
+  const int nkb = min(qb + 1, (S + WB - 1) / WB);
+  const int ld = (H + 2 * Hkv) * HD, HDall = H * HD;
+  const int xq = h * HD, xk = (H + kvh) * HD, xv = (H + Hkv + kvh) * HD;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    mbar_init(qfull, 1);
+    mbar_init(sfull, 1);
+    mbar_init(sempty, NEW);
+    mbar_init(dsfull, NEW);
+    mbar_init(dsempty, 1);
+    mbar_init(ofull, 1);
+    mbar_init(fin, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc512(tbase);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tbase;   // S: columns 0-127, dP: 128-255, dQ: 256 + HD
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    int issued[NST];
+#pragma unroll
+    for (int s = 0; s < NST; ++s) issued[s] = -1;
+    const bool leader = elect_one();
+    if (leader) {
+      mbar_expect_tx(qfull, 2 * C_::T128);
+#pragma unroll
+      for (int c = 0; c < HD / 64; ++c) {
+        tma3d(sq + c * 16384, &tq, qfull, xq + 64 * c, q0, b);
+        tma3d(sdo + c * 16384, &tdo, qfull, h * HD + 64 * c, q0, b);
+      }
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      if (!uwait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+      issued[stage] = (int)phase;
+      if (leader) {
+        mbar_expect_tx(&full[stage], 2 * C_::T128);
+        uint8_t* st = sst + stage * 2 * C_::T128;
+#pragma unroll
+        for (int c = 0; c < HD / 64; ++c) {
+          tma3d(st + c * 16384, &tkv, &full[stage], xk + 64 * c, j * WB, b);
+          tma3d(st + C_::T128 + c * 16384, &tkv, &full[stage], xv + 64 * c, j * WB, b);
+        }
+      }
+      __syncwarp();
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (!ok && lane == 0) drain<NST>(full, issued, qfull);
+  } else if (warp == 1) {
+    constexpr uint32_t id_s = idesc_f16(128, WB, false, false);
+    constexpr uint32_t id_q = idesc_f16(128, HD, false, true);
+    const uint32_t q_addr = su32(sq), do_addr = su32(sdo), ds_addr = su32(sds);
+    const bool leader = elect_one();   // issues every product and every commit that tracks them
+    bool ok = uwait(qfull, 0, abort_flag, err);
+    fence_after();
+    int stage = 0, pstage = 0;
+    uint32_t phase = 0;
+    auto dq = [&](int jb, int st) -> bool {   // dQ += dS_jb K_jb
+      if (!uwait(dsfull, (uint32_t)(jb & 1), abort_flag, err)) return false;
+      fence_after();
+      if (leader) {
+        const uint32_t k_addr = su32(sst + st * 2 * C_::T128);
+#pragma unroll
+        for (int ks = 0; ks < WB / 16; ++ks)
+          mma_bf16(tmem + 256, sdesc(ds_addr + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024),
+                   sdesc(k_addr + ks * 2048, 16384, 1024), id_q, (jb > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&empty[st]);
+        mma_commit(dsempty);
+      }
+      __syncwarp();
+      return true;
+    };
+    for (int j = 0; ok && j < nkb; ++j) {
+      if (!uwait(sempty, ((uint32_t)j & 1u) ^ 1u, abort_flag, err) || !uwait(&full[stage], phase, abort_flag, err)) {
+        ok = false;
+        break;
+      }
+      fence_after();
+      if (leader) {
+        const uint32_t k_addr = su32(sst + stage * 2 * C_::T128), v_addr = k_addr + C_::T128;
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          const int kq = ks / 4, kr = ks % 4;
+          mma_bf16(tmem, sdesc(q_addr + kq * 16384 + kr * 32, 16, 1024), sdesc(k_addr + kq * 16384 + kr * 32, 16, 1024),
+                   id_s, ks > 0 ? 1u : 0u);
+          mma_bf16(tmem + 128, sdesc(do_addr + kq * 16384 + kr * 32, 16, 1024),
+                   sdesc(v_addr + kq * 16384 + kr * 32, 16, 1024), id_s, ks > 0 ? 1u : 0u);
+        }
+        mma_commit(sfull);
+      }
+      __syncwarp();
+      if (j > 0 && !dq(j - 1, pstage)) { ok = false; break; }
+      pstage = stage;
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (ok && !dq(nkb - 1, pstage)) ok = false;
+    if (leader) {
+      if (ok) mma_commit(ofull);
+      mma_commit(fin);
+    }
+    __syncwarp();
+  } else {
+    const int quad = warp & 3, qq = (warp - 2) / 4;   // TMEM lane quadrant, 32-column quarter
+    const int r = quad * 32 + lane;
+    const int q = q0 + r, qc = min(q, S - 1);
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    const size_t si = ((size_t)b * H + h) * S + qc;
+    const float nlse2 = q < S ? -lse[si] * kL2e : -INFINITY;
+    {   // D = rowsum(dO * O): each quarter sums a quarter of the row, fixed-order combination
+      const bf16* orow = outp + ((size_t)b * S + qc) * HDall + (size_t)h * HD + qq * (HD / 4);
+      const bf16* grow = dout + ((size_t)b * S + qc) * HDall + (size_t)h * HD + qq * (HD / 4);
+      float acc = 0.f;
+#pragma unroll
+      for (int c = 0; c < HD / 4; c += 8) {
+        float o8[8], g8[8];
+        Vec8<bf16>::load(orow + c, o8);
+        Vec8<bf16>::load(grow + c, g8);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc = fmaf(o8[e], g8[e], acc);
+      }
+      dpart[qq * 128 + r] = acc;
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * NEW) : "memory");
+    const float Dq = (dpart[r] + dpart[128 + r]) + (dpart[256 + r] + dpart[384 + r]);
+    if (q < S && qq == 0) Dv[si] = Dq;
+    const uint64_t SL2 = f2(scale * kL2e, scale * kL2e), NL = f2(nlse2, nlse2), DD = f2(Dq, Dq);
+    const int qmin = q0 + quad * 32;   // smallest query row of this warp
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      if (!uwait(sfull, (uint32_t)j & 1u, abort_flag, err)) { ok = false; break; }
+      fence_after();
+      for (int sub = 0; sub < 2; ++sub) {
+        const int c0 = qq * 32 + sub * 16;
+        float sv[16], dp[16];
+        tmem_ld16(trow + (uint32_t)c0, sv);
+        tmem_ld16(trow + 128u + (uint32_t)c0, dp);
+        if (sub == 1) {
+          fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sempty);
+        }
+        const int kbase = j * WB + c0;
+        const bool diag = kbase + 15 > qmin;   // warp-uniform: some column may lie above the diagonal
+        const int kmax = q - kbase;            // causal: columns e <= kmax
+        uint32_t pk[8];
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          float2 x = uf2(fma2(f2(sv[e], sv[e + 1]), SL2, NL));
+          if (diag) {
+            if (e > kmax) x.x = -INFINITY;
+            if (e + 1 > kmax) x.y = -INFINITY;
+          }
+          const float p0 = ex2(x.x), p1 = ex2(x.y);
+          const float2 ds = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), DD)));
+          pk[e / 2] = pack2(ds.x, ds.y);
+        }
+        if (sub == 0 && !uwait(dsempty, ((uint32_t)j & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+        put_row16w(sds, qq, sub, r, pk);
+      }
+      if (!ok) break;
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(dsfull);
+    }
+    if (ok && uwait(ofull, 0, abort_flag, err)) {
+      fence_after();
+      bf16* drow = dqkv + ((size_t)b * S + qc) * ld + (size_t)h * HD;
+#pragma unroll
+      for (int c = qq * (HD / 4); c < (qq + 1) * (HD / 4); c += 16) {
+        float v[16];
+        tmem_ld16(trow + 256 + (uint32_t)c, v);
+        if (q < S) {
+#pragma unroll
+          for (int e = 0; e < 16; ++e) v[e] *= scale;
+          Vec8<bf16>::store(drow + c, v);
+          Vec8<bf16>::store(drow + c + 8, v + 8);
+        }
+      }
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_release(fin, tmem);
+}
+
+// dK / dV kernel, 128-query inner blocks; grouped heads and outputs as attn_bwd_dkv_tg_k. Maps: tkv, tq,
+// tdo, all in 128-row boxes.
+template <int HD>
+__global__ void __launch_bounds__(NTHR_B, 1)
+    attn_bwd_dkv_w_k(const __grid_constant__ CUtensorMap tkv, const __grid_constant__ CUtensorMap tq,
+                     const __grid_constant__ CUtensorMap tdo, const float* __restrict__ lse,
+                     const float* __restrict__ Dv, bf16* __restrict__ dqkv, int S, int H, int Hkv, float scale,
+                     float* __restrict__ part, unsigned* err) {
+  using C_ = WCfg<HD>;
+  constexpr int NST = C_::NST;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sk = smem;
+  uint8_t* sv = sk + C_::T128;
+  uint8_t* sst = sv + C_::T128;                   // stage s: Q_i at s * 2 T128, dO_i after it
+  uint8_t* sp = sst + NST * 2 * C_::T128;         // P^T
+  uint8_t* sds = sp + C_::OPB;                    // dS^T
+  float* stats = (float*)(sds + C_::OPB);         // stage s: -lse2[128], D[128]
+  uint64_t* full = (uint64_t*)(stats + NST * 2 * WB);
+  uint64_t* empty = full + NST;
+  uint64_t* kvfull = empty + NST;
+  uint64_t* sfull = kvfull + 1;
+  uint64_t* sempty = sfull + 1;
+  uint64_t* pfull = sempty + 1;
+  uint64_t* pempty = pfull + 1;
+  uint64_t* ofull = pempty + 1;
+  uint64_t* fin = ofull + 1;
+  uint32_t* tbase = (uint32_t*)(fin + 1);
+  volatile int* abort_flag = (volatile int*)(tbase + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x, b = blockIdx.y, kb = blockIdx.z;   // key block 0 (the longest) first
+  const int kvh = part ? h / (H / Hkv) : h;
+  const int k0 = kb * 128;
+  const int nit = (S + WB - 1) / WB - kb;         // query blocks kb .. : the causal ones
+  const int ld = (H + 2 * Hkv) * HD;
+  const int xq = h * HD, xk = (H + kvh) * HD, xv = (H + Hkv + kvh) * HD;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NST; ++s) { mbar_init(&full[s], 2); mbar_init(&empty[s], 1); }
+    mbar_init(kvfull, 1);
+    mbar_init(sfull, 1);
+    mbar_init(sempty, NEW);
+    mbar_init(pfull, NEW);
+    mbar_init(pempty, 1);
+    mbar_init(ofull, 1);
+    mbar_init(fin, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc512(tbase);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tbase;   // S^T 0-127, dP^T 128-255, dV 256 + HD, dK 256 + HD .. 256 + 2 HD
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    // one elected lane: TMA of K, V once and of (Q_i, dO_i) per block; every lane: four of the block's
+    // -lse2 and D, loaded one block ahead
+    int issued[NST];
+#pragma unroll
+    for (int s = 0; s < NST; ++s) issued[s] = -1;
+    const bool leader = elect_one();
+    if (leader) {
+      mbar_expect_tx(kvfull, 2 * C_::T128);
+#pragma unroll
+      for (int c = 0; c < HD / 64; ++c) {
+        tma3d(sk + c * 16384, &tkv, kvfull, xk + 64 * c, k0, b);
+        tma3d(sv + c * 16384, &tkv, kvfull, xv + 64 * c, k0, b);
+      }
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    float nl[4], dd[4];
+    auto fetch = [&](int it) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int qq2 = (kb + it) * WB + lane * 4 + u;
+        const size_t si = ((size_t)b * H + h) * S + (qq2 < S ? qq2 : 0);
+        nl[u] = qq2 < S ? -lse[si] * kL2e : -INFINITY;
+        dd[u] = qq2 < S ? Dv[si] : 0.f;
+      }
+    };
+    fetch(0);
+    for (int it = 0; it < nit; ++it) {
+      const int qi0 = (kb + it) * WB;
+      if (!uwait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+      issued[stage] = (int)phase;
+      if (leader) {
+        mbar_expect_tx(&full[stage], 2 * C_::T128);
+        uint8_t* st = sst + stage * 2 * C_::T128;
+#pragma unroll
+        for (int c = 0; c < HD / 64; ++c) {
+          tma3d(st + c * 16384, &tq, &full[stage], xq + 64 * c, qi0, b);
+          tma3d(st + C_::T128 + c * 16384, &tdo, &full[stage], h * HD + 64 * c, qi0, b);
+        }
+      }
+      float* sl = stats + stage * 2 * WB;
+      *reinterpret_cast<float4*>(sl + lane * 4) = make_float4(nl[0], nl[1], nl[2], nl[3]);
+      *reinterpret_cast<float4*>(sl + WB + lane * 4) = make_float4(dd[0], dd[1], dd[2], dd[3]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&full[stage]);
+      if (it + 1 < nit) fetch(it + 1);
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (!ok && lane == 0) drain<NST>(full, issued, kvfull);
+  } else if (warp == 1) {
+    constexpr uint32_t id_s = idesc_f16(128, WB, false, false);
+    constexpr uint32_t id_g = idesc_f16(128, HD, false, true);
+    const uint32_t k_addr = su32(sk), v_addr = su32(sv), p_addr = su32(sp), ds_addr = su32(sds);
+    const bool leader = elect_one();   // issues every product and every commit that tracks them
+    bool ok = uwait(kvfull, 0, abort_flag, err);
+    fence_after();
+    int stage = 0, pstage = 0;
+    uint32_t phase = 0;
+    auto grads = [&](int ib, int st) -> bool {   // dV += P^T dO_ib, dK += dS^T Q_ib
+      if (!uwait(pfull, (uint32_t)(ib & 1), abort_flag, err)) return false;
+      fence_after();
+      if (leader) {
+        const uint32_t qa = su32(sst + st * 2 * C_::T128), da = qa + C_::T128;
+#pragma unroll
+        for (int ks = 0; ks < WB / 16; ++ks) {
+          const uint32_t acc = (ib > 0 || ks > 0) ? 1u : 0u;
+          const uint32_t ao = (ks / 4) * 16384 + (ks % 4) * 32;
+          mma_bf16(tmem + 256, sdesc(p_addr + ao, 16, 1024), sdesc(da + ks * 2048, 16384, 1024), id_g, acc);
+          mma_bf16(tmem + 256 + HD, sdesc(ds_addr + ao, 16, 1024), sdesc(qa + ks * 2048, 16384, 1024), id_g, acc);
+        }
+        mma_commit(&empty[st]);
+        mma_commit(pempty);
+      }
+      __syncwarp();
+      return true;
+    };
+    for (int it = 0; ok && it < nit; ++it) {
+      if (!uwait(sempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, err) || !uwait(&full[stage], phase, abort_flag, err)) {
+        ok = false;
+        break;
+      }
+      fence_after();
+      if (leader) {
+        const uint32_t qa = su32(sst + stage * 2 * C_::T128), da = qa + C_::T128;
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          const int kq = ks / 4, kr = ks % 4;
+          mma_bf16(tmem, sdesc(k_addr + kq * 16384 + kr * 32, 16, 1024), sdesc(qa + kq * 16384 + kr * 32, 16, 1024),
+                   id_s, ks > 0 ? 1u : 0u);
+          mma_bf16(tmem + 128, sdesc(v_addr + kq * 16384 + kr * 32, 16, 1024),
+                   sdesc(da + kq * 16384 + kr * 32, 16, 1024), id_s, ks > 0 ? 1u : 0u);
+        }
+        mma_commit(sfull);
+      }
+      __syncwarp();
+      if (it > 0 && !grads(it - 1, pstage)) { ok = false; break; }
+      pstage = stage;
+      if (++stage == NST) { stage = 0; phase ^= 1u; }
+    }
+    if (ok && !grads(nit - 1, pstage)) ok = false;
+    if (leader) {
+      if (ok) mma_commit(ofull);
+      mma_commit(fin);
+    }
+    __syncwarp();
+  } else {
+    const int quad = warp & 3, qq = (warp - 2) / 4;   // TMEM lane quadrant, 32-column quarter
+    const int r = quad * 32 + lane;                    // key row = TMEM lane
+    const int key = k0 + r;
+    const int kmaxw = k0 + quad * 32 + 31;             // largest key of this warp
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    const uint64_t SL2 = f2(scale * kL2e, scale * kL2e);
+    // Only the causal mask is applied: queries >= S have -lse2 = -inf (P = 0) and D = 0, and rows of
+    // keys >= S are never stored.
+    bool ok = true;
+    for (int it = 0; it < nit; ++it) {
+      const int stage = it % NST;
+      const uint32_t phase = (uint32_t)(it / NST) & 1u;
+      if (!uwait(sfull, (uint32_t)it & 1u, abort_flag, err)) { ok = false; break; }
+      fence_after();
+      // this stage's statistics: its full phase has completed (the S MMA waited on it); the wait orders
+      // the producer's stores before these loads
+      if (!uwait(&full[stage], phase, abort_flag, err)) { ok = false; break; }
+      for (int sub = 0; sub < 2; ++sub) {
+        const int c0 = qq * 32 + sub * 16;
+        float svv[16], dp[16];
+        tmem_ld16(trow + (uint32_t)c0, svv);
+        tmem_ld16(trow + 128u + (uint32_t)c0, dp);
+        if (sub == 1) {
+          fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sempty);
+        }
+        const float4* sl4 = reinterpret_cast<const float4*>(stats + stage * 2 * WB + c0);
+        const float4* sd4 = reinterpret_cast<const float4*>(stats + stage * 2 * WB + WB + c0);
+        const int qbase = (kb + it) * WB + c0;   // query of column 0 of these 16
+        const bool diag = qbase < kmaxw;          // warp-uniform: some column may precede its key
+        const int qlo = key - qbase;              // causal: columns e >= qlo
+        uint32_t pk[8], dk[8];
+#pragma unroll
+        for (int e4 = 0; e4 < 4; ++e4) {
+          const float4 l = sl4[e4], d = sd4[e4];
+          const int e = 4 * e4;
+          float2 xa = uf2(fma2(f2(svv[e], svv[e + 1]), SL2, f2(l.x, l.y)));
+          float2 xb = uf2(fma2(f2(svv[e + 2], svv[e + 3]), SL2, f2(l.z, l.w)));
+          if (diag) {
+            if (e < qlo) xa.x = -INFINITY;
+            if (e + 1 < qlo) xa.y = -INFINITY;
+            if (e + 2 < qlo) xb.x = -INFINITY;
+            if (e + 3 < qlo) xb.y = -INFINITY;
+          }
+          const float p0 = ex2(xa.x), p1 = ex2(xa.y), p2 = ex2(xb.x), p3 = ex2(xb.y);
+          const float2 da = uf2(mul2(f2(p0, p1), sub2(f2(dp[e], dp[e + 1]), f2(d.x, d.y))));
+          const float2 db = uf2(mul2(f2(p2, p3), sub2(f2(dp[e + 2], dp[e + 3]), f2(d.z, d.w))));
+          pk[2 * e4] = pack2(p0, p1);
+          pk[2 * e4 + 1] = pack2(p2, p3);
+          dk[2 * e4] = pack2(da.x, da.y);
+          dk[2 * e4 + 1] = pack2(db.x, db.y);
+        }
+        if (sub == 0 && !uwait(pempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+        put_row16w(sp, qq, sub, r, pk);
+        put_row16w(sds, qq, sub, r, dk);
+      }
+      if (!ok) break;
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(pfull);
+    }
+    if (ok && uwait(ofull, 0, abort_flag, err)) {
+      fence_after();
+      const int kc = min(key, S - 1);
+      const size_t NS = (size_t)gridDim.y * S;
+#pragma unroll
+      for (int c = qq * (HD / 4); c < (qq + 1) * (HD / 4); c += 16) {
+        float gv[16], gk[16];
+        tmem_ld16(trow + 256 + (uint32_t)c, gv);
+        tmem_ld16(trow + 256 + HD + (uint32_t)c, gk);
+        if (key < S) {
+          if (part) {
+            float* pk2 = part + ((size_t)h * NS + (size_t)b * S + kc) * HD + c;
+            float* pv2 = pk2 + (size_t)H * NS * HD;
+#pragma unroll
+            for (int e = 0; e < 16; e += 4) {
+              *reinterpret_cast<float4*>(pk2 + e) = make_float4(gk[e], gk[e + 1], gk[e + 2], gk[e + 3]);
+              *reinterpret_cast<float4*>(pv2 + e) = make_float4(gv[e], gv[e + 1], gv[e + 2], gv[e + 3]);
+            }
+          } else {
+            bf16* dkr = dqkv + ((size_t)b * S + kc) * ld + (size_t)xk + c;
+            bf16* dvr = dqkv + ((size_t)b * S + kc) * ld + (size_t)xv + c;
+#pragma unroll
+            for (int e = 0; e < 16; ++e) gk[e] *= scale;
+            Vec8<bf16>::store(dkr, gk);
+            Vec8<bf16>::store(dkr + 8, gk + 8);
+            Vec8<bf16>::store(dvr, gv);
+            Vec8<bf16>::store(dvr + 8, gv + 8);
+          }
+        }
+      }
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_release(fin, tmem);
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
 
 bool enc_init() {
@@ -987,6 +1511,43 @@ bool bwd_launch(const void* qkv, const void* out, const void* dout, const float*
   return e == cudaSuccess;
 }
 
+// The 128-wide backward (head dim 64).
+template <int HD>
+bool bwd_w_launch(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B,
+                  int S, int H, int Hkv, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
+  using C_ = WCfg<HD>;
+  static bool attr = false;
+  auto kq = attn_bwd_dq_w_k<HD>;
+  auto kkv = attn_bwd_dkv_w_k<HD>;
+  if (!attr) {
+    if (cudaFuncSetAttribute(kq, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM_DQ) != cudaSuccess ||
+        cudaFuncSetAttribute(kkv, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM_DKV) != cudaSuccess)
+      return false;
+    attr = true;
+  }
+  const int W = (H + 2 * Hkv) * HD, Wo = H * HD;
+  CUtensorMap q128, do128;
+  if (!qkv_map(&q128, qkv, B, S, W, 128) || !qkv_map(&do128, dout, B, S, Wo, 128)) return false;
+  float* part = nullptr;
+  if (H > Hkv) {   // grouped heads: one CTA per query head, then a fixed-order group reduction
+    const size_t bytes = 2ull * H * B * S * HD * sizeof(float);
+    cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&part, bytes, pool, s) : cudaMallocAsync((void**)&part, bytes, s);
+    if (e != cudaSuccess) { cudaGetLastError(); return false; }
+  }
+  const float scale = 1.f / sqrtf((float)HD);
+  const int nqb = (S + 127) / 128;
+  cudaError_t e = launch_pdl(kq, dim3(H, B, nqb), NTHR_B, C_::SMEM_DQ, s, q128, do128, q128, (const bf16*)out,
+                             (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, scale, err);
+  if (e == cudaSuccess)
+    e = launch_pdl(kkv, dim3(part ? H : Hkv, B, nqb), NTHR_B, C_::SMEM_DKV, s, q128, q128, do128, (const float*)lse,
+                   (const float*)D, (bf16*)dqkv, S, H, Hkv, scale, part, err);
+  if (part) {
+    if (e == cudaSuccess) launch_reduce_dkv(part, dqkv, B * S, H, Hkv, HD, scale, s);
+    cudaFreeAsync(part, s);
+  }
+  return e == cudaSuccess;
+}
+
 template <int HD>
 bool fwd1_launch(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, cudaStream_t s, unsigned* err) {
   using C_ = F1Cfg<HD>;
@@ -1027,7 +1588,7 @@ bool attn_bwd_tcgen05(const void* qkv, const void* out, const void* dout, const 
       (S + 127) / 128 > 65535)
     return false;
   if (!tg::enc_init()) return false;
-  return hd == 64 ? tg::bwd_launch<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err)
+  return hd == 64 ? tg::bwd_w_launch<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err)
                   : tg::bwd_launch<128>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err);
 }
 
