@@ -41,7 +41,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="gpt2", choices=list(WORKLOADS))
@@ -113,8 +113,8 @@ GEMM_SOURCES = ["gemm_tc.cu", "tcgen05.cuh"]
 TRAFFIC = {
     # ncu dram__bytes_read.sum + dram__bytes_write.sum of the GPT-2 GEMM shapes (microbench gemm),
     # averaged with the per-step launch mix: 12 layer GEMMs per layer; 5 head forwards, 4 head dX
-    "gemm_layer": {"sources": GEMM_SOURCES, "sha256": "207d8a97ba2abf74", "bytes_per_launch": 22319594.7},
-    "gemm_head": {"sources": GEMM_SOURCES, "sha256": "207d8a97ba2abf74", "bytes_per_launch": 643176106.7},
+    "gemm_layer": {"sources": GEMM_SOURCES, "sha256": "77747b85c3adf6ff", "bytes_per_launch": 22319274.7},
+    "gemm_head": {"sources": GEMM_SOURCES, "sha256": "77747b85c3adf6ff", "bytes_per_launch": 643159296.0},
 }
 
 
