@@ -300,13 +300,17 @@ def run_ours(args):
         if world > 1:
             dist.barrier()
 
-    def timed(fn, steps):
+    def timed(fn, steps, finish=None):
+        """Device time of `steps` calls of fn: the steps are queued back to back (no host sync between
+        them), then `finish` joins every stream of the engine into the timing stream."""
         barrier()
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record(stream)
         for i in range(steps):
             fn(i)
+        if finish is not None:
+            finish()
         t1.record(stream)
         barrier()
         return max_over_ranks(t0.elapsed_time(t1), world)
@@ -314,24 +318,22 @@ def run_ours(args):
     # ---- ZeroLock: device-resident inputs -----------------------------------------------------
     eng = make_engine(args.max_live)
 
+    # Steps are queued as a training loop queues them: chunk k of step i+1 waits only for its own update
+    # of step i and for chunk k-1's output of step i+1, so it may start while later chunks of step i
+    # still run (no update locking across steps either). One join at the end covers all of them.
     def zl(i):
         ids, lab = dev_batches[i % nb]
         zb.zl_step(eng.ctx, ids, lab, w.batch, w.seq, K, want_losses=False)
-        if i % 8 == 7:
-            zb.zl_join(eng.ctx)
-
-    def zl_joined(i):
-        zl(i)
-        zb.zl_join(eng.ctx)
 
     for i in range(args.warmup):
         zl(i)
+    zb.zl_join(eng.ctx)
     eng.synchronize()
     eng.reset_peak()
     clocks = ClockSampler(local)
     clocks.start()
     n0 = zb.zl_kernel_launches()
-    ms = timed(zl_joined, args.steps)
+    ms = timed(zl, args.steps, finish=lambda: zb.zl_join(eng.ctx))
     launches = zb.zl_kernel_launches() - n0
     clk = clocks.stop()
     zl_peak = eng.peak_bytes()[0]
@@ -380,15 +382,14 @@ def run_ours(args):
     if not args.no_bp:
         beng = make_engine(args.max_live)
 
-        def bps(i):
+        def bps(i):   # each backprop step waits for the previous one's update on the engine's streams
             ids, lab = dev_batches[i % nb]
             zb.zl_bp_step(beng.ctx, ids, lab, w.batch, w.seq, want_loss=False)
-            zb.zl_join(beng.ctx)
         for i in range(args.warmup):
             bps(i)
         beng.synchronize()
         beng.reset_peak()
-        bms = timed(bps, args.steps)
+        bms = timed(bps, args.steps, finish=lambda: zb.zl_join(beng.ctx))
         bp = {"value": job_tokens_per_s(tokens, args.steps, world, bms), "unit": "tokens/s",
               "peak_hbm_gb": beng.peak_bytes()[0] / 1e9, "ms_per_step": bms / args.steps}
         beng.close()
