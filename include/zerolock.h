@@ -114,6 +114,12 @@ zl_status zl_set_stream(zl_ctx* ctx, void* stream);
  * on_device, else host) into the master copy (and the compute copy). */
 zl_status zl_set_param(zl_ctx* ctx, const char* name, const void* src, size_t bytes, int on_device);
 
+/* zl_load_weights: the same operation as zl_set_param under the name the problem statement's
+ * interface uses (weights loaded once before training). Same arguments, ownership (src is only
+ * read during the call) and errors (ZL_ERR_ARG for an unknown name or a byte count other than
+ * numel * 4). */
+zl_status zl_load_weights(zl_ctx* ctx, const char* name, const void* src, size_t bytes, int on_device);
+
 /* Copy one tensor out as fp32 (waits for queued work). which: 0 value (master copy),
  * 1 accumulated gradient, 2 AdamW first moment, 3 AdamW second moment (1-3: trainable only). */
 zl_status zl_get_param(zl_ctx* ctx, const char* name, int which, void* dst, size_t bytes, int on_device);

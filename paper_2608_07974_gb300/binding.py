@@ -18,7 +18,7 @@ ZL_ARCH_LLAMA, ZL_ARCH_GPT2 = 0, 1
 ZL_DTYPE_F32, ZL_DTYPE_BF16 = 0, 1
 
 #: every symbol include/zerolock.h declares
-EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_get_param", "zl_param_numel",
+EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_load_weights", "zl_get_param", "zl_param_numel",
            "zl_embed", "zl_forward_chunk", "zl_local_step", "zl_step", "zl_bp_step", "zl_eval_global_loss",
            "zl_read_losses", "zl_join", "zl_synchronize", "zl_peak_bytes", "zl_reset_peak", "zl_last_error",
            "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_gemm_ex", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
@@ -57,6 +57,7 @@ def _load() -> C.CDLL:
         "zl_free": [vp],
         "zl_set_stream": [vp, vp],
         "zl_set_param": [vp, C.c_char_p, vp, sz, i],
+        "zl_load_weights": [vp, C.c_char_p, vp, sz, i],
         "zl_get_param": [vp, C.c_char_p, i, vp, sz, i],
         "zl_param_numel": [vp, C.c_char_p, C.POINTER(sz)],
         "zl_embed": [vp, vp, i, i, vp],
@@ -133,6 +134,12 @@ def zl_set_param(ctx, name: str, t) -> None:
     """t: fp32 torch tensor (host or CUDA), contiguous."""
     t = t.contiguous()
     _check(_lib.zl_set_param(ctx, name.encode(), t.data_ptr(), t.numel() * 4, int(t.is_cuda)))
+
+
+def zl_load_weights(ctx, name: str, t) -> None:
+    """Same as zl_set_param (the problem statement's name for loading a weight). t: fp32 tensor."""
+    t = t.contiguous()
+    _check(_lib.zl_load_weights(ctx, name.encode(), t.data_ptr(), t.numel() * 4, int(t.is_cuda)))
 
 
 def zl_param_numel(ctx, name: str) -> int:

@@ -1191,6 +1191,10 @@ zl_status zl_set_param(zl_ctx* c, const char* name, const void* src, size_t byte
   });
 }
 
+zl_status zl_load_weights(zl_ctx* c, const char* name, const void* src, size_t bytes, int on_device) {
+  return zl_set_param(c, name, src, bytes, on_device);
+}
+
 zl_status zl_get_param(zl_ctx* c, const char* name, int which, void* dst, size_t bytes, int on_device) {
   if (!c || !name || !dst) { g_err = "NULL argument"; return ZL_ERR_ARG; }
   return guarded(c, [&]() -> zl_status {

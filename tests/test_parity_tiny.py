@@ -167,3 +167,23 @@ def test_out_of_range_ids_and_labels_are_reported():
     with pytest.raises(b.ZLError) as e:
         eng.step(ids[:, :0].contiguous().cuda(), labels[:, :0].contiguous().cuda())
     assert e.value.status == b.ZL_ERR_ARG
+
+
+def test_load_weights_is_set_param():
+    """zl_load_weights stores a tensor exactly as zl_set_param does, from host or device memory, and
+    rejects an unknown name or a wrong byte count."""
+    from paper_2608_07974_gb300 import binding as b
+    eng = engine_for(W)
+    eng.load(_params())
+    g = torch.Generator().manual_seed(7)
+    for name, dev in (("layers.0.wqkv", False), ("layers.3.w2", True), ("layers.1.ffn_norm.weight", True)):
+        t = torch.randn(eng.get(name).shape, generator=g)
+        b.zl_load_weights(eng.ctx, name, t.cuda() if dev else t)
+        assert torch.equal(eng.get(name).cpu(), t), name
+    with pytest.raises(b.ZLError) as e:
+        b.zl_load_weights(eng.ctx, "layers.0.no_such", torch.zeros(4))
+    assert e.value.status == b.ZL_ERR_ARG
+    with pytest.raises(b.ZLError) as e:
+        b.zl_load_weights(eng.ctx, "layers.0.wqkv", torch.zeros(4))
+    assert e.value.status == b.ZL_ERR_ARG
+    eng.close()
