@@ -114,3 +114,34 @@ def test_pins_catch_adapter_on_the_teacher(monkeypatch):
     _patch(monkeypatch, "readout", readout_through_adapter)
     with pytest.raises(AssertionError):
         pins.test_adapter_teacher_is_the_frozen_head_and_bp_ignores_adapters()
+
+
+def test_pins_catch_schedule_off_by_one(monkeypatch):
+    def apply_window(self, k, adapters=True):   # eta_0 / sqrt(t + 1 + gamma): the schedule one step late
+        c = self.cfg
+        self.t[k] += 1
+        lr = c.lr if c.lr_schedule == 0 else c.lr / math.sqrt(self.t[k] + c.lr_gamma)
+        for n in self.chunk_names(k):
+            g = self.acc[n] / c.accum_m
+            om.adamw_update(self.P[n], g, self.m[n], self.v[n], self.t[k], lr, c.beta1, c.beta2, c.eps,
+                            c.weight_decay)
+            self.acc[n].zero_()
+        self.micro[k] = 0
+    monkeypatch.setattr(om.Oracle, "_apply_window", apply_window)
+    with pytest.raises(AssertionError):
+        pins.test_lr_schedule_matches_torch_lambda_lr()
+
+
+def test_pins_catch_ignored_consis_first(monkeypatch):
+    monkeypatch.setattr(om.Oracle, "alpha_k", lambda self, k: self.cfg.alpha)
+    with pytest.raises(AssertionError):
+        pins.test_consis_first_zero_is_plain_cross_entropy()
+
+
+def test_pins_catch_swapped_kl_direction(monkeypatch):
+    orig = om.kl_rows
+    _patch(monkeypatch, "kl_rows", lambda z, t, kl_dir=0: orig(z, t, 1 - kl_dir))
+    with pytest.raises(AssertionError):
+        pins.test_reverse_kl_direction_matches_library()
+    with pytest.raises(AssertionError):
+        pins.test_loss_closed_forms()

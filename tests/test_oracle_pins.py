@@ -569,3 +569,82 @@ def test_adapter_teacher_is_the_frozen_head_and_bp_ignores_adapters():
         assert torch.equal(bp.P[n], t), n
     for n, t in base.P.items():
         assert torch.equal(bp.P[n], t), n
+
+
+# ---------------------------------------------------------------------------------------
+# Options of the update rule: the step-size schedule of Theorem 1, chunk 1 without a
+# consistency term, and the reverse distillation direction
+# ---------------------------------------------------------------------------------------
+
+def test_lr_schedule_matches_torch_lambda_lr():
+    """lr_schedule = 1 is eta_t = eta_0 / sqrt(t + gamma), t = 0, 1, .. counting each chunk's own
+    updates (Theorem 1's step size): the oracle's parameters follow torch.optim.AdamW driven by a
+    LambdaLR with that factor, fed the oracle's own gradients (so only the update rule is pinned)."""
+    d = LLAMA_T
+    P = tiny_params(d)
+    lr, gamma = 3e-2, 2.0
+    cfg = OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5, lr=lr, lr_schedule=1, lr_gamma=gamma)
+    orc = Oracle(cfg, P)
+    names = orc.chunk_names(1)
+    ps = [torch.nn.Parameter(orc.P[n].clone()) for n in names]
+    opt = torch.optim.AdamW(ps, lr=lr, betas=(0.9, 0.999), eps=1e-8, weight_decay=0.01)
+    sched = torch.optim.lr_scheduler.LambdaLR(opt, lambda t: 1.0 / math.sqrt(t + gamma))
+    for s in range(4):
+        ids, labels = tiny_batch(d, seed=40 + s)
+        _, grads, _ = orc.local_grad(1, orc.embed(ids), labels)
+        for p, n in zip(ps, names):
+            p.grad = grads[n].clone()
+        opt.step()
+        sched.step()
+        orc.step(ids, labels)
+        assert orc.t[1] == s + 1
+        for p, n in zip(ps, names):
+            assert torch.allclose(orc.P[n], p.detach(), atol=1e-14, rtol=1e-12), (s, n)
+    # the schedule really changed the step: a constant-lr run ends elsewhere
+    const = Oracle(OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5, lr=lr), P)
+    for s in range(4):
+        const.step(*tiny_batch(d, seed=40 + s))
+    assert not torch.allclose(const.P[names[1]], orc.P[names[1]], atol=1e-6, rtol=0)
+
+
+def test_consis_first_zero_is_plain_cross_entropy():
+    """consis_first = 0 gives chunk 1 the task term alone (alpha_1 = 1): its local loss is the
+    library cross-entropy of its readout over Omega; chunk 2 keeps the consistency term."""
+    d = GPT2_T
+    P = tiny_params(d)
+    ids, labels = tiny_batch(d)
+    labels[1, 2] = -1
+    cfg = OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5, consis_first=0)
+    orc = Oracle(cfg, P)
+    h0 = orc.embed(ids)
+    L1, _, h1 = orc.local_grad(1, h0, labels)
+    z1 = oracle.readout(orc.P, h1, d).reshape(-1, d.vocab)
+    ce = F.cross_entropy(z1, labels.reshape(-1).long(), ignore_index=-1)
+    assert abs(L1 - float(ce)) < 1e-13
+    L2, _, h2 = orc.local_grad(2, h1, labels)
+    z2 = oracle.readout(orc.P, h2, d).reshape(-1, d.vocab)
+    ce2 = F.cross_entropy(z2, labels.reshape(-1).long(), ignore_index=-1)
+    assert abs(L2 - float(ce2)) > 1e-6          # 0.5 CE + 0.5 KL(p_2 || p_1), not CE
+    with_first = Oracle(OracleConfig(dims=d, bounds=[0, 1, 2], alpha=0.5), P)
+    L1b, _, _ = with_first.local_grad(1, h0, labels)
+    assert abs(L1b - float(ce)) > 1e-6
+
+
+def test_reverse_kl_direction_matches_library():
+    """kl_dir = 1 is KL(p_{k-1} || p_k) (forward distillation): the library kl_div with the student
+    as input and the teacher as target; its logit gradient is (p - q) / |Omega| per row at alpha 0."""
+    g = torch.Generator().manual_seed(12)
+    V = 23
+    lab = torch.tensor([4, -1, 0, 22, 9])
+    z = torch.randn(5, V, generator=g).requires_grad_(True)
+    t = torch.randn(5, V, generator=g)
+    kl = F.kl_div(F.log_softmax(z, -1), F.log_softmax(t, -1), log_target=True, reduction="none").sum(-1)
+    ref = kl[lab >= 0].sum() / 4
+    ce = F.cross_entropy(z, lab.long(), ignore_index=-1)
+    for a in (0.5, 0.0):
+        val = oracle.local_objective(z, t, lab, a, 1).detach()
+        assert abs(float(val) - float(a * ce + (1 - a) * ref)) < 1e-13
+    (dz,) = torch.autograd.grad(oracle.local_objective(z, t, lab, 0.0, 1), z)
+    pq = (torch.softmax(z.detach(), -1) - torch.softmax(t, -1)) / 4
+    pq[1] = 0
+    assert torch.allclose(dz, pq, atol=1e-16, rtol=0)
