@@ -145,3 +145,30 @@ def test_pins_catch_swapped_kl_direction(monkeypatch):
         pins.test_reverse_kl_direction_matches_library()
     with pytest.raises(AssertionError):
         pins.test_loss_closed_forms()
+
+
+def test_independent_backward_catches_swapped_swiglu_halves(monkeypatch):
+    import tests.test_oracle_independent_bp as ib
+
+    def swapped(P, l, x, d, lora_scale=1.0):   # silu applied to the up half instead of the gate half
+        Q = dict(P)
+        w1 = P[f"layers.{l}.w1"]
+        Q[f"layers.{l}.w1"] = torch.cat([w1[d.d_ff:], w1[:d.d_ff]])
+        return orig(Q, l, x, d, lora_scale)
+    orig = om.layer_forward
+    _patch(monkeypatch, "layer_forward", lambda P, l, x, d, lora_scale=1.0:
+           swapped(P, l, x, d, lora_scale) if d.arch == 0 else orig(P, l, x, d, lora_scale))
+    with pytest.raises(AssertionError):
+        ib.test_backprop_gradient_matches_manual_backward(pins.LLAMA_T, [0, 2])
+
+
+def test_independent_backward_catches_unbiased_layernorm_variance(monkeypatch):
+    import tests.test_oracle_independent_bp as ib
+
+    def ln_unbiased(x, g, b, eps):
+        mu = x.mean(-1, keepdim=True)
+        var = ((x - mu) ** 2).sum(-1, keepdim=True) / (x.shape[-1] - 1)
+        return (x - mu) / torch.sqrt(var + eps) * g + b
+    _patch(monkeypatch, "layernorm", ln_unbiased)
+    with pytest.raises(AssertionError):
+        ib.test_backprop_gradient_matches_manual_backward(pins.GPT2_T, [0, 1, 2])
