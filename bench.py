@@ -213,8 +213,10 @@ class ClockSampler:
 # ---------------------------------------------------------------------------------------------
 # CPU oracle on a bounded sample
 # ---------------------------------------------------------------------------------------------
-def oracle_sample(w, K, params, n_samples: int):
-    """Times the oracle on `n_samples` local steps of one chunk on one 1 x seq sequence each.
+def oracle_sample(w, K, params, n_samples: int, min_seconds: float = 0.0):
+    """Times the oracle on local steps of one chunk on one 1 x seq sequence each, round-robin over the
+    K chunks: `n_samples` of them, or, with `min_seconds` > 0, as many as it takes for the samples after
+    the first to add up to min_seconds (at least K + 1, at most n_samples).
 
     One local step of one chunk costs about 1/K of a full ZeroLock step of the same tokens,
     so the equivalent rate is (seq / K) tokens per sample time.
@@ -229,6 +231,8 @@ def oracle_sample(w, K, params, n_samples: int):
     h0 = orc.embed(ids)
     times = []
     for i in range(n_samples):
+        if min_seconds > 0 and i > K and sum(times[1:]) >= min_seconds:
+            break
         k = i % K + 1
         t0 = time.perf_counter()
         orc.local_grad(k, h0, labels)
@@ -408,9 +412,11 @@ def run_ours(args):
     # ---- CPU oracle on a bounded sample (rank 0, one GPU only) --------------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu and not args.lora and not args.adapter:
-        times, tok, cores = oracle_sample(w, K, params, 2)
-        cpu = {"value": tok / times[-1], "unit": "tokens/s", "cores": cores, "kind": "oracle",
-               "sample": f"one local step of chunk 2 on 1 x {w.seq} tokens (fp32 oracle, after one warm-up sample); "
+        times, tok, cores = oracle_sample(w, K, params, 64, min_seconds=15.0)
+        n, secs = len(times) - 1, sum(times[1:])
+        cpu = {"value": tok * n / secs, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+               "sample": f"{n} local steps of one chunk on 1 x {w.seq} tokens, round-robin over the K chunks "
+                         f"({secs:.1f} s of oracle work after one warm-up sample); "
                          f"rate = ({w.seq}/K) tokens per sample time"}
 
     if rank == 0:
