@@ -310,14 +310,69 @@ def chunk_bwd(P, dh, caches, m: Dims):
     return dh, grads
 
 
-def local_grad(P, d, bounds, k, h_prev, labels, alpha, kl_dir=0):
-    """(L_k, dL_k/dtheta_k, h_k): teacher and input held constant (Eq. 5, Remark 1)."""
+LORA_LINEARS = ("wqkv", "wo", "w1", "w2")
+
+
+def merge_lora(P, n_layers, scale):
+    """Weights with their low-rank updates folded in: w + scale * B A (Section II-A)."""
+    Q = dict(P)
+    for l in range(n_layers):
+        for s in LORA_LINEARS:
+            a = P.get(f"layers.{l}.{s}.lora_a")
+            if a is not None:
+                Q[f"layers.{l}.{s}"] = P[f"layers.{l}.{s}"] + scale * (P[f"layers.{l}.{s}.lora_b"] @ a)
+    return Q
+
+
+def lora_grads(P, grads, scale):
+    """y = x (w + s B A)^T: with G = dL/d(w + s B A), dL/dB = s G A^T and dL/dA = s B^T G; the base
+    weights, norms and biases are frozen."""
+    out = {}
+    for n, G in grads.items():
+        a = P.get(n + ".lora_a")
+        if a is not None:
+            out[n + ".lora_b"] = scale * G @ a.T
+            out[n + ".lora_a"] = scale * P[n + ".lora_b"].T @ G
+    return out
+
+
+def adapter_fwd(P, k, h):
+    """a_k(h) = h + GELU(h D^T) U^T (readout adapter of chunk k, Section III-B (b))."""
+    D, U = P[f"adapters.{k}.down"], P[f"adapters.{k}.up"]
+    act, gc = gelu_fwd(h @ D.T)
+    return h + act @ U.T, (h, act, gc)
+
+
+def adapter_bwd(P, k, da, cache):
+    """dU = da^T GELU(u), du = (da U) GELU'(u), dD = du^T h, dh = da + du D."""
+    h, act, gc = cache
+    D, U = P[f"adapters.{k}.down"], P[f"adapters.{k}.up"]
+    r, dm = D.shape
+    dU = da.reshape(-1, dm).T @ act.reshape(-1, r)
+    du = gelu_bwd(da @ U, gc)
+    dD = du.reshape(-1, r).T @ h.reshape(-1, dm)
+    return da + du @ D, {f"adapters.{k}.down": dD, f"adapters.{k}.up": dU}
+
+
+def local_grad(P, d, bounds, k, h_prev, labels, alpha, kl_dir=0, lora_scale=None, adapters=False):
+    """(L_k, dL_k/dtheta_k, h_k): teacher and input held constant (Eq. 5, Remark 1). lora_scale: only
+    the low-rank factors train; adapters: chunk k's readout goes through its adapter (the teacher is
+    the frozen head on h_{k-1})."""
     m = Dims(d)
-    t = readout_fwd(P, h_prev, m)[0] if alpha < 1.0 else None
-    h, caches = chunk_fwd(P, bounds, k, h_prev, m)
-    z, rc = readout_fwd(P, h, m)
+    W = merge_lora(P, d.n_layers, lora_scale) if lora_scale is not None else P
+    t = readout_fwd(W, h_prev, m)[0] if alpha < 1.0 else None
+    h, caches = chunk_fwd(W, bounds, k, h_prev, m)
+    x, ac = adapter_fwd(P, k, h) if adapters else (h, None)
+    z, rc = readout_fwd(W, x, m)
     L, dz = objective_and_dz(z, t, labels, alpha, kl_dir)
-    _, grads = chunk_bwd(P, readout_bwd(P, dz, rc, m), caches, m)
+    dh = readout_bwd(W, dz, rc, m)
+    extra = {}
+    if adapters:
+        dh, extra = adapter_bwd(P, k, dh, ac)
+    _, grads = chunk_bwd(W, dh, caches, m)
+    if lora_scale is not None:
+        grads = lora_grads(P, grads, lora_scale)
+    grads.update(extra)
     return L, grads, h
 
 

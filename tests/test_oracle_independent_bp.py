@@ -112,3 +112,45 @@ def test_manual_backward_agrees_with_its_own_finite_differences():
             flat[idx] = old
             fd = (lp - lm) / 2e-6
             assert abs(fd - gr.reshape(-1)[idx]) <= 1e-7 + 1e-6 * abs(fd), (n, idx)
+
+
+@pytest.mark.parametrize("d", [LLAMA_T, GPT2_T], ids=["llama", "gpt2"])
+def test_lora_local_gradients_match_manual_backward(d):
+    """LoRA chunks (only A and B train, Delta w = s B A): every factor's gradient element by element."""
+    from tests.test_oracle_pins import _lora_setup
+    P, cfg = _lora_setup(d)
+    ids, labels = _batch(d, seed=17)
+    orc = Oracle(cfg, P)
+    Pn = _np(P)
+    h = orc.embed(ids)
+    hm = h.numpy().copy()
+    for k in (1, 2):
+        L, g, h_next = orc.local_grad(k, h, labels)
+        Lm, gm, hm_next = mb.local_grad(Pn, d, cfg.bounds, k, hm, labels.numpy(), cfg.alpha,
+                                        lora_scale=cfg.lora_scale)
+        assert abs(L - Lm) <= REL * abs(Lm)
+        assert set(g) == set(gm) and all("lora_" in n for n in gm)
+        for n in g:
+            _close(g[n], gm[n], (k, n))
+        _close(h_next, hm_next, f"h_{k}")
+        h, hm = h_next, hm_next
+
+
+@pytest.mark.parametrize("d", [LLAMA_T, GPT2_T], ids=["llama", "gpt2"])
+def test_adapter_local_gradients_match_manual_backward(d):
+    """Readout adapters: every layer tensor and both adapter matrices of chunk k, element by element."""
+    from tests.test_oracle_pins import _adapter_setup
+    P, cfg = _adapter_setup(d)
+    ids, labels = _batch(d, seed=19)
+    orc = Oracle(cfg, P)
+    Pn = _np(P)
+    h = orc.embed(ids)
+    hm = h.numpy().copy()
+    for k in (1, 2):
+        L, g, h_next = orc.local_grad(k, h, labels)
+        Lm, gm, hm_next = mb.local_grad(Pn, d, cfg.bounds, k, hm, labels.numpy(), cfg.alpha, adapters=True)
+        assert abs(L - Lm) <= REL * abs(Lm)
+        assert set(g) == set(gm)
+        for n in g:
+            _close(g[n], gm[n], (k, n))
+        h, hm = h_next, hm_next

@@ -172,3 +172,14 @@ def test_independent_backward_catches_unbiased_layernorm_variance(monkeypatch):
     _patch(monkeypatch, "layernorm", ln_unbiased)
     with pytest.raises(AssertionError):
         ib.test_backprop_gradient_matches_manual_backward(pins.GPT2_T, [0, 1, 2])
+
+
+def test_independent_backward_catches_detached_lora_update(monkeypatch):
+    import tests.test_oracle_independent_bp as ib
+    orig = om.lora_weight
+
+    def merged_constant(P, l, name, scale):   # the merged weight built outside autograd: no factor gradient
+        return orig(P, l, name, scale).detach()
+    monkeypatch.setattr(om, "lora_weight", merged_constant)
+    with pytest.raises((AssertionError, RuntimeError)):
+        ib.test_lora_local_gradients_match_manual_backward(pins.LLAMA_T)
