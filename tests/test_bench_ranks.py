@@ -28,7 +28,7 @@ def _worker(rank, world, port, out):
 
 def test_two_replicas_take_the_slowest_rank_and_count_all_tokens():
     port = _free_port()
-    with mp.Manager() as mgr:
+    with mp.get_context("spawn").Manager() as mgr:
         out = mgr.dict()
         mp.spawn(_worker, args=(2, port, out), nprocs=2, join=True)
         res = dict(out)
