@@ -54,3 +54,65 @@ def test_bad_arguments_are_rejected_on_the_host(lib):
     with pytest.raises(b.ZLError):
         b.zl_create(odd, 2, [0, 2, 4], cfg)
     assert "zl_create" in b.last_error()
+
+
+def _header_struct_fields(name):
+    """(field, C type) pairs, in order, of `typedef struct { ... } name;` in include/zerolock.h."""
+    src = open(os.path.join(ROOT, "include", "zerolock.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    body = re.search(r"typedef struct \{([^{}]*)\}\s*" + name + r"\s*;", src, flags=re.S).group(1)
+    fields = []
+    for decl in body.split(";"):
+        decl = decl.strip()
+        if decl:
+            ctype, rest = decl.split(None, 1)
+            fields += [(v.strip(), ctype) for v in rest.split(",")]
+    return fields
+
+
+@pytest.mark.parametrize("name", ["zl_model_dims", "zl_train_cfg"])
+def test_binding_structs_match_the_header_layout(name):
+    """The ctypes structures list the header's fields in the header's order, with C int / float types
+    matching the declarations (a drift here would shift every later field across the ABI)."""
+    from paper_2608_07974_gb300 import binding
+    want = {"int": ctypes.c_int, "float": ctypes.c_float}
+    fields = _header_struct_fields(name)
+    st = getattr(binding, name)
+    assert [f for f, _ in st._fields_] == [f for f, _ in fields]
+    for (f, t), (_, ct) in zip(st._fields_, fields):
+        assert t is want[ct], (f, ct, t)
+    assert ctypes.sizeof(st) == 4 * len(fields)
+
+
+def test_product_path_never_imports_the_oracle():
+    """Nothing in the package or its CUDA sources refers to the oracle or the tests: the only way to
+    compute is the library."""
+    import ast
+    pkg = os.path.join(ROOT, "paper_2608_07974_gb300")
+    for py in glob.glob(os.path.join(pkg, "*.py")):
+        tree = ast.parse(open(py).read())
+        for node in ast.walk(tree):
+            mods = []
+            if isinstance(node, ast.Import):
+                mods = [a.name for a in node.names]
+            elif isinstance(node, ast.ImportFrom):
+                mods = [node.module or ""]
+            for mod in mods:
+                assert not mod.split(".")[0] in ("oracle", "tests"), (py, mod)
+    for src in glob.glob(os.path.join(pkg, "csrc", "*")):
+        assert "oracle" not in open(src).read().lower(), src
+
+
+def test_binding_refuses_to_load_without_the_library(monkeypatch):
+    """With libzerolock.so absent the binding raises ImportError: there is no CPU fallback."""
+    import importlib
+    import sys
+    from paper_2608_07974_gb300 import binding
+    real = os.path.exists
+    monkeypatch.setattr(os.path, "exists", lambda p: False if p == binding.LIB_PATH else real(p))
+    saved = sys.modules.pop("paper_2608_07974_gb300.binding")
+    try:
+        with pytest.raises(ImportError):
+            importlib.import_module("paper_2608_07974_gb300.binding")
+    finally:
+        sys.modules["paper_2608_07974_gb300.binding"] = saved
