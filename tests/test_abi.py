@@ -116,3 +116,43 @@ def test_binding_refuses_to_load_without_the_library(monkeypatch):
             importlib.import_module("paper_2608_07974_gb300.binding")
     finally:
         sys.modules["paper_2608_07974_gb300.binding"] = saved
+
+
+def _header_prototypes():
+    """name -> list of parameter kinds ('ptr', 'int', 'float', 'size_t') for every zl_ function."""
+    src = open(os.path.join(ROOT, "include", "zerolock.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    protos = {}
+    for name, args in re.findall(r"\b(zl_\w+)\s*\(([^)]*)\)\s*;", src, flags=re.S):
+        kinds = []
+        for a in args.split(","):
+            a = " ".join(a.split())
+            if not a or a == "void":
+                continue
+            if "*" in a:
+                kinds.append("ptr")
+            elif a.startswith("size_t"):
+                kinds.append("size_t")
+            elif a.startswith("float"):
+                kinds.append("float")
+            else:
+                assert a.startswith("int"), a
+                kinds.append("int")
+        protos[name] = kinds
+    return protos
+
+
+def test_binding_argument_types_match_the_header_prototypes():
+    """Every entry point is called with the header's arity and argument kinds (pointer, int, float,
+    size_t): a mismatch would pass garbage across the ABI without any error."""
+    from paper_2608_07974_gb300 import binding
+    kind = {ctypes.c_int: "int", ctypes.c_float: "float", ctypes.c_size_t: "size_t",
+            ctypes.c_void_p: "ptr", ctypes.c_char_p: "ptr"}
+    protos = _header_prototypes()
+    assert set(protos) == set(binding.EXPORTS)
+    for name, want in protos.items():
+        got = getattr(binding._lib, name).argtypes
+        assert got is not None, name
+        got = [kind.get(t, "ptr" if hasattr(t, "contents") or issubclass(t, ctypes._Pointer) else repr(t))
+               for t in got]
+        assert got == want, (name, got, want)
