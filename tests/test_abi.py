@@ -156,3 +156,40 @@ def test_binding_argument_types_match_the_header_prototypes():
         got = [kind.get(t, "ptr" if hasattr(t, "contents") or issubclass(t, ctypes._Pointer) else repr(t))
                for t in got]
         assert got == want, (name, got, want)
+
+
+# Argument checks that every single-kernel entry point makes before it touches the device. The
+# non-NULL pointers below are placeholders that must never be dereferenced; the test runs only where
+# no GPU is present, so even a wrongly accepted call cannot reach a kernel.
+@pytest.mark.skipif(__import__("torch").cuda.is_available(), reason="placeholder pointers: host-only check")
+def test_single_kernel_entry_points_reject_bad_arguments_on_the_host():
+    from paper_2608_07974_gb300 import binding as b
+    L = b._lib
+    P = 256   # placeholder device address
+    cases = [
+        ("zl_op_local_loss", (1, None, None, P, 4, 8, 8, 1.0, 0, P, P, P, None)),        # z NULL
+        ("zl_op_local_loss", (2, P, None, P, 4, 8, 8, 1.0, 0, P, P, P, None)),           # dtype
+        ("zl_op_local_loss", (1, P, None, P, 0, 8, 8, 1.0, 0, P, P, P, None)),           # N = 0
+        ("zl_op_local_loss", (1, P, None, P, 4, 8, 12, 1.0, 0, P, P, P, None)),          # ldz % 8
+        ("zl_op_local_loss", (1, P, None, P, 4, 8, 8, 0.5, 0, P, P, P, None)),           # alpha < 1 without t
+        ("zl_op_local_loss", (1, P, P, P, 4, 8, 8, 1.5, 0, P, P, P, None)),              # alpha > 1
+        ("zl_op_local_loss", (1, P, P, P, 4, 8, 8, 0.5, 2, P, P, P, None)),              # kl_dir
+        ("zl_op_local_loss_noalloc", (1, P, None, P, 65537, 8, 8, 1.0, 0, P, P, None)),  # beyond the scratch
+        ("zl_op_attention", (1, P, P, P, 2, 64, 4, 3, 64, None)),                        # H % Hkv
+        ("zl_op_attention", (1, P, P, P, 2, 64, 4, 4, 130, None)),                       # hd > 128
+        ("zl_op_attention", (1, P, P, P, 2, 64, 4, 4, 63, None)),                        # hd odd
+        ("zl_op_attention_bwd", (1, P, P, P, P, None, 2, 64, 4, 4, 64, None)),           # dqkv NULL
+        ("zl_op_gemm", (1, 3, 8, 8, 8, P, P, P, None)),                                  # mode
+        ("zl_op_gemm", (1, 0, -1, 8, 8, P, P, P, None)),                                 # M < 0
+        ("zl_op_gemm_ex", (1, 0, 8, 8, 8, P, P, P, None, None, 1, None)),                # r_mode 1 without R
+        ("zl_op_gemm_ex", (1, 2, 8, 8, 8, P, P, P, None, P, 0, None)),                   # mode 2 with R
+        ("zl_op_gemm_ex", (1, 2, 12, 8, 8, P, P, P, P, None, 0, None)),                  # column sums, M % 8
+    ]
+    for name, args in cases:
+        assert getattr(L, name)(*args) == b.ZL_ERR_ARG, (name, args)
+        assert b.last_error(), name
+    assert L.zl_kernel_launches(None) == b.ZL_ERR_ARG
+    for name in ("zl_step", "zl_bp_step", "zl_eval_global_loss"):
+        assert getattr(L, name)(None, P, P, 1, 1, None) == b.ZL_ERR_ARG, name
+    assert L.zl_synchronize(None, 0) == b.ZL_ERR_ARG
+    L.zl_free(None)   # NULL-safe
