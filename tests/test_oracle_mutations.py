@@ -183,3 +183,50 @@ def test_independent_backward_catches_detached_lora_update(monkeypatch):
     monkeypatch.setattr(om, "lora_weight", merged_constant)
     with pytest.raises((AssertionError, RuntimeError)):
         ib.test_lora_local_gradients_match_manual_backward(pins.LLAMA_T)
+
+
+def test_pins_catch_mask_hiding_the_diagonal(monkeypatch):
+    def attention_no_self(q, k, v):   # each position may not attend to itself (mask one too wide)
+        B, S, H, hd = q.shape
+        rep = H // k.shape[2]
+        kk, vv = k.repeat_interleave(rep, dim=2), v.repeat_interleave(rep, dim=2)
+        qh, kh, vh = (t.permute(0, 2, 1, 3) for t in (q, kk, vv))
+        s = qh @ kh.transpose(-1, -2) / math.sqrt(hd)
+        mask = torch.triu(torch.ones(S, S, dtype=torch.bool), diagonal=0)
+        mask[0, 0] = False                # keep row 0 defined
+        p = torch.softmax(s.masked_fill(mask, float("-inf")), dim=-1)
+        return (p @ vh).permute(0, 2, 1, 3)
+    _patch(monkeypatch, "attention", attention_no_self)
+    with pytest.raises(AssertionError):
+        pins.test_attention_matches_sdpa(4, 2, 8)
+
+
+def test_pins_catch_mean_over_all_rows(monkeypatch):
+    orig = om.local_objective_rows
+    _patch(monkeypatch, "local_objective",   # |Omega| replaced by the row count
+           lambda z, t, labels, alpha, kl_dir=0: orig(z, t, labels, alpha, kl_dir).sum() / labels.numel())
+    with pytest.raises(AssertionError):
+        pins.test_loss_closed_forms()
+
+
+def test_pins_catch_summed_window(monkeypatch):
+    orig = om.Oracle._apply_window
+
+    def summed(self, k, adapters=True):   # the window gradient summed instead of averaged
+        for n in self.chunk_names(k):
+            self.acc[n] *= self.cfg.accum_m
+        orig(self, k, adapters)
+    monkeypatch.setattr(om.Oracle, "_apply_window", summed)
+    with pytest.raises(AssertionError):
+        pins.test_accumulation_window_is_the_mean()
+
+
+def test_pins_catch_decay_after_the_adam_step(monkeypatch):
+    def late_decay(theta, g, m, v, step, lr, b1, b2, eps, wd):
+        m.mul_(b1).add_((1 - b1) * g)
+        v.mul_(b2).add_((1 - b2) * g * g)
+        theta.sub_(lr * (m / (1 - b1 ** step)) / (torch.sqrt(v / (1 - b2 ** step)) + eps))
+        theta.mul_(1 - lr * wd)
+    _patch(monkeypatch, "adamw_update", late_decay)
+    with pytest.raises(AssertionError):
+        pins.test_adamw_matches_torch_optim()
