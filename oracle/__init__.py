@@ -13,9 +13,11 @@ plain definition of "backpropagate inside the chunk only" (Remark 1).
 Pins (``tests/test_oracle_pins.py``): central finite differences, library
 routines (scaled_dot_product_attention, rms_norm, layer_norm, gelu, AdamW),
 closed forms of the loss, Lemma 1 (three-point identity), Lemma 2 (geometric
-mixture), Lemma 3 (stop-gradient block structure) and K=1, alpha=1 == BP.
-Parity unpinned: the convergence statements (Proposition 1, Theorem 1) need
-trained weights and data and are not checked.
+mixture), Lemma 3 (stop-gradient block structure), K=1, alpha=1 == BP, an
+independent autograd-free backward (tests/manual_backprop.py), and Proposition 1's
+chunk-wise bound in its token-level geometry (random soft targets and chains).
+Parity unpinned: Theorem 1 (a convergence rate over training) and Proposition 1
+for whole trained models need trained weights and data and are not checked.
 """
 from .model import (Oracle, OracleConfig, embed, layer_forward, chunk_forward, readout, adapter,
                     local_objective, local_objective_rows, rmsnorm, layernorm, rope,

@@ -145,6 +145,8 @@ def test_pins_catch_swapped_kl_direction(monkeypatch):
         pins.test_reverse_kl_direction_matches_library()
     with pytest.raises(AssertionError):
         pins.test_loss_closed_forms()
+    with pytest.raises(AssertionError):
+        pins.test_proposition1_chunkwise_bound()
 
 
 def test_independent_backward_catches_swapped_swiglu_halves(monkeypatch):

@@ -649,3 +649,33 @@ def test_reverse_kl_direction_matches_library():
     pq = (torch.softmax(z.detach(), -1) - torch.softmax(t, -1)) / 4
     pq[1] = 0
     assert torch.allclose(dz, pq, atol=1e-16, rtol=0)
+
+
+def test_proposition1_chunkwise_bound():
+    """Proposition 1 in the token-level geometry it is stated in: with psi the negative entropy
+    (D_psi = the oracle's KL), a soft target r and L(p) = KL(p || r) (smooth relative to psi with
+    beta = 1), p_k* the minimiser of the oracle's local objective alpha KL(p || r) + (1 - alpha)
+    KL(p || p_{k-1}) and any p_k with delta_k = KL(p_k || p_k*), the global loss obeys
+    L(p_K) <= L(p_0) - sum_k (1/alpha - 1) KL(p_k || p_{k-1}) + (1/alpha) sum_k delta_k."""
+    g = torch.Generator().manual_seed(21)
+    V, K = 9, 4
+    for a in (0.1, 0.3, 0.5, 0.8, 0.95):
+        for trial in range(300):
+            zr = 2 * torch.randn(1, V, generator=g)
+            zs = [torch.log_softmax(2 * torch.randn(1, V, generator=g), -1)]
+            stars = []
+            for k in range(K):
+                zstar = torch.log_softmax(a * torch.log_softmax(zr, -1) + (1 - a) * zs[-1], -1)
+                if trial == 0:   # p_k* is where the oracle's local objective is stationary
+                    zz = zstar.clone().requires_grad_(True)
+                    obj = a * oracle.kl_rows(zz, zr) + (1 - a) * oracle.kl_rows(zz, zs[-1])
+                    (gz,) = torch.autograd.grad(obj.sum(), zz)
+                    assert float(gz.abs().max()) < 1e-14
+                noise = 0.0 if trial % 5 == 0 else 0.3   # every fifth trial: p_k = p_k* (delta_k = 0)
+                stars.append(zstar)
+                zs.append(torch.log_softmax(zstar + noise * torch.randn(1, V, generator=g), -1))
+            L = lambda z: float(oracle.kl_rows(z, zr))
+            D = lambda u, v: float(oracle.kl_rows(u, v))
+            bound = (L(zs[0]) - sum((1 / a - 1) * D(zs[k + 1], zs[k]) for k in range(K))
+                     + sum(D(zs[k + 1], stars[k]) for k in range(K)) / a)
+            assert L(zs[-1]) <= bound + 1e-12, (a, trial, L(zs[-1]), bound)
