@@ -679,3 +679,27 @@ def test_proposition1_chunkwise_bound():
             bound = (L(zs[0]) - sum((1 / a - 1) * D(zs[k + 1], zs[k]) for k in range(K))
                      + sum(D(zs[k + 1], stars[k]) for k in range(K)) / a)
             assert L(zs[-1]) <= bound + 1e-12, (a, trial, L(zs[-1]), bound)
+
+
+def test_global_update_equivalence_gradient_is_jacobian_times_log_gap():
+    """Lemma 3 (global update equivalence, Section II-C): the gradient of the local objective
+    alpha KL(p || r) + (1 - alpha) KL(p || p_{k-1}) (the oracle's KL) is J^T e with
+    e = log p - log p*, p* the geometric mixture of Lemma 2. At the logits
+    J = diag(p) - p p^T, so dL/dz = p (e - <p, e>); and through a linear readout z = h W^T the chain
+    rule carries the same J^T e to the parameters."""
+    g = torch.Generator().manual_seed(31)
+    V, Dm = 11, 5
+    for a in (0.2, 0.5, 0.9):
+        zr, zq = torch.randn(4, V, generator=g), torch.randn(4, V, generator=g)
+        h = torch.randn(4, Dm, generator=g)
+        W = torch.randn(V, Dm, generator=g).requires_grad_(True)
+        z = h @ W.T
+        L = (a * oracle.kl_rows(z, zr) + (1 - a) * oracle.kl_rows(z, zq)).sum()
+        (gW,) = torch.autograd.grad(L, W)
+        with torch.no_grad():
+            lp = torch.log_softmax(z, -1)
+            lstar = torch.log_softmax(a * torch.log_softmax(zr, -1) + (1 - a) * torch.log_softmax(zq, -1), -1)
+            e = lp - lstar
+            p = lp.exp()
+            dz = p * (e - (p * e).sum(-1, keepdim=True))
+        assert torch.allclose(gW, dz.T @ h, atol=1e-13, rtol=1e-11)
