@@ -20,6 +20,7 @@
  *     ZL_DTYPE_BF16: bfloat16) unless stated otherwise. ids and labels are
  *     int32 device arrays of B*S entries; a label of -1 marks a position
  *     outside Omega; ids must lie in [0, vocab), labels in [-1, vocab).
+ *     A micro-batch holds 1 <= B*S <= 2^24 tokens, B <= 65535, S <= max_seq.
  *   - Pointers passed in are borrowed: the library never frees them, and
  *     device pointers given to a call must stay valid and unmodified until the
  *     next zl_synchronize() on that context returns (work is asynchronous).
@@ -208,7 +209,8 @@ zl_status zl_kernel_launches(uint64_t* count);
 
 /* Fused local objective (Eq. 3-5) over N rows of logits. z, t: [N, ldz] in `dtype`
  * (columns >= V are padding and ignored); t may be NULL when alpha == 1.
- * labels: [N] int32. Writes dz = dL/dz [N, ldz] (dtype; padding columns 0) and
+ * labels: [N] int32; 1 <= N <= 2^24 (|Omega| is counted exactly up to 2^24 rows, so larger N is
+ * rejected with ZL_ERR_ARG). Writes dz = dL/dz [N, ldz] (dtype; padding columns 0) and
  * row_loss[N] (fp32, alpha*CE_i + (1-alpha)*KL_i, 0 outside Omega), and *loss
  * (one fp32 on the device) = sum(row_loss) / |Omega|. */
 zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_t* labels, int N,

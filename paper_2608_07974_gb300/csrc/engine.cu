@@ -788,7 +788,8 @@ void start_on(zl_ctx* c, cudaStream_t s) {   // order s after the user's stream
 void check_bs(zl_ctx* c, int B, int S) {
   if (B <= 0 || S <= 0) raise_err(ZL_ERR_ARG, "empty micro-batch (B and S must be >= 1)");
   if (S > c->dims.max_seq) raise_err(ZL_ERR_ARG, "S exceeds max_seq");
-  if ((long)B * S > (1L << 26)) raise_err(ZL_ERR_ARG, "B*S too large");
+  // |Omega| is counted in fp32 partial sums, exact up to 2^24 positions
+  if ((long)B * S > (1L << 24)) raise_err(ZL_ERR_ARG, "B*S above 2^24 tokens");
   if (B > 65535) raise_err(ZL_ERR_ARG, "B above 65535");
 }
 
@@ -1867,6 +1868,7 @@ zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_
   if (!z || !labels || !dz || !row_loss || !loss) { g_err = "NULL argument"; return ZL_ERR_ARG; }
   if (dtype != 0 && dtype != 1) { g_err = "dtype"; return ZL_ERR_ARG; }
   if (N < 1 || V < 2 || ldz < V || ldz % 8 != 0) { g_err = "need N >= 1, V >= 2, ldz >= V, ldz % 8 == 0"; return ZL_ERR_ARG; }
+  if (N > (1 << 24)) { g_err = "N above 2^24 rows (|Omega| is counted exactly up to 2^24)"; return ZL_ERR_ARG; }
   if (!(alpha > 0.f && alpha <= 1.f) || (alpha < 1.f && !t) || (kl_dir != 0 && kl_dir != 1)) {
     g_err = "alpha in (0,1], t required when alpha < 1, kl_dir 0/1";
     return ZL_ERR_ARG;

@@ -174,6 +174,7 @@ def test_single_kernel_entry_points_reject_bad_arguments_on_the_host():
         ("zl_op_local_loss", (1, P, None, P, 4, 8, 8, 0.5, 0, P, P, P, None)),           # alpha < 1 without t
         ("zl_op_local_loss", (1, P, P, P, 4, 8, 8, 1.5, 0, P, P, P, None)),              # alpha > 1
         ("zl_op_local_loss", (1, P, P, P, 4, 8, 8, 0.5, 2, P, P, P, None)),              # kl_dir
+        ("zl_op_local_loss", (1, P, None, P, (1 << 24) + 1, 8, 8, 1.0, 0, P, P, P, None)),  # N above 2^24
         ("zl_op_local_loss_noalloc", (1, P, None, P, 65537, 8, 8, 1.0, 0, P, P, None)),  # beyond the scratch
         ("zl_op_attention", (1, P, P, P, 2, 64, 4, 3, 64, None)),                        # H % Hkv
         ("zl_op_attention", (1, P, P, P, 2, 64, 4, 4, 130, None)),                       # hd > 128
