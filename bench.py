@@ -191,23 +191,29 @@ class ClockSampler:
             self.proc.kill()
         self.out.flush()
         self.out.seek(0)
-        rows = [r.split(",") for r in self.out.read().strip().splitlines() if r.strip()]
+        text = self.out.read()
         os.unlink(self.out.name)
-        sm, mx, reasons = [], 0.0, set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for r in rows:
-            try:
-                sm.append(float(r[1]))
-                mx = max(mx, float(r[2]))
-                for n, v in zip(names, r[5:9]):
-                    if v.strip() == "Active":
-                        reasons.add(n)
-            except (ValueError, IndexError):
-                continue
-        if not sm:
-            return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+        return parse_clocks(text)
+
+
+def parse_clocks(text: str):
+    """Summary of nvidia-smi samples in ClockSampler.FIELDS order (csv, no header, no units): median SM
+    clock, the maximum SM clock, and every throttle reason seen Active in any sample."""
+    rows = [r.split(",") for r in text.strip().splitlines() if r.strip()]
+    sm, mx, reasons = [], 0.0, set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for r in rows:
+        try:
+            sm.append(float(r[1]))
+            mx = max(mx, float(r[2]))
+            for n, v in zip(names, r[5:9]):
+                if v.strip() == "Active":
+                    reasons.add(n)
+        except (ValueError, IndexError):
+            continue
+    if not sm:
+        return None
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
 
 
 # ---------------------------------------------------------------------------------------------

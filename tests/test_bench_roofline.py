@@ -30,3 +30,13 @@ def test_traffic_figures_are_tied_to_the_kernel_sources(monkeypatch):
                         {"sources": bench.GEMM_SOURCES, "sha256": "0" * 16, "bytes_per_launch": 123.0})
     assert bench.measured_traffic("gemm_layer") is None
     assert bench.measured_traffic("no_such_class") is None
+
+
+def test_clock_summary_keeps_the_median_the_max_and_every_active_reason():
+    text = ("0, 1980, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active\n"
+            "0, 2040, 2070, 1390.5, 0x4, Not Active, Not Active, Not Active, Active\n"
+            "0, 1500, 2070, 1380.0, 0x8, Active, Not Active, Not Active, Not Active\n"
+            "garbage line\n")
+    c = bench.parse_clocks(text)
+    assert c == {"sm_mhz": 1980.0, "sm_max_mhz": 2070.0, "reasons": ["hw_slowdown", "sw_power_cap"], "samples": 3}
+    assert bench.parse_clocks("") is None
