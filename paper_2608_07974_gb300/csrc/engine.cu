@@ -3,6 +3,7 @@
 // (Eq. 6 as AdamW), and the K-stream scheduler with early forwarding, per-entry readiness
 // events and a bound on live activation arenas (Section III-A/B).
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <atomic>
@@ -229,6 +230,28 @@ const void* TrainC(zl_ctx* c, Chunk& k, size_t off) {
 }
 
 size_t esz(zl_ctx* c) { return dt_size(c->dt); }
+
+// Consecutive host-side NVTX ranges over the phases a call enqueues, named by chunk and phase, so a
+// profiler can select one chunk's or one phase's kernels (ncu --nvtx --nvtx-include "zl chunk 2 loss/").
+// Without an attached tool each range is a cheap no-op.
+class NvtxPhases {
+ public:
+  ~NvtxPhases() { end(); }
+  void next(const char* fmt, int k = 0) {
+    end();
+    char name[64];
+    std::snprintf(name, sizeof name, fmt, k);
+    nvtxRangePushA(name);
+    open_ = true;
+  }
+  void end() {
+    if (open_) nvtxRangePop();
+    open_ = false;
+  }
+
+ private:
+  bool open_ = false;
+};
 
 void wait_ev(cudaStream_t s, cudaEvent_t e) { CK(cudaStreamWaitEvent(s, e, 0)); }
 void rec(cudaEvent_t e, cudaStream_t s) { CK(cudaEventRecord(e, s)); }
@@ -1273,6 +1296,8 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
   cudaStream_t s = ck.s;
   const int N = B * S;
   const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
+  NvtxPhases ph;
+  ph.next("zl chunk %d forward", k);
   void* h0 = nullptr;
   if (!h_in) {
     h0 = palloc(c, hb, s);
@@ -1289,13 +1314,16 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
   ChunkActs acts;
   chunk_fwd_save(c, ck, h_in, hk, B, S, acts, s);
   if (h_out) CK(cudaMemcpyAsync(h_out, hk, hb, cudaMemcpyDeviceToDevice, s));
+  ph.next("zl chunk %d readout", k);
   void* z = palloc(c, zb, s);
   ReadoutSave rs;
   Chunk* ad = c->cfg.adapter_dim > 0 ? &ck : nullptr;
   readout_fwd(c, hk, z, &rs, N, s, ad);
+  ph.next("zl chunk %d loss", k);
   void* dz = local_loss(c, z, t, labels, a, N, k, s);
   pfree(z, s);
   pfree(t, s);
+  ph.next("zl chunk %d backward", k);
   void* dh = palloc(c, hb, s);
   readout_bwd(c, hk, rs, dz, dh, N, s, ad);
   pfree(dz, s);
@@ -1304,7 +1332,9 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
   pfree(acts.mem, s);
   pfree(hk, s);
   pfree(h0, s);
+  ph.next("zl chunk %d adamw", k);
   adamw_window(c, ck, s);
+  ph.end();
   ck.done += 1;
 }
 
@@ -1519,6 +1549,8 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
   rec(c->ev_start, c->user);
   for (int k = 1; k <= K; ++k) wait_ev(c->ch[k].s, c->ev_start);
   wait_ev(c->aux, c->ev_start);
+  NvtxPhases ph;
+  ph.next("zl step embedding and teacher");
   std::vector<void*> h(K + 1, nullptr), z(K + 1, nullptr);
   // h_0 = E(x) on s_1; the teacher of chunk 1, z_0 = readout(h_0), on the auxiliary stream
   cudaStream_t s1 = c->ch[1].s;
@@ -1540,6 +1572,7 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
     Chunk& ck = c->ch[k];
     cudaStream_t s = ck.s;
     const float a = alpha_of(c, k);
+    ph.next("zl chunk %d forward", k);
     // S1: the upstream entry (h_{k-1}) and a free arena slot
     if (k > 1) wait_ev(s, c->ch[k - 1].ev_h);
     ring_put(c, ck, c->seq, h[k - 1], labels, B, S, s);
@@ -1554,10 +1587,12 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
     ChunkActs acts;
     chunk_fwd_save(c, ck, h[k - 1], h[k], B, S, acts, s);
     rec(ck.ev_h, s);
+    ph.next("zl chunk %d readout", k);
     z[k] = palloc(c, zb, s);
     ReadoutSave rs;
     readout_fwd(c, h[k], z[k], &rs, N, s, adp ? &ck : nullptr);
     rec(ck.ev_z, s);
+    ph.next("zl chunk %d loss", k);
     // S3: local objective against the stop-gradient teacher: the frozen head on h_{k-1}, which is
     // chunk k-1's own readout z_{k-1} (reused) unless chunk k-1 read out through its adapter
     void* teacher = nullptr;
@@ -1586,6 +1621,7 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
       pfree(z[k - 1], s);
     }
     if (k == K || adp) pfree(z[k], s);   // with adapters no later chunk reads z_k
+    ph.next("zl chunk %d backward", k);
     void* dh = palloc(c, hb, s);
     readout_bwd(c, h[k], rs, dz, dh, N, s, adp ? &ck : nullptr);
     pfree(dz, s);
@@ -1599,8 +1635,10 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
     else wait_ev(s, c->ch[k - 1].ev_hb);
     pfree(h[k - 1], s);
     if (k == K) pfree(h[K], s);
+    ph.next("zl chunk %d adamw", k);
     adamw_window(c, ck, s);
   }
+  ph.end();
   c->last_nloss = K;
   c->seq += 1;
 }
@@ -1655,6 +1693,8 @@ void bp_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int
       rec(c->ch[k].ev_done, c->ch[k].s);
       wait_ev(s, c->ch[k].ev_done);
     }
+  NvtxPhases ph;
+  ph.next("zl bp forward");
   std::vector<void*> h(K + 1, nullptr);
   std::vector<ChunkActs> acts(K + 1);
   h[0] = palloc(c, hb, s);
@@ -1663,11 +1703,13 @@ void bp_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int
     h[k] = palloc(c, hb, s);
     chunk_fwd_save(c, c->ch[k], h[k - 1], h[k], B, S, acts[k], s);
   }
+  ph.next("zl bp readout and loss");
   void* z = palloc(c, zb, s);
   ReadoutSave rs;
   readout_fwd(c, h[K], z, &rs, N, s);
   void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
   pfree(z, s);
+  ph.next("zl bp backward");
   void* dh = palloc(c, hb, s);
   void* dh2 = palloc(c, hb, s);
   readout_bwd(c, h[K], rs, dz, dh, N, s);
@@ -1681,6 +1723,7 @@ void bp_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int
   pfree(h[0], s);
   pfree(dh, s);
   pfree(dh2, s);
+  ph.next("zl bp adamw");
   for (int k = 1; k <= K; ++k) {
     if (k > 1) {   // the optimizer step of chunk k stays on its own stream
       rec(c->ch[1].ev_done, s);
