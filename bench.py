@@ -2,8 +2,9 @@
 """Throughput of ZeroLock's concurrent per-chunk update on GB300 (one JSON line on stdout).
 
 A step is one micro-batch through all K chunks (forward, readout, local objective, local
-backward, AdamW) via zl_step. Default workload: the GPT-2-small-shaped bf16 model (12 layers,
-d 768, vocab 50257, micro-batch 8 x 512 tokens, K = 4). Also reported: the same-engine
+backward, AdamW) via zl_step. Default workload: the largest configuration, the Llama-2-7B-shaped
+bf16 full fine-tune (32 layers, d 4096, SwiGLU 11008, vocab 32000, micro-batch 2 x 1024 tokens,
+K = 8 chunks of 4 layers); --workload gpt2|llama1b|llama3b|tiny selects the others. Also reported: the same-engine
 backpropagation baseline (zl_bp_step), peak HBM of both, the GEMM roofline fraction measured
 live with CUDA events, the CPU oracle on a bounded sample, an end-to-end figure through the
 public API with host buffers, and SM clocks sampled during the timed region.
@@ -41,10 +42,10 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="gpt2", choices=list(WORKLOADS))
+    ap.add_argument("--workload", default="llama7b", choices=list(WORKLOADS))
     ap.add_argument("--K", type=int, default=0, help="chunk count (default: the workload's)")
     ap.add_argument("--max-live", type=int, default=2, help="chunks whose activations may be alive at once")
     ap.add_argument("--lora", type=int, default=0, help="LoRA rank (0: full fine-tune); scale 16 / rank")
@@ -219,31 +220,78 @@ def parse_clocks(text: str):
 # ---------------------------------------------------------------------------------------------
 # CPU oracle on a bounded sample
 # ---------------------------------------------------------------------------------------------
-def oracle_sample(w, K, params, n_samples: int, min_seconds: float = 0.0):
-    """Times the oracle on local steps of one chunk on one 1 x seq sequence each, round-robin over the
-    K chunks: `n_samples` of them, or, with `min_seconds` > 0, as many as it takes for the samples after
-    the first to add up to min_seconds (at least K + 1, at most n_samples).
+ORACLE_SAMPLE_FLOP = 0.5e12      # about the oracle work of one CPU-baseline sample
+ORACLE_WHOLE_MODEL_PARAMS = 3e9  # above this the sample runs chunk 1 alone (every chunk costs about the same)
 
-    One local step of one chunk costs about 1/K of a full ZeroLock step of the same tokens,
-    so the equivalent rate is (seq / K) tokens per sample time.
+
+def oracle_sample_plan(w, K):
+    """(chunks sampled, tokens per sample sequence) of the CPU-baseline sample.
+
+    One sample is chunk k's local step on one sequence. Its length is the longest power of two up to
+    the workload's sequence length whose estimated cost (6 FLOP per chunk parameter and token for the
+    forward and backward, plus the student and teacher heads) stays near ORACLE_SAMPLE_FLOP, at least
+    64. Models above ORACLE_WHOLE_MODEL_PARAMS sample chunk 1 only (as a one-chunk model of its own
+    layers, whose teacher is the readout of h_0 exactly as in the full model); smaller ones go
+    round-robin over all K chunks.
+    """
+    d = w.dims
+    layer = sum(int(torch.tensor(shp).prod()) for _, shp in synth.layer_param_shapes(d))
+    per_tok = 6.0 * layer * d.n_layers / K + 6.0 * d.d_model * d.vocab
+    seq = 64
+    while seq * 2 <= w.seq and seq * 2 * per_tok <= ORACLE_SAMPLE_FLOP:
+        seq *= 2
+    seq = min(seq, w.seq)
+    chunks = list(range(1, K + 1)) if layer * d.n_layers <= ORACLE_WHOLE_MODEL_PARAMS else [1]
+    return chunks, seq
+
+
+def oracle_params(w, K, chunks, params=None):
+    """fp32 CPU tensors the oracle needs for the sampled chunks (drawn on the GPU when one is present)."""
+    import dataclasses
+    bounds = synth.chunk_bounds(w.dims.n_layers, K)
+    if chunks == list(range(1, K + 1)):
+        dims, layers = w.dims, None
+    else:
+        dims, layers = dataclasses.replace(w.dims, n_layers=bounds[1]), range(bounds[1])
+    if params is None:
+        dev = "cuda" if torch.cuda.is_available() else "cpu"
+        params = synth.make_params(w.dims, w.seed, layers=layers, device=dev)
+    keep = set(n for n, _ in synth.frozen_param_shapes(w.dims)) | set(n for n, _ in synth.param_names(dims))
+    return dims, {n: t.cpu() for n, t in params.items() if n in keep}
+
+
+def oracle_sample(w, K, params, n_samples: int, min_seconds: float = 0.0):
+    """Times the oracle on local steps of one chunk on one sequence each (oracle_sample_plan: the
+    chunks, round-robin, and the sequence length): `n_samples` of them, or, with `min_seconds` > 0, as
+    many as it takes for the samples after the first to add up to min_seconds (at least one per sampled
+    chunk after the first sample, at most n_samples). `params` may be None (drawn here) or the
+    workload's tensors on any device.
+
+    One local step of one chunk costs about 1/K of a full ZeroLock step of the same tokens, so the
+    equivalent rate is (sequence length / K) tokens per sample time. Returns (times, tokens per
+    sample, intra-op threads, a description of the sample).
     """
     from oracle import Oracle, OracleConfig
-    bounds = synth.chunk_bounds(w.dims.n_layers, K)
-    P = {n: (synth.round_bf16(t) if (w.dtype == "bf16" and t.dim() == 2) else t) for n, t in params.items()}
+    chunks, seq = oracle_sample_plan(w, K)
+    dims, P = oracle_params(w, K, chunks, params)
+    bounds = synth.chunk_bounds(dims.n_layers, K) if dims is w.dims else [0, dims.n_layers]
+    P = {n: (synth.round_bf16(t) if (w.dtype == "bf16" and t.dim() == 2) else t) for n, t in P.items()}
     dt = torch.float32 if w.dtype == "bf16" else torch.float64
-    orc = Oracle(OracleConfig(dims=w.dims, bounds=bounds, alpha=w.alpha, lr=w.lr), P, dtype=dt)
-    ids = synth.zipf_ids(w.seed + 77, 1, w.seq, w.dims.vocab)
+    orc = Oracle(OracleConfig(dims=dims, bounds=bounds, alpha=w.alpha, lr=w.lr), P, dtype=dt)
+    ids = synth.zipf_ids(w.seed + 77, 1, seq, w.dims.vocab)
     labels = synth.next_token_labels(ids)
     h0 = orc.embed(ids)
     times = []
     for i in range(n_samples):
-        if min_seconds > 0 and i > K and sum(times[1:]) >= min_seconds:
+        if min_seconds > 0 and i > len(chunks) and sum(times[1:]) >= min_seconds:
             break
-        k = i % K + 1
+        k = chunks[i % len(chunks)]
         t0 = time.perf_counter()
         orc.local_grad(k, h0, labels)
         times.append(time.perf_counter() - t0)
-    return times, (w.seq / K), torch.get_num_threads()
+    which = "round-robin over the K chunks" if len(chunks) == K else "of chunk 1 (every chunk has about its size)"
+    desc = f"local steps of one chunk on 1 x {seq} tokens, {which}; rate = ({seq}/K) tokens per sample time"
+    return times, (seq / K), torch.get_num_threads(), desc
 
 
 def run_reference(args):
@@ -252,17 +300,17 @@ def run_reference(args):
         return
     w = WORKLOADS[args.workload]
     K = args.K or w.K
-    params = synth.make_params(w.dims, w.seed)
-    times, tok, cores = oracle_sample(w, K, params, args.warmup + args.steps)
+    times, tok, cores, desc = oracle_sample(w, K, None, args.warmup + args.steps)
     t = sum(times[args.warmup:])
     value = tok * args.steps / t
-    sample = f"{args.steps} local steps of one chunk on 1 x {w.seq} tokens, round-robin over the K chunks"
+    sample = f"{args.steps} {desc}"
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f32" if w.dtype == "bf16" else "f64", "data": "synthetic",
             "config": {"workload": workload_desc(w, K), "K": K},
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "nproc": os.cpu_count(),
+                             "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -285,11 +333,12 @@ def run_ours(args):
     w = WORKLOADS[args.workload]
     K = args.K or w.K
     bounds = synth.chunk_bounds(w.dims.n_layers, K)
-    params = synth.make_params(w.dims, w.seed)
+    # drawn on the device (the same counter-based draws as on the host; the 7B-shaped model has 6.7 B)
+    params = synth.make_params(w.dims, w.seed, device="cuda")
     if args.lora:
-        params.update(synth.make_lora_params(w.dims, w.seed, args.lora))
+        params.update({n: t.cuda() for n, t in synth.make_lora_params(w.dims, w.seed, args.lora).items()})
     if args.adapter:
-        params.update(synth.make_adapter_params(w.dims, K, w.seed, args.adapter))
+        params.update({n: t.cuda() for n, t in synth.make_adapter_params(w.dims, K, w.seed, args.adapter).items()})
 
     def make_engine(max_live, serialize=False):
         e = zb.ZeroLock(w.dims, K, bounds, dtype=w.dtype, alpha=w.alpha, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
@@ -403,6 +452,8 @@ def run_ours(args):
         bp = {"value": job_tokens_per_s(tokens, args.steps, world, bms), "unit": "tokens/s",
               "peak_hbm_gb": beng.peak_bytes()[0] / 1e9, "ms_per_step": bms / args.steps}
         beng.close()
+        del beng
+        torch.cuda.empty_cache()
 
     # ---- the same step with every chunk on one stream: per-launch times without the other chunks' kernels
     seng = make_engine(args.max_live, serialize=True)
@@ -413,17 +464,17 @@ def run_ours(args):
         zb.zl_step(seng.ctx, dev_batches[i % nb][0], dev_batches[i % nb][1], w.batch, w.seq, K, want_losses=False)
     sprof = zb.zl_profile_read(seng.ctx)
     seng.close()
+    del seng
+    torch.cuda.empty_cache()
     roof_serial = roofline_of(sprof)
 
     # ---- CPU oracle on a bounded sample (rank 0, one GPU only) --------------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu and not args.lora and not args.adapter:
-        times, tok, cores = oracle_sample(w, K, params, 64, min_seconds=15.0)
+        times, tok, cores, desc = oracle_sample(w, K, params, 64, min_seconds=15.0)
         n, secs = len(times) - 1, sum(times[1:])
-        cpu = {"value": tok * n / secs, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-               "sample": f"{n} local steps of one chunk on 1 x {w.seq} tokens, round-robin over the K chunks "
-                         f"({secs:.1f} s of oracle work after one warm-up sample); "
-                         f"rate = ({w.seq}/K) tokens per sample time"}
+        cpu = {"value": tok * n / secs, "unit": "tokens/s", "cores": cores, "nproc": os.cpu_count(),
+               "kind": "oracle", "sample": f"{n} {desc} ({secs:.1f} s of oracle work after one warm-up sample)"}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,

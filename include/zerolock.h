@@ -51,6 +51,12 @@ typedef enum {
   ZL_ERR_UNSUPPORTED = -6   /* valid but not implemented combination                           */
 } zl_status;
 
+/* Device-side error bits: kernels OR them into an error word, which zl_synchronize reports as
+ * ZL_ERR_ARG (bad ids or labels) with a message naming each bit, and zl_wait_selftest returns. */
+#define ZL_DEVERR_BAD_ID 1u      /* a token id outside [0, vocab)                   */
+#define ZL_DEVERR_BAD_LABEL 2u   /* a label outside [-1, vocab)                     */
+#define ZL_DEVERR_TIMEOUT 4u     /* a bounded wait inside a kernel gave up          */
+
 enum { ZL_ARCH_LLAMA = 0, ZL_ARCH_GPT2 = 1 };
 enum { ZL_DTYPE_F32 = 0, ZL_DTYPE_BF16 = 1 };
 
@@ -85,6 +91,10 @@ typedef struct {
   int graph;                /* 1: zl_step / zl_bp_step are captured as a CUDA graph once per micro-batch */
                             /*   shape (after one eager call at that shape) and replayed; taken only    */
                             /*   with accum_m = 1, replay_depth = 0 and profiling off (else eager)      */
+  int fuzz_delay_us;        /* scheduler fuzz (tests): > 0 sleeps the host a pseudo-random 0..this many  */
+  unsigned fuzz_seed;       /*   microseconds (SplitMix64 stream of fuzz_seed) at every phase boundary of */
+                            /*   an enqueue, so the GPU runs ahead in varying interleavings; 0 is off,   */
+                            /*   at most 100000. Results do not depend on it.                           */
 } zl_train_cfg;
 
 /* Create a context: parameters, AdamW state, K streams and events, a stream-ordered
@@ -212,7 +222,9 @@ zl_status zl_kernel_launches(uint64_t* count);
  * labels: [N] int32; 1 <= N <= 2^24 (|Omega| is counted exactly up to 2^24 rows, so larger N is
  * rejected with ZL_ERR_ARG). Writes dz = dL/dz [N, ldz] (dtype; padding columns 0) and
  * row_loss[N] (fp32, alpha*CE_i + (1-alpha)*KL_i, 0 outside Omega), and *loss
- * (one fp32 on the device) = sum(row_loss) / |Omega|. */
+ * (one fp32 on the device) = sum(row_loss) / |Omega|. A label outside [-1, V) is treated as
+ * -1 (the row leaves Omega); this call does not report it, since reporting would need a
+ * synchronisation (the engine's step calls do report it, through zl_synchronize). */
 zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_t* labels, int N,
                            int V, int ldz, float alpha, int kl_dir, void* dz, float* row_loss,
                            float* loss, void* stream);
@@ -231,12 +243,13 @@ zl_status zl_op_attention_bwd(int dtype, const void* qkv, const void* out, const
  * cannot allocate device memory: a host framework whose own caching allocator has reserved the
  * device budget, so an outside cudaMalloc fails or breaks its accounting, or a latency-critical
  * loop that must not take the synchronisation cudaMalloc / cudaFree can imply. Same inputs and
- * outputs as zl_op_local_loss except that the per-row losses stay internal; the scratch
- * (per-row losses, |Omega|, an error word) is a file-scope device array of
+ * outputs as zl_op_local_loss except that the per-row losses stay internal (out-of-range labels
+ * leave Omega without being reported, as there); the scratch (per-row losses, |Omega|, a word the
+ * label check writes) is a file-scope device array of
  * ZL_NOALLOC_MAX_ROWS + 128 floats (257 KB) that every GPU which loads the library holds until
- * process exit. N > ZL_NOALLOC_MAX_ROWS is rejected with ZL_ERR_ARG. The first call on a device
- * looks up the array's device address (cudaGetSymbolAddress, with that device current); make
- * that first call before any stream capture. All calls share the array: calls whose work
+ * process exit. N > ZL_NOALLOC_MAX_ROWS is rejected with ZL_ERR_ARG. The first call in each CUDA
+ * context looks up the array's device address (cudaGetSymbolAddress, with that device current);
+ * make that first call before any stream capture. All calls share the array: calls whose work
  * overlaps on the GPU race on it, so order them on one stream (or synchronise between them).
  * Calls no cudaMalloc, cudaFree or allocating library routine. */
 #define ZL_NOALLOC_MAX_ROWS 65536
@@ -258,6 +271,17 @@ zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, co
  * and r_mode 0 (else ZL_ERR_ARG). */
 zl_status zl_op_gemm_ex(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C,
                         float* bias, const void* R, int r_mode, void* stream);
+
+/* Self-test of the bounded waits (no counterpart in the paper; failure detection without a GPU
+ * fault). Every wait of the tcgen05 kernels on an mbarrier (a TMA copy landing, a product completing,
+ * a tile drained) gives up after about 2 s of SM clock (longer at lower clocks), ORs
+ * ZL_DEVERR_TIMEOUT into the error word and unwinds the kernel, so a lost arrival ends as an error
+ * status instead of a hung GPU. This call runs that same wait on an mbarrier that nothing ever
+ * arrives at (one CTA, its own stream), waits for the kernel, and writes the kernel's error bits to
+ * *bits_out (host): ZL_DEVERR_TIMEOUT when the wait gave up as designed. It takes the wait's full
+ * limit (seconds). Returns ZL_OK with the bits written, or ZL_ERR_CUDA / ZL_ERR_STATE if the launch
+ * or the synchronisation failed. The device and any context on it stay usable afterwards. */
+zl_status zl_wait_selftest(unsigned* bits_out);
 
 #ifdef __cplusplus
 }

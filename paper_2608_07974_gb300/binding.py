@@ -15,14 +15,16 @@ LIB_PATH = os.path.join(HERE, "libzerolock.so")
 
 ZL_OK, ZL_ERR_ARG, ZL_ERR_CUDA, ZL_ERR_OOM, ZL_ERR_STATE, ZL_ERR_TIMEOUT, ZL_ERR_UNSUPPORTED = 0, -1, -2, -3, -4, -5, -6
 ZL_ARCH_LLAMA, ZL_ARCH_GPT2 = 0, 1
+ZL_DEVERR_BAD_ID, ZL_DEVERR_BAD_LABEL, ZL_DEVERR_TIMEOUT = 1, 2, 4
 ZL_DTYPE_F32, ZL_DTYPE_BF16 = 0, 1
+ZL_NOALLOC_MAX_ROWS = 65536   # rows of zl_op_local_loss_noalloc's static scratch (include/zerolock.h)
 
 #: every symbol include/zerolock.h declares
 EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_load_weights", "zl_get_param", "zl_param_numel",
            "zl_embed", "zl_forward_chunk", "zl_local_step", "zl_step", "zl_bp_step", "zl_eval_global_loss",
            "zl_read_losses", "zl_join", "zl_synchronize", "zl_peak_bytes", "zl_reset_peak", "zl_last_error",
            "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_gemm_ex", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
-           "zl_chunk_load", "zl_replay"]
+           "zl_chunk_load", "zl_replay", "zl_wait_selftest"]
 
 
 class zl_model_dims(C.Structure):
@@ -37,7 +39,7 @@ class zl_train_cfg(C.Structure):
                 ("accum_m", C.c_int), ("max_live_chunks", C.c_int), ("lr_schedule", C.c_int),
                 ("lr_gamma", C.c_float), ("serialize", C.c_int), ("lora_rank", C.c_int),
                 ("lora_scale", C.c_float), ("replay_depth", C.c_int), ("adapter_dim", C.c_int),
-                ("graph", C.c_int)]
+                ("graph", C.c_int), ("fuzz_delay_us", C.c_int), ("fuzz_seed", C.c_uint)]
 
 
 class ZLError(RuntimeError):
@@ -85,6 +87,7 @@ def _load() -> C.CDLL:
         "zl_chunk_save": [vp, i, vp, sz],
         "zl_chunk_load": [vp, i, vp, sz],
         "zl_replay": [vp, i, C.POINTER(C.c_int), C.POINTER(f)],
+        "zl_wait_selftest": [C.POINTER(C.c_uint)],
     }
     for name, args in sig.items():
         fn = getattr(lib, name)
@@ -221,6 +224,21 @@ def _need(t, dtypes, what):
         raise TypeError(f"{what}: dtype {t.dtype}, expected {dtypes}")
 
 
+def _need_numel(t, n: int, what: str) -> None:
+    """Raise ZLError(ZL_ERR_ARG) when a tensor argument holds fewer than n elements."""
+    if t is not None and not isinstance(t, int) and t.numel() < n:
+        raise ZLError(ZL_ERR_ARG, f"{what}: {t.numel()} elements, the call reads or writes {n}")
+
+
+def _loss_sizes(z, t, labels, dz, N: int, ldz: int, loss, row_loss=None) -> None:
+    if N >= 1 and ldz >= 1:
+        for x, nm in ((z, "z"), (t, "t"), (dz, "dz")):
+            _need_numel(x, N * ldz, nm)
+        _need_numel(labels, N, "labels")
+        _need_numel(row_loss, N, "row_loss")
+        _need_numel(loss, 1, "loss")
+
+
 def zl_op_local_loss(dtype: int, z, t, labels, N: int, V: int, ldz: int, alpha: float, kl_dir: int, dz, row_loss,
                      loss, stream: int = 0) -> None:
     act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
@@ -229,6 +247,7 @@ def zl_op_local_loss(dtype: int, z, t, labels, N: int, V: int, ldz: int, alpha: 
     _need(labels, ("int32",), "labels")
     _need(row_loss, ("float32",), "row_loss")
     _need(loss, ("float32",), "loss")
+    _loss_sizes(z, t, labels, dz, N, ldz, loss, row_loss)
     _check(_lib.zl_op_local_loss(dtype, _p(z), _p(t), _p(labels), N, V, ldz, alpha, kl_dir, _p(dz), _p(row_loss),
                                  _p(loss), stream))
 
@@ -241,6 +260,8 @@ def zl_op_local_loss_noalloc(dtype: int, z, t, labels, N: int, V: int, ldz: int,
         _need(x, act, nm)
     _need(labels, ("int32",), "labels")
     _need(loss, ("float32",), "loss")
+    if N <= ZL_NOALLOC_MAX_ROWS:   # larger N is the library's own error (beyond its scratch)
+        _loss_sizes(z, t, labels, dz, N, ldz, loss)
     _check(_lib.zl_op_local_loss_noalloc(dtype, _p(z), _p(t), _p(labels), N, V, ldz, alpha, kl_dir, _p(dz),
                                          _p(loss), stream))
 
@@ -319,6 +340,13 @@ def zl_replay(ctx, k: int):
     return n.value, loss.value
 
 
+def zl_wait_selftest() -> int:
+    """Runs the bounded-wait self-test (seconds); returns the kernel's device error bits."""
+    bits = C.c_uint()
+    _check(_lib.zl_wait_selftest(C.byref(bits)))
+    return bits.value
+
+
 # ---- convenience object ----------------------------------------------------------------------
 class ZeroLock:
     """One engine context: a model cut into K chunks, its AdamW state and K CUDA streams."""
@@ -328,7 +356,7 @@ class ZeroLock:
                  beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.01, accum_m: int = 1,
                  max_live_chunks: int = 0, lr_schedule: int = 0, lr_gamma: float = 1.0, serialize: bool = False,
                  lora_rank: int = 0, lora_scale: float = 1.0, replay_depth: int = 0, adapter_dim: int = 0,
-                 graph: bool = False, stream=None):
+                 graph: bool = False, fuzz_delay_us: int = 0, fuzz_seed: int = 0, stream=None):
         import torch
         self.dims = dims
         self.K = K
@@ -338,7 +366,7 @@ class ZeroLock:
                            dims.norm_eps, dims.rope_theta)
         cfg = zl_train_cfg(alpha, kl_dir, consis_first, lr, beta1, beta2, eps, weight_decay, accum_m,
                            max_live_chunks, lr_schedule, lr_gamma, int(serialize), lora_rank, lora_scale,
-                           replay_depth, adapter_dim, int(graph))
+                           replay_depth, adapter_dim, int(graph), fuzz_delay_us, fuzz_seed)
         self.ctx = zl_create(md, K, list(bounds), cfg)
         s = stream if stream is not None else torch.cuda.current_stream()
         zl_set_stream(self.ctx, s.cuda_stream)

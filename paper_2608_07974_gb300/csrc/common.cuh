@@ -8,12 +8,9 @@
 
 typedef __nv_bfloat16 bf16;
 
-// Device-side error bits, OR-ed into the context's error word and reported by zl_synchronize.
-enum : unsigned {
-  ZL_DEVERR_BAD_ID = 1u,       // a token id outside [0, vocab)
-  ZL_DEVERR_BAD_LABEL = 2u,    // a label outside [-1, vocab)
-  ZL_DEVERR_TIMEOUT = 4u,      // a bounded wait inside a kernel gave up
-};
+// Device-side error bits (ZL_DEVERR_*, declared with the C ABI), OR-ed into the context's error word
+// and reported by zl_synchronize.
+#include "zerolock.h"
 
 __device__ __forceinline__ float to_f(float x) { return x; }
 __device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }

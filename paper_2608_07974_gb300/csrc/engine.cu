@@ -169,6 +169,7 @@ struct zl_ctx {
   } zg, bg;
   bool capturing = false;
   cudaStream_t cap = nullptr;   // capture origin (the user's stream may be the uncapturable legacy stream)
+  uint64_t fuzz_state = 0;      // scheduler fuzz stream (cfg.fuzz_seed)
 };
 
 namespace {
@@ -231,14 +232,28 @@ const void* TrainC(zl_ctx* c, Chunk& k, size_t off) {
 
 size_t esz(zl_ctx* c) { return dt_size(c->dt); }
 
+// Scheduler fuzz (cfg.fuzz_delay_us > 0): the host sleeps a pseudo-random 0..fuzz_delay_us microseconds,
+// drawn from a SplitMix64 stream seeded by cfg.fuzz_seed, so the GPU runs ahead of the enqueues in
+// varying interleavings. Only the timing changes; every dependency is an event or stream order.
+void fuzz_pause(zl_ctx* c) {
+  if (c->cfg.fuzz_delay_us <= 0) return;
+  uint64_t z = (c->fuzz_state += 0x9E3779B97F4A7C15ull);
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  z ^= z >> 31;
+  std::this_thread::sleep_for(std::chrono::microseconds(z % (uint64_t)(c->cfg.fuzz_delay_us + 1)));
+}
+
 // Consecutive host-side NVTX ranges over the phases a call enqueues, named by chunk and phase, so a
 // profiler can select one chunk's or one phase's kernels (ncu --nvtx --nvtx-include "zl chunk 2 loss/").
-// Without an attached tool each range is a cheap no-op.
+// Without an attached tool each range is a cheap no-op. Each phase boundary is also a fuzz point.
 class NvtxPhases {
  public:
+  explicit NvtxPhases(zl_ctx* c) : c_(c) {}
   ~NvtxPhases() { end(); }
   void next(const char* fmt, int k = 0) {
     end();
+    fuzz_pause(c_);
     char name[64];
     std::snprintf(name, sizeof name, fmt, k);
     nvtxRangePushA(name);
@@ -250,6 +265,7 @@ class NvtxPhases {
   }
 
  private:
+  zl_ctx* c_;
   bool open_ = false;
 };
 
@@ -980,6 +996,7 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (cfg->lora_rank < 0 || cfg->lora_rank > 256) why = "lora_rank must be in [0, 256]";
   else if (cfg->replay_depth < 0 || cfg->replay_depth > 4096) why = "replay_depth must be in [0, 4096]";
   else if (cfg->lora_rank > 0 && !(std::isfinite(cfg->lora_scale))) why = "lora_scale must be finite";
+  else if (cfg->fuzz_delay_us < 0 || cfg->fuzz_delay_us > 100000) why = "fuzz_delay_us must be in [0, 100000]";
   for (int k = 1; why.empty() && k <= K; ++k)
     if (bounds[k] <= bounds[k - 1]) why = "bounds must be strictly increasing";
   if (!why.empty()) { g_err = "zl_create: " + why; return ZL_ERR_ARG; }
@@ -988,6 +1005,7 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   zl_status st = guarded(nullptr, [&]() -> zl_status {
     c->dims = D;
     c->cfg = *cfg;
+    c->fuzz_state = (uint64_t)cfg->fuzz_seed * 0x9E3779B97F4A7C15ull;
     c->K = K;
     c->bounds.assign(bounds, bounds + K + 1);
     c->dt = D.dtype;
@@ -1296,7 +1314,7 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
   cudaStream_t s = ck.s;
   const int N = B * S;
   const size_t hb = (size_t)N * c->d * esz(c), zb = (size_t)N * c->Vp * esz(c);
-  NvtxPhases ph;
+  NvtxPhases ph(c);
   ph.next("zl chunk %d forward", k);
   void* h0 = nullptr;
   if (!h_in) {
@@ -1549,7 +1567,7 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
   rec(c->ev_start, c->user);
   for (int k = 1; k <= K; ++k) wait_ev(c->ch[k].s, c->ev_start);
   wait_ev(c->aux, c->ev_start);
-  NvtxPhases ph;
+  NvtxPhases ph(c);
   ph.next("zl step embedding and teacher");
   std::vector<void*> h(K + 1, nullptr), z(K + 1, nullptr);
   // h_0 = E(x) on s_1; the teacher of chunk 1, z_0 = readout(h_0), on the auxiliary stream
@@ -1693,7 +1711,7 @@ void bp_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int
       rec(c->ch[k].ev_done, c->ch[k].s);
       wait_ev(s, c->ch[k].ev_done);
     }
-  NvtxPhases ph;
+  NvtxPhases ph(c);
   ph.next("zl bp forward");
   std::vector<void*> h(K + 1, nullptr);
   std::vector<ChunkActs> acts(K + 1);

@@ -965,13 +965,8 @@ void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labe
   // being read still fit in L2 for the second pass. Three rows per SM (40 registers) where the rows in
   // flight on every SM stay well inside L2 (V = 32000: 58 MB), two otherwise (V = 50257: three would
   // hold 92 MB, and pass 2 would go back to DRAM: 293 against 260 us at 4096 rows).
-  int cap = 512;
-  if (const char* e = std::getenv("ZL_LOSS_THREADS")) {   // tuning override
-    const int v = std::atoi(e);
-    if (v == 128 || v == 256 || v == 512) cap = v;
-  }
   int th = 32;
-  while (th < cap && th * 8 < ldz) th *= 2;
+  while (th < 512 && th * 8 < ldz) th *= 2;
   const size_t row_bytes = (size_t)ldz * dt_size(dt) * (t ? 2 : 1);
   const bool three = dt == BF16 && 3ull * 152 * row_bytes <= (64ull << 20);
 #define LL2(T, TE, KD)                                                                                            \

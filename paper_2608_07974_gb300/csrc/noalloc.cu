@@ -8,10 +8,12 @@
 // input and output.
 //
 // The array is a host-side stand-in in host code, not a device address: the address handed to
-// the kernels comes from cudaGetSymbolAddress, taken once per device with that device current,
-// by the first call of this entry point on that device. Every call shares the array, so calls
-// whose work overlaps on the GPU race on it; the error word is cleared on each call, the other
-// scratch entries are fully rewritten.
+// the kernels comes from cudaGetSymbolAddress, looked up with the device current by the first call
+// in each CUDA context (the cache is keyed on the context's process-unique id, so a context created
+// after cudaDeviceReset, or a caller's own context, gets its own lookup). Every call shares the
+// array, so calls whose work overlaps on the GPU race on it; |Omega| and the error word are written
+// before they are read on each call, the per-row losses are fully rewritten.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -29,8 +31,36 @@ constexpr int kErrSlot = kMaxRows + 64;     // device-side argument error bits
 static __device__ __align__(256) float g_scratch[kMaxRows + 128];
 
 std::mutex g_mu;
-constexpr int kMaxDevices = 64;
-void* g_addr[kMaxDevices] = {};
+struct CtxAddr {
+  unsigned long long ctx_id;
+  void* addr;
+};
+constexpr int kMaxContexts = 64;
+CtxAddr g_addr[kMaxContexts];
+int g_naddr = 0;
+
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+template <typename F>
+F driver_fn(const char* name) {
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess)
+    return nullptr;
+  return reinterpret_cast<F>(fn);
+}
+
+// Id of the calling thread's current CUDA context (0 if there is none or it cannot be read).
+unsigned long long current_ctx_id() {
+  static CtxGetCurrentFn get_cur = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+  static CtxGetIdFn get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+  CUcontext cx = nullptr;
+  unsigned long long id = 0;
+  if (!get_cur || !get_id || get_cur(&cx) != CUDA_SUCCESS || !cx || get_id(cx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
 
 zl_status fail(zl_status st, const std::string& m) {
   zl::set_last_error(m);
@@ -50,21 +80,22 @@ extern "C" zl_status zl_op_local_loss_noalloc(int dtype, const void* z, const vo
                                 std::to_string(kMaxRows) + " rows");
   if (!(alpha > 0.f && alpha <= 1.f) || (alpha < 1.f && !t) || (kl_dir != 0 && kl_dir != 1))
     return fail(ZL_ERR_ARG, "alpha in (0,1], t required when alpha < 1, kl_dir 0/1");
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return fail(ZL_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
-  if (dev < 0 || dev >= kMaxDevices) return fail(ZL_ERR_UNSUPPORTED, "device index beyond 63");
   float* base = nullptr;
+  cudaError_t e = cudaSuccess;
   {
     std::lock_guard<std::mutex> lk(g_mu);
-    if (!g_addr[dev]) {   // once per device, with that device current
+    const unsigned long long id = current_ctx_id();
+    for (int i = 0; id && i < g_naddr; ++i)
+      if (g_addr[i].ctx_id == id) base = static_cast<float*>(g_addr[i].addr);
+    if (!base) {   // first call in this context: look the array up with the device current
       void* p = nullptr;
       e = cudaGetSymbolAddress(&p, g_scratch);
       if (e != cudaSuccess || !p)
         return fail(ZL_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
-      g_addr[dev] = p;
+      base = static_cast<float*>(p);
+      const unsigned long long id2 = current_ctx_id();   // the lookup may have made the context current
+      if (id2 && g_naddr < kMaxContexts) g_addr[g_naddr++] = CtxAddr{id2, p};
     }
-    base = static_cast<float*>(g_addr[dev]);
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   float* row_loss = base;

@@ -1,12 +1,13 @@
 """Single-kernel timings through the C ABI (CUDA events, after warm-up), for tuning and profiling.
 
     python -m paper_2608_07974_gb300.microbench loss [--rows 1024] [--vocab 50257] [--reps 4]
-    python -m paper_2608_07974_gb300.microbench gemm [--sweep] [--workload gpt2|llama-1b]
+    python -m paper_2608_07974_gb300.microbench gemm [--workload gpt2|llama-1b]
     python -m paper_2608_07974_gb300.microbench attention [--batch 8 --seq 512 --heads 12 --kv-heads 12 --head-dim 64]
 
 `loss` runs the fused local objective on random bf16 logits; `gemm` times the GEMM shapes of the
 GPT-2-small workload (12 layers, d 768, FFN 3072, vocab 50304 padded, 4096 tokens) or of the
-Llama-style 1.1B one, with --sweep every tile width / split-K count; `attention` the causal attention forward and backward.
+Llama-style 1.1B one, each with the tile width and split-K count the library's planner picks;
+`attention` the causal attention forward and backward.
 """
 from __future__ import annotations
 
@@ -75,7 +76,6 @@ LLAMA1B_SHAPES = _shapes_of(2048, 2560, 11264, 5632, 32000)
 
 def gemm(args):
     B = _lib()
-    tiles = ["auto"] + ([f"{bn}:{s}" for bn in (64, 128, 256) for s in (1, 2, 3, 4, 6)] if args.sweep else [])
     shapes = {"gpt2": GPT2_SHAPES, "llama-1b": LLAMA1B_SHAPES}[args.workload]
     for name, mode, M, N, K in shapes:
         bf = torch.bfloat16
@@ -86,19 +86,9 @@ def gemm(args):
         else:
             a, b = torch.randn(K, M, device="cuda").to(bf), torch.randn(K, N, device="cuda").to(bf)
         c = torch.zeros(M, N, device="cuda", dtype=torch.float32 if mode == 2 else bf)
-        res = []
-        for t in tiles:
-            if t == "auto":
-                os.environ.pop("ZL_GEMM_TILE", None)
-            else:
-                os.environ["ZL_GEMM_TILE"] = t
-            ms = _time(lambda: B.zl_op_gemm(1, mode, M, N, K, a, b, c), args.reps)
-            res.append((t, ms))
-        os.environ.pop("ZL_GEMM_TILE", None)
-        line = f"{name:9s} M={M:5d} N={N:6d} K={K:6d} auto {res[0][1] * 1e3:7.1f} us {2 * M * N * K / res[0][1] / 1e9:7.1f} TFLOP/s"
-        if args.sweep:
-            line += " | " + " ".join(f"{t}={ms * 1e3:.1f}" for t, ms in res[1:])
-        print(line, flush=True)
+        ms = _time(lambda: B.zl_op_gemm(1, mode, M, N, K, a, b, c), args.reps)
+        print(f"{name:9s} M={M:5d} N={N:6d} K={K:6d} {ms * 1e3:7.1f} us {2 * M * N * K / ms / 1e9:7.1f} TFLOP/s",
+              flush=True)
 
 
 def attention(args):
@@ -126,7 +116,6 @@ def main():
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--reps", type=int, default=4)
     p = sub.add_parser("gemm")
-    p.add_argument("--sweep", action="store_true")
     p.add_argument("--workload", choices=["gpt2", "llama-1b"], default="gpt2")
     p.add_argument("--reps", type=int, default=20)
     p = sub.add_parser("attention")

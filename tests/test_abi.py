@@ -75,7 +75,7 @@ def test_binding_structs_match_the_header_layout(name):
     """The ctypes structures list the header's fields in the header's order, with C int / float types
     matching the declarations (a drift here would shift every later field across the ABI)."""
     from paper_2608_07974_gb300 import binding
-    want = {"int": ctypes.c_int, "float": ctypes.c_float}
+    want = {"int": ctypes.c_int, "float": ctypes.c_float, "unsigned": ctypes.c_uint}
     fields = _header_struct_fields(name)
     st = getattr(binding, name)
     assert [f for f, _ in st._fields_] == [f for f, _ in fields]
@@ -194,3 +194,30 @@ def test_single_kernel_entry_points_reject_bad_arguments_on_the_host():
         assert getattr(L, name)(None, P, P, 1, 1, None) == b.ZL_ERR_ARG, name
     assert L.zl_synchronize(None, 0) == b.ZL_ERR_ARG
     L.zl_free(None)   # NULL-safe
+
+
+def test_loss_bindings_reject_undersized_tensors_before_the_call():
+    """The loss bindings check every tensor against the sizes the call reads or writes (N * ldz for z,
+    t and dz; N for labels and per-row losses) and raise before any pointer reaches the library (CPU
+    tensors stand in: a wrongly accepted call would fail on the host pointers, not pass)."""
+    import torch
+    from paper_2608_07974_gb300 import binding as b
+    N, V, ldz = 4, 8, 8
+    z, dz = torch.zeros(N * ldz), torch.zeros(N * ldz)
+    lab, rl, loss = torch.zeros(N, dtype=torch.int32), torch.zeros(N), torch.zeros(1)
+    short = torch.zeros(N * ldz - 1)
+    cases = [dict(z=short), dict(dz=short), dict(t=short), dict(labels=torch.zeros(N - 1, dtype=torch.int32)),
+             dict(row_loss=torch.zeros(N - 1)), dict(loss=torch.zeros(0))]
+    for bad in cases:
+        a = dict(z=z, t=None, labels=lab, dz=dz, row_loss=rl, loss=loss)
+        a.update(bad)
+        alpha = 0.5 if "t" in bad else 1.0
+        with pytest.raises(b.ZLError) as e:
+            b.zl_op_local_loss(b.ZL_DTYPE_F32, a["z"], a["t"], a["labels"], N, V, ldz, alpha, 0, a["dz"],
+                               a["row_loss"], a["loss"])
+        assert e.value.status == b.ZL_ERR_ARG, bad
+        if "row_loss" not in bad:
+            with pytest.raises(b.ZLError) as e:
+                b.zl_op_local_loss_noalloc(b.ZL_DTYPE_F32, a["z"], a["t"], a["labels"], N, V, ldz, alpha, 0, a["dz"],
+                                           a["loss"])
+            assert e.value.status == b.ZL_ERR_ARG, bad

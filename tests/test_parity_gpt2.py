@@ -96,3 +96,52 @@ def test_zerolock_peak_memory_below_backprop():
         peaks[mode] = eng.peak_bytes()[0]
         eng.close()
     assert peaks["zl"] < peaks["bp"], peaks
+
+
+def _reanchored_oracle(eng, P, names):
+    """The oracle (fp32) at the engine's current weights: its fp32 masters rounded to bf16, the values its
+    bf16 compute copy must hold after the optimizer step (frozen tensors as loaded)."""
+    Q = dict(P)
+    for n in names:
+        Q[n] = synth.round_bf16(eng.get(n, 0).view(P[n].shape)) if P[n].dim() == 2 else eng.get(n, 0).view(P[n].shape)
+    return oracle_for(W, Q, dtype=torch.float32, accum_m=2)
+
+
+def test_full_model_three_steps_full_size():
+    """All K = 4 chunks at the full 8 x 512 micro-batch for three consecutive concurrent steps (accum_m = 2:
+    the second step ends the window and applies AdamW, the third starts the next window).
+
+    Losses of every chunk at every step are within 2e-2 of the oracle's own uninterrupted fp32 trajectory
+    (Eq. 1-6 from the same bf16-rounded start). The third step's gradients, read from the accumulator,
+    are checked (cosine >= 0.999) against the oracle at the engine's updated weights rounded to bf16,
+    which is what the bf16 compute copy refreshed by the optimizer step must hold. The update itself is
+    checked element-wise against the decoupled AdamW step written out from the engine's own moments."""
+    P = _params()
+    eng = engine_for(W, accum_m=2)
+    eng.load(P)
+    orc = oracle_for(W, P, dtype=torch.float32, accum_m=2)
+    names = [n for k in range(1, W.K + 1) for n in orc.chunk_names(k)]
+    batches = [synth.make_batch(W, s) for s in range(3)]
+    for s, (ids, labels) in enumerate(batches[:2]):
+        lg = eng.step(ids.cuda(), labels.cuda())
+        lo = orc.step(ids, labels)
+        for k in range(W.K):
+            assert rel(lg[k], lo[k]) <= LOSS_TOL, (s, k, lg, lo)
+    # the window's AdamW step (t = 1), element by element from the engine's own m and v
+    bc1, bc2 = 1.0 - W.beta1, 1.0 - W.beta2
+    for n in names:
+        th0 = P[n].reshape(-1).double()
+        m, v, th = (eng.get(n, i).double() for i in (2, 3, 0))
+        want = th0 * (1.0 - W.lr * W.weight_decay) - W.lr * (m / bc1) / (torch.sqrt(v / bc2) + W.eps)
+        assert float((th - want).abs().max()) <= 1e-6 * max(float(th0.abs().max()), 1.0), n
+    ref = _reanchored_oracle(eng, P, names)
+    ids, labels = batches[2]
+    lg = eng.step(ids.cuda(), labels.cuda())
+    lo = orc.step(ids, labels)
+    h = ref.embed(ids)
+    for k in range(1, W.K + 1):
+        assert rel(lg[k - 1], lo[k - 1]) <= LOSS_TOL, (2, k, lg, lo)
+        L, g, h = ref.local_grad(k, h, labels)
+        assert rel(lg[k - 1], L) <= LOSS_TOL, (k, lg, L)
+        _check_grads(eng, ref, g, ref.chunk_names(k))
+    eng.close()

@@ -7,6 +7,11 @@ Chunks are checked in isolation (input h_{k-1} taken from the engine), which is 
 method: chunk k's step depends on the rest of the model only through h_{k-1} (Lemma 3).
 For 3B and 7B the engine holds just the first chunk's layers (a K = 1 model over them): its
 input is h_0 and its teacher readout(h_0), the same computation as chunk 1 of the full model.
+
+Steps 1 and 2 of the optimizer: with accum_m = 2, micro-batch 1's gradient is read from the
+accumulator (step 1, at the loaded weights), micro-batch 2 ends the window (AdamW), and micro-batch
+3's gradient is read again (step 2) and checked against the oracle at the engine's updated weights
+rounded to bf16 (what the refreshed bf16 compute copy must hold), from the engine's own h_{k-1}.
 """
 import dataclasses
 import functools
@@ -87,3 +92,56 @@ def test_first_chunk_full_width(name):
     orc = oracle_for(sub, P, dtype=torch.float32)
     _check_chunk(eng, orc, 1, orc.embed(ids), labels, losses[0])
     eng.close()
+
+
+def _reanchored(w, eng, P, names, **kw):
+    Q = dict(P)
+    for n in names:
+        t = eng.get(n, 0).view(P[n].shape)
+        Q[n] = synth.round_bf16(t) if t.dim() == 2 else t
+    return oracle_for(w, Q, dtype=torch.float32, **kw)
+
+
+def _two_steps_of_chunk(w, P, K, k, **okw):
+    """Chunk k of a K-chunk engine over w, isolated, at optimizer steps 1 and 2 (module docstring)."""
+    eng = engine_for(w, K=K, accum_m=2)
+    eng.load(P)
+    orc = oracle_for(w, P, K=K, dtype=torch.float32, accum_m=2, **okw)
+    names = orc.chunk_names(k)
+    view = lambda t: t.float().cpu().view(w.batch, w.seq, -1)
+
+    def h_in(ids):
+        h = None
+        for j in range(1, k):
+            h = eng.forward_chunk(j, h, ids.cuda() if j == 1 else None, w.batch, w.seq)
+        return orc.embed(ids) if k == 1 else view(h)
+
+    for mb in range(3):
+        ids, labels = synth.make_batch(w, mb)
+        h = h_in(ids) if mb != 1 else None
+        losses = eng.step(ids.cuda(), labels.cuda())
+        if mb == 0:
+            _check_chunk(eng, orc, k, h, labels, losses[k - 1])
+        elif mb == 2:
+            ref = _reanchored(w, eng, P, names, K=K, **okw)
+            _check_chunk(eng, ref, k, h if k > 1 else ref.embed(ids), labels, losses[k - 1])
+    eng.close()
+
+
+@pytest.mark.parametrize("K", [1, 2, 4])
+def test_llama_1b_deepest_chunk_two_steps(K):
+    """The deepest (last) chunk of the 1.1B model split into K = 1, 2 or 4 chunks (22, 11 or 6 layers),
+    full micro-batch (4 x 1024), optimizer steps 1 and 2."""
+    w = synth.LLAMA_1B
+    P = _params("1b", w.dims.n_layers)
+    _two_steps_of_chunk(w, P, K, K)
+
+
+@pytest.mark.parametrize("name", ["3b", "7b"])
+def test_first_chunk_full_width_step_two(name):
+    """Chunk 1 of the 3B and 7B-shaped models (a K = 1 model over its layers) at optimizer steps 1 and 2."""
+    w = {"3b": synth.LLAMA_3B, "7b": synth.LLAMA_7B}[name]
+    nl = synth.chunk_bounds(w.dims.n_layers, w.K)[1]
+    sub = dataclasses.replace(w, dims=dataclasses.replace(w.dims, n_layers=nl), K=1)
+    P = _params(name, nl)
+    _two_steps_of_chunk(sub, P, 1, 1)

@@ -2,13 +2,14 @@
 
 Failures are made on the host (a chunk's state is thrown away and restored); nothing faults the
 GPU. Replaying a chunk from its buffered inputs must reproduce the uninterrupted run bit for bit,
-and the other chunks keep their state.
+and the other chunks keep their state; the recovered parameters also match the oracle's uninterrupted
+trajectory (fp64, Eq. 1-6) within the fp32 bar of 1e-4 (per-tensor Frobenius relative error).
 """
 import pytest
 import torch
 
 import synth
-from tests.gpu_common import engine_for
+from tests.gpu_common import engine_for, fro_rel, oracle_for
 
 pytestmark = pytest.mark.gpu
 W = synth.TINY
@@ -53,6 +54,12 @@ def test_failed_chunk_recovers_by_replay(accum_m):
         if not name.startswith("layers.1."):
             assert torch.equal(after[name], before[name]), name    # other chunks kept their state
     eng.close(); ref.close()
+    orc = oracle_for(W, synth.make_params(W.dims, W.seed), K=4, bounds=BOUNDS, accum_m=accum_m)
+    for s in range(7):                                 # the uninterrupted run, by the oracle
+        ids, labels = synth.make_batch(W, s)
+        orc.step(ids, labels)
+    for name in want:
+        assert fro_rel(after[name], orc.P[name]) <= 1e-4, name
 
 
 def test_checkpoint_round_trip_and_rejections():
