@@ -91,6 +91,10 @@ typedef struct {
   int graph;                /* 1: zl_step / zl_bp_step are captured as a CUDA graph once per micro-batch */
                             /*   shape (after one eager call at that shape) and replayed; taken only    */
                             /*   with accum_m = 1, replay_depth = 0 and profiling off (else eager)      */
+  int unfused_update;       /* 0: at a window's last micro-batch the weight-gradient products of the    */
+                            /*   chunk's matrices apply AdamW in their epilogue (no gradient stored), the */
+                            /*   other trainable tensors get AdamW after the backward; 1: one AdamW over */
+                            /*   the whole slab after the backward. Same results either way.            */
   int fuzz_delay_us;        /* scheduler fuzz (tests): > 0 sleeps the host a pseudo-random 0..this many  */
   unsigned fuzz_seed;       /*   microseconds (SplitMix64 stream of fuzz_seed) at every phase boundary of */
                             /*   an enqueue, so the GPU runs ahead in varying interleavings; 0 is off,   */

@@ -39,7 +39,8 @@ class zl_train_cfg(C.Structure):
                 ("accum_m", C.c_int), ("max_live_chunks", C.c_int), ("lr_schedule", C.c_int),
                 ("lr_gamma", C.c_float), ("serialize", C.c_int), ("lora_rank", C.c_int),
                 ("lora_scale", C.c_float), ("replay_depth", C.c_int), ("adapter_dim", C.c_int),
-                ("graph", C.c_int), ("fuzz_delay_us", C.c_int), ("fuzz_seed", C.c_uint)]
+                ("graph", C.c_int), ("unfused_update", C.c_int), ("fuzz_delay_us", C.c_int),
+                ("fuzz_seed", C.c_uint)]
 
 
 class ZLError(RuntimeError):
@@ -356,17 +357,19 @@ class ZeroLock:
                  beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.01, accum_m: int = 1,
                  max_live_chunks: int = 0, lr_schedule: int = 0, lr_gamma: float = 1.0, serialize: bool = False,
                  lora_rank: int = 0, lora_scale: float = 1.0, replay_depth: int = 0, adapter_dim: int = 0,
-                 graph: bool = False, fuzz_delay_us: int = 0, fuzz_seed: int = 0, stream=None):
+                 graph: bool = False, unfused_update: bool = False, fuzz_delay_us: int = 0, fuzz_seed: int = 0,
+                 stream=None):
         import torch
         self.dims = dims
         self.K = K
         self.dtype = dtype
+        self.adapter_dim = adapter_dim
         md = zl_model_dims(dims.arch, ZL_DTYPE_BF16 if dtype == "bf16" else ZL_DTYPE_F32, dims.n_layers,
                            dims.d_model, dims.n_heads, dims.n_kv_heads, dims.d_ff, dims.vocab, dims.max_seq,
                            dims.norm_eps, dims.rope_theta)
         cfg = zl_train_cfg(alpha, kl_dir, consis_first, lr, beta1, beta2, eps, weight_decay, accum_m,
                            max_live_chunks, lr_schedule, lr_gamma, int(serialize), lora_rank, lora_scale,
-                           replay_depth, adapter_dim, int(graph), fuzz_delay_us, fuzz_seed)
+                           replay_depth, adapter_dim, int(graph), int(unfused_update), fuzz_delay_us, fuzz_seed)
         self.ctx = zl_create(md, K, list(bounds), cfg)
         s = stream if stream is not None else torch.cuda.current_stream()
         zl_set_stream(self.ctx, s.cuda_stream)

@@ -146,3 +146,32 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
+
+// The decoupled AdamW step of one parameter (Eq. 6, as AdamW): m <- b1 m + (1 - b1) g;
+// v <- b2 v + (1 - b2) g^2; theta <- theta (1 - lr wd) - lr (m / bc1) / (sqrt(v / bc2) + eps), with
+// bc1 = 1 - b1^t, bc2 = 1 - b2^t. Every operation is an explicitly rounded intrinsic, so every kernel
+// that applies the step (the slab and range updates, the weight-gradient GEMM's fused epilogue, the
+// split-K reduction) computes the same bits from the same gradient.
+struct AdamHP {
+  float lr, decay, bc1, bc2, b1, omb1, b2, omb2, eps;
+};
+// hp = {lr_t, 1 - b1^t, 1 - b2^t} as written by the step-count kernel.
+__device__ __forceinline__ AdamHP adam_hp(const float* hp, float b1, float b2, float eps, float wd) {
+  AdamHP h;
+  h.lr = hp[0];
+  h.bc1 = hp[1];
+  h.bc2 = hp[2];
+  h.decay = __fsub_rn(1.f, __fmul_rn(h.lr, wd));
+  h.b1 = b1;
+  h.omb1 = __fsub_rn(1.f, b1);
+  h.b2 = b2;
+  h.omb2 = __fsub_rn(1.f, b2);
+  h.eps = eps;
+  return h;
+}
+__device__ __forceinline__ void adamw_elem(float& th, float& m, float& v, float g, const AdamHP& h) {
+  m = __fadd_rn(__fmul_rn(h.b1, m), __fmul_rn(h.omb1, g));
+  v = __fadd_rn(__fmul_rn(h.b2, v), __fmul_rn(__fmul_rn(h.omb2, g), g));
+  const float den = __fadd_rn(__fsqrt_rn(__fdiv_rn(v, h.bc2)), h.eps);
+  th = __fsub_rn(__fmul_rn(th, h.decay), __fdiv_rn(__fmul_rn(h.lr, __fdiv_rn(m, h.bc1)), den));
+}

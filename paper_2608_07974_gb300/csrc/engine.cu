@@ -30,9 +30,9 @@ namespace {
 using namespace zl;
 
 // Kernel classes of the per-launch profile (zl_profile).
-enum { PC_GEMM, PC_GEMM_HEAD, PC_ATTN_F, PC_ATTN_B, PC_LOSS, PC_NORM, PC_ADAMW, PC_ELEM, PC_COUNT };
-const char* kPCName[PC_COUNT] = {"gemm_layer", "gemm_head", "attn_fwd", "attn_bwd", "local_loss", "norm", "adamw",
-                                 "elementwise"};
+enum { PC_GEMM, PC_GEMM_HEAD, PC_GEMM_UPD, PC_ATTN_F, PC_ATTN_B, PC_LOSS, PC_NORM, PC_ADAMW, PC_ELEM, PC_COUNT };
+const char* kPCName[PC_COUNT] = {"gemm_layer", "gemm_head", "gemm_update", "attn_fwd", "attn_bwd", "local_loss",
+                                 "norm", "adamw", "elementwise"};
 struct ProfRec {
   int cls;
   cudaEvent_t a, b;
@@ -102,6 +102,14 @@ struct Chunk {
   long long* d_t = nullptr;  // optimizer steps on the device, advanced by the AdamW launch
   float* d_hp = nullptr;     // this step's lr and bias corrections (written on the device)
   long done = 0;             // micro-batches this chunk has processed (progress metadata)
+  // Fused update: at a window's last micro-batch the weight-gradient products of the chunk's matrices
+  // apply the optimizer step in their epilogue; the other trainable ranges (norm gains, biases, readout
+  // adapter) get a range update after the backward.
+  bool fuse = false;          // this micro-batch's backward updates the matrices in place
+  long long* d_ranges = nullptr;   // device (offset, length) pairs of the non-matrix trainable ranges
+  std::vector<long long> h_ranges; // the same on the host
+  int n_ranges = 0, n_ranges_layers = 0;   // all of them / those before the readout adapter
+  size_t max_range = 0;
   // hidden-state buffer (Section III-B-3): the last replay_depth inputs h_{k-1} with their labels
   struct Entry {
     long seq = -1;
@@ -320,6 +328,34 @@ void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, 
   ProfScope p(c, s, head ? PC_GEMM_HEAD : PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
   gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool, alpha);
 }
+// Weight gradient of matrix p of layer li: C += A^T B into its gradient accumulator, or, when this
+// micro-batch ends the update window with the fused update on (k.fuse), the AdamW step of the matrix in
+// the product's epilogue (the accumulator is read if earlier micro-batches of the window filled it, and
+// left at zero). Where the tensor-core product does not apply (fp32, or a shape outside its rules) the
+// gradient is formed with gemm() and the step applied to the matrix's range right after it: the same
+// arithmetic either way.
+void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, const void* A, const void* B) {
+  float* g = Gm(k, li, p);
+  if (!g) return;   // frozen
+  if (!k.fuse) {
+    G(c, s, 2, M, N, K, A, B, g, nullptr, nullptr);
+    return;
+  }
+  const zl_train_cfg& cf = c->cfg;
+  const size_t off = k.layers[li].off[p];
+  const GemmUpdate u{k.master + off, k.m + off, k.v + off, cf.accum_m > 1 ? g : nullptr,
+                     c->dt == BF16 ? (void*)((bf16*)k.comp + off) : nullptr, k.d_hp, cf.beta1, cf.beta2, cf.eps,
+                     cf.weight_decay, 1.f / (float)cf.accum_m};
+  const double e = (double)esz(c), mn = (double)M * N;
+  // operands, then read theta, m, v (and g) and write them back (g zeroed), plus the compute copy
+  const double upd = (cf.accum_m > 1 ? 32.0 : 24.0) * mn + (c->dt == BF16 ? 2.0 : 0.0) * mn;
+  ProfScope ps(c, s, PC_GEMM_UPD, 2.0 * mn * (double)K, e * ((double)M * K + (double)N * K) + upd);
+  if (c->dt == BF16 && gemm_tc_update(M, N, K, A, B, u, c->d_err, s, c->pool)) return;
+  gemm(c->dt, 2, M, N, K, A, B, g, nullptr, nullptr, s, c->d_err, c->pool);
+  launch_adamw_span(u.theta, g, u.m, u.v, u.comp, (size_t)M * N, k.d_hp, cf.beta1, cf.beta2, cf.eps, cf.weight_decay,
+                    u.gscale, s);
+}
+
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
   const double e = (double)esz(c), N = (double)B * S;
   ProfScope p(c, s, PC_ATTN_F, 2.0 * B * c->H * (double)S * S * c->hd, e * N * (c->qkvw + c->ad));
@@ -526,39 +562,41 @@ void layer_bwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* dy, void*
   const int N = B * S, dt = c->dt;
   // the layer above queued sums over dy's buffer, dhid, dx2 and dqkv, which this layer overwrites
   q.need(k.ev_layer, q.layer);
+  // Every dX product comes before the weight-gradient product of the same matrix, which may update the
+  // matrix in place (fused update).
   // FFN
-  G(c, s, 2, c->d, c->f, N, dy, sv.act, Gm(k, li, P_W2), nullptr, nullptr);
-  bias_grad(c, dy, N, c->d, Gm(k, li, P_B2), w, q);
   G(c, s, 1, N, c->f, c->d, dy, Wc(c, k, li, P_W2), w.da, nullptr, nullptr);
+  GW(c, s, k, li, P_W2, c->d, c->f, N, dy, sv.act);
+  bias_grad(c, dy, N, c->d, Gm(k, li, P_B2), w, q);
   lora_bwd(c, k, li, 3, sv.act, sv.u[3], dy, w.da, w.du, N, s);
   {
     ProfScope p(c, s, PC_ELEM, 0, esz(c) * (double)N * (2.0 * c->f1 + c->f));
     if (c->llama) launch_swiglu_bwd(dt, sv.hid, w.da, w.dhid, N, c->f, s);
     else launch_gelu_bwd(dt, sv.hid, w.da, w.dhid, (size_t)N * c->f, s);
   }
-  G(c, s, 2, c->f1, c->d, N, w.dhid, sv.xn2, Gm(k, li, P_W1), nullptr, nullptr);
-  bias_grad(c, w.dhid, N, c->f1, Gm(k, li, P_B1), w, q);
   q.need(k.ev_ln1, q.ln1);   // the layer above's LN1 parameter sums read dxn
   G(c, s, 1, N, c->d, c->f1, w.dhid, Wc(c, k, li, P_W1), w.dxn, nullptr, nullptr);
+  GW(c, s, k, li, P_W1, c->f1, c->d, N, w.dhid, sv.xn2);
+  bias_grad(c, w.dhid, N, c->f1, Gm(k, li, P_B1), w, q);
   lora_bwd(c, k, li, 2, sv.xn2, sv.u[2], w.dhid, w.dxn, w.du, N, s);
   NBX(c, s, sv.x2, Wm(k, li, P_N2W), sv.rstd2, sv.mean2, w.dxn, dy, w.dx2, N);
   norm_param_grad(c, sv.x2, sv.rstd2, sv.mean2, w.dxn, N, Gm(k, li, P_N2W), Gm(k, li, P_N2B), w, q);
   q.ln2 = q.mark(k.ev_ln2);
   // attention
-  G(c, s, 2, c->d, c->ad, N, w.dx2, sv.att, Gm(k, li, P_WO), nullptr, nullptr);
-  bias_grad(c, w.dx2, N, c->d, Gm(k, li, P_BO), w, q);
   G(c, s, 1, N, c->ad, c->d, w.dx2, Wc(c, k, li, P_WO), w.datt, nullptr, nullptr);
+  GW(c, s, k, li, P_WO, c->d, c->ad, N, w.dx2, sv.att);
+  bias_grad(c, w.dx2, N, c->d, Gm(k, li, P_BO), w, q);
   lora_bwd(c, k, li, 1, sv.att, sv.u[1], w.dx2, w.datt, w.du, N, s);
   AB(c, s, sv.qkv, sv.att, w.datt, sv.lse, w.D, w.dqkv, B, S);
   if (c->llama) {
     ProfScope p(c, s, PC_ELEM, 0, 2.0 * esz(c) * (double)N * (c->H + c->Hkv) * c->hd);
     launch_rope(dt, w.dqkv, c->rope_cs, N, S, c->H, c->Hkv, c->hd, 1, s);
   }
-  G(c, s, 2, c->qkvw, c->d, N, w.dqkv, sv.xn1, Gm(k, li, P_WQKV), nullptr, nullptr);
-  bias_grad(c, w.dqkv, N, c->qkvw, Gm(k, li, P_BQKV), w, q);
-  q.layer = q.mark(k.ev_layer);   // after this layer's sums over dy, dhid, dx2 and dqkv
   q.need(k.ev_ln2, q.ln2);        // LN2 parameter sums read dxn, which the next product overwrites
   G(c, s, 1, N, c->d, c->qkvw, w.dqkv, Wc(c, k, li, P_WQKV), w.dxn, nullptr, nullptr);
+  GW(c, s, k, li, P_WQKV, c->qkvw, c->d, N, w.dqkv, sv.xn1);
+  bias_grad(c, w.dqkv, N, c->qkvw, Gm(k, li, P_BQKV), w, q);
+  q.layer = q.mark(k.ev_layer);   // after this layer's sums over dy, dhid, dx2 and dqkv
   lora_bwd(c, k, li, 0, sv.xn1, sv.u[0], w.dqkv, w.dxn, w.du, N, s);
   norm_param_grad(c, sv.x, sv.rstd1, sv.mean1, w.dxn, N, Gm(k, li, P_N1W), Gm(k, li, P_N1B), w, q);
   q.ln1 = q.mark(k.ev_ln1);
@@ -636,19 +674,41 @@ void chunk_bwd(zl_ctx* c, Chunk& k, ChunkActs& acts, const void* dh, void* dh_in
   pfree(a.base, s);
 }
 
-// adapters = false (the backpropagation step): the readout adapter, at the end of the slab, is left as is.
+// Before the backward of one micro-batch of chunk k: when the micro-batch ends the update window and
+// the fused update applies (full fine-tune, cfg.unfused_update = 0), advance the step count and write
+// this step's lr and bias corrections now, so the weight-gradient products can apply the step.
+void window_begin(zl_ctx* c, Chunk& k, cudaStream_t s) {
+  const zl_train_cfg& g = c->cfg;
+  k.fuse = k.micro + 1 >= g.accum_m && !g.unfused_update && g.lora_rank == 0;
+  if (k.fuse) launch_adamw_tick(k.d_t, k.d_hp, g.lr, g.lr_schedule, g.lr_gamma, g.beta1, g.beta2, s);
+}
+
+// After the backward: at the window's end the AdamW step of whatever the backward did not update (all of
+// the slab, or, after a fused backward, its non-matrix ranges). adapters = false (the backpropagation
+// step): the readout adapter, at the end of the slab, is left as is.
 void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s, bool adapters = true) {
   k.micro += 1;
   if (k.micro < c->cfg.accum_m) return;
   k.t += 1;
   const zl_train_cfg& g = c->cfg;
-  const size_t n = (adapters || g.adapter_dim == 0) ? k.n : k.n_layers_slab;
   k.micro = 0;
+  const float gscale = 1.f / (float)g.accum_m;
+  if (k.fuse) {
+    const int nr = adapters ? k.n_ranges : k.n_ranges_layers;
+    double n = 0;
+    for (int i = 0; i < nr; ++i) n += (double)k.h_ranges[2 * i + 1];
+    ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * n);
+    launch_adamw_ranges(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, k.d_ranges, nr, k.max_range,
+                        k.d_hp, g.beta1, g.beta2, g.eps, g.weight_decay, gscale, s);
+    k.fuse = false;
+    CHECK_LAUNCH();
+    return;
+  }
+  const size_t n = (adapters || g.adapter_dim == 0) ? k.n : k.n_layers_slab;
   ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * (double)n);
   launch_adamw(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, n, k.d_t, k.d_hp, g.lr, g.lr_schedule,
-               g.lr_gamma, g.beta1, g.beta2, g.eps, g.weight_decay, 1.f / (float)g.accum_m, s);
+               g.lr_gamma, g.beta1, g.beta2, g.eps, g.weight_decay, gscale, s);
   CHECK_LAUNCH();
-  k.micro = 0;
 }
 
 float alpha_of(zl_ctx* c, int k) { return (k == 1 && !c->cfg.consis_first) ? 1.f : c->cfg.alpha; }
@@ -997,6 +1057,7 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (cfg->replay_depth < 0 || cfg->replay_depth > 4096) why = "replay_depth must be in [0, 4096]";
   else if (cfg->lora_rank > 0 && !(std::isfinite(cfg->lora_scale))) why = "lora_scale must be finite";
   else if (cfg->fuzz_delay_us < 0 || cfg->fuzz_delay_us > 100000) why = "fuzz_delay_us must be in [0, 100000]";
+  else if (cfg->unfused_update != 0 && cfg->unfused_update != 1) why = "unfused_update must be 0 or 1";
   for (int k = 1; why.empty() && k <= K; ++k)
     if (bounds[k] <= bounds[k - 1]) why = "bounds must be strictly increasing";
   if (!why.empty()) { g_err = "zl_create: " + why; return ZL_ERR_ARG; }
@@ -1127,6 +1188,30 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       ck.d_t = (long long*)salloc(c, 64);
       ck.d_hp = (float*)(ck.d_t + 1);
       CK(cudaMemset(ck.d_t, 0, 64));
+      // the trainable ranges a fused backward leaves to the range update: every vector of the layers,
+      // then the readout adapter (lengths rounded up to 4 inside the slab's 64-element padding)
+      if (r == 0) {
+        for (const Layer& L : ck.layers)
+          for (int p = 0; p < P_COUNT; ++p)
+            if (L.has[p] && L.slab[p] == S_TRAIN && p != P_WQKV && p != P_WO && p != P_W1 && p != P_W2) {
+              ck.h_ranges.push_back((long long)L.off[p]);
+              ck.h_ranges.push_back((long long)round_up(L.numel[p], 4));
+            }
+        ck.n_ranges_layers = (int)ck.h_ranges.size() / 2;
+        if (cfg->adapter_dim > 0)
+          for (size_t o : {ck.ad_down, ck.ad_up}) {
+            ck.h_ranges.push_back((long long)o);
+            ck.h_ranges.push_back((long long)round_up((size_t)cfg->adapter_dim * d, 4));
+          }
+        ck.n_ranges = (int)ck.h_ranges.size() / 2;
+        for (int i = 0; i < ck.n_ranges; ++i) ck.max_range = std::max(ck.max_range, (size_t)ck.h_ranges[2 * i + 1]);
+        if (ck.n_ranges > 65535) raise_err(ZL_ERR_UNSUPPORTED, "too many trainable vectors in one chunk");
+        if (ck.n_ranges > 0) {
+          ck.d_ranges = (long long*)salloc(c, ck.h_ranges.size() * sizeof(long long));
+          CK(cudaMemcpy(ck.d_ranges, ck.h_ranges.data(), ck.h_ranges.size() * sizeof(long long),
+                        cudaMemcpyHostToDevice));
+        }
+      }
       ck.master = (float*)salloc(c, ck.n * 4);
       ck.grad = (float*)salloc(c, ck.n * 4);
       ck.m = (float*)salloc(c, ck.n * 4);
@@ -1345,6 +1430,7 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
   void* dh = palloc(c, hb, s);
   readout_bwd(c, hk, rs, dz, dh, N, s, ad);
   pfree(dz, s);
+  window_begin(c, ck, s);
   chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
   pfree(dh, s);
   pfree(acts.mem, s);
@@ -1644,6 +1730,7 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
     readout_bwd(c, h[k], rs, dz, dh, N, s, adp ? &ck : nullptr);
     pfree(dz, s);
     rec(ck.ev_hb, s);
+    window_begin(c, ck, s);
     chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
     pfree(dh, s);
     pfree(acts.mem, s);
@@ -1733,6 +1820,7 @@ void bp_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int
   readout_bwd(c, h[K], rs, dz, dh, N, s);
   pfree(dz, s);
   for (int k = K; k >= 1; --k) {
+    window_begin(c, c->ch[k], s);
     chunk_bwd(c, c->ch[k], acts[k], dh, k > 1 ? dh2 : nullptr, B, S, s);
     std::swap(dh, dh2);
     pfree(acts[k].mem, s);

@@ -34,7 +34,8 @@ struct Cfg {
 };
 
 struct Args {
-  int M, N, K, mode;       // mode 0/1: bf16 C (+bias, +R); 2: fp32 C += acc; 3: fp32 store into split slice
+  int M, N, K, mode;       // mode 0/1: bf16 C (+bias, +R); 2: fp32 C += acc; 3: fp32 store into split slice;
+                           // 4: the AdamW step of the tensor in `u` with this tile as (the last part of) its gradient
   void* C;
   const float* bias;
   const bf16* R;
@@ -43,7 +44,50 @@ struct Args {
   int splits, kb_per_split;   // split-K: unit u -> split u / tiles, k blocks [s*kps, min(nk, (s+1)*kps))
   float alpha;                // scale of the product
   int rmode;                  // R in modes 0/1: 0 adds it (residual); 1 multiplies by GELU'(R) (R = the GELU input)
+  GemmUpdate u;               // mode 4
 };
+
+// Mode 4 on one accumulator row's columns [base, base + ncols) of the tensor (ncols <= 32, a multiple of
+// 4): G = gscale * (g + acc), then the AdamW step of each parameter (adamw_elem), written back to the
+// fp32 master, both moments and the bf16 compute copy; g (if any) is zeroed. 16 columns at a time, their
+// twelve (sixteen with g) 16-byte loads issued before any arithmetic.
+__device__ __forceinline__ void update_row32(const GemmUpdate& u, const AdamHP& h, size_t base, int ncols,
+                                             const float* acc) {
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    float4 th[4], mm[4], vv[4], gg[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int col = 16 * half + 4 * j;
+      if (col < ncols) {
+        th[j] = *reinterpret_cast<const float4*>(u.theta + base + col);
+        mm[j] = *reinterpret_cast<const float4*>(u.m + base + col);
+        vv[j] = *reinterpret_cast<const float4*>(u.v + base + col);
+        gg[j] = u.g ? *reinterpret_cast<const float4*>(u.g + base + col) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int col = 16 * half + 4 * j;
+      if (col < ncols) {
+        float* tp = &th[j].x; float* mp = &mm[j].x; float* vp = &vv[j].x; const float* gp = &gg[j].x;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float gsum = u.g ? __fadd_rn(gp[q], acc[col + q]) : acc[col + q];
+          adamw_elem(tp[q], mp[q], vp[q], __fmul_rn(gsum, u.gscale), h);
+        }
+        *reinterpret_cast<float4*>(u.theta + base + col) = th[j];
+        *reinterpret_cast<float4*>(u.m + base + col) = mm[j];
+        *reinterpret_cast<float4*>(u.v + base + col) = vv[j];
+        if (u.comp) {
+          __nv_bfloat162 c2[2] = {__floats2bfloat162_rn(tp[0], tp[1]), __floats2bfloat162_rn(tp[2], tp[3])};
+          *reinterpret_cast<uint2*>((bf16*)u.comp + base + col) = *reinterpret_cast<const uint2*>(c2);
+        }
+        if (u.g) *reinterpret_cast<float4*>(u.g + base + col) = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+  }
+}
 
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, operand majors, N, M.
 template <int BN, bool A_MN, bool B_MN>
@@ -191,6 +235,40 @@ __global__ void __launch_bounds__(kThreads, 1)
     // all MMAs issued by the leader complete before TMEM is released
     if (leader) mma_commit(fin);
     __syncwarp();
+  } else if (A_MN && B_MN && g.mode == 4) {
+    // ---------------- fused optimizer epilogue (mode 4): warps 2..5, one accumulator row per thread ----
+    // Each 32-column piece of the row goes from TMEM to registers and through the AdamW step of its 32
+    // parameters (loads and stores straight from the thread's row: each is a full 128-byte line).
+    const int q = warp & 3;
+    const AdamHP hpv = adam_hp(g.u.hp, g.u.b1, g.u.b2, g.u.eps, g.u.wd);
+    int it = 0;
+    for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
+      int tm, tn;
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      const int acc = it & 1;
+      const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], aph, abort_flag, g.err) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      fence_after();
+      const int m = tm * BM + q * 32 + lane;
+      const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        const int nh = tn * BN + c;
+        float v[32];
+        tmem_ld32(trow + (uint32_t)c, v);
+        if (g.alpha != 1.f) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] *= g.alpha;
+        }
+        if (m < g.M && nh < g.N) update_row32(g.u, hpv, (size_t)m * g.N + nh, min(32, g.N - nh), v);
+      }
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+    }
   } else {
     // ---------------- epilogue: warps 2..5, one accumulator row per thread ----------------
     // Per 128-byte column chunk (64 bf16 or 32 fp32 columns): TMEM -> registers (alpha, bias,
@@ -311,12 +389,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Sums the split-K partials in split order (deterministic) and applies the epilogue.
+// Sums the split-K partials in split order (deterministic) and applies the epilogue (mode 4: the fused
+// optimizer step of `u`, as update_row32 does it).
 __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M, int N, int mode, void* C,
-                                const float* __restrict__ bias, const bf16* R, float alpha, int rmode) {
+                                const float* __restrict__ bias, const bf16* R, float alpha, int rmode,
+                                const GemmUpdate u) {
   pdl_wait();
   pdl_trigger();
   const size_t n8 = (size_t)M * N / 8, MN = (size_t)M * N;
+  AdamHP hpv;
+  if (mode == 4) hpv = adam_hp(u.hp, u.b1, u.b2, u.eps, u.wd);
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
     const size_t e = i * 8;
     float acc[8];
@@ -329,7 +411,26 @@ __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M,
     }
 #pragma unroll
     for (int q = 0; q < 8; ++q) acc[q] *= alpha;
-    if (mode == 2) {
+    if (mode == 4) {
+      float th[8], mm[8], vv[8], gg[8];
+      Vec8<float>::load(u.theta + e, th);
+      Vec8<float>::load(u.m + e, mm);
+      Vec8<float>::load(u.v + e, vv);
+      if (u.g) Vec8<float>::load(u.g + e, gg);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float gsum = u.g ? __fadd_rn(gg[q], acc[q]) : acc[q];
+        adamw_elem(th[q], mm[q], vv[q], __fmul_rn(gsum, u.gscale), hpv);
+      }
+      Vec8<float>::store(u.theta + e, th);
+      Vec8<float>::store(u.m + e, mm);
+      Vec8<float>::store(u.v + e, vv);
+      if (u.comp) Vec8<bf16>::store((bf16*)u.comp + e, th);
+      if (u.g) {
+        const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        Vec8<float>::store(u.g + e, z);
+      }
+    } else if (mode == 2) {
       float c[8];
       Vec8<float>::load((float*)C + e, c);
 #pragma unroll
@@ -478,19 +579,24 @@ void choose(int mode, int M, int N, int K, int& bn_out, int& splits_out) {
 
 bool gemm_tc_available() { return tc::init(); }
 
-// Returns false when the shape / alignment is outside what the tensor-core path handles.
-bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode) {
+namespace {
+
+// Plans and launches one tensor-core GEMM (modes 0-2, or 4 with `u`); false if the shape or alignment
+// is outside the kernel's rules.
+bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
+            unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode, const GemmUpdate* u) {
   if (!tc::init()) return false;
   if (M < 16 || N < 16 || K < 16) return false;
   auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
   if (!al16(A) || !al16(B) || !al16(C) || (R && !al16(R))) return false;
+  if (u && (!al16(u->theta) || !al16(u->m) || !al16(u->v) || (u->g && !al16(u->g)) || (u->comp && !al16(u->comp))))
+    return false;
   if (N % 8 != 0) return false;
   if ((mode == 0 || mode == 1) && K % 8 != 0) return false;
-  if (mode == 2 && M % 8 != 0) return false;
+  if (mode >= 2 && M % 8 != 0) return false;
   int bn = 128, splits = 1;
-  tc::choose(mode, M, N, K, bn, splits);
-  if (const char* force = std::getenv("ZL_GEMM_TILE")) {   // tuning override "BN:SPLITS"
+  tc::choose(mode == 4 ? 2 : mode, M, N, K, bn, splits);
+  if (const char* force = std::getenv("ZL_GEMM_TILE")) {   // test hook "BN:SPLITS": forces the tile and split count
     int fb = 0, fs = 0;
     if (std::sscanf(force, "%d:%d", &fb, &fs) == 2 && (fb == 64 || fb == 128 || fb == 256) && fs >= 1 && fs <= 16) {
       bn = fb;
@@ -500,6 +606,7 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
   tc::Args a;
   a.M = M; a.N = N; a.K = K; a.mode = mode;
   a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err; a.alpha = alpha; a.rmode = rmode;
+  a.u = u ? *u : GemmUpdate{};
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
   a.tiles_n = (N + bn - 1) / bn;
   const int nk = (K + tc::BK - 1) / tc::BK;
@@ -533,11 +640,24 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
       const size_t n8 = (size_t)M * N / 8;
       const int blocks = (int)std::min<size_t>((n8 + 255) / 256, (size_t)tc::g_sms * 8);
       launch_pdl(tc::splitk_reduce_k, blocks, 256, 0, s, ws, a.splits, M, N, mode, C, bias, (const bf16*)R, alpha,
-                 rmode);
+                 rmode, a.u);
     }
     cudaFreeAsync(ws, s);
   }
   return ok;
+}
+
+}  // namespace
+
+// Returns false when the shape / alignment is outside what the tensor-core path handles.
+bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
+             unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode) {
+  return run_tc(mode, M, N, K, A, B, C, bias, R, err, s, pool, alpha, rmode, nullptr);
+}
+
+bool gemm_tc_update(int M, int N, int K, const void* A, const void* B, const GemmUpdate& u, unsigned* err,
+                    cudaStream_t s, cudaMemPool_t pool, float alpha) {
+  return run_tc(4, M, N, K, A, B, u.theta, nullptr, nullptr, err, s, pool, alpha, 0, &u);
 }
 
 }  // namespace zl

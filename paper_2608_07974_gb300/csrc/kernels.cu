@@ -1,6 +1,8 @@
 // Memory-bound kernels of the ZeroLock local step: embedding gather, norms, RoPE, activations,
 // the fused local objective (Eq. 3-5) and the per-chunk AdamW update.
 #include <math.h>
+
+#include <algorithm>
 #include <stdlib.h>
 
 #include <type_traits>
@@ -1064,18 +1066,12 @@ __global__ void adamw_k(float4* __restrict__ th, float4* __restrict__ g, float4*
                         const float* __restrict__ hp, float b1, float b2, float eps, float wd, float gscale) {
   pdl_wait();
   pdl_trigger();
-  const float lr = hp[0], bc1 = hp[1], bc2 = hp[2];
-  const float decay = 1.f - lr * wd;
+  const AdamHP h = adam_hp(hp, b1, b2, eps, wd);
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
     float4 t = th[i], gg = g[i], mm = m[i], vv = v[i];
     float* tp = &t.x; float* gp = &gg.x; float* mp = &mm.x; float* vp = &vv.x;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float gq = gp[q] * gscale;
-      mp[q] = b1 * mp[q] + (1.f - b1) * gq;
-      vp[q] = b2 * vp[q] + (1.f - b2) * gq * gq;
-      tp[q] = tp[q] * decay - lr * (mp[q] / bc1) / (sqrtf(vp[q] / bc2) + eps);
-    }
+    for (int q = 0; q < 4; ++q) adamw_elem(tp[q], mp[q], vp[q], __fmul_rn(gp[q], gscale), h);
     th[i] = t; m[i] = mm; v[i] = vv;
     g[i] = make_float4(0.f, 0.f, 0.f, 0.f);
     if (comp) {
@@ -1085,16 +1081,72 @@ __global__ void adamw_k(float4* __restrict__ th, float4* __restrict__ g, float4*
   }
 }
 
+void launch_adamw_tick(long long* t, float* hp, float lr0, int schedule, float gamma, float b1, float b2,
+                       cudaStream_t s) {
+  note_launch(1);
+  launch_pdl(adamw_tick_k, 1, 1, 0, s, t, hp, lr0, schedule, gamma, b1, b2);
+}
+
 void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, long long* t, float* hp,
                   float lr0, int schedule, float gamma, float b1, float b2, float eps, float wd, float gscale,
                   cudaStream_t s) {
-  note_launch(2);
-  launch_pdl(adamw_tick_k, 1, 1, 0, s, t, hp, lr0, schedule, gamma, b1, b2);
+  launch_adamw_tick(t, hp, lr0, schedule, gamma, b1, b2, s);
+  note_launch(1);
   const size_t n4 = n / 4;   // slabs are padded to a multiple of 64 elements
   if (n4 == 0) return;
   const int th = 256, gr = grid_for(n4, th, 152 * 8);
   launch_pdl(adamw_k, gr, th, 0, s, (float4*)theta, (float4*)g, (float4*)m, (float4*)v, (__nv_bfloat162*)comp, n4,
              (const float*)hp, b1, b2, eps, wd, gscale);
+}
+
+void launch_adamw_span(float* theta, float* g, float* m, float* v, void* comp, size_t n, const float* hp, float b1,
+                       float b2, float eps, float wd, float gscale, cudaStream_t s) {
+  const size_t n4 = n / 4;
+  if (n4 == 0) return;
+  note_launch(1);
+  const int th = 256, gr = grid_for(n4, th, 152 * 8);
+  launch_pdl(adamw_k, gr, th, 0, s, (float4*)theta, (float4*)g, (float4*)m, (float4*)v, (__nv_bfloat162*)comp, n4,
+             hp, b1, b2, eps, wd, gscale);
+}
+
+// AdamW over a list of ranges of one slab (offsets and lengths in floats, multiples of 4), with this
+// step's lr and bias corrections already in hp (no tick): the parameters the weight-gradient GEMMs did
+// not update in their epilogue. blockIdx.y is the range.
+__global__ void adamw_ranges_k(float* __restrict__ th, float* __restrict__ g, float* __restrict__ m,
+                               float* __restrict__ v, bf16* __restrict__ comp, const long long* __restrict__ ranges,
+                               const float* __restrict__ hp, float b1, float b2, float eps, float wd, float gscale) {
+  pdl_wait();
+  pdl_trigger();
+  const AdamHP h = adam_hp(hp, b1, b2, eps, wd);
+  const size_t off = (size_t)ranges[2 * blockIdx.y], n4 = (size_t)ranges[2 * blockIdx.y + 1] / 4;
+  float4* th4 = reinterpret_cast<float4*>(th + off);
+  float4* g4 = reinterpret_cast<float4*>(g + off);
+  float4* m4 = reinterpret_cast<float4*>(m + off);
+  float4* v4 = reinterpret_cast<float4*>(v + off);
+  __nv_bfloat162* c2 = comp ? reinterpret_cast<__nv_bfloat162*>(comp + off) : nullptr;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
+    float4 t = th4[i], gg = g4[i], mm = m4[i], vv = v4[i];
+    float* tp = &t.x; float* gp = &gg.x; float* mp = &mm.x; float* vp = &vv.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) adamw_elem(tp[q], mp[q], vp[q], __fmul_rn(gp[q], gscale), h);
+    th4[i] = t; m4[i] = mm; v4[i] = vv;
+    g4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c2) {
+      c2[2 * i] = __floats2bfloat162_rn(t.x, t.y);
+      c2[2 * i + 1] = __floats2bfloat162_rn(t.z, t.w);
+    }
+  }
+}
+
+void launch_adamw_ranges(float* theta, float* g, float* m, float* v, void* comp, const long long* ranges,
+                         int nranges, size_t max_len, const float* hp, float b1, float b2, float eps, float wd,
+                         float gscale, cudaStream_t s) {
+  if (nranges <= 0) return;
+  note_launch(1);
+  const int th = 256;
+  const unsigned bx = (unsigned)std::max<size_t>(1, std::min<size_t>((max_len / 4 + th - 1) / th, 64));
+  launch_pdl(adamw_ranges_k, dim3(bx, (unsigned)nranges), th, 0, s, theta, g, m, v, (bf16*)comp, ranges, hp, b1,
+             b2, eps, wd, gscale);
 }
 
 __global__ void f32_to_bf16_k(const float* __restrict__ a, bf16* __restrict__ b, size_t n) {

@@ -66,6 +66,17 @@ void launch_loss_reduce(const float* row_loss, int N, const int* count, float* o
 void launch_adamw(float* theta, float* g, float* m, float* v, void* comp, size_t n, long long* t, float* hp,
                   float lr0, int schedule, float gamma, float b1, float b2, float eps, float wd, float gscale,
                   cudaStream_t s);
+// Advances the step count and writes hp = {lr_t, 1 - b1^t, 1 - b2^t} (the first kernel of launch_adamw).
+void launch_adamw_tick(long long* t, float* hp, float lr0, int schedule, float gamma, float b1, float b2,
+                       cudaStream_t s);
+// AdamW over one contiguous span of n floats (a multiple of 4), hp already written for this step.
+void launch_adamw_span(float* theta, float* g, float* m, float* v, void* comp, size_t n, const float* hp, float b1,
+                       float b2, float eps, float wd, float gscale, cudaStream_t s);
+// AdamW over `nranges` (offset, length) pairs of a slab (device array ranges[2 * nranges], lengths and
+// offsets multiples of 4, the longest max_len), with hp already written for this step; zeroes g there.
+void launch_adamw_ranges(float* theta, float* g, float* m, float* v, void* comp, const long long* ranges,
+                         int nranges, size_t max_len, const float* hp, float b1, float b2, float eps, float wd,
+                         float gscale, cudaStream_t s);
 void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
 
 // GEMM (row-major): mode 0: C = A[M,K] B[N,K]^T (+ bias[N]) (+ R[M,N]); mode 1: C = A[M,K] B[K,N] (+ R);
@@ -78,6 +89,22 @@ void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
 void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
           const void* R, cudaStream_t s, unsigned* err = nullptr, cudaMemPool_t pool = nullptr, float alpha = 1.f,
           int rmode = 0);
+// The optimizer step fused into a weight-gradient product (mode 2's C += alpha A^T B, here the last
+// micro-batch of an update window): for the [M, N] tensor whose fp32 master, AdamW moments and bf16
+// compute copy are theta, m, v and comp (comp may be NULL), the window's gradient is
+// G = gscale * (g + alpha A^T B), g the accumulated gradient of the window's earlier micro-batches
+// (NULL when there are none; zeroed here otherwise), and AdamW (hp as written by the step-count
+// kernel) updates theta, m, v and comp in place; no gradient is stored.
+struct GemmUpdate {
+  float *theta, *m, *v, *g;
+  void* comp;
+  const float* hp;
+  float b1, b2, eps, wd, gscale;
+};
+// bf16 operands on the tcgen05 kernel; false when the shape or alignment rules of mode 2 do not hold
+// (the caller then forms the gradient with gemm() and applies the step with launch_adamw_ranges).
+bool gemm_tc_update(int M, int N, int K, const void* A, const void* B, const GemmUpdate& u, unsigned* err,
+                    cudaStream_t s, cudaMemPool_t pool, float alpha = 1.f);
 bool gemm_tc_available();
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
              unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode = 0);
