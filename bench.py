@@ -467,6 +467,8 @@ def run_ours(args):
     del seng
     torch.cuda.empty_cache()
     roof_serial = roofline_of(sprof)
+    classes_serial = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / prof_steps}
+                      for k, v in sprof.items() if v["launches"]}
 
     # ---- CPU oracle on a bounded sample (rank 0, one GPU only) --------------------------------
     cpu = None
@@ -488,7 +490,8 @@ def run_ours(args):
                 "peak_hbm_gb": zl_peak / 1e9, "bp": bp,
                 "zl_vs_bp": {"throughput": value / bp["value"], "peak_hbm": (zl_peak / 1e9) / bp["peak_hbm_gb"]}
                 if bp else None,
-                "roofline": roof, "roofline_serial": roof_serial, "step_roofline": step_roof, "kernel_classes": classes, "cpu_baseline": cpu, "e2e": e2e,
+                "roofline": roof, "roofline_serial": roof_serial, "step_roofline": step_roof, "kernel_classes": classes,
+                "kernel_classes_serial": classes_serial, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": launches, "clocks": clk}
         print(json.dumps(line), flush=True)
     if world > 1:

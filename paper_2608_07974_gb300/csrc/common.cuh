@@ -148,20 +148,22 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 }
 
 // The decoupled AdamW step of one parameter (Eq. 6, as AdamW): m <- b1 m + (1 - b1) g;
-// v <- b2 v + (1 - b2) g^2; theta <- theta (1 - lr wd) - lr (m / bc1) / (sqrt(v / bc2) + eps), with
-// bc1 = 1 - b1^t, bc2 = 1 - b2^t. Every operation is an explicitly rounded intrinsic, so every kernel
-// that applies the step (the slab and range updates, the weight-gradient GEMM's fused epilogue, the
-// split-K reduction) computes the same bits from the same gradient.
+// v <- b2 v + (1 - b2) g^2; theta <- theta (1 - lr wd) - (lr / bc1) m / (sqrt(v / bc2) + eps), with
+// bc1 = 1 - b1^t, bc2 = 1 - b2^t. Every operation is an explicitly rounded intrinsic or a hardware
+// approximation instruction (square root and reciprocal, a few ulp, far inside the fp32 parameter
+// tolerance), so every kernel that applies the step (the slab and range updates, the weight-gradient
+// GEMM's fused epilogue, the split-K reduction) computes the same bits from the same gradient, in about
+// a dozen instructions.
 struct AdamHP {
-  float lr, decay, bc1, bc2, b1, omb1, b2, omb2, eps;
+  float step, decay, inv_bc2, b1, omb1, b2, omb2, eps;   // step = lr / bc1, inv_bc2 = 1 / bc2
 };
 // hp = {lr_t, 1 - b1^t, 1 - b2^t} as written by the step-count kernel.
 __device__ __forceinline__ AdamHP adam_hp(const float* hp, float b1, float b2, float eps, float wd) {
   AdamHP h;
-  h.lr = hp[0];
-  h.bc1 = hp[1];
-  h.bc2 = hp[2];
-  h.decay = __fsub_rn(1.f, __fmul_rn(h.lr, wd));
+  const float lr = hp[0];
+  h.step = __fdiv_rn(lr, hp[1]);
+  h.inv_bc2 = __fdiv_rn(1.f, hp[2]);
+  h.decay = __fsub_rn(1.f, __fmul_rn(lr, wd));
   h.b1 = b1;
   h.omb1 = __fsub_rn(1.f, b1);
   h.b2 = b2;
@@ -169,9 +171,19 @@ __device__ __forceinline__ AdamHP adam_hp(const float* hp, float b1, float b2, f
   h.eps = eps;
   return h;
 }
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float r;
+  asm("sqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
 __device__ __forceinline__ void adamw_elem(float& th, float& m, float& v, float g, const AdamHP& h) {
-  m = __fadd_rn(__fmul_rn(h.b1, m), __fmul_rn(h.omb1, g));
-  v = __fadd_rn(__fmul_rn(h.b2, v), __fmul_rn(__fmul_rn(h.omb2, g), g));
-  const float den = __fadd_rn(__fsqrt_rn(__fdiv_rn(v, h.bc2)), h.eps);
-  th = __fsub_rn(__fmul_rn(th, h.decay), __fdiv_rn(__fmul_rn(h.lr, __fdiv_rn(m, h.bc1)), den));
+  m = __fmaf_rn(h.b1, m, __fmul_rn(h.omb1, g));
+  v = __fmaf_rn(h.b2, v, __fmul_rn(__fmul_rn(h.omb2, g), g));
+  const float den = __fadd_rn(sqrt_approx(__fmul_rn(v, h.inv_bc2)), h.eps);
+  th = __fmaf_rn(th, h.decay, -__fmul_rn(__fmul_rn(h.step, m), rcp_approx(den)));
 }

@@ -328,12 +328,11 @@ void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, 
   ProfScope p(c, s, head ? PC_GEMM_HEAD : PC_GEMM, 2.0 * M * N * (double)K, e * ((double)M * K + (double)N * K) + out);
   gemm(c->dt, mode, M, N, K, A, B, C, bias, R, s, c->d_err, c->pool, alpha);
 }
-// Weight gradient of matrix p of layer li: C += A^T B into its gradient accumulator, or, when this
-// micro-batch ends the update window with the fused update on (k.fuse), the AdamW step of the matrix in
-// the product's epilogue (the accumulator is read if earlier micro-batches of the window filled it, and
-// left at zero). Where the tensor-core product does not apply (fp32, or a shape outside its rules) the
-// gradient is formed with gemm() and the step applied to the matrix's range right after it: the same
-// arithmetic either way.
+// Weight gradient of matrix p of layer li: C += A^T B into its gradient accumulator, or, with the fused
+// update on (k.fuse: one micro-batch per window), the AdamW step of the matrix in the product's epilogue,
+// with no gradient stored. Where the tensor-core product does not apply (fp32, or a shape outside its
+// rules) the gradient is formed with gemm() in the accumulator and the step applied to the matrix's
+// range right after it: the same arithmetic either way.
 void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, const void* A, const void* B) {
   float* g = Gm(k, li, p);
   if (!g) return;   // frozen
@@ -343,12 +342,12 @@ void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, 
   }
   const zl_train_cfg& cf = c->cfg;
   const size_t off = k.layers[li].off[p];
-  const GemmUpdate u{k.master + off, k.m + off, k.v + off, cf.accum_m > 1 ? g : nullptr,
+  const GemmUpdate u{k.master + off, k.m + off, k.v + off, nullptr,
                      c->dt == BF16 ? (void*)((bf16*)k.comp + off) : nullptr, k.d_hp, cf.beta1, cf.beta2, cf.eps,
-                     cf.weight_decay, 1.f / (float)cf.accum_m};
+                     cf.weight_decay, 1.f};
   const double e = (double)esz(c), mn = (double)M * N;
-  // operands, then read theta, m, v (and g) and write them back (g zeroed), plus the compute copy
-  const double upd = (cf.accum_m > 1 ? 32.0 : 24.0) * mn + (c->dt == BF16 ? 2.0 : 0.0) * mn;
+  // operands, then read theta, m, v and write them back, plus the compute copy
+  const double upd = 24.0 * mn + (c->dt == BF16 ? 2.0 : 0.0) * mn;
   ProfScope ps(c, s, PC_GEMM_UPD, 2.0 * mn * (double)K, e * ((double)M * K + (double)N * K) + upd);
   if (c->dt == BF16 && gemm_tc_update(M, N, K, A, B, u, c->d_err, s, c->pool)) return;
   gemm(c->dt, 2, M, N, K, A, B, g, nullptr, nullptr, s, c->d_err, c->pool);
@@ -674,12 +673,12 @@ void chunk_bwd(zl_ctx* c, Chunk& k, ChunkActs& acts, const void* dh, void* dh_in
   pfree(a.base, s);
 }
 
-// Before the backward of one micro-batch of chunk k: when the micro-batch ends the update window and
-// the fused update applies (full fine-tune, cfg.unfused_update = 0), advance the step count and write
-// this step's lr and bias corrections now, so the weight-gradient products can apply the step.
+// Before the backward of one micro-batch of chunk k: when the fused update applies (one micro-batch per
+// window, full fine-tune, cfg.unfused_update = 0), advance the step count and write this step's lr and
+// bias corrections now, so the weight-gradient products can apply the step.
 void window_begin(zl_ctx* c, Chunk& k, cudaStream_t s) {
   const zl_train_cfg& g = c->cfg;
-  k.fuse = k.micro + 1 >= g.accum_m && !g.unfused_update && g.lora_rank == 0;
+  k.fuse = g.accum_m == 1 && !g.unfused_update && g.lora_rank == 0;
   if (k.fuse) launch_adamw_tick(k.d_t, k.d_hp, g.lr, g.lr_schedule, g.lr_gamma, g.beta1, g.beta2, s);
 }
 

@@ -9,6 +9,7 @@
 #include <algorithm>
 #include <cstdio>
 #include <cstdlib>
+#include <cstring>
 
 #include "common.cuh"
 #include "ops.h"
@@ -18,9 +19,10 @@ namespace zl {
 namespace tc {
 
 constexpr int BM = 128, BK = 64;
-constexpr int kThreads = 192;
+constexpr int kThreads = 192;      // TMA warp, MMA warp, four epilogue warps
+constexpr int kThreadsUpd = 320;   // fused-update kernels (mode 4): eight epilogue warps, two per TMEM lane quadrant
 
-template <int BN>
+template <int BN, bool UPD = false>
 struct Cfg {
   // BN = 64 stays under 114 KB of shared memory so two CTAs (and TMEM allocations) fit on an SM.
   static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 3);
@@ -28,9 +30,63 @@ struct Cfg {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
-  // epilogue staging: per epilogue warp two buffers of 32 rows x 128 B (the TMA store box)
+  // epilogue staging: per epilogue warp two buffers of 32 rows x 128 B (the TMA store box), or, in the
+  // fused-update kernels, one 32 x 32 accumulator piece for each of eight warps
   static constexpr int OUT_BYTES = 4 * 2 * 32 * 128;
   static constexpr int SMEM = STAGES * STAGE_BYTES + OUT_BYTES + 1024 + 256;
+};
+
+// Mode 4, one chunk: 16 rows x 32 columns of the tensor (rows row0 + 16 h .., columns col0 ..), whose
+// accumulator piece is staged (fp32, 128-byte rows, 16-byte pieces XOR-swizzled by row) in `sp`. Lane l
+// takes columns col0 + 4 (l % 8) .. + 3 of rows 16 h + l / 8 + 4 j, j = 0..3: every warp-wide load or
+// store covers four whole 128-byte lines. upd_load issues the chunk's loads; upd_apply applies the AdamW
+// step (adamw_elem) with G = gscale * acc to the loaded state and writes the fp32 master, both moments
+// and the bf16 compute copy back. The state is streamed (evict-first): it is touched once, and L2 is
+// kept for the operand tiles.
+struct UpdRegs {
+  float4 th[4], mm[4], vv[4];
+  size_t at[4];
+  unsigned ok;   // bit j: row j is inside the tensor
+};
+__device__ __forceinline__ void upd_load(const GemmUpdate& u, UpdRegs& r, int row0, int h, int col0, int M, int N,
+                                         bool valid, int lane) {
+  r.ok = 0;
+  const int col = col0 + 4 * (lane & 7);
+  if (!valid || col >= N) return;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int row = row0 + 16 * h + (lane >> 3) + 4 * j;
+    r.at[j] = (size_t)row * N + col;
+    if (row < M) {
+      r.ok |= 1u << j;
+      r.th[j] = __ldcs(reinterpret_cast<const float4*>(u.theta + r.at[j]));
+      r.mm[j] = __ldcs(reinterpret_cast<const float4*>(u.m + r.at[j]));
+      r.vv[j] = __ldcs(reinterpret_cast<const float4*>(u.v + r.at[j]));
+    }
+  }
+}
+__device__ __forceinline__ void upd_apply(const GemmUpdate& u, const AdamHP& h, UpdRegs& r, const uint8_t* sp,
+                                          int hh, int lane) {
+  const int piece = lane & 7;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (!(r.ok >> j & 1u)) continue;
+    const int rr = 16 * hh + (lane >> 3) + 4 * j;
+    const float4 a4 = *reinterpret_cast<const float4*>(sp + rr * 128 + ((piece ^ (rr & 7)) << 4));
+    const float acc[4] = {a4.x, a4.y, a4.z, a4.w};
+    float* tp = &r.th[j].x; float* mp = &r.mm[j].x; float* vp = &r.vv[j].x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) adamw_elem(tp[q], mp[q], vp[q], __fmul_rn(acc[q], u.gscale), h);
+    __stcs(reinterpret_cast<float4*>(u.theta + r.at[j]), r.th[j]);
+    __stcs(reinterpret_cast<float4*>(u.m + r.at[j]), r.mm[j]);
+    __stcs(reinterpret_cast<float4*>(u.v + r.at[j]), r.vv[j]);
+    __nv_bfloat162 c2[2] = {__floats2bfloat162_rn(tp[0], tp[1]), __floats2bfloat162_rn(tp[2], tp[3])};
+    __stcs(reinterpret_cast<uint2*>((bf16*)u.comp + r.at[j]), *reinterpret_cast<const uint2*>(c2));
+  }
+}
+
+struct UpdMaps {   // (reserved: the fused update reads and writes its state directly)
+  CUtensorMap unused;
 };
 
 struct Args {
@@ -46,48 +102,6 @@ struct Args {
   int rmode;                  // R in modes 0/1: 0 adds it (residual); 1 multiplies by GELU'(R) (R = the GELU input)
   GemmUpdate u;               // mode 4
 };
-
-// Mode 4 on one accumulator row's columns [base, base + ncols) of the tensor (ncols <= 32, a multiple of
-// 4): G = gscale * (g + acc), then the AdamW step of each parameter (adamw_elem), written back to the
-// fp32 master, both moments and the bf16 compute copy; g (if any) is zeroed. 16 columns at a time, their
-// twelve (sixteen with g) 16-byte loads issued before any arithmetic.
-__device__ __forceinline__ void update_row32(const GemmUpdate& u, const AdamHP& h, size_t base, int ncols,
-                                             const float* acc) {
-#pragma unroll
-  for (int half = 0; half < 2; ++half) {
-    float4 th[4], mm[4], vv[4], gg[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int col = 16 * half + 4 * j;
-      if (col < ncols) {
-        th[j] = *reinterpret_cast<const float4*>(u.theta + base + col);
-        mm[j] = *reinterpret_cast<const float4*>(u.m + base + col);
-        vv[j] = *reinterpret_cast<const float4*>(u.v + base + col);
-        gg[j] = u.g ? *reinterpret_cast<const float4*>(u.g + base + col) : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int col = 16 * half + 4 * j;
-      if (col < ncols) {
-        float* tp = &th[j].x; float* mp = &mm[j].x; float* vp = &vv[j].x; const float* gp = &gg[j].x;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const float gsum = u.g ? __fadd_rn(gp[q], acc[col + q]) : acc[col + q];
-          adamw_elem(tp[q], mp[q], vp[q], __fmul_rn(gsum, u.gscale), h);
-        }
-        *reinterpret_cast<float4*>(u.theta + base + col) = th[j];
-        *reinterpret_cast<float4*>(u.m + base + col) = mm[j];
-        *reinterpret_cast<float4*>(u.v + base + col) = vv[j];
-        if (u.comp) {
-          __nv_bfloat162 c2[2] = {__floats2bfloat162_rn(tp[0], tp[1]), __floats2bfloat162_rn(tp[2], tp[3])};
-          *reinterpret_cast<uint2*>((bf16*)u.comp + base + col) = *reinterpret_cast<const uint2*>(c2);
-        }
-        if (u.g) *reinterpret_cast<float4*>(u.g + base + col) = make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-    }
-  }
-}
 
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, operand majors, N, M.
 template <int BN, bool A_MN, bool B_MN>
@@ -106,11 +120,13 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
   tn = r / gm;
 }
 
-template <int BN, bool A_MN, bool B_MN>
-__global__ void __launch_bounds__(kThreads, 1)
+// UPD: the fused optimizer epilogue (mode 4) is compiled in (a kernel of its own, so the other modes keep
+// their register budget).
+template <int BN, bool A_MN, bool B_MN, bool UPD = false>
+__global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     gemm_tc_k(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
-              const __grid_constant__ CUtensorMap tcm, const Args g) {
-  using C_ = Cfg<BN>;
+              const __grid_constant__ CUtensorMap tcm, const Args g, const __grid_constant__ UpdMaps um) {
+  using C_ = Cfg<BN, UPD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* outbuf = smem + C_::STAGES * C_::STAGE_BYTES;   // 1024-byte aligned (stage sizes are)
@@ -125,7 +141,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C_::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
-    for (int a = 0; a < 2; ++a) { mbar_init(&tfull[a], 1); mbar_init(&tempty[a], 4); }
+    for (int a = 0; a < 2; ++a) { mbar_init(&tfull[a], 1); mbar_init(&tempty[a], UPD ? 8 : 4); }
     mbar_init(fin, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -235,12 +251,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     // all MMAs issued by the leader complete before TMEM is released
     if (leader) mma_commit(fin);
     __syncwarp();
-  } else if (A_MN && B_MN && g.mode == 4) {
-    // ---------------- fused optimizer epilogue (mode 4): warps 2..5, one accumulator row per thread ----
-    // Each 32-column piece of the row goes from TMEM to registers and through the AdamW step of its 32
-    // parameters (loads and stores straight from the thread's row: each is a full 128-byte line).
-    const int q = warp & 3;
+  } else if (UPD && g.mode == 4) {
+    // ---------------- fused optimizer epilogue (mode 4): warps 2..9 ----------------
+    // Two warps per TMEM lane quadrant take alternate 32-column pieces of the quadrant's 32 accumulator
+    // rows (BN 128: pieces 0, 2 or 1, 3). Per tile a warp reads both its pieces from TMEM and hands TMEM
+    // back at once; then per piece it stages the accumulator in its shared-memory buffer and works
+    // through the piece's two 16-row chunks (upd_load, then upd_apply).
+    const int q = warp & 3, part = (warp - 2) >> 2;
+    uint8_t* sbuf = outbuf + (warp - 2) * (32 * 128);
     const AdamHP hpv = adam_hp(g.u.hp, g.u.b1, g.u.b2, g.u.eps, g.u.wd);
+    constexpr int NP = BN / 64;   // pieces per warp and tile
+    constexpr int NC = 2 * NP;    // 16-row chunks per warp and tile: chunk k = piece k / 2, half k % 2
+    // L2 prefetch of chunk `k` of tile `unit` (lanes 0-15 one row each: its 128-byte line of the master
+    // and of both moments), issued PD chunks ahead of the loads that read it
+    auto prefetch_chunk = [&](int unit, int k) {
+      if (unit >= num_units || lane >= 16) return;
+      int tm, tn;
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * part + 64 * (k >> 1);
+      if (row >= g.M || col >= g.N) return;
+      const size_t at = (size_t)row * g.N + col;
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.theta + at));
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.m + at));
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.v + at));
+    };
+    constexpr int PD = 2;   // prefetch distance in chunks (2 and 3 measured alike, 4 slower)
+#pragma unroll
+    for (int k = 0; k < PD; ++k) prefetch_chunk(blockIdx.x + (k / NC) * gridDim.x, k % NC);
     int it = 0;
     for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
       int tm, tn;
@@ -252,22 +289,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       fence_after();
-      const int m = tm * BM + q * 32 + lane;
+      const int row0 = tm * BM + q * 32;
       const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-#pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        const int nh = tn * BN + c;
-        float v[32];
-        tmem_ld32(trow + (uint32_t)c, v);
-        if (g.alpha != 1.f) {
+      float v[NP][32];
 #pragma unroll
-          for (int e = 0; e < 32; ++e) v[e] *= g.alpha;
-        }
-        if (m < g.M && nh < g.N) update_row32(g.u, hpv, (size_t)m * g.N + nh, min(32, g.N - nh), v);
-      }
+      for (int p = 0; p < NP; ++p) tmem_ld32(trow + (uint32_t)(32 * part + 64 * p), v[p]);
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
+#pragma unroll
+      for (int p = 0; p < NP; ++p) {
+        const int c = 32 * part + 64 * p;
+        if (g.alpha != 1.f) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[p][e] *= g.alpha;
+        }
+        __syncwarp();   // the previous piece's reads of the staging buffer are done
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          *reinterpret_cast<float4*>(sbuf + lane * 128 + ((k ^ (lane & 7)) << 4)) =
+              make_float4(v[p][4 * k], v[p][4 * k + 1], v[p][4 * k + 2], v[p][4 * k + 3]);
+        __syncwarp();
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int k2 = 2 * p + h + PD;   // PD chunks ahead, into the next tiles at the end
+          prefetch_chunk(unit + (k2 / NC) * gridDim.x, k2 % NC);
+          UpdRegs r;
+          upd_load(g.u, r, row0, h, tn * BN + c, g.M, g.N, c < BN, lane);
+          upd_apply(g.u, hpv, r, sbuf, h, lane);
+        }
+      }
     }
   } else {
     // ---------------- epilogue: warps 2..5, one accumulator row per thread ----------------
@@ -510,11 +561,11 @@ bool make_map_c(CUtensorMap* m, const Args& a) {
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool A_MN, bool B_MN>
+template <int BN, bool A_MN, bool B_MN, bool UPD = false>
 bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int ctas_per_sm) {
-  using C_ = Cfg<BN>;
+  using C_ = Cfg<BN, UPD>;
   static bool attr = false;
-  auto kern = gemm_tc_k<BN, A_MN, B_MN>;
+  auto kern = gemm_tc_k<BN, A_MN, B_MN, UPD>;
   if (!attr) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM) != cudaSuccess) return false;
     attr = true;
@@ -526,12 +577,14 @@ bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int cta
                         : make_map(&tb, B, (uint64_t)a.K, (uint64_t)a.N, 64, BN);
   CUtensorMap tcm;
   if (!okA || !okB || !make_map_c(&tcm, a)) return false;
+  UpdMaps um;
+  std::memset(&um, 0, sizeof um);
   const int units = a.tiles_m * a.tiles_n * a.splits;
   const int slots = g_sms * ctas_per_sm;
   const int grid = units < slots ? units : slots;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3((unsigned)kThreads);
+  cfg.blockDim = dim3((unsigned)(UPD ? kThreadsUpd : kThreads));
   cfg.dynamicSmemBytes = C_::SMEM;
   cfg.stream = s;
   cudaLaunchAttribute at[1];
@@ -539,7 +592,7 @@ bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int cta
   at[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, ta, tb, tcm, a) == cudaSuccess;
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, tcm, a, um) == cudaSuccess;
 }
 
 template <bool A_MN, bool B_MN>
@@ -549,15 +602,21 @@ bool launch_bn(int bn, const Args& a, const void* A, const void* B, cudaStream_t
   return launch<64, A_MN, B_MN>(a, A, B, s, 2);
 }
 
+// The fused-update kernel (mode 4): 128 x 128 tiles, one CTA per SM.
+bool launch_upd(const Args& a, const void* A, const void* B, cudaStream_t s) {
+  return launch<128, true, true, true>(a, A, B, s, 1);
+}
+
 // Tile width and split count from a wave model: units of 128 x BN x (K / splits) run on 152 (BN
 // 256/128) or 304 (BN 64) slots, each k block (64 deep) of a unit taking the time measured for that
 // tile on GB300 (4096^3 and transformer-shape sweeps; the operands of the mode-2 kernel are both
 // MN-major and load in more boxes), plus, for splits, the fp32 partial traffic and the reduction.
-void choose(int mode, int M, int N, int K, int& bn_out, int& splits_out) {
+void choose(int mode, int M, int N, int K, int& bn_out, int& splits_out, bool only128 = false) {
   const double hbm = 6.0e12;                  // bytes/s for the partials
   const int nk = (K + BK - 1) / BK;
   double best = 1e30;
   for (int bn : {256, 128, 64}) {
+    if (only128 && bn != 128) continue;
     const double kb = mode == 2 ? (bn == 256 ? 0.40e-6 : bn == 128 ? 0.30e-6 : 0.36e-6)
                                 : (bn == 256 ? 0.36e-6 : bn == 128 ? 0.29e-6 : 0.32e-6);
     const long tiles = (long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
@@ -589,17 +648,18 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   if (M < 16 || N < 16 || K < 16) return false;
   auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
   if (!al16(A) || !al16(B) || !al16(C) || (R && !al16(R))) return false;
-  if (u && (!al16(u->theta) || !al16(u->m) || !al16(u->v) || (u->g && !al16(u->g)) || (u->comp && !al16(u->comp))))
+  // the fused update: 16-byte aligned state rows, a compute copy, no accumulated gradient
+  if (u && (!al16(u->theta) || !al16(u->m) || !al16(u->v) || u->g || !u->comp || !al16(u->comp) || N % 8 != 0))
     return false;
   if (N % 8 != 0) return false;
   if ((mode == 0 || mode == 1) && K % 8 != 0) return false;
   if (mode >= 2 && M % 8 != 0) return false;
   int bn = 128, splits = 1;
-  tc::choose(mode == 4 ? 2 : mode, M, N, K, bn, splits);
+  tc::choose(mode == 4 ? 2 : mode, M, N, K, bn, splits, mode == 4);
   if (const char* force = std::getenv("ZL_GEMM_TILE")) {   // test hook "BN:SPLITS": forces the tile and split count
     int fb = 0, fs = 0;
     if (std::sscanf(force, "%d:%d", &fb, &fs) == 2 && (fb == 64 || fb == 128 || fb == 256) && fs >= 1 && fs <= 16) {
-      bn = fb;
+      bn = mode == 4 ? 128 : fb;
       splits = std::max(1, std::min(fs, (K + tc::BK - 1) / tc::BK));
     }
   }
@@ -633,6 +693,7 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   bool ok;
   if (mode == 0) ok = tc::launch_bn<false, false>(bn, a, A, B, s);
   else if (mode == 1) ok = tc::launch_bn<false, true>(bn, a, A, B, s);
+  else if (a.mode == 4) ok = tc::launch_upd(a, A, B, s);
   else ok = tc::launch_bn<true, true>(bn, a, A, B, s);
   if (ws) {
     if (ok) {
