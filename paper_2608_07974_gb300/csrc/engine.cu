@@ -96,7 +96,8 @@ struct Chunk {
   size_t fvec_n = 0, fmat_n = 0;
   std::vector<Layer> layers;
   size_t ad_down = 0, ad_up = 0;   // readout adapter D [r, d] and U [d, r] in the trainable slab
-  size_t n_layers_slab = 0;        // trainable floats before the adapter (what backpropagation updates)
+  size_t ad_end = 0;               // end of the adapter (= ad_down without one): vectors before, matrices after
+  size_t grad_n = 0;               // floats of the gradient accumulator (n, or ad_end with the fused update)
   int micro = 0;
   long t = 0;                // optimizer steps (host mirror of *d_t)
   long long* d_t = nullptr;  // optimizer steps on the device, advanced by the AdamW launch
@@ -228,9 +229,13 @@ float* Wm(Chunk& k, int li, PK p) {   // fp32 pointer of a vector (gain or bias)
   if (!L.has[p]) return nullptr;
   return L.slab[p] == S_FVEC ? k.fvec + L.off[p] : k.master + L.off[p];
 }
-float* Gm(Chunk& k, int li, PK p) {   // gradient accumulator; NULL for frozen tensors
+bool trainable(Chunk& k, int li, PK p) {
   const Layer& L = k.layers[li];
-  return (L.has[p] && L.slab[p] == S_TRAIN) ? k.grad + L.off[p] : nullptr;
+  return L.has[p] && L.slab[p] == S_TRAIN;
+}
+float* Gm(Chunk& k, int li, PK p) {   // gradient accumulator; NULL for frozen tensors and unstored gradients
+  const Layer& L = k.layers[li];
+  return (trainable(k, li, p) && L.off[p] < k.grad_n) ? k.grad + L.off[p] : nullptr;
 }
 int lora_r16(int r) { return r > 0 ? (r + 15) / 16 * 16 : 0; }
 
@@ -334,9 +339,10 @@ void G(zl_ctx* c, cudaStream_t s, int mode, int M, int N, int K, const void* A, 
 // rules) the gradient is formed with gemm() in the accumulator and the step applied to the matrix's
 // range right after it: the same arithmetic either way.
 void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, const void* A, const void* B) {
+  if (!trainable(k, li, p)) return;   // frozen
   float* g = Gm(k, li, p);
-  if (!g) return;   // frozen
   if (!k.fuse) {
+    if (!g) raise_err(ZL_ERR_STATE, "internal: unfused weight gradient without an accumulator");
     G(c, s, 2, M, N, K, A, B, g, nullptr, nullptr);
     return;
   }
@@ -350,9 +356,17 @@ void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, 
   const double upd = 24.0 * mn + (c->dt == BF16 ? 2.0 : 0.0) * mn;
   ProfScope ps(c, s, PC_GEMM_UPD, 2.0 * mn * (double)K, e * ((double)M * K + (double)N * K) + upd);
   if (c->dt == BF16 && gemm_tc_update(M, N, K, A, B, u, c->d_err, s, c->pool)) return;
-  gemm(c->dt, 2, M, N, K, A, B, g, nullptr, nullptr, s, c->d_err, c->pool);
-  launch_adamw_span(u.theta, g, u.m, u.v, u.comp, (size_t)M * N, k.d_hp, cf.beta1, cf.beta2, cf.eps, cf.weight_decay,
+  // the gradient in the accumulator (or, where the matrix has none, a zeroed pool buffer), then the step
+  float* tmp = nullptr;
+  if (!g) {
+    tmp = (float*)palloc(c, (size_t)M * N * 4, s);
+    CK(cudaMemsetAsync(tmp, 0, (size_t)M * N * 4, s));
+  }
+  float* gg = g ? g : tmp;
+  gemm(c->dt, 2, M, N, K, A, B, gg, nullptr, nullptr, s, c->d_err, c->pool);
+  launch_adamw_span(u.theta, gg, u.m, u.v, u.comp, (size_t)M * N, k.d_hp, cf.beta1, cf.beta2, cf.eps, cf.weight_decay,
                     u.gscale, s);
+  pfree(tmp, s);
 }
 
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
@@ -703,10 +717,18 @@ void adamw_window(zl_ctx* c, Chunk& k, cudaStream_t s, bool adapters = true) {
     CHECK_LAUNCH();
     return;
   }
-  const size_t n = (adapters || g.adapter_dim == 0) ? k.n : k.n_layers_slab;
-  ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * (double)n);
-  launch_adamw(k.master, k.grad, k.m, k.v, c->dt == BF16 ? k.comp : nullptr, n, k.d_t, k.d_hp, g.lr, g.lr_schedule,
-               g.lr_gamma, g.beta1, g.beta2, g.eps, g.weight_decay, gscale, s);
+  if (k.grad_n < k.n) raise_err(ZL_ERR_STATE, "internal: slab update without a full gradient accumulator");
+  void* comp = c->dt == BF16 ? k.comp : nullptr;
+  const bool skip_ad = !adapters && g.adapter_dim > 0;   // the slab but the adapter [ad_down, ad_end)
+  const size_t n1 = skip_ad ? k.ad_down : k.n;
+  const double nu = (double)(skip_ad ? k.n - (k.ad_end - k.ad_down) : k.n);
+  ProfScope p(c, s, PC_ADAMW, 0, (c->dt == BF16 ? 34.0 : 32.0) * nu);
+  launch_adamw(k.master, k.grad, k.m, k.v, comp, n1, k.d_t, k.d_hp, g.lr, g.lr_schedule, g.lr_gamma, g.beta1, g.beta2,
+               g.eps, g.weight_decay, gscale, s);
+  if (skip_ad)
+    launch_adamw_span(k.master + k.ad_end, k.grad + k.ad_end, k.m + k.ad_end, k.v + k.ad_end,
+                      comp ? (void*)((bf16*)comp + k.ad_end) : nullptr, k.n - k.ad_end, k.d_hp, g.beta1, g.beta2,
+                      g.eps, g.weight_decay, gscale, s);
   CHECK_LAUNCH();
 }
 
@@ -1132,21 +1154,43 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       // Full fine-tune: every layer tensor in the trainable slab. LoRA: the base matrices and the
       // vectors are frozen and only the factors A [r, in], B [out, r] of the four linears train.
       const int r = cfg->lora_rank;
+      // Trainable slab layout: every layer's vectors (norm gains, biases), then the readout adapter, then
+      // every layer's matrices (or LoRA factors). The gradient accumulator may stop after the adapter: with
+      // the fused update the matrices never need one.
       size_t off = 0, fvec = 0, fmat = 0;
+      const bool is_mat[P_COUNT] = {false, false, true, false, true, false, false, false, true, false, true, false};
       for (int l = ck.l0; l < ck.l1; ++l) {
         Layer L;
         size_t shp[P_COUNT] = {(size_t)d, (size_t)d, (size_t)c->qkvw * d, (size_t)c->qkvw, (size_t)d * c->ad, (size_t)d,
                                (size_t)d, (size_t)d, (size_t)c->f1 * d, (size_t)c->f, (size_t)d * c->f, (size_t)d};
         for (int p = 0; p < P_COUNT; ++p) {
           const bool bias = (p == P_N1B || p == P_BQKV || p == P_BO || p == P_N2B || p == P_B1 || p == P_B2);
-          const bool mat = (p == P_WQKV || p == P_WO || p == P_W1 || p == P_W2);
           L.has[p] = !(c->llama && bias);
           L.numel[p] = L.has[p] ? shp[p] : 0;
-          L.slab[p] = r == 0 ? S_TRAIN : (mat ? S_FMAT : S_FVEC);
+          L.slab[p] = r == 0 ? S_TRAIN : (is_mat[p] ? S_FMAT : S_FVEC);
+          L.off[p] = 0;
+          if (L.slab[p] == S_TRAIN && is_mat[p]) continue;   // second pass
           size_t& cur = L.slab[p] == S_TRAIN ? off : (L.slab[p] == S_FMAT ? fmat : fvec);
           L.off[p] = cur;
           if (L.has[p]) cur += round_up(shp[p], 64);
         }
+        ck.layers.push_back(L);
+      }
+      ck.ad_down = ck.ad_up = off;
+      if (cfg->adapter_dim > 0) {
+        const size_t ra = (size_t)cfg->adapter_dim;
+        ck.ad_down = off;
+        off += round_up(ra * d, 64);
+        ck.ad_up = off;
+        off += round_up((size_t)d * ra, 64);
+      }
+      ck.ad_end = off;
+      for (Layer& L : ck.layers) {
+        for (int p = 0; p < P_COUNT; ++p)
+          if (L.has[p] && L.slab[p] == S_TRAIN && is_mat[p]) {
+            L.off[p] = off;
+            off += round_up(L.numel[p], 64);
+          }
         // LoRA factors are stored with the rank padded to a multiple of 16 (rows beyond r stay exactly
         // zero: zero start, zero gradient), A as [r16, in] and B transposed as [r16, out], so every
         // LoRA product is a tensor-core GEMM.
@@ -1163,15 +1207,6 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
             off += round_up(r16 * outs[i], 64);
           }
         }
-        ck.layers.push_back(L);
-      }
-      ck.n_layers_slab = off;
-      if (cfg->adapter_dim > 0) {
-        const size_t ra = (size_t)cfg->adapter_dim;
-        ck.ad_down = off;
-        off += round_up(ra * d, 64);
-        ck.ad_up = off;
-        off += round_up((size_t)d * ra, 64);
       }
       ck.n = std::max<size_t>(off, 64);
       ck.fvec_n = fvec;
@@ -1211,12 +1246,17 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
                         cudaMemcpyHostToDevice));
         }
       }
+      // With the fused update always on (bf16 on the tensor cores, one micro-batch per window, full
+      // fine-tune) the matrices never hold a gradient: the accumulator covers the vectors and adapter only.
+      const bool fused_always = c->dt == BF16 && cfg->accum_m == 1 && !cfg->unfused_update && r == 0 &&
+                                gemm_tc_available();
+      ck.grad_n = fused_always ? std::max<size_t>(ck.ad_end, 64) : ck.n;
       ck.master = (float*)salloc(c, ck.n * 4);
-      ck.grad = (float*)salloc(c, ck.n * 4);
+      ck.grad = (float*)salloc(c, ck.grad_n * 4);
       ck.m = (float*)salloc(c, ck.n * 4);
       ck.v = (float*)salloc(c, ck.n * 4);
       CK(cudaMemset(ck.master, 0, ck.n * 4));
-      CK(cudaMemset(ck.grad, 0, ck.n * 4));
+      CK(cudaMemset(ck.grad, 0, ck.grad_n * 4));
       CK(cudaMemset(ck.m, 0, ck.n * 4));
       CK(cudaMemset(ck.v, 0, ck.n * 4));
       if (c->dt == BF16) {
@@ -1330,6 +1370,11 @@ zl_status zl_get_param(zl_ctx* c, const char* name, int which, void* dst, size_t
     if (which < 0 || which > 3 || (which > 0 && !f.chunk)) raise_err(ZL_ERR_ARG, "which: 0..3, 1..3 trainable only");
     sync_all(c, -1);
     const void* srcp = f.dev;
+    if (which == 1 && f.off >= f.chunk->grad_n) {   // a matrix whose gradient is never stored: it is zero
+      if (on_device) CK(cudaMemset(dst, 0, bytes));
+      else std::memset(dst, 0, bytes);
+      return ZL_OK;
+    }
     if (which > 0) {
       float* base = which == 1 ? f.chunk->grad : which == 2 ? f.chunk->m : f.chunk->v;
       srcp = base + f.off;
@@ -1517,7 +1562,8 @@ zl_status zl_chunk_save(zl_ctx* c, int k, void* dst, size_t bytes) {
     float* p = reinterpret_cast<float*>(static_cast<char*>(dst) + sizeof h);
     const size_t sz = ck.n * sizeof(float);
     CK(cudaMemcpy(p, ck.master, sz, cudaMemcpyDeviceToHost));
-    CK(cudaMemcpy(p + ck.n, ck.grad, sz, cudaMemcpyDeviceToHost));
+    CK(cudaMemcpy(p + ck.n, ck.grad, ck.grad_n * sizeof(float), cudaMemcpyDeviceToHost));
+    std::memset(p + ck.n + ck.grad_n, 0, (ck.n - ck.grad_n) * sizeof(float));   // unstored gradients are zero
     CK(cudaMemcpy(p + 2 * ck.n, ck.m, sz, cudaMemcpyDeviceToHost));
     CK(cudaMemcpy(p + 3 * ck.n, ck.v, sz, cudaMemcpyDeviceToHost));
     return ZL_OK;
@@ -1539,7 +1585,7 @@ zl_status zl_chunk_load(zl_ctx* c, int k, const void* src, size_t bytes) {
     const float* p = reinterpret_cast<const float*>(static_cast<const char*>(src) + sizeof h);
     const size_t sz = ck.n * sizeof(float);
     CK(cudaMemcpy(ck.master, p, sz, cudaMemcpyHostToDevice));
-    CK(cudaMemcpy(ck.grad, p + ck.n, sz, cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(ck.grad, p + ck.n, ck.grad_n * sizeof(float), cudaMemcpyHostToDevice));
     CK(cudaMemcpy(ck.m, p + 2 * ck.n, sz, cudaMemcpyHostToDevice));
     CK(cudaMemcpy(ck.v, p + 3 * ck.n, sz, cudaMemcpyHostToDevice));
     if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
