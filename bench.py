@@ -53,6 +53,8 @@ def parse():
                     help="replay each step as a captured CUDA graph (same GPU time here; more peak memory)")
     ap.add_argument("--adapter", type=int, default=0,
                     help="readout adapter width per chunk (0: static head; a multiple of 16)")
+    ap.add_argument("--loss-rows", type=int, default=0,
+                    help="readout, local objective and head backward in row slices of this many rows (0: whole)")
     ap.add_argument("--no-bp", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -344,7 +346,7 @@ def run_ours(args):
         e = zb.ZeroLock(w.dims, K, bounds, dtype=w.dtype, alpha=w.alpha, lr=w.lr, beta1=w.beta1, beta2=w.beta2,
                         eps=w.eps, weight_decay=w.weight_decay, max_live_chunks=max_live, serialize=serialize,
                         lora_rank=args.lora, lora_scale=16.0 / args.lora if args.lora else 1.0,
-                        adapter_dim=args.adapter, graph=args.graph)
+                        adapter_dim=args.adapter, graph=args.graph, loss_rows=args.loss_rows)
         e.load(params)
         return e
 
@@ -484,7 +486,7 @@ def run_ours(args):
                 "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
                 "config": {"workload": workload_desc(w, K, args.lora, args.adapter), "K": K, "bounds": bounds,
                            "global_batch": w.batch * world, "seq_len": w.seq, "max_live_chunks": args.max_live,
-                           "cuda_graph": args.graph,
+                           "cuda_graph": args.graph, "loss_rows": args.loss_rows,
                            "parallelism": f"replicas x{world}" if world > 1 else "single GPU, K streams",
                            "l2": "no flush: every step's working set (weights, AdamW state, logits) exceeds L2"},
                 "peak_hbm_gb": zl_peak / 1e9, "bp": bp,

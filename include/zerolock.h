@@ -95,6 +95,13 @@ typedef struct {
                             /*   chunk's matrices apply AdamW in their epilogue (no gradient stored), the */
                             /*   other trainable tensors get AdamW after the backward; 1: one AdamW over */
                             /*   the whole slab after the backward. Same results either way.            */
+  int loss_rows;            /* 0: each chunk's logits z_k (and the teacher's) exist for the whole       */
+                            /*   micro-batch, z_{k-1} reused as chunk k's teacher; R > 0: the readout,   */
+                            /*   local objective and head backward run over row slices of R rows (the    */
+                            /*   head fused with the loss, Eq. 2-5): per slice z and the teacher's logits */
+                            /*   (the frozen head on h_{k-1}, recomputed) are formed, the loss writes dz  */
+                            /*   over z and dn = dz W_lm follows, so vocab-sized buffers hold R rows.    */
+                            /*   Not with readout adapters (ZL_ERR_UNSUPPORTED).                         */
   int fuzz_delay_us;        /* scheduler fuzz (tests): > 0 sleeps the host a pseudo-random 0..this many  */
   unsigned fuzz_seed;       /*   microseconds (SplitMix64 stream of fuzz_seed) at every phase boundary of */
                             /*   an enqueue, so the GPU runs ahead in varying interleavings; 0 is off,   */
@@ -232,6 +239,17 @@ zl_status zl_kernel_launches(uint64_t* count);
 zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_t* labels, int N,
                            int V, int ldz, float alpha, int kl_dir, void* dz, float* row_loss,
                            float* loss, void* stream);
+
+/* The frozen head fused with the local objective (Eq. 2-5), over row slices: for rows i of n [N, d]
+ * (the final norm of h_k) and tn [N, d] (of h_{k-1}; NULL when alpha == 1), z = n W^T and t = tn W^T
+ * with W [ldw, d] the head (rows V.. ldw - 1 are padding and must be zero), the loss of
+ * zl_op_local_loss, and dn = dL/dn = dz W [N, d] (dtype; may alias n). Logits exist for
+ * rows_per_slice rows at a time only (1 <= rows_per_slice; the slice buffers and |Omega| come from the
+ * stream-ordered default pool of the device). row_loss [N] and *loss (device, fp32) as for
+ * zl_op_local_loss. ldw >= V, ldw % 8 == 0, d % 8 == 0; 1 <= N <= 2^24. */
+zl_status zl_op_head_loss(int dtype, const void* n, const void* tn, const void* W, const int32_t* labels, int N,
+                          int d, int V, int ldw, float alpha, int kl_dir, int rows_per_slice, void* dn,
+                          float* row_loss, float* loss, void* stream);
 
 /* Causal softmax attention with grouped KV heads (the attention of every transformer layer of
  * Eq. 1): qkv [B*S, (H + 2*Hkv)*hd] token-major (per row: H query heads, Hkv key heads, Hkv value

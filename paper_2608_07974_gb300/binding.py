@@ -23,7 +23,7 @@ ZL_NOALLOC_MAX_ROWS = 65536   # rows of zl_op_local_loss_noalloc's static scratc
 EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_load_weights", "zl_get_param", "zl_param_numel",
            "zl_embed", "zl_forward_chunk", "zl_local_step", "zl_step", "zl_bp_step", "zl_eval_global_loss",
            "zl_read_losses", "zl_join", "zl_synchronize", "zl_peak_bytes", "zl_reset_peak", "zl_last_error",
-           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_gemm", "zl_op_gemm_ex", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
+           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_head_loss", "zl_op_gemm", "zl_op_gemm_ex", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
            "zl_chunk_load", "zl_replay", "zl_wait_selftest"]
 
 
@@ -39,7 +39,7 @@ class zl_train_cfg(C.Structure):
                 ("accum_m", C.c_int), ("max_live_chunks", C.c_int), ("lr_schedule", C.c_int),
                 ("lr_gamma", C.c_float), ("serialize", C.c_int), ("lora_rank", C.c_int),
                 ("lora_scale", C.c_float), ("replay_depth", C.c_int), ("adapter_dim", C.c_int),
-                ("graph", C.c_int), ("unfused_update", C.c_int), ("fuzz_delay_us", C.c_int),
+                ("graph", C.c_int), ("unfused_update", C.c_int), ("loss_rows", C.c_int), ("fuzz_delay_us", C.c_int),
                 ("fuzz_seed", C.c_uint)]
 
 
@@ -77,6 +77,7 @@ def _load() -> C.CDLL:
         "zl_last_error": [],
         "zl_op_local_loss": [i, vp, vp, vp, i, i, i, f, i, vp, vp, vp, vp],
         "zl_op_local_loss_noalloc": [i, vp, vp, vp, i, i, i, f, i, vp, vp, vp],
+        "zl_op_head_loss": [i, vp, vp, vp, vp, i, i, i, i, f, i, i, vp, vp, vp, vp],
         "zl_op_gemm": [i, i, i, i, i, vp, vp, vp, vp],
         "zl_op_gemm_ex": [i, i, i, i, i, vp, vp, vp, vp, vp, i, vp],
         "zl_op_attention": [i, vp, vp, vp, i, i, i, i, i, vp],
@@ -267,6 +268,26 @@ def zl_op_local_loss_noalloc(dtype: int, z, t, labels, N: int, V: int, ldz: int,
                                          _p(loss), stream))
 
 
+def zl_op_head_loss(dtype: int, n, tn, W, labels, N: int, d: int, V: int, ldw: int, alpha: float, kl_dir: int,
+                    rows_per_slice: int, dn, row_loss, loss, stream: int = 0) -> None:
+    """The frozen head fused with the local objective over row slices (include/zerolock.h)."""
+    act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
+    for x, nm in ((n, "n"), (tn, "tn"), (W, "W"), (dn, "dn")):
+        _need(x, act, nm)
+    _need(labels, ("int32",), "labels")
+    _need(row_loss, ("float32",), "row_loss")
+    _need(loss, ("float32",), "loss")
+    if N >= 1 and d >= 1:
+        for x, nm in ((n, "n"), (tn, "tn"), (dn, "dn")):
+            _need_numel(x, N * d, nm)
+        _need_numel(W, ldw * d, "W")
+        _need_numel(labels, N, "labels")
+        _need_numel(row_loss, N, "row_loss")
+        _need_numel(loss, 1, "loss")
+    _check(_lib.zl_op_head_loss(dtype, _p(n), _p(tn), _p(W), _p(labels), N, d, V, ldw, alpha, kl_dir, rows_per_slice,
+                                _p(dn), _p(row_loss), _p(loss), stream))
+
+
 def zl_op_attention(dtype: int, qkv, out, lse, B: int, S: int, H: int, Hkv: int, hd: int, stream: int = 0) -> None:
     act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
     _need(qkv, act, "qkv")
@@ -357,8 +378,8 @@ class ZeroLock:
                  beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.01, accum_m: int = 1,
                  max_live_chunks: int = 0, lr_schedule: int = 0, lr_gamma: float = 1.0, serialize: bool = False,
                  lora_rank: int = 0, lora_scale: float = 1.0, replay_depth: int = 0, adapter_dim: int = 0,
-                 graph: bool = False, unfused_update: bool = False, fuzz_delay_us: int = 0, fuzz_seed: int = 0,
-                 stream=None):
+                 graph: bool = False, unfused_update: bool = False, loss_rows: int = 0, fuzz_delay_us: int = 0,
+                 fuzz_seed: int = 0, stream=None):
         import torch
         self.dims = dims
         self.K = K
@@ -369,7 +390,8 @@ class ZeroLock:
                            dims.norm_eps, dims.rope_theta)
         cfg = zl_train_cfg(alpha, kl_dir, consis_first, lr, beta1, beta2, eps, weight_decay, accum_m,
                            max_live_chunks, lr_schedule, lr_gamma, int(serialize), lora_rank, lora_scale,
-                           replay_depth, adapter_dim, int(graph), int(unfused_update), fuzz_delay_us, fuzz_seed)
+                           replay_depth, adapter_dim, int(graph), int(unfused_update), loss_rows, fuzz_delay_us,
+                           fuzz_seed)
         self.ctx = zl_create(md, K, list(bounds), cfg)
         s = stream if stream is not None else torch.cuda.current_stream()
         zl_set_stream(self.ctx, s.cuda_stream)

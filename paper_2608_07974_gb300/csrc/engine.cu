@@ -303,7 +303,7 @@ struct ProfScope {
   cudaEvent_t a = nullptr;
   ProfScope(zl_ctx* c_, cudaStream_t s_, int cls_, double fl, double by, double nl = 1)
       : c(c_), s(s_), cls(cls_), flops(fl), bytes(by), launches(nl) {
-    if (c->prof) {
+    if (c && c->prof) {
       a = take_ev(c);
       CK(cudaEventRecord(a, s));
     }
@@ -844,6 +844,65 @@ void readout_bwd(zl_ctx* c, const void* h, ReadoutSave& rs, const void* dz, void
   rs = ReadoutSave{};
 }
 
+// Readout (Eq. 2), local objective (Eq. 3-5) and head backward over row slices of R rows, so that the
+// vocab-sized logits exist for R rows at a time only (the head fused with the loss): for each slice
+// z_s = n_s W^T, t_s = tn_s W^T (the stop-gradient teacher, when tn is given), the fused loss writes
+// dz_s in place of z_s and the per-row losses, and (backward) dn_s = dz_s W. n, tn [N, d]: the final-norm
+// outputs of the chunk's hidden state and of its input; W [Vp, d] the frozen head (rows >= V zero);
+// count: |Omega| of all N rows (already counted); dn [N, d] may be n (slice s of n is read before dn_s
+// is written, in stream order); zb, tb: [R, Vp] slice buffers. c may be NULL (no profiling).
+void head_loss_rows(zl_ctx* c, int dt, const void* n, const void* tn, const void* W, const int32_t* labels, int N,
+                    int d, int V, int Vp, float alpha, int kl_dir, int R, const int* count, void* dn, float* rl,
+                    void* zb, void* tb, bool backward, cudaStream_t s, unsigned* err, cudaMemPool_t pool) {
+  const size_t e = dt_size(dt);
+  const double ed = (double)e;
+  auto gm = [&](int mode, int M, int Nn, int K, const void* A, const void* B, void* C) {
+    ProfScope p(c, s, PC_GEMM_HEAD, 2.0 * M * Nn * (double)K, ed * ((double)M * K + (double)Nn * K + (double)M * Nn));
+    gemm(dt, mode, M, Nn, K, A, B, C, nullptr, nullptr, s, err, pool);
+  };
+  const bool teacher = alpha < 1.f && tn;
+  for (int r0 = 0; r0 < N; r0 += R) {
+    const int rows = std::min(R, N - r0);
+    const size_t ro = (size_t)r0 * d * e;
+    gm(0, rows, Vp, d, (const char*)n + ro, W, zb);
+    if (teacher) gm(0, rows, Vp, d, (const char*)tn + ro, W, tb);
+    {
+      ProfScope p(c, s, PC_LOSS, 0, (teacher ? 3.0 : 2.0) * ed * (double)rows * Vp);
+      launch_local_loss(dt, zb, teacher ? tb : nullptr, labels + r0, rows, V, Vp, alpha, kl_dir, count, zb, rl + r0, s);
+    }
+    if (backward) gm(1, rows, d, Vp, zb, W, (char*)dn + ro);
+  }
+}
+
+// The readout, local objective and head backward of one chunk with the logits in row slices of
+// cfg.loss_rows rows (head_loss_rows): the teacher p_{k-1} is the frozen head on h_prev, the loss goes to
+// d_losses[slot] and, with backward, dh receives Norm_f'(h)^T dn. alpha == 1: no teacher (h_prev unused).
+void readout_loss_sliced(zl_ctx* c, const void* h, const void* h_prev, const int32_t* labels, float alpha, int N,
+                         int slot, void* dh, bool backward, cudaStream_t s) {
+  const size_t e = esz(c);
+  const int R = std::min(N, c->cfg.loss_rows);
+  void* n = palloc(c, (size_t)N * c->d * e, s);
+  float* st = (float*)palloc(c, (size_t)N * 8, s);
+  NF(c, s, h, c->normf_w, c->normf_b, n, st, st + N, N);
+  void *tn = nullptr, *tb = nullptr;
+  float* tst = nullptr;
+  if (alpha < 1.f) {
+    tn = palloc(c, (size_t)N * c->d * e, s);
+    tst = (float*)palloc(c, (size_t)N * 8, s);
+    NF(c, s, h_prev, c->normf_w, c->normf_b, tn, tst, tst + N, N);
+    tb = palloc(c, (size_t)R * c->Vp * e, s);
+  }
+  void* zb = palloc(c, (size_t)R * c->Vp * e, s);
+  float* rl = (float*)palloc(c, (size_t)N * 4, s);
+  launch_count_valid(labels, N, c->V, c->d_count + slot, c->d_err, s);
+  head_loss_rows(c, c->dt, n, tn, c->lm_head, labels, N, c->d, c->V, c->Vp, alpha, c->cfg.kl_dir, R, c->d_count + slot,
+                 n, rl, zb, tb, backward, s, c->d_err, c->pool);
+  launch_loss_reduce(rl, N, c->d_count + slot, c->d_losses + slot, s);
+  if (backward) NBX(c, s, h, c->normf_w, st, st + N, n, nullptr, dh, N);
+  CHECK_LAUNCH();
+  for (void* p : {(void*)rl, zb, tb, tn, (void*)tst, n, (void*)st}) pfree(p, s);
+}
+
 // Loss of chunk slot `slot` into d_losses[slot]; returns dz (pool memory, caller frees).
 void* local_loss(zl_ctx* c, const void* z, const void* t, const int32_t* labels, float alpha, int N, int slot,
                  cudaStream_t s) {
@@ -1079,9 +1138,14 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
   else if (cfg->lora_rank > 0 && !(std::isfinite(cfg->lora_scale))) why = "lora_scale must be finite";
   else if (cfg->fuzz_delay_us < 0 || cfg->fuzz_delay_us > 100000) why = "fuzz_delay_us must be in [0, 100000]";
   else if (cfg->unfused_update != 0 && cfg->unfused_update != 1) why = "unfused_update must be 0 or 1";
+  else if (cfg->loss_rows < 0) why = "loss_rows must be >= 0";
   for (int k = 1; why.empty() && k <= K; ++k)
     if (bounds[k] <= bounds[k - 1]) why = "bounds must be strictly increasing";
   if (!why.empty()) { g_err = "zl_create: " + why; return ZL_ERR_ARG; }
+  if (cfg->loss_rows > 0 && cfg->adapter_dim > 0) {
+    g_err = "zl_create: the row-sliced head (loss_rows > 0) does not take readout adapters";
+    return ZL_ERR_UNSUPPORTED;
+  }
 
   zl_ctx* c = new zl_ctx();
   zl_status st = guarded(nullptr, [&]() -> zl_status {
@@ -1452,8 +1516,9 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
     h_in = h0;
   }
   const float a = alpha_of(c, k);
+  const bool sliced = c->cfg.loss_rows > 0;
   void* t = nullptr;
-  if (a < 1.f) {   // teacher p_{k-1} = readout(h_{k-1}), recomputed from the detached input
+  if (a < 1.f && !sliced) {   // teacher p_{k-1} = readout(h_{k-1}), recomputed from the detached input
     t = palloc(c, zb, s);
     readout_fwd(c, h_in, t, nullptr, N, s);
   }
@@ -1461,19 +1526,25 @@ void local_step_impl(zl_ctx* c, int k, const void* h_in, const int32_t* ids, con
   ChunkActs acts;
   chunk_fwd_save(c, ck, h_in, hk, B, S, acts, s);
   if (h_out) CK(cudaMemcpyAsync(h_out, hk, hb, cudaMemcpyDeviceToDevice, s));
-  ph.next("zl chunk %d readout", k);
-  void* z = palloc(c, zb, s);
-  ReadoutSave rs;
-  Chunk* ad = c->cfg.adapter_dim > 0 ? &ck : nullptr;
-  readout_fwd(c, hk, z, &rs, N, s, ad);
-  ph.next("zl chunk %d loss", k);
-  void* dz = local_loss(c, z, t, labels, a, N, k, s);
-  pfree(z, s);
-  pfree(t, s);
-  ph.next("zl chunk %d backward", k);
   void* dh = palloc(c, hb, s);
-  readout_bwd(c, hk, rs, dz, dh, N, s, ad);
-  pfree(dz, s);
+  if (sliced) {
+    ph.next("zl chunk %d readout, loss and head backward", k);
+    readout_loss_sliced(c, hk, h_in, labels, a, N, k, dh, true, s);
+    ph.next("zl chunk %d backward", k);
+  } else {
+    ph.next("zl chunk %d readout", k);
+    void* z = palloc(c, zb, s);
+    ReadoutSave rs;
+    Chunk* ad = c->cfg.adapter_dim > 0 ? &ck : nullptr;
+    readout_fwd(c, hk, z, &rs, N, s, ad);
+    ph.next("zl chunk %d loss", k);
+    void* dz = local_loss(c, z, t, labels, a, N, k, s);
+    pfree(z, s);
+    pfree(t, s);
+    ph.next("zl chunk %d backward", k);
+    readout_bwd(c, hk, rs, dz, dh, N, s, ad);
+    pfree(dz, s);
+  }
   window_begin(c, ck, s);
   chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
   pfree(dh, s);
@@ -1709,7 +1780,8 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
   rec(c->ch[1].ev_h, s1);   // reused below as "h_0 ready" before chunk 1 records h_1
   cudaEvent_t ev_h0 = c->ev_aux;
   const float a1 = alpha_of(c, 1);
-  if (a1 < 1.f) {
+  const bool sliced = c->cfg.loss_rows > 0;   // each chunk forms its teacher slices from h_{k-1} itself
+  if (a1 < 1.f && !sliced) {
     wait_ev(c->aux, c->ch[1].ev_h);
     z[0] = palloc(c, zb, c->aux);
     readout_fwd(c, h[0], z[0], nullptr, N, c->aux);
@@ -1736,45 +1808,55 @@ void step_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, i
     ChunkActs acts;
     chunk_fwd_save(c, ck, h[k - 1], h[k], B, S, acts, s);
     rec(ck.ev_h, s);
-    ph.next("zl chunk %d readout", k);
-    z[k] = palloc(c, zb, s);
-    ReadoutSave rs;
-    readout_fwd(c, h[k], z[k], &rs, N, s, adp ? &ck : nullptr);
-    rec(ck.ev_z, s);
-    ph.next("zl chunk %d loss", k);
-    // S3: local objective against the stop-gradient teacher: the frozen head on h_{k-1}, which is
-    // chunk k-1's own readout z_{k-1} (reused) unless chunk k-1 read out through its adapter
-    void* teacher = nullptr;
-    void* own_t = nullptr;
-    if (a < 1.f) {
-      if (k == 1) {
-        wait_ev(s, ev_h0);
-        teacher = z[0];
-      } else if (adp) {
-        own_t = palloc(c, zb, s);
-        readout_fwd(c, h[k - 1], own_t, nullptr, N, s);
-        teacher = own_t;
-      } else {
-        wait_ev(s, c->ch[k - 1].ev_z);
-        teacher = z[k - 1];
-      }
-    }
-    void* dz = local_loss(c, z[k], teacher, labels, a, N, k, s);
-    rec(ck.ev_loss, s);
-    pfree(own_t, s);
-    // z_{k-1} is no longer needed once this loss and chunk k-1's own loss are done
-    if (k == 1) {
-      if (z[0]) { wait_ev(s, ev_h0); pfree(z[0], s); }
-    } else if (!adp) {
-      wait_ev(s, c->ch[k - 1].ev_loss);
-      pfree(z[k - 1], s);
-    }
-    if (k == K || adp) pfree(z[k], s);   // with adapters no later chunk reads z_k
-    ph.next("zl chunk %d backward", k);
     void* dh = palloc(c, hb, s);
-    readout_bwd(c, h[k], rs, dz, dh, N, s, adp ? &ck : nullptr);
-    pfree(dz, s);
-    rec(ck.ev_hb, s);
+    if (sliced) {
+      // readout, local objective against the frozen head on h_{k-1}, head backward, in row slices
+      ph.next("zl chunk %d readout, loss and head backward", k);
+      readout_loss_sliced(c, h[k], h[k - 1], labels, a, N, k, dh, true, s);
+      rec(ck.ev_z, s);
+      rec(ck.ev_loss, s);
+      rec(ck.ev_hb, s);
+      ph.next("zl chunk %d backward", k);
+    } else {
+      ph.next("zl chunk %d readout", k);
+      z[k] = palloc(c, zb, s);
+      ReadoutSave rs;
+      readout_fwd(c, h[k], z[k], &rs, N, s, adp ? &ck : nullptr);
+      rec(ck.ev_z, s);
+      ph.next("zl chunk %d loss", k);
+      // S3: local objective against the stop-gradient teacher: the frozen head on h_{k-1}, which is
+      // chunk k-1's own readout z_{k-1} (reused) unless chunk k-1 read out through its adapter
+      void* teacher = nullptr;
+      void* own_t = nullptr;
+      if (a < 1.f) {
+        if (k == 1) {
+          wait_ev(s, ev_h0);
+          teacher = z[0];
+        } else if (adp) {
+          own_t = palloc(c, zb, s);
+          readout_fwd(c, h[k - 1], own_t, nullptr, N, s);
+          teacher = own_t;
+        } else {
+          wait_ev(s, c->ch[k - 1].ev_z);
+          teacher = z[k - 1];
+        }
+      }
+      void* dz = local_loss(c, z[k], teacher, labels, a, N, k, s);
+      rec(ck.ev_loss, s);
+      pfree(own_t, s);
+      // z_{k-1} is no longer needed once this loss and chunk k-1's own loss are done
+      if (k == 1) {
+        if (z[0]) { wait_ev(s, ev_h0); pfree(z[0], s); }
+      } else if (!adp) {
+        wait_ev(s, c->ch[k - 1].ev_loss);
+        pfree(z[k - 1], s);
+      }
+      if (k == K || adp) pfree(z[k], s);   // with adapters no later chunk reads z_k
+      ph.next("zl chunk %d backward", k);
+      readout_bwd(c, h[k], rs, dz, dh, N, s, adp ? &ck : nullptr);
+      pfree(dz, s);
+      rec(ck.ev_hb, s);
+    }
     window_begin(c, ck, s);
     chunk_bwd(c, ck, acts, dh, nullptr, B, S, s);
     pfree(dh, s);
@@ -1854,16 +1936,21 @@ void bp_enqueue(zl_ctx* c, const int32_t* ids, const int32_t* labels, int B, int
     chunk_fwd_save(c, c->ch[k], h[k - 1], h[k], B, S, acts[k], s);
   }
   ph.next("zl bp readout and loss");
-  void* z = palloc(c, zb, s);
-  ReadoutSave rs;
-  readout_fwd(c, h[K], z, &rs, N, s);
-  void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
-  pfree(z, s);
-  ph.next("zl bp backward");
   void* dh = palloc(c, hb, s);
   void* dh2 = palloc(c, hb, s);
-  readout_bwd(c, h[K], rs, dz, dh, N, s);
-  pfree(dz, s);
+  if (c->cfg.loss_rows > 0) {
+    readout_loss_sliced(c, h[K], nullptr, labels, 1.f, N, 0, dh, true, s);
+    ph.next("zl bp backward");
+  } else {
+    void* z = palloc(c, zb, s);
+    ReadoutSave rs;
+    readout_fwd(c, h[K], z, &rs, N, s);
+    void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
+    pfree(z, s);
+    ph.next("zl bp backward");
+    readout_bwd(c, h[K], rs, dz, dh, N, s);
+    pfree(dz, s);
+  }
   for (int k = K; k >= 1; --k) {
     window_begin(c, c->ch[k], s);
     chunk_bwd(c, c->ch[k], acts[k], dh, k > 1 ? dh2 : nullptr, B, S, s);
@@ -1935,11 +2022,15 @@ zl_status zl_eval_global_loss(zl_ctx* c, const int32_t* ids, const int32_t* labe
       chunk_fwd_nosave(c, c->ch[k], a, b, B, S, s);
       std::swap(a, b);
     }
-    void* z = palloc(c, zb, s);
-    readout_fwd(c, a, z, nullptr, N, s);
-    void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
-    pfree(dz, s);
-    pfree(z, s);
+    if (c->cfg.loss_rows > 0) {
+      readout_loss_sliced(c, a, nullptr, labels, 1.f, N, 0, nullptr, false, s);
+    } else {
+      void* z = palloc(c, zb, s);
+      readout_fwd(c, a, z, nullptr, N, s);
+      void* dz = local_loss(c, z, nullptr, labels, 1.f, N, 0, s);
+      pfree(dz, s);
+      pfree(z, s);
+    }
     pfree(a, s);
     pfree(b, s);
     CK(cudaMemcpyAsync(c->h_losses, c->d_losses, 4, cudaMemcpyDeviceToHost, s));
@@ -2078,6 +2169,43 @@ zl_status zl_op_local_loss(int dtype, const void* z, const void* t, const int32_
     launch_local_loss(dtype, z, t, labels, N, V, ldz, alpha, kl_dir, cnt, dz, row_loss, s);
     launch_loss_reduce(row_loss, N, cnt, loss, s);
     CHECK_LAUNCH();
+    CK(cudaFreeAsync(cnt, s));
+    return ZL_OK;
+  });
+}
+
+zl_status zl_op_head_loss(int dtype, const void* n, const void* tn, const void* W, const int32_t* labels, int N, int d,
+                          int V, int ldw, float alpha, int kl_dir, int rows_per_slice, void* dn, float* row_loss,
+                          float* loss, void* stream) {
+  if (!n || !W || !labels || !dn || !row_loss || !loss) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if (dtype != 0 && dtype != 1) { g_err = "dtype"; return ZL_ERR_ARG; }
+  if (N < 1 || d < 8 || d % 8 != 0 || V < 2 || ldw < V || ldw % 8 != 0 || rows_per_slice < 1) {
+    g_err = "need N >= 1, d >= 8 with d % 8 == 0, V >= 2, ldw >= V with ldw % 8 == 0, rows_per_slice >= 1";
+    return ZL_ERR_ARG;
+  }
+  if (N > (1 << 24)) { g_err = "N above 2^24 rows (|Omega| is counted exactly up to 2^24)"; return ZL_ERR_ARG; }
+  if (!(alpha > 0.f && alpha <= 1.f) || (alpha < 1.f && !tn) || (kl_dir != 0 && kl_dir != 1)) {
+    g_err = "alpha in (0,1], tn required when alpha < 1, kl_dir 0/1";
+    return ZL_ERR_ARG;
+  }
+  return guarded(nullptr, [&]() -> zl_status {
+    cudaStream_t s = (cudaStream_t)stream;
+    const int R = std::min(N, rows_per_slice);
+    const size_t zb = (size_t)R * ldw * dt_size(dtype);
+    int* cnt = nullptr;
+    void *z = nullptr, *t = nullptr;
+    CK(cudaMallocAsync((void**)&cnt, 256, s));
+    CK(cudaMallocAsync(&z, zb, s));
+    if (alpha < 1.f) CK(cudaMallocAsync(&t, zb, s));
+    unsigned* err = (unsigned*)((char*)cnt + 128);
+    CK(cudaMemsetAsync(err, 0, 4, s));
+    launch_count_valid(labels, N, V, cnt, err, s);
+    head_loss_rows(nullptr, dtype, n, alpha < 1.f ? tn : nullptr, W, labels, N, d, V, ldw, alpha, kl_dir, R, cnt, dn,
+                   row_loss, z, t, true, s, nullptr, nullptr);
+    launch_loss_reduce(row_loss, N, cnt, loss, s);
+    CHECK_LAUNCH();
+    CK(cudaFreeAsync(z, s));
+    if (t) CK(cudaFreeAsync(t, s));
     CK(cudaFreeAsync(cnt, s));
     return ZL_OK;
   });

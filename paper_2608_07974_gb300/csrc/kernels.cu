@@ -805,11 +805,12 @@ __device__ __forceinline__ void loss_pass1_bf16(const bf16* zp, const bf16* tp, 
 }
 
 // One block per row of logits. Pass 1: base-2 online log-sum-exp of z and t and the KL cross term
-// (two full vectors per trip for loads in flight); pass 2 (the row is still in L2) writes dz.
+// (two full vectors per trip for loads in flight); pass 2 (the row is still in L2) writes dz. dz may be
+// z itself (in place): every element is read before it is written, by the same thread.
 template <typename T, bool TEACHER, int KLDIR>
-__device__ __forceinline__ void local_loss_row(const T* __restrict__ z, const T* __restrict__ t,
+__device__ __forceinline__ void local_loss_row(const T* z, const T* __restrict__ t,
                                                const int32_t* __restrict__ labels, int V, int ldz, float alpha,
-                                               const int* __restrict__ count, T* __restrict__ dz,
+                                               const int* __restrict__ count, T* dz,
                                                float* __restrict__ row_loss) {
   pdl_wait();
   pdl_trigger();
@@ -945,17 +946,17 @@ __device__ __forceinline__ void local_loss_row(const T* __restrict__ z, const T*
 
 // Two rows per SM (the compiler's own register choice) and three rows per SM (at most 40 registers).
 template <typename T, bool TEACHER, int KLDIR>
-__global__ void __launch_bounds__(1024) local_loss_k(const T* __restrict__ z, const T* __restrict__ t,
+__global__ void __launch_bounds__(1024) local_loss_k(const T* z, const T* __restrict__ t,
                                                      const int32_t* __restrict__ labels, int V, int ldz,
                                                      float alpha, const int* __restrict__ count,
-                                                     T* __restrict__ dz, float* __restrict__ row_loss) {
+                                                     T* dz, float* __restrict__ row_loss) {
   local_loss_row<T, TEACHER, KLDIR>(z, t, labels, V, ldz, alpha, count, dz, row_loss);
 }
 template <typename T, bool TEACHER, int KLDIR>
-__global__ void __launch_bounds__(512, 3) local_loss3_k(const T* __restrict__ z, const T* __restrict__ t,
+__global__ void __launch_bounds__(512, 3) local_loss3_k(const T* z, const T* __restrict__ t,
                                                         const int32_t* __restrict__ labels, int V, int ldz,
                                                         float alpha, const int* __restrict__ count,
-                                                        T* __restrict__ dz, float* __restrict__ row_loss) {
+                                                        T* dz, float* __restrict__ row_loss) {
   local_loss_row<T, TEACHER, KLDIR>(z, t, labels, V, ldz, alpha, count, dz, row_loss);
 }
 

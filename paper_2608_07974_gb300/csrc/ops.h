@@ -54,7 +54,7 @@ void launch_gelu_bwd(int dt, const void* x, const void* dy, void* dx, size_t n, 
 
 // |Omega| = #(labels >= 0); labels outside [-1, V) set ZL_DEVERR_BAD_LABEL.
 void launch_count_valid(const int32_t* labels, int N, int V, int* count, unsigned* err, cudaStream_t s);
-// Fused local objective: dz and per-row loss (Eq. 3-5). t may be NULL iff alpha == 1.
+// Fused local objective: dz and per-row loss (Eq. 3-5). t may be NULL iff alpha == 1. dz may be z.
 void launch_local_loss(int dt, const void* z, const void* t, const int32_t* labels, int N, int V, int ldz,
                        float alpha, int kl_dir, const int* count, void* dz, float* row_loss, cudaStream_t s);
 // *out = sum(row_loss) / count.
