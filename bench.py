@@ -76,13 +76,25 @@ def job_tokens_per_s(tokens_per_step: int, steps: int, world: int, max_ms: float
     return tokens_per_step * steps * world / (max_ms / 1e3)
 
 
+def class_ideal_s(v, pk):
+    """Ideal time of one kernel class: the larger of its algorithmic FLOPs at the measured sustained bf16
+    peak and its algorithmic bytes at the measured HBM copy rate (a GEMM with the optimizer step fused
+    into its epilogue is bound by the second)."""
+    return max(v["flops"] / (pk["bf16_tflops_sustained"] * 1e12), v["bytes"] / (pk["hbm_gbs"] * 1e9))
+
+
 def step_roofline(prof, steps: int, ms_per_step: float):
-    """Whole-step roofline: the step time if every tensor-core class ran at the measured sustained bf16
-    peak and every memory-bound class at the measured HBM copy rate (algorithmic FLOPs and bytes per
-    step from the live profile), and the measured step's fraction of it."""
+    """Whole-step roofline: the step time if every class ran at its bound (class_ideal_s; algorithmic FLOPs
+    and bytes per step from the live profile), split into tensor-bound and HBM-bound classes, and the
+    measured step's fraction of it."""
     pk, pk_kind = peaks()
-    t_tensor = sum(v["flops"] for v in prof.values() if v["flops"] > 0) / steps / (pk["bf16_tflops_sustained"] * 1e12)
-    t_hbm = sum(v["bytes"] for v in prof.values() if v["flops"] == 0) / steps / (pk["hbm_gbs"] * 1e9)
+    t_tensor = t_hbm = 0.0
+    for v in prof.values():
+        t = class_ideal_s(v, pk) / steps
+        if v["flops"] / (pk["bf16_tflops_sustained"] * 1e12) >= v["bytes"] / (pk["hbm_gbs"] * 1e9):
+            t_tensor += t
+        else:
+            t_hbm += t
     ideal_ms = (t_tensor + t_hbm) * 1e3
     return {"ideal_ms": ideal_ms, "tensor_ms": t_tensor * 1e3, "hbm_ms": t_hbm * 1e3, "measured_ms": ms_per_step,
             "frac": ideal_ms / ms_per_step if ms_per_step > 0 else None,
@@ -95,7 +107,7 @@ def roofline_of(prof):
     tot_ms = sum(v["ms"] for v in prof.values())
     dom = max(prof, key=lambda k: prof[k]["ms"])
     g = prof[dom]
-    tensor = g["flops"] > 0
+    tensor = g["flops"] / (pk["bf16_tflops_sustained"] * 1e12) >= g["bytes"] / (pk["hbm_gbs"] * 1e9)
     if tensor:
         achieved = g["flops"] / (g["ms"] / 1e3) / 1e12
         peak_v, unit, kind = pk["bf16_tflops_sustained"], "TFLOP/s", f"{pk_kind} bf16 sustained"

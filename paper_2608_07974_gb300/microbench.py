@@ -1,8 +1,9 @@
 """Single-kernel timings through the C ABI (CUDA events, after warm-up), for tuning and profiling.
 
     python -m paper_2608_07974_gb300.microbench loss [--rows 1024] [--vocab 50257] [--reps 4]
-    python -m paper_2608_07974_gb300.microbench gemm [--workload gpt2|llama-1b]
+    python -m paper_2608_07974_gb300.microbench gemm [--workload gpt2|llama-1b|llama-7b]
     python -m paper_2608_07974_gb300.microbench attention [--batch 8 --seq 512 --heads 12 --kv-heads 12 --head-dim 64]
+    python -m paper_2608_07974_gb300.microbench layer-step [--width 4096 --ffn 11008 --steps 2 --unfused]
 
 `loss` runs the fused local objective on random bf16 logits; `gemm` times the GEMM shapes of the
 GPT-2-small workload (12 layers, d 768, FFN 3072, vocab 50304 padded, 4096 tokens) or of the
@@ -72,11 +73,13 @@ def _shapes_of(d, d_qkv, f1, f, V, n=4096):
 
 # Llama-style 1.1B: d 2048, 32 query / 4 key-value heads of 64, SwiGLU 5632 (gate and up fused), vocab 32000
 LLAMA1B_SHAPES = _shapes_of(2048, 2560, 11264, 5632, 32000)
+# Llama-2-7B-shaped: d 4096, 32 heads of 128, SwiGLU 11008, vocab 32000, 2 x 1024 tokens
+LLAMA7B_SHAPES = _shapes_of(4096, 12288, 22016, 11008, 32000, n=2048)
 
 
 def gemm(args):
     B = _lib()
-    shapes = {"gpt2": GPT2_SHAPES, "llama-1b": LLAMA1B_SHAPES}[args.workload]
+    shapes = {"gpt2": GPT2_SHAPES, "llama-1b": LLAMA1B_SHAPES, "llama-7b": LLAMA7B_SHAPES}[args.workload]
     for name, mode, M, N, K in shapes:
         bf = torch.bfloat16
         if mode == 0:
@@ -107,6 +110,22 @@ def attention(args):
           f"bwd {b * 1e3:.1f} us ({2 * fl / b / 1e9:.0f} TFLOP/s, 4 matmuls counted)")
 
 
+def layer_step(args):
+    """Concurrent steps of one Llama-style layer as a one-chunk model (small enough for a full ncu capture
+    of every kernel of a step, with the optimizer step fused into the dW products unless --unfused)."""
+    _lib()
+    import synth
+    from paper_2608_07974_gb300.binding import ZeroLock
+    d = synth.ModelDims(synth.ARCH_LLAMA, 1, args.width, args.heads, args.heads, args.ffn, args.vocab, args.seq)
+    w = synth.Workload("layer", d, "bf16", batch=args.batch, seq=args.seq, K=1, steps=args.steps)
+    eng = ZeroLock(d, 1, [0, 1], dtype="bf16", alpha=0.5, unfused_update=args.unfused)
+    eng.load(synth.make_params(d, 1, device="cuda"))
+    ids, labels = (t.cuda() for t in synth.make_batch(w, 0))
+    ms = _time(lambda: eng.step(ids, labels, want_losses=False), args.steps)
+    eng.synchronize()
+    print(f"layer step d={args.width} ffn={args.ffn} {args.batch}x{args.seq} tokens: {ms * 1e3:.1f} us per step")
+
+
 def main():
     ap = argparse.ArgumentParser()
     sub = ap.add_subparsers(dest="cmd", required=True)
@@ -116,7 +135,7 @@ def main():
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--reps", type=int, default=4)
     p = sub.add_parser("gemm")
-    p.add_argument("--workload", choices=["gpt2", "llama-1b"], default="gpt2")
+    p.add_argument("--workload", choices=["gpt2", "llama-1b", "llama-7b"], default="gpt2")
     p.add_argument("--reps", type=int, default=20)
     p = sub.add_parser("attention")
     p.add_argument("--batch", type=int, default=8)
@@ -125,8 +144,17 @@ def main():
     p.add_argument("--kv-heads", type=int, default=12)
     p.add_argument("--head-dim", type=int, default=64)
     p.add_argument("--reps", type=int, default=10)
+    p = sub.add_parser("layer-step")
+    p.add_argument("--width", type=int, default=4096)
+    p.add_argument("--ffn", type=int, default=11008)
+    p.add_argument("--heads", type=int, default=32)
+    p.add_argument("--vocab", type=int, default=1024)
+    p.add_argument("--batch", type=int, default=2)
+    p.add_argument("--seq", type=int, default=1024)
+    p.add_argument("--steps", type=int, default=2)
+    p.add_argument("--unfused", action="store_true")
     args = ap.parse_args()
-    {"loss": loss, "gemm": gemm, "attention": attention}[args.cmd](args)
+    {"loss": loss, "gemm": gemm, "attention": attention, "layer-step": layer_step}[args.cmd](args)
 
 
 if __name__ == "__main__":

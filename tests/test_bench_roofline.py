@@ -40,3 +40,16 @@ def test_clock_summary_keeps_the_median_the_max_and_every_active_reason():
     c = bench.parse_clocks(text)
     assert c == {"sm_mhz": 1980.0, "sm_max_mhz": 2070.0, "reasons": ["hw_slowdown", "sw_power_cap"], "samples": 3}
     assert bench.parse_clocks("") is None
+
+
+def test_fused_update_class_is_bound_by_its_bytes():
+    """A class with both FLOPs and bytes (the dW product with the optimizer step in its epilogue) counts the
+    larger of its compute time and its memory time, and the roofline entry names the memory bound then."""
+    pk, _ = bench.peaks()
+    prof = {"gemm_update": {"flops": 1e-3 * pk["bf16_tflops_sustained"] * 1e12,
+                            "bytes": 3e-3 * pk["hbm_gbs"] * 1e9, "ms": 4.0, "launches": 2}}
+    r = bench.step_roofline(prof, 1, ms_per_step=4.0)
+    assert r["hbm_ms"] == pytest.approx(3.0) and r["tensor_ms"] == pytest.approx(0.0)
+    e = bench.roofline_of(prof)
+    assert e["bound"] == "hbm" and e["unit"] == "GB/s"
+    assert e["achieved"] == pytest.approx(3e-3 * pk["hbm_gbs"] / 4e-3)
