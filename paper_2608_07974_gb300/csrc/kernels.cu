@@ -557,10 +557,52 @@ __global__ void rope_k(T* __restrict__ qkv, const float2* __restrict__ cs, int N
   }
 }
 
+// Head dims with hd / 2 a multiple of 8: one thread per 8 rotation pairs (16-byte loads of both halves and
+// 64 bytes of the (cos, sin) table), blocks striding over token rows, no 64-bit index divisions.
+template <typename T>
+__global__ void rope8_k(T* __restrict__ qkv, const float2* __restrict__ cs, int N, int S, int nh, int hd, int ld,
+                        int inverse) {
+  pdl_wait();
+  pdl_trigger();
+  const int half = hd / 2, g8 = half / 8, per_row = nh * g8;
+  const float sg = inverse ? -1.f : 1.f;
+  for (int n = blockIdx.x; n < N; n += gridDim.x) {
+    const float2* c = cs + (size_t)(n % S) * half;
+    T* row = qkv + (size_t)n * ld;
+    for (int w = threadIdx.x; w < per_row; w += blockDim.x) {
+      const int hh = w / g8, i0 = (w - hh * g8) * 8;
+      T* p = row + hh * hd + i0;
+      float x1[8], x2[8], y1[8], y2[8];
+      Vec8<T>::load(p, x1);
+      Vec8<T>::load(p + half, x2);
+      const float4* c4 = reinterpret_cast<const float4*>(c + i0);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 t = c4[j];   // (cos, sin) of pairs i0 + 2j and i0 + 2j + 1
+        const float co[2] = {t.x, t.z}, sn[2] = {sg * t.y, sg * t.w};
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int q = 2 * j + e;
+          y1[q] = x1[q] * co[e] - x2[q] * sn[e];
+          y2[q] = x2[q] * co[e] + x1[q] * sn[e];
+        }
+      }
+      Vec8<T>::store(p, y1);
+      Vec8<T>::store(p + half, y2);
+    }
+  }
+}
+
 void launch_rope(int dt, void* qkv, const float* cs, int N, int S, int H, int Hkv, int hd, int inverse,
                  cudaStream_t s) {
   note_launch(1);
   const int nh = H + Hkv, ld = (H + 2 * Hkv) * hd;
+  if (hd % 16 == 0) {
+    const int th = 128, g = std::min(N, 152 * 16);
+    if (dt == BF16) launch_pdl(rope8_k<bf16>, g, th, 0, s, (bf16*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
+    else launch_pdl(rope8_k<float>, g, th, 0, s, (float*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
+    return;
+  }
   const int th = 256, g = grid_for((size_t)N * nh * (hd / 2), th);
   if (dt == BF16) launch_pdl(rope_k<bf16>, g, th, 0, s, (bf16*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);
   else launch_pdl(rope_k<float>, g, th, 0, s, (float*)qkv, (const float2*)cs, N, S, nh, hd, ld, inverse);

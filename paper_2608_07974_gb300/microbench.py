@@ -121,7 +121,12 @@ def layer_step(args):
     eng = ZeroLock(d, 1, [0, 1], dtype="bf16", alpha=0.5, unfused_update=args.unfused)
     eng.load(synth.make_params(d, 1, device="cuda"))
     ids, labels = (t.cuda() for t in synth.make_batch(w, 0))
-    ms = _time(lambda: eng.step(ids, labels, want_losses=False), args.steps)
+    from paper_2608_07974_gb300.binding import zl_join
+
+    def step():
+        eng.step(ids, labels, want_losses=False)
+        zl_join(eng.ctx)   # every stream of the engine back into the timing stream
+    ms = _time(step, args.steps)
     eng.synchronize()
     print(f"layer step d={args.width} ffn={args.ffn} {args.batch}x{args.seq} tokens: {ms * 1e3:.1f} us per step")
 
