@@ -97,6 +97,7 @@ struct Args {
   const bf16* R;
   unsigned* err;
   int tiles_m, tiles_n;
+  int group_m;                // tile rows per raster group (tile_coords)
   int splits, kb_per_split;   // split-K: unit u -> split u / tiles, k blocks [s*kps, min(nk, (s+1)*kps))
   float alpha;                // scale of the product
   int rmode;                  // R in modes 0/1: 0 adds it (residual); 1 multiplies by GELU'(R) (R = the GELU input)
@@ -110,8 +111,10 @@ __device__ __forceinline__ constexpr uint32_t idesc() {
          ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 }
 
-__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int& tm, int& tn) {
-  constexpr int G = 8;   // groups of 8 tile rows share B tiles in L2
+// Tile order: groups of G tile rows sweep the tile columns, so the rows of A a group reads and the
+// B tile a column of the group reads are each fetched from DRAM about once. The host picks G: all the
+// tile rows when the whole A operand fits well inside L2 (then every B tile is read once), else 8.
+__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int G, int& tm, int& tn) {
   const int per_group = G * tiles_n;
   const int gid = tile / per_group, first = gid * G;
   const int gm = min(tiles_m - first, G);
@@ -178,7 +181,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
     for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
       const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
       for (int kb = kb0; kb < kb1; ++kb) {
         if (!uwait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
@@ -267,7 +270,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     auto prefetch_chunk = [&](int unit, int k) {
       if (unit >= num_units || lane >= 16) return;
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
       const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * part + 64 * (k >> 1);
       if (row >= g.M || col >= g.N) return;
       const size_t at = (size_t)row * g.N + col;
@@ -281,7 +284,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     int it = 0;
     for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
       int ok = 1;
@@ -334,7 +337,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     int it = 0, nchunk = 0;
     for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, tm, tn);
+      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
       const int split = unit / num_tiles;
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
@@ -669,6 +672,7 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   a.u = u ? *u : GemmUpdate{};
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
   a.tiles_n = (N + bn - 1) / bn;
+  a.group_m = (double)M * K * 2.0 <= 48e6 ? a.tiles_m : std::min(8, a.tiles_m);
   const int nk = (K + tc::BK - 1) / tc::BK;
   a.kb_per_split = (nk + splits - 1) / splits;
   a.splits = (nk + a.kb_per_split - 1) / a.kb_per_split;   // no empty split (its slice would never be formed)
