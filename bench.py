@@ -101,7 +101,7 @@ def step_roofline(prof, steps: int, ms_per_step: float):
             "peak_kind": f"{pk_kind} bf16 sustained / HBM copy"}
 
 
-def roofline_of(prof):
+def roofline_of(prof, workload="llama7b"):
     """Roofline entry of the kernel class with the largest time share in a zl_profile_read result."""
     pk, pk_kind = peaks()
     tot_ms = sum(v["ms"] for v in prof.values())
@@ -114,7 +114,7 @@ def roofline_of(prof):
     else:
         achieved = g["bytes"] / (g["ms"] / 1e3) / 1e9
         peak_v, unit, kind = pk["hbm_gbs"], "GB/s", f"{pk_kind} HBM copy"
-    traffic = measured_traffic(dom)
+    traffic = measured_traffic(dom, workload)
     return {"bound": "tensor" if tensor else "hbm", "kernel": dom, "achieved": achieved, "peak": peak_v,
             "unit": unit, "frac": achieved / peak_v, "peak_kind": kind, "traffic": traffic,
             "launches": g["launches"],
@@ -123,13 +123,18 @@ def roofline_of(prof):
 
 
 # DRAM bytes per launch (read + write) from ncu captures, valid only for the kernel sources they were
-# taken on (sha256 prefix over the listed files, in order); any change to them makes the figure null.
+# taken on (sha256 prefix over the listed files, in order) and for the workload named; any change to the
+# sources makes the figure null. Llama-7B-shaped step (profiles/gemm_tc_llama7b_shapes.md and
+# profiles/gemm_update_llama7b_layer.md): layer GEMMs are the mean over the eight forward and dX shapes of
+# a layer (each once per layer and step); head GEMMs weight nine forwards (eight students and the first
+# teacher) against eight dX products; the fused dW + AdamW products are the mean over a layer's four.
 GEMM_SOURCES = ["gemm_tc.cu", "tcgen05.cuh"]
 TRAFFIC = {
-    # ncu dram__bytes_read.sum + dram__bytes_write.sum of the GPT-2 GEMM shapes (microbench gemm),
-    # averaged with the per-step launch mix: 12 layer GEMMs per layer; 5 head forwards, 4 head dX
-    "gemm_layer": {"sources": GEMM_SOURCES, "sha256": "77747b85c3adf6ff", "bytes_per_launch": 22319274.7},
-    "gemm_head": {"sources": GEMM_SOURCES, "sha256": "77747b85c3adf6ff", "bytes_per_launch": 643159296.0},
+    "llama7b": {
+        "gemm_layer": {"sources": GEMM_SOURCES, "sha256": "91a4a0621d6ae14d", "bytes_per_launch": 195639776.0},
+        "gemm_head": {"sources": GEMM_SOURCES, "sha256": "91a4a0621d6ae14d", "bytes_per_launch": 524555791.0},
+        "gemm_update": {"sources": GEMM_SOURCES, "sha256": "91a4a0621d6ae14d", "bytes_per_launch": 1392006656.0},
+    },
 }
 
 
@@ -142,8 +147,8 @@ def sources_sha(names):
     return h.hexdigest()[:16]
 
 
-def measured_traffic(cls):
-    ent = TRAFFIC.get(cls)
+def measured_traffic(cls, workload="llama7b"):
+    ent = TRAFFIC.get(workload, {}).get(cls)
     if not ent or ent["bytes_per_launch"] is None:
         return None
     if sources_sha(ent["sources"]) != ent["sha256"]:
@@ -419,7 +424,7 @@ def run_ours(args):
         zl(i)
     prof = zb.zl_profile_read(eng.ctx)
     zb.zl_profile(eng.ctx, False)
-    roof = roofline_of(prof)
+    roof = roofline_of(prof, args.workload if not (args.K or args.lora or args.adapter or args.loss_rows) else "")
     step_roof = step_roofline(prof, prof_steps, ms / args.steps)
     classes = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / prof_steps,
                    "TFLOP/s" if v["flops"] else "GB/s":
@@ -480,7 +485,7 @@ def run_ours(args):
     seng.close()
     del seng
     torch.cuda.empty_cache()
-    roof_serial = roofline_of(sprof)
+    roof_serial = roofline_of(sprof, args.workload if not (args.K or args.lora or args.adapter or args.loss_rows) else "")
     classes_serial = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / prof_steps}
                       for k, v in sprof.items() if v["launches"]}
 

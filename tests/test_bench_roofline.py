@@ -23,13 +23,14 @@ def test_step_roofline_is_flops_over_tensor_peak_plus_bytes_over_hbm():
 
 def test_traffic_figures_are_tied_to_the_kernel_sources(monkeypatch):
     sha = bench.sources_sha(bench.GEMM_SOURCES)
-    monkeypatch.setitem(bench.TRAFFIC, "gemm_layer",
-                        {"sources": bench.GEMM_SOURCES, "sha256": sha, "bytes_per_launch": 123.0})
-    assert bench.measured_traffic("gemm_layer") == 123.0
-    monkeypatch.setitem(bench.TRAFFIC, "gemm_layer",
-                        {"sources": bench.GEMM_SOURCES, "sha256": "0" * 16, "bytes_per_launch": 123.0})
-    assert bench.measured_traffic("gemm_layer") is None
-    assert bench.measured_traffic("no_such_class") is None
+    monkeypatch.setitem(bench.TRAFFIC, "w", {"gemm_layer": {"sources": bench.GEMM_SOURCES, "sha256": sha,
+                                                           "bytes_per_launch": 123.0}})
+    assert bench.measured_traffic("gemm_layer", "w") == 123.0
+    assert bench.measured_traffic("gemm_layer", "other") is None       # figures belong to one workload
+    monkeypatch.setitem(bench.TRAFFIC, "w", {"gemm_layer": {"sources": bench.GEMM_SOURCES, "sha256": "0" * 16,
+                                                           "bytes_per_launch": 123.0}})
+    assert bench.measured_traffic("gemm_layer", "w") is None
+    assert bench.measured_traffic("no_such_class", "w") is None
 
 
 def test_clock_summary_keeps_the_median_the_max_and_every_active_reason():
