@@ -155,19 +155,110 @@ __global__ void attn_bwd_dkv_k(const T* __restrict__ qkv, const T* __restrict__ 
 }
 
 inline int warps_grid(long rows) { return (int)((rows * 32 + 255) / 256); }
+
+// Head padding for the tcgen05 kernels (head dims 64 and 128): dst [N, nh * hp] from src [N, nh * hd] with
+// each head's columns hd .. hp - 1 zero (pad), or src [N, nh * hp] back to dst [N, nh * hd] (unpad).
+// Zero query and key columns add nothing to Q K^T, zero value columns give zero output columns, and the
+// gradients of the padding columns are zero, so the padded products are the unpadded ones. bf16 pairs.
+__global__ void heads_pad_k(const __nv_bfloat162* __restrict__ src, __nv_bfloat162* __restrict__ dst, int N, int nh,
+                            int hd, int hp, int pad) {
+  pdl_wait();
+  pdl_trigger();
+  const int h2 = hd / 2, p2 = hp / 2;
+  const int src_w = (pad ? h2 : p2) * nh, dst_w = (pad ? p2 : h2) * nh, cols = nh * (pad ? p2 : h2);
+  const __nv_bfloat162 zero = __floats2bfloat162_rn(0.f, 0.f);
+  for (int n = blockIdx.x; n < N; n += gridDim.x) {
+    const __nv_bfloat162* sr = src + (size_t)n * src_w;
+    __nv_bfloat162* dr = dst + (size_t)n * dst_w;
+    for (int c = threadIdx.x; c < cols; c += blockDim.x) {
+      if (pad) {
+        const int h = c / p2, e = c - h * p2;
+        dr[c] = e < h2 ? sr[h * h2 + e] : zero;
+      } else {
+        const int h = c / h2, e = c - h * h2;
+        dr[c] = sr[h * p2 + e];
+      }
+    }
+  }
+}
+
+void heads_pad(const void* src, void* dst, int N, int nh, int hd, int hp, bool pad, cudaStream_t s) {
+  note_launch(1);
+  launch_pdl(heads_pad_k, std::min(N, 152 * 16), 256, 0, s, (const __nv_bfloat162*)src, (__nv_bfloat162*)dst, N, nh, hd,
+             hp, pad ? 1 : 0);
+}
+
+// The tcgen05 head dim a bf16 head of hd columns is padded to, or 0 when it runs as it is (64, 128) or
+// on the mma.sync kernels (odd, or above 128).
+int padded_hd(int hd) {
+  if (hd == 64 || hd == 128 || hd % 2 != 0 || hd > 128) return 0;
+  return hd < 64 ? 64 : 128;
+}
+
+void* scratch(size_t bytes, cudaStream_t s, cudaMemPool_t pool) {
+  void* p = nullptr;
+  const cudaError_t e = pool ? cudaMallocFromPoolAsync(&p, bytes, pool, s) : cudaMallocAsync(&p, bytes, s);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return p;
+}
 }  // namespace
 
 bool attn_fwd_tc(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s);
 bool attn_fwd_tcgen05(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
-                      unsigned* err);
+                      unsigned* err, float scale);
 bool attn_bwd_tc(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B, int S,
                  int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool);
 bool attn_bwd_tcgen05(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv,
-                      int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err);
+                      int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err,
+                      float scale);
+
+namespace {
+// bf16 heads of a dim the tcgen05 kernels do not take: zero-padded copies through them (padded_hd).
+bool attn_fwd_padded(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
+                     unsigned* err, cudaMemPool_t pool) {
+  const int hp = padded_hd(hd), N = B * S, nh = H + 2 * Hkv;
+  if (!hp) return false;
+  void* qp = scratch((size_t)N * nh * hp * 2, s, pool);
+  void* op = qp ? scratch((size_t)N * H * hp * 2, s, pool) : nullptr;
+  bool ok = op != nullptr;
+  if (ok) {
+    heads_pad(qkv, qp, N, nh, hd, hp, true, s);
+    ok = attn_fwd_tcgen05(qp, op, lse, B, S, H, Hkv, hp, s, err, 1.f / sqrtf((float)hd));
+    if (ok) heads_pad(op, out, N, H, hd, hp, false, s);
+  }
+  if (op) cudaFreeAsync(op, s);
+  if (qp) cudaFreeAsync(qp, s);
+  return ok;
+}
+
+bool attn_bwd_padded(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B,
+                     int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
+  const int hp = padded_hd(hd), N = B * S, nh = H + 2 * Hkv;
+  if (!hp) return false;
+  const size_t wq = (size_t)N * nh * hp * 2, wo = (size_t)N * H * hp * 2;
+  void* buf = scratch(2 * wq + 2 * wo, s, pool);
+  if (!buf) return false;
+  char* qp = (char*)buf;
+  char* dqp = qp + wq;
+  char* op = dqp + wq;
+  char* dop = op + wo;
+  heads_pad(qkv, qp, N, nh, hd, hp, true, s);
+  heads_pad(out, op, N, H, hd, hp, true, s);
+  heads_pad(dout, dop, N, H, hd, hp, true, s);
+  const bool ok = attn_bwd_tcgen05(qp, op, dop, lse, D, dqp, B, S, H, Hkv, hp, s, pool, err, 1.f / sqrtf((float)hd));
+  if (ok) heads_pad(dqp, dqkv, N, nh, hd, hp, false, s);
+  cudaFreeAsync(buf, s);
+  return ok;
+}
+}  // namespace
 
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
-              unsigned* err) {
-  if (dt == BF16 && attn_fwd_tcgen05(qkv, out, lse, B, S, H, Hkv, hd, s, err)) return;
+              unsigned* err, cudaMemPool_t pool) {
+  if (dt == BF16 && attn_fwd_tcgen05(qkv, out, lse, B, S, H, Hkv, hd, s, err, 1.f / sqrtf((float)hd))) return;
+  if (dt == BF16 && attn_fwd_padded(qkv, out, lse, B, S, H, Hkv, hd, s, err, pool)) return;
   note_launch(1);
   if (dt == BF16 && attn_fwd_tc(qkv, out, lse, B, S, H, Hkv, hd, s)) return;
   const float scale = 1.f / sqrtf((float)hd);
@@ -181,7 +272,8 @@ void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const 
   note_launch(dt == BF16 ? (H > Hkv ? 3 : 2) : 3);
   const float scale = 1.f / sqrtf((float)hd);
   const int gq = warps_grid((long)B * H * S), gk = warps_grid((long)B * Hkv * S);
-  if (dt == BF16 && attn_bwd_tcgen05(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s, pool, err)) return;
+  if (dt == BF16 && attn_bwd_tcgen05(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s, pool, err, scale)) return;
+  if (dt == BF16 && attn_bwd_padded(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s, pool, err)) return;
   if (dt == BF16 && attn_bwd_tc(qkv, out, dout, lse, Dbuf, dqkv, B, S, H, Hkv, hd, s, pool)) return;
   if (dt == BF16) {
     attn_bwd_d_k<bf16><<<gq, 256, 0, s>>>((const bf16*)out, (const bf16*)dout, Dbuf, B, S, H, hd);

@@ -1475,7 +1475,7 @@ bool qkv_map(CUtensorMap* m, const void* qkv, int B, int S, int W, int rows) {
 
 template <int HD>
 bool bwd_launch(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B,
-                int S, int H, int Hkv, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
+                int S, int H, int Hkv, cudaStream_t s, cudaMemPool_t pool, unsigned* err, float scale) {
   using C_ = BCfg<HD>;
   static bool attr = false;
   auto kq = attn_bwd_dq_tg_k<HD>;
@@ -1497,7 +1497,6 @@ bool bwd_launch(const void* qkv, const void* out, const void* dout, const float*
     cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&part, bytes, pool, s) : cudaMallocAsync((void**)&part, bytes, s);
     if (e != cudaSuccess) { cudaGetLastError(); return false; }
   }
-  const float scale = 1.f / sqrtf((float)HD);
   const int nqb = (S + 127) / 128;
   cudaError_t e = launch_pdl(kq, dim3(H, B, nqb), NTHR_B, C_::SMEM_DQ, s, q128, do128, q64, (const bf16*)out,
                              (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, scale, err);
@@ -1514,7 +1513,7 @@ bool bwd_launch(const void* qkv, const void* out, const void* dout, const float*
 // The 128-wide backward (head dim 64).
 template <int HD>
 bool bwd_w_launch(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv, int B,
-                  int S, int H, int Hkv, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
+                  int S, int H, int Hkv, cudaStream_t s, cudaMemPool_t pool, unsigned* err, float scale) {
   using C_ = WCfg<HD>;
   static bool attr = false;
   auto kq = attn_bwd_dq_w_k<HD>;
@@ -1534,7 +1533,6 @@ bool bwd_w_launch(const void* qkv, const void* out, const void* dout, const floa
     cudaError_t e = pool ? cudaMallocFromPoolAsync((void**)&part, bytes, pool, s) : cudaMallocAsync((void**)&part, bytes, s);
     if (e != cudaSuccess) { cudaGetLastError(); return false; }
   }
-  const float scale = 1.f / sqrtf((float)HD);
   const int nqb = (S + 127) / 128;
   cudaError_t e = launch_pdl(kq, dim3(H, B, nqb), NTHR_B, C_::SMEM_DQ, s, q128, do128, q128, (const bf16*)out,
                              (const bf16*)dout, lse, D, (bf16*)dqkv, S, H, Hkv, scale, err);
@@ -1549,7 +1547,8 @@ bool bwd_w_launch(const void* qkv, const void* out, const void* dout, const floa
 }
 
 template <int HD>
-bool fwd1_launch(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, cudaStream_t s, unsigned* err) {
+bool fwd1_launch(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, cudaStream_t s, unsigned* err,
+                 float scale) {
   using C_ = F1Cfg<HD>;
   static bool attr = false;
   auto kern = attn_fwd1_tg_k<HD>;
@@ -1561,35 +1560,36 @@ bool fwd1_launch(const void* qkv, void* out, float* lse, int B, int S, int H, in
   CUtensorMap tqk, tvv;
   if (!qkv_map(&tqk, qkv, B, S, W, 128) || !qkv_map(&tvv, qkv, B, S, W, 64)) return false;
   const dim3 grid(H, B, (S + QB - 1) / QB);
-  return launch_pdl(kern, grid, NTHR, C_::SMEM, s, tqk, tvv, (bf16*)out, lse, S, H, Hkv, 1.f / sqrtf((float)HD),
-                    err) == cudaSuccess;
+  return launch_pdl(kern, grid, NTHR, C_::SMEM, s, tqk, tvv, (bf16*)out, lse, S, H, Hkv, scale, err) == cudaSuccess;
 }
 
 }  // namespace tg
 
 // Returns false when the shape is outside this kernel (head dim 64 or 128, alignment, no sm_103a); the
-// caller uses the mma.sync kernel then.
+// caller uses the mma.sync kernel then. scale: the softmax scale (1 / sqrt of the true head dim when the
+// heads are zero-padded up to hd).
 bool attn_fwd_tcgen05(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
-                      unsigned* err) {
+                      unsigned* err, float scale) {
   if (hd != 64 && hd != 128) return false;
   if (((uintptr_t)qkv & 15u) || ((uintptr_t)out & 15u) || B > 65535 || (S + tg::QB - 1) / tg::QB > 65535) return false;
   if (!tg::enc_init()) return false;
   note_launch(1);
-  return hd == 64 ? tg::fwd1_launch<64>(qkv, out, lse, B, S, H, Hkv, s, err)
-                  : tg::fwd1_launch<128>(qkv, out, lse, B, S, H, Hkv, s, err);
+  return hd == 64 ? tg::fwd1_launch<64>(qkv, out, lse, B, S, H, Hkv, s, err, scale)
+                  : tg::fwd1_launch<128>(qkv, out, lse, B, S, H, Hkv, s, err, scale);
 }
 
 // Returns false when the shape is outside these kernels (head dim 64 or 128, alignment, no sm_103a) or the
 // grouped-head partials could not be allocated; the caller then uses the mma.sync kernels.
 bool attn_bwd_tcgen05(const void* qkv, const void* out, const void* dout, const float* lse, float* D, void* dqkv,
-                      int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err) {
+                      int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool, unsigned* err,
+                      float scale) {
   if (hd != 64 && hd != 128) return false;
   if ((((uintptr_t)qkv | (uintptr_t)out | (uintptr_t)dout | (uintptr_t)dqkv) & 15u) || B > 65535 ||
       (S + 127) / 128 > 65535)
     return false;
   if (!tg::enc_init()) return false;
-  return hd == 64 ? tg::bwd_w_launch<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err)
-                  : tg::bwd_launch<128>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err);
+  return hd == 64 ? tg::bwd_w_launch<64>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err, scale)
+                  : tg::bwd_launch<128>(qkv, out, dout, lse, D, dqkv, B, S, H, Hkv, s, pool, err, scale);
 }
 
 }  // namespace zl

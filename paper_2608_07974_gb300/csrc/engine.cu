@@ -372,7 +372,7 @@ void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, 
 void AF(zl_ctx* c, cudaStream_t s, const void* qkv, void* out, float* lse, int B, int S) {
   const double e = (double)esz(c), N = (double)B * S;
   ProfScope p(c, s, PC_ATTN_F, 2.0 * B * c->H * (double)S * S * c->hd, e * N * (c->qkvw + c->ad));
-  attn_fwd(c->dt, qkv, out, lse, B, S, c->H, c->Hkv, c->hd, s, c->d_err);
+  attn_fwd(c->dt, qkv, out, lse, B, S, c->H, c->Hkv, c->hd, s, c->d_err, c->pool);
 }
 void AB(zl_ctx* c, cudaStream_t s, const void* qkv, const void* out, const void* dout, const float* lse, float* D,
         void* dqkv, int B, int S) {

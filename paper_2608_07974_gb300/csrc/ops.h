@@ -113,11 +113,14 @@ void gemm_simt(int dt, int mode, int M, int N, int K, const void* A, const void*
 
 // Causal attention over qkv [N, (H + 2 Hkv) hd] (token-major, rows b*S + s): out [N, H hd], lse [B, H, S].
 // bf16 with head dim 64 or 128: the one-pass tcgen05 kernel (err: device word for its bounded waits, may
-// be NULL); other bf16 shapes: mma.sync; fp32: CUDA cores.
+// be NULL); other even bf16 head dims up to 128: the same kernel on copies zero-padded to 64 or 128 (pool:
+// where the copies come from, NULL = the device's default pool), mma.sync if they cannot be had; fp32:
+// CUDA cores.
 void attn_fwd(int dt, const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd,
-              cudaStream_t s, unsigned* err = nullptr);
+              cudaStream_t s, unsigned* err = nullptr, cudaMemPool_t pool = nullptr);
 // Gradients into dqkv (same layout as qkv). Dbuf: [B, H, S] scratch. bf16 with head dim 64 or 128: the
-// tcgen05 kernels (err as for attn_fwd); other bf16 shapes: mma.sync; fp32: CUDA cores.
+// tcgen05 kernels (err as for attn_fwd); other even bf16 head dims up to 128: the tcgen05 kernels on
+// zero-padded copies; else mma.sync; fp32: CUDA cores.
 void attn_bwd(int dt, const void* qkv, const void* out, const void* dout, const float* lse, float* Dbuf,
               void* dqkv, int B, int S, int H, int Hkv, int hd, cudaStream_t s, cudaMemPool_t pool = nullptr,
               unsigned* err = nullptr);
