@@ -123,13 +123,24 @@ __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, 
   tn = r / gm;
 }
 
+// Tile (tm, tn) of work unit `unit`. PAIR: units are pairs of vertically adjacent tiles sharing their B
+// tile; the CTA of cluster rank r takes the pair's tile row 2 tmp + r.
+__device__ __forceinline__ void unit_tile(const Args& g, int unit, int num_tiles, bool pair, uint32_t crank, int& tm,
+                                          int& tn) {
+  tile_coords(unit % num_tiles, pair ? (g.tiles_m + 1) / 2 : g.tiles_m, g.tiles_n, g.group_m, tm, tn);
+  if (pair) tm = 2 * tm + (int)crank;
+}
+
 // UPD: the fused optimizer epilogue (mode 4) is compiled in (a kernel of its own, so the other modes keep
-// their register budget).
-template <int BN, bool A_MN, bool B_MN, bool UPD = false>
+// their register budget). PAIR: the CTA runs in a cluster of two that share each B tile: each loads half
+// of it and multicasts it to both (TMA), each CTA's MMA commit frees the stage in both, so every SM copies
+// half as much of B from L2 as alone.
+template <int BN, bool A_MN, bool B_MN, bool UPD = false, bool PAIR = false>
 __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     gemm_tc_k(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
               const __grid_constant__ CUtensorMap tcm, const Args g, const __grid_constant__ UpdMaps um) {
   using C_ = Cfg<BN, UPD>;
+  constexpr uint16_t kPairMask = 3;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* outbuf = smem + C_::STAGES * C_::STAGE_BYTES;   // 1024-byte aligned (stage sizes are)
@@ -143,7 +154,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < C_::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int s = 0; s < C_::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], PAIR ? 2 : 1); }
     for (int a = 0; a < 2; ++a) { mbar_init(&tfull[a], 1); mbar_init(&tempty[a], UPD ? 8 : 4); }
     mbar_init(fin, 1);
     *abort_flag = 0;
@@ -158,6 +169,11 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
   fence_before();
   __syncthreads();
   fence_after();
+  // a pair's copies land in both CTAs' shared memory: both sets of barriers exist before any is issued
+  if (PAIR) cluster_sync();
+  const uint32_t crank = PAIR ? cluster_rank() : 0u;
+  const int unit0 = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int ustride = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
   const uint32_t tmem = *tbase;
   // Programmatic dependent launch: the set-up above may overlap the previous kernel of the stream;
   // every thread waits for that kernel (and its memory) before touching global memory, and lets the
@@ -165,7 +181,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int nk = (g.K + BK - 1) / BK;
-  const int num_tiles = g.tiles_m * g.tiles_n;
+  const int num_tiles = (PAIR ? (g.tiles_m + 1) / 2 : g.tiles_m) * g.tiles_n;
   const int num_units = num_tiles * g.splits;
 
   if (warp == 0) {
@@ -179,9 +195,9 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     int issued[C_::STAGES];   // parity of the last fill of each stage, -1 if none
 #pragma unroll
     for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
-    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
+    for (int unit = unit0; ok && unit < num_units; unit += ustride) {
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
+      unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
       const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
       for (int kb = kb0; kb < kb1; ++kb) {
         if (!uwait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
@@ -197,7 +213,18 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
             tma2d(sa, &ta, &full[stage], tm * BM, k0);
             tma2d(sa + 8192, &ta, &full[stage], tm * BM + 64, k0);
           }
-          if (!B_MN) {
+          if (PAIR) {   // this CTA's half of the B tile, into both CTAs
+            constexpr int HB = BN / 2;
+            if (!B_MN) {
+              tma2d_mc(sb + crank * (HB * 128), &tb, &full[stage], k0, tn * BN + (int)crank * HB, kPairMask);
+            } else {
+#pragma unroll
+              for (int j = 0; j < HB / 64; ++j) {
+                const int jj = (int)crank * (HB / 64) + j;
+                tma2d_mc(sb + jj * 8192, &tb, &full[stage], tn * BN + 64 * jj, k0, kPairMask);
+              }
+            }
+          } else if (!B_MN) {
             tma2d(sb, &tb, &full[stage], k0, tn * BN);
           } else {
 #pragma unroll
@@ -207,6 +234,13 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
         __syncwarp();
         if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
       }
+    }
+    if (PAIR && ok) {
+      // both CTAs' commits for the last fill of every stage have arrived: no arrival from the peer (and no
+      // copy of this CTA's into the peer) is still on its way when the CTAs exit
+#pragma unroll 1
+      for (int s = 0; s < C_::STAGES; ++s)
+        if (issued[s] >= 0 && !uwait(&empty[s], (uint32_t)issued[s], abort_flag, g.err)) break;
     }
     if (!ok && lane == 0) {   // unwinding: let the copies already in flight land before the CTA exits
       for (int s = 0; s < C_::STAGES; ++s) {
@@ -225,7 +259,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     int stage = 0, it = 0;
     uint32_t phase = 0;
     bool ok = true;
-    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++it) {
+    for (int unit = unit0; ok && unit < num_units; unit += ustride, ++it) {
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
       if (!uwait(&tempty[acc], aph ^ 1u, abort_flag, g.err)) break;
@@ -243,7 +277,8 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
             const uint64_t bd = B_MN ? sdesc(b0 + kk * 2048, 8192, 1024) : sdesc(b0 + kk * 32, 16, 1024);
             mma_bf16(d, ad, bd, id, (kb > kb0 || kk > 0) ? 1u : 0u);
           }
-          mma_commit(&empty[stage]);
+          if (PAIR) mma_commit_mc(&empty[stage], kPairMask);   // the stage is free in both CTAs' view
+          else mma_commit(&empty[stage]);
         }
         __syncwarp();
         if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
@@ -270,7 +305,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     auto prefetch_chunk = [&](int unit, int k) {
       if (unit >= num_units || lane >= 16) return;
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
+      unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
       const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * part + 64 * (k >> 1);
       if (row >= g.M || col >= g.N) return;
       const size_t at = (size_t)row * g.N + col;
@@ -280,11 +315,11 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     };
     constexpr int PD = 2;   // prefetch distance in chunks (2 and 3 measured alike, 4 slower)
 #pragma unroll
-    for (int k = 0; k < PD; ++k) prefetch_chunk(blockIdx.x + (k / NC) * gridDim.x, k % NC);
+    for (int k = 0; k < PD; ++k) prefetch_chunk(unit0 + (k / NC) * ustride, k % NC);
     int it = 0;
-    for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
+    for (int unit = unit0; unit < num_units; unit += ustride, ++it) {
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
+      unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
       int ok = 1;
@@ -316,7 +351,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int k2 = 2 * p + h + PD;   // PD chunks ahead, into the next tiles at the end
-          prefetch_chunk(unit + (k2 / NC) * gridDim.x, k2 % NC);
+          prefetch_chunk(unit + (k2 / NC) * ustride, k2 % NC);
           UpdRegs r;
           upd_load(g.u, r, row0, h, tn * BN + c, g.M, g.N, c < BN, lane);
           upd_apply(g.u, hpv, r, sbuf, h, lane);
@@ -335,9 +370,9 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     const bool f32out = g.mode >= 2;
     const int ccols = f32out ? 32 : 64;   // columns per chunk
     int it = 0, nchunk = 0;
-    for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
+    for (int unit = unit0; unit < num_units; unit += ustride, ++it) {
       int tm, tn;
-      tile_coords(unit % num_tiles, g.tiles_m, g.tiles_n, g.group_m, tm, tn);
+      unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
       const int split = unit / num_tiles;
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
@@ -437,6 +472,12 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
       }
     }
     __syncwarp();
+  }
+  if (PAIR) {   // neither CTA of a pair leaves while the other may still use its shared memory
+    __syncthreads();
+    cluster_sync();
+  }
+  if (warp == 1) {
     fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)C_::TMEM_COLS)
                  : "memory");
@@ -564,50 +605,79 @@ bool make_map_c(CUtensorMap* m, const Args& a) {
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool A_MN, bool B_MN, bool UPD = false>
+template <int BN, bool A_MN, bool B_MN, bool UPD = false, bool PAIR = false>
 bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int ctas_per_sm) {
   using C_ = Cfg<BN, UPD>;
   static bool attr = false;
-  auto kern = gemm_tc_k<BN, A_MN, B_MN, UPD>;
+  static int max_pairs = 0;   // clusters of two that can be resident at once
+  auto kern = gemm_tc_k<BN, A_MN, B_MN, UPD, PAIR>;
   if (!attr) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM) != cudaSuccess) return false;
+    if (PAIR) {
+      cudaLaunchConfig_t oc = {};
+      oc.gridDim = dim3(2u * (unsigned)g_sms);
+      oc.blockDim = dim3((unsigned)(UPD ? kThreadsUpd : kThreads));
+      oc.dynamicSmemBytes = C_::SMEM;
+      cudaLaunchAttribute ca[1];
+      ca[0].id = cudaLaunchAttributeClusterDimension;
+      ca[0].val.clusterDim.x = 2;
+      ca[0].val.clusterDim.y = 1;
+      ca[0].val.clusterDim.z = 1;
+      oc.attrs = ca;
+      oc.numAttrs = 1;
+      if (cudaOccupancyMaxActiveClusters(&max_pairs, kern, &oc) != cudaSuccess || max_pairs < 1) {
+        cudaGetLastError();
+        return false;
+      }
+    }
     attr = true;
   }
   CUtensorMap ta, tb;
   const bool okA = A_MN ? make_map(&ta, A, (uint64_t)a.M, (uint64_t)a.K, 64, 64)
                         : make_map(&ta, A, (uint64_t)a.K, (uint64_t)a.M, 64, BM);
+  // a pair's CTA loads half of a K-major B tile (BN / 2 rows); MN-major B tiles are 64-column boxes
   const bool okB = B_MN ? make_map(&tb, B, (uint64_t)a.N, (uint64_t)a.K, 64, 64)
-                        : make_map(&tb, B, (uint64_t)a.K, (uint64_t)a.N, 64, BN);
+                        : make_map(&tb, B, (uint64_t)a.K, (uint64_t)a.N, 64, PAIR ? BN / 2 : BN);
   CUtensorMap tcm;
   if (!okA || !okB || !make_map_c(&tcm, a)) return false;
   UpdMaps um;
   std::memset(&um, 0, sizeof um);
-  const int units = a.tiles_m * a.tiles_n * a.splits;
-  const int slots = g_sms * ctas_per_sm;
-  const int grid = units < slots ? units : slots;
+  int grid;
+  if (PAIR) {   // one cluster of two per pair of tile rows, as many as can be resident
+    const int units = (a.tiles_m + 1) / 2 * a.tiles_n * a.splits;
+    grid = 2 * std::min(units, max_pairs);
+  } else {
+    const int units = a.tiles_m * a.tiles_n * a.splits;
+    const int slots = g_sms * ctas_per_sm;
+    grid = units < slots ? units : slots;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3((unsigned)(UPD ? kThreadsUpd : kThreads));
   cfg.dynamicSmemBytes = C_::SMEM;
   cfg.stream = s;
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = 2;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = PAIR ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, kern, ta, tb, tcm, a, um) == cudaSuccess;
 }
 
 template <bool A_MN, bool B_MN>
-bool launch_bn(int bn, const Args& a, const void* A, const void* B, cudaStream_t s) {
-  if (bn == 256) return launch<256, A_MN, B_MN>(a, A, B, s, 1);
-  if (bn == 128) return launch<128, A_MN, B_MN>(a, A, B, s, 1);
+bool launch_bn(int bn, bool pair, const Args& a, const void* A, const void* B, cudaStream_t s) {
+  if (bn == 256) return pair ? launch<256, A_MN, B_MN, false, true>(a, A, B, s, 1) : launch<256, A_MN, B_MN>(a, A, B, s, 1);
+  if (bn == 128) return pair ? launch<128, A_MN, B_MN, false, true>(a, A, B, s, 1) : launch<128, A_MN, B_MN>(a, A, B, s, 1);
   return launch<64, A_MN, B_MN>(a, A, B, s, 2);
 }
 
 // The fused-update kernel (mode 4): 128 x 128 tiles, one CTA per SM.
-bool launch_upd(const Args& a, const void* A, const void* B, cudaStream_t s) {
-  return launch<128, true, true, true>(a, A, B, s, 1);
+bool launch_upd(bool pair, const Args& a, const void* A, const void* B, cudaStream_t s) {
+  return pair ? launch<128, true, true, true, true>(a, A, B, s, 1) : launch<128, true, true, true>(a, A, B, s, 1);
 }
 
 // Tile width and split count from a wave model: units of 128 x BN x (K / splits) run on 152 (BN
@@ -659,11 +729,16 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   if (mode >= 2 && M % 8 != 0) return false;
   int bn = 128, splits = 1;
   tc::choose(mode == 4 ? 2 : mode, M, N, K, bn, splits, mode == 4);
-  if (const char* force = std::getenv("ZL_GEMM_TILE")) {   // test hook "BN:SPLITS": forces the tile and split count
-    int fb = 0, fs = 0;
-    if (std::sscanf(force, "%d:%d", &fb, &fs) == 2 && (fb == 64 || fb == 128 || fb == 256) && fs >= 1 && fs <= 16) {
+  // CTA pairs sharing B tiles wherever there are two tile rows to pair (BN 64 runs two CTAs per SM instead)
+  int pair = bn >= 128 && M > tc::BM ? 1 : 0;
+  if (const char* force = std::getenv("ZL_GEMM_TILE")) {   // test hook "BN:SPLITS[:PAIR]": forces the plan
+    int fb = 0, fs = 0, fp = -1;
+    const int nf = std::sscanf(force, "%d:%d:%d", &fb, &fs, &fp);
+    if (nf >= 2 && (fb == 64 || fb == 128 || fb == 256) && fs >= 1 && fs <= 16) {
       bn = mode == 4 ? 128 : fb;
       splits = std::max(1, std::min(fs, (K + tc::BK - 1) / tc::BK));
+      pair = bn >= 128 && M > tc::BM ? 1 : 0;
+      if (nf == 3 && (fp == 0 || fp == 1)) pair = fp && bn >= 128 ? 1 : 0;
     }
   }
   tc::Args a;
@@ -673,6 +748,7 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
   a.tiles_n = (N + bn - 1) / bn;
   a.group_m = (double)M * K * 2.0 <= 48e6 ? a.tiles_m : std::min(8, a.tiles_m);
+  if (pair) a.group_m = (a.group_m + 1) / 2;   // in pairs of tile rows
   const int nk = (K + tc::BK - 1) / tc::BK;
   a.kb_per_split = (nk + splits - 1) / splits;
   a.splits = (nk + a.kb_per_split - 1) / a.kb_per_split;   // no empty split (its slice would never be formed)
@@ -695,10 +771,10 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   }
   note_launch(1);
   bool ok;
-  if (mode == 0) ok = tc::launch_bn<false, false>(bn, a, A, B, s);
-  else if (mode == 1) ok = tc::launch_bn<false, true>(bn, a, A, B, s);
-  else if (a.mode == 4) ok = tc::launch_upd(a, A, B, s);
-  else ok = tc::launch_bn<true, true>(bn, a, A, B, s);
+  if (mode == 0) ok = tc::launch_bn<false, false>(bn, pair, a, A, B, s);
+  else if (mode == 1) ok = tc::launch_bn<false, true>(bn, pair, a, A, B, s);
+  else if (a.mode == 4) ok = tc::launch_upd(pair, a, A, B, s);
+  else ok = tc::launch_bn<true, true>(bn, pair, a, A, B, s);
   if (ws) {
     if (ok) {
       note_launch(1);

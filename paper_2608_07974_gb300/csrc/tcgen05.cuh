@@ -102,6 +102,33 @@ __device__ __forceinline__ void tma2d(void* dst, const CUtensorMap* m, uint64_t*
       : "memory");
 }
 
+// 2-D TMA load multicast to the CTAs of `mask` in this CTA's cluster: the box lands at the same shared
+// offset in each of them and completes bytes on the mbarrier at the same offset in each.
+__device__ __forceinline__ void tma2d_mc(void* dst, const CUtensorMap* m, uint64_t* bar, int c0, int c1,
+                                         uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(su32(dst)),
+      "l"((unsigned long long)m), "r"(su32(bar)), "r"(c0), "r"(c1), "h"(mask)
+      : "memory");
+}
+// Commit of this thread's prior tcgen05 operations, arriving on the mbarrier at the same shared offset in
+// every CTA of `mask` (cluster).
+__device__ __forceinline__ void mma_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::
+                   "r"(su32(bar)), "h"(mask)
+               : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Every thread of every CTA of the cluster arrives and waits (release / acquire).
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // Shared-memory matrix descriptor: start, leading / stride byte offsets, sm100 version bit,
 // 128-byte swizzle.
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {

@@ -72,7 +72,7 @@ def test_fused_update_equals_unfused_bitwise(w, kind, accum_m):
         assert torch.equal(a[1][key], b[1][key]), key
 
 
-@pytest.mark.parametrize("tile", ["128:2", "256:3", "64:1"])
+@pytest.mark.parametrize("tile", ["128:2", "256:3", "64:1", "128:1:0", "128:1:1", "128:3:1"])
 def test_fused_update_with_forced_tiles_and_split_k(tile, monkeypatch):
     """The fused step in the split-K reduction and under every tile width (the test hook ZL_GEMM_TILE
     forces the tile and split count of every product, fused and unfused alike)."""

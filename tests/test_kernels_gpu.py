@@ -203,10 +203,13 @@ def test_gemm_tensor_core_matches_fp32(B, mode, M, N, K):
     assert err <= (1e-5 if mode == 2 else 8e-3), err
 
 
-@pytest.mark.parametrize("tile", ["64:1", "128:1", "256:1", "64:3", "128:4", "256:2"])
-@pytest.mark.parametrize("mode,M,N,K", [(0, 384, 200, 1024), (1, 260, 136, 3000), (2, 136, 264, 2100)])
+@pytest.mark.parametrize("tile", ["64:1", "128:1:0", "256:1:0", "64:3", "128:4:0", "256:2:0",
+                                  "128:1:1", "256:1:1", "128:4:1", "256:2:1"])
+@pytest.mark.parametrize("mode,M,N,K", [(0, 384, 200, 1024), (1, 260, 136, 3000), (2, 136, 264, 2100),
+                                        (0, 1000, 520, 777), (2, 904, 392, 640)])
 def test_gemm_every_tile_and_split(B, monkeypatch, tile, mode, M, N, K):
-    """Each tile width and split-K count (forced) agrees with the fp32 reference on ragged shapes."""
+    """Each tile width, split-K count and CTA-pair choice (forced: BN:SPLITS:PAIR) agrees with the fp32
+    reference on ragged shapes, including an odd number of tile rows (the last pair's second tile lies past M)."""
     monkeypatch.setenv("ZL_GEMM_TILE", tile)
     test_gemm_tensor_core_matches_fp32(B, mode, M, N, K)
 
