@@ -113,7 +113,8 @@ __device__ __forceinline__ constexpr uint32_t idesc() {
 
 // Tile order: groups of G tile rows sweep the tile columns, so the rows of A a group reads and the
 // B tile a column of the group reads are each fetched from DRAM about once. The host picks G: all the
-// tile rows when the whole A operand fits well inside L2 (then every B tile is read once), else 8.
+// tile rows when A fits well inside L2 or is the smaller operand (then every B tile is read once and A
+// about once per wave), else 8.
 __device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int G, int& tm, int& tn) {
   const int per_group = G * tiles_n;
   const int gid = tile / per_group, first = gid * G;
@@ -747,7 +748,10 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   a.u = u ? *u : GemmUpdate{};
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
   a.tiles_n = (N + bn - 1) / bn;
-  a.group_m = (double)M * K * 2.0 <= 48e6 ? a.tiles_m : std::min(8, a.tiles_m);
+  // one group of every tile row (each B tile fetched once, A once per wave of tile columns) when A fits
+  // well inside L2 or is the smaller operand; else groups of 8 tile rows (A once, B once per group)
+  const double a_bytes = (double)M * K * 2.0, b_bytes = (double)N * K * 2.0;
+  a.group_m = (a_bytes <= 48e6 || a_bytes <= b_bytes) ? a.tiles_m : std::min(8, a.tiles_m);
   if (pair) a.group_m = (a.group_m + 1) / 2;   // in pairs of tile rows
   const int nk = (K + tc::BK - 1) / tc::BK;
   a.kb_per_split = (nk + splits - 1) / splits;
