@@ -20,19 +20,20 @@ namespace tc {
 
 constexpr int BM = 128, BK = 64;
 constexpr int kThreads = 192;      // TMA warp, MMA warp, four epilogue warps
-constexpr int kThreadsUpd = 320;   // fused-update kernels (mode 4): eight epilogue warps, two per TMEM lane quadrant
+constexpr int kUpdWarps = 8;       // fused-update kernels (mode 4): epilogue warps, kUpdWarps / 4 per TMEM lane quadrant (16: 41.2 against 36.3 ms per 7B step, spills)
+constexpr int kThreadsUpd = 64 + 32 * kUpdWarps;
 
 template <int BN, bool UPD = false>
 struct Cfg {
   // BN = 64 stays under 114 KB of shared memory so two CTAs (and TMEM allocations) fit on an SM.
-  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 3);
+  static constexpr int STAGES = UPD ? (kUpdWarps > 8 ? 5 : 6) : (BN == 256 ? 4 : (BN == 128 ? 6 : 3));
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
   // epilogue staging: per epilogue warp two buffers of 32 rows x 128 B (the TMA store box), or, in the
-  // fused-update kernels, one 32 x 32 accumulator piece for each of eight warps
-  static constexpr int OUT_BYTES = 4 * 2 * 32 * 128;
+  // fused-update kernels, one 32 x 32 accumulator piece per epilogue warp
+  static constexpr int OUT_BYTES = UPD ? kUpdWarps * 32 * 128 : 4 * 2 * 32 * 128;
   static constexpr int SMEM = STAGES * STAGE_BYTES + OUT_BYTES + 1024 + 256;
 };
 
@@ -156,7 +157,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C_::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], PAIR ? 2 : 1); }
-    for (int a = 0; a < 2; ++a) { mbar_init(&tfull[a], 1); mbar_init(&tempty[a], UPD ? 8 : 4); }
+    for (int a = 0; a < 2; ++a) { mbar_init(&tfull[a], 1); mbar_init(&tempty[a], UPD ? kUpdWarps : 4); }
     mbar_init(fin, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -291,15 +292,17 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     if (leader) mma_commit(fin);
     __syncwarp();
   } else if (UPD && g.mode == 4) {
-    // ---------------- fused optimizer epilogue (mode 4): warps 2..9 ----------------
-    // Two warps per TMEM lane quadrant take alternate 32-column pieces of the quadrant's 32 accumulator
-    // rows (BN 128: pieces 0, 2 or 1, 3). Per tile a warp reads both its pieces from TMEM and hands TMEM
+    // ---------------- fused optimizer epilogue (mode 4): warps 2 .. 2 + kUpdWarps - 1 ----------------
+    // WQ warps per TMEM lane quadrant take interleaved 32-column pieces of the quadrant's 32 accumulator
+    // rows (piece column 32 (part + WQ p)). Per tile a warp reads all its pieces from TMEM and hands TMEM
     // back at once; then per piece it stages the accumulator in its shared-memory buffer and works
     // through the piece's two 16-row chunks (upd_load, then upd_apply).
+    constexpr int WQ = kUpdWarps / 4;
     const int q = warp & 3, part = (warp - 2) >> 2;
     uint8_t* sbuf = outbuf + (warp - 2) * (32 * 128);
     const AdamHP hpv = adam_hp(g.u.hp, g.u.b1, g.u.b2, g.u.eps, g.u.wd);
-    constexpr int NP = BN / 64;   // pieces per warp and tile
+    constexpr int NP = UPD ? BN / (32 * WQ) : 1;   // pieces per warp and tile
+    static_assert(!UPD || NP >= 1, "at least one 32-column piece per epilogue warp");
     constexpr int NC = 2 * NP;    // 16-row chunks per warp and tile: chunk k = piece k / 2, half k % 2
     // L2 prefetch of chunk `k` of tile `unit` (lanes 0-15 one row each: its 128-byte line of the master
     // and of both moments), issued PD chunks ahead of the loads that read it
@@ -307,7 +310,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
       if (unit >= num_units || lane >= 16) return;
       int tm, tn;
       unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
-      const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * part + 64 * (k >> 1);
+      const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * (part + WQ * (k >> 1));
       if (row >= g.M || col >= g.N) return;
       const size_t at = (size_t)row * g.N + col;
       asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.theta + at));
@@ -332,13 +335,13 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
       const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       float v[NP][32];
 #pragma unroll
-      for (int p = 0; p < NP; ++p) tmem_ld32(trow + (uint32_t)(32 * part + 64 * p), v[p]);
+      for (int p = 0; p < NP; ++p) tmem_ld32(trow + (uint32_t)(32 * (part + WQ * p)), v[p]);
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
 #pragma unroll
       for (int p = 0; p < NP; ++p) {
-        const int c = 32 * part + 64 * p;
+        const int c = 32 * (part + WQ * p);
         if (g.alpha != 1.f) {
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[p][e] *= g.alpha;
