@@ -170,6 +170,15 @@ def workload_desc(w, K, lora=0, adapter=0):
             f"K={K} chunks, alpha {w.alpha}, AdamW, {tune}" + (f", readout adapters of width {adapter}" if adapter else ""))
 
 
+def run_config(args, w, K, world):
+    """The `config` object of both arms' JSON lines (the workload they measure)."""
+    return {"workload": workload_desc(w, K, args.lora, args.adapter), "K": K,
+            "bounds": synth.chunk_bounds(w.dims.n_layers, K), "global_batch": w.batch * world, "seq_len": w.seq,
+            "max_live_chunks": args.max_live, "cuda_graph": args.graph, "loss_rows": args.loss_rows,
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU, K streams",
+            "l2": "no flush: every step's working set (weights, AdamW state, logits) exceeds L2"}
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -327,7 +336,7 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f32" if w.dtype == "bf16" else "f64", "data": "synthetic",
-            "config": {"workload": workload_desc(w, K), "K": K},
+            "config": run_config(args, w, K, int(os.environ.get("WORLD_SIZE", "1"))),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "nproc": os.cpu_count(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -501,11 +510,7 @@ def run_ours(args):
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-                "config": {"workload": workload_desc(w, K, args.lora, args.adapter), "K": K, "bounds": bounds,
-                           "global_batch": w.batch * world, "seq_len": w.seq, "max_live_chunks": args.max_live,
-                           "cuda_graph": args.graph, "loss_rows": args.loss_rows,
-                           "parallelism": f"replicas x{world}" if world > 1 else "single GPU, K streams",
-                           "l2": "no flush: every step's working set (weights, AdamW state, logits) exceeds L2"},
+                "config": run_config(args, w, K, world),
                 "peak_hbm_gb": zl_peak / 1e9, "bp": bp,
                 "zl_vs_bp": {"throughput": value / bp["value"], "peak_hbm": (zl_peak / 1e9) / bp["peak_hbm_gb"]}
                 if bp else None,
