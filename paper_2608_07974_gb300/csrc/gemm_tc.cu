@@ -26,7 +26,7 @@ constexpr int kThreadsUpd = 64 + 32 * kUpdWarps;
 template <int BN, bool UPD = false>
 struct Cfg {
   // BN = 64 stays under 114 KB of shared memory so two CTAs (and TMEM allocations) fit on an SM.
-  static constexpr int STAGES = UPD ? (kUpdWarps > 8 ? 5 : 6) : (BN == 256 ? 4 : (BN == 128 ? 6 : 3));
+  static constexpr int STAGES = UPD ? (BN == 256 ? 4 : (kUpdWarps > 8 ? 5 : 6)) : (BN == 256 ? 4 : (BN == 128 ? 6 : 3));
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -333,24 +333,38 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
       fence_after();
       const int row0 = tm * BM + q * 32;
       const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-      float v[NP][32];
+      // up to two pieces are read before TMEM goes back; wider tiles read each piece when it is due and
+      // release TMEM after the last
+      constexpr int NV = NP <= 2 ? NP : 1;
+      float v[NV][32];
+      if (NP <= 2) {
 #pragma unroll
-      for (int p = 0; p < NP; ++p) tmem_ld32(trow + (uint32_t)(32 * (part + WQ * p)), v[p]);
-      fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
+        for (int p = 0; p < NV; ++p) tmem_ld32(trow + (uint32_t)(32 * (part + WQ * p)), v[p]);
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+      }
 #pragma unroll
       for (int p = 0; p < NP; ++p) {
         const int c = 32 * (part + WQ * p);
+        float* vp = v[NP <= 2 ? p : 0];
+        if (NP > 2) {
+          tmem_ld32(trow + (uint32_t)c, vp);
+          if (p == NP - 1) {
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+          }
+        }
         if (g.alpha != 1.f) {
 #pragma unroll
-          for (int e = 0; e < 32; ++e) v[p][e] *= g.alpha;
+          for (int e = 0; e < 32; ++e) vp[e] *= g.alpha;
         }
         __syncwarp();   // the previous piece's reads of the staging buffer are done
 #pragma unroll
         for (int k = 0; k < 8; ++k)
           *reinterpret_cast<float4*>(sbuf + lane * 128 + ((k ^ (lane & 7)) << 4)) =
-              make_float4(v[p][4 * k], v[p][4 * k + 1], v[p][4 * k + 2], v[p][4 * k + 3]);
+              make_float4(vp[4 * k], vp[4 * k + 1], vp[4 * k + 2], vp[4 * k + 3]);
         __syncwarp();
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -679,8 +693,10 @@ bool launch_bn(int bn, bool pair, const Args& a, const void* A, const void* B, c
   return launch<64, A_MN, B_MN>(a, A, B, s, 2);
 }
 
-// The fused-update kernel (mode 4): 128 x 128 tiles, one CTA per SM.
-bool launch_upd(bool pair, const Args& a, const void* A, const void* B, cudaStream_t s) {
+// The fused-update kernels (mode 4): 128 x 128 or 128 x 256 tiles, one CTA per SM.
+bool launch_upd(int bn, bool pair, const Args& a, const void* A, const void* B, cudaStream_t s) {
+  if (bn == 256)
+    return pair ? launch<256, true, true, true, true>(a, A, B, s, 1) : launch<256, true, true, true>(a, A, B, s, 1);
   return pair ? launch<128, true, true, true, true>(a, A, B, s, 1) : launch<128, true, true, true>(a, A, B, s, 1);
 }
 
@@ -688,12 +704,12 @@ bool launch_upd(bool pair, const Args& a, const void* A, const void* B, cudaStre
 // 256/128) or 304 (BN 64) slots, each k block (64 deep) of a unit taking the time measured for that
 // tile on GB300 (4096^3 and transformer-shape sweeps; the operands of the mode-2 kernel are both
 // MN-major and load in more boxes), plus, for splits, the fp32 partial traffic and the reduction.
-void choose(int mode, int M, int N, int K, int& bn_out, int& splits_out, bool only128 = false) {
+void choose(int mode, int M, int N, int K, int& bn_out, int& splits_out, bool no64 = false) {
   const double hbm = 6.0e12;                  // bytes/s for the partials
   const int nk = (K + BK - 1) / BK;
   double best = 1e30;
   for (int bn : {256, 128, 64}) {
-    if (only128 && bn != 128) continue;
+    if (no64 && bn == 64) continue;
     const double kb = mode == 2 ? (bn == 256 ? 0.40e-6 : bn == 128 ? 0.30e-6 : 0.36e-6)
                                 : (bn == 256 ? 0.36e-6 : bn == 128 ? 0.29e-6 : 0.32e-6);
     const long tiles = (long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
@@ -739,7 +755,7 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
     int fb = 0, fs = 0, fp = -1;
     const int nf = std::sscanf(force, "%d:%d:%d", &fb, &fs, &fp);
     if (nf >= 2 && (fb == 64 || fb == 128 || fb == 256) && fs >= 1 && fs <= 16) {
-      bn = mode == 4 ? 128 : fb;
+      bn = mode == 4 && fb == 64 ? 128 : fb;
       splits = std::max(1, std::min(fs, (K + tc::BK - 1) / tc::BK));
       pair = bn >= 128 && M > tc::BM ? 1 : 0;
       if (nf == 3 && (fp == 0 || fp == 1)) pair = fp && bn >= 128 ? 1 : 0;
@@ -780,7 +796,7 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   bool ok;
   if (mode == 0) ok = tc::launch_bn<false, false>(bn, pair, a, A, B, s);
   else if (mode == 1) ok = tc::launch_bn<false, true>(bn, pair, a, A, B, s);
-  else if (a.mode == 4) ok = tc::launch_upd(pair, a, A, B, s);
+  else if (a.mode == 4) ok = tc::launch_upd(bn, pair, a, A, B, s);
   else ok = tc::launch_bn<true, true>(bn, pair, a, A, B, s);
   if (ws) {
     if (ok) {
