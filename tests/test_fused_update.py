@@ -21,6 +21,9 @@ GPT2S = synth.Workload("fused-gpt2-bf16", synth.ModelDims(synth.ARCH_GPT2, 4, 25
                        batch=2, seq=256, K=2, steps=4, seed=1234 + 1)
 LLAMAS = synth.Workload("fused-llama-bf16", synth.ModelDims(synth.ARCH_LLAMA, 2, 256, 4, 2, 704, 512, 256), "bf16",
                         batch=2, seq=128, K=2, steps=4, seed=1234 + 2)
+# ragged everywhere: d 200 (head dim 50, padded to 64 in attention), gate/up 688 rows, FFN 344 columns
+ODD = synth.Workload("fused-llama-odd", synth.ModelDims(synth.ARCH_LLAMA, 2, 200, 4, 2, 344, 500, 192), "bf16",
+                     batch=3, seq=96, K=2, steps=4, seed=1234 + 3)
 
 
 def _params(w):
@@ -60,7 +63,7 @@ def _run(w, P, kind, steps, **kw):
     return losses, st
 
 
-@pytest.mark.parametrize("w", [GPT2S, LLAMAS, synth.TINY], ids=["gpt2s-bf16", "llama-bf16", "tiny-f32"])
+@pytest.mark.parametrize("w", [GPT2S, LLAMAS, ODD, synth.TINY], ids=["gpt2s-bf16", "llama-bf16", "odd-bf16", "tiny-f32"])
 @pytest.mark.parametrize("kind", ["zl", "bp", "local"])
 @pytest.mark.parametrize("accum_m", [1, 2])
 def test_fused_update_equals_unfused_bitwise(w, kind, accum_m):
