@@ -1,7 +1,8 @@
 // Tensor-core GEMM for sm_103a: TMA tiles (128-byte swizzle) -> tcgen05.mma (bf16 operands,
 // fp32 accumulator in TMEM, double buffered) -> tcgen05.ld epilogue (bias, residual, bf16 store,
-// or fp32 accumulate into a gradient). Persistent, warp-specialised: warp 0 issues TMA loads,
-// warp 1 owns TMEM and issues the MMAs (one thread), warps 2-5 drain the accumulator.
+// or fp32 accumulate into a gradient, or the fused AdamW step of the weight). Persistent,
+// warp-specialised: warp 0 issues TMA loads, warp 1 owns TMEM and issues the MMAs (one thread),
+// warps 2-5 (fused update: 4-11) drain the accumulator.
 // Every mbarrier wait is bounded: on expiry the kernel raises ZL_DEVERR_TIMEOUT and unwinds.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -20,8 +21,15 @@ namespace tc {
 
 constexpr int BM = 128, BK = 64;
 constexpr int kThreads = 192;      // TMA warp, MMA warp, four epilogue warps
-constexpr int kUpdWarps = 8;       // fused-update kernels (mode 4): epilogue warps, kUpdWarps / 4 per TMEM lane quadrant (16: 41.2 against 36.3 ms per 7B step, spills)
-constexpr int kThreadsUpd = 64 + 32 * kUpdWarps;
+// Fused-update kernels (mode 4): warpgroup 0 = TMA warp, MMA warp and two idle warps on kRegsLow
+// registers each; then kUpdWarps epilogue warps (two per TMEM lane quadrant) on kRegsUpd, which hold the
+// optimizer state of two chunks at once. The split uses exactly the registers of the launch (384 threads
+// x 168, the most a 384-thread CTA gets); the host checks the kernel's register count before it runs.
+// (40 for warpgroup 0 spills in the MMA loop; 56 + 224 spills nowhere.)
+constexpr int kUpdWarps = 8;
+constexpr int kThreadsUpd = 128 + 32 * kUpdWarps;
+constexpr int kRegsLow = 56, kRegsUpd = 224;
+static_assert(128 * kRegsLow + 32 * kUpdWarps * kRegsUpd <= kThreadsUpd * 168, "register split above the pool");
 
 template <int BN, bool UPD = false>
 struct Cfg {
@@ -46,7 +54,7 @@ struct Cfg {
 // kept for the operand tiles.
 struct UpdRegs {
   float4 th[4], mm[4], vv[4];
-  size_t at[4];
+  size_t at;     // element offset of row j = 0; row j sits 4 j rows further down
   unsigned ok;   // bit j: row j is inside the tensor
 };
 __device__ __forceinline__ void upd_load(const GemmUpdate& u, UpdRegs& r, int row0, int h, int col0, int M, int N,
@@ -54,35 +62,37 @@ __device__ __forceinline__ void upd_load(const GemmUpdate& u, UpdRegs& r, int ro
   r.ok = 0;
   const int col = col0 + 4 * (lane & 7);
   if (!valid || col >= N) return;
+  const int row = row0 + 16 * h + (lane >> 3);
+  r.at = (size_t)row * N + col;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
-    const int row = row0 + 16 * h + (lane >> 3) + 4 * j;
-    r.at[j] = (size_t)row * N + col;
-    if (row < M) {
+    if (row + 4 * j < M) {
+      const size_t a = r.at + (size_t)(4 * j) * N;
       r.ok |= 1u << j;
-      r.th[j] = __ldcs(reinterpret_cast<const float4*>(u.theta + r.at[j]));
-      r.mm[j] = __ldcs(reinterpret_cast<const float4*>(u.m + r.at[j]));
-      r.vv[j] = __ldcs(reinterpret_cast<const float4*>(u.v + r.at[j]));
+      r.th[j] = __ldcs(reinterpret_cast<const float4*>(u.theta + a));
+      r.mm[j] = __ldcs(reinterpret_cast<const float4*>(u.m + a));
+      r.vv[j] = __ldcs(reinterpret_cast<const float4*>(u.v + a));
     }
   }
 }
 __device__ __forceinline__ void upd_apply(const GemmUpdate& u, const AdamHP& h, UpdRegs& r, const uint8_t* sp,
-                                          int hh, int lane) {
+                                          int hh, int N, int lane) {
   const int piece = lane & 7;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     if (!(r.ok >> j & 1u)) continue;
+    const size_t a = r.at + (size_t)(4 * j) * N;
     const int rr = 16 * hh + (lane >> 3) + 4 * j;
     const float4 a4 = *reinterpret_cast<const float4*>(sp + rr * 128 + ((piece ^ (rr & 7)) << 4));
     const float acc[4] = {a4.x, a4.y, a4.z, a4.w};
     float* tp = &r.th[j].x; float* mp = &r.mm[j].x; float* vp = &r.vv[j].x;
 #pragma unroll
     for (int q = 0; q < 4; ++q) adamw_elem(tp[q], mp[q], vp[q], __fmul_rn(acc[q], u.gscale), h);
-    __stcs(reinterpret_cast<float4*>(u.theta + r.at[j]), r.th[j]);
-    __stcs(reinterpret_cast<float4*>(u.m + r.at[j]), r.mm[j]);
-    __stcs(reinterpret_cast<float4*>(u.v + r.at[j]), r.vv[j]);
+    __stcs(reinterpret_cast<float4*>(u.theta + a), r.th[j]);
+    __stcs(reinterpret_cast<float4*>(u.m + a), r.mm[j]);
+    __stcs(reinterpret_cast<float4*>(u.v + a), r.vv[j]);
     __nv_bfloat162 c2[2] = {__floats2bfloat162_rn(tp[0], tp[1]), __floats2bfloat162_rn(tp[2], tp[3])};
-    __stcs(reinterpret_cast<uint2*>((bf16*)u.comp + r.at[j]), *reinterpret_cast<const uint2*>(c2));
+    __stcs(reinterpret_cast<uint2*>((bf16*)u.comp + a), *reinterpret_cast<const uint2*>(c2));
   }
 }
 
@@ -154,7 +164,6 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
   uint32_t* tbase = (uint32_t*)(fin + 1);
   volatile int* abort_flag = (volatile int*)(tbase + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
   if (threadIdx.x == 0) {
     for (int s = 0; s < C_::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], PAIR ? 2 : 1); }
     for (int a = 0; a < 2; ++a) { mbar_init(&tfull[a], 1); mbar_init(&tempty[a], UPD ? kUpdWarps : 4); }
@@ -186,193 +195,195 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
   const int num_tiles = (PAIR ? (g.tiles_m + 1) / 2 : g.tiles_m) * g.tiles_n;
   const int num_units = num_tiles * g.splits;
 
-  if (warp == 0) {
-    // ---------------- TMA producer ----------------
-    // The whole warp runs the loop (uniform control flow keeps coordinates and addresses in uniform
-    // registers); one elected lane issues the copies.
-    const bool leader = elect_one();
-    int stage = 0;
-    uint32_t phase = 0;
-    bool ok = true;
-    int issued[C_::STAGES];   // parity of the last fill of each stage, -1 if none
-#pragma unroll
-    for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
-    for (int unit = unit0; ok && unit < num_units; unit += ustride) {
-      int tm, tn;
-      unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
-      const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
-      for (int kb = kb0; kb < kb1; ++kb) {
-        if (!uwait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
-        issued[stage] = (int)phase;
-        if (leader) {
-          mbar_expect_tx(&full[stage], C_::STAGE_BYTES);
-          uint8_t* sa = smem + stage * C_::STAGE_BYTES;
-          uint8_t* sb = sa + C_::A_BYTES;
-          const int k0 = kb * BK;
-          if (!A_MN) {
-            tma2d(sa, &ta, &full[stage], k0, tm * BM);
-          } else {
-            tma2d(sa, &ta, &full[stage], tm * BM, k0);
-            tma2d(sa + 8192, &ta, &full[stage], tm * BM + 64, k0);
-          }
-          if (PAIR) {   // this CTA's half of the B tile, into both CTAs
-            constexpr int HB = BN / 2;
-            if (!B_MN) {
-              tma2d_mc(sb + crank * (HB * 128), &tb, &full[stage], k0, tn * BN + (int)crank * HB, kPairMask);
+  if (warp < 2 || (UPD && warp < 4)) {
+    // warpgroup 0 of a fused-update kernel hands most of its registers to the epilogue warpgroups
+    if constexpr (UPD) regs_dec<kRegsLow>();
+    if (warp == 0) {
+      // ---------------- TMA producer ----------------
+      // The whole warp runs the loop (uniform control flow keeps coordinates and addresses in uniform
+      // registers); one elected lane issues the copies.
+      const bool leader = elect_one();
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int issued[C_::STAGES];   // parity of the last fill of each stage, -1 if none
+  #pragma unroll
+      for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
+      for (int unit = unit0; ok && unit < num_units; unit += ustride) {
+        int tm, tn;
+        unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
+        const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!uwait(&empty[stage], phase ^ 1u, abort_flag, g.err)) { ok = false; break; }
+          issued[stage] = (int)phase;
+          if (leader) {
+            mbar_expect_tx(&full[stage], C_::STAGE_BYTES);
+            uint8_t* sa = smem + stage * C_::STAGE_BYTES;
+            uint8_t* sb = sa + C_::A_BYTES;
+            const int k0 = kb * BK;
+            if (!A_MN) {
+              tma2d(sa, &ta, &full[stage], k0, tm * BM);
             } else {
-#pragma unroll
-              for (int j = 0; j < HB / 64; ++j) {
-                const int jj = (int)crank * (HB / 64) + j;
-                tma2d_mc(sb + jj * 8192, &tb, &full[stage], tn * BN + 64 * jj, k0, kPairMask);
-              }
+              tma2d(sa, &ta, &full[stage], tm * BM, k0);
+              tma2d(sa + 8192, &ta, &full[stage], tm * BM + 64, k0);
             }
-          } else if (!B_MN) {
-            tma2d(sb, &tb, &full[stage], k0, tn * BN);
-          } else {
-#pragma unroll
-            for (int j = 0; j < BN / 64; ++j) tma2d(sb + j * 8192, &tb, &full[stage], tn * BN + 64 * j, k0);
+            if (PAIR) {   // this CTA's half of the B tile, into both CTAs
+              constexpr int HB = BN / 2;
+              if (!B_MN) {
+                tma2d_mc(sb + crank * (HB * 128), &tb, &full[stage], k0, tn * BN + (int)crank * HB, kPairMask);
+              } else {
+  #pragma unroll
+                for (int j = 0; j < HB / 64; ++j) {
+                  const int jj = (int)crank * (HB / 64) + j;
+                  tma2d_mc(sb + jj * 8192, &tb, &full[stage], tn * BN + 64 * jj, k0, kPairMask);
+                }
+              }
+            } else if (!B_MN) {
+              tma2d(sb, &tb, &full[stage], k0, tn * BN);
+            } else {
+  #pragma unroll
+              for (int j = 0; j < BN / 64; ++j) tma2d(sb + j * 8192, &tb, &full[stage], tn * BN + 64 * j, k0);
+            }
+          }
+          __syncwarp();
+          if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (PAIR && ok) {
+        // both CTAs' commits for the last fill of every stage have arrived: no arrival from the peer (and no
+        // copy of this CTA's into the peer) is still on its way when the CTAs exit
+  #pragma unroll 1
+        for (int s = 0; s < C_::STAGES; ++s)
+          if (issued[s] >= 0 && !uwait(&empty[s], (uint32_t)issued[s], abort_flag, g.err)) break;
+      }
+      if (!ok && lane == 0) {   // unwinding: let the copies already in flight land before the CTA exits
+        for (int s = 0; s < C_::STAGES; ++s) {
+          if (issued[s] < 0) continue;
+          const unsigned long long t0 = gtimer();
+          while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
           }
         }
-        __syncwarp();
-        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
       }
-    }
-    if (PAIR && ok) {
-      // both CTAs' commits for the last fill of every stage have arrived: no arrival from the peer (and no
-      // copy of this CTA's into the peer) is still on its way when the CTAs exit
-#pragma unroll 1
-      for (int s = 0; s < C_::STAGES; ++s)
-        if (issued[s] >= 0 && !uwait(&empty[s], (uint32_t)issued[s], abort_flag, g.err)) break;
-    }
-    if (!ok && lane == 0) {   // unwinding: let the copies already in flight land before the CTA exits
-      for (int s = 0; s < C_::STAGES; ++s) {
-        if (issued[s] < 0) continue;
-        const unsigned long long t0 = gtimer();
-        while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
-        }
-      }
-    }
-  } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
-    // The whole warp runs the loop and the waits; one elected lane issues every product and every
-    // commit that tracks them.
-    constexpr uint32_t id = idesc<BN, A_MN, B_MN>();
-    const bool leader = elect_one();
-    int stage = 0, it = 0;
-    uint32_t phase = 0;
-    bool ok = true;
-    for (int unit = unit0; ok && unit < num_units; unit += ustride, ++it) {
-      const int acc = it & 1;
-      const uint32_t aph = (uint32_t)(it >> 1) & 1u;
-      if (!uwait(&tempty[acc], aph ^ 1u, abort_flag, g.err)) break;
-      fence_after();
-      const uint32_t d = tmem + (uint32_t)(acc * BN);
-      const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
-      for (int kb = kb0; kb < kb1; ++kb) {
-        if (!uwait(&full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+    } else if (warp == 1) {
+      // ---------------- MMA issuer ----------------
+      // The whole warp runs the loop and the waits; one elected lane issues every product and every
+      // commit that tracks them.
+      constexpr uint32_t id = idesc<BN, A_MN, B_MN>();
+      const bool leader = elect_one();
+      int stage = 0, it = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int unit = unit0; ok && unit < num_units; unit += ustride, ++it) {
+        const int acc = it & 1;
+        const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+        if (!uwait(&tempty[acc], aph ^ 1u, abort_flag, g.err)) break;
         fence_after();
-        if (leader) {
-          const uint32_t a0 = su32(smem + stage * C_::STAGE_BYTES), b0 = a0 + C_::A_BYTES;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t ad = A_MN ? sdesc(a0 + kk * 2048, 8192, 1024) : sdesc(a0 + kk * 32, 16, 1024);
-            const uint64_t bd = B_MN ? sdesc(b0 + kk * 2048, 8192, 1024) : sdesc(b0 + kk * 32, 16, 1024);
-            mma_bf16(d, ad, bd, id, (kb > kb0 || kk > 0) ? 1u : 0u);
+        const uint32_t d = tmem + (uint32_t)(acc * BN);
+        const int kb0 = (unit / num_tiles) * g.kb_per_split, kb1 = min(nk, kb0 + g.kb_per_split);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!uwait(&full[stage], phase, abort_flag, g.err)) { ok = false; break; }
+          fence_after();
+          if (leader) {
+            const uint32_t a0 = su32(smem + stage * C_::STAGE_BYTES), b0 = a0 + C_::A_BYTES;
+  #pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+              const uint64_t ad = A_MN ? sdesc(a0 + kk * 2048, 8192, 1024) : sdesc(a0 + kk * 32, 16, 1024);
+              const uint64_t bd = B_MN ? sdesc(b0 + kk * 2048, 8192, 1024) : sdesc(b0 + kk * 32, 16, 1024);
+              mma_bf16(d, ad, bd, id, (kb > kb0 || kk > 0) ? 1u : 0u);
+            }
+            if (PAIR) mma_commit_mc(&empty[stage], kPairMask);   // the stage is free in both CTAs' view
+            else mma_commit(&empty[stage]);
           }
-          if (PAIR) mma_commit_mc(&empty[stage], kPairMask);   // the stage is free in both CTAs' view
-          else mma_commit(&empty[stage]);
+          __syncwarp();
+          if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
         }
+        if (ok && leader) mma_commit(&tfull[acc]);
         __syncwarp();
-        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
       }
-      if (ok && leader) mma_commit(&tfull[acc]);
+      // all MMAs issued by the leader complete before TMEM is released
+      if (leader) mma_commit(fin);
       __syncwarp();
     }
-    // all MMAs issued by the leader complete before TMEM is released
-    if (leader) mma_commit(fin);
-    __syncwarp();
-  } else if (UPD && g.mode == 4) {
-    // ---------------- fused optimizer epilogue (mode 4): warps 2 .. 2 + kUpdWarps - 1 ----------------
-    // WQ warps per TMEM lane quadrant take interleaved 32-column pieces of the quadrant's 32 accumulator
-    // rows (piece column 32 (part + WQ p)). Per tile a warp reads all its pieces from TMEM and hands TMEM
-    // back at once; then per piece it stages the accumulator in its shared-memory buffer and works
-    // through the piece's two 16-row chunks (upd_load, then upd_apply).
-    constexpr int WQ = kUpdWarps / 4;
-    const int q = warp & 3, part = (warp - 2) >> 2;
-    uint8_t* sbuf = outbuf + (warp - 2) * (32 * 128);
-    const AdamHP hpv = adam_hp(g.u.hp, g.u.b1, g.u.b2, g.u.eps, g.u.wd);
-    constexpr int NP = UPD ? BN / (32 * WQ) : 1;   // pieces per warp and tile
-    static_assert(!UPD || NP >= 1, "at least one 32-column piece per epilogue warp");
-    constexpr int NC = 2 * NP;    // 16-row chunks per warp and tile: chunk k = piece k / 2, half k % 2
-    // L2 prefetch of chunk `k` of tile `unit` (lanes 0-15 one row each: its 128-byte line of the master
-    // and of both moments), issued PD chunks ahead of the loads that read it
-    auto prefetch_chunk = [&](int unit, int k) {
-      if (unit >= num_units || lane >= 16) return;
-      int tm, tn;
-      unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
-      const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * (part + WQ * (k >> 1));
-      if (row >= g.M || col >= g.N) return;
-      const size_t at = (size_t)row * g.N + col;
-      asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.theta + at));
-      asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.m + at));
-      asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.v + at));
-    };
-    constexpr int PD = 2;   // prefetch distance in chunks (2 and 3 measured alike, 4 slower)
-#pragma unroll
-    for (int k = 0; k < PD; ++k) prefetch_chunk(unit0 + (k / NC) * ustride, k % NC);
-    int it = 0;
-    for (int unit = unit0; unit < num_units; unit += ustride, ++it) {
-      int tm, tn;
-      unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
-      const int acc = it & 1;
-      const uint32_t aph = (uint32_t)(it >> 1) & 1u;
-      int ok = 1;
-      if (lane == 0) ok = mbar_wait(&tfull[acc], aph, abort_flag, g.err) ? 1 : 0;
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      fence_after();
-      const int row0 = tm * BM + q * 32;
-      const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-      // up to two pieces are read before TMEM goes back; wider tiles read each piece when it is due and
-      // release TMEM after the last
-      constexpr int NV = NP <= 2 ? NP : 1;
-      float v[NV][32];
-      if (NP <= 2) {
-#pragma unroll
-        for (int p = 0; p < NV; ++p) tmem_ld32(trow + (uint32_t)(32 * (part + WQ * p)), v[p]);
-        fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[acc]);
-      }
-#pragma unroll
-      for (int p = 0; p < NP; ++p) {
+  } else if constexpr (UPD) {
+    // ---------------- fused optimizer epilogue (mode 4): warps 4 .. 4 + kUpdWarps - 1 ----------------
+    regs_inc<kRegsUpd>();
+    if (g.mode == 4) {
+      // WQ warps per TMEM lane quadrant take interleaved 32-column pieces of the quadrant's 32 accumulator
+      // rows (piece column 32 (part + WQ p)). Per piece a warp stages the accumulator in its shared-memory
+      // buffer and works through the piece's two 16-row chunks (upd_load, then upd_apply).
+      constexpr int WQ = kUpdWarps / 4;
+      const int q = warp & 3, part = (warp - 4) >> 2;
+      uint8_t* sbuf = outbuf + (warp - 4) * (32 * 128);
+      const AdamHP hpv = adam_hp(g.u.hp, g.u.b1, g.u.b2, g.u.eps, g.u.wd);
+      constexpr int NP = UPD ? BN / (32 * WQ) : 1;   // pieces per warp and tile
+      static_assert(!UPD || NP >= 1, "at least one 32-column piece per epilogue warp");
+      constexpr int NC = 2 * NP;    // 16-row chunks per warp and tile: chunk k = piece k / 2, half k % 2
+      // L2 prefetch of chunk `k` of tile `unit` (lanes 0-15 one row each: its 128-byte line of the master
+      // and of both moments), issued PD chunks ahead of the loads that read it
+      auto prefetch_chunk = [&](int unit, int k) {
+        if (unit >= num_units || lane >= 16) return;
+        int tm, tn;
+        unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
+        const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * (part + WQ * (k >> 1));
+        if (row >= g.M || col >= g.N) return;
+        const size_t at = (size_t)row * g.N + col;
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.theta + at));
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.m + at));
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.v + at));
+      };
+      constexpr int PD = 2;   // prefetch distance in chunks (2 and 3 measured alike, 4 slower)
+  #pragma unroll
+      for (int k = 0; k < PD; ++k) prefetch_chunk(unit0 + (k / NC) * ustride, k % NC);
+      // chunk (p, h) of tile `unit`: rows 16 h .. of the quadrant, columns 32 (part + WQ p) ..
+      auto load_chunk = [&](UpdRegs& r, int unit, int p, int h) {
+        if (unit >= num_units) { r.ok = 0; return; }
+        int tm, tn;
+        unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
         const int c = 32 * (part + WQ * p);
-        float* vp = v[NP <= 2 ? p : 0];
-        if (NP > 2) {
-          tmem_ld32(trow + (uint32_t)c, vp);
+        upd_load(g.u, r, tm * BM + q * 32, h, tn * BN + c, g.M, g.N, c < BN, lane);
+      };
+      // The state loads of the next chunk are always in flight while a chunk is worked on (two register
+      // sets), across pieces and into the CTA's next tile; each piece is read from TMEM when it is due and
+      // TMEM goes back to the MMA warp after the tile's last piece is read.
+      UpdRegs ra, rb;
+      load_chunk(ra, unit0, 0, 0);
+      int it = 0;
+      for (int unit = unit0; unit < num_units; unit += ustride, ++it) {
+        const int acc = it & 1;
+        const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait(&tfull[acc], aph, abort_flag, g.err) ? 1 : 0;
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
+        fence_after();
+        const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+  #pragma unroll 1
+        for (int p = 0; p < NP; ++p) {
+          const int c = 32 * (part + WQ * p);
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
           if (p == NP - 1) {
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[acc]);
           }
-        }
-        if (g.alpha != 1.f) {
-#pragma unroll
-          for (int e = 0; e < 32; ++e) vp[e] *= g.alpha;
-        }
-        __syncwarp();   // the previous piece's reads of the staging buffer are done
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-          *reinterpret_cast<float4*>(sbuf + lane * 128 + ((k ^ (lane & 7)) << 4)) =
-              make_float4(vp[4 * k], vp[4 * k + 1], vp[4 * k + 2], vp[4 * k + 3]);
-        __syncwarp();
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int k2 = 2 * p + h + PD;   // PD chunks ahead, into the next tiles at the end
-          prefetch_chunk(unit + (k2 / NC) * ustride, k2 % NC);
-          UpdRegs r;
-          upd_load(g.u, r, row0, h, tn * BN + c, g.M, g.N, c < BN, lane);
-          upd_apply(g.u, hpv, r, sbuf, h, lane);
+          if (g.alpha != 1.f) {
+  #pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] *= g.alpha;
+          }
+          __syncwarp();   // the previous piece's reads of the staging buffer are done
+  #pragma unroll
+          for (int k = 0; k < 8; ++k)
+            *reinterpret_cast<float4*>(sbuf + lane * 128 + ((k ^ (lane & 7)) << 4)) =
+                make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+          __syncwarp();
+          prefetch_chunk(unit + ((2 * p + PD) / NC) * ustride, (2 * p + PD) % NC);
+          load_chunk(rb, unit, p, 1);
+          upd_apply(g.u, hpv, ra, sbuf, 0, g.N, lane);
+          prefetch_chunk(unit + ((2 * p + 1 + PD) / NC) * ustride, (2 * p + 1 + PD) % NC);
+          if (p + 1 < NP) load_chunk(ra, unit, p + 1, 0);
+          else load_chunk(ra, unit + ustride, 0, 0);
+          upd_apply(g.u, hpv, rb, sbuf, 1, g.N, lane);
         }
       }
     }
@@ -630,6 +641,14 @@ bool launch(const Args& a, const void* A, const void* B, cudaStream_t s, int cta
   static int max_pairs = 0;   // clusters of two that can be resident at once
   auto kern = gemm_tc_k<BN, A_MN, B_MN, UPD, PAIR>;
   if (!attr) {
+    if (UPD) {   // the register split of the fused-update kernels must fit the pool the CTA is launched with
+      cudaFuncAttributes fa;
+      if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess ||
+          128 * kRegsLow + 32 * kUpdWarps * kRegsUpd > kThreadsUpd * fa.numRegs) {
+        cudaGetLastError();
+        return false;
+      }
+    }
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C_::SMEM) != cudaSuccess) return false;
     if (PAIR) {
       cudaLaunchConfig_t oc = {};

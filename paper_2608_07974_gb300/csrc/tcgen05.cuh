@@ -125,6 +125,17 @@ __device__ __forceinline__ uint32_t cluster_rank() {
   return r;
 }
 // Every thread of every CTA of the cluster arrives and waits (release / acquire).
+// Per-warpgroup register budgets (all four warps of a warpgroup execute the same one): `dec` hands
+// registers back to the CTA's pool, `inc` waits until the pool holds enough and takes them. The pool is
+// what the CTA was launched with (threads x registers per thread).
+template <int N>
+__device__ __forceinline__ void regs_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <int N>
+__device__ __forceinline__ void regs_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
