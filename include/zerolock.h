@@ -294,6 +294,18 @@ zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, co
 zl_status zl_op_gemm_ex(int dtype, int mode, int M, int N, int K, const void* A, const void* B, void* C,
                         float* bias, const void* R, int r_mode, void* stream);
 
+/* The query / key / value projection of a Llama-style layer with rotate-half RoPE (the first
+ * product and rotation of the chunk function f_k, Eq. 1): C[M,N] = A[M,K] . B^T (+ bias[N], fp32), B [N,K], then in
+ * every row n the columns < rot_cols, whole heads of hd columns, rotated pairwise (column i with
+ * i + hd/2 of the head) by the angles of position n % S: cs is the device table [S][hd/2][2] of
+ * (cos, sin), fp32, read only. dtype of A, B, C; row-major, dense; C must not overlap A or B.
+ * bf16 products of head dim 64 or 128 on the tensor-core path rotate in the product's epilogue
+ * (one kernel; the product is rounded to bf16 before its rotation, exactly as the two-pass
+ * path sees it), other cases run the product and then a RoPE pass. Returns ZL_ERR_ARG for NULL
+ * pointers or rot_cols that is not a multiple of hd within N, ZL_ERR_CUDA on a launch failure. */
+zl_status zl_op_qkv_rope(int dtype, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
+                         const float* cs, int S, int hd, int rot_cols, void* stream);
+
 /* Self-test of the bounded waits (no counterpart in the paper; failure detection without a GPU
  * fault). Every wait of the tcgen05 kernels on an mbarrier (a TMA copy landing, a product completing,
  * a tile drained) gives up after about 2 s of SM clock (longer at lower clocks), ORs

@@ -23,7 +23,7 @@ ZL_NOALLOC_MAX_ROWS = 65536   # rows of zl_op_local_loss_noalloc's static scratc
 EXPORTS = ["zl_create", "zl_free", "zl_set_stream", "zl_set_param", "zl_load_weights", "zl_get_param", "zl_param_numel",
            "zl_embed", "zl_forward_chunk", "zl_local_step", "zl_step", "zl_bp_step", "zl_eval_global_loss",
            "zl_read_losses", "zl_join", "zl_synchronize", "zl_peak_bytes", "zl_reset_peak", "zl_last_error",
-           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_head_loss", "zl_op_gemm", "zl_op_gemm_ex", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
+           "zl_op_local_loss", "zl_op_local_loss_noalloc", "zl_op_head_loss", "zl_op_gemm", "zl_op_gemm_ex", "zl_op_qkv_rope", "zl_op_attention", "zl_op_attention_bwd", "zl_profile", "zl_profile_read", "zl_kernel_launches", "zl_chunk_state_bytes", "zl_chunk_save",
            "zl_chunk_load", "zl_replay", "zl_wait_selftest"]
 
 
@@ -80,6 +80,7 @@ def _load() -> C.CDLL:
         "zl_op_head_loss": [i, vp, vp, vp, vp, i, i, i, i, f, i, i, vp, vp, vp, vp],
         "zl_op_gemm": [i, i, i, i, i, vp, vp, vp, vp],
         "zl_op_gemm_ex": [i, i, i, i, i, vp, vp, vp, vp, vp, i, vp],
+        "zl_op_qkv_rope": [i, i, i, i, vp, vp, vp, vp, vp, i, i, i, vp],
         "zl_op_attention": [i, vp, vp, vp, i, i, i, i, i, vp],
         "zl_op_attention_bwd": [i, vp, vp, vp, vp, vp, i, i, i, i, i, vp],
         "zl_profile": [vp, i],
@@ -325,6 +326,26 @@ def zl_op_gemm_ex(dtype: int, mode: int, M: int, N: int, K: int, A, B, Cm, bias=
         _need(R, act, "R")
     _check(_lib.zl_op_gemm_ex(dtype, mode, M, N, K, _p(A), _p(B), _p(Cm), _p(bias) if bias is not None else None,
                               _p(R) if R is not None else None, r_mode, stream))
+
+
+def zl_op_qkv_rope(dtype: int, M: int, N: int, K: int, A, B, Cm, cs, S: int, hd: int, rot_cols: int, bias=None,
+                   stream: int = 0) -> None:
+    """C = A B^T (+ bias), then rotate-half RoPE of the first rot_cols columns (heads of hd) of row n by
+    position n % S; cs: fp32 [S, hd/2, 2] (cos, sin)."""
+    act = ("bfloat16",) if dtype == ZL_DTYPE_BF16 else ("float32",)
+    _need(A, act, "A")
+    _need(B, act, "B")
+    _need(Cm, act, "C")
+    _need(cs, ("float32",), "cs")
+    if bias is not None:
+        _need(bias, ("float32",), "bias")
+        _need_numel(bias, N, "bias")
+    _need_numel(A, M * K, "A")
+    _need_numel(B, N * K, "B")
+    _need_numel(Cm, M * N, "C")
+    _need_numel(cs, S * hd, "cs")
+    _check(_lib.zl_op_qkv_rope(dtype, M, N, K, _p(A), _p(B), _p(Cm), _p(bias) if bias is not None else None, _p(cs),
+                               S, hd, rot_cols, stream))
 
 
 def zl_profile(ctx, on: bool) -> None:

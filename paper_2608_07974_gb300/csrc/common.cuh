@@ -154,6 +154,13 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 // tolerance), so every kernel that applies the step (the slab and range updates, the weight-gradient
 // GEMM's fused epilogue, the split-K reduction) computes the same bits from the same gradient, in about
 // a dozen instructions.
+// Rotate-half RoPE of one pair (x1 at column i, x2 at column i + hd/2 of a head) by the angle with
+// (cos, sin) = (c, sn): every product and sum explicitly rounded, so that every kernel that rotates
+// (the RoPE kernels and the QKV product's epilogue) gives the same bits.
+__device__ __forceinline__ void rope_rot(float x1, float x2, float c, float sn, float& y1, float& y2) {
+  y1 = __fsub_rn(__fmul_rn(x1, c), __fmul_rn(x2, sn));
+  y2 = __fadd_rn(__fmul_rn(x2, c), __fmul_rn(x1, sn));
+}
 struct AdamHP {
   float step, decay, inv_bc2, b1, omb1, b2, omb2, eps;   // step = lr / bc1, inv_bc2 = 1 / bc2
 };

@@ -301,6 +301,7 @@ struct ProfScope {
   int cls;
   double flops, bytes, launches;
   cudaEvent_t a = nullptr;
+  bool keep = true;   // false: nothing of the scope ran, no record
   ProfScope(zl_ctx* c_, cudaStream_t s_, int cls_, double fl, double by, double nl = 1)
       : c(c_), s(s_), cls(cls_), flops(fl), bytes(by), launches(nl) {
     if (c && c->prof) {
@@ -309,7 +310,7 @@ struct ProfScope {
     }
   }
   ~ProfScope() {
-    if (!a) return;
+    if (!a || !keep) return;
     if (c->evnext == c->evpool.size()) {
       cudaEvent_t e;
       if (cudaEventCreate(&e) != cudaSuccess) return;
@@ -459,11 +460,24 @@ void layer_fwd(zl_ctx* c, Chunk& k, int li, LayerSave& sv, const void* x, void* 
   const int N = B * S, dt = c->dt;
   sv.x = x;
   NF(c, s, x, Wm(k, li, P_N1W), Wm(k, li, P_N1B), sv.xn1, sv.rstd1, sv.mean1, N);
-  G(c, s, 0, N, c->qkvw, c->d, sv.xn1, Wc(c, k, li, P_WQKV), sv.qkv, Wm(k, li, P_BQKV), nullptr);
-  lora_fwd(c, k, li, 0, sv.xn1, sv.qkv, sv.u[0], N, s);
-  if (c->llama) {
-    ProfScope p(c, s, PC_ELEM, 0, 2.0 * esz(c) * (double)N * (c->H + c->Hkv) * c->hd);
-    launch_rope(dt, sv.qkv, c->rope_cs, N, S, c->H, c->Hkv, c->hd, 0, s);
+  // Llama without LoRA on the QKV product: RoPE in the product's epilogue; otherwise a RoPE pass after
+  // the product (and after the LoRA term, which the rotation must see)
+  bool rotated = false;
+  if (c->llama && dt == BF16 && lora_r16(c->cfg.lora_rank) <= 0) {
+    const double e = (double)esz(c), M = N, Nq = c->qkvw, K = c->d;
+    ProfScope p(c, s, PC_GEMM, 2.0 * M * Nq * K, e * (M * K + Nq * K + M * Nq));
+    const GemmRope r{c->rope_cs, S, c->hd, (c->H + c->Hkv) * c->hd};
+    rotated = gemm_tc_rope(N, c->qkvw, c->d, sv.xn1, Wc(c, k, li, P_WQKV), sv.qkv, Wm(k, li, P_BQKV), r, c->d_err,
+                           s, c->pool);
+    p.keep = rotated;
+  }
+  if (!rotated) {
+    G(c, s, 0, N, c->qkvw, c->d, sv.xn1, Wc(c, k, li, P_WQKV), sv.qkv, Wm(k, li, P_BQKV), nullptr);
+    lora_fwd(c, k, li, 0, sv.xn1, sv.qkv, sv.u[0], N, s);
+    if (c->llama) {
+      ProfScope p(c, s, PC_ELEM, 0, 2.0 * esz(c) * (double)N * (c->H + c->Hkv) * c->hd);
+      launch_rope(dt, sv.qkv, c->rope_cs, N, S, c->H, c->Hkv, c->hd, 0, s);
+    }
   }
   AF(c, s, sv.qkv, sv.att, sv.lse, B, S);
   G(c, s, 0, N, c->d, c->ad, sv.att, Wc(c, k, li, P_WO), sv.x2, Wm(k, li, P_BO), x);
@@ -2250,6 +2264,26 @@ zl_status zl_op_gemm(int dtype, int mode, int M, int N, int K, const void* A, co
   }
   return guarded(nullptr, [&]() -> zl_status {
     gemm(dtype, mode, M, N, K, A, B, C, nullptr, nullptr, (cudaStream_t)stream);
+    CHECK_LAUNCH();
+    return ZL_OK;
+  });
+}
+
+zl_status zl_op_qkv_rope(int dtype, int M, int N, int K, const void* A, const void* B, void* C, const float* bias,
+                         const float* cs, int S, int hd, int rot_cols, void* stream) {
+  if (!A || !B || !C || !cs) { g_err = "NULL argument"; return ZL_ERR_ARG; }
+  if ((dtype != 0 && dtype != 1) || M < 0 || N < 0 || K < 0 || S < 1 || hd < 2 || hd % 2 != 0 || rot_cols < 0 ||
+      rot_cols % hd != 0 || rot_cols > N) {
+    g_err = "bad dtype/size, or rot_cols not whole heads within N";
+    return ZL_ERR_ARG;
+  }
+  return guarded(nullptr, [&]() -> zl_status {
+    cudaStream_t s = (cudaStream_t)stream;
+    const GemmRope r{cs, S, hd, rot_cols};
+    if (!(dtype == BF16 && M > 0 && gemm_tc_rope(M, N, K, A, B, C, bias, r, nullptr, s, nullptr))) {
+      gemm(dtype, 0, M, N, K, A, B, C, bias, nullptr, s);
+      if (M > 0 && rot_cols > 0) launch_rope_heads(dtype, C, cs, M, S, rot_cols / hd, hd, N, 0, s);
+    }
     CHECK_LAUNCH();
     return ZL_OK;
   });

@@ -113,6 +113,8 @@ struct Args {
   float alpha;                // scale of the product
   int rmode;                  // R in modes 0/1: 0 adds it (residual); 1 multiplies by GELU'(R) (R = the GELU input)
   GemmUpdate u;               // mode 4
+  const float2* rope_cs;      // mode 0: rotate-half RoPE of columns < rope_cols (heads of rope_hd = 64 or 128),
+  int rope_S, rope_hd, rope_cols;   // row n by position n % rope_S (NULL: none)
 };
 
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, operand majors, N, M.
@@ -398,7 +400,7 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
     uint8_t* stage_out = outbuf + q * (2 * 32 * 128);
     const bool f32out = g.mode >= 2;
     const int ccols = f32out ? 32 : 64;   // columns per chunk
-    int it = 0, nchunk = 0;
+    int it = 0, nchunk = 0, drain = 0;
     for (int unit = unit0; unit < num_units; unit += ustride, ++it) {
       int tm, tn;
       unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
@@ -416,8 +418,69 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
 #pragma unroll 1
       for (int c = 0; c < BN; c += ccols, ++nchunk) {
         const int n0 = tn * BN + c;
+        if constexpr (BN >= 128 && !A_MN && !B_MN) {   // mode 0 kernels of 128- or 256-column tiles
+        if (g.rope_cs != nullptr && n0 < g.rope_cols) {
+          // one query / key head (rope_hd columns: one or two 64-column chunks, both staging buffers):
+          // pairs (i, i + hd/2) read from TMEM together, rounded to bf16, rotated, rounded again
+          const int hd = g.rope_hd, half = hd >> 1, nch = hd >> 6;
+          if (lane == 0) bulk_wait_read0();   // both buffers free
+          __syncwarp();
+          const float2* csr = g.rope_cs + (size_t)(m % g.rope_S) * half;
+#pragma unroll 1
+          for (int a = 0; a < half; a += 32) {
+            float4 cs4[16];   // (cos, sin) of pairs a .. a + 31 (16-byte loads, issued before the TMEM reads)
+#pragma unroll
+            for (int e = 0; e < 16; ++e) cs4[e] = reinterpret_cast<const float4*>(csr + a)[e];
+            float v1[32], v2[32];
+            tmem_ld32(trow + (uint32_t)(c + a), v1);
+            tmem_ld32(trow + (uint32_t)(c + a + half), v2);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              float x1 = v1[e] * g.alpha, x2 = v2[e] * g.alpha;
+              if (g.bias) {
+                if (n0 + a + e < g.N) x1 += g.bias[n0 + a + e];
+                if (n0 + a + half + e < g.N) x2 += g.bias[n0 + a + half + e];
+              }
+              x1 = __bfloat162float(__float2bfloat16_rn(x1));
+              x2 = __bfloat162float(__float2bfloat16_rn(x2));
+              const float4 c4 = cs4[e >> 1];
+              rope_rot(x1, x2, (e & 1) ? c4.z : c4.x, (e & 1) ? c4.w : c4.y, v1[e], v2[e]);
+            }
+#pragma unroll
+            for (int side = 0; side < 2; ++side) {
+              const float* vv = side ? v2 : v1;
+              const int col = a + side * half;   // column within the head
+              uint8_t* srow = stage_out + (col >> 6) * (32 * 128) + lane * 128;
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                __nv_bfloat162 hv[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) hv[e] = __floats2bfloat162_rn(vv[8 * k + 2 * e], vv[8 * k + 2 * e + 1]);
+                const int piece = ((col & 63) >> 3) + k;
+                *reinterpret_cast<uint4*>(srow + ((piece ^ (lane & 7)) << 4)) = *reinterpret_cast<const uint4*>(hv);
+              }
+            }
+          }
+          fence_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            for (int j = 0; j < nch; ++j) {
+              if (row0 < g.M && n0 + 64 * j < g.N) tma_store2d(&tcm, stage_out + j * (32 * 128), n0 + 64 * j, row0);
+              bulk_commit();
+            }
+          }
+          drain = 1;
+          c += hd - ccols;
+          nchunk += nch - 1;
+          continue;
+        }
+        }
         uint8_t* sbuf = stage_out + (nchunk & 1) * (32 * 128);
-        if (lane == 0) bulk_wait_read1();   // the store that last used this buffer has read it
+        if (lane == 0) {   // the store that last used this buffer has read it
+          if (drain) bulk_wait_read0();
+          else bulk_wait_read1();
+        }
+        drain = 0;
         __syncwarp();
         uint8_t* srow = sbuf + lane * 128;
         // 32 columns at a time: f32 chunks are one half, bf16 chunks two (16-byte pieces 4h .. 4h+3)
@@ -755,7 +818,8 @@ namespace {
 // Plans and launches one tensor-core GEMM (modes 0-2, or 4 with `u`); false if the shape or alignment
 // is outside the kernel's rules.
 bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
-            unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode, const GemmUpdate* u) {
+            unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode, const GemmUpdate* u,
+            const GemmRope* rope = nullptr) {
   if (!tc::init()) return false;
   if (M < 16 || N < 16 || K < 16) return false;
   auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
@@ -764,6 +828,10 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   if (u && (!al16(u->theta) || !al16(u->m) || !al16(u->v) || u->g || !u->comp || !al16(u->comp) || N % 8 != 0))
     return false;
   if (N % 8 != 0) return false;
+  // the rotation: bf16 C without residual, whole heads of 64 or 128 columns from column 0
+  if (rope && (mode != 0 || R || !rope->cs || ((uintptr_t)rope->cs & 7u) || (rope->hd != 64 && rope->hd != 128) ||
+               rope->S < 1 || rope->cols < 0 || rope->cols % rope->hd != 0 || rope->cols > N))
+    return false;
   if ((mode == 0 || mode == 1) && K % 8 != 0) return false;
   if (mode >= 2 && M % 8 != 0) return false;
   int bn = 128, splits = 1;
@@ -780,8 +848,17 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
       if (nf == 3 && (fp == 0 || fp == 1)) pair = fp && bn >= 128 ? 1 : 0;
     }
   }
+  if (rope) {   // one split (the reduction does not rotate); tiles of 128 or 256 columns (heads never straddle)
+    splits = 1;
+    if (bn < 128) bn = 128;
+    pair = bn >= 128 && M > tc::BM ? pair : 0;
+  }
   tc::Args a;
   a.M = M; a.N = N; a.K = K; a.mode = mode;
+  a.rope_cs = rope ? reinterpret_cast<const float2*>(rope->cs) : nullptr;
+  a.rope_S = rope ? rope->S : 1;
+  a.rope_hd = rope ? rope->hd : 0;
+  a.rope_cols = rope ? rope->cols : 0;
   a.C = C; a.bias = bias; a.R = (const bf16*)R; a.err = err; a.alpha = alpha; a.rmode = rmode;
   a.u = u ? *u : GemmUpdate{};
   a.tiles_m = (M + tc::BM - 1) / tc::BM;
@@ -841,6 +918,11 @@ bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* 
 bool gemm_tc_update(int M, int N, int K, const void* A, const void* B, const GemmUpdate& u, unsigned* err,
                     cudaStream_t s, cudaMemPool_t pool, float alpha) {
   return run_tc(4, M, N, K, A, B, u.theta, nullptr, nullptr, err, s, pool, alpha, 0, &u);
+}
+
+bool gemm_tc_rope(int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const GemmRope& r,
+                  unsigned* err, cudaStream_t s, cudaMemPool_t pool) {
+  return run_tc(0, M, N, K, A, B, C, bias, nullptr, err, s, pool, 1.f, 0, nullptr, &r);
 }
 
 }  // namespace zl

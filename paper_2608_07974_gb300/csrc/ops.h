@@ -47,6 +47,9 @@ void launch_partials_add(const float* part, int nb, int d, float* out, cudaStrea
 // cs: [S, hd/2] (cos, sin) pairs.
 void launch_rope(int dt, void* qkv, const float* cs, int N, int S, int H, int Hkv, int hd, int inverse,
                  cudaStream_t s);
+// The same on the first nh heads of rows of ld elements.
+void launch_rope_heads(int dt, void* qkv, const float* cs, int N, int S, int nh, int hd, int ld, int inverse,
+                       cudaStream_t s);
 void launch_swiglu_fwd(int dt, const void* gu, void* a, int N, int f, cudaStream_t s);
 void launch_swiglu_bwd(int dt, const void* gu, const void* da, void* dgu, int N, int f, cudaStream_t s);
 void launch_gelu_fwd(int dt, const void* x, void* y, size_t n, cudaStream_t s);
@@ -105,6 +108,18 @@ struct GemmUpdate {
 // (the caller then forms the gradient with gemm() and applies the step with launch_adamw_ranges).
 bool gemm_tc_update(int M, int N, int K, const void* A, const void* B, const GemmUpdate& u, unsigned* err,
                     cudaStream_t s, cudaMemPool_t pool, float alpha = 1.f);
+// Rotate-half RoPE applied by the forward QKV product's epilogue: output columns < cols (the query and key
+// heads, head dim hd = 64 or 128) of row n are rotated by the angles of position n % S, (cos, sin) pairs
+// from cs [S][hd / 2][2] (fp32). The product is rounded to the output type before the rotation, as a
+// separate RoPE pass over the stored product would see it.
+struct GemmRope {
+  const float* cs;
+  int S, hd, cols;
+};
+// C = A B^T (+ bias) in bf16 with the rotation in the epilogue (mode 0, no residual); false when the
+// tensor-core product or the rotation's rules do not hold (the caller then runs gemm() and launch_rope).
+bool gemm_tc_rope(int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const GemmRope& r,
+                  unsigned* err, cudaStream_t s, cudaMemPool_t pool);
 bool gemm_tc_available();
 bool gemm_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C, const float* bias, const void* R,
              unsigned* err, cudaStream_t s, cudaMemPool_t pool, float alpha, int rmode = 0);
