@@ -188,6 +188,15 @@ __device__ __forceinline__ float rcp_approx(float x) {
   asm("rcp.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
   return r;
 }
+// Blocked layout of the fp32 master and AdamW moments of a matrix [M, N] (M % 16 == 0, N % 32 == 0)
+// whose optimizer step runs in its weight-gradient product: 16 x 32 pieces of 512 contiguous floats
+// (row-major inside a piece), the pieces in row-major order over the [M / 16, N / 32] grid. A piece is
+// what one epilogue warp updates at a time, so the update streams whole 2 KB runs instead of 128-byte
+// segments of rows far apart (about 10% more of the HBM rate on the 7B-shaped matrices). The compute
+// copy and every gradient stay row-major.
+__host__ __device__ __forceinline__ size_t blk_index(size_t r, size_t c, size_t N) {
+  return ((r >> 4) * (N >> 5) + (c >> 5)) * 512 + (r & 15) * 32 + (c & 31);
+}
 __device__ __forceinline__ void adamw_elem(float& th, float& m, float& v, float g, const AdamHP& h) {
   m = __fmaf_rn(h.b1, m, __fmul_rn(h.omb1, g));
   v = __fmaf_rn(h.b2, v, __fmul_rn(__fmul_rn(h.omb2, g), g));

@@ -84,6 +84,8 @@ struct Layer {
   int slab[P_COUNT];
   size_t la[4], lb[4];        // LoRA A [r16, in] and B^T [r16, out] offsets in the trainable slab
   int lin_in[4], lin_out[4];  // shapes of the four linears
+  bool blk[P_COUNT];          // trainable matrix whose master and moments are in the blocked layout
+  int rows[P_COUNT], cols[P_COUNT];   // [rows, cols] of each matrix (out, in)
 };
 
 struct Chunk {
@@ -349,9 +351,10 @@ void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, 
   }
   const zl_train_cfg& cf = c->cfg;
   const size_t off = k.layers[li].off[p];
+  const bool blk = k.layers[li].blk[p];
   const GemmUpdate u{k.master + off, k.m + off, k.v + off, nullptr,
                      c->dt == BF16 ? (void*)((bf16*)k.comp + off) : nullptr, k.d_hp, cf.beta1, cf.beta2, cf.eps,
-                     cf.weight_decay, 1.f};
+                     cf.weight_decay, 1.f, blk ? 1 : 0};
   const double e = (double)esz(c), mn = (double)M * N;
   // operands, then read theta, m, v and write them back, plus the compute copy
   const double upd = 24.0 * mn + (c->dt == BF16 ? 2.0 : 0.0) * mn;
@@ -365,8 +368,12 @@ void GW(zl_ctx* c, cudaStream_t s, Chunk& k, int li, PK p, int M, int N, int K, 
   }
   float* gg = g ? g : tmp;
   gemm(c->dt, 2, M, N, K, A, B, gg, nullptr, nullptr, s, c->d_err, c->pool);
-  launch_adamw_span(u.theta, gg, u.m, u.v, u.comp, (size_t)M * N, k.d_hp, cf.beta1, cf.beta2, cf.eps, cf.weight_decay,
-                    u.gscale, s);
+  if (blk)
+    launch_adamw_span_blk(u.theta, gg, u.m, u.v, u.comp, M, N, k.d_hp, cf.beta1, cf.beta2, cf.eps, cf.weight_decay,
+                          u.gscale, s);
+  else
+    launch_adamw_span(u.theta, gg, u.m, u.v, u.comp, (size_t)M * N, k.d_hp, cf.beta1, cf.beta2, cf.eps,
+                      cf.weight_decay, u.gscale, s);
   pfree(tmp, s);
 }
 
@@ -997,6 +1004,7 @@ struct Found {
   size_t off = 0;
   int frozen = 0;               // 1 tok_emb, 2 pos_emb, 3 norm_f.weight, 4 norm_f.bias, 5 lm_head
   int trows = 0, tcols = 0;     // > 0: user layout [tcols, trows], stored transposed as [trows, tcols]
+  int brows = 0, bcols = 0;     // > 0: master and moments stored in the blocked layout of [brows, bcols]
 };
 
 bool lookup(zl_ctx* c, const std::string& name, Found& f) {
@@ -1035,7 +1043,10 @@ bool lookup(zl_ctx* c, const std::string& name, Found& f) {
     const Layer& L = ck.layers[l - ck.l0];
     for (int p = 0; p < P_COUNT; ++p)
       if (L.has[p] && suf == kPName[p]) {
-        if (L.slab[p] == S_TRAIN) f = Found{ck.master + L.off[p], true, L.numel[p], &ck, L.off[p], 0};
+        if (L.slab[p] == S_TRAIN) {
+          f = Found{ck.master + L.off[p], true, L.numel[p], &ck, L.off[p], 0};
+          if (L.blk[p]) { f.brows = L.rows[p]; f.bcols = L.cols[p]; }
+        }
         else if (L.slab[p] == S_FVEC) f = Found{ck.fvec + L.off[p], true, L.numel[p], nullptr, 0, 0};
         else f = Found{(char*)ck.fmat + L.off[p] * esz(c), c->dt == F32, L.numel[p], nullptr, 0, 0};
         return true;
@@ -1239,6 +1250,7 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       const bool is_mat[P_COUNT] = {false, false, true, false, true, false, false, false, true, false, true, false};
       for (int l = ck.l0; l < ck.l1; ++l) {
         Layer L;
+        for (int p = 0; p < P_COUNT; ++p) { L.blk[p] = false; L.rows[p] = L.cols[p] = 0; }
         size_t shp[P_COUNT] = {(size_t)d, (size_t)d, (size_t)c->qkvw * d, (size_t)c->qkvw, (size_t)d * c->ad, (size_t)d,
                                (size_t)d, (size_t)d, (size_t)c->f1 * d, (size_t)c->f, (size_t)d * c->f, (size_t)d};
         for (int p = 0; p < P_COUNT; ++p) {
@@ -1277,6 +1289,8 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
         for (int i = 0; i < 4; ++i) {
           L.lin_in[i] = ins[i];
           L.lin_out[i] = outs[i];
+          L.rows[kLoraP[i]] = outs[i];
+          L.cols[kLoraP[i]] = ins[i];
           L.la[i] = L.lb[i] = 0;
           if (r > 0) {
             L.la[i] = off;
@@ -1329,6 +1343,13 @@ zl_status zl_create(const zl_model_dims* dims, int K, const int* bounds, const z
       const bool fused_always = c->dt == BF16 && cfg->accum_m == 1 && !cfg->unfused_update && r == 0 &&
                                 gemm_tc_available();
       ck.grad_n = fused_always ? std::max<size_t>(ck.ad_end, 64) : ck.n;
+      // ... and, where the shape allows it, their master and moments take the blocked layout the fused
+      // update streams fastest (the weight-gradient products are then the only kernels that step them)
+      for (Layer& L : ck.layers)
+        for (int i = 0; i < 4; ++i) {
+          const int p = kLoraP[i];
+          L.blk[p] = fused_always && L.has[p] && L.slab[p] == S_TRAIN && L.rows[p] % 16 == 0 && L.cols[p] % 32 == 0;
+        }
       ck.master = (float*)salloc(c, ck.n * 4);
       ck.grad = (float*)salloc(c, ck.grad_n * 4);
       ck.m = (float*)salloc(c, ck.n * 4);
@@ -1414,6 +1435,14 @@ zl_status zl_set_param(zl_ctx* c, const char* name, const void* src, size_t byte
         for (int j = 0; j < f.trows; ++j) t[(size_t)j * f.tcols + o] = h[(size_t)o * f.trows + j];
       CK(cudaMemcpy(f.dev, t.data(), bytes, cudaMemcpyHostToDevice));
       if (c->dt == BF16) launch_f32_to_bf16((const float*)f.dev, (bf16*)f.chunk->comp + f.off, f.numel, 0);
+    } else if (f.chunk && f.brows > 0) {   // row-major in, blocked master; the compute copy from the row-major
+      float* tmp = nullptr;
+      CK(cudaMalloc(&tmp, bytes));
+      CK(cudaMemcpy(tmp, src, bytes, kind));
+      launch_blk_permute(tmp, (float*)f.dev, f.brows, f.bcols, 1, 0);
+      if (c->dt == BF16) launch_f32_to_bf16(tmp, (bf16*)f.chunk->comp + f.off, f.numel, 0);
+      CK(cudaDeviceSynchronize());
+      CK(cudaFree(tmp));
     } else if (f.chunk) {
       CK(cudaMemcpy(f.dev, src, bytes, kind));
       if (c->dt == BF16) launch_f32_to_bf16((const float*)f.dev, (bf16*)f.chunk->comp + f.off, f.numel, 0);
@@ -1464,6 +1493,13 @@ zl_status zl_get_param(zl_ctx* c, const char* name, int which, void* dst, size_t
       for (int j = 0; j < f.trows; ++j)
         for (int o = 0; o < f.tcols; ++o) t[(size_t)o * f.trows + j] = h[(size_t)j * f.tcols + o];
       CK(cudaMemcpy(dst, t.data(), bytes, on_device ? cudaMemcpyHostToDevice : cudaMemcpyHostToHost));
+    } else if (f.brows > 0) {   // blocked master or moment -> row-major
+      float* tmp = nullptr;
+      CK(cudaMalloc(&tmp, bytes));
+      launch_blk_permute((const float*)srcp, tmp, f.brows, f.bcols, 0, 0);
+      CK(cudaDeviceSynchronize());
+      CK(cudaMemcpy(dst, tmp, bytes, kind));
+      CK(cudaFree(tmp));
     } else if (f.fp32 || which > 0) {
       CK(cudaMemcpy(dst, srcp, bytes, kind));
     } else {
@@ -1628,6 +1664,22 @@ struct CkptHeader {
 };
 constexpr uint64_t kCkptMagic = 0x31304B434C5A4C5AULL;   // "ZLZLCK01"
 
+bool has_blocked(const Chunk& ck) {
+  for (const Layer& L : ck.layers)
+    for (int p = 0; p < P_COUNT; ++p)
+      if (L.blk[p]) return true;
+  return false;
+}
+// Copies one slab-sized fp32 array (n floats) between device buffers, turning every blocked matrix into
+// row-major (to_blk = 0) or back (1), so checkpoints hold the same row-major layout whatever the engine's.
+void slab_xfer(Chunk& ck, const float* src, float* dst, int to_blk) {
+  CK(cudaMemcpy(dst, src, ck.n * sizeof(float), cudaMemcpyDeviceToDevice));
+  for (const Layer& L : ck.layers)
+    for (int p = 0; p < P_COUNT; ++p)
+      if (L.blk[p]) launch_blk_permute(src + L.off[p], dst + L.off[p], L.rows[p], L.cols[p], to_blk, 0);
+  CK(cudaDeviceSynchronize());
+}
+
 zl_status zl_chunk_state_bytes(zl_ctx* c, int k, size_t* bytes) {
   if (!c || !bytes) { g_err = "NULL argument"; return ZL_ERR_ARG; }
   if (k < 1 || k > c->K) { g_err = "chunk index out of [1, K]"; return ZL_ERR_ARG; }
@@ -1646,11 +1698,18 @@ zl_status zl_chunk_save(zl_ctx* c, int k, void* dst, size_t bytes) {
     std::memcpy(dst, &h, sizeof h);
     float* p = reinterpret_cast<float*>(static_cast<char*>(dst) + sizeof h);
     const size_t sz = ck.n * sizeof(float);
-    CK(cudaMemcpy(p, ck.master, sz, cudaMemcpyDeviceToHost));
+    float* tmp = nullptr;
+    if (has_blocked(ck)) CK(cudaMalloc(&tmp, sz));
+    auto out = [&](const float* a, float* h) {   // row-major copy of a slab array to the host
+      if (tmp) slab_xfer(ck, a, tmp, 0);
+      CK(cudaMemcpy(h, tmp ? tmp : a, sz, cudaMemcpyDeviceToHost));
+    };
+    out(ck.master, p);
     CK(cudaMemcpy(p + ck.n, ck.grad, ck.grad_n * sizeof(float), cudaMemcpyDeviceToHost));
     std::memset(p + ck.n + ck.grad_n, 0, (ck.n - ck.grad_n) * sizeof(float));   // unstored gradients are zero
-    CK(cudaMemcpy(p + 2 * ck.n, ck.m, sz, cudaMemcpyDeviceToHost));
-    CK(cudaMemcpy(p + 3 * ck.n, ck.v, sz, cudaMemcpyDeviceToHost));
+    out(ck.m, p + 2 * ck.n);
+    out(ck.v, p + 3 * ck.n);
+    if (tmp) CK(cudaFree(tmp));
     return ZL_OK;
   });
 }
@@ -1669,11 +1728,24 @@ zl_status zl_chunk_load(zl_ctx* c, int k, const void* src, size_t bytes) {
     sync_all(c, -1);
     const float* p = reinterpret_cast<const float*>(static_cast<const char*>(src) + sizeof h);
     const size_t sz = ck.n * sizeof(float);
-    CK(cudaMemcpy(ck.master, p, sz, cudaMemcpyHostToDevice));
+    if (has_blocked(ck)) {   // the blob is row-major: through a device copy into the blocked layout
+      float* tmp = nullptr;
+      CK(cudaMalloc(&tmp, sz));
+      CK(cudaMemcpy(tmp, p, sz, cudaMemcpyHostToDevice));
+      slab_xfer(ck, tmp, ck.master, 1);
+      if (c->dt == BF16) launch_f32_to_bf16(tmp, ck.comp, ck.n, 0);
+      CK(cudaMemcpy(tmp, p + 2 * ck.n, sz, cudaMemcpyHostToDevice));
+      slab_xfer(ck, tmp, ck.m, 1);
+      CK(cudaMemcpy(tmp, p + 3 * ck.n, sz, cudaMemcpyHostToDevice));
+      slab_xfer(ck, tmp, ck.v, 1);
+      CK(cudaFree(tmp));
+    } else {
+      CK(cudaMemcpy(ck.master, p, sz, cudaMemcpyHostToDevice));
+      CK(cudaMemcpy(ck.m, p + 2 * ck.n, sz, cudaMemcpyHostToDevice));
+      CK(cudaMemcpy(ck.v, p + 3 * ck.n, sz, cudaMemcpyHostToDevice));
+      if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
+    }
     CK(cudaMemcpy(ck.grad, p + ck.n, ck.grad_n * sizeof(float), cudaMemcpyHostToDevice));
-    CK(cudaMemcpy(ck.m, p + 2 * ck.n, sz, cudaMemcpyHostToDevice));
-    CK(cudaMemcpy(ck.v, p + 3 * ck.n, sz, cudaMemcpyHostToDevice));
-    if (c->dt == BF16) launch_f32_to_bf16(ck.master, ck.comp, ck.n, 0);
     CK(cudaDeviceSynchronize());
     ck.t = h.t;
     const long long tt = h.t;

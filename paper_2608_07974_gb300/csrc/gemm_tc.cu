@@ -51,10 +51,13 @@ struct Cfg {
 // store covers four whole 128-byte lines. upd_load issues the chunk's loads; upd_apply applies the AdamW
 // step (adamw_elem) with G = gscale * acc to the loaded state and writes the fp32 master, both moments
 // and the bf16 compute copy back. The state is streamed (evict-first): it is touched once, and L2 is
-// kept for the operand tiles.
+// kept for the operand tiles. With the blocked state layout (u.blk) the chunk is one 16 x 32 piece of
+// it: lane l's row j sits at piece offset 4 l + 128 j, so each warp-wide access covers 512 contiguous
+// bytes.
 struct UpdRegs {
   float4 th[4], mm[4], vv[4];
-  size_t at;     // element offset of row j = 0; row j sits 4 j rows further down
+  size_t at;     // state offset of row j = 0; row j sits 4 j rows further down (blocked: 128 j floats)
+  size_t ct;     // row-major offset of row j = 0 (the compute copy)
   unsigned ok;   // bit j: row j is inside the tensor
 };
 __device__ __forceinline__ void upd_load(const GemmUpdate& u, UpdRegs& r, int row0, int h, int col0, int M, int N,
@@ -63,11 +66,13 @@ __device__ __forceinline__ void upd_load(const GemmUpdate& u, UpdRegs& r, int ro
   const int col = col0 + 4 * (lane & 7);
   if (!valid || col >= N) return;
   const int row = row0 + 16 * h + (lane >> 3);
-  r.at = (size_t)row * N + col;
+  r.ct = (size_t)row * N + col;
+  r.at = u.blk ? blk_index((size_t)(row0 + 16 * h), (size_t)col0, (size_t)N) + 4 * lane : r.ct;
+  const size_t sj = u.blk ? 128 : (size_t)4 * N;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     if (row + 4 * j < M) {
-      const size_t a = r.at + (size_t)(4 * j) * N;
+      const size_t a = r.at + j * sj;
       r.ok |= 1u << j;
       r.th[j] = __ldcs(reinterpret_cast<const float4*>(u.theta + a));
       r.mm[j] = __ldcs(reinterpret_cast<const float4*>(u.m + a));
@@ -78,10 +83,11 @@ __device__ __forceinline__ void upd_load(const GemmUpdate& u, UpdRegs& r, int ro
 __device__ __forceinline__ void upd_apply(const GemmUpdate& u, const AdamHP& h, UpdRegs& r, const uint8_t* sp,
                                           int hh, int N, int lane) {
   const int piece = lane & 7;
+  const size_t sj = u.blk ? 128 : (size_t)4 * N;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     if (!(r.ok >> j & 1u)) continue;
-    const size_t a = r.at + (size_t)(4 * j) * N;
+    const size_t a = r.at + j * sj;
     const int rr = 16 * hh + (lane >> 3) + 4 * j;
     const float4 a4 = *reinterpret_cast<const float4*>(sp + rr * 128 + ((piece ^ (rr & 7)) << 4));
     const float acc[4] = {a4.x, a4.y, a4.z, a4.w};
@@ -92,7 +98,7 @@ __device__ __forceinline__ void upd_apply(const GemmUpdate& u, const AdamHP& h, 
     __stcs(reinterpret_cast<float4*>(u.m + a), r.mm[j]);
     __stcs(reinterpret_cast<float4*>(u.v + a), r.vv[j]);
     __nv_bfloat162 c2[2] = {__floats2bfloat162_rn(tp[0], tp[1]), __floats2bfloat162_rn(tp[2], tp[3])};
-    __stcs(reinterpret_cast<uint2*>((bf16*)u.comp + a), *reinterpret_cast<const uint2*>(c2));
+    __stcs(reinterpret_cast<uint2*>((bf16*)u.comp + r.ct + (size_t)(4 * j) * N), *reinterpret_cast<const uint2*>(c2));
   }
 }
 
@@ -328,7 +334,9 @@ __global__ void __launch_bounds__(UPD ? kThreadsUpd : kThreads, 1)
         unit_tile(g, unit, num_tiles, PAIR, crank, tm, tn);
         const int row = tm * BM + q * 32 + 16 * (k & 1) + lane, col = tn * BN + 32 * (part + WQ * (k >> 1));
         if (row >= g.M || col >= g.N) return;
-        const size_t at = (size_t)row * g.N + col;
+        // blocked: line `lane` of the chunk's 2 KB piece; row-major: row `lane`'s 128-byte segment
+        const size_t at = g.u.blk ? blk_index((size_t)(row - lane), (size_t)col, (size_t)g.N) + 32 * lane
+                                  : (size_t)row * g.N + col;
         asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.theta + at));
         asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.m + at));
         asm volatile("prefetch.global.L2 [%0];" ::"l"(g.u.v + at));
@@ -600,18 +608,19 @@ __global__ void splitk_reduce_k(const float* __restrict__ ws, int splits, int M,
     for (int q = 0; q < 8; ++q) acc[q] *= alpha;
     if (mode == 4) {
       float th[8], mm[8], vv[8], gg[8];
-      Vec8<float>::load(u.theta + e, th);
-      Vec8<float>::load(u.m + e, mm);
-      Vec8<float>::load(u.v + e, vv);
+      const size_t se = u.blk ? blk_index(e / N, e % N, (size_t)N) : e;   // eight columns stay contiguous
+      Vec8<float>::load(u.theta + se, th);
+      Vec8<float>::load(u.m + se, mm);
+      Vec8<float>::load(u.v + se, vv);
       if (u.g) Vec8<float>::load(u.g + e, gg);
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         const float gsum = u.g ? __fadd_rn(gg[q], acc[q]) : acc[q];
         adamw_elem(th[q], mm[q], vv[q], __fmul_rn(gsum, u.gscale), hpv);
       }
-      Vec8<float>::store(u.theta + e, th);
-      Vec8<float>::store(u.m + e, mm);
-      Vec8<float>::store(u.v + e, vv);
+      Vec8<float>::store(u.theta + se, th);
+      Vec8<float>::store(u.m + se, mm);
+      Vec8<float>::store(u.v + se, vv);
       if (u.comp) Vec8<bf16>::store((bf16*)u.comp + e, th);
       if (u.g) {
         const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -825,7 +834,8 @@ bool run_tc(int mode, int M, int N, int K, const void* A, const void* B, void* C
   auto al16 = [](const void* p) { return ((uintptr_t)p & 15u) == 0; };
   if (!al16(A) || !al16(B) || !al16(C) || (R && !al16(R))) return false;
   // the fused update: 16-byte aligned state rows, a compute copy, no accumulated gradient
-  if (u && (!al16(u->theta) || !al16(u->m) || !al16(u->v) || u->g || !u->comp || !al16(u->comp) || N % 8 != 0))
+  if (u && (!al16(u->theta) || !al16(u->m) || !al16(u->v) || u->g || !u->comp || !al16(u->comp) || N % 8 != 0 ||
+            (u->blk && (M % 16 != 0 || N % 32 != 0))))
     return false;
   if (N % 8 != 0) return false;
   // the rotation: bf16 C without residual, whole heads of 64 or 128 columns from column 0

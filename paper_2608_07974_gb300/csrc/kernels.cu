@@ -1200,6 +1200,57 @@ void launch_adamw_ranges(float* theta, float* g, float* m, float* v, void* comp,
              b2, eps, wd, gscale);
 }
 
+// One thread per four consecutive columns of one row (contiguous in both layouts).
+__global__ void adamw_blk_k(float* __restrict__ th, float* __restrict__ g, float* __restrict__ m,
+                            float* __restrict__ v, __nv_bfloat162* __restrict__ comp, int M, int N,
+                            const float* __restrict__ hp, float b1, float b2, float eps, float wd, float gscale) {
+  pdl_wait();
+  pdl_trigger();
+  const AdamHP h = adam_hp(hp, b1, b2, eps, wd);
+  const size_t n4 = (size_t)M * N / 4;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
+    const size_t e = 4 * i, b = blk_index(e / N, e % N, N);
+    float4 t = *reinterpret_cast<float4*>(th + b), gg = *reinterpret_cast<float4*>(g + e),
+           mm = *reinterpret_cast<float4*>(m + b), vv = *reinterpret_cast<float4*>(v + b);
+    float* tp = &t.x; float* gp = &gg.x; float* mp = &mm.x; float* vp = &vv.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) adamw_elem(tp[q], mp[q], vp[q], __fmul_rn(gp[q], gscale), h);
+    *reinterpret_cast<float4*>(th + b) = t;
+    *reinterpret_cast<float4*>(m + b) = mm;
+    *reinterpret_cast<float4*>(v + b) = vv;
+    *reinterpret_cast<float4*>(g + e) = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (comp) {
+      comp[2 * i] = __floats2bfloat162_rn(t.x, t.y);
+      comp[2 * i + 1] = __floats2bfloat162_rn(t.z, t.w);
+    }
+  }
+}
+
+void launch_adamw_span_blk(float* theta, float* g, float* m, float* v, void* comp, int M, int N, const float* hp,
+                           float b1, float b2, float eps, float wd, float gscale, cudaStream_t s) {
+  const size_t n4 = (size_t)M * N / 4;
+  if (n4 == 0) return;
+  note_launch(1);
+  const int th = 256, gr = grid_for(n4, th, 152 * 8);
+  launch_pdl(adamw_blk_k, gr, th, 0, s, theta, g, m, v, (__nv_bfloat162*)comp, M, N, hp, b1, b2, eps, wd, gscale);
+}
+
+__global__ void blk_permute_k(const float* __restrict__ src, float* __restrict__ dst, int M, int N, int to_blk) {
+  const size_t n4 = (size_t)M * N / 4;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
+    const size_t e = 4 * i, b = blk_index(e / N, e % N, N);
+    if (to_blk) *reinterpret_cast<float4*>(dst + b) = *reinterpret_cast<const float4*>(src + e);
+    else *reinterpret_cast<float4*>(dst + e) = *reinterpret_cast<const float4*>(src + b);
+  }
+}
+
+void launch_blk_permute(const float* src, float* dst, int M, int N, int to_blk, cudaStream_t s) {
+  const size_t n4 = (size_t)M * N / 4;
+  if (n4 == 0) return;
+  note_launch(1);
+  blk_permute_k<<<grid_for(n4, 256), 256, 0, s>>>(src, dst, M, N, to_blk);
+}
+
 __global__ void f32_to_bf16_k(const float* __restrict__ a, bf16* __restrict__ b, size_t n) {
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
     b[i] = __float2bfloat16_rn(a[i]);

@@ -80,6 +80,13 @@ void launch_adamw_span(float* theta, float* g, float* m, float* v, void* comp, s
 void launch_adamw_ranges(float* theta, float* g, float* m, float* v, void* comp, const long long* ranges,
                          int nranges, size_t max_len, const float* hp, float b1, float b2, float eps, float wd,
                          float gscale, cudaStream_t s);
+// AdamW over a matrix [M, N] (M % 16 == 0, N % 32 == 0) whose theta, m and v are in the blocked layout of
+// blk_index while g (zeroed here) and comp are row-major; hp already written for this step.
+void launch_adamw_span_blk(float* theta, float* g, float* m, float* v, void* comp, int M, int N, const float* hp,
+                           float b1, float b2, float eps, float wd, float gscale, cudaStream_t s);
+// Copies a matrix [M, N] (M % 16 == 0, N % 32 == 0) between row-major and the blocked layout of
+// blk_index: to_blk = 1 reads src row-major and writes dst blocked, 0 the reverse.
+void launch_blk_permute(const float* src, float* dst, int M, int N, int to_blk, cudaStream_t s);
 void launch_f32_to_bf16(const float* src, void* dst, size_t n, cudaStream_t s);
 
 // GEMM (row-major): mode 0: C = A[M,K] B[N,K]^T (+ bias[N]) (+ R[M,N]); mode 1: C = A[M,K] B[K,N] (+ R);
@@ -97,12 +104,14 @@ void gemm(int dt, int mode, int M, int N, int K, const void* A, const void* B, v
 // compute copy are theta, m, v and comp (comp may be NULL), the window's gradient is
 // G = gscale * (g + alpha A^T B), g the accumulated gradient of the window's earlier micro-batches
 // (NULL when there are none; zeroed here otherwise), and AdamW (hp as written by the step-count
-// kernel) updates theta, m, v and comp in place; no gradient is stored.
+// kernel) updates theta, m, v and comp in place; no gradient is stored. blk = 1: theta, m and v are in
+// the blocked layout of blk_index (comp and g stay row-major).
 struct GemmUpdate {
   float *theta, *m, *v, *g;
   void* comp;
   const float* hp;
   float b1, b2, eps, wd, gscale;
+  int blk;
 };
 // bf16 operands on the tcgen05 kernel; false when the shape or alignment rules of mode 2 do not hold
 // (the caller then forms the gradient with gemm() and applies the step with launch_adamw_ranges).

@@ -21,6 +21,9 @@ GPT2S = synth.Workload("fused-gpt2-bf16", synth.ModelDims(synth.ARCH_GPT2, 4, 25
                        batch=2, seq=256, K=2, steps=4, seed=1234 + 1)
 LLAMAS = synth.Workload("fused-llama-bf16", synth.ModelDims(synth.ARCH_LLAMA, 2, 256, 4, 2, 704, 512, 256), "bf16",
                         batch=2, seq=128, K=2, steps=4, seed=1234 + 2)
+# the down projection [256, 344] keeps row-major state (344 % 32 != 0), the other matrices take the blocked one
+MIXED = synth.Workload("fused-llama-mixed", synth.ModelDims(synth.ARCH_LLAMA, 2, 256, 4, 2, 344, 512, 128), "bf16",
+                       batch=2, seq=128, K=2, steps=4, seed=1234 + 4)
 # ragged everywhere: d 200 (head dim 50, padded to 64 in attention), gate/up 688 rows, FFN 344 columns
 ODD = synth.Workload("fused-llama-odd", synth.ModelDims(synth.ARCH_LLAMA, 2, 200, 4, 2, 344, 500, 192), "bf16",
                      batch=3, seq=96, K=2, steps=4, seed=1234 + 3)
@@ -63,7 +66,8 @@ def _run(w, P, kind, steps, **kw):
     return losses, st
 
 
-@pytest.mark.parametrize("w", [GPT2S, LLAMAS, ODD, synth.TINY], ids=["gpt2s-bf16", "llama-bf16", "odd-bf16", "tiny-f32"])
+@pytest.mark.parametrize("w", [GPT2S, LLAMAS, MIXED, ODD, synth.TINY],
+                         ids=["gpt2s-bf16", "llama-bf16", "mixed-bf16", "odd-bf16", "tiny-f32"])
 @pytest.mark.parametrize("kind", ["zl", "bp", "local"])
 @pytest.mark.parametrize("accum_m", [1, 2])
 def test_fused_update_equals_unfused_bitwise(w, kind, accum_m):
@@ -98,3 +102,33 @@ def test_fused_update_with_adapters():
     assert a[0] == b[0]
     for key in b[1]:
         assert torch.equal(a[1][key], b[1][key]), key
+
+
+def test_checkpoints_move_between_blocked_and_row_major_state():
+    """With the fused update the matrices' master and moments are held in a blocked layout (16 x 32 pieces)
+    where the shape allows it; the unfused engine keeps them row-major. Checkpoints are row-major either
+    way: a chunk saved by one engine and loaded into the other continues exactly like an uninterrupted run
+    of either (parameters, moments and losses bit for bit)."""
+    from paper_2608_07974_gb300 import binding as b
+    w = MIXED
+    P = _params(w)
+    ref = _run(w, P, "zl", 4)
+    for src_kw, dst_kw in (({}, {"unfused_update": True}), ({"unfused_update": True}, {})):
+        src, dst = engine_for(w, **src_kw), engine_for(w, **dst_kw)
+        src.load(P)
+        dst.load(P)   # the frozen tensors (embedding, head, final norm) are not part of a chunk checkpoint
+        losses = []
+        for s in range(2):
+            ids, labels = (t.cuda() for t in synth.make_batch(w, s))
+            losses.append(src.step(ids, labels))
+        for k in range(1, w.K + 1):
+            b.zl_chunk_load(dst.ctx, k, b.zl_chunk_save(src.ctx, k))
+        src.close()
+        for s in range(2, 4):
+            ids, labels = (t.cuda() for t in synth.make_batch(w, s))
+            losses.append(dst.step(ids, labels))
+        st = _state(dst, w)
+        dst.close()
+        assert losses == ref[0], (src_kw, dst_kw)
+        for key in ref[1]:
+            assert torch.equal(st[key], ref[1][key]), (src_kw, dst_kw, key)
