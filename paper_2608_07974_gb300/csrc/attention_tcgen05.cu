@@ -34,16 +34,19 @@ __device__ __forceinline__ float ex2(float x) {
 }
 
 // ==============================================================================================
-// Forward, one pass with lazy rescaling. Per 128-key block j: S_j = Q K_j^T (TMEM, double-buffered),
-// then O += P_{j-1} V_{j-1}. The softmax warps (two per lane quadrant, one 64-key half each) exchange
-// the half-row maxima of S_j through shared memory, so both take the same decisions, and keep a
-// running maximum m that moves only when the block maximum exceeds it by more than 8 (log2 units):
-// P = 2^(s - m) then stays at most 256 (exact in fp32 sums, the usual bf16 rounding), and O and the
-// row sum l are rescaled (in TMEM / registers) only on such a move. The rescale happens after the
-// wait that P's buffer is free, which is also the completion of the previous P V product, so no
-// product touches O meanwhile. At the end O / l is the softmax-weighted sum and m + log2 l the
-// row's log-sum-exp. One exponential per score and 12 (head dim 64) or 16 (128) products per block,
-// against two and 16 / 20 for the two-pass kernel.
+// Forward, one pass with lazy rescaling, persistent. Each CTA takes its share of the tiles (128 query
+// rows of one batch and head; snake_tile's deal of a longest-first order), so the next tile's Q and K/V
+// loads and first S product overlap the current tile's last softmax block and its output; the output
+// accumulator O is double-buffered in TMEM by tile parity. Per 128-key block j: S_j = Q K_j^T (TMEM,
+// double-buffered), then O += P_{j-1} V_{j-1} (across a tile boundary: the previous tile's last block).
+// The softmax warps (two per lane quadrant, one 64-key half each) exchange the half-row maxima of S_j
+// through shared memory, so both take the same decisions, and keep a running maximum m that moves only
+// when the block maximum exceeds it by more than 8 (log2 units): P = 2^(s - m) then stays at most 256
+// (exact in fp32 sums, the usual bf16 rounding), and O and the row sum l are rescaled (in TMEM /
+// registers) only on such a move. The rescale happens after the wait that P's buffer is free, which is
+// also the completion of the previous P V product, so no product touches O meanwhile. At the end O / l
+// is the softmax-weighted sum and m + log2 l the row's log-sum-exp. Barrier phases follow global block
+// and tile counters, so they run on across tiles.
 // ==============================================================================================
 template <int HD>
 struct F1Cfg {
@@ -55,13 +58,32 @@ struct F1Cfg {
   static constexpr int PBYTES = QB * KB * 2;
   static constexpr int XBYTES = (2 * 2 * QB + 2 * QB) * 4;   // maxima [2 buffers][2 halves][rows], sums [2][rows]
   static constexpr int SMEM = QBYTES + STAGES * STAGE + PBYTES + XBYTES + 256 + 1024;
+  static constexpr uint32_t OCOL = 256;                        // O of even tiles; odd tiles at OCOL + HD
   static_assert(SMEM <= 232448, "shared memory per CTA");
+  static_assert(OCOL + 2 * HD <= 512, "TMEM columns");
 };
+
+// The it-th tile of CTA c among G: the tiles are sorted longest first and dealt out in rounds of G whose
+// direction alternates (round 0: c, round 1: 2G - 1 - c, ...), so every CTA's long and short tiles even
+// out; past the last tile it returns a value >= every tile count (every later round is past it too).
+__device__ __forceinline__ int snake_tile(int it, int c, int G) {
+  return (it & 1) ? (it + 1) * G - 1 - c : it * G + c;
+}
+
+// Tile t of the longest-first order: query block (longest first), then batch, then head (heads that share
+// a K/V head are adjacent, so their K/V tiles come from L2).
+__device__ __forceinline__ void fwd_tile(int t, int H, int B, int nqb, int& h, int& b, int& qb) {
+  const int hb = H * B;
+  qb = nqb - 1 - t / hb;
+  const int r = t % hb;
+  h = r % H;
+  b = r / H;
+}
 
 template <int HD>
 __global__ void __launch_bounds__(NTHR, 1)
     attn_fwd1_tg_k(const __grid_constant__ CUtensorMap tqk, const __grid_constant__ CUtensorMap tvv,
-                   bf16* __restrict__ out, float* __restrict__ lse, int S, int H, int Hkv, float scale,
+                   bf16* __restrict__ out, float* __restrict__ lse, int S, int B, int H, int Hkv, float scale,
                    unsigned* err) {
   using C_ = F1Cfg<HD>;
   extern __shared__ uint8_t smem_raw[];
@@ -74,27 +96,32 @@ __global__ void __launch_bounds__(NTHR, 1)
   uint64_t* full = (uint64_t*)(xsum + 2 * QB);
   uint64_t* empty = full + C_::STAGES;
   uint64_t* qfull = empty + C_::STAGES;
-  uint64_t* sfull = qfull + 1;                         // [2]
+  uint64_t* qempty = qfull + 1;
+  uint64_t* sfull = qempty + 1;                        // [2]
   uint64_t* sempty = sfull + 2;                        // [2]
   uint64_t* pfull = sempty + 2;
   uint64_t* pempty = pfull + 1;
-  uint64_t* ofull = pempty + 1;
-  uint64_t* fin = ofull + 1;
+  uint64_t* ofull = pempty + 1;                        // [2]
+  uint64_t* oempty = ofull + 2;                        // [2]
+  uint64_t* fin = oempty + 2;
   uint32_t* tbase = (uint32_t*)(fin + 1);
   volatile int* abort_flag = (volatile int*)(tbase + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x, b = blockIdx.y, qb = gridDim.z - 1 - blockIdx.z;   // longest blocks first
-  const int kvh = h / (H / Hkv);
-  const int q0 = qb * QB, nkb = qb + 1;                // causal: key blocks 0 .. qb
-  const int xq = h * HD, xk = (H + kvh) * HD, xv = (H + Hkv + kvh) * HD;
+  const int nqb = (S + QB - 1) / QB, ntiles = nqb * B * H;
+  const int group = H / Hkv;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C_::STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     mbar_init(qfull, 1);
-    for (int i = 0; i < 2; ++i) { mbar_init(&sfull[i], 1); mbar_init(&sempty[i], NSM); }
+    mbar_init(qempty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sfull[i], 1);
+      mbar_init(&sempty[i], NSM);
+      mbar_init(&ofull[i], 1);
+      mbar_init(&oempty[i], NSM);
+    }
     mbar_init(pfull, NSM);
     mbar_init(pempty, 1);
-    mbar_init(ofull, 1);
     mbar_init(fin, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -115,33 +142,46 @@ __global__ void __launch_bounds__(NTHR, 1)
     // ---------------- TMA producer (whole warp, one elected lane issues) ----------------
     const bool leader = elect_one();
     bool ok = true;
+    int qlast = -1;   // tile count of the last Q load issued
     int issued[C_::STAGES];
 #pragma unroll
     for (int s = 0; s < C_::STAGES; ++s) issued[s] = -1;
-    if (leader) {
-      mbar_expect_tx(qfull, C_::QBYTES);
-#pragma unroll
-      for (int c = 0; c < HD / 64; ++c) tma3d(sq + c * 16384, &tqk, qfull, xq + 64 * c, q0, b);
-    }
-    int stage = 0;
+    int stage = 0, it = 0;
     uint32_t phase = 0;
-    for (int j = 0; ok && j < nkb; ++j) {
-      if (!uwait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
-      issued[stage] = (int)phase;
+    for (; ok; ++it) {
+      const int t = snake_tile(it, blockIdx.x, gridDim.x);
+      if (t >= ntiles) break;
+      int h, b, qb;
+      fwd_tile(t, H, B, nqb, h, b, qb);
+      const int kvh = h / group, nkb = qb + 1;
+      const int xq = h * HD, xk = (H + kvh) * HD, xv = (H + Hkv + kvh) * HD;
+      // Q's buffer is free once the previous tile's S products have completed
+      if (!uwait(qempty, ((uint32_t)it & 1u) ^ 1u, abort_flag, err)) { ok = false; break; }
+      qlast = it;
       if (leader) {
-        mbar_expect_tx(&full[stage], C_::STAGE);
-        uint8_t* sk = sst + stage * C_::STAGE;
-        uint8_t* sv = sk + C_::KBYTES;
+        mbar_expect_tx(qfull, C_::QBYTES);
 #pragma unroll
-        for (int c = 0; c < HD / 64; ++c) tma3d(sk + c * 16384, &tqk, &full[stage], xk + 64 * c, j * KB, b);
-#pragma unroll
-        for (int kh = 0; kh < 2; ++kh)
-#pragma unroll
-          for (int nb = 0; nb < HD / 64; ++nb)
-            tma3d(sv + (kh * (HD / 64) + nb) * 8192, &tvv, &full[stage], xv + 64 * nb, j * KB + 64 * kh, b);
+        for (int c = 0; c < HD / 64; ++c) tma3d(sq + c * 16384, &tqk, qfull, xq + 64 * c, qb * QB, b);
       }
       __syncwarp();
-      if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
+      for (int j = 0; j < nkb; ++j) {
+        if (!uwait(&empty[stage], phase ^ 1u, abort_flag, err)) { ok = false; break; }
+        issued[stage] = (int)phase;
+        if (leader) {
+          mbar_expect_tx(&full[stage], C_::STAGE);
+          uint8_t* sk = sst + stage * C_::STAGE;
+          uint8_t* sv = sk + C_::KBYTES;
+#pragma unroll
+          for (int c = 0; c < HD / 64; ++c) tma3d(sk + c * 16384, &tqk, &full[stage], xk + 64 * c, j * KB, b);
+#pragma unroll
+          for (int kh = 0; kh < 2; ++kh)
+#pragma unroll
+            for (int nb = 0; nb < HD / 64; ++nb)
+              tma3d(sv + (kh * (HD / 64) + nb) * 8192, &tvv, &full[stage], xv + 64 * nb, j * KB + 64 * kh, b);
+        }
+        __syncwarp();
+        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
+      }
     }
     if (!ok && lane == 0) {   // unwinding: let the copies in flight land before the CTA exits
       for (int s = 0; s < C_::STAGES; ++s) {
@@ -150,170 +190,194 @@ __global__ void __launch_bounds__(NTHR, 1)
         while (!mbar_test(&full[s], (uint32_t)issued[s]) && gtimer() - t0 < 100000000ull) {
         }
       }
-      const unsigned long long t0 = gtimer();
-      while (!mbar_test(qfull, 0) && gtimer() - t0 < 100000000ull) {
+      if (qlast >= 0) {   // the last Q load (phase parity = its tile count)
+        const unsigned long long t0 = gtimer();
+        while (!mbar_test(qfull, (uint32_t)qlast & 1u) && gtimer() - t0 < 100000000ull) {
+        }
       }
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer (whole warp, one elected lane issues and commits) ----------------
     constexpr uint32_t id_s = idesc_f16(QB, KB, false, false);
     constexpr uint32_t id_o = idesc_f16(QB, HD, false, true);
-    const uint32_t tso = tmem + 256;   // O
     const bool leader = elect_one();
-    bool ok = uwait(qfull, 0, abort_flag, err);
-    fence_after();
-    int stage = 0, pstage = 0;
+    bool ok = true;
+    int stage = 0, jg = 0, it = 0;
     uint32_t phase = 0;
     const uint32_t q_addr = su32(sq), p_addr = su32(sp);
-    // O += P_jb V_jb, then the stage and P are free and O holds blocks 0 .. jb
-    auto pv = [&](int jb, int st) -> bool {
-      if (!uwait(pfull, (uint32_t)(jb & 1), abort_flag, err)) return false;
+    // the P V product still to issue: block jl (of its tile) with global index pg, in stage pst, of tile pit
+    struct Pending { bool on; int jl, pg, pst, pit; bool last; } pend{false, 0, 0, 0, 0, false};
+    // O[tile parity] += P V: waits for P (and, on a tile's first block, for O's buffer to be read out);
+    // then the stage and P are free, and after a tile's last block O is complete
+    auto pv = [&](const Pending& p) -> bool {
+      if (!uwait(pfull, (uint32_t)p.pg & 1u, abort_flag, err)) return false;
+      const int ob = p.pit & 1;
+      if (p.jl == 0 && !uwait(&oempty[ob], ((uint32_t)(p.pit >> 1) & 1u) ^ 1u, abort_flag, err)) return false;
       fence_after();
       if (leader) {
-        const uint32_t v_addr = su32(sst + st * C_::STAGE + C_::KBYTES);
+        const uint32_t tso = tmem + C_::OCOL + (uint32_t)(ob * HD);
+        const uint32_t v_addr = su32(sst + p.pst * C_::STAGE + C_::KBYTES);
 #pragma unroll
         for (int ks = 0; ks < KB / 16; ++ks) {
           const int kh = ks / 4, kr = ks % 4;
           const uint64_t ad = sdesc(p_addr + kh * 16384 + kr * 32, 16, 1024);
           const uint64_t bd = sdesc(v_addr + kh * (HD / 64) * 8192 + kr * 2048, 8192, 1024);
-          mma_bf16(tso, ad, bd, id_o, (jb > 0 || ks > 0) ? 1u : 0u);
+          mma_bf16(tso, ad, bd, id_o, (p.jl > 0 || ks > 0) ? 1u : 0u);
         }
-        mma_commit(&empty[st]);
+        mma_commit(&empty[p.pst]);
         mma_commit(pempty);
+        if (p.last) mma_commit(&ofull[ob]);
       }
       __syncwarp();
       return true;
     };
-    for (int j = 0; ok && j < nkb; ++j) {
-      const int sb = j & 1;
-      if (!uwait(&sempty[sb], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort_flag, err) ||
-          !uwait(&full[stage], phase, abort_flag, err)) {
-        ok = false;
-        break;
-      }
-      fence_after();
-      if (leader) {
-        const uint32_t k_addr = su32(sst + stage * C_::STAGE);
-#pragma unroll
-        for (int ks = 0; ks < HD / 16; ++ks) {
-          const int kq = ks / 4, kr = ks % 4;
-          mma_bf16(tmem + sb * 128, sdesc(q_addr + kq * 16384 + kr * 32, 16, 1024),
-                   sdesc(k_addr + kq * 16384 + kr * 32, 16, 1024), id_s, ks > 0 ? 1u : 0u);
+    for (; ok; ++it) {
+      const int t = snake_tile(it, blockIdx.x, gridDim.x);
+      if (t >= ntiles) break;
+      int h, b, qb;
+      fwd_tile(t, H, B, nqb, h, b, qb);
+      const int nkb = qb + 1;
+      if (!uwait(qfull, (uint32_t)it & 1u, abort_flag, err)) { ok = false; break; }
+      for (int j = 0; j < nkb; ++j, ++jg) {
+        const int sb = jg & 1;
+        if (!uwait(&sempty[sb], ((uint32_t)(jg >> 1) & 1u) ^ 1u, abort_flag, err) ||
+            !uwait(&full[stage], phase, abort_flag, err)) {
+          ok = false;
+          break;
         }
-        mma_commit(&sfull[sb]);
+        fence_after();
+        if (leader) {
+          const uint32_t k_addr = su32(sst + stage * C_::STAGE);
+#pragma unroll
+          for (int ks = 0; ks < HD / 16; ++ks) {
+            const int kq = ks / 4, kr = ks % 4;
+            mma_bf16(tmem + sb * 128, sdesc(q_addr + kq * 16384 + kr * 32, 16, 1024),
+                     sdesc(k_addr + kq * 16384 + kr * 32, 16, 1024), id_s, ks > 0 ? 1u : 0u);
+          }
+          mma_commit(&sfull[sb]);
+          if (j == nkb - 1) mma_commit(qempty);   // Q is free once the tile's last S product completes
+        }
+        __syncwarp();
+        if (pend.on && !pv(pend)) { ok = false; break; }
+        pend = Pending{true, j, jg, stage, it, j == nkb - 1};
+        if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
       }
-      __syncwarp();
-      if (j > 0 && !pv(j - 1, pstage)) { ok = false; break; }
-      pstage = stage;
-      if (++stage == C_::STAGES) { stage = 0; phase ^= 1u; }
     }
-    if (ok && !pv(nkb - 1, pstage)) ok = false;
-    if (leader) {
-      if (ok) mma_commit(ofull);
-      mma_commit(fin);   // every MMA of the leader completes before TMEM is released
-    }
+    if (ok && pend.on && !pv(pend)) ok = false;
+    if (leader) mma_commit(fin);   // every MMA of the leader completes before TMEM is released
     __syncwarp();
   } else {
     // ---------------- softmax and output: warps 2..9, one query row per thread ----------------
     const int quad = warp & 3, half = (warp - 2) / 4;    // TMEM lane quadrant; key half of every block
     const int r = quad * 32 + lane;                       // row within the block = TMEM lane
-    const int q = q0 + r;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     const float sl2 = scale * kL2e;
-    float m = -INFINITY, l = 0.f;                         // running maximum (log2 units), this half's sum
-    // A failed wait only skips work: both warps of a quadrant still pass every named barrier.
+    // A failed wait only skips work: both warps of a quadrant still pass every named barrier (the same
+    // tiles and blocks on both).
     bool ok = true;
-    for (int j = 0; j < nkb; ++j) {
-      const int sb = j & 1;
-      if (ok && !uwait(&sfull[sb], (uint32_t)(j >> 1) & 1u, abort_flag, err)) ok = false;
-      float v[64];
-      float mh = -INFINITY;
-      if (ok) {
-        fence_after();
-        const int kmax = min(q, S - 1) - j * KB - half * 64;   // last visible key offset in the half
-        const uint32_t tcol = trow + (uint32_t)(sb * 128 + half * 64);
-        tmem_ld32(tcol, v);
-        tmem_ld32(tcol + 32u, v + 32);
-        fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sempty[sb]);
+    int jg = 0, it = 0;
+    for (;; ++it) {
+      const int t = snake_tile(it, blockIdx.x, gridDim.x);
+      if (t >= ntiles) break;
+      int h, b, qb;
+      fwd_tile(t, H, B, nqb, h, b, qb);
+      const int nkb = qb + 1, q = qb * QB + r;
+      const uint32_t ocol = C_::OCOL + (uint32_t)((it & 1) * HD);
+      float m = -INFINITY, l = 0.f;                       // running maximum (log2 units), this half's sum
+      for (int j = 0; j < nkb; ++j, ++jg) {
+        const int sb = jg & 1;
+        if (ok && !uwait(&sfull[sb], (uint32_t)(jg >> 1) & 1u, abort_flag, err)) ok = false;
+        float v[64];
+        float mh = -INFINITY;
+        if (ok) {
+          fence_after();
+          const int kmax = min(q, S - 1) - j * KB - half * 64;   // last visible key offset in the half
+          const uint32_t tcol = trow + (uint32_t)(sb * 128 + half * 64);
+          tmem_ld32(tcol, v);
+          tmem_ld32(tcol + 32u, v + 32);
+          fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sempty[sb]);
 #pragma unroll
-        for (int e = 0; e < 64; ++e) {
-          v[e] = e <= kmax ? v[e] * sl2 : -INFINITY;
-          mh = fmaxf(mh, v[e]);
-        }
-      }
-      // the partner half's maximum (double-buffered by block parity; one barrier per block)
-      float* xm = xmax + (j & 1) * 2 * QB;
-      xm[half * QB + r] = mh;
-      asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory");
-      if (!ok) continue;
-      const float mblk = fmaxf(mh, xm[(1 - half) * QB + r]);
-      const float mnew = fmaxf(m, mblk);
-      const bool move = mnew > m + 8.f;   // also true on the first block (m = -inf)
-      // P's buffer is free once the previous P V product has completed; O then holds blocks < j
-      if (!uwait(pempty, ((uint32_t)j & 1u) ^ 1u, abort_flag, err)) { ok = false; continue; }
-      if (j > 0 && __any_sync(0xffffffffu, move)) {   // rescale this half of the O row (warp-wide TMEM access)
-        const float a = move ? ex2(m - mnew) : 1.f;
-        l *= a;
-        fence_after();
-#pragma unroll 1
-        for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
-          float o[32];
-          tmem_ld32(trow + 256u + (uint32_t)c, o);
-#pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] *= a;
-          tmem_st32(trow + 256u + (uint32_t)c, o);
-        }
-      }
-      if (move) m = mnew;
-      uint8_t* prow = sp + half * 16384 + r * 128;   // this half's P block, row r (128-byte swizzle)
-      float sum = 0.f;
-#pragma unroll
-      for (int c = 0; c < 64; c += 32) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          const float p0 = ex2(v[c + e] - m), p1 = ex2(v[c + e + 1] - m);   // masked scores are -inf: 0
-          sum += p0 + p1;
-          __nv_bfloat162 hv = __floats2bfloat162_rn(p0, p1);
-          pk[e / 2] = *reinterpret_cast<uint32_t*>(&hv);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int piece = c / 8 + u;
-          *reinterpret_cast<uint4*>(prow + ((piece ^ (r & 7)) << 4)) =
-              make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-        }
-      }
-      l += sum;
-      fence_before();
-      fence_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(pfull);
-    }
-    // output: both halves use the same m; O / (l_0 + l_1), log-sum-exp m + log2(l_0 + l_1)
-    xsum[half * QB + r] = l;
-    asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory");
-    if (ok) {
-      const float lt = l + xsum[(1 - half) * QB + r];
-      const float inv = lt > 0.f ? 1.f / lt : 0.f;
-      if (uwait(ofull, 0, abort_flag, err)) {
-        fence_after();
-        bf16* orow = out + ((size_t)b * S + min(q, S - 1)) * ((size_t)H * HD) + (size_t)h * HD;
-#pragma unroll 1
-        for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {   // every lane loads (tcgen05.ld is
-          float o[32];                                                        // warp-wide); rows >= S store nothing
-          tmem_ld32(trow + 256u + (uint32_t)c, o);
-          if (q < S) {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] *= inv;
-#pragma unroll
-            for (int u = 0; u < 4; ++u) Vec8<bf16>::store(orow + c + 8 * u, o + 8 * u);
+          for (int e = 0; e < 64; ++e) {
+            v[e] = e <= kmax ? v[e] * sl2 : -INFINITY;
+            mh = fmaxf(mh, v[e]);
           }
         }
-        if (q < S && half == 0) lse[((size_t)b * H + h) * S + q] = (lt > 0.f ? m + log2f(lt) : INFINITY) * kLn2;
+        // the partner half's maximum (double-buffered by block parity; one barrier per block)
+        float* xm = xmax + (jg & 1) * 2 * QB;
+        xm[half * QB + r] = mh;
+        asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory");
+        if (!ok) continue;
+        const float mblk = fmaxf(mh, xm[(1 - half) * QB + r]);
+        const float mnew = fmaxf(m, mblk);
+        const bool move = mnew > m + 8.f;   // also true on the first block (m = -inf)
+        // P's buffer is free once the previous P V product has completed; O then holds blocks < j
+        if (!uwait(pempty, ((uint32_t)jg & 1u) ^ 1u, abort_flag, err)) { ok = false; continue; }
+        if (j > 0 && __any_sync(0xffffffffu, move)) {   // rescale this half of the O row (warp-wide TMEM access)
+          const float a = move ? ex2(m - mnew) : 1.f;
+          l *= a;
+          fence_after();
+#pragma unroll 1
+          for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {
+            float o[32];
+            tmem_ld32(trow + ocol + (uint32_t)c, o);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] *= a;
+            tmem_st32(trow + ocol + (uint32_t)c, o);
+          }
+        }
+        if (move) m = mnew;
+        uint8_t* prow = sp + half * 16384 + r * 128;   // this half's P block, row r (128-byte swizzle)
+        float sum = 0.f;
+#pragma unroll
+        for (int c = 0; c < 64; c += 32) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            const float p0 = ex2(v[c + e] - m), p1 = ex2(v[c + e + 1] - m);   // masked scores are -inf: 0
+            sum += p0 + p1;
+            __nv_bfloat162 hv = __floats2bfloat162_rn(p0, p1);
+            pk[e / 2] = *reinterpret_cast<uint32_t*>(&hv);
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int piece = c / 8 + u;
+            *reinterpret_cast<uint4*>(prow + ((piece ^ (r & 7)) << 4)) =
+                make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+          }
+        }
+        l += sum;
+        fence_before();
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pfull);
       }
+      // output: both halves use the same m; O / (l_0 + l_1), log-sum-exp m + log2(l_0 + l_1)
+      xsum[half * QB + r] = l;
+      asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory");
+      if (!ok) continue;
+      const float lt = l + xsum[(1 - half) * QB + r];
+      const float inv = lt > 0.f ? 1.f / lt : 0.f;
+      if (!uwait(&ofull[it & 1], (uint32_t)(it >> 1) & 1u, abort_flag, err)) { ok = false; continue; }
+      fence_after();
+      bf16* orow = out + ((size_t)b * S + min(q, S - 1)) * ((size_t)H * HD) + (size_t)h * HD;
+#pragma unroll 1
+      for (int c = half * (HD / 2); c < (half + 1) * (HD / 2); c += 32) {   // every lane loads (tcgen05.ld is
+        float o[32];                                                        // warp-wide); rows >= S store nothing
+        tmem_ld32(trow + ocol + (uint32_t)c, o);
+        if (q < S) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] *= inv;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) Vec8<bf16>::store(orow + c + 8 * u, o + 8 * u);
+        }
+      }
+      // this warp's half of O has been read: the buffer may take the tile after next
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&oempty[it & 1]);
+      if (q < S && half == 0) lse[((size_t)b * H + h) * S + q] = (lt > 0.f ? m + log2f(lt) : INFINITY) * kLn2;
     }
   }
 
@@ -1442,6 +1506,7 @@ __global__ void __launch_bounds__(NTHR_B, 1)
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
+int g_nsm = 0;
 
 bool enc_init() {
   static int avail = -1;
@@ -1451,7 +1516,8 @@ bool enc_init() {
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-  if (major != 10 || minor != 3) return false;
+  cudaDeviceGetAttribute(&g_nsm, cudaDevAttrMultiProcessorCount, dev);
+  if (major != 10 || minor != 3 || g_nsm < 1) return false;
   void* fn = nullptr;
   cudaDriverEntryPointQueryResult qr;
   if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &qr) != cudaSuccess ||
@@ -1559,8 +1625,10 @@ bool fwd1_launch(const void* qkv, void* out, float* lse, int B, int S, int H, in
   const int W = (H + 2 * Hkv) * HD;
   CUtensorMap tqk, tvv;
   if (!qkv_map(&tqk, qkv, B, S, W, 128) || !qkv_map(&tvv, qkv, B, S, W, 64)) return false;
-  const dim3 grid(H, B, (S + QB - 1) / QB);
-  return launch_pdl(kern, grid, NTHR, C_::SMEM, s, tqk, tvv, (bf16*)out, lse, S, H, Hkv, scale, err) == cudaSuccess;
+  const long ntiles = (long)H * B * ((S + QB - 1) / QB);   // persistent: at most one CTA per SM
+  const int grid = (int)std::min<long>(ntiles, g_nsm);
+  return launch_pdl(kern, dim3(grid), NTHR, C_::SMEM, s, tqk, tvv, (bf16*)out, lse, S, B, H, Hkv, scale, err) ==
+         cudaSuccess;
 }
 
 }  // namespace tg
@@ -1571,7 +1639,8 @@ bool fwd1_launch(const void* qkv, void* out, float* lse, int B, int S, int H, in
 bool attn_fwd_tcgen05(const void* qkv, void* out, float* lse, int B, int S, int H, int Hkv, int hd, cudaStream_t s,
                       unsigned* err, float scale) {
   if (hd != 64 && hd != 128) return false;
-  if (((uintptr_t)qkv & 15u) || ((uintptr_t)out & 15u) || B > 65535 || (S + tg::QB - 1) / tg::QB > 65535) return false;
+  if (((uintptr_t)qkv & 15u) || ((uintptr_t)out & 15u) || (long)B * H * ((S + tg::QB - 1) / tg::QB) > 0x7fffffffL)
+    return false;
   if (!tg::enc_init()) return false;
   note_launch(1);
   return hd == 64 ? tg::fwd1_launch<64>(qkv, out, lse, B, S, H, Hkv, s, err, scale)

@@ -238,7 +238,9 @@ ATTN_SHAPES = [(2, 512, 12, 12, 64), (1, 1024, 32, 4, 64), (1, 200, 4, 4, 32), (
                (1, 300, 8, 8, 128), (3, 1, 4, 2, 64), (1, 64, 2, 1, 32), (2, 1500, 4, 2, 128),
                (2, 333, 6, 3, 64), (1, 130, 2, 2, 64), (1, 65, 2, 2, 128),
                # head dims the tcgen05 kernels take zero-padded to 128 or 64 (the 3B workload's is 100)
-               (1, 2048, 4, 4, 100), (2, 257, 4, 2, 96), (1, 700, 2, 2, 80), (1, 300, 4, 4, 48)]
+               (1, 2048, 4, 4, 100), (2, 257, 4, 2, 96), (1, 700, 2, 2, 80), (1, 300, 4, 4, 48),
+               # more tiles than SMs: the persistent forward runs several tiles per CTA (O in both buffers)
+               (4, 1024, 32, 4, 64), (2, 1024, 32, 32, 128), (8, 300, 16, 16, 128)]
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
@@ -291,7 +293,8 @@ def test_attention_matches_sdpa(B, dtype, Bb, S, H, Hkv, hd):
 # 128-key block's maximum exceeds the previous one by far more than the rescale threshold, so the
 # one-pass forward rescales O in TMEM at every block; outputs, log-sum-exp and gradients against the
 # fp32 reference as in test_attention_matches_sdpa.
-@pytest.mark.parametrize("Bb,S,H,Hkv,hd", [(1, 700, 2, 2, 64), (2, 520, 4, 2, 64), (1, 600, 2, 2, 128)])
+@pytest.mark.parametrize("Bb,S,H,Hkv,hd", [(1, 700, 2, 2, 64), (2, 520, 4, 2, 64), (1, 600, 2, 2, 128),
+                                            (16, 520, 16, 8, 64)])
 def test_attention_rescales_on_growing_scores(B, Bb, S, H, Hkv, hd):
     g = torch.Generator(device="cuda").manual_seed(S + hd)
     W = (H + 2 * Hkv) * hd
