@@ -80,7 +80,11 @@ LLAMA7B_SHAPES = _shapes_of(4096, 12288, 22016, 11008, 32000, n=2048)
 def gemm(args):
     B = _lib()
     shapes = {"gpt2": GPT2_SHAPES, "llama-1b": LLAMA1B_SHAPES, "llama-7b": LLAMA7B_SHAPES}[args.workload]
+    if args.only and args.only not in [sh[0] for sh in shapes]:
+        raise SystemExit(f"no shape named {args.only!r}")
     for name, mode, M, N, K in shapes:
+        if args.only and name != args.only:
+            continue
         bf = torch.bfloat16
         if mode == 0:
             a, b = torch.randn(M, K, device="cuda").to(bf), torch.randn(N, K, device="cuda").to(bf)
@@ -142,6 +146,7 @@ def main():
     p = sub.add_parser("gemm")
     p.add_argument("--workload", choices=["gpt2", "llama-1b", "llama-7b"], default="gpt2")
     p.add_argument("--reps", type=int, default=20)
+    p.add_argument("--only", default="", help="run this shape only (its name, e.g. 'qkv fwd')")
     p = sub.add_parser("attention")
     p.add_argument("--batch", type=int, default=8)
     p.add_argument("--seq", type=int, default=512)
