@@ -1,9 +1,10 @@
-// Causal attention on the 5th-generation tensor cores (sm_103a), head dims 64 and 128: a one-pass
-// forward with lazy rescaling and a two-kernel backward (dQ; dK and dV) with 64-row (head dim 128) or
-// 128-row (head dim 64) inner blocks.
+// Causal attention on the 5th-generation tensor cores (sm_103a), head dims 64 and 128: a persistent
+// one-pass forward with lazy rescaling and a two-kernel backward (dQ; dK and dV) with 64-row (head dim
+// 128) or 128-row (head dim 64) inner blocks.
 //
-// One CTA per 128 rows of one (batch, head). TMA brings the CTA's fixed tile once and the streamed tiles
-// through a stage ring (128-byte swizzle; a 3-D tensor map over [batch, token, feature] reads rows past
+// A tile is 128 rows of one (batch, head): the forward runs at most one CTA per SM over a deal of the
+// tiles, the backward kernels one CTA per tile. TMA brings a tile's fixed operands once and the streamed
+// tiles through a stage ring (128-byte swizzle; a 3-D tensor map over [batch, token, feature] reads rows past
 // the sequence end as zeros); one elected lane of the MMA warp issues tcgen05.mma with fp32
 // accumulators in TMEM; the elementwise warps own TMEM lane quadrants (one row per thread). Every
 // mbarrier wait is bounded (about 2 s); on expiry the kernel raises ZL_DEVERR_TIMEOUT and unwinds.
