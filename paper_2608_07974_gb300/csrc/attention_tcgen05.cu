@@ -64,9 +64,10 @@ struct F1Cfg {
   static_assert(OCOL + 2 * HD <= 512, "TMEM columns");
 };
 
-// The it-th tile of CTA c among G: the tiles are sorted longest first and dealt out in rounds of G whose
-// direction alternates (round 0: c, round 1: 2G - 1 - c, ...), so every CTA's long and short tiles even
-// out; past the last tile it returns a value >= every tile count (every later round is past it too).
+// The it-th tile of CTA c among G: the tiles are sorted longest first and dealt out G at a time, the
+// direction alternating between deals (deal 0: c, deal 1: 2G - 1 - c, ...), so every CTA's long and short
+// tiles even out; past the last tile it returns a value >= every tile count (every later deal is past it
+// too).
 __device__ __forceinline__ int snake_tile(int it, int c, int G) {
   return (it & 1) ? (it + 1) * G - 1 - c : it * G + c;
 }
